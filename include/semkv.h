@@ -122,8 +122,9 @@ uint32_t semkv_block_high_count(uint32_t n, uint32_t r_num, uint32_t r_den);
 
 /* Gaussian N(0,1) Lloyd-Max codebook with L levels (Sec. 4.9: "Gaussian-optimal
  * Lloyd-Max codebook", extended to any integer L).  Computed on the host in fp64
- * by Lloyd iteration to convergence; centroids[L] = fp32(c_l), thresholds[L-1] =
- * fp32((c_l + c_{l+1})/2) taken in fp64.  Host pointers. */
+ * by Lloyd iteration to convergence, then made exactly symmetric (c_l = -c_{L-1-l});
+ * centroids[L] = fp32(c_l), thresholds[L-1] = fp32((c_l + c_{l+1})/2) taken in fp64.
+ * Host pointers. */
 semkv_status semkv_lloyd_max_gaussian(int32_t levels, float* centroids, float* thresholds);
 
 /* Top-r selection, Eqs. 4-5 / Algorithm 1.  For each sequence b of `batch`:

@@ -242,6 +242,10 @@ def lloyd_max_gaussian(L: int, iters: int = 200000, tol: float = 1e-15):
         c = nc
         if delta < tol:
             break
+    # N(0,1) is symmetric, so is its Lloyd-Max codebook: symmetrize the converged
+    # centroids exactly (the middle centroid of an odd L, and the middle threshold of
+    # an even L, become exactly 0 rather than +-1e-16 of iteration noise)
+    c = [0.5 * (c[i] - c[L - 1 - i]) for i in range(L)]
     t = [(c[i] + c[i + 1]) / 2 for i in range(L - 1)]
     edges = [-math.inf] + t + [math.inf]
     # MSE = E[X^2] - sum_l P_l c_l^2 for centroid-condition quantizers

@@ -215,7 +215,8 @@ void orc_unpack_row(const uint8_t* row, int L, uint8_t* codes) {
 /* ------------------------------------------------------------ quantizers ------ */
 
 /* Affine row quantizer Q_b (Eq. 7 with the Sec. 4.1 per-row asymmetric quantizer):
- *   mn, mx = min, max of the row;  s32 = (mx - mn) / (L - 1)
+ *   mn, mx = min, max of the row (a zero extreme taken as +0);
+ *   s32 = (mx - mn) / (L - 1)
  *   s16 = fp16(s32) (limited to 65504);  z16 = fp16(mn)  (= mn, an fp16 value)
  *   codes c_j = clamp(rint((x_j - z) * fl(1/s)), 0, L-1) with z, s the fp32 values
  *   of the stored parameters; all codes 0 when s == 0. */
@@ -228,6 +229,10 @@ void orc_affine_row(const uint16_t* x, int L, uint8_t* codes, uint16_t* s_out,
     if (xf[j] < mn) mn = xf[j];
     if (xf[j] > mx) mx = xf[j];
   }
+  /* a zero extreme is taken as +0, so the stored offset does not depend on the
+   * order in which equal zeros of either sign were met */
+  if (mn == 0.0f) mn = 0.0f;
+  if (mx == 0.0f) mx = 0.0f;
   float range = mx - mn;
   float s32 = range / (float)(L - 1);
   uint16_t s16 = f16_param(s32);

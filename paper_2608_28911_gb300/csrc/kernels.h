@@ -1,0 +1,75 @@
+// kernels.h — launch interfaces between the C ABI (api.cu) and the kernels.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace semkv {
+
+// Quantize tokens 0..n-1 of a source K/V tensor [B][NL][H][Tsrc][128] into the
+// pools at slot base + slot[b][i] (Eq. 7).
+struct QuantArgs {
+  int base, L_hi, L_lo;
+  const uint16_t* k;
+  const uint16_t* v;
+  int B, NL, H, Tsrc, n;
+  const uint8_t* is_high;   // [B][n]
+  const uint32_t* slot;     // [B][n]
+  int64_t hi_base, lo_base, tok_base;
+  const int8_t* signs;      // [NL][H][128] (TQ)
+  const float* thr_hi;
+  const float* thr_lo;
+  uint8_t* hi_pool;
+  uint8_t* lo_pool;
+  int64_t hi_cap, lo_cap;
+  int32_t* hi_tok;
+  int32_t* lo_tok;
+  int32_t* err;
+};
+cudaError_t launch_quantize_pack(const QuantArgs& a, int num_sms, cudaStream_t stream);
+
+// Top-r selection of each sequence (Eqs. 4-5).
+struct RankArgs {
+  const float* scores;      // [B][T] (row stride ld)
+  int B, T;
+  int64_t ld;
+  uint32_t n_high;
+  uint8_t* is_high;         // [B][T]
+  uint32_t* slot;           // [B][T]
+};
+cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream);
+
+// Decode attention over one layer of the cache (split-K + combine).
+struct DecodePlan {
+  int tiles_hi, tiles_lo, tiles_st;     // 16-token tiles per (b, h) per source
+  int splits_hi, splits_lo, splits_st;  // CTAs per (b, h) per source
+  int splits;                            // total partials per (b, h)
+};
+struct DecodeArgs {
+  int base, L_hi, L_lo;
+  int B, NL, H, Hq, layer;
+  const uint8_t* hi_pool;
+  const uint8_t* lo_pool;
+  int64_t hi_cap, lo_cap, hi_count, lo_count;
+  const uint16_t* stage_k;   // [B][NL][H][block][128]
+  const uint16_t* stage_v;
+  int block, stage_n;
+  const uint16_t* q;         // [B][Hq][128]
+  float* out;                // [B][Hq][128]
+  float scale_log2;          // softmax scale * log2(e)
+  float* partials;           // [B][H][splits][kPartialFloats]
+  const int8_t* signs;       // TQ
+  const float* cb_hi;        // TQ centroids
+  const float* cb_lo;
+  float* qrot;               // TQ: [B][Hq][128] rotated queries (workspace)
+  int32_t* err;
+  DecodePlan plan;
+};
+constexpr int kPartialFloats = 16 + 8 * 128;  // m[8], l[8], o[8][128]
+DecodePlan make_decode_plan(int B, int H, int64_t hi_count, int64_t lo_count, int stage_n,
+                            int num_sms);
+size_t decode_workspace_floats(int B, int H, int Hq);
+cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream);
+
+int device_sm_count();
+
+}  // namespace semkv

@@ -1,0 +1,162 @@
+// rank.cu — top-r selection of Eqs. 4-5 / Algorithm 1 (and of each block in
+// Algorithm 2): is_high marks the n_high largest scores of a sequence, ties going to
+// the lower token index; slot is each token's position in its pool.
+//
+// One 1024-thread CTA per sequence.  Scores become order-preserving 32-bit keys
+// (NaN -> 0, below every number; -0 -> +0).  A 4-pass MSB-first radix select over
+// 8-bit digits finds theta, the key of the n_high-th largest score, and `need`, how
+// many keys equal to theta are taken (the earliest ones).  One sweep with a block
+// scan of packed (greater, equal) counts then gives, for token i,
+//   high(i)        = key_i > theta  or  (key_i == theta and eq_before(i) < need)
+//   high_before(i) = gt_before(i) + min(eq_before(i), need)
+//   slot(i)        = high(i) ? high_before(i) : i - high_before(i).
+#include "common.cuh"
+#include "kernels.h"
+
+namespace semkv {
+
+namespace {
+
+constexpr int kThreads = 1024;
+constexpr int kItems = 4;
+
+__device__ __forceinline__ uint32_t order_key(float f) {
+  if (f != f) return 0u;  // NaN ranks below every number
+  uint32_t b = __float_as_uint(f);
+  if (f == 0.0f) b = 0u;  // -0 == +0
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// exclusive scan of a 64-bit value over the CTA; returns the prefix, sets *total
+__device__ __forceinline__ uint64_t block_exclusive_scan(uint64_t v, uint64_t* warp_sums,
+                                                         uint64_t* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint64_t x = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    uint64_t y = __shfl_up_sync(0xffffffffu, x, off);
+    if (lane >= off) x += y;
+  }
+  if (lane == 31) warp_sums[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    uint64_t w = warp_sums[lane];
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      uint64_t y = __shfl_up_sync(0xffffffffu, w, off);
+      if (lane >= off) w += y;
+    }
+    warp_sums[lane] = w;  // inclusive over warps
+  }
+  __syncthreads();
+  const uint64_t before_warp = warp == 0 ? 0ull : warp_sums[warp - 1];
+  *total = warp_sums[31];
+  const uint64_t r = before_warp + x - v;
+  __syncthreads();  // warp_sums is reused by the next call
+  return r;
+}
+
+__global__ void __launch_bounds__(kThreads) rank_assign_kernel(RankArgs a) {
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t sel_prefix, sel_k;
+  __shared__ uint64_t warp_sums[32];
+  const int b = blockIdx.x;
+  const float* s = a.scores + (int64_t)b * a.ld;
+  uint8_t* is_high = a.is_high + (int64_t)b * a.T;
+  uint32_t* slot = a.slot + (int64_t)b * a.T;
+  const uint32_t T = (uint32_t)a.T;
+  const int tid = threadIdx.x;
+
+  if (a.n_high == 0 || a.n_high == T) {
+    const uint8_t all = a.n_high == T ? 1 : 0;
+    for (uint32_t i = tid; i < T; i += kThreads) {
+      is_high[i] = all;
+      slot[i] = i;
+    }
+    return;
+  }
+
+  // ---- radix select: theta = key of the n_high-th largest, need = ties taken
+  uint32_t prefix = 0, mask = 0, k = a.n_high;
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    for (int i = tid; i < 256; i += kThreads) hist[i] = 0;
+    __syncthreads();
+    for (uint32_t i0 = 0; i0 < T; i0 += kThreads) {
+      const uint32_t i = i0 + tid;
+      bool cand = false;
+      uint32_t bin = 0;
+      if (i < T) {
+        const uint32_t key = order_key(s[i]);
+        cand = (key & mask) == prefix;
+        bin = (key >> shift) & 0xFFu;
+      }
+      // warp-aggregated histogram update: equal bins of a warp add once
+      const uint32_t active = __ballot_sync(0xffffffffu, cand);
+      if (cand) {
+        const uint32_t peers = __match_any_sync(active, bin);
+        const int leader = __ffs(peers) - 1;
+        if ((tid & 31) == leader) atomicAdd(&hist[bin], (uint32_t)__popc(peers));
+      }
+    }
+    __syncthreads();
+    if (tid == 0) {
+      uint32_t cum = 0, chosen = 0;
+      for (int bin = 255; bin >= 0; --bin) {
+        const uint32_t c = hist[bin];
+        if (cum + c >= k) {
+          chosen = (uint32_t)bin;
+          break;
+        }
+        cum += c;
+      }
+      sel_prefix = prefix | (chosen << shift);
+      sel_k = k - cum;
+    }
+    __syncthreads();
+    prefix = sel_prefix;
+    k = sel_k;
+    mask |= 0xFFu << shift;
+    __syncthreads();
+  }
+  const uint32_t theta = prefix, need = k;
+
+  // ---- one sweep: flags and slots from a scan of packed (eq << 32 | gt) counts
+  uint64_t run = 0;  // totals of all earlier chunks
+  for (uint32_t c0 = 0; c0 < T; c0 += kThreads * kItems) {
+    uint32_t keys[kItems];
+    uint64_t local = 0;
+#pragma unroll
+    for (int j = 0; j < kItems; ++j) {
+      const uint32_t i = c0 + tid * kItems + j;
+      keys[j] = i < T ? order_key(s[i]) : 0u;
+      if (i < T) local += (keys[j] > theta ? 1ull : 0ull) | ((keys[j] == theta ? 1ull : 0ull) << 32);
+    }
+    uint64_t total;
+    uint64_t before = run + block_exclusive_scan(local, warp_sums, &total);
+#pragma unroll
+    for (int j = 0; j < kItems; ++j) {
+      const uint32_t i = c0 + tid * kItems + j;
+      if (i >= T) break;
+      const uint32_t gt_b = (uint32_t)(before & 0xFFFFFFFFu);
+      const uint32_t eq_b = (uint32_t)(before >> 32);
+      const bool gt = keys[j] > theta, eq = keys[j] == theta;
+      const bool hi = gt || (eq && eq_b < need);
+      const uint32_t hib = gt_b + min(eq_b, need);
+      is_high[i] = hi ? 1 : 0;
+      slot[i] = hi ? hib : i - hib;
+      before += (gt ? 1ull : 0ull) | ((eq ? 1ull : 0ull) << 32);
+    }
+    run += total;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream) {
+  if (a.B == 0 || a.T == 0) return cudaSuccess;
+  rank_assign_kernel<<<a.B, kThreads, 0, stream>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace semkv

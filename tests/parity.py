@@ -1,0 +1,90 @@
+"""Shared set-up for the GPU parity tests: the same seeded inputs are fed to the
+CUDA library (through the C ABI) and to the CPU oracle, independently."""
+import math
+
+import numpy as np
+
+import oracle
+from paper_2608_28911_gb300 import synthetic
+
+ATOL = 2e-3       # attention max-abs error vs the oracle's fp64 result
+RTOL_L2 = 1e-3    # attention relative L2 error over the whole output
+
+
+def attention_errors(got, ref):
+    got = np.asarray(got, np.float64)
+    mask = ~np.isnan(ref)
+    d = got[mask] - ref[mask]
+    return float(np.abs(d).max()), float(np.linalg.norm(d) / np.linalg.norm(ref[mask]))
+
+
+class Pair:
+    """A GPU cache and an oracle cache built from the same inputs."""
+
+    def __init__(self, base, L_hi, L_lo, B, NL, H, Hq, T, r_num, r_den, seed, block=128,
+                 extra_cap=0, tiefree=False):
+        import torch
+        from paper_2608_28911_gb300 import semkv
+        self.torch, self.semkv = torch, semkv
+        self.dev = torch.device("cuda:0")
+        self.base, self.B, self.NL, self.H, self.Hq, self.T = base, B, NL, H, Hq, T
+        self.r_num, self.r_den, self.seed = r_num, r_den, seed
+        self.n_high = oracle.high_count_floor(T, r_num, r_den)
+        signs = synthetic.signs(seed, NL, H) if base == oracle.BASE_TQ else None
+        self.desc = semkv.QuantDesc(base, L_hi, L_lo, signs=signs, device=self.dev)
+        self.cache = semkv.KVCache(self.desc, B, NL, H, Hq, hi_cap=self.n_high + extra_cap,
+                                   lo_cap=T - self.n_high + extra_cap, block=block,
+                                   device=self.dev)
+        self.oc = oracle.Cache(base=base, L_hi=L_hi, L_lo=L_lo, batch=B, layers=NL, kv_heads=H,
+                               q_heads=Hq, block=block, hi_cap=self.cache.s.hi_cap,
+                               lo_cap=self.cache.s.lo_cap)
+        if base == oracle.BASE_TQ:
+            self.oc.signs = signs
+            _, c32, t32, _ = oracle.lloyd_max_gaussian(L_hi)
+            self.oc.cb_hi = (c32, t32)
+            _, c32, t32, _ = oracle.lloyd_max_gaussian(L_lo)
+            self.oc.cb_lo = (c32, t32)
+        self.k, self.v = synthetic.kv(seed, B, NL, H, T)
+        self.s = (synthetic.scores_tiefree(seed, B, T) if tiefree
+                  else synthetic.scores_zipf(seed, B, T))
+
+    def quantize(self):
+        torch, semkv = self.torch, self.semkv
+        d = self.dev
+        scores = torch.from_numpy(self.s).to(d)
+        self.is_high = torch.empty((self.B, self.T), dtype=torch.uint8, device=d)
+        self.slot = torch.empty((self.B, self.T), dtype=torch.int32, device=d)
+        semkv.semkv_rank_assign(scores, self.n_high, self.is_high, self.slot)
+        semkv.semkv_quantize_pack(self.desc, torch.from_numpy(self.k).to(d),
+                                  torch.from_numpy(self.v).to(d), self.is_high, self.slot,
+                                  self.n_high, self.cache)
+        torch.cuda.synchronize()
+        self.o_is_high, self.o_slot = oracle.quantize_prompt(
+            self.oc, synthetic.f16_bits(self.k), synthetic.f16_bits(self.v), self.s,
+            self.r_num, self.r_den)
+
+    def assert_records_equal(self):
+        c, oc = self.cache, self.oc
+        assert c.hi_count == oc.hi_count and c.lo_count == oc.lo_count
+        assert c.n_tokens == oc.n_tokens
+        hp = c.hi_pool.cpu().numpy()[..., :oc.hi_count, :]
+        lp = c.lo_pool.cpu().numpy()[..., :oc.lo_count, :]
+        for name, got, want in (("hi", hp, oc.hi_pool[..., :oc.hi_count, :]),
+                                ("lo", lp, oc.lo_pool[..., :oc.lo_count, :])):
+            if not np.array_equal(got, want):
+                bad = np.argwhere(np.any(got != want, axis=-1))
+                raise AssertionError(f"{name} pool differs at {len(bad)} records, first {bad[:3]}")
+        assert np.array_equal(c.hi_tok.cpu().numpy()[:, :oc.hi_count], oc.hi_tok[:, :oc.hi_count])
+        assert np.array_equal(c.lo_tok.cpu().numpy()[:, :oc.lo_count], oc.lo_tok[:, :oc.lo_count])
+
+    def decode(self, layer=0, qseed=0, heads=None):
+        torch, semkv = self.torch, self.semkv
+        q = synthetic.queries(self.seed + 100 * qseed, self.B, self.Hq)
+        out = torch.empty((self.B, self.Hq, 128), dtype=torch.float32, device=self.dev)
+        ws = self.cache.workspace()
+        scale = 1.0 / math.sqrt(128)
+        semkv.semkv_decode_attention(self.desc, self.cache, layer, torch.from_numpy(q).to(self.dev),
+                                     out, scale, ws)
+        torch.cuda.synchronize()
+        ref = oracle.decode_attention(self.oc, layer, synthetic.f16_bits(q), scale, heads=heads)
+        return out.cpu().numpy(), ref

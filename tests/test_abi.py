@@ -1,0 +1,73 @@
+"""CPU checks of the C-ABI library: it loads, exports every entry point that
+include/semkv.h declares, and its host-only logic (sizes, counts, argument
+validation, the host Lloyd-Max codebook) behaves as documented.  No kernel runs."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from conftest import ROOT
+
+HEADER = os.path.join(ROOT, "include", "semkv.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_28911_gb300 import build
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"\b(semkv_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 12
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_host_sizes_and_counts_match_oracle(lib):
+    lib.semkv_record_bytes.restype = ctypes.c_size_t
+    lib.semkv_row_bytes.restype = ctypes.c_size_t
+    for L in range(2, 9):
+        assert lib.semkv_row_bytes(L) == oracle.row_bytes(L)
+        for base in (0, 1):
+            assert lib.semkv_record_bytes(base, L) == oracle.record_bytes(base, L)
+    assert lib.semkv_row_bytes(9) == 0 and lib.semkv_row_bytes(1) == 0
+    lib.semkv_high_count_floor.restype = ctypes.c_uint32
+    lib.semkv_block_high_count.restype = ctypes.c_uint32
+    for T in (0, 1, 7, 128, 1024, 32768, 131072):
+        for num, den in ((26, 100), (1, 4), (35, 100), (3, 4), (1, 1), (0, 5)):
+            assert lib.semkv_high_count_floor(T, num, den) == oracle.high_count_floor(T, num, den)
+            assert lib.semkv_block_high_count(T, num, den) == oracle.block_high_count(T, num, den)
+
+
+def test_host_lloyd_max_agrees_with_oracle(lib):
+    lib.semkv_lloyd_max_gaussian.argtypes = [ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p]
+    for L in range(2, 9):
+        c = np.zeros(L, np.float32)
+        t = np.zeros(L - 1, np.float32)
+        assert lib.semkv_lloyd_max_gaussian(L, c.ctypes.data, t.ctypes.data) == 0
+        _, oc, ot, _ = oracle.lloyd_max_gaussian(L)
+        assert np.array_equal(c, oc) and np.array_equal(t, ot), L
+
+
+def test_argument_validation_returns_status(lib):
+    p = ctypes.c_void_p
+    lib.semkv_rank_assign.argtypes = [p, ctypes.c_int32, ctypes.c_int32, ctypes.c_uint32, p, p, p,
+                                      p, ctypes.c_size_t, p]
+    assert lib.semkv_rank_assign(None, 1, 10, 1, None, None, None, None, 0, None) == 1
+    lib.semkv_quantize_pack.argtypes = [p, p, p, ctypes.c_int32, p, p, ctypes.c_uint32, p, p]
+    assert lib.semkv_quantize_pack(None, None, None, 10, None, None, 0, None, None) == 1
+    lib.semkv_decode_attention.argtypes = [p, p, ctypes.c_int32, p, p, ctypes.c_float, p,
+                                           ctypes.c_size_t, p]
+    assert lib.semkv_decode_attention(None, None, 0, None, None, 1.0, None, 0, None) == 1
+    lib.semkv_status_string.restype = ctypes.c_char_p
+    assert lib.semkv_status_string(3) == b"pool or staging capacity exceeded"

@@ -1,0 +1,155 @@
+"""GPU parity: the CUDA library (through the C ABI) against the CPU oracle.
+
+Bit-exact: top-r flags and slots, every packed record byte, slot->token arrays.
+Attention: max-abs error <= 2e-3 and relative L2 error <= 1e-3 against the
+oracle's fp64 attention over the same dequantized cache.
+Sizes span several 16-token tiles with ragged tails, every level count, both
+bases, GQA group sizes 1..8, the fp16 staged tail and the degenerate splits.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_28911_gb300 import synthetic
+from parity import ATOL, RTOL_L2, Pair, attention_errors
+
+pytestmark = pytest.mark.gpu
+
+
+# ------------------------------------------------------------------ rank -----
+
+@pytest.mark.parametrize("T", [1, 7, 16, 1000, 4097, 70001])
+def test_rank_assign_bit_exact(T):
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    B = 3
+    s = synthetic.scores_zipf(T, B, T)
+    rng = np.random.default_rng(T)
+    if T > 20:
+        s[0, rng.choice(T, 5, replace=False)] = np.nan
+        s[1, rng.choice(T, 5, replace=False)] = -0.0
+        s[1, rng.choice(T, 5, replace=False)] = 0.0
+        s[2, rng.choice(T, 3, replace=False)] = np.inf
+        s[2, rng.choice(T, 3, replace=False)] = -np.inf
+        s[2, rng.choice(T, 10, replace=False)] *= -1
+    d = torch.device("cuda:0")
+    st = torch.from_numpy(s).to(d)
+    for n_high in sorted({0, 1, T // 4, max(T - 1, 0), T}):
+        ih = torch.empty((B, T), dtype=torch.uint8, device=d)
+        sl = torch.empty((B, T), dtype=torch.int32, device=d)
+        semkv.semkv_rank_assign(st, n_high, ih, sl)
+        o_ih, o_sl, _ = oracle.rank_assign(s, n_high)
+        assert np.array_equal(ih.cpu().numpy(), o_ih), n_high
+        assert np.array_equal(sl.cpu().numpy().view(np.uint32), o_sl), n_high
+
+
+# -------------------------------------------------------------- quantize -----
+
+@pytest.mark.parametrize("base,L_hi,L_lo,B,NL,H,T,r", [
+    (0, 5, 5, 1, 1, 1, 1024, (0, 100)),     # tiny uniform 5-level affine
+    (0, 6, 5, 2, 2, 2, 333, (26, 100)),     # mixed 6/5, ragged
+    (0, 2, 3, 1, 1, 2, 70, (1, 2)),
+    (0, 4, 7, 1, 1, 2, 70, (1, 3)),
+    (0, 8, 8, 1, 2, 1, 50, (1, 2)),
+    (1, 4, 3, 1, 2, 2, 200, (3, 4)),        # TQ 4/3
+    (1, 6, 5, 1, 1, 2, 90, (1, 4)),
+    (1, 8, 2, 1, 1, 2, 90, (1, 4)),
+])
+def test_quantize_pack_bit_exact(base, L_hi, L_lo, B, NL, H, T, r):
+    p = Pair(base, L_hi, L_lo, B, NL, H, 4 * H, T, r[0], r[1], seed=T + L_hi)
+    p.quantize()
+    assert np.array_equal(p.is_high.cpu().numpy(), p.o_is_high)
+    p.assert_records_equal()
+    assert int(p.cache.dev_error.item()) == 0
+
+
+def test_quantize_edge_rows_bit_exact():
+    # constant rows, signed zeros, tiny (subnormal-step) ranges and huge ranges
+    p = Pair(0, 6, 5, 1, 1, 2, 8, 64, 1, 2, seed=3)
+    k = p.k.astype(np.float32)
+    v = p.v.astype(np.float32)
+    k[0, 0, 0, 0] = 1.5
+    k[0, 0, 0, 1] = 0.0
+    k[0, 0, 0, 1, ::2] = -0.0
+    k[0, 0, 0, 2] = np.linspace(0, 6e-5, 128)
+    k[0, 0, 0, 3] = np.linspace(-60000, 60000, 128)
+    v[0, 0, 1, 4] = -0.0
+    v[0, 0, 1, 5, 0] = 65504.0
+    v[0, 0, 1, 5, 1] = -65504.0
+    p.k, p.v = k.astype(np.float16), v.astype(np.float16)
+    p.quantize()
+    p.assert_records_equal()
+
+
+# ---------------------------------------------------------------- decode -----
+
+def check_attention(p, layer=0, qseed=0):
+    got, ref = p.decode(layer, qseed)
+    err, rel = attention_errors(got, ref)
+    assert err <= ATOL and rel <= RTOL_L2, (err, rel)
+    assert int(p.cache.dev_error.item()) == 0
+    return err, rel
+
+
+@pytest.mark.parametrize("L_hi,L_lo,B,NL,H,Hq,T,r", [
+    (5, 5, 1, 1, 1, 4, 1024, (0, 100)),     # tiny uniform 5-level, 4 query heads
+    (6, 5, 2, 2, 2, 8, 333, (26, 100)),     # mixed, ragged tiles, layer 1 checked too
+    (6, 5, 1, 1, 8, 32, 2048, (26, 100)),   # Llama-3.1-8B layer shape, short context
+    (2, 2, 1, 1, 2, 8, 100, (0, 1)),
+    (3, 4, 1, 1, 2, 8, 100, (1, 2)),
+    (7, 8, 1, 1, 2, 8, 100, (1, 2)),
+    (6, 5, 1, 1, 2, 2, 200, (1, 4)),        # GQA group of 1
+    (6, 5, 1, 1, 2, 16, 200, (1, 4)),       # GQA group of 8
+    (6, 5, 1, 1, 1, 3, 150, (1, 4)),        # GQA group of 3
+    (6, 5, 1, 1, 1, 4, 1, (0, 1)),          # a single token
+    (6, 5, 1, 1, 1, 4, 40, (1, 1)),         # every token high
+])
+def test_decode_attention_matches_oracle(L_hi, L_lo, B, NL, H, Hq, T, r):
+    p = Pair(0, L_hi, L_lo, B, NL, H, Hq, T, r[0], r[1], seed=7 + T)
+    p.quantize()
+    for layer in range(NL):
+        check_attention(p, layer)
+
+
+def test_decode_attention_with_staged_tail():
+    p = Pair(0, 6, 5, 2, 1, 2, 8, 300, 26, 100, seed=11, block=32)
+    p.quantize()
+    k, v = synthetic.kv(12, 2, 1, 2, 20)
+    s = synthetic.scores_zipf(12, 2, 20)
+    import torch
+    for g in range(20):
+        kt = torch.from_numpy(np.ascontiguousarray(k[:, :, :, g])).to(p.dev)
+        vt = torch.from_numpy(np.ascontiguousarray(v[:, :, :, g])).to(p.dev)
+        p.cache.stage_token(kt, vt, torch.from_numpy(np.ascontiguousarray(s[:, g])).to(p.dev))
+        oracle.stage_token(p.oc, synthetic.f16_bits(k[:, :, :, g]), synthetic.f16_bits(v[:, :, :, g]),
+                           s[:, g])
+    check_attention(p)
+
+
+def test_append_blocks_and_flush_match_oracle():
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    blk, T0, ngen = 32, 200, 2 * 32 + 9
+    p = Pair(0, 6, 5, 2, 2, 2, 8, T0, 26, 100, seed=21, block=blk, extra_cap=ngen)
+    p.quantize()
+    k, v = synthetic.kv(22, 2, 2, 2, ngen)
+    s = synthetic.scores_zipf(22, 2, ngen)
+    for g in range(ngen):
+        kt = torch.from_numpy(np.ascontiguousarray(k[:, :, :, g])).to(p.dev)
+        vt = torch.from_numpy(np.ascontiguousarray(v[:, :, :, g])).to(p.dev)
+        p.cache.stage_token(kt, vt, torch.from_numpy(np.ascontiguousarray(s[:, g])).to(p.dev))
+        oracle.stage_token(p.oc, synthetic.f16_bits(k[:, :, :, g]), synthetic.f16_bits(v[:, :, :, g]),
+                           s[:, g])
+        if p.cache.stage_n == blk:
+            semkv.semkv_append_block(p.desc, p.cache, 26, 100)
+            oracle.append_block(p.oc, 26, 100)
+            torch.cuda.synchronize()
+            p.assert_records_equal()
+        if g % 13 == 0:
+            check_attention(p, layer=g % 2, qseed=g)
+    semkv.semkv_append_block(p.desc, p.cache, 26, 100)   # end-of-turn flush
+    oracle.append_block(p.oc, 26, 100)
+    torch.cuda.synchronize()
+    p.assert_records_equal()
+    assert p.cache.stage_n == 0 and p.cache.n_tokens == T0 + ngen
+    check_attention(p, layer=1, qseed=99)

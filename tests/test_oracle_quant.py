@@ -72,6 +72,15 @@ def test_affine_constant_row_and_hand_example():
     assert list(codes[:6]) == [0, 4, 0, 2, 2, 3]
 
 
+def test_affine_signed_zero_offset_is_positive():
+    # all-zero rows with either zero sign store offset +0 and scale +0
+    x = np.zeros(128, np.float16)
+    x[::3] = -0.0
+    for row in (x, -x, np.full(128, -0.0, np.float16)):
+        codes, s16, z16 = oracle.affine_row(f16(row), 5)
+        assert s16 == 0 and z16 == 0 and not codes.any()
+
+
 @pytest.mark.parametrize("L", [5, 6])
 def test_affine_matches_fp64_nearest_level(L):
     # away from half-way points the code is the nearest level z + s*k (fp64 search)
