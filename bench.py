@@ -1,0 +1,433 @@
+"""Benchmark of the SemKV packed mixed-precision KV cache on GB300.
+
+Workload (default): one layer of the Llama-3.1-8B KV shape (8 KV heads, 32 query
+heads, head_dim 128), batch 16 x 65536-token context, affine 6/5 levels with the
+top 26% of tokens (Zipf(1.1) scores) at 6 levels, block B = 128.  Inputs are seeded
+synthetic tensors (fp16 N(0,1) K/V with 4 outlier channels x8 per head), standing
+in for LongBench prompts run through the model.
+
+One step = one pass of the generation-time hot path over the batch:
+  A6  block-exact deferred quantization of a block of 128 staged tokens
+      (semkv_append_block: top-r rank in the block, quantize, pack, append), and
+  A7  decode attention for all 32 query heads over the whole cache
+      (65536 prompt tokens + the appended block), split-K + combine.
+The appended slots are reused every step (counts rewound), so the work per step is
+constant.  The prompt's own rank + quantize (A1-A5 at full size) is timed apart and
+reported as quantize_gbs.
+
+value = algorithmic bytes of the step (records read by decode attention, q and out,
+plus the block's fp16 K/V read and records written) / step time, in GB/s: decode
+dominates (722 MB of records per step, larger than the 129 MB L2, so every timed step
+streams from HBM).  roofline: decode attention's bytes per launch / its mean launch
+time (CUDA events on the launching stream) against the measured HBM copy peak.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+for _v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")   # the CPU oracle baseline runs on one core
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_28911_gb300 import synthetic  # noqa: E402
+
+METRIC = ("packed-KV decode attention µs/step and HBM GB/s (% of peak); quantize GB/s")
+
+CONFIGS = {
+    # name: batch, context, layers, kv heads, q heads, L_hi, L_lo, r, block, seed
+    "b16x64k": dict(B=16, T=65536, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100), block=128,
+                    seed=3, desc="batch 16 x 64K context, 1 layer of the Llama-3.1-8B KV shape "
+                                 "(8 KV heads, 32 q heads, d=128), affine 6/5 levels at r=26%"),
+    "b4x64k": dict(B=4, T=65536, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100), block=128,
+                   seed=3, desc="batch 4 x 64K context, 1 layer of the Llama-3.1-8B KV shape "
+                                "(8 KV heads, 32 q heads, d=128), affine 6/5 levels at r=26% "
+                                "(profiling size: 180 MB of records, above L2)"),
+    "b1x32k": dict(B=1, T=32768, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100), block=128,
+                   seed=2, desc="batch 1 x 32K context, 1 layer of the Llama-3.1-8B KV shape, "
+                                "affine 6/5 levels at r=26%"),
+}
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples taken while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.25)
+        return self
+
+    def __exit__(self, *exc):
+        time.sleep(0.15)
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in self.lines:
+            parts = [p.strip() for p in l.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------ GPU arm ---------
+
+def build_workload(cfg, dev):
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    B, T, NL, H, Hq = cfg["B"], cfg["T"], cfg["NL"], cfg["H"], cfg["Hq"]
+    r_num, r_den = cfg["r"]
+    blk = cfg["block"]
+    n_high = semkv.semkv_high_count_floor(T, r_num, r_den)
+    n_high_blk = semkv.semkv_block_high_count(blk, r_num, r_den)
+    desc = semkv.QuantDesc(semkv.BASE_AFFINE, cfg["L_hi"], cfg["L_lo"], device=dev)
+    cache = semkv.KVCache(desc, B, NL, H, Hq, hi_cap=n_high + n_high_blk,
+                          lo_cap=T - n_high + blk - n_high_blk, block=blk, device=dev)
+    k = torch.empty((B, NL, H, T, 128), dtype=torch.float16, device=dev)
+    v = torch.empty_like(k)
+    scores = torch.empty((B, T), dtype=torch.float32, device=dev)
+    for b in range(B):   # one seeded stream per sequence keeps host memory small
+        kb, vb = synthetic.kv(cfg["seed"] * 100 + b, 1, NL, H, T)
+        k[b].copy_(torch.from_numpy(kb[0]))
+        v[b].copy_(torch.from_numpy(vb[0]))
+        scores[b].copy_(torch.from_numpy(synthetic.scores_zipf(cfg["seed"] * 100 + b, 1, T)[0]))
+    return dict(desc=desc, cache=cache, k=k, v=v, scores=scores, n_high=n_high,
+                n_high_blk=n_high_blk)
+
+
+def step_bytes(cfg, cache, desc):
+    """Algorithmic bytes of one step (see module docstring)."""
+    from paper_2608_28911_gb300 import semkv
+    B, H, Hq, blk = cfg["B"], cfg["H"], cfg["Hq"], cfg["block"]
+    rh = semkv.semkv_record_bytes(desc.base, desc.levels_hi)
+    rl = semkv.semkv_record_bytes(desc.base, desc.levels_lo)
+    nh_b = semkv.semkv_block_high_count(blk, *cfg["r"])
+    hi = cache.hi_count + nh_b
+    lo = cache.lo_count + blk - nh_b
+    decode = B * H * (hi * rh + lo * rl) + B * Hq * 128 * (2 + 4)   # one layer
+    append = B * cfg["NL"] * H * (blk * 2 * 128 * 2 + nh_b * rh + (blk - nh_b) * rl) + B * blk * 4
+    return decode, append
+
+
+def gpu_arm(args, cfg, rank, world):
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    w = build_workload(cfg, dev)
+    desc, cache = w["desc"], w["cache"]
+    B, T, NL, H, Hq, blk = cfg["B"], cfg["T"], cfg["NL"], cfg["H"], cfg["Hq"], cfg["block"]
+    r_num, r_den = cfg["r"]
+
+    # ---- prompt: rank + quantize + pack (A1-A5), timed for quantize GB/s
+    is_high = torch.empty((B, T), dtype=torch.uint8, device=dev)
+    slot = torch.empty((B, T), dtype=torch.int32, device=dev)
+    qt = []
+    for it in range(4):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        semkv.semkv_rank_assign(w["scores"], w["n_high"], is_high, slot)
+        semkv.semkv_quantize_pack(desc, w["k"], w["v"], is_high, slot, w["n_high"], cache)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if it > 0:
+            qt.append(e0.elapsed_time(e1) * 1e-3)
+    rh = semkv.semkv_record_bytes(desc.base, desc.levels_hi)
+    rl = semkv.semkv_record_bytes(desc.base, desc.levels_lo)
+    q_bytes = B * NL * H * (T * 2 * 128 * 2 + w["n_high"] * rh + (T - w["n_high"]) * rl) + B * T * 4
+    quantize_gbs = q_bytes / statistics.median(qt) / 1e9
+    del w["k"], w["v"]
+
+    # ---- generation-time step: stage a block, append it (A6), decode (A7)
+    nblocks = 4
+    gk, gv = synthetic.kv(cfg["seed"] * 100 + 99, B, NL, H, blk * nblocks)
+    gs = synthetic.scores_zipf(cfg["seed"] * 100 + 99, B, blk * nblocks)
+    blocks_k = torch.from_numpy(gk).to(dev)
+    blocks_v = torch.from_numpy(gv).to(dev)
+    blocks_s = torch.from_numpy(gs).to(dev)
+    q_all = torch.from_numpy(np.stack([synthetic.queries(cfg["seed"], B, Hq, step=i)
+                                       for i in range(nblocks)])).to(dev)
+    out = torch.empty((B, Hq, 128), dtype=torch.float32, device=dev)
+    ws = cache.workspace()
+    scale = 1.0 / math.sqrt(128)
+    base_counts = (cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens)
+
+    def stage_block(i):
+        j = i % nblocks
+        cache.stage_k.copy_(blocks_k[:, :, :, j * blk:(j + 1) * blk])
+        cache.stage_v.copy_(blocks_v[:, :, :, j * blk:(j + 1) * blk])
+        cache.stage_score.copy_(blocks_s[:, j * blk:(j + 1) * blk])
+        cache.s.stage_n = blk
+
+    def step(i, ev=None):
+        cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+        stage_block(i)
+        semkv.semkv_append_block(desc, cache, r_num, r_den)
+        if ev is not None:
+            ev[0].record(stream)
+        semkv.semkv_decode_attention(desc, cache, 0, q_all[i % nblocks], out, scale, ws)
+        if ev is not None:
+            ev[1].record(stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    dec_bytes, app_bytes = step_bytes(cfg, cache_after_rewind(cache, base_counts), desc)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index) as clk:
+        barrier()
+        t0.record(stream)
+        for i in range(args.steps):
+            step(i, evs[i])
+        t1.record(stream)
+        barrier()
+    elapsed = t0.elapsed_time(t1) * 1e-3
+    dec_times = [a.elapsed_time(b) * 1e-3 for a, b in evs]
+    err = int(cache.dev_error.item())
+
+    # ---- end to end through the public API with host buffers
+    # per-block contiguous pinned host buffers, as a serving loop would hand them over
+    pin_k = [torch.from_numpy(np.ascontiguousarray(gk[:, :, :, j * blk:(j + 1) * blk])).pin_memory()
+             for j in range(nblocks)]
+    pin_v = [torch.from_numpy(np.ascontiguousarray(gv[:, :, :, j * blk:(j + 1) * blk])).pin_memory()
+             for j in range(nblocks)]
+    pin_s = [torch.from_numpy(np.ascontiguousarray(gs[:, j * blk:(j + 1) * blk])).pin_memory()
+             for j in range(nblocks)]
+    pin_q = q_all.cpu().pin_memory()
+    pin_out = torch.empty((B, Hq, 128), dtype=torch.float32).pin_memory()
+    h2d = (blk * B * NL * H * 128 * 2 * 2) + blk * B * 4 + B * Hq * 128 * 2
+    d2h = B * Hq * 128 * 4
+    qdev = torch.empty((B, Hq, 128), dtype=torch.float16, device=dev)
+
+    def step_e2e(i):
+        j = i % nblocks
+        cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+        cache.stage_k.copy_(pin_k[j], non_blocking=True)
+        cache.stage_v.copy_(pin_v[j], non_blocking=True)
+        cache.stage_score.copy_(pin_s[j], non_blocking=True)
+        qdev.copy_(pin_q[j], non_blocking=True)
+        cache.s.stage_n = blk
+        semkv.semkv_append_block(desc, cache, r_num, r_den)
+        semkv.semkv_decode_attention(desc, cache, 0, qdev, out, scale, ws)
+        pin_out.copy_(out, non_blocking=True)
+
+    e2e_steps = max(3, min(args.steps, 200))
+    for i in range(3):
+        step_e2e(i)
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(e2e_steps):
+        step_e2e(i)
+    e1.record(stream)
+    barrier()
+    e2e_time = e0.elapsed_time(e1) * 1e-3 / e2e_steps
+
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([elapsed, e2e_time], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed, e2e_time = float(t[0]), float(t[1])
+    return dict(elapsed=elapsed, dec_times=dec_times, dec_bytes=dec_bytes, app_bytes=app_bytes,
+                quantize_gbs=quantize_gbs, clocks=clk.summary(), err=err, e2e_time=e2e_time,
+                h2d=h2d, d2h=d2h)
+
+
+def cache_after_rewind(cache, base_counts):
+    cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+    return cache
+
+
+# ------------------------------------------------------------ CPU oracle ------
+
+def oracle_sample(cfg, budget_s: float, max_steps: int | None = None):
+    """The CPU oracle as it stands on a bounded sample of the same workload: one
+    (sequence, KV head) of the batch at full context -- append one block and run
+    fp64 decode attention for that head's 4 query heads -- repeated until the time
+    budget is spent.  Returns (GB/s of algorithmic bytes, sample description, steps)."""
+    import oracle
+    T, Hq, H, blk = cfg["T"], cfg["Hq"], cfg["H"], cfg["block"]
+    r_num, r_den = cfg["r"]
+    G = Hq // H
+    n_high = oracle.high_count_floor(T, r_num, r_den)
+    nh_b = oracle.block_high_count(blk, r_num, r_den)
+    oc = oracle.Cache(base=0, L_hi=cfg["L_hi"], L_lo=cfg["L_lo"], batch=1, layers=1, kv_heads=1,
+                      q_heads=G, block=blk, hi_cap=((n_high + nh_b + 15) // 16) * 16,
+                      lo_cap=((T - n_high + blk + 15) // 16) * 16)
+    kb, vb = synthetic.kv(cfg["seed"] * 100, 1, 1, H, T)
+    s = synthetic.scores_zipf(cfg["seed"] * 100, 1, T)
+    oracle.quantize_prompt(oc, synthetic.f16_bits(kb[:, :, :1]), synthetic.f16_bits(vb[:, :, :1]),
+                           s, r_num, r_den)
+    gk, gv = synthetic.kv(cfg["seed"] * 100 + 99, 1, 1, H, blk)
+    gs = synthetic.scores_zipf(cfg["seed"] * 100 + 99, 1, blk)
+    q = synthetic.f16_bits(synthetic.queries(cfg["seed"], 1, Hq)[:, :G])
+    base = (oc.hi_count, oc.lo_count, oc.n_tokens)
+    rh, rl = oracle.record_bytes(0, cfg["L_hi"]), oracle.record_bytes(0, cfg["L_lo"])
+    per_step = ((n_high + nh_b) * rh + (T - n_high + blk - nh_b) * rl + G * 128 * 6
+                + blk * 2 * 128 * 2 + nh_b * rh + (blk - nh_b) * rl + blk * 4)
+    steps, t_start = 0, time.perf_counter()
+    while True:
+        oc.hi_count, oc.lo_count, oc.n_tokens = base
+        oc.stage_k[0, 0, 0, :blk] = synthetic.f16_bits(gk[0, 0, 0])
+        oc.stage_v[0, 0, 0, :blk] = synthetic.f16_bits(gv[0, 0, 0])
+        oc.stage_score[0, :blk] = gs[0]
+        oc.stage_n = blk
+        oracle.append_block(oc, r_num, r_den)
+        oracle.decode_attention(oc, 0, q, 1 / math.sqrt(128))
+        steps += 1
+        el = time.perf_counter() - t_start
+        if (max_steps is not None and steps >= max_steps) or (max_steps is None and el >= budget_s):
+            break
+    sample = (f"1 of {cfg['B'] * H} (sequence, KV head) pairs at full {T}-token context: "
+              f"append one {blk}-token block + fp64 decode attention for its {G} query heads, "
+              f"x{steps} repetitions")
+    return per_step * steps / el / 1e9, sample, steps, el
+
+
+# ------------------------------------------------------------------ main ------
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="b16x64k", choices=sorted(CONFIGS))
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    cfg = CONFIGS[args.config]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    peaks, peak_kind = load_peaks()
+    config = {"workload": cfg["desc"], "batch": cfg["B"], "context": cfg["T"],
+              "layers": cfg["NL"], "kv_heads": cfg["H"], "q_heads": cfg["Hq"],
+              "levels": [cfg["L_hi"], cfg["L_lo"]], "r": f"{cfg['r'][0]}/{cfg['r'][1]}",
+              "block": cfg["block"], "l2": "inputs larger than L2 (records read per step > 129 MB)"
+              if cfg["B"] * cfg["T"] >= 100000 else "fits L2"}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        gbs, sample, steps, el = oracle_sample(cfg, 0, max_steps=args.warmup + args.steps)
+        line = {"impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s",
+                "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": el / steps * 1e3, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config,
+                "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                 "sample": sample},
+                "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return
+
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+        dist.init_process_group("nccl")
+    r = gpu_arm(args, cfg, rank, world)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    if rank != 0:
+        return
+    step_s = r["elapsed"] / args.steps
+    total_bytes = (r["dec_bytes"] + r["app_bytes"]) * world
+    dec_mean = sum(r["dec_times"]) / len(r["dec_times"])
+    achieved = r["dec_bytes"] / dec_mean / 1e9
+    peak = peaks["hbm_gbs"]
+    line = {
+        "metric": METRIC, "value": total_bytes / step_s / 1e9, "unit": "GB/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f16 codes x f16 -> f32 (mma), f32 softmax",
+        "data": "synthetic", "config": config,
+        "decode_us_per_step": dec_mean * 1e6,
+        "decode_gbs": achieved,
+        "decode_frac_of_peak": achieved / peak,
+        "decode_frac_of_nominal_8tbs": achieved / 8000.0,
+        "quantize_gbs": r["quantize_gbs"],
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None,
+                     "kernel": "decode_kernel+combine_kernel (semkv_decode_attention)",
+                     "peak_kind": f"{peak_kind} hbm_gbs"},
+        "e2e": {"value": total_bytes / r["e2e_time"] / 1e9, "unit": "GB/s",
+                "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
+        "gpu_launches": 4 * args.steps,
+        "clocks": r["clocks"],
+        "device_error": r["err"],
+    }
+    if world == 1 and args.cpu_seconds > 0:
+        gbs, sample, steps, el = oracle_sample(cfg, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": gbs, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                "sample": sample}
+    print(json.dumps(line))
+
+
+if __name__ == "__main__":
+    main()

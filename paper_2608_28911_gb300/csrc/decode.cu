@@ -10,19 +10,30 @@
 // tiles of ONE source (so its level count L is uniform), the warps taking tiles
 // round-robin; a final kernel merges the per-CTA partials (m, l, o) per (b, qh).
 //
-// Per warp and tile (affine, level L):
-//  - a 4-deep ring of cp.async.bulk copies (one 16-record tile each) completes on
-//    per-stage mbarriers; waits are bounded and report a timeout in the error word;
-//  - QK^T as S^T = Kc * Q^T on mma.sync m16n8k16 (M = 16 tokens, N = 8 query heads
-//    of the group, K = 128 dims): the A fragments are built straight from the packed
-//    symbols.  Each lane decodes a quarter row of two tokens; two symbols ride in the
-//    16-bit halves of a register and each digit is peeled with one multiply
-//    (y = x*L, digit = y >> W), landing as the fp16 value 8 + c.  q is permuted to
-//    match the decode order once per CTA;
-//  - logits = scale*log2e * (s*(acc - 8*sum q) + z*sum q); online softmax in base 2;
-//  - P V as O^T = Vc^T * P'^T (M = 128 dims, N = 8 heads, K = 16 tokens) with
-//    P' = p * s_v in fp16; the offset 8 and the zero point are added back per head
-//    from the same rounded P' (sum p' * 8) and from sum p * z_v.
+// Decoding on the FMA pipe.  A group symbol is stored as the W-bit integer
+// beta = ceil(t 2^W / L^G), so F_k = floor(beta L^(k+1) / 2^W) is the number formed by
+// the first k+1 digits and c_k = F_k - L F_{k-1}.  Read as an fp32 bit pattern, beta
+// is the denormal beta * 2^-149; one multiply rounded toward zero by the exact
+// constant L^(k+1)/2^W yields a float whose bit pattern is F_k.  Two symbols' F
+// values are paired into the 16-bit halves of a register with one integer
+// multiply-add, and one more multiply-add per digit position forms c_k lane-wise
+// (P_k - L P_{k-1}; digits are never negative, so nothing borrows across halves).
+// The integer c < 8 read as fp16 is the exact subnormal c * 2^-24: the tensor cores
+// take the digits as they are, and the 2^24 is folded into the scales.  (Feeding the
+// F values themselves and undoing the mixing after accumulation was tried and
+// rejected: the subtraction cancels ~30x and amplified the tensor cores' fp32
+// accumulation error past the attention tolerance.)
+//  - QK^T as S^T = C Q^T on mma.sync m16n8k16 (M = 16 tokens, N = 8 query heads of
+//    the group, K = 128 dims), q permuted to this decode order once per CTA;
+//    logit = scale log2e (s * 2^24 acc + z sum q), online softmax in base 2;
+//  - P V as O^T = C^T P'^T (M = 128 dims, N = 8 heads, K = 16 tokens) with
+//    P' = p * s_v in fp16, plus sum p * z_v per head.
+// Six-level groups (F_4 up to 7775 would not fit) restart the chain after two
+// digits from the remainder x = beta * 36 mod 2^13.
+//
+// Per warp: a 4-deep ring of cp.async.bulk tile copies completing on per-stage
+// mbarriers (bounded waits that report a timeout in the error word), online
+// softmax in base 2, lazy rescaling only when a running max grows.
 #include <float.h>
 
 #include "common.cuh"
@@ -41,9 +52,10 @@ constexpr int kStageBytes = kTile * kMaxRec + 16;  // +16: window loads may run 
 constexpr int kRingBytes = kWarps * kStages * kStageBytes;
 constexpr int kMaxSplits = 64;                     // pool splits per (b, h)
 constexpr uint32_t kSpinLimit = 1u << 22;
+constexpr float kTwo24 = 16777216.0f;              // a digit c enters the mma as c * 2^-24
 
 static_assert(kStageBytes % 16 == 0, "bulk copies need 16-byte aligned stages");
-static_assert(kRingBytes >= kWarps * (8 * 128 + 16) * 4, "merge area reuses the ring");
+static_assert(kRingBytes >= (kWarps * 8 * 128 + 8 * 128) * 4, "merge area reuses the ring");
 
 // ------------------------------------------------------------------ PTX -------
 
@@ -91,7 +103,20 @@ __device__ __forceinline__ void mma16816(float c[4], uint32_t a0, uint32_t a1, u
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
+// two 16-bit values into one register with a multiply-add (keeps the ALU pipe free)
+__device__ __forceinline__ uint32_t pair16(uint32_t lo, uint32_t hi) {
+  uint32_t r;
+  asm("mad.lo.u32 %0, %1, 65536, %2;" : "=r"(r) : "r"(hi), "r"(lo));
+  return r;
+}
+
+// F = floor(beta * c) for the exact constant c: beta read as a denormal float,
+// multiplied with rounding toward zero; the result's bit pattern is the integer F.
+__device__ __forceinline__ uint32_t fdig(uint32_t beta, float c) {
+  return __float_as_uint(__fmul_rz(__uint_as_float(beta), c));
+}
+
+__device__ __forceinline__ uint32_t h2(float lo, float hi) {
   return (uint32_t)__half_as_ushort(__float2half_rn(lo)) |
          ((uint32_t)__half_as_ushort(__float2half_rn(hi)) << 16);
 }
@@ -112,7 +137,7 @@ __device__ __forceinline__ Window load_window(const uint8_t* rec, int pos) {
   r.q2 = __funnelshift_r(w2, w3, sh);
   return r;
 }
-// bits [p, p+n) of a window, n <= 16 (p, n compile-time after unrolling)
+// bits [p, p+n) of a window (p, n compile-time after unrolling)
 __device__ __forceinline__ uint32_t wbits(const Window& w, int p, int n) {
   const uint32_t mask = (1u << n) - 1u;
   uint32_t v;
@@ -130,108 +155,144 @@ __device__ __forceinline__ uint32_t wbits_rt(const Window& w, int p, int n) {
   return __funnelshift_r(lo, hi, p & 31) & ((1u << n) - 1u);
 }
 
-// fp16 (8 + digit) in both halves: digit sits at bits [Wd, Wd+3) of each 16-bit lane
-template <int Wd>
-__device__ __forceinline__ uint32_t digit_half2(uint32_t y) {
-  uint32_t t;
-  if constexpr (Wd >= 7) t = y >> (Wd - 7);
-  else t = y << (7 - Wd);
-  return (t & 0x03800380u) | 0x48004800u;
-}
-
-// Peel the G digits of two symbols held in the 16-bit halves of x (most
-// significant first) into out[0..G).
-template <int L, int G, int Wd>
-__device__ __forceinline__ void peel(uint32_t x, uint32_t* out) {
-  constexpr uint32_t kMask = ((1u << Wd) - 1u) * 0x00010001u;
+template <int L>
+struct Dec {
+  using F = Fmt<L>;
+  static constexpr int G = F::G;
+  static constexpr int kHalf = F::NG / 2;                     // symbols per half quarter
+  static constexpr int kRestart = (L == 6) ? 2 : G;           // F chain restarts here
+  static constexpr bool kPow2 = (L & (L - 1)) == 0;
+  // F values of one full symbol
+  __device__ __forceinline__ static void sym(uint32_t beta, uint32_t* f) {
+    if constexpr (G == 1) {
+      f[0] = kPow2 ? beta : fdig(beta, (float)L / (float)(1u << F::W));
+    } else if constexpr (L == 6) {
+      constexpr float c1 = 6.0f / 8192.0f, c2 = 36.0f / 8192.0f, c3 = 216.0f / 8192.0f;
+      f[0] = fdig(beta, c1);
+      f[1] = fdig(beta, c2);
+      const uint32_t x = (beta * 36u) & 8191u;  // remainder after two digits
+      f[2] = fdig(x, c1);
+      f[3] = fdig(x, c2);
+      f[4] = fdig(x, c3);
+    } else {
+      float c = (float)L / (float)(1u << F::W);
 #pragma unroll
-  for (int k = 0; k < G; ++k) {
-    const uint32_t y = x * (uint32_t)L;
-    out[k] = digit_half2<Wd>(y);
-    x = y & kMask;
+      for (int k = 0; k < G; ++k) {
+        f[k] = fdig(beta, c);
+        c *= (float)L;
+      }
+    }
+  }
+  // F values of the two-code tail symbol
+  __device__ __forceinline__ static void tail(uint32_t beta, uint32_t* f) {
+    constexpr float c = (float)L / (float)(1u << F::WT);
+    f[0] = fdig(beta, c);
+    f[1] = fdig(beta, c * (float)L);
+  }
+  // does F slot k of a group carry a share of digit k+1?
+  __host__ __device__ static constexpr bool chained(int k) { return k + 1 < G && k + 1 != kRestart; }
+};
+
+// digits of two symbols from their F values, one register per digit position:
+// P_k = F_k(a) + 65536 F_k(b), digit_k = P_k - L P_{k-1} lane-wise (never negative,
+// so no borrow crosses the halves); the chain restarts at kRestart
+template <int L>
+__device__ __forceinline__ void pair_digits(const uint32_t* fa, const uint32_t* fb, uint32_t* h) {
+  using D = Dec<L>;
+  uint32_t prev = 0;
+#pragma unroll
+  for (int k = 0; k < D::G; ++k) {
+    const uint32_t P = pair16(fa[k], fb[k]);
+    if (k == 0 || k == D::kRestart) h[k] = P;
+    else asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(h[k]) : "r"(prev), "r"((uint32_t)(-L)), "r"(P));
+    prev = P;
   }
 }
 
-// The 16 half2 of one quarter row of one token (K side: both halves of a register
-// are codes of the same token).  Order p: symbol pairs (s, s + NG/2) digit by digit,
-// then the tail symbol's two codes.
+// K side: the 16 half2 of one quarter row of one token (both halves are digits of
+// the same token).  Slot p < kHalf*G holds digit k of symbols s and s + kHalf
+// (s = p / G, k = p % G); slot 15 holds the tail's two digits.
 template <int L>
-__device__ __forceinline__ void decode_quarter(const Window& w, uint32_t h[16]) {
-  using F = Fmt<L>;
-  constexpr int kHalf = F::NG / 2;
+__device__ __forceinline__ void k_quarter(const Window& w, uint32_t h[16]) {
+  using D = Dec<L>;
+  using F = typename D::F;
 #pragma unroll
-  for (int s = 0; s < kHalf; ++s) {
-    const uint32_t x = wbits(w, s * F::W, F::W) | (wbits(w, (s + kHalf) * F::W, F::W) << 16);
-    peel<L, F::G, F::W>(x, h + s * F::G);
+  for (int s = 0; s < D::kHalf; ++s) {
+    uint32_t fa[D::G], fb[D::G];
+    D::sym(wbits(w, s * F::W, F::W), fa);
+    D::sym(wbits(w, (s + D::kHalf) * F::W, F::W), fb);
+    pair_digits<L>(fa, fb, h + s * D::G);
   }
   if constexpr (F::R > 0) {
-    static_assert(F::R == 2 && kHalf * F::G == 15, "tail layout");
-    // the two tail digits: peel the tail symbol twice in one lane
-    const uint32_t t = wbits(w, F::NG * F::W, F::WT);
-    const uint32_t y0 = t * (uint32_t)L;
-    const uint32_t d0 = y0 >> F::WT;
-    const uint32_t y1 = (y0 & ((1u << F::WT) - 1u)) * (uint32_t)L;
-    const uint32_t d1 = y1 >> F::WT;
-    h[15] = ((d0 << 7) | (d1 << 23)) | 0x48004800u;
+    static_assert(F::R == 2 && D::kHalf * D::G == 15, "tail layout");
+    uint32_t ft[2];
+    D::tail(wbits(w, F::NG * F::W, F::WT), ft);
+    uint32_t d1;
+    asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(d1) : "r"(ft[0]), "r"((uint32_t)(-L)), "r"(ft[1]));
+    h[15] = pair16(ft[0], d1);
   } else {
-    static_assert(kHalf * F::G == 16, "layout");
+    static_assert(D::kHalf * D::G == 16, "layout");
   }
 }
 
-// dims (lo half, hi half) of K-side half2 p of quarter t
+// dims (lo half, hi half) of K-side slot p of quarter t
 template <int L>
 __device__ __forceinline__ void k_dims(int t, int p, int& dlo, int& dhi) {
-  using F = Fmt<L>;
-  constexpr int kHalf = F::NG / 2;
+  using D = Dec<L>;
+  using F = typename D::F;
   if (F::R > 0 && p == 15) {
     dlo = 32 * t + 30;
     dhi = 32 * t + 31;
   } else {
-    const int s = p / F::G, k = p % F::G;
-    dlo = 32 * t + s * F::G + k;
-    dhi = 32 * t + (s + kHalf) * F::G + k;
+    const int s = p / D::G, k = p % D::G;
+    dlo = 32 * t + s * D::G + k;
+    dhi = 32 * t + (s + D::kHalf) * D::G + k;
   }
 }
 
-// V side: lane group g decodes half `hh` of quarter qv for two tokens at once (the
-// halves of each register are the two tokens).  Output u = 0..15: symbol s' digit k
-// at u = s'*G + k, then (when present) tail digit hh at u = 15.
+// V side: lane group g holds half hh of quarter qv for two tokens at once (the two
+// halves of each register are the two tokens).  Row u = j*G + k is digit k of
+// symbol hh*kHalf + j; row 15 is the tail's digit hh.
 template <int L>
-__device__ __forceinline__ void decode_half_quarter_pair(const Window& wa, const Window& wb,
-                                                         const Window& ta, const Window& tb,
-                                                         int hh, uint32_t h[16]) {
-  using F = Fmt<L>;
-  constexpr int kHalf = F::NG / 2;
+__device__ __forceinline__ void v_half_pair(const Window& wa, const Window& wb, int tpos, int hh,
+                                            uint32_t h[16]) {
+  using D = Dec<L>;
+  using F = typename D::F;
 #pragma unroll
-  for (int s = 0; s < kHalf; ++s) {
-    const uint32_t x = wbits(wa, s * F::W, F::W) | (wbits(wb, s * F::W, F::W) << 16);
-    peel<L, F::G, F::W>(x, h + s * F::G);
+  for (int j = 0; j < D::kHalf; ++j) {
+    uint32_t fa[D::G], fb[D::G];
+    D::sym(wbits(wa, j * F::W, F::W), fa);
+    D::sym(wbits(wb, j * F::W, F::W), fb);
+    pair_digits<L>(fa, fb, h + j * D::G);
   }
   if constexpr (F::R > 0) {
-    const uint32_t x = wbits(ta, F::NG * F::W, F::WT) | (wbits(tb, F::NG * F::W, F::WT) << 16);
-    const uint32_t y0 = x * (uint32_t)L;
-    const uint32_t y1 = (y0 & (((1u << F::WT) - 1u) * 0x00010001u)) * (uint32_t)L;
-    h[15] = digit_half2<F::WT>(hh ? y1 : y0);
+    uint32_t fa[2], fb[2];
+    D::tail(wbits_rt(wa, tpos, F::WT), fa);
+    D::tail(wbits_rt(wb, tpos, F::WT), fb);
+    const uint32_t P0 = pair16(fa[0], fb[0]), P1 = pair16(fa[1], fb[1]);
+    uint32_t d1;
+    asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(d1) : "r"(P0), "r"((uint32_t)(-L)), "r"(P1));
+    h[15] = hh ? d1 : P0;
   }
 }
 
+// output dim of V row u of lane group g
 template <int L>
 __device__ __forceinline__ int v_dim(int g, int u) {
-  using F = Fmt<L>;
-  constexpr int kHalf = F::NG / 2;
+  using D = Dec<L>;
+  using F = typename D::F;
   const int qv = g >> 1, hh = g & 1;
   if (F::R > 0 && u == 15) return 32 * qv + 30 + hh;
-  const int s = u / F::G, k = u % F::G;
-  return 32 * qv + (hh * kHalf + s) * F::G + k;
+  const int s = u / D::G, k = u % D::G;
+  return 32 * qv + (hh * D::kHalf + s) * D::G + k;
 }
 
 // ------------------------------------------------------- per-warp state -------
 
 struct WarpState {
-  float O[8][4];     // O^T accumulators: rows (dims) x columns (heads 2t, 2t+1)
-  float m[2];        // running max (base-2 logits) of heads 2t, 2t+1
+  float O[8][4];     // O^T accumulators: V rows x columns (heads 2t, 2t+1)
+  float m[2];        // running max (base-2 logits) of this lane's two heads
   float l[2];        // partial sum of p over this lane's tokens
-  float poff[2];     // partial sum of the rounded p*s_v (offset correction)
   float zs[2];       // partial sum of p*z_v
 };
 
@@ -244,7 +305,6 @@ __device__ __forceinline__ void state_init(WarpState& st) {
   for (int e = 0; e < 2; ++e) {
     st.m[e] = -INFINITY;
     st.l[e] = 0.0f;
-    st.poff[e] = 0.0f;
     st.zs[e] = 0.0f;
   }
 }
@@ -260,7 +320,8 @@ template <int L>
 __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
                          uint64_t* bars, const uint8_t* pool_bh, int64_t count, int t_begin,
                          int t_end, int G, WarpState& st) {
-  using F = Fmt<L>;
+  using D = Dec<L>;
+  using F = typename D::F;
   constexpr int kRec = 2 * F::RB + 8;
   constexpr uint32_t kTileBytes = kTile * kRec;
   static_assert(kTileBytes % 16 == 0, "tile size must be a multiple of 16 bytes");
@@ -269,7 +330,7 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
   uint8_t* my_ring = ring + warp * kStages * kStageBytes;
   uint64_t* my_bar = bars + warp * kStages;
 
-  // q fragments (B of S^T = Kc Q^T): column n = g, rows = this quarter's decode order
+  // B fragments of S^T = C Q^T: column n = g (head g), rows = this quarter's slots
   uint32_t bq[16];
 #pragma unroll
   for (int p = 0; p < 16; ++p) {
@@ -279,17 +340,16 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
   }
   float sumq[2];
 #pragma unroll
-  for (int e = 0; e < 2; ++e) {
+  for (int c = 0; c < 2; ++c) {
     float s = 0.0f;
-    for (int d = 0; d < 128; ++d) s += f16_to_f32(sh.q[2 * t + e][d]);
-    sumq[e] = s;
+    for (int d = 0; d < 128; ++d) s += f16_to_f32(sh.q[2 * t + c][d]);
+    sumq[c] = s;
   }
   const int qv = g >> 1, hh = g & 1;
-  const int vpos = 8 * F::RB + qv * F::QB + hh * (F::NG / 2) * F::W;  // V half-quarter
-  const int vtail = 8 * F::RB + qv * F::QB;                           // V quarter (tail)
+  const int vpos = 8 * F::RB + qv * F::QB + hh * D::kHalf * F::W;  // V half quarter
+  const int tpos = F::NG * F::W - hh * D::kHalf * F::W;           // tail, relative
 
   const int nmine = t_end - t_begin <= warp ? 0 : (t_end - t_begin - warp + kWarps - 1) / kWarps;
-  // prologue: fill the ring
   if (lane == 0) {
     for (int i = 0; i < kStages && i < nmine; ++i) {
       const int tile = t_begin + warp + i * kWarps;
@@ -311,22 +371,24 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
     const uint8_t* tb = my_ring + stage * kStageBytes;
     const int nvalid = (int)min((int64_t)kTile, count - (int64_t)tile * kTile);
 
-    // ---- S^T = Kc Q^T
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    // ---- S^T = C Q^T (two accumulators: two short dependency chains)
+    float acc[4] = {0.f, 0.f, 0.f, 0.f}, acc2[4] = {0.f, 0.f, 0.f, 0.f};
     {
       uint32_t h0[16], h1[16];
-      decode_quarter<L>(load_window(tb + g * kRec, t * F::QB), h0);
-      decode_quarter<L>(load_window(tb + (g + 8) * kRec, t * F::QB), h1);
+      k_quarter<L>(load_window(tb + g * kRec, t * F::QB), h0);
+      k_quarter<L>(load_window(tb + (g + 8) * kRec, t * F::QB), h1);
 #pragma unroll
       for (int j = 0; j < 8; ++j)
-        mma16816(acc, h0[2 * j], h1[2 * j], h0[2 * j + 1], h1[2 * j + 1], bq[2 * j], bq[2 * j + 1]);
+        mma16816((j & 1) ? acc2 : acc, h0[2 * j], h1[2 * j], h0[2 * j + 1], h1[2 * j + 1],
+                 bq[2 * j], bq[2 * j + 1]);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[e] += acc2[e];
     }
     // ---- logits and online softmax (base 2)
-    float p[2][2], ph_sum[2] = {0.f, 0.f}, zadd[2] = {0.f, 0.f};
+    float p[2][2];
     uint32_t X[2];
     {
-      float lg[2][2];
-      float sv[2], zv[2];
+      float lg[2][2], sv[2], zv[2];
       bool valid[2];
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
@@ -337,8 +399,8 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
         sv[e] = f16_to_f32((uint16_t)(vp & 0xFFFF));
         zv[e] = f16_to_f32((uint16_t)(vp >> 16));
         valid[e] = tok < nvalid;
-        const float A = a.scale_log2 * sk;
-        const float Bz = a.scale_log2 * (zk - 8.0f * sk);
+        const float A = a.scale_log2 * kTwo24 * sk;
+        const float Bz = a.scale_log2 * zk;
 #pragma unroll
         for (int c = 0; c < 2; ++c)
           lg[e][c] = valid[e] ? fmaf(A, acc[2 * e + c], Bz * sumq[c]) : -INFINITY;
@@ -360,7 +422,6 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
           al[c] = (st.m[c] == -INFINITY) ? 0.0f : exp2f(st.m[c] - mnew[c]);
           st.m[c] = mnew[c];
           st.l[c] *= al[c];
-          st.poff[c] *= al[c];
           st.zs[c] *= al[c];
         }
 #pragma unroll
@@ -375,17 +436,9 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
       for (int c = 0; c < 2; ++c) {
 #pragma unroll
         for (int e = 0; e < 2; ++e) p[e][c] = valid[e] ? exp2f(lg[e][c] - st.m[c]) : 0.0f;
-      }
-#pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        const __half a0 = __float2half_rn(p[0][c] * sv[0]);
-        const __half a1 = __float2half_rn(p[1][c] * sv[1]);
-        X[c] = (uint32_t)__half_as_ushort(a0) | ((uint32_t)__half_as_ushort(a1) << 16);
-        ph_sum[c] = __half2float(a0) + __half2float(a1);
-        zadd[c] = p[0][c] * zv[0] + p[1][c] * zv[1];
+        X[c] = h2(p[0][c] * sv[0], p[1][c] * sv[1]);
         st.l[c] += p[0][c] + p[1][c];
-        st.poff[c] += ph_sum[c];
-        st.zs[c] += zadd[c];
+        st.zs[c] += p[0][c] * zv[0] + p[1][c] * zv[1];
       }
     }
     // ---- P'^T into the B fragment: column g (head g), rows = tokens 2t, 2t+1, 2t+8, 2t+9
@@ -401,25 +454,18 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
       b0 = g < G ? __byte_perm(A, B, 0x5410) : 0u;
       b1 = g < G ? __byte_perm(A, B, 0x7632) : 0u;
     }
-    // ---- O^T += Vc^T P'^T
+    // ---- O^T += C^T P'^T
     {
       uint32_t ha[16], hb[16];
-      const Window wa0 = load_window(tb + (2 * t) * kRec, vpos);
-      const Window wa1 = load_window(tb + (2 * t + 1) * kRec, vpos);
-      const Window ta0 = load_window(tb + (2 * t) * kRec, vtail);
-      const Window ta1 = load_window(tb + (2 * t + 1) * kRec, vtail);
-      decode_half_quarter_pair<L>(wa0, wa1, ta0, ta1, hh, ha);
-      const Window wb0 = load_window(tb + (2 * t + 8) * kRec, vpos);
-      const Window wb1 = load_window(tb + (2 * t + 9) * kRec, vpos);
-      const Window tb0 = load_window(tb + (2 * t + 8) * kRec, vtail);
-      const Window tb1 = load_window(tb + (2 * t + 9) * kRec, vtail);
-      decode_half_quarter_pair<L>(wb0, wb1, tb0, tb1, hh, hb);
+      v_half_pair<L>(load_window(tb + (2 * t) * kRec, vpos),
+                     load_window(tb + (2 * t + 1) * kRec, vpos), tpos, hh, ha);
+      v_half_pair<L>(load_window(tb + (2 * t + 8) * kRec, vpos),
+                     load_window(tb + (2 * t + 9) * kRec, vpos), tpos, hh, hb);
 #pragma unroll
       for (int m = 0; m < 8; ++m)
         mma16816(st.O[m], ha[2 * m], ha[2 * m + 1], hb[2 * m], hb[2 * m + 1], b0, b1);
     }
     __syncwarp();
-    // refill this stage with the tile kStages ahead
     if (lane == 0 && it + kStages < nmine) {
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       const int nt = t_begin + warp + (it + kStages) * kWarps;
@@ -441,8 +487,9 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
 // ------------------------------------------------------- fp16 stage tokens ----
 
 // Staged tokens are few (< block): one warp per token, lane = 4 dims, CUDA cores.
+// Writes rows in natural dim order and zs = 0.
 __device__ void run_stage(const DecodeArgs& a, const Shared& sh, int b, int h, int G,
-                          float* m_out, float* l_out, float* o_out /* [8][128] */) {
+                          float* m_out, float* l_out, float* z_out, float* o_out) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   float qf[8][4];
 #pragma unroll
@@ -487,6 +534,7 @@ __device__ void run_stage(const DecodeArgs& a, const Shared& sh, int b, int h, i
     if (lane == 0) {
       m_out[warp * 8 + c] = m[c];
       l_out[warp * 8 + c] = l[c];
+      z_out[warp * 8 + c] = 0.0f;
     }
 #pragma unroll
     for (int j = 0; j < 4; ++j) o_out[(warp * 8 + c) * 128 + 4 * lane + j] = o[c][j];
@@ -498,9 +546,10 @@ __device__ void run_stage(const DecodeArgs& a, const Shared& sh, int b, int h, i
 __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
   extern __shared__ __align__(128) uint8_t dyn[];
   __shared__ Shared sh;
-  __shared__ float merge_m[kWarps * 8], merge_l[kWarps * 8];
+  __shared__ float merge_m[kWarps * 8], merge_l[kWarps * 8], merge_z[kWarps * 8];
+  __shared__ float cta_scale[kWarps * 8], cta_z[8];
   uint8_t* ring = dyn;
-  float* merge_o = reinterpret_cast<float*>(dyn);  // [kWarps][8][128], after the loop
+  float* merge_o = reinterpret_cast<float*>(dyn);  // [kWarps][8][128] output rows
 
   const int b = blockIdx.z, h = blockIdx.y, split = blockIdx.x;
   const int G = a.Hq / a.H;
@@ -511,13 +560,10 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
     const int c = i >> 7, d = i & 127;
     sh.q[c][d] = c < G ? a.q[((int64_t)b * a.Hq + h * G + c) * 128 + d] : (uint16_t)0;
   }
-  if (threadIdx.x < kWarps * kStages) {
-    mbar_init(&sh.bar[0][0] + threadIdx.x);
-  }
+  if (threadIdx.x < kWarps * kStages) mbar_init(&sh.bar[0][0] + threadIdx.x);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncthreads();
 
-  // which source and which tiles
   int src, s_idx, nsrc, ntiles;
   if (split < P.splits_hi) {
     src = 0; s_idx = split; nsrc = P.splits_hi; ntiles = P.tiles_hi;
@@ -528,27 +574,27 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
   }
   const int per = (ntiles + nsrc - 1) / nsrc;
   const int t_begin = min(ntiles, s_idx * per), t_end = min(ntiles, t_begin + per);
+  const int L = src == 0 ? a.L_hi : a.L_lo;
 
   if (src == 2) {
-    __syncthreads();
-    run_stage(a, sh, b, h, G, merge_m, merge_l, merge_o);
+    run_stage(a, sh, b, h, G, merge_m, merge_l, merge_z, merge_o);
   } else {
     WarpState st;
     state_init(st);
-    const int L = src == 0 ? a.L_hi : a.L_lo;
     const int64_t cap = src == 0 ? a.hi_cap : a.lo_cap;
     const int64_t count = src == 0 ? a.hi_count : a.lo_count;
     const uint8_t* pool = src == 0 ? a.hi_pool : a.lo_pool;
     const int rec = record_bytes_rt(SEMKV_BASE_AFFINE, L);
     const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
+    uint64_t* bars = &sh.bar[0][0];
     switch (L) {
-      case 2: run_pool<2>(a, sh, ring, &sh.bar[0][0], pool_bh, count, t_begin, t_end, G, st); break;
-      case 3: run_pool<3>(a, sh, ring, &sh.bar[0][0], pool_bh, count, t_begin, t_end, G, st); break;
-      case 4: run_pool<4>(a, sh, ring, &sh.bar[0][0], pool_bh, count, t_begin, t_end, G, st); break;
-      case 5: run_pool<5>(a, sh, ring, &sh.bar[0][0], pool_bh, count, t_begin, t_end, G, st); break;
-      case 6: run_pool<6>(a, sh, ring, &sh.bar[0][0], pool_bh, count, t_begin, t_end, G, st); break;
-      case 7: run_pool<7>(a, sh, ring, &sh.bar[0][0], pool_bh, count, t_begin, t_end, G, st); break;
-      case 8: run_pool<8>(a, sh, ring, &sh.bar[0][0], pool_bh, count, t_begin, t_end, G, st); break;
+      case 2: run_pool<2>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 3: run_pool<3>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 4: run_pool<4>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 5: run_pool<5>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 6: run_pool<6>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 7: run_pool<7>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 8: run_pool<8>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
       default: break;
     }
     // reduce the per-lane partial sums over the 8 token rows (lanes with equal t)
@@ -557,21 +603,27 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
 #pragma unroll
       for (int off = 4; off <= 16; off <<= 1) {
         st.l[c] += __shfl_xor_sync(0xffffffffu, st.l[c], off);
-        st.poff[c] += __shfl_xor_sync(0xffffffffu, st.poff[c], off);
         st.zs[c] += __shfl_xor_sync(0xffffffffu, st.zs[c], off);
       }
     }
     __syncthreads();  // every warp is done with the ring: reuse it as the merge area
     const int g = lane >> 2, t = lane & 3;
+    if (g == 0) {
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        if (2 * t + c < G) {
+          merge_m[warp * 8 + 2 * t + c] = st.m[c];
+          merge_l[warp * 8 + 2 * t + c] = st.l[c];
+          merge_z[warp * 8 + 2 * t + c] = st.zs[c];
+        }
+      }
+    }
+    // O columns are heads 2t, 2t+1; rows 16m + g (+8) are V rows u = 2m (+1) of
+    // lane group g, i.e. output dims v_dim(g, u)
 #pragma unroll
     for (int c = 0; c < 2; ++c) {
       const int qh = 2 * t + c;
       if (qh < G) {
-        const float corr = st.zs[c] - 8.0f * st.poff[c];
-        if (g == 0) {
-          merge_m[warp * 8 + qh] = st.m[c];
-          merge_l[warp * 8 + qh] = st.l[c];
-        }
 #pragma unroll
         for (int m = 0; m < 8; ++m) {
 #pragma unroll
@@ -586,7 +638,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
               case 7: dim = v_dim<7>(g, 2 * m + r); break;
               default: dim = v_dim<8>(g, 2 * m + r); break;
             }
-            merge_o[(warp * 8 + qh) * 128 + dim] = st.O[m][2 * r + c] + corr;
+            merge_o[(warp * 8 + qh) * 128 + dim] = st.O[m][2 * r + c];
           }
         }
       }
@@ -594,27 +646,40 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
   }
   __syncthreads();
 
-  // merge the warps into this CTA's partial (unnormalised o, base-2 max m, sum l)
+  // merge the warps: scale factors per (warp, head), then the rows
   float* part = a.partials + (((int64_t)b * a.H + h) * P.splits + split) * kPartialFloats;
-  for (int i = threadIdx.x; i < G * 128; i += kThreads) {
-    const int qh = i >> 7, d = i & 127;
+  if (threadIdx.x < 8) {
+    const int qh = threadIdx.x;
     float M = -INFINITY;
-    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + qh]);
-    float o = 0.0f, lsum = 0.0f;
-    if (M != -INFINITY) {
-      for (int w = 0; w < kWarps; ++w) {
-        const float mw = merge_m[w * 8 + qh];
-        if (mw == -INFINITY) continue;
-        const float sc = exp2f(mw - M);
-        o += sc * merge_o[(w * 8 + qh) * 128 + d];
+    if (qh < G)
+      for (int w = 0; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + qh]);
+    float lsum = 0.0f, zsum = 0.0f;
+    for (int w = 0; w < kWarps; ++w) {
+      const float mw = qh < G ? merge_m[w * 8 + qh] : -INFINITY;
+      const float sc = (M == -INFINITY || mw == -INFINITY) ? 0.0f : exp2f(mw - M);
+      cta_scale[w * 8 + qh] = sc;
+      if (sc != 0.0f) {
         lsum += sc * merge_l[w * 8 + qh];
+        zsum += sc * merge_z[w * 8 + qh];
       }
     }
-    part[16 + qh * 128 + d] = o;
-    if (d == 0) {
+    if (qh < G) {
       part[qh] = M;
       part[8 + qh] = lsum;
     }
+    cta_z[qh] = zsum;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < G * 128; i += kThreads) {
+    const int qh = i >> 7, d = i & 127;
+    float o = 0.0f;
+    for (int w = 0; w < kWarps; ++w) {
+      const float sc = cta_scale[w * 8 + qh];
+      if (sc != 0.0f) o += sc * merge_o[(w * 8 + qh) * 128 + d];
+    }
+    // pool rows hold sum p' c (c as the fp16 value c * 2^-24); the offset part is
+    // sum p z; staged rows are plain sums of p v
+    part[16 + qh * 128 + d] = src == 2 ? o : kTwo24 * o + cta_z[qh];
   }
 }
 
