@@ -14,20 +14,22 @@
 // beta = ceil(t 2^W / L^G), so F_k = floor(beta L^(k+1) / 2^W) is the number formed by
 // the first k+1 digits and c_k = F_k - L F_{k-1}.  Read as an fp32 bit pattern, beta
 // is the denormal beta * 2^-149; one multiply rounded toward zero by the exact
-// constant L^(k+1)/2^W yields a float whose bit pattern is F_k.  Two symbols' F
-// values are paired into the 16-bit halves of a register with one integer
-// multiply-add, and one more multiply-add per digit position forms c_k lane-wise
-// (P_k - L P_{k-1}; digits are never negative, so nothing borrows across halves).
-// The integer c < 8 read as fp16 is the exact subnormal c * 2^-24: the tensor cores
-// take the digits as they are, and the 2^24 is folded into the scales.  (Feeding the
-// F values themselves and undoing the mixing after accumulation was tried and
-// rejected: the subtraction cancels ~30x and amplified the tensor cores' fp32
-// accumulation error past the attention tolerance.)
-//  - QK^T as S^T = C Q^T on mma.sync m16n8k16 (M = 16 tokens, N = 8 query heads of
-//    the group, K = 128 dims), q permuted to this decode order once per CTA;
-//    logit = scale log2e (s * 2^24 acc + z sum q), online softmax in base 2;
-//  - P V as O^T = C^T P'^T (M = 128 dims, N = 8 heads, K = 16 tokens) with
-//    P' = p * s_v in fp16, plus sum p * z_v per head.
+// constant L^(k+1)/2^W yields a float whose bit pattern is F_k.  For five-level
+// groups two symbols share one multiply (beta_a + 65536 beta_b is still a denormal)
+// and a mask separates the halves.  Integers (all < 256) become fp16 values with a
+// byte permute (1024 + v) and one f16x2 subtract.
+//  - QK^T as S^T = F Q'^T on mma.sync m16n8k16 (M = 16 tokens, K = 128 F slots,
+//    N = 8 columns): the q coefficient of F_k is q'_k = q_{d_k} - L q_{d_{k+1}}
+//    when F_k carries a share of digit k+1, split into fp16 hi + lo parts (the lo
+//    parts ride in the spare columns 4..7 when G <= 4, else a second pass);
+//    logit = scale log2e (s acc + z sum q), online softmax in base 2, rescaling only
+//    when some logit exceeds the running max;
+//  - P V as O^T = C^T P'^T (M = 128 dims, N = 8 heads, K = 16 tokens) on the digits
+//    c_k (formed lane-wise as P_k - L P_{k-1}, never negative, so nothing borrows
+//    across halves), with P' = p * s_v as fp16 hi + lo (lo again in columns 4..7),
+//    plus sum p * z_v per head.  (Feeding F values to PV and undoing the mixing after
+//    accumulation was tried and rejected: the subtraction cancels ~30x and amplified
+//    the tensor cores' fp32 accumulation error past the attention tolerance.)
 // Six-level groups (F_4 up to 7775 would not fit) restart the chain after two
 // digits from the remainder x = beta * 36 mod 2^13.
 //
@@ -52,7 +54,6 @@ constexpr int kStageBytes = kTile * kMaxRec + 16;  // +16: window loads may run 
 constexpr int kRingBytes = kWarps * kStages * kStageBytes;
 constexpr int kMaxSplits = 64;                     // pool splits per (b, h)
 constexpr uint32_t kSpinLimit = 1u << 22;
-constexpr float kTwo24 = 16777216.0f;              // a digit c enters the mma as c * 2^-24
 
 static_assert(kStageBytes % 16 == 0, "bulk copies need 16-byte aligned stages");
 static_assert(kRingBytes >= (kWarps * 8 * 128 + 8 * 128) * 4, "merge area reuses the ring");
@@ -107,6 +108,18 @@ __device__ __forceinline__ void mma16816(float c[4], uint32_t a0, uint32_t a1, u
 __device__ __forceinline__ uint32_t pair16(uint32_t lo, uint32_t hi) {
   uint32_t r;
   asm("mad.lo.u32 %0, %1, 65536, %2;" : "=r"(r) : "r"(hi), "r"(lo));
+  return r;
+}
+
+// two integers < 256 in the 16-bit halves -> the same integers as fp16 values: the
+// byte 0x64 over each makes 1024 + v, and one f16x2 subtract of 1024 leaves v.  (The
+// integers read directly as fp16 subnormals v * 2^-24 were tried first: the tensor
+// cores lose products of subnormal operands with small weights, biasing attention by
+// ~1e-5 of the low-weight mass per mma.)
+__device__ __forceinline__ uint32_t ints_to_h2(uint32_t P) {
+  const uint32_t x = __byte_perm(P, 0x64646464u, 0x7250);
+  uint32_t r;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(x), "r"(0x64006400u));
   return r;
 }
 
@@ -193,9 +206,16 @@ struct Dec {
   __host__ __device__ static constexpr bool chained(int k) { return k + 1 < G && k + 1 != kRestart; }
 };
 
+// lane-wise P_k - L P_{k-1}: digits are never negative, so no borrow crosses halves
+template <int L>
+__device__ __forceinline__ uint32_t digit_step(uint32_t prev, uint32_t P) {
+  uint32_t r;
+  asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(r) : "r"(prev), "r"((uint32_t)(-L)), "r"(P));
+  return r;
+}
+
 // digits of two symbols from their F values, one register per digit position:
-// P_k = F_k(a) + 65536 F_k(b), digit_k = P_k - L P_{k-1} lane-wise (never negative,
-// so no borrow crosses the halves); the chain restarts at kRestart
+// P_k = F_k(a) + 65536 F_k(b), digit_k = P_k - L P_{k-1}; the chain restarts at kRestart
 template <int L>
 __device__ __forceinline__ void pair_digits(const uint32_t* fa, const uint32_t* fb, uint32_t* h) {
   using D = Dec<L>;
@@ -203,76 +223,144 @@ __device__ __forceinline__ void pair_digits(const uint32_t* fa, const uint32_t* 
 #pragma unroll
   for (int k = 0; k < D::G; ++k) {
     const uint32_t P = pair16(fa[k], fb[k]);
-    if (k == 0 || k == D::kRestart) h[k] = P;
-    else asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(h[k]) : "r"(prev), "r"((uint32_t)(-L)), "r"(P));
+    h[k] = (k == 0 || k == D::kRestart) ? P : digit_step<L>(prev, P);
     prev = P;
   }
 }
 
-// K side: the 16 half2 of one quarter row of one token (both halves are digits of
-// the same token).  Slot p < kHalf*G holds digit k of symbols s and s + kHalf
-// (s = p / G, k = p % G); slot 15 holds the tail's two digits.
+// ---- five-level fast path: two 7-bit symbols per register ---------------------
+// u = beta_a + 65536 beta_b is still a denormal (beta < 128), and
+// floor(u * L^(k+1)/128) = F_k(a) + 65536 F_k(b) + (fraction of b) * 512: one
+// multiply and one mask give both halves' F_k at once (F_k <= 124).
+constexpr uint32_t kM7 = 0x007F007Fu;
+__device__ __forceinline__ uint32_t lo16hi16(uint32_t a, uint32_t b) {
+  return __byte_perm(a, b, 0x5410);
+}
+__device__ __forceinline__ void l5_fpairs(uint32_t u, uint32_t* P) {
+  P[0] = fdig(u, 5.0f / 128.0f) & kM7;
+  P[1] = fdig(u, 25.0f / 128.0f) & kM7;
+  P[2] = fdig(u, 125.0f / 128.0f) & kM7;
+}
+// symbol pairs from two 96-bit windows: symbol j of window a in the low half and of
+// window b in the high half, j = 0..4 (bits 7j)
+__device__ __forceinline__ void l5_pairs(uint32_t a0, uint32_t a1, uint32_t b0, uint32_t b1,
+                                         uint32_t u[5]) {
+  uint32_t C = lo16hi16(a0, b0);
+  u[0] = C & kM7;
+  u[1] = (C >> 7) & kM7;
+  C = lo16hi16(a0 >> 14, b0 >> 14);
+  u[2] = C & kM7;
+  u[3] = (C >> 7) & kM7;
+  C = lo16hi16(__funnelshift_r(a0, a1, 28), __funnelshift_r(b0, b1, 28));
+  u[4] = C & kM7;
+}
+
+// K side: the 16 F-value pairs of one quarter row of one token (both halves are the
+// same token).  Slot p < kHalf*G holds F_k of symbols s and s + kHalf (s = p / G,
+// k = p % G); slot 15 holds the tail's F_0 and F_1.
+template <int L>
+__device__ __forceinline__ void k_quarter_ints(const Window& w, uint32_t h[16]);
 template <int L>
 __device__ __forceinline__ void k_quarter(const Window& w, uint32_t h[16]) {
+  k_quarter_ints<L>(w, h);
+#pragma unroll
+  for (int p = 0; p < 16; ++p) h[p] = ints_to_h2(h[p]);
+}
+template <int L>
+__device__ __forceinline__ void k_quarter_ints(const Window& w, uint32_t h[16]) {
   using D = Dec<L>;
   using F = typename D::F;
+  if constexpr (L == 5) {
+    uint32_t u[5];
+    // symbol s + 5 sits 35 bits after symbol s
+    l5_pairs(w.q0, w.q1, __funnelshift_r(w.q1, w.q2, 3), w.q2 >> 3, u);
 #pragma unroll
-  for (int s = 0; s < D::kHalf; ++s) {
-    uint32_t fa[D::G], fb[D::G];
-    D::sym(wbits(w, s * F::W, F::W), fa);
-    D::sym(wbits(w, (s + D::kHalf) * F::W, F::W), fb);
-    pair_digits<L>(fa, fb, h + s * D::G);
-  }
-  if constexpr (F::R > 0) {
-    static_assert(F::R == 2 && D::kHalf * D::G == 15, "tail layout");
-    uint32_t ft[2];
-    D::tail(wbits(w, F::NG * F::W, F::WT), ft);
-    uint32_t d1;
-    asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(d1) : "r"(ft[0]), "r"((uint32_t)(-L)), "r"(ft[1]));
-    h[15] = pair16(ft[0], d1);
+    for (int s = 0; s < 5; ++s) l5_fpairs(u[s], h + 3 * s);
+    const uint32_t bt = wbits(w, 70, 5);
+    h[15] = pair16(fdig(bt, 5.0f / 32.0f), fdig(bt, 25.0f / 32.0f));
   } else {
-    static_assert(D::kHalf * D::G == 16, "layout");
+#pragma unroll
+    for (int s = 0; s < D::kHalf; ++s) {
+      uint32_t fa[D::G], fb[D::G];
+      D::sym(wbits(w, s * F::W, F::W), fa);
+      D::sym(wbits(w, (s + D::kHalf) * F::W, F::W), fb);
+#pragma unroll
+      for (int k = 0; k < D::G; ++k) h[s * D::G + k] = pair16(fa[k], fb[k]);
+    }
+    if constexpr (F::R > 0) {
+      static_assert(F::R == 2 && D::kHalf * D::G == 15, "tail layout");
+      uint32_t ft[2];
+      D::tail(wbits(w, F::NG * F::W, F::WT), ft);
+      h[15] = pair16(ft[0], ft[1]);
+    } else {
+      static_assert(D::kHalf * D::G == 16, "layout");
+    }
   }
 }
 
-// dims (lo half, hi half) of K-side slot p of quarter t
+// q coefficient of K-side slot p (lo or hi half) of quarter t for one head: the
+// digit k weight minus the share of digit k+1 that F_k carries
 template <int L>
-__device__ __forceinline__ void k_dims(int t, int p, int& dlo, int& dhi) {
+__device__ __forceinline__ float k_coef(const uint16_t* qrow, int t, int p, int half) {
   using D = Dec<L>;
   using F = typename D::F;
-  if (F::R > 0 && p == 15) {
-    dlo = 32 * t + 30;
-    dhi = 32 * t + 31;
-  } else {
-    const int s = p / D::G, k = p % D::G;
-    dlo = 32 * t + s * D::G + k;
-    dhi = 32 * t + (s + D::kHalf) * D::G + k;
-  }
+  const int base = 32 * t;
+  if (F::R > 0 && p == 15)
+    return half == 0 ? f16_to_f32(qrow[base + 30]) - (float)L * f16_to_f32(qrow[base + 31])
+                     : f16_to_f32(qrow[base + 31]);
+  const int s = p / D::G + (half ? D::kHalf : 0), k = p % D::G;
+  const int d = base + s * D::G + k;
+  return D::chained(k) ? f16_to_f32(qrow[d]) - (float)L * f16_to_f32(qrow[d + 1])
+                       : f16_to_f32(qrow[d]);
 }
 
 // V side: lane group g holds half hh of quarter qv for two tokens at once (the two
 // halves of each register are the two tokens).  Row u = j*G + k is digit k of
 // symbol hh*kHalf + j; row 15 is the tail's digit hh.
 template <int L>
+__device__ __forceinline__ void v_half_pair_ints(const Window& wa, const Window& wb, int tpos,
+                                                 int hh, uint32_t h[16]);
+template <int L>
 __device__ __forceinline__ void v_half_pair(const Window& wa, const Window& wb, int tpos, int hh,
                                             uint32_t h[16]) {
+  v_half_pair_ints<L>(wa, wb, tpos, hh, h);
+#pragma unroll
+  for (int u = 0; u < 16; ++u) h[u] = ints_to_h2(h[u]);
+}
+template <int L>
+__device__ __forceinline__ void v_half_pair_ints(const Window& wa, const Window& wb, int tpos,
+                                                 int hh, uint32_t h[16]) {
   using D = Dec<L>;
   using F = typename D::F;
+  if constexpr (L == 5) {
+    uint32_t u[5];
+    l5_pairs(wa.q0, wa.q1, wb.q0, wb.q1, u);
 #pragma unroll
-  for (int j = 0; j < D::kHalf; ++j) {
-    uint32_t fa[D::G], fb[D::G];
-    D::sym(wbits(wa, j * F::W, F::W), fa);
-    D::sym(wbits(wb, j * F::W, F::W), fb);
-    pair_digits<L>(fa, fb, h + j * D::G);
-  }
-  if constexpr (F::R > 0) {
-    uint32_t fa[2], fb[2];
-    D::tail(wbits_rt(wa, tpos, F::WT), fa);
-    D::tail(wbits_rt(wb, tpos, F::WT), fb);
-    const uint32_t P0 = pair16(fa[0], fb[0]), P1 = pair16(fa[1], fb[1]);
-    uint32_t d1;
-    asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(d1) : "r"(P0), "r"((uint32_t)(-L)), "r"(P1));
-    h[15] = hh ? d1 : P0;
+    for (int j = 0; j < 5; ++j) {
+      uint32_t P[3];
+      l5_fpairs(u[j], P);
+      h[3 * j] = P[0];
+      h[3 * j + 1] = digit_step<5>(P[0], P[1]);
+      h[3 * j + 2] = digit_step<5>(P[1], P[2]);
+    }
+    const uint32_t ut = lo16hi16(wbits_rt(wa, tpos, 5), wbits_rt(wb, tpos, 5));
+    const uint32_t P0 = fdig(ut, 5.0f / 32.0f) & kM7, P1 = fdig(ut, 25.0f / 32.0f) & kM7;
+    h[15] = hh ? digit_step<5>(P0, P1) : P0;
+  } else {
+#pragma unroll
+    for (int j = 0; j < D::kHalf; ++j) {
+      uint32_t fa[D::G], fb[D::G];
+      D::sym(wbits(wa, j * F::W, F::W), fa);
+      D::sym(wbits(wb, j * F::W, F::W), fb);
+      pair_digits<L>(fa, fb, h + j * D::G);
+    }
+    if constexpr (F::R > 0) {
+      uint32_t fa[2], fb[2];
+      D::tail(wbits_rt(wa, tpos, F::WT), fa);
+      D::tail(wbits_rt(wb, tpos, F::WT), fb);
+      const uint32_t P0 = pair16(fa[0], fb[0]), P1 = pair16(fa[1], fb[1]);
+      h[15] = hh ? digit_step<L>(P0, P1) : P0;
+    }
   }
 }
 
@@ -316,7 +404,9 @@ struct Shared {
 
 // ------------------------------------------------------------ pool tiles ------
 
-template <int L>
+// PACKED (G <= 4): the lo parts of the q coefficients ride in B columns 4..7 and one
+// mma per k-step serves both; otherwise a second pass with the lo parts.
+template <int L, bool PACKED>
 __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
                          uint64_t* bars, const uint8_t* pool_bh, int64_t count, int t_begin,
                          int t_end, int G, WarpState& st) {
@@ -330,19 +420,34 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
   uint8_t* my_ring = ring + warp * kStages * kStageBytes;
   uint64_t* my_bar = bars + warp * kStages;
 
-  // B fragments of S^T = C Q^T: column n = g (head g), rows = this quarter's slots
-  uint32_t bq[16];
+  // B fragments of S^T = F Q'^T: column n = g, rows = this quarter's F slots; the
+  // coefficient q'_k = q_k - L q_{k+1} (when F_k carries a share of digit k+1) is
+  // split into fp16 hi + lo, exact to 2^-22 relative
+  uint32_t bq[16], bq2[16];
+  {
+    const int head = PACKED ? (g & 3) : g;
+    const bool lo_col = PACKED && g >= 4;
 #pragma unroll
-  for (int p = 0; p < 16; ++p) {
-    int dlo, dhi;
-    k_dims<L>(t, p, dlo, dhi);
-    bq[p] = (uint32_t)sh.q[g][dlo] | ((uint32_t)sh.q[g][dhi] << 16);
+    for (int p = 0; p < 16; ++p) {
+      float c0 = 0.0f, c1 = 0.0f;
+      if (head < G) {
+        c0 = k_coef<L>(sh.q[head], t, p, 0);
+        c1 = k_coef<L>(sh.q[head], t, p, 1);
+      }
+      const float h0 = __half2float(__float2half_rn(c0)), h1 = __half2float(__float2half_rn(c1));
+      const uint32_t hi = h2(h0, h1), lo = h2(c0 - h0, c1 - h1);
+      bq[p] = lo_col ? lo : hi;
+      bq2[p] = lo;
+    }
   }
+  // logit heads of this lane: PACKED folds column c+4 (lo) onto column c (hi)
+  const int hc0 = PACKED ? 2 * (t & 1) : 2 * t;
   float sumq[2];
 #pragma unroll
   for (int c = 0; c < 2; ++c) {
     float s = 0.0f;
-    for (int d = 0; d < 128; ++d) s += f16_to_f32(sh.q[2 * t + c][d]);
+    if (hc0 + c < G)
+      for (int d = 0; d < 128; ++d) s += f16_to_f32(sh.q[hc0 + c][d]);
     sumq[c] = s;
   }
   const int qv = g >> 1, hh = g & 1;
@@ -371,22 +476,29 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
     const uint8_t* tb = my_ring + stage * kStageBytes;
     const int nvalid = (int)min((int64_t)kTile, count - (int64_t)tile * kTile);
 
-    // ---- S^T = C Q^T (two accumulators: two short dependency chains)
+    // ---- S^T = F Q'^T (two accumulators: two short dependency chains)
     float acc[4] = {0.f, 0.f, 0.f, 0.f}, acc2[4] = {0.f, 0.f, 0.f, 0.f};
     {
       uint32_t h0[16], h1[16];
       k_quarter<L>(load_window(tb + g * kRec, t * F::QB), h0);
       k_quarter<L>(load_window(tb + (g + 8) * kRec, t * F::QB), h1);
 #pragma unroll
-      for (int j = 0; j < 8; ++j)
+      for (int j = 0; j < 8; ++j) {
         mma16816((j & 1) ? acc2 : acc, h0[2 * j], h1[2 * j], h0[2 * j + 1], h1[2 * j + 1],
                  bq[2 * j], bq[2 * j + 1]);
+        if constexpr (!PACKED)
+          mma16816((j & 1) ? acc : acc2, h0[2 * j], h1[2 * j], h0[2 * j + 1], h1[2 * j + 1],
+                   bq2[2 * j], bq2[2 * j + 1]);
+      }
 #pragma unroll
-      for (int e = 0; e < 4; ++e) acc[e] += acc2[e];
+      for (int e = 0; e < 4; ++e) {
+        acc[e] += acc2[e];
+        if constexpr (PACKED) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], 2);
+      }
     }
     // ---- logits and online softmax (base 2)
     float p[2][2];
-    uint32_t X[2];
+    uint32_t X[2], Xl[2];
     {
       float lg[2][2], sv[2], zv[2];
       bool valid[2];
@@ -399,31 +511,31 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
         sv[e] = f16_to_f32((uint16_t)(vp & 0xFFFF));
         zv[e] = f16_to_f32((uint16_t)(vp >> 16));
         valid[e] = tok < nvalid;
-        const float A = a.scale_log2 * kTwo24 * sk;
+        const float A = a.scale_log2 * sk;
         const float Bz = a.scale_log2 * zk;
 #pragma unroll
         for (int c = 0; c < 2; ++c)
           lg[e][c] = valid[e] ? fmaf(A, acc[2 * e + c], Bz * sumq[c]) : -INFINITY;
       }
-      float mnew[2];
-#pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        float mx = fmaxf(lg[0][c], lg[1][c]);
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-        mnew[c] = fmaxf(st.m[c], mx);
-      }
-      const bool grow = (mnew[0] > st.m[0]) || (mnew[1] > st.m[1]);
-      if (__any_sync(0xffffffffu, grow)) {
+      // rescale only when some logit of the warp exceeds its running max (rare once
+      // the max has settled); then the tile max comes from the shuffles
+      const bool over = lg[0][0] > st.m[0] || lg[1][0] > st.m[0] || lg[0][1] > st.m[1] ||
+                        lg[1][1] > st.m[1];
+      if (__any_sync(0xffffffffu, over)) {
         float al[2];
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
-          al[c] = (st.m[c] == -INFINITY) ? 0.0f : exp2f(st.m[c] - mnew[c]);
-          st.m[c] = mnew[c];
+          float mx = fmaxf(lg[0][c], lg[1][c]);
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+          const float mnew = fmaxf(st.m[c], mx);
+          al[c] = (st.m[c] == -INFINITY) ? 0.0f : exp2f(st.m[c] - mnew);
+          st.m[c] = mnew;
           st.l[c] *= al[c];
           st.zs[c] *= al[c];
         }
+        // O columns are heads 2t, 2t+1: for PACKED lanes t >= 2 they are padding
 #pragma unroll
         for (int m = 0; m < 8; ++m) {
           st.O[m][0] *= al[0];
@@ -436,23 +548,40 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
       for (int c = 0; c < 2; ++c) {
 #pragma unroll
         for (int e = 0; e < 2; ++e) p[e][c] = valid[e] ? exp2f(lg[e][c] - st.m[c]) : 0.0f;
-        X[c] = h2(p[0][c] * sv[0], p[1][c] * sv[1]);
+        // P' = p * s_v as fp16 hi + lo (exact to 2^-22 relative)
+        const float P0 = p[0][c] * sv[0], P1 = p[1][c] * sv[1];
+        const float H0 = __half2float(__float2half_rn(P0)), H1 = __half2float(__float2half_rn(P1));
+        X[c] = h2(H0, H1);
+        Xl[c] = h2(P0 - H0, P1 - H1);
         st.l[c] += p[0][c] + p[1][c];
         st.zs[c] += p[0][c] * zv[0] + p[1][c] * zv[1];
       }
     }
-    // ---- P'^T into the B fragment: column g (head g), rows = tokens 2t, 2t+1, 2t+8, 2t+9
-    uint32_t b0, b1;
+    // ---- P'^T into the B fragment: rows = tokens 2t, 2t+1, 2t+8, 2t+9; column g is
+    // head g (hi parts), or for PACKED columns 4..7 the lo parts of heads 0..3
+    uint32_t b0, b1, b0l = 0u, b1l = 0u;
     {
-      const int src0 = (2 * t) * 4 + (g >> 1), src1 = (2 * t + 1) * 4 + (g >> 1);
+      const int hd = PACKED ? (g & 3) : g;
+      const int src0 = (2 * t) * 4 + (hd >> 1), src1 = (2 * t + 1) * 4 + (hd >> 1);
       const uint32_t v0 = __shfl_sync(0xffffffffu, X[0], src0);
       const uint32_t v1 = __shfl_sync(0xffffffffu, X[1], src0);
       const uint32_t w0 = __shfl_sync(0xffffffffu, X[0], src1);
       const uint32_t w1 = __shfl_sync(0xffffffffu, X[1], src1);
-      const uint32_t A = (g & 1) ? v1 : v0;  // tokens 2t (lo), 2t+8 (hi)
-      const uint32_t B = (g & 1) ? w1 : w0;  // tokens 2t+1 (lo), 2t+9 (hi)
-      b0 = g < G ? __byte_perm(A, B, 0x5410) : 0u;
-      b1 = g < G ? __byte_perm(A, B, 0x7632) : 0u;
+      const uint32_t vl0 = __shfl_sync(0xffffffffu, Xl[0], src0);
+      const uint32_t vl1 = __shfl_sync(0xffffffffu, Xl[1], src0);
+      const uint32_t wl0 = __shfl_sync(0xffffffffu, Xl[0], src1);
+      const uint32_t wl1 = __shfl_sync(0xffffffffu, Xl[1], src1);
+      const bool odd = hd & 1, live = hd < G;
+      const uint32_t Ah = odd ? v1 : v0, Bh = odd ? w1 : w0;    // tokens 2t|2t+8, 2t+1|2t+9
+      const uint32_t Al = odd ? vl1 : vl0, Bl = odd ? wl1 : wl0;
+      const bool use_lo = PACKED && g >= 4;
+      const uint32_t A = use_lo ? Al : Ah, B = use_lo ? Bl : Bh;
+      b0 = live ? __byte_perm(A, B, 0x5410) : 0u;
+      b1 = live ? __byte_perm(A, B, 0x7632) : 0u;
+      if constexpr (!PACKED) {
+        b0l = live ? __byte_perm(Al, Bl, 0x5410) : 0u;
+        b1l = live ? __byte_perm(Al, Bl, 0x7632) : 0u;
+      }
     }
     // ---- O^T += C^T P'^T
     {
@@ -462,8 +591,11 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
       v_half_pair<L>(load_window(tb + (2 * t + 8) * kRec, vpos),
                      load_window(tb + (2 * t + 9) * kRec, vpos), tpos, hh, hb);
 #pragma unroll
-      for (int m = 0; m < 8; ++m)
+      for (int m = 0; m < 8; ++m) {
         mma16816(st.O[m], ha[2 * m], ha[2 * m + 1], hb[2 * m], hb[2 * m + 1], b0, b1);
+        if constexpr (!PACKED)
+          mma16816(st.O[m], ha[2 * m], ha[2 * m + 1], hb[2 * m], hb[2 * m + 1], b0l, b1l);
+      }
     }
     __syncwarp();
     if (lane == 0 && it + kStages < nmine) {
@@ -588,13 +720,20 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
     const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
     uint64_t* bars = &sh.bar[0][0];
     switch (L) {
-      case 2: run_pool<2>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 3: run_pool<3>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 4: run_pool<4>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 5: run_pool<5>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 6: run_pool<6>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 7: run_pool<7>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 8: run_pool<8>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 2: G <= 4 ? run_pool<2, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<2, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 3: G <= 4 ? run_pool<3, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<3, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 4: G <= 4 ? run_pool<4, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<4, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 5: G <= 4 ? run_pool<5, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<5, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 6: G <= 4 ? run_pool<6, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<6, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 7: G <= 4 ? run_pool<7, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<7, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 8: G <= 4 ? run_pool<8, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<8, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
       default: break;
     }
     // reduce the per-lane partial sums over the 8 token rows (lanes with equal t)
@@ -608,22 +747,25 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
     }
     __syncthreads();  // every warp is done with the ring: reuse it as the merge area
     const int g = lane >> 2, t = lane & 3;
-    if (g == 0) {
+    // logit heads of this lane: 2t+c, or 2(t&1)+c when the lo parts were folded
+    const int hc0 = G <= 4 ? 2 * (t & 1) : 2 * t;
+    if (g == 0 && (G > 4 || t < 2)) {
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
-        if (2 * t + c < G) {
-          merge_m[warp * 8 + 2 * t + c] = st.m[c];
-          merge_l[warp * 8 + 2 * t + c] = st.l[c];
-          merge_z[warp * 8 + 2 * t + c] = st.zs[c];
+        if (hc0 + c < G) {
+          merge_m[warp * 8 + hc0 + c] = st.m[c];
+          merge_l[warp * 8 + hc0 + c] = st.l[c];
+          merge_z[warp * 8 + hc0 + c] = st.zs[c];
         }
       }
     }
-    // O columns are heads 2t, 2t+1; rows 16m + g (+8) are V rows u = 2m (+1) of
-    // lane group g, i.e. output dims v_dim(g, u)
+    // O columns are heads 2t, 2t+1 (for G <= 4, columns 4..7 hold the lo parts of
+    // heads 0..3; they are written as rows 4..7 and folded in below); rows 16m + g
+    // (+8) are V rows u = 2m (+1) of lane group g, i.e. output dims v_dim(g, u)
 #pragma unroll
     for (int c = 0; c < 2; ++c) {
       const int qh = 2 * t + c;
-      if (qh < G) {
+      if (qh < G || (G <= 4 && qh >= 4 && qh - 4 < G)) {
 #pragma unroll
         for (int m = 0; m < 8; ++m) {
 #pragma unroll
@@ -675,11 +817,15 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
     float o = 0.0f;
     for (int w = 0; w < kWarps; ++w) {
       const float sc = cta_scale[w * 8 + qh];
-      if (sc != 0.0f) o += sc * merge_o[(w * 8 + qh) * 128 + d];
+      if (sc != 0.0f) {
+        float v = merge_o[(w * 8 + qh) * 128 + d];
+        if (src != 2 && G <= 4) v += merge_o[(w * 8 + qh + 4) * 128 + d];
+        o += sc * v;
+      }
     }
-    // pool rows hold sum p' c (c as the fp16 value c * 2^-24); the offset part is
-    // sum p z; staged rows are plain sums of p v
-    part[16 + qh * 128 + d] = src == 2 ? o : kTwo24 * o + cta_z[qh];
+    // pool rows hold sum p' c; the offset part is sum p z; staged rows are plain
+    // sums of p v
+    part[16 + qh * 128 + d] = src == 2 ? o : o + cta_z[qh];
   }
 }
 
