@@ -104,29 +104,46 @@ __device__ __forceinline__ void mma16816(float c[4], uint32_t a0, uint32_t a1, u
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// two 16-bit values into one register with a multiply-add (keeps the ALU pipe free)
-__device__ __forceinline__ uint32_t pair16(uint32_t lo, uint32_t hi) {
-  uint32_t r;
-  asm("mad.lo.u32 %0, %1, 65536, %2;" : "=r"(r) : "r"(hi), "r"(lo));
-  return r;
-}
-
-// two integers < 256 in the 16-bit halves -> the same integers as fp16 values: the
-// byte 0x64 over each makes 1024 + v, and one f16x2 subtract of 1024 leaves v.  (The
-// integers read directly as fp16 subnormals v * 2^-24 were tried first: the tensor
-// cores lose products of subnormal operands with small weights, biasing attention by
-// ~1e-5 of the low-weight mass per mma.)
-__device__ __forceinline__ uint32_t ints_to_h2(uint32_t P) {
-  const uint32_t x = __byte_perm(P, 0x64646464u, 0x7250);
-  uint32_t r;
-  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(x), "r"(0x64006400u));
-  return r;
-}
+// ---------------------------------------------------------- digit helpers -----
 
 // F = floor(beta * c) for the exact constant c: beta read as a denormal float,
 // multiplied with rounding toward zero; the result's bit pattern is the integer F.
 __device__ __forceinline__ uint32_t fdig(uint32_t beta, float c) {
   return __float_as_uint(__fmul_rz(__uint_as_float(beta), c));
+}
+// the same with 0x6400 added in the denormal grid: the low 16 bits are then the fp16
+// value 1024 + F (F < 1024)
+__device__ __forceinline__ uint32_t fdig1024(uint32_t beta, float c) {
+  return __float_as_uint(__fmaf_rz(__uint_as_float(beta), c, __uint_as_float(0x6400u)));
+}
+__device__ __forceinline__ uint32_t lo16hi16(uint32_t a, uint32_t b) {
+  return __byte_perm(a, b, 0x5410);
+}
+// subtract 1024 from both fp16 halves: 1024 + v -> v exactly (v < 1024)
+__device__ __forceinline__ uint32_t hsub1024(uint32_t x) {
+  uint32_t r;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(x), "r"(0x64006400u));
+  return r;
+}
+// integers in bytes 0 and 2 (< 256; bytes 1 and 3 ignored) -> fp16 values: the byte
+// 0x64 over each makes 1024 + v.  (The integers read directly as fp16 subnormals
+// v * 2^-24 were tried first: the tensor cores lose products of subnormal operands
+// with small weights, biasing attention by ~1e-5 of the low-weight mass per mma.)
+__device__ __forceinline__ uint32_t bytes_to_h2(uint32_t P) {
+  return hsub1024(__byte_perm(P, 0x64646464u, 0x7250));
+}
+// fp16 bit pattern of -L
+__host__ __device__ constexpr uint32_t neg_half_bits(int L) {
+  return L == 2 ? 0xC000u : L == 3 ? 0xC200u : L == 4 ? 0xC400u : L == 5 ? 0xC500u
+       : L == 6 ? 0xC600u : L == 7 ? 0xC700u : 0xC800u;
+}
+// digit pair cur - L prev on fp16 integers (exact: all values are small integers)
+template <int L>
+__device__ __forceinline__ uint32_t hdigit(uint32_t prev, uint32_t cur) {
+  constexpr uint32_t kNegL = neg_half_bits(L) * 0x00010001u;
+  uint32_t r;
+  asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(r) : "r"(prev), "r"(kNegL), "r"(cur));
+  return r;
 }
 
 __device__ __forceinline__ uint32_t h2(float lo, float hi) {
@@ -174,75 +191,63 @@ struct Dec {
   static constexpr int G = F::G;
   static constexpr int kHalf = F::NG / 2;                     // symbols per half quarter
   static constexpr int kRestart = (L == 6) ? 2 : G;           // F chain restarts here
-  static constexpr bool kPow2 = (L & (L - 1)) == 0;
-  // F values of one full symbol
+  // 1024 + F values of one full symbol, in the low 16 bits of each word (F < 256)
   __device__ __forceinline__ static void sym(uint32_t beta, uint32_t* f) {
     if constexpr (G == 1) {
-      f[0] = kPow2 ? beta : fdig(beta, (float)L / (float)(1u << F::W));
+      f[0] = fdig1024(beta, (float)L / (float)(1u << F::W));
     } else if constexpr (L == 6) {
       constexpr float c1 = 6.0f / 8192.0f, c2 = 36.0f / 8192.0f, c3 = 216.0f / 8192.0f;
-      f[0] = fdig(beta, c1);
-      f[1] = fdig(beta, c2);
+      f[0] = fdig1024(beta, c1);
+      f[1] = fdig1024(beta, c2);
       const uint32_t x = (beta * 36u) & 8191u;  // remainder after two digits
-      f[2] = fdig(x, c1);
-      f[3] = fdig(x, c2);
-      f[4] = fdig(x, c3);
+      f[2] = fdig1024(x, c1);
+      f[3] = fdig1024(x, c2);
+      f[4] = fdig1024(x, c3);
     } else {
       float c = (float)L / (float)(1u << F::W);
 #pragma unroll
       for (int k = 0; k < G; ++k) {
-        f[k] = fdig(beta, c);
+        f[k] = fdig1024(beta, c);
         c *= (float)L;
       }
     }
   }
-  // F values of the two-code tail symbol
+  // 1024 + F values of the two-code tail symbol
   __device__ __forceinline__ static void tail(uint32_t beta, uint32_t* f) {
     constexpr float c = (float)L / (float)(1u << F::WT);
-    f[0] = fdig(beta, c);
-    f[1] = fdig(beta, c * (float)L);
+    f[0] = fdig1024(beta, c);
+    f[1] = fdig1024(beta, c * (float)L);
   }
   // does F slot k of a group carry a share of digit k+1?
   __host__ __device__ static constexpr bool chained(int k) { return k + 1 < G && k + 1 != kRestart; }
 };
 
-// lane-wise P_k - L P_{k-1}: digits are never negative, so no borrow crosses halves
+// fp16 F pairs (low half symbol a, high half symbol b) of two symbols
 template <int L>
-__device__ __forceinline__ uint32_t digit_step(uint32_t prev, uint32_t P) {
-  uint32_t r;
-  asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(r) : "r"(prev), "r"((uint32_t)(-L)), "r"(P));
-  return r;
-}
-
-// digits of two symbols from their F values, one register per digit position:
-// P_k = F_k(a) + 65536 F_k(b), digit_k = P_k - L P_{k-1}; the chain restarts at kRestart
-template <int L>
-__device__ __forceinline__ void pair_digits(const uint32_t* fa, const uint32_t* fb, uint32_t* h) {
-  using D = Dec<L>;
-  uint32_t prev = 0;
+__device__ __forceinline__ void pair_F(const uint32_t* fa, const uint32_t* fb, uint32_t* X) {
 #pragma unroll
-  for (int k = 0; k < D::G; ++k) {
-    const uint32_t P = pair16(fa[k], fb[k]);
-    h[k] = (k == 0 || k == D::kRestart) ? P : digit_step<L>(prev, P);
-    prev = P;
-  }
+  for (int k = 0; k < Dec<L>::G; ++k) X[k] = hsub1024(lo16hi16(fa[k], fb[k]));
+}
+// digits from fp16 F pairs: c_k = F_k - L F_{k-1}, the chain restarting at kRestart
+template <int L>
+__device__ __forceinline__ void F_to_digits(const uint32_t* X, uint32_t* h) {
+#pragma unroll
+  for (int k = 0; k < Dec<L>::G; ++k)
+    h[k] = (k == 0 || k == Dec<L>::kRestart) ? X[k] : hdigit<L>(X[k - 1], X[k]);
 }
 
 // ---- five-level fast path: two 7-bit symbols per register ---------------------
 // u = beta_a + 65536 beta_b is still a denormal (beta < 128), and
 // floor(u * L^(k+1)/128) = F_k(a) + 65536 F_k(b) + (fraction of b) * 512: one
-// multiply and one mask give both halves' F_k at once (F_k <= 124).
+// multiply gives both halves' F_k (bytes 0 and 2; the fraction lands in byte 1).
 constexpr uint32_t kM7 = 0x007F007Fu;
-__device__ __forceinline__ uint32_t lo16hi16(uint32_t a, uint32_t b) {
-  return __byte_perm(a, b, 0x5410);
+__device__ __forceinline__ void l5_fpairs(uint32_t u, uint32_t* X) {
+  X[0] = bytes_to_h2(fdig(u, 5.0f / 128.0f));
+  X[1] = bytes_to_h2(fdig(u, 25.0f / 128.0f));
+  X[2] = bytes_to_h2(fdig(u, 125.0f / 128.0f));
 }
-__device__ __forceinline__ void l5_fpairs(uint32_t u, uint32_t* P) {
-  P[0] = fdig(u, 5.0f / 128.0f) & kM7;
-  P[1] = fdig(u, 25.0f / 128.0f) & kM7;
-  P[2] = fdig(u, 125.0f / 128.0f) & kM7;
-}
-// symbol pairs from two 96-bit windows: symbol j of window a in the low half and of
-// window b in the high half, j = 0..4 (bits 7j)
+// symbol pairs from two windows: symbol j of window a in the low half and of window b
+// in the high half, j = 0..4 (bits 7j)
 __device__ __forceinline__ void l5_pairs(uint32_t a0, uint32_t a1, uint32_t b0, uint32_t b1,
                                          uint32_t u[5]) {
   uint32_t C = lo16hi16(a0, b0);
@@ -255,19 +260,11 @@ __device__ __forceinline__ void l5_pairs(uint32_t a0, uint32_t a1, uint32_t b0, 
   u[4] = C & kM7;
 }
 
-// K side: the 16 F-value pairs of one quarter row of one token (both halves are the
-// same token).  Slot p < kHalf*G holds F_k of symbols s and s + kHalf (s = p / G,
-// k = p % G); slot 15 holds the tail's F_0 and F_1.
-template <int L>
-__device__ __forceinline__ void k_quarter_ints(const Window& w, uint32_t h[16]);
+// K side: the 16 fp16 F-value pairs of one quarter row of one token (both halves are
+// the same token).  Slot p < kHalf*G holds F_k of symbols s and s + kHalf
+// (s = p / G, k = p % G); slot 15 holds the tail's F_0 and F_1.
 template <int L>
 __device__ __forceinline__ void k_quarter(const Window& w, uint32_t h[16]) {
-  k_quarter_ints<L>(w, h);
-#pragma unroll
-  for (int p = 0; p < 16; ++p) h[p] = ints_to_h2(h[p]);
-}
-template <int L>
-__device__ __forceinline__ void k_quarter_ints(const Window& w, uint32_t h[16]) {
   using D = Dec<L>;
   using F = typename D::F;
   if constexpr (L == 5) {
@@ -276,22 +273,22 @@ __device__ __forceinline__ void k_quarter_ints(const Window& w, uint32_t h[16]) 
     l5_pairs(w.q0, w.q1, __funnelshift_r(w.q1, w.q2, 3), w.q2 >> 3, u);
 #pragma unroll
     for (int s = 0; s < 5; ++s) l5_fpairs(u[s], h + 3 * s);
-    const uint32_t bt = wbits(w, 70, 5);
-    h[15] = pair16(fdig(bt, 5.0f / 32.0f), fdig(bt, 25.0f / 32.0f));
+    uint32_t ft[2];
+    D::tail(wbits(w, 70, 5), ft);
+    h[15] = hsub1024(lo16hi16(ft[0], ft[1]));
   } else {
 #pragma unroll
     for (int s = 0; s < D::kHalf; ++s) {
       uint32_t fa[D::G], fb[D::G];
       D::sym(wbits(w, s * F::W, F::W), fa);
       D::sym(wbits(w, (s + D::kHalf) * F::W, F::W), fb);
-#pragma unroll
-      for (int k = 0; k < D::G; ++k) h[s * D::G + k] = pair16(fa[k], fb[k]);
+      pair_F<L>(fa, fb, h + s * D::G);
     }
     if constexpr (F::R > 0) {
       static_assert(F::R == 2 && D::kHalf * D::G == 15, "tail layout");
       uint32_t ft[2];
       D::tail(wbits(w, F::NG * F::W, F::WT), ft);
-      h[15] = pair16(ft[0], ft[1]);
+      h[15] = hsub1024(lo16hi16(ft[0], ft[1]));
     } else {
       static_assert(D::kHalf * D::G == 16, "layout");
     }
@@ -316,20 +313,10 @@ __device__ __forceinline__ float k_coef(const uint16_t* qrow, int t, int p, int 
 
 // V side: lane group g holds half hh of quarter qv for two tokens at once (the two
 // halves of each register are the two tokens).  Row u = j*G + k is digit k of
-// symbol hh*kHalf + j; row 15 is the tail's digit hh.
-template <int L>
-__device__ __forceinline__ void v_half_pair_ints(const Window& wa, const Window& wb, int tpos,
-                                                 int hh, uint32_t h[16]);
+// symbol hh*kHalf + j; row 15 is the tail's digit hh.  Digits as fp16 values.
 template <int L>
 __device__ __forceinline__ void v_half_pair(const Window& wa, const Window& wb, int tpos, int hh,
                                             uint32_t h[16]) {
-  v_half_pair_ints<L>(wa, wb, tpos, hh, h);
-#pragma unroll
-  for (int u = 0; u < 16; ++u) h[u] = ints_to_h2(h[u]);
-}
-template <int L>
-__device__ __forceinline__ void v_half_pair_ints(const Window& wa, const Window& wb, int tpos,
-                                                 int hh, uint32_t h[16]) {
   using D = Dec<L>;
   using F = typename D::F;
   if constexpr (L == 5) {
@@ -337,29 +324,30 @@ __device__ __forceinline__ void v_half_pair_ints(const Window& wa, const Window&
     l5_pairs(wa.q0, wa.q1, wb.q0, wb.q1, u);
 #pragma unroll
     for (int j = 0; j < 5; ++j) {
-      uint32_t P[3];
-      l5_fpairs(u[j], P);
-      h[3 * j] = P[0];
-      h[3 * j + 1] = digit_step<5>(P[0], P[1]);
-      h[3 * j + 2] = digit_step<5>(P[1], P[2]);
+      uint32_t X[3];
+      l5_fpairs(u[j], X);
+      F_to_digits<5>(X, h + 3 * j);
     }
     const uint32_t ut = lo16hi16(wbits_rt(wa, tpos, 5), wbits_rt(wb, tpos, 5));
-    const uint32_t P0 = fdig(ut, 5.0f / 32.0f) & kM7, P1 = fdig(ut, 25.0f / 32.0f) & kM7;
-    h[15] = hh ? digit_step<5>(P0, P1) : P0;
+    const uint32_t X0 = bytes_to_h2(fdig(ut, 5.0f / 32.0f));
+    const uint32_t X1 = bytes_to_h2(fdig(ut, 25.0f / 32.0f));
+    h[15] = hh ? hdigit<5>(X0, X1) : X0;
   } else {
 #pragma unroll
     for (int j = 0; j < D::kHalf; ++j) {
-      uint32_t fa[D::G], fb[D::G];
+      uint32_t fa[D::G], fb[D::G], X[D::G];
       D::sym(wbits(wa, j * F::W, F::W), fa);
       D::sym(wbits(wb, j * F::W, F::W), fb);
-      pair_digits<L>(fa, fb, h + j * D::G);
+      pair_F<L>(fa, fb, X);
+      F_to_digits<L>(X, h + j * D::G);
     }
     if constexpr (F::R > 0) {
       uint32_t fa[2], fb[2];
       D::tail(wbits_rt(wa, tpos, F::WT), fa);
       D::tail(wbits_rt(wb, tpos, F::WT), fb);
-      const uint32_t P0 = pair16(fa[0], fb[0]), P1 = pair16(fa[1], fb[1]);
-      h[15] = hh ? digit_step<L>(P0, P1) : P0;
+      const uint32_t X0 = hsub1024(lo16hi16(fa[0], fb[0]));
+      const uint32_t X1 = hsub1024(lo16hi16(fa[1], fb[1]));
+      h[15] = hh ? hdigit<L>(X0, X1) : X0;
     }
   }
 }
