@@ -180,6 +180,32 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
                                     float softmax_scale, void* ws, size_t ws_bytes,
                                     void* stream);
 
+/* Decode attention for callers that cannot allocate device memory.  The paper has
+ * no counterpart: this is a deployment variant of semkv_decode_attention.
+ * Who needs it: a caller whose host framework owns all device memory and gives this
+ * library only the cache and the tensors of the call, or a serving loop that must
+ * not call cudaMalloc between decode steps (an allocation can synchronise the device).
+ * It computes exactly what semkv_decode_attention computes (same kernels, affine base
+ * only), but keeps the split-K partial results in a static device array of 8 MiB
+ * (2016 partials) that the library owns, instead of a caller workspace; it calls no
+ * cudaMalloc, cudaFree or allocating routine.  Every GPU that loads the library
+ * holds that array until the process exits.
+ *  - Set-up: the first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call before
+ *    any stream capture.
+ *  - Limit: batch * kv_heads * (one partial per non-empty pool, plus one when tokens
+ *    are staged) must fit in 2016 partials; larger requests return SEMKV_EWORKSPACE.
+ *    Within the limit the split count is reduced to fit.
+ *  - All calls share the array, which keeps the last call's contents (each call
+ *    overwrites every partial it reads, so nothing needs clearing).  Calls whose
+ *    kernels overlap on the GPU (e.g. on two streams, or two host threads) race on
+ *    it: serialise them.
+ * Arguments and errors otherwise as semkv_decode_attention (no ws / ws_bytes). */
+semkv_status semkv_decode_attention_noalloc(const semkv_quant_desc* desc,
+                                            const semkv_cache* cache, int32_t layer,
+                                            const uint16_t* q, float* out, float softmax_scale,
+                                            void* stream);
+
 /* Human-readable name of a status code (static string). */
 const char* semkv_status_string(semkv_status s);
 

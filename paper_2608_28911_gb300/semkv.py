@@ -86,6 +86,10 @@ def _load():
                                          ctypes.POINTER(CacheStruct), i32, p, p,
                                          ctypes.c_float, p, sz, p]
     L.semkv_decode_attention.restype = ctypes.c_int
+    L.semkv_decode_attention_noalloc.argtypes = [ctypes.POINTER(QuantDescStruct),
+                                                 ctypes.POINTER(CacheStruct), i32, p, p,
+                                                 ctypes.c_float, p]
+    L.semkv_decode_attention_noalloc.restype = ctypes.c_int
     L.semkv_status_string.argtypes = [ctypes.c_int]
     L.semkv_status_string.restype = ctypes.c_char_p
     return L
@@ -95,7 +99,8 @@ LIB = _load()
 EXPORTED = ["semkv_row_bytes", "semkv_record_bytes", "semkv_high_count_floor",
             "semkv_block_high_count", "semkv_lloyd_max_gaussian", "semkv_rank_workspace_bytes",
             "semkv_rank_assign", "semkv_quantize_pack", "semkv_append_block",
-            "semkv_decode_workspace_bytes", "semkv_decode_attention", "semkv_status_string"]
+            "semkv_decode_workspace_bytes", "semkv_decode_attention",
+            "semkv_decode_attention_noalloc", "semkv_status_string"]
 
 
 def _ptr(t):
@@ -177,6 +182,17 @@ def semkv_decode_attention(desc: "QuantDesc", cache: "KVCache", layer: int, q: t
            LIB.semkv_decode_attention(ctypes.byref(desc.s), ctypes.byref(cache.s), layer,
                                       _ptr(q), _ptr(out), softmax_scale, _ptr(ws),
                                       ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def semkv_decode_attention_noalloc(desc: "QuantDesc", cache: "KVCache", layer: int,
+                                   q: torch.Tensor, out: torch.Tensor, softmax_scale: float,
+                                   stream=None):
+    """Decode attention with the library's static split-K scratch (no workspace):
+    for callers that cannot allocate device memory.  See include/semkv.h."""
+    _check("semkv_decode_attention_noalloc",
+           LIB.semkv_decode_attention_noalloc(ctypes.byref(desc.s), ctypes.byref(cache.s), layer,
+                                              _ptr(q), _ptr(out), softmax_scale,
+                                              _stream(stream)))
 
 
 # ------------------------------------------------------- owning wrappers ------
