@@ -278,7 +278,6 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
   if (s != SEMKV_OK) return s;
   s = check_cache(cache);
   if (s != SEMKV_OK) return s;
-  if (desc->base != SEMKV_BASE_AFFINE) return SEMKV_EUNSUPPORTED;
   if (!q || !out || layer < 0 || layer >= cache->layers) return SEMKV_EINVAL;
   if (!aligned(out, 16)) return SEMKV_EALIGN;
   if (cache->hi_count + cache->lo_count + cache->stage_n == 0) return SEMKV_EINVAL;
@@ -316,7 +315,8 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
   a.signs = desc->signs;
   a.cb_hi = desc->centroids_hi;
   a.cb_lo = desc->centroids_lo;
-  a.qrot = nullptr;
+  // rotated queries (TQ base) after the split-K partials in the workspace
+  a.qrot = a.partials + (decode_workspace_floats(a.B, a.H, a.Hq) - (size_t)a.B * a.Hq * 128);
   a.err = cache->dev_error;
   a.plan = make_decode_plan(a.B, a.H, a.hi_count, a.lo_count, a.stage_n, sms);
   return from_cuda(launch_decode_attention(a, (cudaStream_t)stream));

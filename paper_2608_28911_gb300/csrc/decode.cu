@@ -387,6 +387,8 @@ __device__ __forceinline__ void state_init(WarpState& st) {
 
 struct Shared {
   uint16_t q[8][128];       // the group's query heads (rows >= G are zero)
+  float qr[8][128];         // TQ base: rotated queries q' = H S q
+  float cb[2][8];           // TQ base: centroids of the high / low level count
   uint64_t bar[kWarps][kStages];
 };
 
@@ -604,6 +606,163 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
   }
 }
 
+// ------------------------------------------------- TurboQuant-MSE records -----
+// Dequantized rows are x^ = (n/128) S H cb[c] (Sec. 4.9), so q . x^ = (n/128) q' . cb[c]
+// with q' = H S q, and sum p x^ = S H (sum p (n/128) cb[c]): scores and the weighted
+// sum run in the rotated domain and each CTA rotates its partial back at the end.
+// One warp per token on the CUDA cores: lane l holds dims 4l..4l+3 of both rows.
+
+// digit k of the group symbol beta (compile-time level, run-time k)
+template <int L>
+__device__ __forceinline__ uint32_t digit_rt(uint32_t beta, int k) {
+  using D = Dec<L>;
+  using F = typename D::F;
+  if constexpr (D::G == 1) {
+    return fdig(beta, (float)L / (float)(1u << F::W));
+  } else {
+    // chain start and the multiplier of F_k within its chain
+    const int k0 = (k >= D::kRestart) ? D::kRestart : 0;
+    const uint32_t x = (k0 == 0) ? beta : ((beta * 36u) & 8191u);  // restart: six levels only
+    float c = (float)L / (float)(1u << F::W);
+    for (int j = k0; j < k; ++j) c *= (float)L;
+    const uint32_t Fk = fdig(x, c);
+    if (k == k0) return Fk;
+    return Fk - (uint32_t)L * fdig(x, c / (float)L);
+  }
+}
+template <int L>
+__device__ __forceinline__ uint32_t tail_digit(uint32_t beta, int k) {
+  using F = Fmt<L>;
+  const float c = (float)L / (float)(1u << F::WT);
+  const uint32_t F0 = fdig(beta, c);
+  return k == 0 ? F0 : fdig(beta, c * (float)L) - (uint32_t)L * F0;
+}
+// 96 bits from bit `pos` of a record in global memory, reading no word at or past
+// bit `end` (the end of the row): the last record of a pool may end its allocation
+__device__ __forceinline__ Window load_window_bounded(const uint8_t* rec, int pos, int end) {
+  const uint32_t* w = reinterpret_cast<const uint32_t*>(rec) + (pos >> 5);
+  const int first = pos >> 5, last = (end - 1) >> 5;
+  uint32_t v[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) v[i] = (first + i <= last) ? w[i] : 0u;
+  const int sh = pos & 31;
+  Window r;
+  r.q0 = __funnelshift_r(v[0], v[1], sh);
+  r.q1 = __funnelshift_r(v[1], v[2], sh);
+  r.q2 = __funnelshift_r(v[2], v[3], sh);
+  return r;
+}
+
+// the codes of dims 4l..4l+3 of the row starting at bit `row_bit` of a record
+template <int L>
+__device__ __forceinline__ void tq_codes4(const uint8_t* rec, int row_bit, int lane, uint32_t c[4]) {
+  using D = Dec<L>;
+  using F = typename D::F;
+  const int q = lane >> 3, i0 = 4 * (lane & 7);
+  const Window w = load_window_bounded(rec, row_bit + q * F::QB, row_bit + 8 * F::RB);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int i = i0 + j;
+    if (F::R > 0 && i >= 32 - F::R) {
+      c[j] = tail_digit<L>(wbits(w, F::NG * F::W, F::WT), i - (32 - F::R));
+    } else {
+      const int s = i / D::G, k = i % D::G;
+      c[j] = digit_rt<L>(wbits_rt(w, s * F::W, F::W), k);
+    }
+  }
+}
+
+template <int L>
+__device__ void run_pool_tq(const DecodeArgs& a, const Shared& sh, int which,
+                            const uint8_t* pool_bh, int64_t count, int t_begin, int t_end,
+                            int G, float* m_out, float* l_out, float* z_out, float* o_out) {
+  using F = Fmt<L>;
+  constexpr int kRec = 2 * F::RB + 4;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float qf[8][4];
+#pragma unroll
+  for (int c = 0; c < 8; ++c)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) qf[c][j] = c < G ? sh.qr[c][4 * lane + j] : 0.0f;
+  float m[8], l[8], o[8][4];
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    m[c] = -INFINITY;
+    l[c] = 0.0f;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) o[c][j] = 0.0f;
+  }
+  const int64_t i_end = min((int64_t)t_end * kTile, count);
+  for (int64_t i = (int64_t)t_begin * kTile + warp; i < i_end; i += kWarps) {
+    const uint8_t* rec = pool_bh + i * kRec;
+    uint32_t ck[4], cv[4];
+    tq_codes4<L>(rec, 0, lane, ck);
+    tq_codes4<L>(rec, 8 * F::RB, lane, cv);
+    const uint32_t nn = *reinterpret_cast<const uint32_t*>(rec + 2 * F::RB);
+    const float nk = f16_to_f32((uint16_t)(nn & 0xFFFF)) * (1.0f / 128.0f);
+    const float nv = f16_to_f32((uint16_t)(nn >> 16)) * (1.0f / 128.0f);
+    float kv[4], vv[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      kv[j] = sh.cb[which][ck[j]] * nk;
+      vv[j] = sh.cb[which][cv[j]] * nv;
+    }
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      if (c >= G) break;
+      float d = qf[c][0] * kv[0] + qf[c][1] * kv[1] + qf[c][2] * kv[2] + qf[c][3] * kv[3];
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) d += __shfl_xor_sync(0xffffffffu, d, off);
+      const float lg = d * a.scale_log2;
+      const float mn = fmaxf(m[c], lg);
+      const float al = m[c] == -INFINITY ? 0.0f : exp2f(m[c] - mn);
+      const float pp = exp2f(lg - mn);
+      m[c] = mn;
+      l[c] = l[c] * al + pp;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) o[c][j] = o[c][j] * al + pp * vv[j];
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    if (c >= G) break;
+    if (lane == 0) {
+      m_out[warp * 8 + c] = m[c];
+      l_out[warp * 8 + c] = l[c];
+      z_out[warp * 8 + c] = 0.0f;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) o_out[(warp * 8 + c) * 128 + 4 * lane + j] = o[c][j];
+  }
+}
+
+// q' = H S q for every (sequence, query head): one warp each, lane l = dims 4l..4l+3
+__global__ void qrot_kernel(DecodeArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (gw >= a.B * a.Hq) return;
+  const int b = gw / a.Hq, qh = gw % a.Hq, h = qh / (a.Hq / a.H);
+  const int8_t* sg = a.signs + ((int64_t)a.layer * a.H + h) * 128;
+  const uint16_t* qrow = a.q + ((int64_t)b * a.Hq + qh) * 128;
+  float w[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) w[j] = f16_to_f32(qrow[4 * lane + j]) * (float)sg[4 * lane + j];
+  float t0 = w[0] + w[1], t1 = w[0] - w[1], t2 = w[2] + w[3], t3 = w[2] - w[3];
+  w[0] = t0 + t2; w[2] = t0 - t2; w[1] = t1 + t3; w[3] = t1 - t3;
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    const bool upper = (lane >> k) & 1;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float other = __shfl_xor_sync(0xffffffffu, w[j], 1 << k);
+      w[j] = upper ? other - w[j] : w[j] + other;
+    }
+  }
+  float* dst = a.qrot + ((int64_t)b * a.Hq + qh) * 128 + 4 * lane;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) dst[j] = w[j];
+}
+
 // ------------------------------------------------------- fp16 stage tokens ----
 
 // Staged tokens are few (< block): one warp per token, lane = 4 dims, CUDA cores.
@@ -680,6 +839,17 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
     const int c = i >> 7, d = i & 127;
     sh.q[c][d] = c < G ? a.q[((int64_t)b * a.Hq + h * G + c) * 128 + d] : (uint16_t)0;
   }
+  if (a.base == SEMKV_BASE_TQ) {
+    for (int i = threadIdx.x; i < 8 * 128; i += kThreads) {
+      const int c = i >> 7, d = i & 127;
+      sh.qr[c][d] = c < G ? a.qrot[((int64_t)b * a.Hq + h * G + c) * 128 + d] : 0.0f;
+    }
+    if (threadIdx.x < 16) {
+      const int which = threadIdx.x >> 3, k = threadIdx.x & 7;
+      const int L = which == 0 ? a.L_hi : a.L_lo;
+      sh.cb[which][k] = k < L ? (which == 0 ? a.cb_hi : a.cb_lo)[k] : 0.0f;
+    }
+  }
   if (threadIdx.x < kWarps * kStages) mbar_init(&sh.bar[0][0] + threadIdx.x);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncthreads();
@@ -696,8 +866,23 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
   const int t_begin = min(ntiles, s_idx * per), t_end = min(ntiles, t_begin + per);
   const int L = src == 0 ? a.L_hi : a.L_lo;
 
+  const bool tq = a.base == SEMKV_BASE_TQ && src != 2;
   if (src == 2) {
     run_stage(a, sh, b, h, G, merge_m, merge_l, merge_z, merge_o);
+  } else if (tq) {
+    const int64_t cap = src == 0 ? a.hi_cap : a.lo_cap;
+    const int64_t count = src == 0 ? a.hi_count : a.lo_count;
+    const uint8_t* pool = src == 0 ? a.hi_pool : a.lo_pool;
+    const int rec = record_bytes_rt(SEMKV_BASE_TQ, L);
+    const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
+    switch (L) {
+#define SEMKV_TQ_CASE(LV) \
+      case LV: run_pool_tq<LV>(a, sh, src, pool_bh, count, t_begin, t_end, G, merge_m, merge_l, merge_z, merge_o); break;
+      SEMKV_TQ_CASE(2) SEMKV_TQ_CASE(3) SEMKV_TQ_CASE(4) SEMKV_TQ_CASE(5)
+      SEMKV_TQ_CASE(6) SEMKV_TQ_CASE(7) SEMKV_TQ_CASE(8)
+#undef SEMKV_TQ_CASE
+      default: break;
+    }
   } else {
     WarpState st;
     state_init(st);
@@ -800,6 +985,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
     cta_z[qh] = zsum;
   }
   __syncthreads();
+  float* merged = merge_o + kWarps * 8 * 128;  // [8][128], after the warp rows
   for (int i = threadIdx.x; i < G * 128; i += kThreads) {
     const int qh = i >> 7, d = i & 127;
     float o = 0.0f;
@@ -807,13 +993,34 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
       const float sc = cta_scale[w * 8 + qh];
       if (sc != 0.0f) {
         float v = merge_o[(w * 8 + qh) * 128 + d];
-        if (src != 2 && G <= 4) v += merge_o[(w * 8 + qh + 4) * 128 + d];
+        if (src != 2 && !tq && G <= 4) v += merge_o[(w * 8 + qh + 4) * 128 + d];
         o += sc * v;
       }
     }
-    // pool rows hold sum p' c; the offset part is sum p z; staged rows are plain
-    // sums of p v
-    part[16 + qh * 128 + d] = src == 2 ? o : o + cta_z[qh];
+    // affine pool rows hold sum p' c, plus the offset part sum p z; TQ rows and
+    // staged rows are plain weighted sums
+    merged[qh * 128 + d] = (src == 2 || tq) ? o : o + cta_z[qh];
+  }
+  __syncthreads();
+  if (tq) {
+    // back from the rotated domain: o = S H o' (unnormalised transform, stages 1..64)
+    for (int hs = 1; hs < 128; hs <<= 1) {
+      for (int i = threadIdx.x; i < G * 64; i += kThreads) {
+        const int qh = i >> 6, j = i & 63;
+        const int lo = (j / hs) * 2 * hs + (j % hs);
+        float* r = merged + qh * 128;
+        const float x = r[lo], y = r[lo + hs];
+        r[lo] = x + y;
+        r[lo + hs] = x - y;
+      }
+      __syncthreads();
+    }
+  }
+  const int8_t* sg = tq ? a.signs + ((int64_t)a.layer * a.H + h) * 128 : nullptr;
+  for (int i = threadIdx.x; i < G * 128; i += kThreads) {
+    const int qh = i >> 7, d = i & 127;
+    const float o = merged[qh * 128 + d];
+    part[16 + qh * 128 + d] = tq ? o * (float)sg[d] : o;
   }
 }
 
@@ -918,6 +1125,12 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
     attr_set = true;
   }
   if (a.plan.splits == 0) return cudaErrorInvalidValue;
+  if (a.base == SEMKV_BASE_TQ) {
+    const int heads = a.B * a.Hq;
+    qrot_kernel<<<(heads + 7) / 8, 256, 0, stream>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
   dim3 grid(a.plan.splits, a.H, a.B);
   decode_kernel<<<grid, kThreads, kRingBytes, stream>>>(a);
   cudaError_t e = cudaGetLastError();

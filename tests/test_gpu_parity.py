@@ -153,3 +153,35 @@ def test_append_blocks_and_flush_match_oracle():
     p.assert_records_equal()
     assert p.cache.stage_n == 0 and p.cache.n_tokens == T0 + ngen
     check_attention(p, layer=1, qseed=99)
+
+
+# ------------------------------------------------------------ TQ decode -----
+
+@pytest.mark.parametrize("L_hi,L_lo,B,NL,H,Hq,T,r", [
+    (4, 3, 1, 2, 2, 8, 333, (3, 4)),        # the 2.0/1.585-bit TQ mix at r = 75%
+    (4, 3, 2, 1, 8, 32, 1100, (3, 4)),      # Mistral-7B layer shape, short context
+    (2, 2, 1, 1, 2, 4, 100, (0, 1)),
+    (6, 5, 1, 1, 2, 16, 150, (1, 4)),
+    (8, 7, 1, 1, 1, 1, 64, (1, 2)),
+])
+def test_tq_decode_attention_matches_oracle(L_hi, L_lo, B, NL, H, Hq, T, r):
+    p = Pair(1, L_hi, L_lo, B, NL, H, Hq, T, r[0], r[1], seed=40 + T)
+    p.quantize()
+    p.assert_records_equal()
+    for layer in range(NL):
+        check_attention(p, layer)
+
+
+def test_tq_decode_with_staged_tail():
+    import torch
+    p = Pair(1, 4, 3, 1, 1, 2, 8, 200, 3, 4, seed=51, block=32)
+    p.quantize()
+    k, v = synthetic.kv(52, 1, 1, 2, 11)
+    s = synthetic.scores_zipf(52, 1, 11)
+    for g in range(11):
+        kt = torch.from_numpy(np.ascontiguousarray(k[:, :, :, g])).to(p.dev)
+        vt = torch.from_numpy(np.ascontiguousarray(v[:, :, :, g])).to(p.dev)
+        p.cache.stage_token(kt, vt, torch.from_numpy(np.ascontiguousarray(s[:, g])).to(p.dev))
+        oracle.stage_token(p.oc, synthetic.f16_bits(k[:, :, :, g]), synthetic.f16_bits(v[:, :, :, g]),
+                           s[:, g])
+    check_attention(p)
