@@ -27,6 +27,7 @@ import argparse
 import json
 import math
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -57,6 +58,25 @@ CONFIGS = {
                    seed=2, desc="batch 1 x 32K context, 1 layer of the Llama-3.1-8B KV shape, "
                                 "affine 6/5 levels at r=26%"),
 }
+
+
+def profiled_traffic(config_name: str):
+    """DRAM bytes per decode launch from the committed ncu summary, or None when the
+    summary does not cover this workload or the decode kernel source has changed since
+    the counters were taken (its sha256 prefix is recorded beside the figure)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "decode_kernel_b4x64k.md")
+    src = os.path.join(ROOT, "paper_2608_28911_gb300", "csrc", "decode.cu")
+    try:
+        text = open(path).read()
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_launch_%s: (\d+)" % re.escape(config_name), text)
+    h = re.search(r"source_sha256_prefix: ([0-9a-f]+)", text)
+    if not m or not h or not digest.startswith(h.group(1)):
+        return None
+    return int(m.group(1))
 
 
 def load_peaks():
@@ -413,7 +433,7 @@ def main():
         "decode_frac_of_nominal_8tbs": achieved / 8000.0,
         "quantize_gbs": r["quantize_gbs"],
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None,
+                     "frac": achieved / peak, "traffic": profiled_traffic(args.config),
                      "kernel": "decode_kernel+combine_kernel (semkv_decode_attention)",
                      "peak_kind": f"{peak_kind} hbm_gbs"},
         "e2e": {"value": total_bytes / r["e2e_time"] / 1e9, "unit": "GB/s",

@@ -78,3 +78,23 @@ def signs(seed: int, layers: int, kv_heads: int) -> np.ndarray:
 def f16_bits(a: np.ndarray) -> np.ndarray:
     """View a float16 array as its uint16 bit patterns."""
     return np.ascontiguousarray(a, dtype=np.float16).view(np.uint16)
+
+
+def kv_layer_device(seed: int, layer: int, batch: int, kv_heads: int, T: int, device,
+                    outliers: int = 4, factor: float = 8.0):
+    """Like kv_layer, drawn on the GPU (torch's seeded CUDA generator) for caches too
+    large to draw on the host; outlier channels come from the same numpy stream.
+    Returns float16 torch tensors [batch][kv_heads][T][128] on `device`."""
+    import torch
+    ro = _rng(seed, STREAM_OUTLIERS, layer)
+    chans = [ro.choice(HEAD_DIM, outliers, replace=False) for _ in range(kv_heads)]
+    out = []
+    for stream in (STREAM_K, STREAM_V):
+        g = torch.Generator(device=device)
+        g.manual_seed(seed * 1000 + stream + 10000 * layer)
+        x = torch.randn((batch, kv_heads, T, HEAD_DIM), generator=g, device=device,
+                        dtype=torch.float32)
+        for h in range(kv_heads):
+            x[:, h, :, torch.as_tensor(chans[h], device=device)] *= factor
+        out.append(x.to(torch.float16))
+    return out[0], out[1]
