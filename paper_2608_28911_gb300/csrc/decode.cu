@@ -17,25 +17,26 @@
 // constant L^(k+1)/2^W yields a float whose bit pattern is F_k.  For five-level
 // groups two symbols share one multiply (beta_a + 65536 beta_b is still a denormal)
 // and a mask separates the halves.  Integers (all < 256) become fp16 values with a
-// byte permute (1024 + v) and one f16x2 subtract.
-//  - QK^T as S^T = F Q'^T on mma.sync m16n8k16 (M = 16 tokens, K = 128 F slots,
-//    N = 8 columns): the q coefficient of F_k is q'_k = q_{d_k} - L q_{d_{k+1}}
-//    when F_k carries a share of digit k+1, split into fp16 hi + lo parts (the lo
-//    parts ride in the spare columns 4..7 when G <= 4, else a second pass);
-//    logit = scale log2e (s acc + z sum q), online softmax in base 2, rescaling only
-//    when some logit exceeds the running max;
-//  - P V as O^T = C^T P'^T (M = 128 dims, N = 8 heads, K = 16 tokens) on the digits
-//    c_k (formed lane-wise as P_k - L P_{k-1}, never negative, so nothing borrows
-//    across halves), with P' = p * s_v as fp16 hi + lo (lo again in columns 4..7),
-//    plus sum p * z_v per head.  (Feeding F values to PV and undoing the mixing after
-//    accumulation was tried and rejected: the subtraction cancels ~30x and amplified
-//    the tensor cores' fp32 accumulation error past the attention tolerance.)
+// byte placed over them (1024 + v) and one f16x2 subtract.
+//  - QK^T as S = Q' F^T on mma.sync m16n8k16 (M = heads, N = 8 tokens, K = 128 F
+//    slots): the q coefficient of F_k is q'_k = q_{d_k} - L q_{d_{k+1}} when F_k
+//    carries a share of digit k+1, scaled by a power of two and split into fp16 hi
+//    and lo rows; logit = scale log2e (s acc + z sum q).  The output fragment is
+//    the B operand of the PV product as it stands (at most one exchange of halves).
+//  - softmax in base 2 against a per-head reference exponent e that keeps p and
+//    p * s_v below 2^14; e moves, and the running sums are rescaled, only when a tile
+//    would exceed that bound.
+//  - P V as O^T = C^T P'^T (M = 128 dims, N = 8 columns, K = 16 tokens) on the digits
+//    c_k (formed lane-wise as F_k - L F_{k-1} in f16x2), with P' = p * s_v as fp16
+//    hi + lo (lo in columns 4..7 when G <= 4, else a second pass), plus sum p * z_v
+//    per head.  (Feeding F values to PV and undoing the mixing after accumulation was
+//    tried and rejected: the subtraction cancels ~30x and amplified the tensor
+//    cores' truncating fp32 accumulation past the attention tolerance.)
 // Six-level groups (F_4 up to 7775 would not fit) restart the chain after two
 // digits from the remainder x = beta * 36 mod 2^13.
 //
 // Per warp: a 4-deep ring of cp.async.bulk tile copies completing on per-stage
-// mbarriers (bounded waits that report a timeout in the error word), online
-// softmax in base 2, lazy rescaling only when a running max grows.
+// mbarriers (bounded waits that report a timeout in the error word).
 #include <float.h>
 
 #include "common.cuh"
@@ -52,6 +53,8 @@ constexpr int kTile = 16;
 constexpr int kMaxRec = 104;
 constexpr int kStageBytes = kTile * kMaxRec + 16;  // +16: window loads may run 12 B past a tile
 constexpr int kRingBytes = kWarps * kStages * kStageBytes;
+constexpr int kAqBytes = kWarps * 8 * 32 * 16;       // per warp: 8 k-steps x 32 lanes x uint4
+constexpr int kDynBytes = kRingBytes + kAqBytes;
 constexpr int kMaxSplits = 64;                     // pool splits per (b, h)
 constexpr uint32_t kSpinLimit = 1u << 22;
 
@@ -116,19 +119,21 @@ __device__ __forceinline__ uint32_t fdig(uint32_t beta, float c) {
 __device__ __forceinline__ uint32_t fdig1024(uint32_t beta, float c) {
   return __float_as_uint(__fmaf_rz(__uint_as_float(beta), c, __uint_as_float(0x6400u)));
 }
-__device__ __forceinline__ uint32_t lo16hi16(uint32_t a, uint32_t b) {
+// the low halves of a and b side by side
+__device__ __forceinline__ uint32_t fpair(uint32_t a, uint32_t b) {
   return __byte_perm(a, b, 0x5410);
 }
-// subtract 1024 from both fp16 halves: 1024 + v -> v exactly (v < 1024)
+// subtract 1024 from both fp16 halves: 1024 + v -> v exactly (v < 1024).  Integers
+// reach the tensor cores as normal fp16 values: read directly as the subnormals
+// v * 2^-24 they multiply exactly in isolation, but a chained accumulation over
+// subnormal operands loses about 10 bits (measured: ~1e-3 relative attention error).
 __device__ __forceinline__ uint32_t hsub1024(uint32_t x) {
   uint32_t r;
   asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(x), "r"(0x64006400u));
   return r;
 }
-// integers in bytes 0 and 2 (< 256; bytes 1 and 3 ignored) -> fp16 values: the byte
-// 0x64 over each makes 1024 + v.  (The integers read directly as fp16 subnormals
-// v * 2^-24 were tried first: the tensor cores lose products of subnormal operands
-// with small weights, biasing attention by ~1e-5 of the low-weight mass per mma.)
+// integers in bytes 0 and 2 (< 256; bytes 1 and 3 ignored) -> fp16 values: one byte
+// permute lays 0x64 over each (1024 + v) and one f16x2 subtract removes the 1024
 __device__ __forceinline__ uint32_t bytes_to_h2(uint32_t P) {
   return hsub1024(__byte_perm(P, 0x64646464u, 0x7250));
 }
@@ -145,10 +150,25 @@ __device__ __forceinline__ uint32_t hdigit(uint32_t prev, uint32_t cur) {
   asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(r) : "r"(prev), "r"(kNegL), "r"(cur));
   return r;
 }
-
-__device__ __forceinline__ uint32_t h2(float lo, float hi) {
-  return (uint32_t)__half_as_ushort(__float2half_rn(lo)) |
-         ((uint32_t)__half_as_ushort(__float2half_rn(hi)) << 16);
+__device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
+  const __half2 h = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+// x0, x1 as fp16 hi + lo parts, packed pairwise (exact to ~2^-22 relative)
+__device__ __forceinline__ void split_h2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __half2 h = __floats2half2_rn(x0, x1);
+  const float2 f = __half22float2(h);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = pack_h2(x0 - f.x, x1 - f.y);
+}
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+// the largest power of two <= x (x positive and normal)
+__device__ __forceinline__ float pow2_floor(float x) {
+  return __uint_as_float(__float_as_uint(x) & 0x7F800000u);
 }
 
 // ------------------------------------------------------------ decoding --------
@@ -194,7 +214,8 @@ struct Dec {
   // 1024 + F values of one full symbol, in the low 16 bits of each word (F < 256)
   __device__ __forceinline__ static void sym(uint32_t beta, uint32_t* f) {
     if constexpr (G == 1) {
-      f[0] = fdig1024(beta, (float)L / (float)(1u << F::W));
+      // L = 2, 4, 8 store the code itself; seven levels take one multiply
+      f[0] = L == 7 ? fdig1024(beta, 7.0f / 8.0f) : (beta | 0x6400u);
     } else if constexpr (L == 6) {
       constexpr float c1 = 6.0f / 8192.0f, c2 = 36.0f / 8192.0f, c3 = 216.0f / 8192.0f;
       f[0] = fdig1024(beta, c1);
@@ -222,24 +243,10 @@ struct Dec {
   __host__ __device__ static constexpr bool chained(int k) { return k + 1 < G && k + 1 != kRestart; }
 };
 
-// fp16 F pairs (low half symbol a, high half symbol b) of two symbols
-template <int L>
-__device__ __forceinline__ void pair_F(const uint32_t* fa, const uint32_t* fb, uint32_t* X) {
-#pragma unroll
-  for (int k = 0; k < Dec<L>::G; ++k) X[k] = hsub1024(lo16hi16(fa[k], fb[k]));
-}
-// digits from fp16 F pairs: c_k = F_k - L F_{k-1}, the chain restarting at kRestart
-template <int L>
-__device__ __forceinline__ void F_to_digits(const uint32_t* X, uint32_t* h) {
-#pragma unroll
-  for (int k = 0; k < Dec<L>::G; ++k)
-    h[k] = (k == 0 || k == Dec<L>::kRestart) ? X[k] : hdigit<L>(X[k - 1], X[k]);
-}
-
 // ---- five-level fast path: two 7-bit symbols per register ---------------------
 // u = beta_a + 65536 beta_b is still a denormal (beta < 128), and
-// floor(u * L^(k+1)/128) = F_k(a) + 65536 F_k(b) + (fraction of b) * 512: one
-// multiply gives both halves' F_k (bytes 0 and 2; the fraction lands in byte 1).
+// floor(u * 5^(k+1)/128) = F_k(a) + 65536 F_k(b) + 512 * (fraction of b's product):
+// one multiply gives both halves' F_k (bytes 0 and 2; the fraction lands in byte 1).
 constexpr uint32_t kM7 = 0x007F007Fu;
 __device__ __forceinline__ void l5_fpairs(uint32_t u, uint32_t* X) {
   X[0] = bytes_to_h2(fdig(u, 5.0f / 128.0f));
@@ -250,23 +257,31 @@ __device__ __forceinline__ void l5_fpairs(uint32_t u, uint32_t* X) {
 // in the high half, j = 0..4 (bits 7j)
 __device__ __forceinline__ void l5_pairs(uint32_t a0, uint32_t a1, uint32_t b0, uint32_t b1,
                                          uint32_t u[5]) {
-  uint32_t C = lo16hi16(a0, b0);
+  uint32_t C = fpair(a0, b0);
   u[0] = C & kM7;
   u[1] = (C >> 7) & kM7;
-  C = lo16hi16(a0 >> 14, b0 >> 14);
+  C = fpair(a0 >> 14, b0 >> 14);
   u[2] = C & kM7;
   u[3] = (C >> 7) & kM7;
-  C = lo16hi16(__funnelshift_r(a0, a1, 28), __funnelshift_r(b0, b1, 28));
+  C = fpair(__funnelshift_r(a0, a1, 28), __funnelshift_r(b0, b1, 28));
   u[4] = C & kM7;
 }
+// the two-code five-level tail of two windows at once (5-bit symbols, u < 2^21):
+// F_0 and F_1 pairs (bytes 0 and 2); the fraction of the high symbol lands in bits 11..15
+__device__ __forceinline__ void l5_tail_pairs(uint32_t ut, uint32_t& X0, uint32_t& X1) {
+  X0 = bytes_to_h2(fdig(ut, 5.0f / 32.0f));
+  X1 = bytes_to_h2(fdig(ut, 25.0f / 32.0f));
+}
 
-// K side: the 16 fp16 F-value pairs of one quarter row of one token (both halves are
-// the same token).  Slot p < kHalf*G holds F_k of symbols s and s + kHalf
-// (s = p / G, k = p % G); slot 15 holds the tail's F_0 and F_1.
+// F side of S = Q' F^T: the fp16 F-value pairs of one quarter row of one token (both
+// halves are the same token), as the B fragments of the 8 k-steps: slot p = 2j + i
+// goes to f[j][i].  Slot p < kHalf*G holds F_k of symbols s and s + kHalf (s = p / G,
+// k = p % G); slot 15 holds the tail's F_0 and F_1.
 template <int L>
-__device__ __forceinline__ void k_quarter(const Window& w, uint32_t h[16]) {
+__device__ __forceinline__ void k_quarter(const Window& w, uint32_t (&f)[8][2]) {
   using D = Dec<L>;
   using F = typename D::F;
+  uint32_t h[16];
   if constexpr (L == 5) {
     uint32_t u[5];
     // symbol s + 5 sits 35 bits after symbol s
@@ -275,28 +290,31 @@ __device__ __forceinline__ void k_quarter(const Window& w, uint32_t h[16]) {
     for (int s = 0; s < 5; ++s) l5_fpairs(u[s], h + 3 * s);
     uint32_t ft[2];
     D::tail(wbits(w, 70, 5), ft);
-    h[15] = hsub1024(lo16hi16(ft[0], ft[1]));
+    h[15] = hsub1024(fpair(ft[0], ft[1]));
   } else {
 #pragma unroll
     for (int s = 0; s < D::kHalf; ++s) {
       uint32_t fa[D::G], fb[D::G];
       D::sym(wbits(w, s * F::W, F::W), fa);
       D::sym(wbits(w, (s + D::kHalf) * F::W, F::W), fb);
-      pair_F<L>(fa, fb, h + s * D::G);
+#pragma unroll
+      for (int k = 0; k < D::G; ++k) h[s * D::G + k] = hsub1024(fpair(fa[k], fb[k]));
     }
     if constexpr (F::R > 0) {
       static_assert(F::R == 2 && D::kHalf * D::G == 15, "tail layout");
       uint32_t ft[2];
       D::tail(wbits(w, F::NG * F::W, F::WT), ft);
-      h[15] = hsub1024(lo16hi16(ft[0], ft[1]));
+      h[15] = hsub1024(fpair(ft[0], ft[1]));
     } else {
       static_assert(D::kHalf * D::G == 16, "layout");
     }
   }
+#pragma unroll
+  for (int p = 0; p < 16; ++p) f[p >> 1][p & 1] = h[p];
 }
 
-// q coefficient of K-side slot p (lo or hi half) of quarter t for one head: the
-// digit k weight minus the share of digit k+1 that F_k carries
+// q coefficient of F slot p (lo or hi half) of quarter t for one head: the digit k
+// weight minus the share of digit k+1 that F_k carries
 template <int L>
 __device__ __forceinline__ float k_coef(const uint16_t* qrow, int t, int p, int half) {
   using D = Dec<L>;
@@ -314,11 +332,14 @@ __device__ __forceinline__ float k_coef(const uint16_t* qrow, int t, int p, int 
 // V side: lane group g holds half hh of quarter qv for two tokens at once (the two
 // halves of each register are the two tokens).  Row u = j*G + k is digit k of
 // symbol hh*kHalf + j; row 15 is the tail's digit hh.  Digits as fp16 values.
-template <int L>
+// The 16 rows land in the A fragments of the 8 m-blocks: row u = 2m + i goes to
+// A[m][C + i] (C = 0 for tokens 2t, 2t+1 and 2 for tokens 2t+8, 2t+9).
+template <int L, int C>
 __device__ __forceinline__ void v_half_pair(const Window& wa, const Window& wb, int tpos, int hh,
-                                            uint32_t h[16]) {
+                                            uint32_t (&A)[8][4]) {
   using D = Dec<L>;
   using F = typename D::F;
+  uint32_t h[16];
   if constexpr (L == 5) {
     uint32_t u[5];
     l5_pairs(wa.q0, wa.q1, wb.q0, wb.q1, u);
@@ -326,11 +347,12 @@ __device__ __forceinline__ void v_half_pair(const Window& wa, const Window& wb, 
     for (int j = 0; j < 5; ++j) {
       uint32_t X[3];
       l5_fpairs(u[j], X);
-      F_to_digits<5>(X, h + 3 * j);
+      h[3 * j] = X[0];
+      h[3 * j + 1] = hdigit<5>(X[0], X[1]);
+      h[3 * j + 2] = hdigit<5>(X[1], X[2]);
     }
-    const uint32_t ut = lo16hi16(wbits_rt(wa, tpos, 5), wbits_rt(wb, tpos, 5));
-    const uint32_t X0 = bytes_to_h2(fdig(ut, 5.0f / 32.0f));
-    const uint32_t X1 = bytes_to_h2(fdig(ut, 25.0f / 32.0f));
+    uint32_t X0, X1;
+    l5_tail_pairs(fpair(wbits_rt(wa, tpos, 5), wbits_rt(wb, tpos, 5)), X0, X1);
     h[15] = hh ? hdigit<5>(X0, X1) : X0;
   } else {
 #pragma unroll
@@ -338,18 +360,23 @@ __device__ __forceinline__ void v_half_pair(const Window& wa, const Window& wb, 
       uint32_t fa[D::G], fb[D::G], X[D::G];
       D::sym(wbits(wa, j * F::W, F::W), fa);
       D::sym(wbits(wb, j * F::W, F::W), fb);
-      pair_F<L>(fa, fb, X);
-      F_to_digits<L>(X, h + j * D::G);
+#pragma unroll
+      for (int k = 0; k < D::G; ++k) X[k] = hsub1024(fpair(fa[k], fb[k]));
+#pragma unroll
+      for (int k = 0; k < D::G; ++k)
+        h[j * D::G + k] = (k == 0 || k == D::kRestart) ? X[k] : hdigit<L>(X[k - 1], X[k]);
     }
     if constexpr (F::R > 0) {
       uint32_t fa[2], fb[2];
       D::tail(wbits_rt(wa, tpos, F::WT), fa);
       D::tail(wbits_rt(wb, tpos, F::WT), fb);
-      const uint32_t X0 = hsub1024(lo16hi16(fa[0], fb[0]));
-      const uint32_t X1 = hsub1024(lo16hi16(fa[1], fb[1]));
+      const uint32_t X0 = hsub1024(fpair(fa[0], fb[0]));
+      const uint32_t X1 = hsub1024(fpair(fa[1], fb[1]));
       h[15] = hh ? hdigit<L>(X0, X1) : X0;
     }
   }
+#pragma unroll
+  for (int u = 0; u < 16; ++u) A[u >> 1][C + (u & 1)] = h[u];
 }
 
 // output dim of V row u of lane group g
@@ -366,10 +393,10 @@ __device__ __forceinline__ int v_dim(int g, int u) {
 // ------------------------------------------------------- per-warp state -------
 
 struct WarpState {
-  float O[8][4];     // O^T accumulators: V rows x columns (heads 2t, 2t+1)
-  float m[2];        // running max (base-2 logits) of this lane's two heads
-  float l[2];        // partial sum of p over this lane's tokens
-  float zs[2];       // partial sum of p*z_v
+  float O[8][4];     // O^T accumulators: V rows x columns 2t, 2t+1
+  float e;           // reference exponent of head g (base 2)
+  float l;           // partial sum of p over this lane's tokens
+  float zs;          // partial sum of p*z_v
 };
 
 __device__ __forceinline__ void state_init(WarpState& st) {
@@ -377,27 +404,36 @@ __device__ __forceinline__ void state_init(WarpState& st) {
   for (int m = 0; m < 8; ++m)
 #pragma unroll
     for (int e = 0; e < 4; ++e) st.O[m][e] = 0.0f;
-#pragma unroll
-  for (int e = 0; e < 2; ++e) {
-    st.m[e] = -INFINITY;
-    st.l[e] = 0.0f;
-    st.zs[e] = 0.0f;
-  }
+  st.e = -INFINITY;
+  st.l = 0.0f;
+  st.zs = 0.0f;
 }
 
 struct Shared {
   uint16_t q[8][128];       // the group's query heads (rows >= G are zero)
   float qr[8][128];         // TQ base: rotated queries q' = H S q
   float cb[2][8];           // TQ base: centroids of the high / low level count
+  float sumq[8];            // sum over dims of each head's q
+  float qmax[8];            // max |q_d| of each head
   uint64_t bar[kWarps][kStages];
 };
 
 // ------------------------------------------------------------ pool tiles ------
 
-// PACKED (G <= 4): the lo parts of the q coefficients ride in B columns 4..7 and one
-// mma per k-step serves both; otherwise a second pass with the lo parts.
+// One warp streams its tiles.  Per 16-token tile:
+//  S = Q' F^T on m16n8k16 in two 8-token halves (N = tokens g, g+8 of lane group g):
+//   A rows g and g+8 are head g's q' coefficients, scaled by a power of two so the
+//   largest is near 2^13 and split into fp16 hi (row g) and lo (row g+8) parts.  The
+//   output fragment (rows = heads, columns = tokens 2t, 2t+1) is, after adding hi and
+//   lo, already laid out as the B fragment the PV product needs: no transposition.
+//  p = 2^(logit - e) with a per-head reference e chosen so p and p*s_v stay <= 2^14:
+//   e moves (and the sums are rescaled) only when a tile would exceed that.
+//  O^T += C^T P'^T (M = 128 V rows, K = 16 tokens) with P' = p*s_v as fp16 hi + lo
+//   (PACKED: columns 0..3 hi and 4..7 lo of heads 0..3; else two passes).
+// Codes enter as exact fp16 integers; the partners' power-of-two scales keep every
+// operand within the fp16 range.
 template <int L, bool PACKED>
-__device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
+__device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint4* aq_all,
                          uint64_t* bars, const uint8_t* pool_bh, int64_t count, int t_begin,
                          int t_end, int G, WarpState& st) {
   using D = Dec<L>;
@@ -410,36 +446,34 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
   uint8_t* my_ring = ring + warp * kStages * kStageBytes;
   uint64_t* my_bar = bars + warp * kStages;
 
-  // B fragments of S^T = F Q'^T: column n = g, rows = this quarter's F slots; the
-  // coefficient q'_k = q_k - L q_{k+1} (when F_k carries a share of digit k+1) is
-  // split into fp16 hi + lo, exact to 2^-22 relative
-  uint32_t bq[16], bq2[16];
-  {
-    const int head = PACKED ? (g & 3) : g;
-    const bool lo_col = PACKED && g >= 4;
+  const bool live = g < G;   // head g: A rows g (hi) and g + 8 (lo), softmax of head g
+  const float qmax = sh.qmax[g];
+  const float qscale =
+      qmax > 0.0f ? pow2_floor(fminf(8192.0f / ((float)(L + 1) * qmax), 1e30f)) : 1.0f;
+  // A fragments of the 8 k-steps, {hi 2j, lo 2j, hi 2j+1, lo 2j+1} per lane, kept in
+  // this warp's slice of shared memory (one conflict-free 16-byte load per k-step)
+  uint4* aq = aq_all + warp * 8 * 32 + lane;
 #pragma unroll
-    for (int p = 0; p < 16; ++p) {
+  for (int j = 0; j < 8; ++j) {
+    uint32_t r[4];
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int p = 2 * j + i;
       float c0 = 0.0f, c1 = 0.0f;
-      if (head < G) {
-        c0 = k_coef<L>(sh.q[head], t, p, 0);
-        c1 = k_coef<L>(sh.q[head], t, p, 1);
+      if (live) {
+        c0 = k_coef<L>(sh.q[g], t, p, 0) * qscale;
+        c1 = k_coef<L>(sh.q[g], t, p, 1) * qscale;
       }
-      const float h0 = __half2float(__float2half_rn(c0)), h1 = __half2float(__float2half_rn(c1));
-      const uint32_t hi = h2(h0, h1), lo = h2(c0 - h0, c1 - h1);
-      bq[p] = lo_col ? lo : hi;
-      bq2[p] = lo;
+      split_h2(c0, c1, r[2 * i], r[2 * i + 1]);
     }
+    aq[32 * j] = make_uint4(r[0], r[1], r[2], r[3]);
   }
-  // logit heads of this lane: PACKED folds column c+4 (lo) onto column c (hi)
-  const int hc0 = PACKED ? 2 * (t & 1) : 2 * t;
-  float sumq[2];
-#pragma unroll
-  for (int c = 0; c < 2; ++c) {
-    float s = 0.0f;
-    if (hc0 + c < G)
-      for (int d = 0; d < 128; ++d) s += f16_to_f32(sh.q[hc0 + c][d]);
-    sumq[c] = s;
-  }
+  __syncwarp();
+  const float cS = a.scale_log2 / qscale;   // logit weight of s_k * S
+  const float cZ = a.scale_log2 * sh.sumq[g];  // logit weight of z_k
+  // O columns 2t, 2t+1 belong to these heads (their e lives in lane 4*head)
+  const int oh0 = PACKED ? ((2 * t) & 3) : 2 * t, oh1 = oh0 + 1;
+
   const int qv = g >> 1, hh = g & 1;
   const int vpos = 8 * F::RB + qv * F::QB + hh * D::kHalf * F::W;  // V half quarter
   const int tpos = F::NG * F::W - hh * D::kHalf * F::W;           // tail, relative
@@ -466,125 +500,97 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
     const uint8_t* tb = my_ring + stage * kStageBytes;
     const int nvalid = (int)min((int64_t)kTile, count - (int64_t)tile * kTile);
 
-    // ---- S^T = F Q'^T (two accumulators: two short dependency chains)
-    float acc[4] = {0.f, 0.f, 0.f, 0.f}, acc2[4] = {0.f, 0.f, 0.f, 0.f};
+    // ---- S = Q' F^T, tokens 0..7 and 8..15
+    float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
     {
-      uint32_t h0[16], h1[16];
-      k_quarter<L>(load_window(tb + g * kRec, t * F::QB), h0);
-      k_quarter<L>(load_window(tb + (g + 8) * kRec, t * F::QB), h1);
+      uint32_t f0[8][2], f1[8][2];
+      k_quarter<L>(load_window(tb + g * kRec, t * F::QB), f0);
+      k_quarter<L>(load_window(tb + (g + 8) * kRec, t * F::QB), f1);
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        mma16816((j & 1) ? acc2 : acc, h0[2 * j], h1[2 * j], h0[2 * j + 1], h1[2 * j + 1],
-                 bq[2 * j], bq[2 * j + 1]);
-        if constexpr (!PACKED)
-          mma16816((j & 1) ? acc : acc2, h0[2 * j], h1[2 * j], h0[2 * j + 1], h1[2 * j + 1],
-                   bq2[2 * j], bq2[2 * j + 1]);
-      }
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        acc[e] += acc2[e];
-        if constexpr (PACKED) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], 2);
+        const uint4 A = aq[32 * j];
+        mma16816(s0, A.x, A.y, A.z, A.w, f0[j][0], f0[j][1]);
+        mma16816(s1, A.x, A.y, A.z, A.w, f1[j][0], f1[j][1]);
       }
     }
-    // ---- logits and online softmax (base 2)
-    float p[2][2];
-    uint32_t X[2], Xl[2];
-    {
-      float lg[2][2], sv[2], zv[2];
-      bool valid[2];
+    // ---- logits of head g for tokens 2t, 2t+1, 2t+8, 2t+9 (hi + lo rows)
+    const float S[4] = {s0[0] + s0[2], s0[1] + s0[3], s1[0] + s1[2], s1[1] + s1[3]};
+    float lg[4], sv[4], zv[4], p[4], P[4];
+    bool valid[4];
+    bool bad = false;
 #pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int tok = g + 8 * e;
-        const uint32_t* prm = reinterpret_cast<const uint32_t*>(tb + tok * kRec + 2 * F::RB);
-        const uint32_t kp = prm[0], vp = prm[1];
-        const float sk = f16_to_f32((uint16_t)(kp & 0xFFFF)), zk = f16_to_f32((uint16_t)(kp >> 16));
-        sv[e] = f16_to_f32((uint16_t)(vp & 0xFFFF));
-        zv[e] = f16_to_f32((uint16_t)(vp >> 16));
-        valid[e] = tok < nvalid;
-        const float A = a.scale_log2 * sk;
-        const float Bz = a.scale_log2 * zk;
+    for (int i = 0; i < 4; ++i) {
+      const int tok = 2 * t + (i & 1) + 8 * (i >> 1);
+      const uint32_t* prm = reinterpret_cast<const uint32_t*>(tb + tok * kRec + 2 * F::RB);
+      const uint32_t kp = prm[0], vp = prm[1];
+      const float sk = f16_to_f32((uint16_t)(kp & 0xFFFF)), zk = f16_to_f32((uint16_t)(kp >> 16));
+      valid[i] = live && tok < nvalid;
+      // rows past the pool's count are not data: keep whatever they hold out of the sums
+      sv[i] = valid[i] ? f16_to_f32((uint16_t)(vp & 0xFFFF)) : 0.0f;
+      zv[i] = valid[i] ? f16_to_f32((uint16_t)(vp >> 16)) : 0.0f;
+      lg[i] = fmaf(sk * cS, S[i], zk * cZ);
+      p[i] = valid[i] ? ex2(lg[i] - st.e) : 0.0f;
+      P[i] = p[i] * sv[i];
+      bad |= !(p[i] <= 16384.0f) || !(P[i] <= 16384.0f);
+    }
+    if (__any_sync(0xffffffffu, bad)) {
+      // move e up to (max over the head's tokens of logit + log2 max(s_v, 1)) - 12
+      float mx = -INFINITY;
 #pragma unroll
-        for (int c = 0; c < 2; ++c)
-          lg[e][c] = valid[e] ? fmaf(A, acc[2 * e + c], Bz * sumq[c]) : -INFINITY;
-      }
-      // rescale only when some logit of the warp exceeds its running max (rare once
-      // the max has settled); then the tile max comes from the shuffles
-      const bool over = lg[0][0] > st.m[0] || lg[1][0] > st.m[0] || lg[0][1] > st.m[1] ||
-                        lg[1][1] > st.m[1];
-      if (__any_sync(0xffffffffu, over)) {
-        float al[2];
+      for (int i = 0; i < 4; ++i)
+        if (valid[i]) mx = fmaxf(mx, lg[i] + fmaxf(0.0f, __log2f(sv[i])));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float e_new = fmaxf(st.e, mx - 12.0f);
+      const float al = st.e == -INFINITY ? 0.0f : ex2(st.e - e_new);
+      st.e = e_new;
+      st.l *= al;
+      st.zs *= al;
+      const float a0 = __shfl_sync(0xffffffffu, al, 4 * oh0);
+      const float a1 = __shfl_sync(0xffffffffu, al, 4 * oh1);
 #pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          float mx = fmaxf(lg[0][c], lg[1][c]);
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-          const float mnew = fmaxf(st.m[c], mx);
-          al[c] = (st.m[c] == -INFINITY) ? 0.0f : exp2f(st.m[c] - mnew);
-          st.m[c] = mnew;
-          st.l[c] *= al[c];
-          st.zs[c] *= al[c];
-        }
-        // O columns are heads 2t, 2t+1: for PACKED lanes t >= 2 they are padding
-#pragma unroll
-        for (int m = 0; m < 8; ++m) {
-          st.O[m][0] *= al[0];
-          st.O[m][1] *= al[1];
-          st.O[m][2] *= al[0];
-          st.O[m][3] *= al[1];
-        }
+      for (int m = 0; m < 8; ++m) {
+        st.O[m][0] *= a0;
+        st.O[m][1] *= a1;
+        st.O[m][2] *= a0;
+        st.O[m][3] *= a1;
       }
 #pragma unroll
-      for (int c = 0; c < 2; ++c) {
-#pragma unroll
-        for (int e = 0; e < 2; ++e) p[e][c] = valid[e] ? exp2f(lg[e][c] - st.m[c]) : 0.0f;
-        // P' = p * s_v as fp16 hi + lo (exact to 2^-22 relative)
-        const float P0 = p[0][c] * sv[0], P1 = p[1][c] * sv[1];
-        const float H0 = __half2float(__float2half_rn(P0)), H1 = __half2float(__float2half_rn(P1));
-        X[c] = h2(H0, H1);
-        Xl[c] = h2(P0 - H0, P1 - H1);
-        st.l[c] += p[0][c] + p[1][c];
-        st.zs[c] += p[0][c] * zv[0] + p[1][c] * zv[1];
+      for (int i = 0; i < 4; ++i) {
+        p[i] = valid[i] ? ex2(lg[i] - st.e) : 0.0f;
+        P[i] = p[i] * sv[i];
       }
     }
-    // ---- P'^T into the B fragment: rows = tokens 2t, 2t+1, 2t+8, 2t+9; column g is
-    // head g (hi parts), or for PACKED columns 4..7 the lo parts of heads 0..3
-    uint32_t b0, b1, b0l = 0u, b1l = 0u;
-    {
-      const int hd = PACKED ? (g & 3) : g;
-      const int src0 = (2 * t) * 4 + (hd >> 1), src1 = (2 * t + 1) * 4 + (hd >> 1);
-      const uint32_t v0 = __shfl_sync(0xffffffffu, X[0], src0);
-      const uint32_t v1 = __shfl_sync(0xffffffffu, X[1], src0);
-      const uint32_t w0 = __shfl_sync(0xffffffffu, X[0], src1);
-      const uint32_t w1 = __shfl_sync(0xffffffffu, X[1], src1);
-      const uint32_t vl0 = __shfl_sync(0xffffffffu, Xl[0], src0);
-      const uint32_t vl1 = __shfl_sync(0xffffffffu, Xl[1], src0);
-      const uint32_t wl0 = __shfl_sync(0xffffffffu, Xl[0], src1);
-      const uint32_t wl1 = __shfl_sync(0xffffffffu, Xl[1], src1);
-      const bool odd = hd & 1, live = hd < G;
-      const uint32_t Ah = odd ? v1 : v0, Bh = odd ? w1 : w0;    // tokens 2t|2t+8, 2t+1|2t+9
-      const uint32_t Al = odd ? vl1 : vl0, Bl = odd ? wl1 : wl0;
-      const bool use_lo = PACKED && g >= 4;
-      const uint32_t A = use_lo ? Al : Ah, B = use_lo ? Bl : Bh;
-      b0 = live ? __byte_perm(A, B, 0x5410) : 0u;
-      b1 = live ? __byte_perm(A, B, 0x7632) : 0u;
-      if constexpr (!PACKED) {
-        b0l = live ? __byte_perm(Al, Bl, 0x5410) : 0u;
-        b1l = live ? __byte_perm(Al, Bl, 0x7632) : 0u;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      st.l += p[i];
+      st.zs = fmaf(p[i], zv[i], st.zs);
+    }
+    // ---- P'^T as the B fragment: rows = tokens (2t, 2t+1 | 2t+8, 2t+9), column g
+    uint32_t b0, b1, b0l, b1l;
+    split_h2(P[0], P[1], b0, b0l);
+    split_h2(P[2], P[3], b1, b1l);
+    if constexpr (PACKED) {
+      // columns 4..7 carry the lo parts of heads 0..3, computed by lanes g - 4
+      const uint32_t r0 = __shfl_xor_sync(0xffffffffu, b0l, 16);
+      const uint32_t r1 = __shfl_xor_sync(0xffffffffu, b1l, 16);
+      if (g >= 4) {
+        b0 = r0;
+        b1 = r1;
       }
     }
     // ---- O^T += C^T P'^T
     {
-      uint32_t ha[16], hb[16];
-      v_half_pair<L>(load_window(tb + (2 * t) * kRec, vpos),
-                     load_window(tb + (2 * t + 1) * kRec, vpos), tpos, hh, ha);
-      v_half_pair<L>(load_window(tb + (2 * t + 8) * kRec, vpos),
-                     load_window(tb + (2 * t + 9) * kRec, vpos), tpos, hh, hb);
+      uint32_t VA[8][4];
+      v_half_pair<L, 0>(load_window(tb + (2 * t) * kRec, vpos),
+                        load_window(tb + (2 * t + 1) * kRec, vpos), tpos, hh, VA);
+      v_half_pair<L, 2>(load_window(tb + (2 * t + 8) * kRec, vpos),
+                        load_window(tb + (2 * t + 9) * kRec, vpos), tpos, hh, VA);
 #pragma unroll
       for (int m = 0; m < 8; ++m) {
-        mma16816(st.O[m], ha[2 * m], ha[2 * m + 1], hb[2 * m], hb[2 * m + 1], b0, b1);
+        mma16816(st.O[m], VA[m][0], VA[m][1], VA[m][2], VA[m][3], b0, b1);
         if constexpr (!PACKED)
-          mma16816(st.O[m], ha[2 * m], ha[2 * m + 1], hb[2 * m], hb[2 * m + 1], b0l, b1l);
+          mma16816(st.O[m], VA[m][0], VA[m][1], VA[m][2], VA[m][3], b0l, b1l);
       }
     }
     __syncwarp();
@@ -828,6 +834,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
   __shared__ float merge_m[kWarps * 8], merge_l[kWarps * 8], merge_z[kWarps * 8];
   __shared__ float cta_scale[kWarps * 8], cta_z[8];
   uint8_t* ring = dyn;
+  uint4* aq_all = reinterpret_cast<uint4*>(dyn + kRingBytes);
   float* merge_o = reinterpret_cast<float*>(dyn);  // [kWarps][8][128] output rows
 
   const int b = blockIdx.z, h = blockIdx.y, split = blockIdx.x;
@@ -852,6 +859,27 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
   }
   if (threadIdx.x < kWarps * kStages) mbar_init(&sh.bar[0][0] + threadIdx.x);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  __syncthreads();
+  {
+    // per head: sum of q (the zero-point weight) and max |q| (the coefficient scale)
+    static_assert(kWarps == 8, "one warp per head slot");
+    float s = 0.0f, mx = 0.0f;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float x = f16_to_f32(sh.q[warp][4 * lane + j]);
+      s += x;
+      mx = fmaxf(mx, fabsf(x));
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      s += __shfl_xor_sync(0xffffffffu, s, off);
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    }
+    if (lane == 0) {
+      sh.sumq[warp] = s;
+      sh.qmax[warp] = mx;
+    }
+  }
   __syncthreads();
 
   int src, s_idx, nsrc, ntiles;
@@ -893,44 +921,34 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
     const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
     uint64_t* bars = &sh.bar[0][0];
     switch (L) {
-      case 2: G <= 4 ? run_pool<2, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<2, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 3: G <= 4 ? run_pool<3, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<3, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 4: G <= 4 ? run_pool<4, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<4, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 5: G <= 4 ? run_pool<5, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<5, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 6: G <= 4 ? run_pool<6, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<6, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 7: G <= 4 ? run_pool<7, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<7, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 8: G <= 4 ? run_pool<8, true>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<8, false>(a, sh, ring, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 2: G <= 4 ? run_pool<2, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<2, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 3: G <= 4 ? run_pool<3, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<3, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 4: G <= 4 ? run_pool<4, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<4, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 5: G <= 4 ? run_pool<5, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<5, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 6: G <= 4 ? run_pool<6, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<6, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 7: G <= 4 ? run_pool<7, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<7, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
+      case 8: G <= 4 ? run_pool<8, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
+                     : run_pool<8, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
       default: break;
     }
-    // reduce the per-lane partial sums over the 8 token rows (lanes with equal t)
+    // reduce l and zs over the lanes that share a softmax head
+    const int g = lane >> 2, t = lane & 3;
 #pragma unroll
-    for (int c = 0; c < 2; ++c) {
-#pragma unroll
-      for (int off = 4; off <= 16; off <<= 1) {
-        st.l[c] += __shfl_xor_sync(0xffffffffu, st.l[c], off);
-        st.zs[c] += __shfl_xor_sync(0xffffffffu, st.zs[c], off);
-      }
+    for (int off = 1; off <= 2; off <<= 1) {
+      st.l += __shfl_xor_sync(0xffffffffu, st.l, off);
+      st.zs += __shfl_xor_sync(0xffffffffu, st.zs, off);
     }
     __syncthreads();  // every warp is done with the ring: reuse it as the merge area
-    const int g = lane >> 2, t = lane & 3;
-    // logit heads of this lane: 2t+c, or 2(t&1)+c when the lo parts were folded
-    const int hc0 = G <= 4 ? 2 * (t & 1) : 2 * t;
-    if (g == 0 && (G > 4 || t < 2)) {
-#pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        if (hc0 + c < G) {
-          merge_m[warp * 8 + hc0 + c] = st.m[c];
-          merge_l[warp * 8 + hc0 + c] = st.l[c];
-          merge_z[warp * 8 + hc0 + c] = st.zs[c];
-        }
-      }
+    if (t == 0 && g < G) {
+      merge_m[warp * 8 + g] = st.e;
+      merge_l[warp * 8 + g] = st.l;
+      merge_z[warp * 8 + g] = st.zs;
     }
     // O columns are heads 2t, 2t+1 (for G <= 4, columns 4..7 hold the lo parts of
     // heads 0..3; they are written as rows 4..7 and folded in below); rows 16m + g
@@ -1120,7 +1138,7 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kRingBytes);
+                                         kDynBytes);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
@@ -1132,7 +1150,7 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
   }
   dim3 grid(a.plan.splits, a.H, a.B);
-  decode_kernel<<<grid, kThreads, kRingBytes, stream>>>(a);
+  decode_kernel<<<grid, kThreads, kDynBytes, stream>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int heads = a.B * a.Hq;
