@@ -195,7 +195,7 @@ semkv_status semkv_quantize_pack(const semkv_quant_desc* desc, const uint16_t* k
   a.hi_tok = cache->hi_tok;
   a.lo_tok = cache->lo_tok;
   a.err = cache->dev_error;
-  s = from_cuda(launch_quantize_pack(a, device_sm_count(), (cudaStream_t)stream));
+  s = from_cuda(launch_quantize_pack(a, n_high, device_sm_count(), (cudaStream_t)stream));
   if (s != SEMKV_OK) return s;
   cache->hi_count = n_high;
   cache->lo_count = T - (int64_t)n_high;
@@ -256,7 +256,7 @@ semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache
   a.hi_tok = cache->hi_tok;
   a.lo_tok = cache->lo_tok;
   a.err = cache->dev_error;
-  s = from_cuda(launch_quantize_pack(a, device_sm_count(), (cudaStream_t)stream));
+  s = from_cuda(launch_quantize_pack(a, n_high, device_sm_count(), (cudaStream_t)stream));
   if (s != SEMKV_OK) return s;
   cache->hi_count += n_high;
   cache->lo_count += n - (int64_t)n_high;

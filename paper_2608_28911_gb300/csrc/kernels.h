@@ -25,7 +25,9 @@ struct QuantArgs {
   int32_t* lo_tok;
   int32_t* err;
 };
-cudaError_t launch_quantize_pack(const QuantArgs& a, int num_sms, cudaStream_t stream);
+// n_hi: how many of the n tokens go to the high pool (the rest go to the low pool)
+cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
+                                 cudaStream_t stream);
 
 // Top-r selection of each sequence (Eqs. 4-5).
 struct RankArgs {

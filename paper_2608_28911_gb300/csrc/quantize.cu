@@ -235,18 +235,219 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32)
   }
 }
 
+// ------------------------------------------------- affine pools, by slot -----
+// Affine records are built by destination slot: a warp takes units of 8 consecutive
+// slots of one pool of one (sequence, layer, KV head), so the level count is uniform
+// across the warp and the records it writes are contiguous.  Lane 4i + 2r + f handles
+// half f (dims 64f..64f+63, quarters 2f and 2f+1) of row r (0 = K, 1 = V) of the i-th
+// slot's token: 128 contiguous bytes in, two quarter bit fields out.  The same
+// arithmetic as affine_row, and symbols beta = ceil(t 2^W / L^G) as in pack_rows.
+
+constexpr int kAffineSlots = 8;
+
+// 64 fp16 values of one half row (16-byte loads when the source allows)
+__device__ __forceinline__ void load_half(const uint16_t* src, bool vec16, uint32_t (&h)[32]) {
+  if (vec16) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const uint4 u = __ldg(reinterpret_cast<const uint4*>(src) + j);
+      h[4 * j] = u.x; h[4 * j + 1] = u.y; h[4 * j + 2] = u.z; h[4 * j + 3] = u.w;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const uint2 u = __ldg(reinterpret_cast<const uint2*>(src) + j);
+      h[2 * j] = u.x; h[2 * j + 1] = u.y;
+    }
+  }
+}
+
+// OR the value v (n bits, n <= 32) in at bit pos of a 3-word field (pos, n compile-time)
+__device__ __forceinline__ void put_bits(uint32_t (&w)[3], int pos, int n, uint32_t v) {
+  const int wd = pos >> 5, sh = pos & 31;
+  w[wd] |= v << sh;
+  if (sh + n > 32) w[wd + 1] |= v >> (32 - sh);
+}
+
+// The bit field of one quarter from its 32 rounded values: m[j] is the bit pattern of
+// 1.5 * 2^23 + c_j, so sums of L-weighted patterns give the radix value t modulo 2^32
+// once the weighted 1.5 * 2^23 terms are taken off.
+template <int L>
+__device__ __forceinline__ void quarter_field(const uint32_t (&m)[32], uint32_t (&w)[3]) {
+  using F = Fmt<L>;
+  constexpr uint32_t kMagic = 0x4B400000u;
+  w[0] = w[1] = w[2] = 0u;
+#pragma unroll
+  for (int sy = 0; sy < F::NG; ++sy) {
+    uint32_t t = 0, wsum = 0;
+#pragma unroll
+    for (int k = 0; k < F::G; ++k) {
+      t = t * (uint32_t)L + m[sy * F::G + k];
+      wsum = wsum * (uint32_t)L + 1u;
+    }
+    t -= wsum * kMagic;
+    put_bits(w, sy * F::W, F::W, ((t << F::W) + F::LG - 1u) / F::LG);
+  }
+  if constexpr (F::R > 0) {
+    uint32_t t = 0, wsum = 0;
+#pragma unroll
+    for (int k = 0; k < F::R; ++k) {
+      t = t * (uint32_t)L + m[32 - F::R + k];
+      wsum = wsum * (uint32_t)L + 1u;
+    }
+    t -= wsum * kMagic;
+    put_bits(w, F::NG * F::W, F::WT, ((t << F::WT) + F::LR - 1u) / F::LR);
+  }
+}
+
+template <int L>
+__device__ void affine_units(const QuantArgs& a, int b, int l, int h, bool hi, int64_t n_pool,
+                             int64_t u_begin, int64_t u_step, bool vec16, uint32_t* img) {
+  using F = Fmt<L>;
+  constexpr int kRecW = (2 * F::RB + 8) / 4;
+  static_assert(F::QB <= 96, "a quarter fits three words");
+  const int lane = threadIdx.x & 31;
+  const int ti = lane >> 2, row = (lane >> 1) & 1, hf = lane & 1;
+  const int64_t cap = hi ? a.hi_cap : a.lo_cap;
+  const int64_t base = hi ? a.hi_base : a.lo_base;
+  const int64_t bh = ((int64_t)b * a.NL + l) * a.H + h;
+  const int32_t* tokmap = (hi ? a.hi_tok : a.lo_tok) + (int64_t)b * cap + base;
+  const uint16_t* src = (row ? a.v : a.k) + bh * a.Tsrc * kHeadDim + 64 * hf;
+  const int64_t tok_base = a.tok_base;
+  uint32_t* recs = reinterpret_cast<uint32_t*>(hi ? a.hi_pool : a.lo_pool) + (bh * cap + base) * kRecW;
+  const int64_t units = (n_pool + kAffineSlots - 1) / kAffineSlots;
+  for (int64_t u = u_begin; u < units; u += u_step) {
+    const int64_t s0 = u * kAffineSlots;
+    const int nslots = (int)min((int64_t)kAffineSlots, n_pool - s0);
+    const bool active = ti < nslots;
+    for (int i = lane; i < kAffineSlots * kRecW; i += 32) img[i] = 0u;
+    uint32_t hv[32];
+    if (active) {
+      load_half(src + ((int64_t)tokmap[s0 + ti] - tok_base) * kHeadDim, vec16, hv);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) hv[j] = 0u;
+    }
+    // row minimum and maximum: fp16 pairs (exact), then the row's other half
+    __half2 mn2 = *reinterpret_cast<const __half2*>(&hv[0]), mx2 = mn2;
+#pragma unroll
+    for (int j = 1; j < 32; ++j) {
+      const __half2 x2 = *reinterpret_cast<const __half2*>(&hv[j]);
+      mn2 = __hmin2(mn2, x2);
+      mx2 = __hmax2(mx2, x2);
+    }
+    float mn = fminf(__low2float(mn2), __high2float(mn2));
+    float mx = fmaxf(__low2float(mx2), __high2float(mx2));
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, 1));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+    // a zero extreme is taken as +0 (min/max may return either signed zero)
+    if (mn == 0.0f) mn = 0.0f;
+    if (mx == 0.0f) mx = 0.0f;
+    const float s32 = __fdiv_rn(__fsub_rn(mx, mn), (float)(L - 1));
+    const uint16_t s16 = f16_param(s32), z16 = __half_as_ushort(__float2half_rn(mn));
+    const float sc = f16_to_f32(s16), z = f16_to_f32(z16);
+    // 1/s, or 0 when s == 0 (then every value rounds to code 0)
+    const float inv = sc != 0.0f ? __fdiv_rn(1.0f, sc) : 0.0f;
+    __syncwarp();
+#pragma unroll
+    for (int qq = 0; qq < 2; ++qq) {
+      uint32_t m[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const float x = f16_to_f32((uint16_t)(hv[16 * qq + (j >> 1)] >> (16 * (j & 1))));
+        // rint((x - z) / s) clamped to L-1 (the difference is >= 0: z is the row
+        // minimum); adding 1.5 * 2^23 rounds to nearest even
+        const float y = fminf(__fmul_rn(__fsub_rn(x, z), inv), (float)(L - 1));
+        m[j] = __float_as_uint(__fadd_rn(y, 12582912.0f));
+      }
+      uint32_t w[3];
+      quarter_field<L>(m, w);
+      if (active) {
+        uint32_t* r = img + ti * kRecW;
+        const int pos = row * 8 * F::RB + (2 * hf + qq) * F::QB;  // the quarter's first bit
+        const int wd = pos >> 5, sh = pos & 31;
+        atomicOr(&r[wd], w[0] << sh);
+        if (sh + F::QB > 32) atomicOr(&r[wd + 1], __funnelshift_l(w[0], w[1], sh));
+        if (sh + F::QB > 64) atomicOr(&r[wd + 2], __funnelshift_l(w[1], w[2], sh));
+        if (sh + F::QB > 96) atomicOr(&r[wd + 3], __funnelshift_l(w[2], 0u, sh));
+      }
+    }
+    if (active && hf == 0) img[ti * kRecW + (2 * F::RB) / 4 + row] = (uint32_t)s16 | ((uint32_t)z16 << 16);
+    __syncwarp();
+    uint32_t* dst = recs + s0 * kRecW;
+    for (int i = lane; i < nslots * kRecW; i += 32) dst[i] = img[i];
+    __syncwarp();
+  }
+}
+
+// slot -> token maps of the tokens quantized by this call
+__global__ void scatter_tok_kernel(QuantArgs a) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (int64_t)a.B * a.n) return;
+  const int b = (int)(i / a.n), j = (int)(i % a.n);
+  const bool hi = a.is_high[(int64_t)b * a.n + j] != 0;
+  const int64_t s = (hi ? a.hi_base : a.lo_base) + a.slot[(int64_t)b * a.n + j];
+  const int64_t cap = hi ? a.hi_cap : a.lo_cap;
+  if (s >= cap) {  // cannot happen after the host's capacity check
+    raise_error(a.err, kDevCapacity);
+    return;
+  }
+  (hi ? a.hi_tok : a.lo_tok)[(int64_t)b * cap + s] = (int32_t)(a.tok_base + j);
+}
+
+// grid (x, sequence*layer*head, pool): each warp strides over that pool's units
+__global__ void __launch_bounds__(kWarpsPerBlock * 32)
+    quantize_affine_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
+  __shared__ __align__(16) uint32_t img_sm[kWarpsPerBlock][kAffineSlots * kMaxRecWords];
+  const int wib = threadIdx.x >> 5;
+  const bool hi = blockIdx.z == 0;
+  const int64_t n_pool = hi ? n_hi : n_lo;
+  const int64_t u_begin = (int64_t)blockIdx.x * kWarpsPerBlock + wib;
+  const int64_t u_step = (int64_t)gridDim.x * kWarpsPerBlock;
+  const bool vec16 = ((reinterpret_cast<uintptr_t>(a.k) | reinterpret_cast<uintptr_t>(a.v)) & 15u) == 0;
+  uint32_t* img = img_sm[wib];
+  const int bhs = a.B * a.NL * a.H;
+  for (int bhi = blockIdx.y; bhi < bhs; bhi += gridDim.y) {
+    const int h = bhi % a.H, l = (bhi / a.H) % a.NL, b = bhi / (a.H * a.NL);
+    switch (hi ? a.L_hi : a.L_lo) {
+      case 2: affine_units<2>(a, b, l, h, hi, n_pool, u_begin, u_step, vec16, img); break;
+      case 3: affine_units<3>(a, b, l, h, hi, n_pool, u_begin, u_step, vec16, img); break;
+      case 4: affine_units<4>(a, b, l, h, hi, n_pool, u_begin, u_step, vec16, img); break;
+      case 5: affine_units<5>(a, b, l, h, hi, n_pool, u_begin, u_step, vec16, img); break;
+      case 6: affine_units<6>(a, b, l, h, hi, n_pool, u_begin, u_step, vec16, img); break;
+      case 7: affine_units<7>(a, b, l, h, hi, n_pool, u_begin, u_step, vec16, img); break;
+      case 8: affine_units<8>(a, b, l, h, hi, n_pool, u_begin, u_step, vec16, img); break;
+      default: break;
+    }
+  }
+}
+
 }  // namespace
 
-cudaError_t launch_quantize_pack(const QuantArgs& a, int num_sms, cudaStream_t stream) {
+cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
+                                 cudaStream_t stream) {
   const int64_t total = (int64_t)a.B * a.NL * a.H * a.n;
   if (total == 0) return cudaSuccess;
+  if (a.base == SEMKV_BASE_AFFINE) {
+    const int64_t pairs = (int64_t)a.B * a.n;
+    scatter_tok_kernel<<<(unsigned)((pairs + 255) / 256), 256, 0, stream>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    // about 8 units per warp for the larger pool; the (sequence, layer, head) index
+    // runs over grid y (and loops past its limit of 65535)
+    const int64_t bhs = (int64_t)a.B * a.NL * a.H;
+    const int64_t n_max = n_hi > a.n - n_hi ? n_hi : a.n - n_hi;
+    const int64_t units = (n_max + kAffineSlots - 1) / kAffineSlots;
+    int64_t bx = (units + 8 * kWarpsPerBlock - 1) / (8 * kWarpsPerBlock);
+    if (bx < 1) bx = 1;
+    dim3 grid((unsigned)bx, (unsigned)(bhs < 65535 ? bhs : 65535), 2);
+    quantize_affine_kernel<<<grid, kWarpsPerBlock * 32, 0, stream>>>(a, n_hi, a.n - n_hi);
+    return cudaGetLastError();
+  }
   int64_t blocks = (total + kWarpsPerBlock - 1) / kWarpsPerBlock;
   const int64_t cap_blocks = (int64_t)num_sms * 16;  // grid-stride beyond this
   if (blocks > cap_blocks) blocks = cap_blocks;
-  if (a.base == SEMKV_BASE_AFFINE)
-    quantize_pack_kernel<SEMKV_BASE_AFFINE><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
-  else
-    quantize_pack_kernel<SEMKV_BASE_TQ><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+  quantize_pack_kernel<SEMKV_BASE_TQ><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
   return cudaGetLastError();
 }
 
