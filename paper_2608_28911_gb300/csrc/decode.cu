@@ -82,6 +82,17 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       "l"(src), "r"(bytes), "r"(smem_u32(bar))
       : "memory");
 }
+// expect_tx + bulk copy issued by the lanes where `pred` holds (no branch)
+__device__ __forceinline__ void bulk_refill(bool pred, void* dst, const void* src, uint32_t bytes,
+                                            uint64_t* bar) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.u32 p, %0, 0;\n"
+      " @p mbarrier.arrive.expect_tx.shared::cta.b64 _, [%1], %2;\n"
+      " @p cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%3], [%4], %2, [%1];\n}" ::"r"(
+          (uint32_t)pred),
+      "r"(smem_u32(bar)), "r"(bytes), "r"(smem_u32(dst)), "l"(src)
+      : "memory");
+}
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -446,8 +457,12 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
   uint8_t* my_ring = ring + warp * kStages * kStageBytes;
   uint64_t* my_bar = bars + warp * kStages;
 
-  const bool live = g < G;   // head g: A rows g (hi) and g + 8 (lo), softmax of head g
-  const float qmax = sh.qmax[g];
+  // head hd: A rows g (hi) and g + 8 (lo) belong to head g; for G <= 4 lanes g and g + 4
+  // share the softmax of head g & 3
+  const int hd = PACKED ? (g & 3) : g;
+  const bool live = hd < G;
+  const bool upper = PACKED && g >= 4;
+  const float qmax = sh.qmax[hd];
   const float qscale =
       qmax > 0.0f ? pow2_floor(fminf(8192.0f / ((float)(L + 1) * qmax), 1e30f)) : 1.0f;
   // A fragments of the 8 k-steps, {hi 2j, lo 2j, hi 2j+1, lo 2j+1} per lane, kept in
@@ -460,7 +475,7 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
     for (int i = 0; i < 2; ++i) {
       const int p = 2 * j + i;
       float c0 = 0.0f, c1 = 0.0f;
-      if (live) {
+      if (live && !upper) {
         c0 = k_coef<L>(sh.q[g], t, p, 0) * qscale;
         c1 = k_coef<L>(sh.q[g], t, p, 1) * qscale;
       }
@@ -470,7 +485,7 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
   }
   __syncwarp();
   const float cS = a.scale_log2 / qscale;   // logit weight of s_k * S
-  const float cZ = a.scale_log2 * sh.sumq[g];  // logit weight of z_k
+  const float cZ = a.scale_log2 * sh.sumq[hd];  // logit weight of z_k
   // O columns 2t, 2t+1 belong to these heads (their e lives in lane 4*head)
   const int oh0 = PACKED ? ((2 * t) & 3) : 2 * t, oh1 = oh0 + 1;
 
@@ -513,18 +528,38 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
         mma16816(s1, A.x, A.y, A.z, A.w, f1[j][0], f1[j][1]);
       }
     }
-    // ---- logits of head g for tokens 2t, 2t+1, 2t+8, 2t+9 (hi + lo rows)
-    const float S[4] = {s0[0] + s0[2], s0[1] + s0[3], s1[0] + s1[2], s1[1] + s1[3]};
-    float lg[4], sv[4], zv[4], p[4], P[4];
-    bool valid[4];
+    // ---- logits of head hd (hi + lo rows).  G > 4: lane (g, t) takes tokens 2t, 2t+1,
+    // 2t+8, 2t+9 of head g.  G <= 4 (rows 4..7 empty): lane g < 4 keeps tokens 2t, 2t+1
+    // and hands 2t+8, 2t+9 to lane g + 4, which works for the same head.
+    constexpr int NT = PACKED ? 2 : 4;
+    float S[NT];
+    int tk[NT];
+    if constexpr (PACKED) {
+      const float r0 = __shfl_xor_sync(0xffffffffu, s1[0] + s1[2], 16);
+      const float r1 = __shfl_xor_sync(0xffffffffu, s1[1] + s1[3], 16);
+      S[0] = upper ? r0 : s0[0] + s0[2];
+      S[1] = upper ? r1 : s0[1] + s0[3];
+      tk[0] = 2 * t + (upper ? 8 : 0);
+      tk[1] = tk[0] + 1;
+    } else {
+      S[0] = s0[0] + s0[2];
+      S[1] = s0[1] + s0[3];
+      S[2] = s1[0] + s1[2];
+      S[3] = s1[1] + s1[3];
+      tk[0] = 2 * t;
+      tk[1] = 2 * t + 1;
+      tk[2] = 2 * t + 8;
+      tk[3] = 2 * t + 9;
+    }
+    float lg[NT], sv[NT], zv[NT], p[NT], P[NT];
+    bool valid[NT];
     bool bad = false;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int tok = 2 * t + (i & 1) + 8 * (i >> 1);
-      const uint32_t* prm = reinterpret_cast<const uint32_t*>(tb + tok * kRec + 2 * F::RB);
+    for (int i = 0; i < NT; ++i) {
+      const uint32_t* prm = reinterpret_cast<const uint32_t*>(tb + tk[i] * kRec + 2 * F::RB);
       const uint32_t kp = prm[0], vp = prm[1];
       const float sk = f16_to_f32((uint16_t)(kp & 0xFFFF)), zk = f16_to_f32((uint16_t)(kp >> 16));
-      valid[i] = live && tok < nvalid;
+      valid[i] = live && tk[i] < nvalid;
       // rows past the pool's count are not data: keep whatever they hold out of the sums
       sv[i] = valid[i] ? f16_to_f32((uint16_t)(vp & 0xFFFF)) : 0.0f;
       zv[i] = valid[i] ? f16_to_f32((uint16_t)(vp >> 16)) : 0.0f;
@@ -537,10 +572,11 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
       // move e up to (max over the head's tokens of logit + log2 max(s_v, 1)) - 12
       float mx = -INFINITY;
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+      for (int i = 0; i < NT; ++i)
         if (valid[i]) mx = fmaxf(mx, lg[i] + fmaxf(0.0f, __log2f(sv[i])));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      if (PACKED) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
       const float e_new = fmaxf(st.e, mx - 12.0f);
       const float al = st.e == -INFINITY ? 0.0f : ex2(st.e - e_new);
       st.e = e_new;
@@ -556,28 +592,28 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
         st.O[m][3] *= a1;
       }
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
+      for (int i = 0; i < NT; ++i) {
         p[i] = valid[i] ? ex2(lg[i] - st.e) : 0.0f;
         P[i] = p[i] * sv[i];
       }
     }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < NT; ++i) {
       st.l += p[i];
       st.zs = fmaf(p[i], zv[i], st.zs);
     }
     // ---- P'^T as the B fragment: rows = tokens (2t, 2t+1 | 2t+8, 2t+9), column g
-    uint32_t b0, b1, b0l, b1l;
-    split_h2(P[0], P[1], b0, b0l);
-    split_h2(P[2], P[3], b1, b1l);
+    uint32_t b0, b1, b0l = 0u, b1l = 0u;
     if constexpr (PACKED) {
-      // columns 4..7 carry the lo parts of heads 0..3, computed by lanes g - 4
-      const uint32_t r0 = __shfl_xor_sync(0xffffffffu, b0l, 16);
-      const uint32_t r1 = __shfl_xor_sync(0xffffffffu, b1l, 16);
-      if (g >= 4) {
-        b0 = r0;
-        b1 = r1;
-      }
+      // column g < 4: hi parts of head g; column g + 4: lo parts of head g
+      uint32_t hi, lo;
+      split_h2(P[0], P[1], hi, lo);
+      const uint32_t recv = __shfl_xor_sync(0xffffffffu, upper ? hi : lo, 16);
+      b0 = upper ? recv : hi;
+      b1 = upper ? lo : recv;
+    } else {
+      split_h2(P[0], P[1], b0, b0l);
+      split_h2(P[2], P[3], b1, b1l);
     }
     // ---- O^T += C^T P'^T
     {
@@ -594,12 +630,12 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
       }
     }
     __syncwarp();
-    if (lane == 0 && it + kStages < nmine) {
+    {
+      // the stage is free again: lane 0 starts the copy of the tile kStages ahead
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       const int nt = t_begin + warp + (it + kStages) * kWarps;
-      mbar_expect_tx(&my_bar[stage], kTileBytes);
-      bulk_g2s(my_ring + stage * kStageBytes, pool_bh + (int64_t)nt * kTileBytes, kTileBytes,
-               &my_bar[stage]);
+      bulk_refill(lane == 0 && it + kStages < nmine, my_ring + stage * kStageBytes,
+                  pool_bh + (int64_t)nt * kTileBytes, kTileBytes, &my_bar[stage]);
     }
   }
   if (!ok) {
@@ -940,7 +976,8 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
     // reduce l and zs over the lanes that share a softmax head
     const int g = lane >> 2, t = lane & 3;
 #pragma unroll
-    for (int off = 1; off <= 2; off <<= 1) {
+    for (int off = 1; off <= 16; off <<= 1) {
+      if (off == 4 || off == 8 || (off == 16 && G > 4)) continue;
       st.l += __shfl_xor_sync(0xffffffffu, st.l, off);
       st.zs += __shfl_xor_sync(0xffffffffu, st.zs, off);
     }
