@@ -135,8 +135,11 @@ semkv_status semkv_lloyd_max_gaussian(int32_t levels, float* centroids, float* t
  *   rank[b][i]    = position of i in the (score desc, index asc) order, 0-based
  *                   (u32 [batch][T]; may be NULL).
  * scores: device f32 [batch][T].  ws/ws_bytes: device workspace of at least
- * semkv_rank_workspace_bytes(batch, T) bytes (may be NULL when that is 0).
- * Requires n_high <= T, 1 <= T <= 2^24. */
+ * semkv_rank_workspace_bytes(batch, T, rank != NULL) bytes, 4-byte aligned, owned by
+ * the caller: 16 * batch * T bytes when ranks are wanted (keys and indices of a
+ * stable radix sort, double-buffered), else 0 and ws may be NULL.
+ * Errors: SEMKV_EINVAL (null pointers, T outside 1..2^24, n_high > T),
+ * SEMKV_EWORKSPACE (rank set and ws missing or too small), SEMKV_EALIGN. */
 size_t semkv_rank_workspace_bytes(int32_t batch, int32_t T, int32_t want_rank);
 semkv_status semkv_rank_assign(const float* scores, int32_t batch, int32_t T,
                                uint32_t n_high, uint8_t* is_high, uint32_t* slot,

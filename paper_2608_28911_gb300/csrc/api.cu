@@ -131,21 +131,22 @@ semkv_status semkv_lloyd_max_gaussian(int32_t levels, float* centroids, float* t
 }
 
 size_t semkv_rank_workspace_bytes(int32_t batch, int32_t T, int32_t want_rank) {
-  (void)batch;
-  (void)T;
-  (void)want_rank;
-  return 0;
+  if (!want_rank || batch < 1 || T < 1) return 0;
+  return rank_workspace_words(batch, T) * sizeof(uint32_t);
 }
 
 semkv_status semkv_rank_assign(const float* scores, int32_t batch, int32_t T, uint32_t n_high,
                                uint8_t* is_high, uint32_t* slot, uint32_t* rank, void* ws,
                                size_t ws_bytes, void* stream) {
-  (void)ws;
-  (void)ws_bytes;
   if (!scores || !is_high || !slot || batch < 0 || T < 1 || T > (1 << 24)) return SEMKV_EINVAL;
   if (n_high > (uint32_t)T) return SEMKV_EINVAL;
-  if (rank) return SEMKV_EUNSUPPORTED;  // full ranks are not produced by this version
+  if (rank) {
+    if (!ws || ws_bytes < semkv_rank_workspace_bytes(batch, T, 1)) return SEMKV_EWORKSPACE;
+    if (!aligned(ws, 4)) return SEMKV_EALIGN;
+  }
   RankArgs a;
+  a.rank = rank;
+  a.ws = static_cast<uint32_t*>(ws);
   a.scores = scores;
   a.B = batch;
   a.T = T;
@@ -228,6 +229,8 @@ semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache
   r.n_high = n_high;
   r.is_high = cache->blk_is_high;
   r.slot = cache->blk_slot;
+  r.rank = nullptr;
+  r.ws = nullptr;
   s = from_cuda(launch_rank_assign(r, (cudaStream_t)stream));
   if (s != SEMKV_OK) return s;
   QuantArgs a;

@@ -37,7 +37,10 @@ struct RankArgs {
   uint32_t n_high;
   uint8_t* is_high;         // [B][T]
   uint32_t* slot;           // [B][T]
+  uint32_t* rank;           // [B][T] or null
+  uint32_t* ws;             // rank_workspace_words(B, T) words when rank is set
 };
+size_t rank_workspace_words(int B, int T);
 cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream);
 
 // Decode attention over one layer of the cache (split-K + combine).

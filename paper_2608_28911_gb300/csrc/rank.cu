@@ -151,11 +151,113 @@ __global__ void __launch_bounds__(kThreads) rank_assign_kernel(RankArgs a) {
   }
 }
 
+// ---- full ranks (optional output): a stable LSD radix sort of the inverted keys
+// (ascending inverted key = descending score; a stable pass keeps equal keys in index
+// order, which is the tie rule), 4-bit digits in 8 passes, one CTA per sequence,
+// 1024 keys per step.  Within a step a key's place among the equal digits before it
+// comes from match_any inside its warp plus a scan of the per-warp digit counts.
+// Then rank[index at sorted position p] = p.  Workspace per sequence: keys and
+// indices, double-buffered (4 T words).
+constexpr int kSortBins = 16;
+
+__global__ void __launch_bounds__(kThreads) rank_sort_kernel(RankArgs a, uint32_t* ws) {
+  __shared__ uint32_t wcount[32][kSortBins];  // per-warp digit counts, then offsets
+  __shared__ uint32_t base[kSortBins];        // first output position of each digit
+  __shared__ uint32_t total[kSortBins];
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t T = (uint32_t)a.T;
+  const float* s = a.scores + (int64_t)b * a.ld;
+  uint32_t* kb[2] = {ws + (size_t)b * 4 * T, ws + (size_t)b * 4 * T + 2 * (size_t)T};
+  uint32_t* ib[2] = {kb[0] + T, kb[1] + T};
+  for (uint32_t i = tid; i < T; i += kThreads) {
+    kb[0][i] = ~order_key(s[i]);
+    ib[0][i] = i;
+  }
+  __syncthreads();
+  const uint32_t lt_mask = (1u << lane) - 1u;
+  for (int pass = 0; pass < 8; ++pass) {
+    const int sh = 4 * pass;
+    const uint32_t* ksrc = kb[pass & 1];
+    const uint32_t* isrc = ib[pass & 1];
+    uint32_t* kdst = kb[(pass + 1) & 1];
+    uint32_t* idst = ib[(pass + 1) & 1];
+    // digit histogram of the whole sequence -> first position of each digit
+    if (tid < kSortBins) total[tid] = 0;
+    __syncthreads();
+    for (uint32_t i0 = 0; i0 < T; i0 += kThreads) {
+      const uint32_t i = i0 + tid;
+      const bool ok = i < T;
+      const uint32_t d = ok ? (ksrc[i] >> sh) & (kSortBins - 1) : 0u;
+      const uint32_t act = __ballot_sync(0xffffffffu, ok);
+      if (ok) {
+        const uint32_t peers = __match_any_sync(act, d);
+        if ((peers & lt_mask) == 0) atomicAdd(&total[d], (uint32_t)__popc(peers));
+      }
+    }
+    __syncthreads();
+    if (tid == 0) {
+      uint32_t run = 0;
+      for (int d = 0; d < kSortBins; ++d) {
+        base[d] = run;
+        run += total[d];
+      }
+    }
+    __syncthreads();
+    // stable scatter, 1024 keys at a time in index order
+    for (uint32_t i0 = 0; i0 < T; i0 += kThreads) {
+      const uint32_t i = i0 + tid;
+      const bool ok = i < T;
+      uint32_t key = 0, idx = 0, d = 0;
+      if (ok) {
+        key = ksrc[i];
+        idx = isrc[i];
+        d = (key >> sh) & (kSortBins - 1);
+      }
+      if (lane < kSortBins) wcount[warp][lane] = 0;
+      __syncwarp();
+      const uint32_t act = __ballot_sync(0xffffffffu, ok);
+      uint32_t before = 0;
+      if (ok) {
+        const uint32_t peers = __match_any_sync(act, d);
+        before = __popc(peers & lt_mask);
+        if (before == 0) wcount[warp][d] = (uint32_t)__popc(peers);
+      }
+      __syncthreads();
+      if (tid < kSortBins) {  // exclusive scan over the warps, per digit
+        uint32_t run = 0;
+        for (int w = 0; w < 32; ++w) {
+          const uint32_t c = wcount[w][tid];
+          wcount[w][tid] = run;
+          run += c;
+        }
+        total[tid] = run;
+      }
+      __syncthreads();
+      if (ok) {
+        const uint32_t pos = base[d] + wcount[warp][d] + before;
+        kdst[pos] = key;
+        idst[pos] = idx;
+      }
+      __syncthreads();
+      if (tid < kSortBins) base[tid] += total[tid];
+      __syncthreads();
+    }
+  }
+  // after an even number of passes the sorted order is back in buffer 0
+  uint32_t* rank = a.rank + (int64_t)b * a.T;
+  for (uint32_t p = tid; p < T; p += kThreads) rank[ib[0][p]] = p;
+}
+
 }  // namespace
+
+size_t rank_workspace_words(int B, int T) { return (size_t)B * 4 * (size_t)T; }
 
 cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream) {
   if (a.B == 0 || a.T == 0) return cudaSuccess;
   rank_assign_kernel<<<a.B, kThreads, 0, stream>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || !a.rank) return e;
+  rank_sort_kernel<<<a.B, kThreads, 0, stream>>>(a, a.ws);
   return cudaGetLastError();
 }
 

@@ -147,6 +147,10 @@ def semkv_lloyd_max_gaussian(levels: int):
             torch.tensor(list(t)[:levels - 1], dtype=torch.float32))
 
 
+def semkv_rank_workspace_bytes(batch: int, T: int, want_rank: bool = True) -> int:
+    return LIB.semkv_rank_workspace_bytes(batch, T, 1 if want_rank else 0)
+
+
 def semkv_rank_assign(scores: torch.Tensor, n_high: int, is_high: torch.Tensor,
                       slot: torch.Tensor, rank=None, ws=None, stream=None):
     B, T = scores.shape

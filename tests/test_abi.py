@@ -71,3 +71,19 @@ def test_argument_validation_returns_status(lib):
     assert lib.semkv_decode_attention(None, None, 0, None, None, 1.0, None, 0, None) == 1
     lib.semkv_status_string.restype = ctypes.c_char_p
     assert lib.semkv_status_string(3) == b"pool or staging capacity exceeded"
+
+
+def test_rank_workspace_sizing_and_checks(lib):
+    p = ctypes.c_void_p
+    lib.semkv_rank_workspace_bytes.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]
+    lib.semkv_rank_workspace_bytes.restype = ctypes.c_size_t
+    assert lib.semkv_rank_workspace_bytes(2, 100, 1) == 2 * 4 * 100 * 4
+    assert lib.semkv_rank_workspace_bytes(2, 100, 0) == 0
+    lib.semkv_rank_assign.argtypes = [p, ctypes.c_int32, ctypes.c_int32, ctypes.c_uint32, p, p, p,
+                                      p, ctypes.c_size_t, p]
+    fake = 4096  # never dereferenced: every call below fails validation before a launch
+    # ranks wanted without (enough) workspace -> SEMKV_EWORKSPACE
+    assert lib.semkv_rank_assign(fake, 2, 100, 3, fake, fake, fake, None, 0, None) == 6
+    assert lib.semkv_rank_assign(fake, 2, 100, 3, fake, fake, fake, fake, 3199, None) == 6
+    # misaligned workspace -> SEMKV_EALIGN
+    assert lib.semkv_rank_assign(fake, 2, 100, 3, fake, fake, fake, fake + 2, 3200, None) == 2

@@ -37,10 +37,13 @@ def test_rank_assign_bit_exact(T):
     for n_high in sorted({0, 1, T // 4, max(T - 1, 0), T}):
         ih = torch.empty((B, T), dtype=torch.uint8, device=d)
         sl = torch.empty((B, T), dtype=torch.int32, device=d)
-        semkv.semkv_rank_assign(st, n_high, ih, sl)
-        o_ih, o_sl, _ = oracle.rank_assign(s, n_high)
+        rk = torch.empty((B, T), dtype=torch.int32, device=d)
+        ws = torch.empty(semkv.semkv_rank_workspace_bytes(B, T) // 4, dtype=torch.int32, device=d)
+        semkv.semkv_rank_assign(st, n_high, ih, sl, rank=rk, ws=ws)
+        o_ih, o_sl, o_rk = oracle.rank_assign(s, n_high)
         assert np.array_equal(ih.cpu().numpy(), o_ih), n_high
         assert np.array_equal(sl.cpu().numpy().view(np.uint32), o_sl), n_high
+        assert np.array_equal(rk.cpu().numpy().view(np.uint32), o_rk), n_high
 
 
 # -------------------------------------------------------------- quantize -----
