@@ -79,6 +79,23 @@ def profiled_traffic(config_name: str):
     return int(m.group(1))
 
 
+def max_over_ranks(values, device=None):
+    """Each value's maximum over the ranks of the default process group (the values
+    themselves in a single process): the job is as slow as its slowest replica."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t.cpu()]
+
+
+def job_gbs(bytes_per_rank: float, world: int, seconds: float) -> float:
+    """Whole-job throughput: every replica moves bytes_per_rank in `seconds`."""
+    return bytes_per_rank * world / seconds / 1e9
+
+
 def load_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -306,11 +323,7 @@ def gpu_arm(args, cfg, rank, world):
     barrier()
     e2e_time = e0.elapsed_time(e1) * 1e-3 / e2e_steps
 
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([elapsed, e2e_time], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed, e2e_time = float(t[0]), float(t[1])
+    elapsed, e2e_time = max_over_ranks([elapsed, e2e_time], device=dev)
     return dict(elapsed=elapsed, dec_times=dec_times, dec_bytes=dec_bytes, app_bytes=app_bytes,
                 quantize_gbs=quantize_gbs, clocks=clk.summary(), err=err, e2e_time=e2e_time,
                 h2d=h2d, d2h=d2h)
@@ -417,12 +430,12 @@ def main():
     if rank != 0:
         return
     step_s = r["elapsed"] / args.steps
-    total_bytes = (r["dec_bytes"] + r["app_bytes"]) * world
+    step_bytes = r["dec_bytes"] + r["app_bytes"]
     dec_mean = sum(r["dec_times"]) / len(r["dec_times"])
     achieved = r["dec_bytes"] / dec_mean / 1e9
     peak = peaks["hbm_gbs"]
     line = {
-        "metric": METRIC, "value": total_bytes / step_s / 1e9, "unit": "GB/s",
+        "metric": METRIC, "value": job_gbs(step_bytes, world, step_s), "unit": "GB/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f16 codes x f16 -> f32 (mma), f32 softmax",
@@ -436,7 +449,7 @@ def main():
                      "frac": achieved / peak, "traffic": profiled_traffic(args.config),
                      "kernel": "decode_kernel+combine_kernel (semkv_decode_attention)",
                      "peak_kind": f"{peak_kind} hbm_gbs"},
-        "e2e": {"value": total_bytes / r["e2e_time"] / 1e9, "unit": "GB/s",
+        "e2e": {"value": job_gbs(step_bytes, world, r["e2e_time"]), "unit": "GB/s",
                 "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
         "gpu_launches": 4 * args.steps,
         "clocks": r["clocks"],

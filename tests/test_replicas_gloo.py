@@ -1,0 +1,66 @@
+"""The multi-GPU path of the benchmark is replicas only: every rank runs the whole
+step on its own GPU and no data crosses ranks.  What crosses ranks is the timing:
+the job takes as long as its slowest replica.  These tests run that host logic as
+two gloo ranks on the CPU, and check the reference arm's rank handling."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+
+def _rank_main(rank, world, port, out_dir):
+    import torch.distributed as dist
+    import bench
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    mine = [1.0 + rank, 10.0 - rank]          # rank 1 is slower on the first value
+    got = bench.max_over_ranks(mine)
+    with open(os.path.join(out_dir, f"r{rank}.json"), "w") as f:
+        json.dump(got, f)
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_timing_is_max_over_two_gloo_ranks(tmp_path):
+    import socket
+    import torch.multiprocessing as mp
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    mp.start_processes(_rank_main, args=(2, port, str(tmp_path)), nprocs=2, join=True,
+                       start_method="spawn")
+    for r in range(2):
+        with open(tmp_path / f"r{r}.json") as f:
+            assert json.load(f) == [2.0, 10.0]
+
+
+def test_single_process_timing_and_job_throughput():
+    import bench
+    assert bench.max_over_ranks([3.5, 4.0]) == [3.5, 4.0]
+    # two replicas moving 1 GB each in 0.5 s: 4 GB/s for the job
+    assert bench.job_gbs(1e9, 2, 0.5) == pytest.approx(4.0)
+
+
+def test_reference_arm_runs_on_rank_zero_only():
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--gpus", "2", "--steps", "1", "--warmup", "3"],
+                       capture_output=True, text=True, env=env, timeout=120)
+    assert r.returncode == 0 and r.stdout.strip() == ""
+
+
+def test_reference_arm_line_on_rank_zero():
+    env = dict(os.environ, RANK="0", WORLD_SIZE="1")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--config", "b1x32k", "--steps", "1", "--warmup", "3"],
+                       capture_output=True, text=True, env=env, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["unit"] == "GB/s" and line["value"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
