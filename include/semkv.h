@@ -94,7 +94,8 @@ typedef struct {
   int32_t block;               /* B of Algorithm 2 (1..1024)                       */
   uint8_t* hi_pool;            /* device [batch][layers][kv_heads][hi_cap][rec_hi], 16-B aligned */
   uint8_t* lo_pool;            /* device [batch][layers][kv_heads][lo_cap][rec_lo], 16-B aligned */
-  int64_t hi_cap, lo_cap;      /* slots per (b, layer, head); multiples of 16      */
+  int64_t hi_cap, lo_cap;      /* slots per (b, layer, head); multiples of 16, at
+                                  most 2^30 (else SEMKV_EUNSUPPORTED)               */
   int32_t* hi_tok;             /* device [batch][hi_cap]: token index of each slot */
   int32_t* lo_tok;             /* device [batch][lo_cap]                            */
   int64_t hi_count, lo_count;  /* (lib) slots in use, same for every sequence      */

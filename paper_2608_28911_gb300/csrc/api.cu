@@ -39,6 +39,8 @@ semkv_status check_cache(const semkv_cache* c) {
   if (!c->hi_pool || !c->lo_pool || !c->hi_tok || !c->lo_tok) return SEMKV_EINVAL;
   if (!aligned(c->hi_pool, 16) || !aligned(c->lo_pool, 16)) return SEMKV_EALIGN;
   if (c->hi_cap < 0 || c->lo_cap < 0 || c->hi_cap % 16 || c->lo_cap % 16) return SEMKV_EALIGN;
+  // slot indices are 32-bit inside the kernels
+  if (c->hi_cap > (int64_t)1 << 30 || c->lo_cap > (int64_t)1 << 30) return SEMKV_EUNSUPPORTED;
   if (c->hi_count < 0 || c->lo_count < 0 || c->hi_count > c->hi_cap || c->lo_count > c->lo_cap)
     return SEMKV_EINVAL;
   if (c->stage_n < 0 || c->stage_n > c->block) return SEMKV_EINVAL;
@@ -321,7 +323,8 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
   // rotated queries (TQ base) after the split-K partials in the workspace
   a.qrot = a.partials + (decode_workspace_floats(a.B, a.H, a.Hq) - (size_t)a.B * a.Hq * 128);
   a.err = cache->dev_error;
-  a.plan = make_decode_plan(a.B, a.H, a.hi_count, a.lo_count, a.stage_n, sms);
+  a.plan = make_decode_plan(a.base, a.L_hi, a.L_lo, a.B, a.H, a.hi_count, a.lo_count, a.stage_n,
+                            sms, kMaxPartialsPerPair);
   return from_cuda(launch_decode_attention(a, (cudaStream_t)stream));
 }
 

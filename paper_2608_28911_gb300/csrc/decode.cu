@@ -39,6 +39,8 @@
 // mbarriers (bounded waits that report a timeout in the error word).
 #include <float.h>
 
+#include <cstring>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -53,8 +55,9 @@ constexpr int kTile = 16;
 constexpr int kMaxRec = 104;
 constexpr int kStageBytes = kTile * kMaxRec + 16;  // +16: window loads may run 12 B past a tile
 constexpr int kRingBytes = kWarps * kStages * kStageBytes;
-constexpr int kAqBytes = kWarps * 8 * 32 * 16;       // per warp: 8 k-steps x 32 lanes x uint4
-constexpr int kDynBytes = kRingBytes + kAqBytes;
+constexpr int kAqBytes = 8 * 32 * 16;   // q-coefficient A fragments: 8 k-steps x 32 lanes x uint4
+constexpr int kCtasAffine = 2;          // resident CTAs per SM: affine pools / other sources
+constexpr int kCtasOther = 2;
 constexpr int kMaxSplits = 64;                     // pool splits per (b, h)
 constexpr uint32_t kSpinLimit = 1u << 22;
 
@@ -444,9 +447,11 @@ struct Shared {
 // Codes enter as exact fp16 integers; the partners' power-of-two scales keep every
 // operand within the fp16 range.
 template <int L, bool PACKED>
+// ring_it: tiles this warp has already taken through its ring (kept across calls so
+// the stage and barrier phase of each tile continue from the previous call)
 __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint4* aq_all,
                          uint64_t* bars, const uint8_t* pool_bh, int64_t count, int t_begin,
-                         int t_end, int G, WarpState& st) {
+                         int t_end, int G, WarpState& st, int& ring_it) {
   using D = Dec<L>;
   using F = typename D::F;
   constexpr int kRec = 2 * F::RB + 8;
@@ -465,11 +470,13 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
   const float qmax = sh.qmax[hd];
   const float qscale =
       qmax > 0.0f ? pow2_floor(fminf(8192.0f / ((float)(L + 1) * qmax), 1e30f)) : 1.0f;
-  // A fragments of the 8 k-steps, {hi 2j, lo 2j, hi 2j+1, lo 2j+1} per lane, kept in
-  // this warp's slice of shared memory (one conflict-free 16-byte load per k-step)
-  uint4* aq = aq_all + warp * 8 * 32 + lane;
+  // A fragments of the 8 k-steps, {hi 2j, lo 2j, hi 2j+1, lo 2j+1} per lane, the same
+  // for every warp of the CTA: warp 0 stores them in shared memory, every warp loads
+  // its lane's fragment (one conflict-free 16-byte load per k-step)
+  uint4* aq = aq_all + lane;
+  __syncthreads();  // the previous pool's fragments and the merge area are no longer read
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
+  for (int j = 0; j < 8 && warp == 0; ++j) {
     uint32_t r[4];
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
@@ -483,7 +490,7 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
     }
     aq[32 * j] = make_uint4(r[0], r[1], r[2], r[3]);
   }
-  __syncwarp();
+  __syncthreads();  // every warp of the CTA runs this pool with the same level count
   const float cS = a.scale_log2 / qscale;   // logit weight of s_k * S
   const float cZ = a.scale_log2 * sh.sumq[hd];  // logit weight of z_k
   // O columns 2t, 2t+1 belong to these heads (their e lives in lane 4*head)
@@ -494,26 +501,31 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
   const int tpos = F::NG * F::W - hh * D::kHalf * F::W;           // tail, relative
 
   const int nmine = t_end - t_begin <= warp ? 0 : (t_end - t_begin - warp + kWarps - 1) / kWarps;
+  const int count32 = (int)count;  // a pool holds fewer than 2^31 slots
   if (lane == 0) {
+    // the ring may have been the merge area: order those writes before the copies
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     for (int i = 0; i < kStages && i < nmine; ++i) {
       const int tile = t_begin + warp + i * kWarps;
-      mbar_expect_tx(&my_bar[i], kTileBytes);
-      bulk_g2s(my_ring + i * kStageBytes, pool_bh + (int64_t)tile * kTileBytes, kTileBytes,
-               &my_bar[i]);
+      const int sl = (ring_it + i) % kStages;
+      mbar_expect_tx(&my_bar[sl], kTileBytes);
+      bulk_g2s(my_ring + sl * kStageBytes, pool_bh + (int64_t)tile * kTileBytes, kTileBytes,
+               &my_bar[sl]);
     }
   }
   __syncwarp();
   bool ok = true;
   int it = 0;
   for (; it < nmine; ++it) {
-    const int stage = it % kStages;
-    if (!mbar_wait(&my_bar[stage], (uint32_t)((it / kStages) & 1))) {
+    const int gi = ring_it + it;
+    const int stage = gi % kStages;
+    if (!mbar_wait(&my_bar[stage], (uint32_t)((gi / kStages) & 1))) {
       ok = false;
       break;
     }
     const int tile = t_begin + warp + it * kWarps;
     const uint8_t* tb = my_ring + stage * kStageBytes;
-    const int nvalid = (int)min((int64_t)kTile, count - (int64_t)tile * kTile);
+    const int nvalid = min(kTile, count32 - tile * kTile);
 
     // ---- S = Q' F^T, tokens 0..7 and 8..15
     float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
@@ -643,9 +655,10 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
     // chance to land, and drop this warp's contribution
     if (lane == 0) raise_error(a.err, kDevWaitTimeout);
     for (int j = it; j < nmine && j < it + kStages; ++j)
-      mbar_wait(&my_bar[j % kStages], (uint32_t)((j / kStages) & 1));
+      mbar_wait(&my_bar[(ring_it + j) % kStages], (uint32_t)(((ring_it + j) / kStages) & 1));
     state_init(st);
   }
+  ring_it += nmine;
 }
 
 // ------------------------------------------------- TurboQuant-MSE records -----
@@ -864,180 +877,129 @@ __device__ void run_stage(const DecodeArgs& a, const Shared& sh, int b, int h, i
 
 // -------------------------------------------------------------- kernel --------
 
-__global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
-  extern __shared__ __align__(128) uint8_t dyn[];
-  __shared__ Shared sh;
-  __shared__ float merge_m[kWarps * 8], merge_l[kWarps * 8], merge_z[kWarps * 8];
-  __shared__ float cta_scale[kWarps * 8], cta_z[8];
-  uint8_t* ring = dyn;
-  uint4* aq_all = reinterpret_cast<uint4*>(dyn + kRingBytes);
-  float* merge_o = reinterpret_cast<float*>(dyn);  // [kWarps][8][128] output rows
+// balanced plan: the partial slots of pair bh's hi and lo segments
+__host__ __device__ inline int seg_slots(const DecodePlan& P, int64_t s, int64_t e) {
+  return e > s ? (int)((e - 1) / P.per - s / P.per + 1) : 0;
+}
+__host__ __device__ inline void pair_slots(const DecodePlan& P, int64_t bh, int& n_hi, int& n_lo) {
+  const int64_t s = bh * P.W, m = s + (int64_t)P.w_hi * P.tiles_hi, e = s + P.W;
+  n_hi = seg_slots(P, s, m);
+  n_lo = seg_slots(P, m, e);
+}
+// partial slots used by pair bh (pools, then the stage)
+__host__ __device__ inline int pair_partials(const DecodePlan& P, int64_t bh) {
+  if (!P.balanced) return P.splits;
+  int n_hi, n_lo;
+  pair_slots(P, bh, n_hi, n_lo);
+  return n_hi + n_lo + P.splits_st;
+}
 
-  const int b = blockIdx.z, h = blockIdx.y, split = blockIdx.x;
-  const int G = a.Hq / a.H;
+struct MergeArea {
+  float m[kWarps * 8], l[kWarps * 8], z[kWarps * 8];
+  float scale[kWarps * 8], cta_z[8];
+};
+
+// the group's queries of pair (b, h) into shared memory, with their sums and maxima
+// (every thread of the CTA calls this; the caller orders it after earlier readers)
+__device__ void load_group_q(const DecodeArgs& a, Shared& sh, int b, int h, int G) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const DecodePlan& P = a.plan;
-
   for (int i = threadIdx.x; i < 8 * 128; i += kThreads) {
     const int c = i >> 7, d = i & 127;
     sh.q[c][d] = c < G ? a.q[((int64_t)b * a.Hq + h * G + c) * 128 + d] : (uint16_t)0;
   }
-  if (a.base == SEMKV_BASE_TQ) {
-    for (int i = threadIdx.x; i < 8 * 128; i += kThreads) {
-      const int c = i >> 7, d = i & 127;
-      sh.qr[c][d] = c < G ? a.qrot[((int64_t)b * a.Hq + h * G + c) * 128 + d] : 0.0f;
-    }
-    if (threadIdx.x < 16) {
-      const int which = threadIdx.x >> 3, k = threadIdx.x & 7;
-      const int L = which == 0 ? a.L_hi : a.L_lo;
-      sh.cb[which][k] = k < L ? (which == 0 ? a.cb_hi : a.cb_lo)[k] : 0.0f;
-    }
-  }
-  if (threadIdx.x < kWarps * kStages) mbar_init(&sh.bar[0][0] + threadIdx.x);
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncthreads();
-  {
-    // per head: sum of q (the zero-point weight) and max |q| (the coefficient scale)
-    static_assert(kWarps == 8, "one warp per head slot");
-    float s = 0.0f, mx = 0.0f;
+  // per head: sum of q (the zero-point weight) and max |q| (the coefficient scale)
+  static_assert(kWarps == 8, "one warp per head slot");
+  float s = 0.0f, mx = 0.0f;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float x = f16_to_f32(sh.q[warp][4 * lane + j]);
-      s += x;
-      mx = fmaxf(mx, fabsf(x));
-    }
+  for (int j = 0; j < 4; ++j) {
+    const float x = f16_to_f32(sh.q[warp][4 * lane + j]);
+    s += x;
+    mx = fmaxf(mx, fabsf(x));
+  }
 #pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) {
-      s += __shfl_xor_sync(0xffffffffu, s, off);
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    }
-    if (lane == 0) {
-      sh.sumq[warp] = s;
-      sh.qmax[warp] = mx;
-    }
+  for (int off = 16; off >= 1; off >>= 1) {
+    s += __shfl_xor_sync(0xffffffffu, s, off);
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  }
+  if (lane == 0) {
+    sh.sumq[warp] = s;
+    sh.qmax[warp] = mx;
   }
   __syncthreads();
+}
 
-  int src, s_idx, nsrc, ntiles;
-  if (split < P.splits_hi) {
-    src = 0; s_idx = split; nsrc = P.splits_hi; ntiles = P.tiles_hi;
-  } else if (split < P.splits_hi + P.splits_lo) {
-    src = 1; s_idx = split - P.splits_hi; nsrc = P.splits_lo; ntiles = P.tiles_lo;
-  } else {
-    src = 2; s_idx = 0; nsrc = 1; ntiles = P.tiles_st;
+// An affine warp's state into the merge area: (e, l, zs) per head and its O^T rows.
+// O columns are heads 2t, 2t+1 (for G <= 4, columns 4..7 hold the lo parts of heads
+// 0..3; they are written as rows 4..7 and folded in by merge_warps); rows 16m + g (+8)
+// are V rows u = 2m (+1) of lane group g, i.e. output dims v_dim(g, u).
+__device__ void affine_rows(WarpState& st, int L, int G, MergeArea& mg, float* merge_o) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int g = lane >> 2, t = lane & 3;
+  // reduce l and zs over the lanes that share a softmax head
+#pragma unroll
+  for (int off = 1; off <= 16; off <<= 1) {
+    if (off == 4 || off == 8 || (off == 16 && G > 4)) continue;
+    st.l += __shfl_xor_sync(0xffffffffu, st.l, off);
+    st.zs += __shfl_xor_sync(0xffffffffu, st.zs, off);
   }
-  const int per = (ntiles + nsrc - 1) / nsrc;
-  const int t_begin = min(ntiles, s_idx * per), t_end = min(ntiles, t_begin + per);
-  const int L = src == 0 ? a.L_hi : a.L_lo;
-
-  const bool tq = a.base == SEMKV_BASE_TQ && src != 2;
-  if (src == 2) {
-    run_stage(a, sh, b, h, G, merge_m, merge_l, merge_z, merge_o);
-  } else if (tq) {
-    const int64_t cap = src == 0 ? a.hi_cap : a.lo_cap;
-    const int64_t count = src == 0 ? a.hi_count : a.lo_count;
-    const uint8_t* pool = src == 0 ? a.hi_pool : a.lo_pool;
-    const int rec = record_bytes_rt(SEMKV_BASE_TQ, L);
-    const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
-    switch (L) {
-#define SEMKV_TQ_CASE(LV) \
-      case LV: run_pool_tq<LV>(a, sh, src, pool_bh, count, t_begin, t_end, G, merge_m, merge_l, merge_z, merge_o); break;
-      SEMKV_TQ_CASE(2) SEMKV_TQ_CASE(3) SEMKV_TQ_CASE(4) SEMKV_TQ_CASE(5)
-      SEMKV_TQ_CASE(6) SEMKV_TQ_CASE(7) SEMKV_TQ_CASE(8)
-#undef SEMKV_TQ_CASE
-      default: break;
-    }
-  } else {
-    WarpState st;
-    state_init(st);
-    const int64_t cap = src == 0 ? a.hi_cap : a.lo_cap;
-    const int64_t count = src == 0 ? a.hi_count : a.lo_count;
-    const uint8_t* pool = src == 0 ? a.hi_pool : a.lo_pool;
-    const int rec = record_bytes_rt(SEMKV_BASE_AFFINE, L);
-    const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
-    uint64_t* bars = &sh.bar[0][0];
-    switch (L) {
-      case 2: G <= 4 ? run_pool<2, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<2, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 3: G <= 4 ? run_pool<3, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<3, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 4: G <= 4 ? run_pool<4, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<4, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 5: G <= 4 ? run_pool<5, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<5, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 6: G <= 4 ? run_pool<6, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<6, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 7: G <= 4 ? run_pool<7, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<7, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      case 8: G <= 4 ? run_pool<8, true>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st)
-                     : run_pool<8, false>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st); break;
-      default: break;
-    }
-    // reduce l and zs over the lanes that share a softmax head
-    const int g = lane >> 2, t = lane & 3;
+  __syncthreads();  // every warp is done with the ring: reuse it as the merge area
+  if (t == 0 && g < G) {
+    mg.m[warp * 8 + g] = st.e;
+    mg.l[warp * 8 + g] = st.l;
+    mg.z[warp * 8 + g] = st.zs;
+  }
 #pragma unroll
-    for (int off = 1; off <= 16; off <<= 1) {
-      if (off == 4 || off == 8 || (off == 16 && G > 4)) continue;
-      st.l += __shfl_xor_sync(0xffffffffu, st.l, off);
-      st.zs += __shfl_xor_sync(0xffffffffu, st.zs, off);
-    }
-    __syncthreads();  // every warp is done with the ring: reuse it as the merge area
-    if (t == 0 && g < G) {
-      merge_m[warp * 8 + g] = st.e;
-      merge_l[warp * 8 + g] = st.l;
-      merge_z[warp * 8 + g] = st.zs;
-    }
-    // O columns are heads 2t, 2t+1 (for G <= 4, columns 4..7 hold the lo parts of
-    // heads 0..3; they are written as rows 4..7 and folded in below); rows 16m + g
-    // (+8) are V rows u = 2m (+1) of lane group g, i.e. output dims v_dim(g, u)
+  for (int c = 0; c < 2; ++c) {
+    const int qh = 2 * t + c;
+    if (qh < G || (G <= 4 && qh >= 4 && qh - 4 < G)) {
 #pragma unroll
-    for (int c = 0; c < 2; ++c) {
-      const int qh = 2 * t + c;
-      if (qh < G || (G <= 4 && qh >= 4 && qh - 4 < G)) {
+      for (int m = 0; m < 8; ++m) {
 #pragma unroll
-        for (int m = 0; m < 8; ++m) {
-#pragma unroll
-          for (int r = 0; r < 2; ++r) {
-            int dim;
-            switch (L) {
-              case 2: dim = v_dim<2>(g, 2 * m + r); break;
-              case 3: dim = v_dim<3>(g, 2 * m + r); break;
-              case 4: dim = v_dim<4>(g, 2 * m + r); break;
-              case 5: dim = v_dim<5>(g, 2 * m + r); break;
-              case 6: dim = v_dim<6>(g, 2 * m + r); break;
-              case 7: dim = v_dim<7>(g, 2 * m + r); break;
-              default: dim = v_dim<8>(g, 2 * m + r); break;
-            }
-            merge_o[(warp * 8 + qh) * 128 + dim] = st.O[m][2 * r + c];
+        for (int r = 0; r < 2; ++r) {
+          int dim;
+          switch (L) {
+            case 2: dim = v_dim<2>(g, 2 * m + r); break;
+            case 3: dim = v_dim<3>(g, 2 * m + r); break;
+            case 4: dim = v_dim<4>(g, 2 * m + r); break;
+            case 5: dim = v_dim<5>(g, 2 * m + r); break;
+            case 6: dim = v_dim<6>(g, 2 * m + r); break;
+            case 7: dim = v_dim<7>(g, 2 * m + r); break;
+            default: dim = v_dim<8>(g, 2 * m + r); break;
           }
+          merge_o[(warp * 8 + qh) * 128 + dim] = st.O[m][2 * r + c];
         }
       }
     }
   }
-  __syncthreads();
+}
 
-  // merge the warps: scale factors per (warp, head), then the rows
-  float* part = a.partials + (((int64_t)b * a.H + h) * P.splits + split) * kPartialFloats;
+// Merge the warps' rows into one partial (m, l, o) per head and write it.  kind 0:
+// affine pool rows (sum p' c; plus sum p z; lo rows folded for G <= 4); 1: TQ rows
+// (rotated back); 2: staged rows (plain sums).
+__device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeArea& mg,
+                            float* merge_o, float* part) {
+  __syncthreads();
   if (threadIdx.x < 8) {
     const int qh = threadIdx.x;
     float M = -INFINITY;
     if (qh < G)
-      for (int w = 0; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + qh]);
+      for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mg.m[w * 8 + qh]);
     float lsum = 0.0f, zsum = 0.0f;
     for (int w = 0; w < kWarps; ++w) {
-      const float mw = qh < G ? merge_m[w * 8 + qh] : -INFINITY;
+      const float mw = qh < G ? mg.m[w * 8 + qh] : -INFINITY;
       const float sc = (M == -INFINITY || mw == -INFINITY) ? 0.0f : exp2f(mw - M);
-      cta_scale[w * 8 + qh] = sc;
+      mg.scale[w * 8 + qh] = sc;
       if (sc != 0.0f) {
-        lsum += sc * merge_l[w * 8 + qh];
-        zsum += sc * merge_z[w * 8 + qh];
+        lsum += sc * mg.l[w * 8 + qh];
+        zsum += sc * mg.z[w * 8 + qh];
       }
     }
     if (qh < G) {
       part[qh] = M;
       part[8 + qh] = lsum;
     }
-    cta_z[qh] = zsum;
+    mg.cta_z[qh] = zsum;
   }
   __syncthreads();
   float* merged = merge_o + kWarps * 8 * 128;  // [8][128], after the warp rows
@@ -1045,19 +1007,17 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
     const int qh = i >> 7, d = i & 127;
     float o = 0.0f;
     for (int w = 0; w < kWarps; ++w) {
-      const float sc = cta_scale[w * 8 + qh];
+      const float sc = mg.scale[w * 8 + qh];
       if (sc != 0.0f) {
         float v = merge_o[(w * 8 + qh) * 128 + d];
-        if (src != 2 && !tq && G <= 4) v += merge_o[(w * 8 + qh + 4) * 128 + d];
+        if (kind == 0 && G <= 4) v += merge_o[(w * 8 + qh + 4) * 128 + d];
         o += sc * v;
       }
     }
-    // affine pool rows hold sum p' c, plus the offset part sum p z; TQ rows and
-    // staged rows are plain weighted sums
-    merged[qh * 128 + d] = (src == 2 || tq) ? o : o + cta_z[qh];
+    merged[qh * 128 + d] = kind == 0 ? o + mg.cta_z[qh] : o;
   }
   __syncthreads();
-  if (tq) {
+  if (kind == 1) {
     // back from the rotated domain: o = S H o' (unnormalised transform, stages 1..64)
     for (int hs = 1; hs < 128; hs <<= 1) {
       for (int i = threadIdx.x; i < G * 64; i += kThreads) {
@@ -1071,12 +1031,150 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a) {
       __syncthreads();
     }
   }
-  const int8_t* sg = tq ? a.signs + ((int64_t)a.layer * a.H + h) * 128 : nullptr;
+  const int8_t* sg = kind == 1 ? a.signs + ((int64_t)a.layer * a.H + h) * 128 : nullptr;
   for (int i = threadIdx.x; i < G * 128; i += kThreads) {
     const int qh = i >> 7, d = i & 127;
     const float o = merged[qh * 128 + d];
-    part[16 + qh * 128 + d] = tq ? o * (float)sg[d] : o;
+    part[16 + qh * 128 + d] = kind == 1 ? o * (float)sg[d] : o;
   }
+  __syncthreads();  // the merge area (the ring) is free again
+}
+
+template <int L>
+__device__ void run_pool_any_g(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint4* aq_all,
+                               uint64_t* bars, const uint8_t* pool_bh, int64_t count, int t0,
+                               int t1, int G, WarpState& st, int& ring_it) {
+  if (G <= 4)
+    run_pool<L, true>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it);
+  else
+    run_pool<L, false>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it);
+}
+
+// Affine pools, balanced plan: CTA c takes the weighted range [c per, (c+1) per) of the
+// concatenated [hi | lo] tile sequence of every (b, h) (a tile belongs to the CTA whose
+// range holds its start), one partial per (pair, pool) segment it touches.  One wave of
+// equal CTAs: no quantisation into waves and no per-split start-up beyond that.
+__global__ void __launch_bounds__(kThreads, kCtasAffine) decode_affine_kernel(DecodeArgs a) {
+  extern __shared__ __align__(128) uint8_t dyn[];
+  __shared__ Shared sh;
+  __shared__ MergeArea mg;
+  uint8_t* ring = dyn;
+  uint4* aq_all = reinterpret_cast<uint4*>(dyn + kRingBytes);
+  float* merge_o = reinterpret_cast<float*>(dyn);  // [kWarps][8][128] rows, then [8][128]
+  const DecodePlan& P = a.plan;
+  const int G = a.Hq / a.H;
+  const int64_t pairs = (int64_t)a.B * a.H;
+  const int64_t total = pairs * P.W;
+  const int64_t start = (int64_t)blockIdx.x * P.per;
+  const int64_t end = min(start + P.per, total);
+
+  if (threadIdx.x < kWarps * kStages) mbar_init(&sh.bar[0][0] + threadIdx.x);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  __syncthreads();
+  int ring_it = 0;  // tiles this warp has taken through its ring (barrier phases)
+  int64_t loaded = -1;
+  for (int64_t bh = start / P.W; bh < pairs && bh * P.W < end; ++bh) {
+    const int b = (int)(bh / a.H), h = (int)(bh % a.H);
+    for (int src = 0; src < 2; ++src) {
+      const int tiles = src ? P.tiles_lo : P.tiles_hi;
+      const int w = src ? P.w_lo : P.w_hi;
+      const int64_t S = bh * P.W + (src ? (int64_t)P.w_hi * P.tiles_hi : 0);
+      const int64_t E = S + (int64_t)w * tiles;
+      if (E <= S || E <= start || S >= end) continue;
+      const int64_t x0 = max(start, S) - S, x1 = min(end, E) - S;
+      const int t0 = (int)((x0 + w - 1) / w);
+      const int t1 = (int)min((int64_t)tiles, (x1 + w - 1) / w);
+      int n_hi, n_lo;
+      pair_slots(P, bh, n_hi, n_lo);
+      const int slot = (int)((int64_t)blockIdx.x - S / P.per) + (src ? n_hi : 0);
+      if (bh != loaded) {
+        load_group_q(a, sh, b, h, G);
+        loaded = bh;
+      }
+      WarpState st;
+      state_init(st);
+      const int L = src ? a.L_lo : a.L_hi;
+      const int64_t cap = src ? a.lo_cap : a.hi_cap;
+      const int64_t count = src ? a.lo_count : a.hi_count;
+      const uint8_t* pool = src ? a.lo_pool : a.hi_pool;
+      const uint8_t* pool_bh =
+          pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * record_bytes_rt(SEMKV_BASE_AFFINE, L);
+      uint64_t* bars = &sh.bar[0][0];
+      switch (L) {
+        case 2: run_pool_any_g<2>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it); break;
+        case 3: run_pool_any_g<3>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it); break;
+        case 4: run_pool_any_g<4>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it); break;
+        case 5: run_pool_any_g<5>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it); break;
+        case 6: run_pool_any_g<6>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it); break;
+        case 7: run_pool_any_g<7>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it); break;
+        case 8: run_pool_any_g<8>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it); break;
+        default: break;
+      }
+      affine_rows(st, L, G, mg, merge_o);
+      merge_warps(a, 0, h, G, mg, merge_o, a.partials + (bh * P.stride + slot) * kPartialFloats);
+    }
+  }
+}
+
+// TQ pools (KIND 1, one CTA per split) and the fp16 stage (KIND 2, one CTA per pair).
+template <int KIND>
+__global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs a) {
+  extern __shared__ __align__(128) uint8_t dyn[];
+  __shared__ Shared sh;
+  __shared__ MergeArea mg;
+  float* merge_o = reinterpret_cast<float*>(dyn);  // [kWarps][8][128] rows, then [8][128]
+  const DecodePlan& P = a.plan;
+  const int b = blockIdx.z, h = blockIdx.y;
+  const int64_t bh = (int64_t)b * a.H + h;
+  const int G = a.Hq / a.H;
+  int split = blockIdx.x;
+  if (KIND == 2) {
+    if (P.balanced) {
+      int n_hi, n_lo;
+      pair_slots(P, bh, n_hi, n_lo);
+      split = n_hi + n_lo;
+    } else {
+      split = P.splits_hi + P.splits_lo;
+    }
+  }
+  load_group_q(a, sh, b, h, G);
+  if (KIND == 1) {
+    for (int i = threadIdx.x; i < 8 * 128; i += kThreads) {
+      const int c = i >> 7, d = i & 127;
+      sh.qr[c][d] = c < G ? a.qrot[((int64_t)b * a.Hq + h * G + c) * 128 + d] : 0.0f;
+    }
+    if (threadIdx.x < 16) {
+      const int which = threadIdx.x >> 3, k = threadIdx.x & 7;
+      const int L = which == 0 ? a.L_hi : a.L_lo;
+      sh.cb[which][k] = k < L ? (which == 0 ? a.cb_hi : a.cb_lo)[k] : 0.0f;
+    }
+  }
+  __syncthreads();
+  if constexpr (KIND == 2) {
+    run_stage(a, sh, b, h, G, mg.m, mg.l, mg.z, merge_o);
+  } else {
+    const int src = split < P.splits_hi ? 0 : 1;
+    const int s_idx = src == 0 ? split : split - P.splits_hi;
+    const int nsrc = src == 0 ? P.splits_hi : P.splits_lo;
+    const int ntiles = src == 0 ? P.tiles_hi : P.tiles_lo;
+    const int per = (ntiles + nsrc - 1) / nsrc;
+    const int t_begin = min(ntiles, s_idx * per), t_end = min(ntiles, t_begin + per);
+    const int L = src == 0 ? a.L_hi : a.L_lo;
+    const int64_t cap = src == 0 ? a.hi_cap : a.lo_cap;
+    const int64_t count = src == 0 ? a.hi_count : a.lo_count;
+    const uint8_t* pool = src == 0 ? a.hi_pool : a.lo_pool;
+    const int rec = record_bytes_rt(SEMKV_BASE_TQ, L);
+    const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
+    switch (L) {
+#define SEMKV_TQ_CASE(LV) \
+      case LV: run_pool_tq<LV>(a, sh, src, pool_bh, count, t_begin, t_end, G, mg.m, mg.l, mg.z, merge_o); break;
+      SEMKV_TQ_CASE(2) SEMKV_TQ_CASE(3) SEMKV_TQ_CASE(4) SEMKV_TQ_CASE(5)
+      SEMKV_TQ_CASE(6) SEMKV_TQ_CASE(7) SEMKV_TQ_CASE(8)
+#undef SEMKV_TQ_CASE
+      default: break;
+    }
+  }
+  merge_warps(a, KIND, h, G, mg, merge_o, a.partials + (bh * P.stride + split) * kPartialFloats);
 }
 
 // merge the splits of each (b, qh): one warp per head, 4 dims per lane
@@ -1086,8 +1184,9 @@ __global__ void combine_kernel(DecodeArgs a) {
   if (gw >= a.B * a.Hq) return;
   const int b = gw / a.Hq, qh = gw % a.Hq;
   const int G = a.Hq / a.H, h = qh / G, c = qh % G;
-  const int S = a.plan.splits;
-  const float* base = a.partials + ((int64_t)b * a.H + h) * S * kPartialFloats;
+  const int64_t bh = (int64_t)b * a.H + h;
+  const int S = pair_partials(a.plan, bh);
+  const float* base = a.partials + bh * a.plan.stride * kPartialFloats;
   float M = -INFINITY;
   for (int s = 0; s < S; ++s) M = fmaxf(M, base[s * kPartialFloats + c]);
   float o[4] = {0.f, 0.f, 0.f, 0.f}, lsum = 0.0f;
@@ -1112,19 +1211,74 @@ __global__ void combine_kernel(DecodeArgs a) {
 
 }  // namespace
 
-DecodePlan make_decode_plan(int B, int H, int64_t hi_count, int64_t lo_count, int stage_n,
-                            int num_sms) {
+// relative cost of a 16-token tile per level count (decode instructions per tile)
+static int tile_cost(int L) {
+  switch (L) {
+    case 3: case 6: return 8;   // five-code groups: five multiplies per symbol
+    case 5: return 7;
+    case 7: case 8: return 6;
+    default: return 5;          // L = 2, 4: one code per symbol
+  }
+}
+
+DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int64_t hi_count,
+                            int64_t lo_count, int stage_n, int num_sms, int max_stride) {
   DecodePlan p;
+  std::memset(&p, 0, sizeof(p));
   p.tiles_hi = (int)((hi_count + kTile - 1) / kTile);
   p.tiles_lo = (int)((lo_count + kTile - 1) / kTile);
   p.tiles_st = (stage_n + kTile - 1) / kTile;
   const int st = stage_n > 0 ? 1 : 0;
+  p.splits_st = st;
   const int64_t pairs = (int64_t)B * H;
-  const int64_t slots = (int64_t)num_sms * 2;  // two 8-warp CTAs per SM
+  if (max_stride > kMaxSplits + 1) max_stride = kMaxSplits + 1;
+  if (base == SEMKV_BASE_AFFINE) {
+    // balanced: one wave of equal CTAs over the weighted tiles of every pair
+    p.balanced = 1;
+    p.w_hi = tile_cost(L_hi);
+    p.w_lo = tile_cost(L_lo);
+    p.W = (int64_t)p.w_hi * p.tiles_hi + (int64_t)p.w_lo * p.tiles_lo;
+    const int64_t total = pairs * p.W;
+    if (total == 0) {
+      p.per = 1;
+      p.ctas = 0;
+      p.stride = st;
+      return p;
+    }
+    const int64_t target = (int64_t)num_sms * kCtasAffine;
+    int64_t per = (total + target - 1) / target;
+    const int64_t min_work = (int64_t)(p.w_hi > p.w_lo ? p.w_hi : p.w_lo) * kWarps * 2;
+    if (per < min_work) per = min_work;
+    // a segment of length x meets at most x / per + 2 CTAs: keep a pair's partials
+    // (hi + lo + stage) within max_stride
+    const int64_t avail = (int64_t)max_stride - st - 4;
+    if (avail < 1) {
+      p.per = per;
+      p.ctas = 0;
+      p.stride = max_stride + 1;  // infeasible: the caller reports the workspace as short
+      return p;
+    }
+    const int64_t per_min = (p.W + avail - 1) / avail;
+    if (per < per_min) per = per_min;
+    p.per = per;
+    p.ctas = (int)((total + per - 1) / per);
+    int worst = 0;
+    for (int64_t bh = 0; bh < pairs; ++bh) {
+      int n_hi, n_lo;
+      pair_slots(p, bh, n_hi, n_lo);
+      if (n_hi + n_lo > worst) worst = n_hi + n_lo;
+    }
+    p.stride = worst + st;
+    p.splits = 0;
+    return p;
+  }
+  // split plan (TQ pools): S CTAs per pair, divided between the pools by tile count
+  const int64_t slots = (int64_t)num_sms * kCtasOther;  // resident CTAs
   const int nt = p.tiles_hi + p.tiles_lo;
+  const int s_max = max_stride - st < kMaxSplits ? max_stride - st : kMaxSplits;
   int best_s = 1;
   double best_cost = 1e300;
-  for (int S = 1; S <= kMaxSplits; ++S) {
+  for (int S = 1; S <= s_max; ++S) {
     int shi = 0, slo = 0;
     if (p.tiles_hi > 0 && p.tiles_lo > 0) {
       if (S < 2) continue;
@@ -1154,16 +1308,24 @@ DecodePlan make_decode_plan(int B, int H, int64_t hi_count, int64_t lo_count, in
   if (nt == 0) {
     p.splits_hi = p.splits_lo = 0;
   } else if (p.tiles_hi > 0 && p.tiles_lo > 0) {
+    if (s_max < 2) {
+      p.stride = max_stride + 1;  // infeasible
+      return p;
+    }
     int shi = (int)((double)best_s * p.tiles_hi / nt + 0.5);
     shi = shi < 1 ? 1 : (shi > best_s - 1 ? best_s - 1 : shi);
     p.splits_hi = shi;
     p.splits_lo = best_s - shi;
   } else {
+    if (s_max < 1) {
+      p.stride = max_stride + 1;
+      return p;
+    }
     p.splits_hi = p.tiles_hi > 0 ? best_s : 0;
     p.splits_lo = p.tiles_lo > 0 ? best_s : 0;
   }
-  p.splits_st = st;
   p.splits = p.splits_hi + p.splits_lo + p.splits_st;
+  p.stride = p.splits;
   return p;
 }
 
@@ -1174,22 +1336,39 @@ size_t decode_workspace_floats(int B, int H, int Hq) {
 cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kDynBytes);
+    cudaError_t e = cudaFuncSetAttribute(decode_affine_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kRingBytes + kAqBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               kRingBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(decode_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               kRingBytes);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  if (a.plan.splits == 0) return cudaErrorInvalidValue;
+  const DecodePlan& P = a.plan;
+  if (P.stride < 1 || P.stride > kMaxSplits + 1) return cudaErrorInvalidValue;
+  cudaError_t e = cudaSuccess;
   if (a.base == SEMKV_BASE_TQ) {
     const int heads = a.B * a.Hq;
     qrot_kernel<<<(heads + 7) / 8, 256, 0, stream>>>(a);
-    cudaError_t e = cudaGetLastError();
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int pool_splits = P.splits_hi + P.splits_lo;
+    if (pool_splits > 0)
+      decode_kernel<1><<<dim3(pool_splits, a.H, a.B), kThreads, kRingBytes, stream>>>(a);
+  } else if (P.ctas > 0) {
+    decode_affine_kernel<<<P.ctas, kThreads, kRingBytes + kAqBytes, stream>>>(a);
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (P.splits_st > 0) {
+    decode_kernel<2><<<dim3(1, a.H, a.B), kThreads, kRingBytes, stream>>>(a);
+    e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  dim3 grid(a.plan.splits, a.H, a.B);
-  decode_kernel<<<grid, kThreads, kDynBytes, stream>>>(a);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
   const int heads = a.B * a.Hq;
   combine_kernel<<<(heads + 7) / 8, 256, 0, stream>>>(a);
   return cudaGetLastError();

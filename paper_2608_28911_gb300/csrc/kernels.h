@@ -46,8 +46,16 @@ cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream);
 // Decode attention over one layer of the cache (split-K + combine).
 struct DecodePlan {
   int tiles_hi, tiles_lo, tiles_st;     // 16-token tiles per (b, h) per source
-  int splits_hi, splits_lo, splits_st;  // CTAs per (b, h) per source
-  int splits;                            // total partials per (b, h)
+  int splits_hi, splits_lo, splits_st;  // split plan: CTAs per (b, h) per source
+  int splits;                            // split plan: partials per (b, h)
+  int stride;                            // partial slots reserved per (b, h)
+  // balanced plan (affine pools): one wave of CTAs over the weighted tiles of every
+  // (b, h) in the order [hi | lo]; a hi tile weighs w_hi, a lo tile w_lo
+  int balanced;
+  int w_hi, w_lo;
+  int64_t W;                             // weighted length of one (b, h)
+  int64_t per;                           // weighted length per CTA
+  int ctas;
 };
 struct DecodeArgs {
   int base, L_hi, L_lo;
@@ -70,8 +78,11 @@ struct DecodeArgs {
   DecodePlan plan;
 };
 constexpr int kPartialFloats = 16 + 8 * 128;  // m[8], l[8], o[8][128]
-DecodePlan make_decode_plan(int B, int H, int64_t hi_count, int64_t lo_count, int stage_n,
-                            int num_sms);
+// max_stride: partial slots available per (b, h); a plan whose stride exceeds it
+// cannot be run with that workspace
+DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int64_t hi_count,
+                            int64_t lo_count, int stage_n, int num_sms, int max_stride);
+constexpr int kMaxPartialsPerPair = 65;
 size_t decode_workspace_floats(int B, int H, int Hq);
 cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream);
 

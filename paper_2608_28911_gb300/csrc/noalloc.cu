@@ -72,28 +72,15 @@ extern "C" semkv_status semkv_decode_attention_noalloc(const semkv_quant_desc* d
 
   const int sms = device_sm_count();
   if (sms <= 0) return SEMKV_ECUDA;
-  // Fit the split plan to the array: each (sequence, KV head) gets at most
-  // cap = capacity / (batch * kv_heads) partials; at least one per non-empty source.
+  // Fit the plan to the array: each (sequence, KV head) gets at most
+  // cap = capacity / (batch * kv_heads) partial slots.
   const int64_t pairs = (int64_t)c->batch * c->kv_heads;
-  const int64_t cap = (int64_t)(kScratchFloats / kPartialFloats) / pairs;
-  DecodePlan plan = make_decode_plan(c->batch, c->kv_heads, c->hi_count, c->lo_count, c->stage_n, sms);
-  const int need = (plan.tiles_hi > 0) + (plan.tiles_lo > 0) + plan.splits_st;
-  if (cap < need) return SEMKV_EWORKSPACE;  // the request exceeds the static scratch
-  if (plan.splits > cap) {
-    const int pool_cap = (int)cap - plan.splits_st;
-    const int pools = plan.splits_hi + plan.splits_lo;
-    if (plan.splits_hi > 0 && plan.splits_lo > 0) {
-      int hi = (int)((int64_t)plan.splits_hi * pool_cap / pools);
-      hi = hi < 1 ? 1 : (hi > pool_cap - 1 ? pool_cap - 1 : hi);
-      plan.splits_hi = hi;
-      plan.splits_lo = pool_cap - hi;
-    } else if (plan.splits_hi > 0) {
-      plan.splits_hi = pool_cap;
-    } else if (plan.splits_lo > 0) {
-      plan.splits_lo = pool_cap;
-    }
-    plan.splits = plan.splits_hi + plan.splits_lo + plan.splits_st;
-  }
+  const int64_t cap64 = (int64_t)(kScratchFloats / kPartialFloats) / pairs;
+  const int cap = (int)(cap64 < kMaxPartialsPerPair ? cap64 : kMaxPartialsPerPair);
+  const DecodePlan plan = make_decode_plan(desc->base, desc->levels_hi, desc->levels_lo, c->batch,
+                                           c->kv_heads, c->hi_count, c->lo_count, c->stage_n,
+                                           sms, cap);
+  if (cap < 1 || plan.stride > cap) return SEMKV_EWORKSPACE;  // exceeds the static scratch
 
   float* scratch = nullptr;
   semkv_status s = scratch_address(&scratch);
