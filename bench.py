@@ -451,7 +451,9 @@ def main():
                      "peak_kind": f"{peak_kind} hbm_gbs"},
         "e2e": {"value": job_gbs(step_bytes, world, r["e2e_time"]), "unit": "GB/s",
                 "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
-        "gpu_launches": 4 * args.steps,
+        # per step: the block append (rank, slot->token scatter, quantize) and the
+        # decode (pool kernel, combine); the stage is empty when decode runs
+        "gpu_launches": 5 * args.steps,
         "clocks": r["clocks"],
         "device_error": r["err"],
     }
