@@ -1,25 +1,30 @@
 """Benchmark of the SemKV packed mixed-precision KV cache on GB300.
 
-Workload (default): one layer of the Llama-3.1-8B KV shape (8 KV heads, 32 query
-heads, head_dim 128), batch 16 x 65536-token context, affine 6/5 levels with the
-top 26% of tokens (Zipf(1.1) scores) at 6 levels, block B = 128.  Inputs are seeded
-synthetic tensors (fp16 N(0,1) K/V with 4 outlier channels x8 per head), standing
-in for LongBench prompts run through the model.
+Workload (default, --config b16x64k): one layer of the Llama-3.1-8B KV shape (8 KV
+heads, 32 query heads, head_dim 128), batch 16 x 65536-token context, affine 6/5
+levels with the top 26% of tokens (Zipf(1.1) scores) at 6 levels, block B = 128.
+Inputs are seeded synthetic tensors (fp16 N(0,1) K/V with 4 outlier channels x8 per
+head), standing in for LongBench prompts run through the model.  Other --config
+values measure the other workloads (tiny, b1x32k, l32x128k, blk4k, tq32k).
 
 One step = one pass of the generation-time hot path over the batch:
   A6  block-exact deferred quantization of a block of 128 staged tokens
       (semkv_append_block: top-r rank in the block, quantize, pack, append), and
-  A7  decode attention for all 32 query heads over the whole cache
-      (65536 prompt tokens + the appended block), split-K + combine.
+  A7  decode attention for all query heads over the whole cache (the prompt + the
+      appended block), for every layer of the config, split-K + combine.
 The appended slots are reused every step (counts rewound), so the work per step is
-constant.  The prompt's own rank + quantize (A1-A5 at full size) is timed apart and
+constant.  In the block-wise config (blk4k) a step stages ONE generated token, runs
+the block append when the stage is full, and decodes over the pools plus the fp16
+stage.  The prompt's own rank + quantize (A1-A5 at full size) is timed apart and
 reported as quantize_gbs.
 
-value = algorithmic bytes of the step (records read by decode attention, q and out,
-plus the block's fp16 K/V read and records written) / step time, in GB/s: decode
-dominates (722 MB of records per step, larger than the 129 MB L2, so every timed step
-streams from HBM).  roofline: decode attention's bytes per launch / its mean launch
-time (CUDA events on the launching stream) against the measured HBM copy peak.
+value = algorithmic bytes of the step (records and staged fp16 rows read by decode
+attention, q and out, plus the appended block's fp16 K/V read and records written) /
+step time, in GB/s.  The default workload moves 722 MB of records per step, more
+than the 129 MB L2; workloads smaller than twice the L2 are timed step by step with
+an L2 flush (a 512 MB write) between steps, outside the timed events.  roofline:
+decode attention's bytes per step / its mean time (CUDA events on the launching
+stream) against the measured HBM copy peak.
 """
 from __future__ import annotations
 
@@ -45,19 +50,40 @@ from paper_2608_28911_gb300 import synthetic  # noqa: E402
 
 METRIC = ("packed-KV decode attention µs/step and HBM GB/s (% of peak); quantize GB/s")
 
+_LLAMA = "8 KV heads, 32 q heads, d=128"
 CONFIGS = {
-    # name: batch, context, layers, kv heads, q heads, L_hi, L_lo, r, block, seed
-    "b16x64k": dict(B=16, T=65536, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100), block=128,
-                    seed=3, desc="batch 16 x 64K context, 1 layer of the Llama-3.1-8B KV shape "
-                                 "(8 KV heads, 32 q heads, d=128), affine 6/5 levels at r=26%"),
-    "b4x64k": dict(B=4, T=65536, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100), block=128,
-                   seed=3, desc="batch 4 x 64K context, 1 layer of the Llama-3.1-8B KV shape "
-                                "(8 KV heads, 32 q heads, d=128), affine 6/5 levels at r=26% "
-                                "(profiling size: 180 MB of records, above L2)"),
-    "b1x32k": dict(B=1, T=32768, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100), block=128,
-                   seed=2, desc="batch 1 x 32K context, 1 layer of the Llama-3.1-8B KV shape, "
-                                "affine 6/5 levels at r=26%"),
+    # base 0 = affine, 1 = TQ-MSE; mode "block": stage + append a 128-token block per
+    # step; "token": stage one token per step, append when the stage is full
+    "b16x64k": dict(base=0, B=16, T=65536, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100),
+                    block=128, seed=3, mode="block",
+                    desc=f"batch 16 x 64K context, 1 layer of the Llama-3.1-8B KV shape "
+                         f"({_LLAMA}), affine 6/5 levels at r=26%"),
+    "b4x64k": dict(base=0, B=4, T=65536, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100),
+                   block=128, seed=3, mode="block",
+                   desc=f"batch 4 x 64K context, 1 layer of the Llama-3.1-8B KV shape "
+                        f"({_LLAMA}), affine 6/5 levels at r=26% (profiling size: 180 MB "
+                        f"of records, above L2)"),
+    "b1x32k": dict(base=0, B=1, T=32768, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100),
+                   block=128, seed=2, mode="block",
+                   desc=f"batch 1 x 32K context, 1 layer of the Llama-3.1-8B KV shape "
+                        f"({_LLAMA}), affine 6/5 levels at r=26%"),
+    "tiny": dict(base=0, B=1, T=1024, NL=1, H=1, Hq=4, L_hi=5, L_lo=5, r=(0, 100), block=128,
+                 seed=0, mode="block",
+                 desc="1 layer, 1 KV head, 4 q heads, 1024 tokens, uniform 5-level affine"),
+    "l32x128k": dict(base=0, B=1, T=131072, NL=32, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100),
+                     block=128, seed=3, mode="block",
+                     desc=f"batch 1 x 128K context, all 32 layers of the Llama-3.1-8B KV shape "
+                          f"({_LLAMA}), affine 6/5 levels at r=26%, every layer decoded"),
+    "blk4k": dict(base=0, B=1, T=4096, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100),
+                  block=128, seed=4, mode="token",
+                  desc=f"4K-token prompt + generated tokens one per step, block-wise "
+                       f"deferred quantization every 128 tokens, 1 layer ({_LLAMA}), affine 6/5"),
+    "tq32k": dict(base=1, B=1, T=32768, NL=1, H=8, Hq=32, L_hi=4, L_lo=3, r=(3, 4), block=128,
+                  seed=5, mode="block",
+                  desc=f"batch 1 x 32K context, 1 layer of the Mistral-7B KV shape ({_LLAMA}), "
+                       f"rotated TurboQuant-MSE-style base at 4/3 levels, r=75%"),
 }
+L2_BYTES = 129 * 2**20
 
 
 def profiled_traffic(config_name: str):
@@ -169,33 +195,49 @@ def build_workload(cfg, dev):
     blk = cfg["block"]
     n_high = semkv.semkv_high_count_floor(T, r_num, r_den)
     n_high_blk = semkv.semkv_block_high_count(blk, r_num, r_den)
-    desc = semkv.QuantDesc(semkv.BASE_AFFINE, cfg["L_hi"], cfg["L_lo"], device=dev)
+    signs = synthetic.signs(cfg["seed"], NL, H) if cfg["base"] == semkv.BASE_TQ else None
+    desc = semkv.QuantDesc(cfg["base"], cfg["L_hi"], cfg["L_lo"], signs=signs, device=dev)
     cache = semkv.KVCache(desc, B, NL, H, Hq, hi_cap=n_high + n_high_blk,
                           lo_cap=T - n_high + blk - n_high_blk, block=blk, device=dev)
     k = torch.empty((B, NL, H, T, 128), dtype=torch.float16, device=dev)
     v = torch.empty_like(k)
     scores = torch.empty((B, T), dtype=torch.float32, device=dev)
+    big = NL * H * T > 2**24   # draw large caches on the device, layer by layer
     for b in range(B):   # one seeded stream per sequence keeps host memory small
-        kb, vb = synthetic.kv(cfg["seed"] * 100 + b, 1, NL, H, T)
-        k[b].copy_(torch.from_numpy(kb[0]))
-        v[b].copy_(torch.from_numpy(vb[0]))
-        scores[b].copy_(torch.from_numpy(synthetic.scores_zipf(cfg["seed"] * 100 + b, 1, T)[0]))
+        sd = cfg["seed"] * 100 + b
+        if big:
+            for l in range(NL):
+                kl, vl = synthetic.kv_layer_device(sd, l, 1, H, T, dev)
+                k[b, l].copy_(kl[0])
+                v[b, l].copy_(vl[0])
+        else:
+            kb, vb = synthetic.kv(sd, 1, NL, H, T)
+            k[b].copy_(torch.from_numpy(kb[0]))
+            v[b].copy_(torch.from_numpy(vb[0]))
+        scores[b].copy_(torch.from_numpy(synthetic.scores_zipf(sd, 1, T)[0]))
     return dict(desc=desc, cache=cache, k=k, v=v, scores=scores, n_high=n_high,
                 n_high_blk=n_high_blk)
 
 
-def step_bytes(cfg, cache, desc):
-    """Algorithmic bytes of one step (see module docstring)."""
+def decode_bytes(cfg, desc, hi, lo, stage_n):
+    """Algorithmic bytes of one decode attention call (one layer): the records of both
+    pools, the staged fp16 rows, q and out."""
     from paper_2608_28911_gb300 import semkv
-    B, H, Hq, blk = cfg["B"], cfg["H"], cfg["Hq"], cfg["block"]
+    B, H, Hq = cfg["B"], cfg["H"], cfg["Hq"]
+    rh = semkv.semkv_record_bytes(desc.base, desc.levels_hi)
+    rl = semkv.semkv_record_bytes(desc.base, desc.levels_lo)
+    return B * H * (hi * rh + lo * rl + stage_n * 2 * 128 * 2) + B * Hq * 128 * (2 + 4)
+
+
+def append_bytes(cfg, desc):
+    """Algorithmic bytes of one block append: the block's fp16 K/V read, its scores,
+    and its records written."""
+    from paper_2608_28911_gb300 import semkv
+    B, NL, H, blk = cfg["B"], cfg["NL"], cfg["H"], cfg["block"]
     rh = semkv.semkv_record_bytes(desc.base, desc.levels_hi)
     rl = semkv.semkv_record_bytes(desc.base, desc.levels_lo)
     nh_b = semkv.semkv_block_high_count(blk, *cfg["r"])
-    hi = cache.hi_count + nh_b
-    lo = cache.lo_count + blk - nh_b
-    decode = B * H * (hi * rh + lo * rl) + B * Hq * 128 * (2 + 4)   # one layer
-    append = B * cfg["NL"] * H * (blk * 2 * 128 * 2 + nh_b * rh + (blk - nh_b) * rl) + B * blk * 4
-    return decode, append
+    return B * NL * H * (blk * 2 * 128 * 2 + nh_b * rh + (blk - nh_b) * rl) + B * blk * 4
 
 
 def gpu_arm(args, cfg, rank, world):
@@ -208,6 +250,8 @@ def gpu_arm(args, cfg, rank, world):
     desc, cache = w["desc"], w["cache"]
     B, T, NL, H, Hq, blk = cfg["B"], cfg["T"], cfg["NL"], cfg["H"], cfg["Hq"], cfg["block"]
     r_num, r_den = cfg["r"]
+    token_mode = cfg["mode"] == "token"
+    tq = cfg["base"] == semkv.BASE_TQ
 
     # ---- prompt: rank + quantize + pack (A1-A5), timed for quantize GB/s
     is_high = torch.empty((B, T), dtype=torch.uint8, device=dev)
@@ -228,8 +272,9 @@ def gpu_arm(args, cfg, rank, world):
     q_bytes = B * NL * H * (T * 2 * 128 * 2 + w["n_high"] * rh + (T - w["n_high"]) * rl) + B * T * 4
     quantize_gbs = q_bytes / statistics.median(qt) / 1e9
     del w["k"], w["v"]
+    torch.cuda.empty_cache()
 
-    # ---- generation-time step: stage a block, append it (A6), decode (A7)
+    # ---- generation-time step
     nblocks = 4
     gk, gv = synthetic.kv(cfg["seed"] * 100 + 99, B, NL, H, blk * nblocks)
     gs = synthetic.scores_zipf(cfg["seed"] * 100 + 99, B, blk * nblocks)
@@ -242,28 +287,64 @@ def gpu_arm(args, cfg, rank, world):
     ws = cache.workspace()
     scale = 1.0 / math.sqrt(128)
     base_counts = (cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens)
+    nh_b = semkv.semkv_block_high_count(blk, r_num, r_den)
+    # launches per decode call: (rotation for TQ,) pools, (stage,) combine
+    dec_launch = (1 if tq else 0) + 1 + 1
+    app_launch = 2 if tq else 3      # rank, (slot -> token scatter,) quantize
 
-    def stage_block(i):
-        j = i % nblocks
-        cache.stage_k.copy_(blocks_k[:, :, :, j * blk:(j + 1) * blk])
-        cache.stage_v.copy_(blocks_v[:, :, :, j * blk:(j + 1) * blk])
-        cache.stage_score.copy_(blocks_s[:, j * blk:(j + 1) * blk])
-        cache.s.stage_n = blk
-
-    def step(i, ev=None):
-        cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
-        stage_block(i)
-        semkv.semkv_append_block(desc, cache, r_num, r_den)
+    def decode_all(qv, ev=None):
         if ev is not None:
             ev[0].record(stream)
-        semkv.semkv_decode_attention(desc, cache, 0, q_all[i % nblocks], out, scale, ws)
+        for layer in range(NL):
+            semkv.semkv_decode_attention(desc, cache, layer, qv, out, scale, ws)
         if ev is not None:
             ev[1].record(stream)
 
+    if not token_mode:
+        def step(i, ev=None):
+            j = i % nblocks
+            cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+            cache.stage_k.copy_(blocks_k[:, :, :, j * blk:(j + 1) * blk])
+            cache.stage_v.copy_(blocks_v[:, :, :, j * blk:(j + 1) * blk])
+            cache.stage_score.copy_(blocks_s[:, j * blk:(j + 1) * blk])
+            cache.s.stage_n = blk
+            semkv.semkv_append_block(desc, cache, r_num, r_den)
+            decode_all(q_all[j], ev)
+        dec_bytes = NL * decode_bytes(cfg, desc, base_counts[0] + nh_b,
+                                      base_counts[1] + blk - nh_b, 0)
+        app_bytes = append_bytes(cfg, desc)
+        launches_per_step = app_launch + NL * dec_launch
+    else:
+        def step(i, ev=None):
+            # one generated token: stage it; append the block when the stage is full
+            n = cache.s.stage_n
+            if n == 0:
+                cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+            j = i % (nblocks * blk)
+            cache.stage_k[:, :, :, n].copy_(blocks_k[:, :, :, j])
+            cache.stage_v[:, :, :, n].copy_(blocks_v[:, :, :, j])
+            cache.stage_score[:, n].copy_(blocks_s[:, j])
+            cache.s.stage_n = n + 1
+            if cache.s.stage_n == blk:
+                semkv.semkv_append_block(desc, cache, r_num, r_den)
+            decode_all(q_all[(i // blk) % nblocks], ev)
+        # over a cycle of blk steps: stages 1..blk-1 hold that many fp16 rows, the
+        # last step decodes the appended block from the pools
+        cyc = sum(decode_bytes(cfg, desc, base_counts[0], base_counts[1], n) for n in range(1, blk))
+        cyc += decode_bytes(cfg, desc, base_counts[0] + nh_b, base_counts[1] + blk - nh_b, 0)
+        dec_bytes = NL * cyc / blk
+        app_bytes = append_bytes(cfg, desc) / blk
+        launches_per_step = (app_launch + NL * (dec_launch + 1) * (blk - 1) + NL * dec_launch) / blk
+
+    flush = NL * dec_bytes < 2 * L2_BYTES
+    scrub = torch.empty(512 * 2**20, dtype=torch.uint8, device=dev) if flush else None
+
     for i in range(args.warmup):
         step(i)
+    if token_mode:   # start the timed steps at a block boundary
+        while cache.s.stage_n != 0:
+            step(0)
     torch.cuda.synchronize()
-    dec_bytes, app_bytes = step_bytes(cfg, cache_after_rewind(cache, base_counts), desc)
 
     def barrier():
         if world > 1:
@@ -273,46 +354,87 @@ def gpu_arm(args, cfg, rank, world):
 
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in range(args.steps)]
-    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(dev.index) as clk:
-        barrier()
-        t0.record(stream)
-        for i in range(args.steps):
-            step(i, evs[i])
-        t1.record(stream)
-        barrier()
-    elapsed = t0.elapsed_time(t1) * 1e-3
+        if not flush:
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            barrier()
+            t0.record(stream)
+            for i in range(args.steps):
+                step(i, evs[i])
+            t1.record(stream)
+            barrier()
+            elapsed = t0.elapsed_time(t1) * 1e-3
+        else:
+            # small workloads: time each step alone, the L2 flushed in between
+            sev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(args.steps)]
+            barrier()
+            for i in range(args.steps):
+                scrub.fill_(i & 0xFF)
+                sev[i][0].record(stream)
+                step(i, evs[i])
+                sev[i][1].record(stream)
+            barrier()
+            elapsed = sum(a.elapsed_time(b) for a, b in sev) * 1e-3
     dec_times = [a.elapsed_time(b) * 1e-3 for a, b in evs]
     err = int(cache.dev_error.item())
 
     # ---- end to end through the public API with host buffers
-    # per-block contiguous pinned host buffers, as a serving loop would hand them over
-    pin_k = [torch.from_numpy(np.ascontiguousarray(gk[:, :, :, j * blk:(j + 1) * blk])).pin_memory()
-             for j in range(nblocks)]
-    pin_v = [torch.from_numpy(np.ascontiguousarray(gv[:, :, :, j * blk:(j + 1) * blk])).pin_memory()
-             for j in range(nblocks)]
-    pin_s = [torch.from_numpy(np.ascontiguousarray(gs[:, j * blk:(j + 1) * blk])).pin_memory()
-             for j in range(nblocks)]
+    # contiguous pinned host buffers per block (per token in the block-wise workload),
+    # as a serving loop would hand them over
+    if not token_mode:
+        pin_k = [torch.from_numpy(np.ascontiguousarray(gk[:, :, :, j * blk:(j + 1) * blk])).pin_memory()
+                 for j in range(nblocks)]
+        pin_v = [torch.from_numpy(np.ascontiguousarray(gv[:, :, :, j * blk:(j + 1) * blk])).pin_memory()
+                 for j in range(nblocks)]
+        pin_s = [torch.from_numpy(np.ascontiguousarray(gs[:, j * blk:(j + 1) * blk])).pin_memory()
+                 for j in range(nblocks)]
+        h2d = (blk * B * NL * H * 128 * 2 * 2) + blk * B * 4 + B * Hq * 128 * 2
+    else:
+        ntok = nblocks * blk
+        pin_k = torch.from_numpy(np.ascontiguousarray(np.moveaxis(gk, 3, 0))).pin_memory()
+        pin_v = torch.from_numpy(np.ascontiguousarray(np.moveaxis(gv, 3, 0))).pin_memory()
+        pin_s = torch.from_numpy(np.ascontiguousarray(gs.T)).pin_memory()
+        h2d = B * NL * H * 128 * 2 * 2 + B * 4 + B * Hq * 128 * 2
     pin_q = q_all.cpu().pin_memory()
     pin_out = torch.empty((B, Hq, 128), dtype=torch.float32).pin_memory()
-    h2d = (blk * B * NL * H * 128 * 2 * 2) + blk * B * 4 + B * Hq * 128 * 2
     d2h = B * Hq * 128 * 4
     qdev = torch.empty((B, Hq, 128), dtype=torch.float16, device=dev)
+    tok_k = torch.empty((B, NL, H, 128), dtype=torch.float16, device=dev)
+    tok_v = torch.empty_like(tok_k)
+    tok_s = torch.empty((B,), dtype=torch.float32, device=dev)
 
     def step_e2e(i):
-        j = i % nblocks
-        cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
-        cache.stage_k.copy_(pin_k[j], non_blocking=True)
-        cache.stage_v.copy_(pin_v[j], non_blocking=True)
-        cache.stage_score.copy_(pin_s[j], non_blocking=True)
-        qdev.copy_(pin_q[j], non_blocking=True)
-        cache.s.stage_n = blk
-        semkv.semkv_append_block(desc, cache, r_num, r_den)
-        semkv.semkv_decode_attention(desc, cache, 0, qdev, out, scale, ws)
+        if not token_mode:
+            j = i % nblocks
+            cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+            cache.stage_k.copy_(pin_k[j], non_blocking=True)
+            cache.stage_v.copy_(pin_v[j], non_blocking=True)
+            cache.stage_score.copy_(pin_s[j], non_blocking=True)
+            qdev.copy_(pin_q[j], non_blocking=True)
+            cache.s.stage_n = blk
+            semkv.semkv_append_block(desc, cache, r_num, r_den)
+        else:
+            n = cache.s.stage_n
+            if n == 0:
+                cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+            j = i % ntok
+            tok_k.copy_(pin_k[j], non_blocking=True)
+            tok_v.copy_(pin_v[j], non_blocking=True)
+            tok_s.copy_(pin_s[j], non_blocking=True)
+            qdev.copy_(pin_q[(i // blk) % nblocks], non_blocking=True)
+            cache.stage_token(tok_k, tok_v, tok_s)
+            if cache.s.stage_n == blk:
+                semkv.semkv_append_block(desc, cache, r_num, r_den)
+        for layer in range(NL):
+            semkv.semkv_decode_attention(desc, cache, layer, qdev, out, scale, ws)
         pin_out.copy_(out, non_blocking=True)
 
     e2e_steps = max(3, min(args.steps, 200))
-    for i in range(3):
+    if token_mode:
+        e2e_steps = max(blk, (e2e_steps // blk) * blk)
+        cache.s.stage_n = 0
+    for i in range(3 if not token_mode else blk):
         step_e2e(i)
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -326,44 +448,47 @@ def gpu_arm(args, cfg, rank, world):
     elapsed, e2e_time = max_over_ranks([elapsed, e2e_time], device=dev)
     return dict(elapsed=elapsed, dec_times=dec_times, dec_bytes=dec_bytes, app_bytes=app_bytes,
                 quantize_gbs=quantize_gbs, clocks=clk.summary(), err=err, e2e_time=e2e_time,
-                h2d=h2d, d2h=d2h)
-
-
-def cache_after_rewind(cache, base_counts):
-    cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
-    return cache
+                h2d=h2d, d2h=d2h, flush=flush, launches=launches_per_step * args.steps)
 
 
 # ------------------------------------------------------------ CPU oracle ------
 
 def oracle_sample(cfg, budget_s: float, max_steps: int | None = None):
     """The CPU oracle as it stands on a bounded sample of the same workload: one
-    (sequence, KV head) of the batch at full context -- append one block and run
-    fp64 decode attention for that head's 4 query heads -- repeated until the time
-    budget is spent.  Returns (GB/s of algorithmic bytes, sample description, steps)."""
+    (sequence, KV head) of the batch and one layer, at full context -- append one
+    block and run fp64 decode attention for that head's query heads -- repeated until
+    the time budget is spent.  Returns (GB/s of algorithmic bytes, sample description,
+    steps, seconds)."""
     import oracle
     T, Hq, H, blk = cfg["T"], cfg["Hq"], cfg["H"], cfg["block"]
+    base = cfg["base"]
     r_num, r_den = cfg["r"]
     G = Hq // H
     n_high = oracle.high_count_floor(T, r_num, r_den)
     nh_b = oracle.block_high_count(blk, r_num, r_den)
-    oc = oracle.Cache(base=0, L_hi=cfg["L_hi"], L_lo=cfg["L_lo"], batch=1, layers=1, kv_heads=1,
+    oc = oracle.Cache(base=base, L_hi=cfg["L_hi"], L_lo=cfg["L_lo"], batch=1, layers=1, kv_heads=1,
                       q_heads=G, block=blk, hi_cap=((n_high + nh_b + 15) // 16) * 16,
                       lo_cap=((T - n_high + blk + 15) // 16) * 16)
-    kb, vb = synthetic.kv(cfg["seed"] * 100, 1, 1, H, T)
+    if base == oracle.BASE_TQ:
+        oc.signs = synthetic.signs(cfg["seed"], 1, H)[:, :1]
+        _, c32, t32, _ = oracle.lloyd_max_gaussian(cfg["L_hi"])
+        oc.cb_hi = (c32, t32)
+        _, c32, t32, _ = oracle.lloyd_max_gaussian(cfg["L_lo"])
+        oc.cb_lo = (c32, t32)
+    kb, vb = synthetic.kv_layer(cfg["seed"] * 100, 0, 1, H, T)
     s = synthetic.scores_zipf(cfg["seed"] * 100, 1, T)
-    oracle.quantize_prompt(oc, synthetic.f16_bits(kb[:, :, :1]), synthetic.f16_bits(vb[:, :, :1]),
+    oracle.quantize_prompt(oc, synthetic.f16_bits(kb[:, None, :1]), synthetic.f16_bits(vb[:, None, :1]),
                            s, r_num, r_den)
     gk, gv = synthetic.kv(cfg["seed"] * 100 + 99, 1, 1, H, blk)
     gs = synthetic.scores_zipf(cfg["seed"] * 100 + 99, 1, blk)
     q = synthetic.f16_bits(synthetic.queries(cfg["seed"], 1, Hq)[:, :G])
-    base = (oc.hi_count, oc.lo_count, oc.n_tokens)
-    rh, rl = oracle.record_bytes(0, cfg["L_hi"]), oracle.record_bytes(0, cfg["L_lo"])
+    counts = (oc.hi_count, oc.lo_count, oc.n_tokens)
+    rh, rl = oracle.record_bytes(base, cfg["L_hi"]), oracle.record_bytes(base, cfg["L_lo"])
     per_step = ((n_high + nh_b) * rh + (T - n_high + blk - nh_b) * rl + G * 128 * 6
                 + blk * 2 * 128 * 2 + nh_b * rh + (blk - nh_b) * rl + blk * 4)
     steps, t_start = 0, time.perf_counter()
     while True:
-        oc.hi_count, oc.lo_count, oc.n_tokens = base
+        oc.hi_count, oc.lo_count, oc.n_tokens = counts
         oc.stage_k[0, 0, 0, :blk] = synthetic.f16_bits(gk[0, 0, 0])
         oc.stage_v[0, 0, 0, :blk] = synthetic.f16_bits(gv[0, 0, 0])
         oc.stage_score[0, :blk] = gs[0]
@@ -374,9 +499,9 @@ def oracle_sample(cfg, budget_s: float, max_steps: int | None = None):
         el = time.perf_counter() - t_start
         if (max_steps is not None and steps >= max_steps) or (max_steps is None and el >= budget_s):
             break
-    sample = (f"1 of {cfg['B'] * H} (sequence, KV head) pairs at full {T}-token context: "
-              f"append one {blk}-token block + fp64 decode attention for its {G} query heads, "
-              f"x{steps} repetitions")
+    sample = (f"1 of {cfg['B'] * H} (sequence, KV head) pairs, 1 of {cfg['NL']} layers, at "
+              f"full {T}-token context: append one {blk}-token block + fp64 decode attention "
+              f"for its {G} query heads, x{steps} repetitions")
     return per_step * steps / el / 1e9, sample, steps, el
 
 
@@ -400,8 +525,9 @@ def main():
     config = {"workload": cfg["desc"], "batch": cfg["B"], "context": cfg["T"],
               "layers": cfg["NL"], "kv_heads": cfg["H"], "q_heads": cfg["Hq"],
               "levels": [cfg["L_hi"], cfg["L_lo"]], "r": f"{cfg['r'][0]}/{cfg['r'][1]}",
-              "block": cfg["block"], "l2": "inputs larger than L2 (records read per step > 129 MB)"
-              if cfg["B"] * cfg["T"] >= 100000 else "fits L2"}
+              "block": cfg["block"], "base": "TQ-MSE" if cfg["base"] == 1 else "affine",
+              "step": "one generated token staged per step, block append every 128 steps"
+              if cfg["mode"] == "token" else "append one 128-token block + decode every layer"}
 
     if args.impl == "reference":
         if rank != 0:
@@ -429,6 +555,8 @@ def main():
         dist.destroy_process_group()
     if rank != 0:
         return
+    config["l2"] = ("flushed between timed steps (512 MB write, outside the events)" if r["flush"]
+                    else "inputs larger than L2 (records read per step > 2 x 129 MB)")
     step_s = r["elapsed"] / args.steps
     step_bytes = r["dec_bytes"] + r["app_bytes"]
     dec_mean = sum(r["dec_times"]) / len(r["dec_times"])
@@ -451,9 +579,7 @@ def main():
                      "peak_kind": f"{peak_kind} hbm_gbs"},
         "e2e": {"value": job_gbs(step_bytes, world, r["e2e_time"]), "unit": "GB/s",
                 "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
-        # per step: the block append (rank, slot->token scatter, quantize) and the
-        # decode (pool kernel, combine); the stage is empty when decode runs
-        "gpu_launches": 5 * args.steps,
+        "gpu_launches": int(round(r["launches"])),
         "clocks": r["clocks"],
         "device_error": r["err"],
     }

@@ -2,7 +2,9 @@
 // Algorithm 2): is_high marks the n_high largest scores of a sequence, ties going to
 // the lower token index; slot is each token's position in its pool.
 //
-// One 1024-thread CTA per sequence.  Scores become order-preserving 32-bit keys
+// One 1024-thread CTA per sequence.  Sequences of at most 1024 tokens (the blocks of
+// Algorithm 2) take a single pass: each thread counts the keys ahead of its own.
+// Longer ones: scores become order-preserving 32-bit keys
 // (NaN -> 0, below every number; -0 -> +0).  A 4-pass MSB-first radix select over
 // 8-bit digits finds theta, the key of the n_high-th largest score, and `need`, how
 // many keys equal to theta are taken (the earliest ones).  One sweep with a block
@@ -54,6 +56,39 @@ __device__ __forceinline__ uint64_t block_exclusive_scan(uint64_t v, uint64_t* w
   const uint64_t r = before_warp + x - v;
   __syncthreads();  // warp_sums is reused by the next call
   return r;
+}
+
+// Short sequences (T <= 1024, e.g. a block of Algorithm 2): thread i counts the keys
+// that precede token i in the (key desc, index asc) order -- its rank -- by comparing
+// against all T keys in shared memory; is_high = rank < n_high, and the slot is the
+// count of earlier tokens of the same class (a block scan of the flags).
+__global__ void __launch_bounds__(kThreads) rank_small_kernel(RankArgs a) {
+  __shared__ uint32_t keys[kThreads];
+  __shared__ uint32_t warp_hi[32];
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int T = a.T;
+  const float* s = a.scores + (int64_t)b * a.ld;
+  const uint32_t mine = tid < T ? order_key(s[tid]) : 0u;
+  keys[tid] = mine;
+  __syncthreads();
+  uint32_t rank = 0;
+  if (tid < T) {
+    for (int j = 0; j < T; ++j) {
+      const uint32_t kj = keys[j];
+      rank += (kj > mine || (kj == mine && j < tid)) ? 1u : 0u;
+    }
+  }
+  const bool hi = tid < T && rank < a.n_high;
+  // exclusive count of earlier high tokens
+  const uint32_t bal = __ballot_sync(0xffffffffu, hi);
+  if (lane == 0) warp_hi[warp] = __popc(bal);
+  __syncthreads();
+  uint32_t before = __popc(bal & ((1u << lane) - 1u));
+  for (int w = 0; w < warp; ++w) before += warp_hi[w];
+  if (tid < T) {
+    a.is_high[(int64_t)b * T + tid] = hi ? 1 : 0;
+    a.slot[(int64_t)b * T + tid] = hi ? before : (uint32_t)tid - before;
+  }
 }
 
 __global__ void __launch_bounds__(kThreads) rank_assign_kernel(RankArgs a) {
@@ -254,7 +289,10 @@ size_t rank_workspace_words(int B, int T) { return (size_t)B * 4 * (size_t)T; }
 
 cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream) {
   if (a.B == 0 || a.T == 0) return cudaSuccess;
-  rank_assign_kernel<<<a.B, kThreads, 0, stream>>>(a);
+  if (a.T <= kThreads)
+    rank_small_kernel<<<a.B, kThreads, 0, stream>>>(a);
+  else
+    rank_assign_kernel<<<a.B, kThreads, 0, stream>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || !a.rank) return e;
   rank_sort_kernel<<<a.B, kThreads, 0, stream>>>(a, a.ws);
