@@ -329,18 +329,27 @@ __device__ __forceinline__ void k_quarter(const Window& w, uint32_t (&f)[8][2]) 
 
 // q coefficient of F slot p (lo or hi half) of quarter t for one head: the digit k
 // weight minus the share of digit k+1 that F_k carries
-template <int L>
-__device__ __forceinline__ float k_coef(const uint16_t* qrow, int t, int p, int half) {
+__device__ __forceinline__ float qval(const uint16_t* qrow, int d) { return f16_to_f32(qrow[d]); }
+__device__ __forceinline__ float qval(const float* qrow, int d) { return qrow[d]; }
+template <int L, typename QT>
+__device__ __forceinline__ float k_coef(const QT* qrow, int t, int p, int half) {
   using D = Dec<L>;
   using F = typename D::F;
   const int base = 32 * t;
   if (F::R > 0 && p == 15)
-    return half == 0 ? f16_to_f32(qrow[base + 30]) - (float)L * f16_to_f32(qrow[base + 31])
-                     : f16_to_f32(qrow[base + 31]);
+    return half == 0 ? qval(qrow, base + 30) - (float)L * qval(qrow, base + 31)
+                     : qval(qrow, base + 31);
   const int s = p / D::G + (half ? D::kHalf : 0), k = p % D::G;
   const int d = base + s * D::G + k;
-  return D::chained(k) ? f16_to_f32(qrow[d]) - (float)L * f16_to_f32(qrow[d + 1])
-                       : f16_to_f32(qrow[d]);
+  return D::chained(k) ? qval(qrow, d) - (float)L * qval(qrow, d + 1) : qval(qrow, d);
+}
+// (2c - 3)^3 of both fp16 halves (c a code of four levels)
+__device__ __forceinline__ uint32_t cube_phi(uint32_t c) {
+  uint32_t f, f2, f3;
+  asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(f) : "r"(c), "r"(0x40004000u), "r"(0xC200C200u));
+  asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(f2) : "r"(f), "r"(f));
+  asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(f3) : "r"(f2), "r"(f));
+  return f3;
 }
 
 // V side: lane group g holds half hh of quarter qv for two tokens at once (the two
@@ -427,8 +436,9 @@ struct Shared {
   uint16_t q[8][128];       // the group's query heads (rows >= G are zero)
   float qr[8][128];         // TQ base: rotated queries q' = H S q
   float cb[2][8];           // TQ base: centroids of the high / low level count
-  float sumq[8];            // sum over dims of each head's q
-  float qmax[8];            // max |q_d| of each head
+  float sumq[8];            // sum over dims of each head's q (q' for TQ records)
+  float qmax[8];            // max |q_d| of each head (q' for TQ records)
+  float cdec[2][3];         // TQ tensor path, per pool: centroids as cz + cs c (+ c3 phi^3)
   uint64_t bar[kWarps][kStages];
 };
 
@@ -446,15 +456,22 @@ struct Shared {
 //   (PACKED: columns 0..3 hi and 4..7 lo of heads 0..3; else two passes).
 // Codes enter as exact fp16 integers; the partners' power-of-two scales keep every
 // operand within the fp16 range.
-template <int L, bool PACKED>
+// CODEC 0: affine records [K][V][Ks Kz Vs Vz], rows z + s c against q.
+// CODEC 1: TQ records [K][V][Kn Vn] whose centroids are linear in the code (two or
+//   three levels, the codebook symmetric): cb[c] = cz + cs c, so the rows (n/128) cb[c]
+//   are affine rows with s = cs n/128, z = cz n/128, taken against q' = H S q.
+// CODEC 2: TQ, four levels: cb[c] = alpha phi + beta phi^3 with phi = 2c - 3; the phi
+//   part as CODEC 1 (cs = 2 alpha, cz = -3 alpha) plus a second pass on phi^3 (beta).
 // ring_it: tiles this warp has already taken through its ring (kept across calls so
 // the stage and barrier phase of each tile continue from the previous call)
+template <int L, bool PACKED, int CODEC = 0>
 __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint4* aq_all,
                          uint64_t* bars, const uint8_t* pool_bh, int64_t count, int t_begin,
-                         int t_end, int G, WarpState& st, int& ring_it) {
+                         int t_end, int G, WarpState& st, int& ring_it, int which = 0) {
   using D = Dec<L>;
   using F = typename D::F;
-  constexpr int kRec = 2 * F::RB + 8;
+  static_assert(CODEC != 2 || L == 4, "the cubic decomposition is for four levels");
+  constexpr int kRec = 2 * F::RB + (CODEC == 0 ? 8 : 4);
   constexpr uint32_t kTileBytes = kTile * kRec;
   static_assert(kTileBytes % 16 == 0, "tile size must be a multiple of 16 bytes");
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -483,8 +500,13 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
       const int p = 2 * j + i;
       float c0 = 0.0f, c1 = 0.0f;
       if (live && !upper) {
-        c0 = k_coef<L>(sh.q[g], t, p, 0) * qscale;
-        c1 = k_coef<L>(sh.q[g], t, p, 1) * qscale;
+        if constexpr (CODEC == 0) {
+          c0 = k_coef<L>(sh.q[g], t, p, 0) * qscale;
+          c1 = k_coef<L>(sh.q[g], t, p, 1) * qscale;
+        } else {
+          c0 = k_coef<L>(sh.qr[g], t, p, 0) * qscale;
+          c1 = k_coef<L>(sh.qr[g], t, p, 1) * qscale;
+        }
       }
       split_h2(c0, c1, r[2 * i], r[2 * i + 1]);
     }
@@ -493,6 +515,10 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
   __syncthreads();  // every warp of the CTA runs this pool with the same level count
   const float cS = a.scale_log2 / qscale;   // logit weight of s_k * S
   const float cZ = a.scale_log2 * sh.sumq[hd];  // logit weight of z_k
+  // TQ: row parameters per unit norm (the record holds n as fp16; rows are n/128 cb[c])
+  const float tq_s = CODEC ? sh.cdec[which][0] * (1.0f / 128.0f) : 0.0f;
+  const float tq_z = CODEC ? sh.cdec[which][1] * (1.0f / 128.0f) : 0.0f;
+  const float tq_3 = CODEC == 2 ? sh.cdec[which][2] * (1.0f / 128.0f) : 0.0f;
   // O columns 2t, 2t+1 belong to these heads (their e lives in lane 4*head)
   const int oh0 = PACKED ? ((2 * t) & 3) : 2 * t, oh1 = oh0 + 1;
 
@@ -527,8 +553,9 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
     const uint8_t* tb = my_ring + stage * kStageBytes;
     const int nvalid = min(kTile, count32 - tile * kTile);
 
-    // ---- S = Q' F^T, tokens 0..7 and 8..15
+    // ---- S = Q' F^T, tokens 0..7 and 8..15 (and the phi^3 pass for CODEC 2)
     float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+    float c0[4] = {0.f, 0.f, 0.f, 0.f}, c1[4] = {0.f, 0.f, 0.f, 0.f};
     {
       uint32_t f0[8][2], f1[8][2];
       k_quarter<L>(load_window(tb + g * kRec, t * F::QB), f0);
@@ -538,19 +565,29 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
         const uint4 A = aq[32 * j];
         mma16816(s0, A.x, A.y, A.z, A.w, f0[j][0], f0[j][1]);
         mma16816(s1, A.x, A.y, A.z, A.w, f1[j][0], f1[j][1]);
+        if constexpr (CODEC == 2) {
+          mma16816(c0, A.x, A.y, A.z, A.w, cube_phi(f0[j][0]), cube_phi(f0[j][1]));
+          mma16816(c1, A.x, A.y, A.z, A.w, cube_phi(f1[j][0]), cube_phi(f1[j][1]));
+        }
       }
     }
     // ---- logits of head hd (hi + lo rows).  G > 4: lane (g, t) takes tokens 2t, 2t+1,
     // 2t+8, 2t+9 of head g.  G <= 4 (rows 4..7 empty): lane g < 4 keeps tokens 2t, 2t+1
     // and hands 2t+8, 2t+9 to lane g + 4, which works for the same head.
     constexpr int NT = PACKED ? 2 : 4;
-    float S[NT];
+    float S[NT], S3[NT];
     int tk[NT];
     if constexpr (PACKED) {
       const float r0 = __shfl_xor_sync(0xffffffffu, s1[0] + s1[2], 16);
       const float r1 = __shfl_xor_sync(0xffffffffu, s1[1] + s1[3], 16);
       S[0] = upper ? r0 : s0[0] + s0[2];
       S[1] = upper ? r1 : s0[1] + s0[3];
+      if constexpr (CODEC == 2) {
+        const float u0 = __shfl_xor_sync(0xffffffffu, c1[0] + c1[2], 16);
+        const float u1 = __shfl_xor_sync(0xffffffffu, c1[1] + c1[3], 16);
+        S3[0] = upper ? u0 : c0[0] + c0[2];
+        S3[1] = upper ? u1 : c0[1] + c0[3];
+      }
       tk[0] = 2 * t + (upper ? 8 : 0);
       tk[1] = tk[0] + 1;
     } else {
@@ -558,34 +595,57 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
       S[1] = s0[1] + s0[3];
       S[2] = s1[0] + s1[2];
       S[3] = s1[1] + s1[3];
+      if constexpr (CODEC == 2) {
+        S3[0] = c0[0] + c0[2];
+        S3[1] = c0[1] + c0[3];
+        S3[2] = c1[0] + c1[2];
+        S3[3] = c1[1] + c1[3];
+      }
       tk[0] = 2 * t;
       tk[1] = 2 * t + 1;
       tk[2] = 2 * t + 8;
       tk[3] = 2 * t + 9;
     }
-    float lg[NT], sv[NT], zv[NT], p[NT], P[NT];
+    float lg[NT], sv[NT], zv[NT], s3v[NT], p[NT], P[NT];
     bool valid[NT];
     bool bad = false;
 #pragma unroll
     for (int i = 0; i < NT; ++i) {
       const uint32_t* prm = reinterpret_cast<const uint32_t*>(tb + tk[i] * kRec + 2 * F::RB);
-      const uint32_t kp = prm[0], vp = prm[1];
-      const float sk = f16_to_f32((uint16_t)(kp & 0xFFFF)), zk = f16_to_f32((uint16_t)(kp >> 16));
       valid[i] = live && tk[i] < nvalid;
-      // rows past the pool's count are not data: keep whatever they hold out of the sums
-      sv[i] = valid[i] ? f16_to_f32((uint16_t)(vp & 0xFFFF)) : 0.0f;
-      zv[i] = valid[i] ? f16_to_f32((uint16_t)(vp >> 16)) : 0.0f;
-      lg[i] = fmaf(sk * cS, S[i], zk * cZ);
+      float sk, zk;
+      if constexpr (CODEC == 0) {
+        const uint32_t kp = prm[0], vp = prm[1];
+        sk = f16_to_f32((uint16_t)(kp & 0xFFFF));
+        zk = f16_to_f32((uint16_t)(kp >> 16));
+        // rows past the pool's count are not data: keep whatever they hold out of the sums
+        sv[i] = valid[i] ? f16_to_f32((uint16_t)(vp & 0xFFFF)) : 0.0f;
+        zv[i] = valid[i] ? f16_to_f32((uint16_t)(vp >> 16)) : 0.0f;
+        lg[i] = fmaf(sk * cS, S[i], zk * cZ);
+      } else {
+        const uint32_t nn = prm[0];
+        const float nk = f16_to_f32((uint16_t)(nn & 0xFFFF));
+        const float nv = valid[i] ? f16_to_f32((uint16_t)(nn >> 16)) : 0.0f;
+        sk = tq_s * nk;
+        zk = tq_z * nk;
+        sv[i] = tq_s * nv;
+        zv[i] = tq_z * nv;
+        lg[i] = fmaf(sk * cS, S[i], zk * cZ);
+        if constexpr (CODEC == 2) {
+          lg[i] = fmaf(tq_3 * nk * cS, S3[i], lg[i]);
+          s3v[i] = tq_3 * nv;
+        }
+      }
       p[i] = valid[i] ? ex2(lg[i] - st.e) : 0.0f;
       P[i] = p[i] * sv[i];
-      bad |= !(p[i] <= 16384.0f) || !(P[i] <= 16384.0f);
+      bad |= !(p[i] <= 16384.0f) || !(fabsf(P[i]) <= 16384.0f);
     }
     if (__any_sync(0xffffffffu, bad)) {
       // move e up to (max over the head's tokens of logit + log2 max(s_v, 1)) - 12
       float mx = -INFINITY;
 #pragma unroll
       for (int i = 0; i < NT; ++i)
-        if (valid[i]) mx = fmaxf(mx, lg[i] + fmaxf(0.0f, __log2f(sv[i])));
+        if (valid[i]) mx = fmaxf(mx, lg[i] + fmaxf(0.0f, __log2f(fabsf(sv[i]))));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
       if (PACKED) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
@@ -639,6 +699,30 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
         mma16816(st.O[m], VA[m][0], VA[m][1], VA[m][2], VA[m][3], b0, b1);
         if constexpr (!PACKED)
           mma16816(st.O[m], VA[m][0], VA[m][1], VA[m][2], VA[m][3], b0l, b1l);
+      }
+      if constexpr (CODEC == 2) {
+        // the phi^3 pass: the same digits cubed, weighted by P3 = p * beta n / 128
+        uint32_t e0, e1, e0l = 0u, e1l = 0u;
+        float P3[NT];
+#pragma unroll
+        for (int i = 0; i < NT; ++i) P3[i] = p[i] * s3v[i];
+        if constexpr (PACKED) {
+          uint32_t hi, lo;
+          split_h2(P3[0], P3[1], hi, lo);
+          const uint32_t recv = __shfl_xor_sync(0xffffffffu, upper ? hi : lo, 16);
+          e0 = upper ? recv : hi;
+          e1 = upper ? lo : recv;
+        } else {
+          split_h2(P3[0], P3[1], e0, e0l);
+          split_h2(P3[2], P3[3], e1, e1l);
+        }
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+          const uint32_t x0 = cube_phi(VA[m][0]), x1 = cube_phi(VA[m][1]);
+          const uint32_t x2 = cube_phi(VA[m][2]), x3 = cube_phi(VA[m][3]);
+          mma16816(st.O[m], x0, x1, x2, x3, e0, e1);
+          if constexpr (!PACKED) mma16816(st.O[m], x0, x1, x2, x3, e0l, e1l);
+        }
       }
     }
     __syncwarp();
@@ -976,7 +1060,8 @@ __device__ void affine_rows(WarpState& st, int L, int G, MergeArea& mg, float* m
 
 // Merge the warps' rows into one partial (m, l, o) per head and write it.  kind 0:
 // affine pool rows (sum p' c; plus sum p z; lo rows folded for G <= 4); 1: TQ rows
-// (rotated back); 2: staged rows (plain sums).
+// from the CUDA-core path (rotated back); 2: staged rows (plain sums); 3: TQ rows from
+// the tensor-core path (as kind 0, then rotated back).
 __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeArea& mg,
                             float* merge_o, float* part) {
   __syncthreads();
@@ -1010,14 +1095,15 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
       const float sc = mg.scale[w * 8 + qh];
       if (sc != 0.0f) {
         float v = merge_o[(w * 8 + qh) * 128 + d];
-        if (kind == 0 && G <= 4) v += merge_o[(w * 8 + qh + 4) * 128 + d];
+        if ((kind == 0 || kind == 3) && G <= 4) v += merge_o[(w * 8 + qh + 4) * 128 + d];
         o += sc * v;
       }
     }
-    merged[qh * 128 + d] = kind == 0 ? o + mg.cta_z[qh] : o;
+    merged[qh * 128 + d] = (kind == 0 || kind == 3) ? o + mg.cta_z[qh] : o;
   }
   __syncthreads();
-  if (kind == 1) {
+  const bool rotated = kind == 1 || kind == 3;
+  if (rotated) {
     // back from the rotated domain: o = S H o' (unnormalised transform, stages 1..64)
     for (int hs = 1; hs < 128; hs <<= 1) {
       for (int i = threadIdx.x; i < G * 64; i += kThreads) {
@@ -1031,11 +1117,11 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
       __syncthreads();
     }
   }
-  const int8_t* sg = kind == 1 ? a.signs + ((int64_t)a.layer * a.H + h) * 128 : nullptr;
+  const int8_t* sg = rotated ? a.signs + ((int64_t)a.layer * a.H + h) * 128 : nullptr;
   for (int i = threadIdx.x; i < G * 128; i += kThreads) {
     const int qh = i >> 7, d = i & 127;
     const float o = merged[qh * 128 + d];
-    part[16 + qh * 128 + d] = kind == 1 ? o * (float)sg[d] : o;
+    part[16 + qh * 128 + d] = rotated ? o * (float)sg[d] : o;
   }
   __syncthreads();  // the merge area (the ring) is free again
 }
@@ -1138,6 +1224,7 @@ __global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs
     }
   }
   load_group_q(a, sh, b, h, G);
+  __shared__ int tq_path;  // TQ: 1 when this pool's codebook takes the tensor-core path
   if (KIND == 1) {
     for (int i = threadIdx.x; i < 8 * 128; i += kThreads) {
       const int c = i >> 7, d = i & 127;
@@ -1150,6 +1237,53 @@ __global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs
     }
   }
   __syncthreads();
+  if (KIND == 1) {
+    // rotated queries: sums and maxima for the tensor-core path
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float s = 0.0f, mx = 0.0f;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float x = sh.qr[warp][4 * lane + j];
+      s += x;
+      mx = fmaxf(mx, fabsf(x));
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      s += __shfl_xor_sync(0xffffffffu, s, off);
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    }
+    if (lane == 0) {
+      sh.sumq[warp] = s;
+      sh.qmax[warp] = mx;
+    }
+    if (threadIdx.x == 0) {
+      // centroids as cz + cs c (two levels; three when equally spaced), or for four
+      // exactly symmetric levels alpha phi + beta phi^3, phi = 2c - 3
+      const int src0 = split < P.splits_hi ? 0 : 1;
+      const int L = src0 == 0 ? a.L_hi : a.L_lo;
+      const float* cb = sh.cb[src0];
+      int path = 0;
+      float cs = 0.0f, cz = 0.0f, c3 = 0.0f;
+      if (L == 2 || (L == 3 && cb[1] - cb[0] == cb[2] - cb[1])) {
+        path = 1;
+        cs = cb[1] - cb[0];
+        cz = cb[0];
+      } else if (L == 4 && cb[0] == -cb[3] && cb[1] == -cb[2]) {
+        path = 2;
+        const float beta = (cb[3] - 3.0f * cb[2]) / 24.0f;
+        const float alpha = cb[2] - beta;
+        cs = 2.0f * alpha;
+        cz = -3.0f * alpha;
+        c3 = beta;
+      }
+      sh.cdec[src0][0] = cs;
+      sh.cdec[src0][1] = cz;
+      sh.cdec[src0][2] = c3;
+      tq_path = path;
+    }
+  }
+  __syncthreads();
+  int kind = KIND;
   if constexpr (KIND == 2) {
     run_stage(a, sh, b, h, G, mg.m, mg.l, mg.z, merge_o);
   } else {
@@ -1165,22 +1299,49 @@ __global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs
     const uint8_t* pool = src == 0 ? a.hi_pool : a.lo_pool;
     const int rec = record_bytes_rt(SEMKV_BASE_TQ, L);
     const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
-    switch (L) {
+    if (tq_path) {
+      uint8_t* ring = dyn;
+      uint4* aq_all = reinterpret_cast<uint4*>(dyn + kRingBytes);
+      uint64_t* bars = &sh.bar[0][0];
+      if (threadIdx.x < kWarps * kStages) mbar_init(bars + threadIdx.x);
+      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+      WarpState st;
+      state_init(st);
+      int ring_it = 0;
+      if (L == 2) {
+        if (G <= 4) run_pool<2, true, 1>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st, ring_it, src);
+        else run_pool<2, false, 1>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st, ring_it, src);
+      } else if (L == 3) {
+        if (G <= 4) run_pool<3, true, 1>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st, ring_it, src);
+        else run_pool<3, false, 1>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st, ring_it, src);
+      } else {
+        if (G <= 4) run_pool<4, true, 2>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st, ring_it, src);
+        else run_pool<4, false, 2>(a, sh, ring, aq_all, bars, pool_bh, count, t_begin, t_end, G, st, ring_it, src);
+      }
+      affine_rows(st, L, G, mg, merge_o);
+      kind = 3;
+    } else {
+      switch (L) {
 #define SEMKV_TQ_CASE(LV) \
-      case LV: run_pool_tq<LV>(a, sh, src, pool_bh, count, t_begin, t_end, G, mg.m, mg.l, mg.z, merge_o); break;
-      SEMKV_TQ_CASE(2) SEMKV_TQ_CASE(3) SEMKV_TQ_CASE(4) SEMKV_TQ_CASE(5)
-      SEMKV_TQ_CASE(6) SEMKV_TQ_CASE(7) SEMKV_TQ_CASE(8)
+        case LV: run_pool_tq<LV>(a, sh, src, pool_bh, count, t_begin, t_end, G, mg.m, mg.l, mg.z, merge_o); break;
+        SEMKV_TQ_CASE(2) SEMKV_TQ_CASE(3) SEMKV_TQ_CASE(4) SEMKV_TQ_CASE(5)
+        SEMKV_TQ_CASE(6) SEMKV_TQ_CASE(7) SEMKV_TQ_CASE(8)
 #undef SEMKV_TQ_CASE
-      default: break;
+        default: break;
+      }
     }
   }
-  merge_warps(a, KIND, h, G, mg, merge_o, a.partials + (bh * P.stride + split) * kPartialFloats);
+  merge_warps(a, kind, h, G, mg, merge_o, a.partials + (bh * P.stride + split) * kPartialFloats);
 }
 
-// merge the splits of each (b, qh): one warp per head, 4 dims per lane
+// merge the partials of each (b, qh): one warp per head, 4 dims per lane.  The lanes
+// first take the partials' maxima and weights in parallel (weights kept in shared
+// memory), then sum the rows with independent loads.
 __global__ void combine_kernel(DecodeArgs a) {
-  const int lane = threadIdx.x & 31;
-  const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  constexpr int kHeadsPerCta = 8;
+  __shared__ float wsm[kHeadsPerCta][kMaxPartialsPerPair];
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  const int gw = blockIdx.x * kHeadsPerCta + wib;
   if (gw >= a.B * a.Hq) return;
   const int b = gw / a.Hq, qh = gw % a.Hq;
   const int G = a.Hq / a.H, h = qh / G, c = qh % G;
@@ -1188,21 +1349,29 @@ __global__ void combine_kernel(DecodeArgs a) {
   const int S = pair_partials(a.plan, bh);
   const float* base = a.partials + bh * a.plan.stride * kPartialFloats;
   float M = -INFINITY;
-  for (int s = 0; s < S; ++s) M = fmaxf(M, base[s * kPartialFloats + c]);
-  float o[4] = {0.f, 0.f, 0.f, 0.f}, lsum = 0.0f;
-  if (M != -INFINITY) {
-    for (int s = 0; s < S; ++s) {
-      const float* p = base + s * kPartialFloats;
-      const float ms = p[c];
-      if (ms == -INFINITY) continue;
-      const float sc = exp2f(ms - M);
-      lsum += sc * p[8 + c];
-      const float4 v = *reinterpret_cast<const float4*>(p + 16 + c * 128 + 4 * lane);
-      o[0] += sc * v.x;
-      o[1] += sc * v.y;
-      o[2] += sc * v.z;
-      o[3] += sc * v.w;
-    }
+  for (int s = lane; s < S; s += 32) M = fmaxf(M, base[s * kPartialFloats + c]);
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+  float lsum = 0.0f;
+  for (int s = lane; s < S; s += 32) {
+    const float ms = base[s * kPartialFloats + c];
+    const float sc = (M == -INFINITY || ms == -INFINITY) ? 0.0f : exp2f(ms - M);
+    wsm[wib][s] = sc;
+    lsum += sc * base[s * kPartialFloats + 8 + c];
+  }
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
+  __syncwarp();
+  float o[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+  for (int s = 0; s < S; ++s) {
+    const float sc = wsm[wib][s];
+    if (sc == 0.0f) continue;
+    const float4 v = *reinterpret_cast<const float4*>(base + s * kPartialFloats + 16 + c * 128 + 4 * lane);
+    o[0] += sc * v.x;
+    o[1] += sc * v.y;
+    o[2] += sc * v.z;
+    o[3] += sc * v.w;
   }
   const float inv = 1.0f / lsum;
   float4 r = make_float4(o[0] * inv, o[1] * inv, o[2] * inv, o[3] * inv);
@@ -1341,7 +1510,7 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
                                          kRingBytes + kAqBytes);
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               kRingBytes);
+                               kRingBytes + kAqBytes);
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(decode_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                kRingBytes);
@@ -1358,7 +1527,7 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     const int pool_splits = P.splits_hi + P.splits_lo;
     if (pool_splits > 0)
-      decode_kernel<1><<<dim3(pool_splits, a.H, a.B), kThreads, kRingBytes, stream>>>(a);
+      decode_kernel<1><<<dim3(pool_splits, a.H, a.B), kThreads, kRingBytes + kAqBytes, stream>>>(a);
   } else if (P.ctas > 0) {
     decode_affine_kernel<<<P.ctas, kThreads, kRingBytes + kAqBytes, stream>>>(a);
   }
