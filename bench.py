@@ -240,6 +240,31 @@ def append_bytes(cfg, desc):
     return B * NL * H * (blk * 2 * 128 * 2 + nh_b * rh + (blk - nh_b) * rl) + B * blk * 4
 
 
+def pre_decode_work(k, cache, blk, token_mode, base_counts, r_num, r_den, desc,
+                    blocks_k, blocks_v, blocks_s, nblocks, semkv):
+    """The host and device work of step k that precedes its decode calls: staging and,
+    when due, the block append (with the appended slots rewound first)."""
+    if not token_mode:
+        j = k % nblocks
+        cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+        cache.stage_k.copy_(blocks_k[:, :, :, j * blk:(j + 1) * blk])
+        cache.stage_v.copy_(blocks_v[:, :, :, j * blk:(j + 1) * blk])
+        cache.stage_score.copy_(blocks_s[:, j * blk:(j + 1) * blk])
+        cache.s.stage_n = blk
+        semkv.semkv_append_block(desc, cache, r_num, r_den)
+    else:
+        n = cache.s.stage_n
+        if n == 0:
+            cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+        j = k % (nblocks * blk)
+        cache.stage_k[:, :, :, n].copy_(blocks_k[:, :, :, j])
+        cache.stage_v[:, :, :, n].copy_(blocks_v[:, :, :, j])
+        cache.stage_score[:, n].copy_(blocks_s[:, j])
+        cache.s.stage_n = n + 1
+        if cache.s.stage_n == blk:
+            semkv.semkv_append_block(desc, cache, r_num, r_den)
+
+
 def gpu_arm(args, cfg, rank, world):
     import torch
     from paper_2608_28911_gb300 import semkv
@@ -300,34 +325,23 @@ def gpu_arm(args, cfg, rank, world):
         if ev is not None:
             ev[1].record(stream)
 
+    def q_for(i):
+        return q_all[(i // blk) % nblocks] if token_mode else q_all[i % nblocks]
+
+    def step(i, ev=None):
+        pre_decode(i)
+        decode_all(q_for(i), ev)
+
+    def pre_decode(i):
+        pre_decode_work(i, cache, blk, token_mode, base_counts, r_num, r_den, desc,
+                        blocks_k, blocks_v, blocks_s, nblocks, semkv)
+
     if not token_mode:
-        def step(i, ev=None):
-            j = i % nblocks
-            cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
-            cache.stage_k.copy_(blocks_k[:, :, :, j * blk:(j + 1) * blk])
-            cache.stage_v.copy_(blocks_v[:, :, :, j * blk:(j + 1) * blk])
-            cache.stage_score.copy_(blocks_s[:, j * blk:(j + 1) * blk])
-            cache.s.stage_n = blk
-            semkv.semkv_append_block(desc, cache, r_num, r_den)
-            decode_all(q_all[j], ev)
         dec_bytes = NL * decode_bytes(cfg, desc, base_counts[0] + nh_b,
                                       base_counts[1] + blk - nh_b, 0)
         app_bytes = append_bytes(cfg, desc)
         launches_per_step = app_launch + NL * dec_launch
     else:
-        def step(i, ev=None):
-            # one generated token: stage it; append the block when the stage is full
-            n = cache.s.stage_n
-            if n == 0:
-                cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
-            j = i % (nblocks * blk)
-            cache.stage_k[:, :, :, n].copy_(blocks_k[:, :, :, j])
-            cache.stage_v[:, :, :, n].copy_(blocks_v[:, :, :, j])
-            cache.stage_score[:, n].copy_(blocks_s[:, j])
-            cache.s.stage_n = n + 1
-            if cache.s.stage_n == blk:
-                semkv.semkv_append_block(desc, cache, r_num, r_den)
-            decode_all(q_all[(i // blk) % nblocks], ev)
         # over a cycle of blk steps: stages 1..blk-1 hold that many fp16 rows, the
         # last step decodes the appended block from the pools
         cyc = sum(decode_bytes(cfg, desc, base_counts[0], base_counts[1], n) for n in range(1, blk))
@@ -345,6 +359,35 @@ def gpu_arm(args, cfg, rank, world):
         while cache.s.stage_n != 0:
             step(0)
     torch.cuda.synchronize()
+
+    if args.graph:
+        # replay each distinct step from CUDA graphs, as a serving loop would: the same
+        # kernels on the same data without the per-call host work.  Captured in step
+        # order, so the host-side counts evolve exactly as in the direct calls; the
+        # pre-decode part and the decode part are separate graphs so events can time
+        # the decode between them.
+        n_distinct = blk if token_mode else nblocks
+        parts = []
+        for k in range(n_distinct):
+            ga, gd = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+            with torch.cuda.graph(ga):
+                pre_decode(k)
+            with torch.cuda.graph(gd):
+                decode_all(q_for(k))
+            parts.append((ga, gd))
+        torch.cuda.synchronize()
+
+        def step(i, ev=None, _parts=parts):   # noqa: F811 (the graph replay of the step)
+            ga, gd = _parts[i % len(_parts)]
+            ga.replay()
+            if ev is not None:
+                ev[0].record(stream)
+            gd.replay()
+            if ev is not None:
+                ev[1].record(stream)
+        for i in range(args.warmup):
+            step(i)
+        torch.cuda.synchronize()
 
     def barrier():
         if world > 1:
@@ -515,6 +558,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="b16x64k", choices=sorted(CONFIGS))
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--graph", action=argparse.BooleanOptionalAction, default=True,
+                    help="replay the device-resident steps from CUDA graphs (the e2e steps "
+                         "always call the API directly)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
