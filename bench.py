@@ -296,6 +296,19 @@ def gpu_arm(args, cfg, rank, world):
     rl = semkv.semkv_record_bytes(desc.base, desc.levels_lo)
     q_bytes = B * NL * H * (T * 2 * 128 * 2 + w["n_high"] * rh + (T - w["n_high"]) * rl) + B * T * 4
     quantize_gbs = q_bytes / statistics.median(qt) / 1e9
+    # the value-norm indicator over the prompt's V cache (Sec. 3.3), the cheapest scorer
+    vn = torch.empty((B, T), dtype=torch.float32, device=dev)
+    st_ = []
+    for it in range(4):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        semkv.semkv_score_kv_norm(w["v"], vn)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if it > 0:
+            st_.append(e0.elapsed_time(e1) * 1e-3)
+    score_gbs = (B * NL * H * T * 128 * 2 + B * T * 4) / statistics.median(st_) / 1e9
     del w["k"], w["v"]
     torch.cuda.empty_cache()
 
@@ -490,7 +503,8 @@ def gpu_arm(args, cfg, rank, world):
 
     elapsed, e2e_time = max_over_ranks([elapsed, e2e_time], device=dev)
     return dict(elapsed=elapsed, dec_times=dec_times, dec_bytes=dec_bytes, app_bytes=app_bytes,
-                quantize_gbs=quantize_gbs, clocks=clk.summary(), err=err, e2e_time=e2e_time,
+                quantize_gbs=quantize_gbs, score_gbs=score_gbs, clocks=clk.summary(), err=err,
+                e2e_time=e2e_time,
                 h2d=h2d, d2h=d2h, flush=flush, launches=launches_per_step * args.steps)
 
 
@@ -619,6 +633,7 @@ def main():
         "decode_frac_of_peak": achieved / peak,
         "decode_frac_of_nominal_8tbs": achieved / 8000.0,
         "quantize_gbs": r["quantize_gbs"],
+        "value_norm_score_gbs": r["score_gbs"],
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": profiled_traffic(args.config),
                      "kernel": "decode_kernel+combine_kernel (semkv_decode_attention)",

@@ -146,6 +146,21 @@ semkv_status semkv_rank_assign(const float* scores, int32_t batch, int32_t T,
                                uint32_t n_high, uint8_t* is_high, uint32_t* slot,
                                uint32_t* rank, void* ws, size_t ws_bytes, void* stream);
 
+/* KV-norm importance indicator (Sec. 3.3, "KV-norm" family: key-norm ||K_i||_2 and
+ * value-norm ||V_i||_2, the magnitude of the tensor being compressed; Sec. 4.5 finds
+ * value-norm the cheapest indicator profiled).  Writes
+ *   scores[b][t] = || x[b][l][h][t][:] ||_2 over l in [layer_begin, layer_end) and all h
+ * (a layer range restricts the score to the last m layers, as Eq. 3 does).
+ * x: device fp16 [batch][layers][kv_heads][T][128] (pass the K cache for key-norm, the V
+ * cache for value-norm), 8-byte aligned; scores: device f32 [batch][T], 4-byte aligned,
+ * both caller-owned.  The summation order is fixed (per dim group of 4, row by row, then
+ * a pairwise tree over the 32 groups), so equal inputs give bit-identical scores.
+ * The scores feed semkv_rank_assign directly (only their ranking matters).
+ * Errors: SEMKV_EINVAL (null pointers, empty or inverted ranges), SEMKV_EALIGN. */
+semkv_status semkv_score_kv_norm(const uint16_t* x, int32_t batch, int32_t layers,
+                                 int32_t kv_heads, int32_t T, int32_t layer_begin,
+                                 int32_t layer_end, float* scores, void* stream);
+
 /* Token-wise quantization, Eq. 7 / Algorithm 1: quantize every row of the prompt
  * K/V with Q_{b_i} and write token i's record (for every layer and KV head) to
  * slot[b][i] of the high pool if is_high[b][i] else of the low pool; writes

@@ -63,6 +63,7 @@ def lib():
                                           p, p]
         L.orc_quantize_tokens.restype = i32
         L.orc_dequant_records.argtypes = [i32, i32, p, i64, p, p, p, p]
+        L.orc_score_kv_norm.argtypes = [p, i32, i32, i32, i32, i32, i32, p]
         _lib = L
     return _lib
 
@@ -446,3 +447,20 @@ def effective_bits(base: int, L_hi: int, L_lo: int, r: float) -> float:
 def layout_bytes_per_token_head(base: int, L_hi: int, L_lo: int, n_high: int, T: int) -> int:
     """Bytes of this build's records (K and V of one KV head) for T tokens."""
     return n_high * record_bytes(base, L_hi) + (T - n_high) * record_bytes(base, L_lo)
+
+
+# ------------------------------------------- KV-norm indicator (Sec. 3.3) -----
+
+def score_kv_norm(x_f16bits, layer_begin: int = 0, layer_end: int | None = None):
+    """Key-norm / value-norm importance score of each token (Sec. 3.3, KV-norm family):
+    ||x_{b,t}||_2 over layers [layer_begin, layer_end) and every KV head of the fp16
+    K or V cache x [B][NL][H][T][128] (bit patterns), in the fixed summation order of
+    orc_score_kv_norm.  Returns float32 [B][T]."""
+    x = np.ascontiguousarray(x_f16bits, dtype=np.uint16)
+    B, NL, H, T, d = x.shape
+    assert d == D
+    le = NL if layer_end is None else layer_end
+    assert 0 <= layer_begin < le <= NL
+    out = np.zeros((B, T), np.float32)
+    lib().orc_score_kv_norm(_ptr(x), B, NL, H, T, layer_begin, le, _ptr(out))
+    return out

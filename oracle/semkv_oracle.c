@@ -17,6 +17,8 @@
  *  - Token-wise quantization of a whole cache into high/low pools (Eq. 7),
  *    precision broadcast over layers and KV heads (Fig. 5 caption).
  *  - Dequantization of records to exact fp64 rows (used by the fp64 attention).
+ *  - The KV-norm importance indicator (Sec. 3.3: key-norm ||K_i||_2 / value-norm
+ *    ||V_i||_2 of the tensor being compressed), in a fixed summation order.
  *
  * Floating point: build with -O2 -ffp-contract=off; every float operation below is
  * one IEEE binary32 operation rounded to nearest-even, in the order written.
@@ -426,6 +428,44 @@ void orc_dequant_records(int base, int L, const uint8_t* recs, int64_t count,
 }
 
 /* Element-wise conversions over arrays (for tests that sweep many values). */
+/* KV-norm indicator (Sec. 3.3, "KV-norm" family): token t of sequence b scores
+ * ||x_{b,t}||_2 over the rows of layers [lb, le) and every KV head, x being the K or V
+ * cache [B][NL][H][T][128] (fp16 bits).  Summation order, fixed so that equal inputs
+ * give equal scores (and hence equal rankings) everywhere: the 128 dims of a row are
+ * 32 consecutive groups of 4; group j's square sum ((x0^2 + x1^2) + x2^2) + x3^2 is
+ * added to accumulator j, rows taken layer by layer, head by head; then the 32
+ * accumulators are combined pairwise a[j] + a[j ^ o] for o = 16, 8, 4, 2, 1 (which
+ * leaves the same total in every a[j]); the score is sqrtf of that total. */
+void orc_score_kv_norm(const uint16_t* x, int B, int NL, int H, int T, int lb, int le,
+                       float* scores) {
+  for (int b = 0; b < B; b++) {
+    for (int t = 0; t < T; t++) {
+      float acc[32];
+      for (int j = 0; j < 32; j++) acc[j] = 0.0f;
+      for (int l = lb; l < le; l++) {
+        for (int h = 0; h < H; h++) {
+          const uint16_t* row = x + ((((int64_t)b * NL + l) * H + h) * T + t) * D;
+          for (int j = 0; j < 32; j++) {
+            float x0 = orc_f16_to_f32(row[4 * j]), x1 = orc_f16_to_f32(row[4 * j + 1]);
+            float x2 = orc_f16_to_f32(row[4 * j + 2]), x3 = orc_f16_to_f32(row[4 * j + 3]);
+            float sq = x0 * x0;
+            sq = sq + x1 * x1;
+            sq = sq + x2 * x2;
+            sq = sq + x3 * x3;
+            acc[j] = acc[j] + sq;
+          }
+        }
+      }
+      for (int o = 16; o >= 1; o >>= 1) {
+        float nxt[32];
+        for (int j = 0; j < 32; j++) nxt[j] = acc[j] + acc[j ^ o];
+        for (int j = 0; j < 32; j++) acc[j] = nxt[j];
+      }
+      scores[(int64_t)b * T + t] = sqrtf(acc[0]);
+    }
+  }
+}
+
 void orc_f32_to_f16_array(const float* x, uint16_t* h, int64_t n) {
   for (int64_t i = 0; i < n; i++) h[i] = orc_f32_to_f16(x[i]);
 }

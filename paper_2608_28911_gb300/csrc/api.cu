@@ -159,6 +159,24 @@ semkv_status semkv_rank_assign(const float* scores, int32_t batch, int32_t T, ui
   return from_cuda(launch_rank_assign(a, (cudaStream_t)stream));
 }
 
+semkv_status semkv_score_kv_norm(const uint16_t* x, int32_t batch, int32_t layers,
+                                 int32_t kv_heads, int32_t T, int32_t layer_begin,
+                                 int32_t layer_end, float* scores, void* stream) {
+  if (!x || !scores || batch < 1 || layers < 1 || kv_heads < 1 || T < 1) return SEMKV_EINVAL;
+  if (layer_begin < 0 || layer_end > layers || layer_begin >= layer_end) return SEMKV_EINVAL;
+  if (!aligned(x, 8) || !aligned(scores, 4)) return SEMKV_EALIGN;
+  ScoreArgs a;
+  a.x = x;
+  a.B = batch;
+  a.NL = layers;
+  a.H = kv_heads;
+  a.T = T;
+  a.lb = layer_begin;
+  a.le = layer_end;
+  a.scores = scores;
+  return from_cuda(launch_score_kv_norm(a, device_sm_count(), (cudaStream_t)stream));
+}
+
 semkv_status semkv_quantize_pack(const semkv_quant_desc* desc, const uint16_t* k,
                                  const uint16_t* v, int32_t T, const uint8_t* is_high,
                                  const uint32_t* slot, uint32_t n_high, semkv_cache* cache,

@@ -43,6 +43,14 @@ struct RankArgs {
 size_t rank_workspace_words(int B, int T);
 cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream);
 
+// KV-norm importance scores (Sec. 3.3): ||x_{b,t}|| over layers [lb, le), all heads.
+struct ScoreArgs {
+  const uint16_t* x;        // [B][NL][H][T][128] fp16
+  int B, NL, H, T, lb, le;
+  float* scores;            // [B][T]
+};
+cudaError_t launch_score_kv_norm(const ScoreArgs& a, int num_sms, cudaStream_t stream);
+
 // Decode attention over one layer of the cache (split-K + combine).
 struct DecodePlan {
   int tiles_hi, tiles_lo, tiles_st;     // 16-token tiles per (b, h) per source

@@ -74,6 +74,8 @@ def _load():
     L.semkv_rank_workspace_bytes.restype = sz
     L.semkv_rank_assign.argtypes = [p, i32, i32, u32, p, p, p, p, sz, p]
     L.semkv_rank_assign.restype = ctypes.c_int
+    L.semkv_score_kv_norm.argtypes = [p, i32, i32, i32, i32, i32, i32, p, p]
+    L.semkv_score_kv_norm.restype = ctypes.c_int
     L.semkv_quantize_pack.argtypes = [ctypes.POINTER(QuantDescStruct), p, p, i32, p, p, u32,
                                       ctypes.POINTER(CacheStruct), p]
     L.semkv_quantize_pack.restype = ctypes.c_int
@@ -98,7 +100,7 @@ def _load():
 LIB = _load()
 EXPORTED = ["semkv_row_bytes", "semkv_record_bytes", "semkv_high_count_floor",
             "semkv_block_high_count", "semkv_lloyd_max_gaussian", "semkv_rank_workspace_bytes",
-            "semkv_rank_assign", "semkv_quantize_pack", "semkv_append_block",
+            "semkv_rank_assign", "semkv_score_kv_norm", "semkv_quantize_pack", "semkv_append_block",
             "semkv_decode_workspace_bytes", "semkv_decode_attention",
             "semkv_decode_attention_noalloc", "semkv_status_string"]
 
@@ -158,6 +160,16 @@ def semkv_rank_assign(scores: torch.Tensor, n_high: int, is_high: torch.Tensor,
     _check("semkv_rank_assign",
            LIB.semkv_rank_assign(_ptr(scores), B, T, n_high, _ptr(is_high), _ptr(slot),
                                  _ptr(rank), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def semkv_score_kv_norm(x: torch.Tensor, scores: torch.Tensor, layer_begin: int = 0,
+                        layer_end=None, stream=None):
+    """KV-norm importance scores of x [B][NL][H][T][128] fp16 into scores [B][T] f32."""
+    B, NL, H, T, _ = x.shape
+    le = NL if layer_end is None else layer_end
+    _check("semkv_score_kv_norm",
+           LIB.semkv_score_kv_norm(_ptr(x), B, NL, H, T, layer_begin, le, _ptr(scores),
+                                   _stream(stream)))
 
 
 def semkv_quantize_pack(desc: "QuantDesc", k: torch.Tensor, v: torch.Tensor, is_high, slot,

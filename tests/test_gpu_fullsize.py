@@ -148,3 +148,23 @@ def test_tq_43_32k_every_record_and_head():
     got, ref = p.decode(0, 0)
     err, rel = attention_errors(got, ref)
     assert err <= ATOL and rel <= RTOL_L2, (err, rel)
+
+
+def test_value_norm_scores_batch16_64k_sampled_sequences():
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    B, T, H = 16, 65536, 8
+    dev = torch.device("cuda:0")
+    v = torch.empty((B, 1, H, T, 128), dtype=torch.float16, device=dev)
+    host = {}
+    for b in range(B):
+        _, vb = synthetic.kv(500 + b, 1, 1, H, T)
+        v[b].copy_(torch.from_numpy(vb[0]))
+        if b in (0, 9):
+            host[b] = vb
+    sc = torch.empty((B, T), dtype=torch.float32, device=dev)
+    semkv.semkv_score_kv_norm(v, sc)
+    got = sc.cpu().numpy()
+    for b, vb in host.items():
+        want = oracle.score_kv_norm(synthetic.f16_bits(vb))[0]
+        assert np.array_equal(got[b].view(np.uint32), want.view(np.uint32)), b

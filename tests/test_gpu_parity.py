@@ -188,3 +188,32 @@ def test_tq_decode_with_staged_tail():
         oracle.stage_token(p.oc, synthetic.f16_bits(k[:, :, :, g]), synthetic.f16_bits(v[:, :, :, g]),
                            s[:, g])
     check_attention(p)
+
+
+# ------------------------------------------------------ KV-norm scoring -----
+
+@pytest.mark.parametrize("B,NL,H,T,lb,le", [
+    (2, 1, 8, 1000, 0, 1),      # value-norm of one Llama-shaped layer
+    (1, 4, 2, 333, 2, 4),       # last-2-layers restriction, ragged T
+    (3, 2, 1, 17, 0, 2),
+])
+def test_score_kv_norm_bit_exact_and_ranks(B, NL, H, T, lb, le):
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    _, v = synthetic.kv(T + NL, B, NL, H, T)
+    v[0, 0, 0, 0] = 0.0                       # an all-zero row
+    d = torch.device("cuda:0")
+    vd = torch.from_numpy(v).to(d)
+    sc = torch.empty((B, T), dtype=torch.float32, device=d)
+    semkv.semkv_score_kv_norm(vd, sc, lb, le)
+    got = sc.cpu().numpy()
+    want = oracle.score_kv_norm(synthetic.f16_bits(v), lb, le)
+    assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+    # the scores drive the top-r selection: identical flags and slots follow
+    n_high = (26 * T) // 100
+    ih = torch.empty((B, T), dtype=torch.uint8, device=d)
+    sl = torch.empty((B, T), dtype=torch.int32, device=d)
+    semkv.semkv_rank_assign(sc, n_high, ih, sl)
+    o_ih, o_sl, _ = oracle.rank_assign(want, n_high)
+    assert np.array_equal(ih.cpu().numpy(), o_ih)
+    assert np.array_equal(sl.cpu().numpy().view(np.uint32), o_sl)
