@@ -146,6 +146,21 @@ semkv_status semkv_rank_assign(const float* scores, int32_t batch, int32_t T,
                                uint32_t n_high, uint8_t* is_high, uint32_t* slot,
                                uint32_t* rank, void* ws, size_t ws_bytes, void* stream);
 
+/* Fake quantization (Sec. 4.1: the quality experiments quantize, dequantize and compute
+ * in fp16).  Every row of K and V is quantized with the same arithmetic as
+ * semkv_quantize_pack at its token's level count (levels_hi where is_high[b][t], else
+ * levels_lo; is_high NULL puts every token at levels_hi, a uniform grid point) and
+ * reconstructed to fp16, in binary32 in this order:
+ *   affine: out_d = fp16( z + s * c_d )
+ *   TQ:     y = unnormalised FWHT(cb[c]) (stages 1..64);  out_d = fp16( (sign_d * y_d) * (n/128) )
+ * k, v, k_out, v_out: device fp16 [batch][layers][kv_heads][T][128], 8-byte aligned,
+ * caller-owned (outputs may not alias inputs); is_high: device u8 [batch][T] or NULL.
+ * Errors: SEMKV_EINVAL, SEMKV_EALIGN, SEMKV_EUNSUPPORTED (level counts, base). */
+semkv_status semkv_fake_quant(const semkv_quant_desc* desc, const uint16_t* k, const uint16_t* v,
+                              int32_t batch, int32_t layers, int32_t kv_heads, int32_t T,
+                              const uint8_t* is_high, uint16_t* k_out, uint16_t* v_out,
+                              void* stream);
+
 /* KV-norm importance indicator (Sec. 3.3, "KV-norm" family: key-norm ||K_i||_2 and
  * value-norm ||V_i||_2, the magnitude of the tensor being compressed; Sec. 4.5 finds
  * value-norm the cheapest indicator profiled).  Writes

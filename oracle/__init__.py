@@ -28,7 +28,7 @@ import numpy as np
 from .build import build_oracle
 
 D = 128
-BASE_AFFINE, BASE_TQ = 0, 1
+BASE_AFFINE, BASE_TQ, BASE_AFFINE_HAD = 0, 1, 2
 
 _lib = None
 
@@ -55,6 +55,10 @@ def lib():
         L.orc_unpack_row.argtypes = [p, i32, p]
         L.orc_affine_row.argtypes = [p, i32, p, p, p]
         L.orc_tq_row.argtypes = [p, p, i32, p, p, p]
+        L.orc_affine_had_row.argtypes = [p, p, i32, p, p, p]
+        L.orc_f32_to_f16_rd.argtypes = [ctypes.c_float]
+        L.orc_f32_to_f16_rd.restype = ctypes.c_uint16
+        L.orc_inv_sqrt_d.restype = ctypes.c_float
         L.orc_fwht_f32.argtypes = [p]
         L.orc_row_norm.argtypes = [p]
         L.orc_row_norm.restype = ctypes.c_float
@@ -64,6 +68,8 @@ def lib():
         L.orc_quantize_tokens.restype = i32
         L.orc_dequant_records.argtypes = [i32, i32, p, i64, p, p, p, p]
         L.orc_score_kv_norm.argtypes = [p, i32, i32, i32, i32, i32, i32, p]
+        L.orc_fake_quant.argtypes = [i32, i32, i32, p, p, i32, i32, i32, i32, p, p, p, p, p, p,
+                                     p, p]
         _lib = L
     return _lib
 
@@ -162,6 +168,28 @@ def tq_row(x_f16bits, signs, L: int, thresholds):
     n = np.zeros(1, dtype=np.uint16)
     lib().orc_tq_row(_ptr(x), _ptr(sg), L, _ptr(thr), _ptr(codes), _ptr(n))
     return codes, int(n[0])
+
+
+def affine_had_row(x_f16bits, signs, L: int):
+    """Hadamard-rotated affine row quantizer (Sec. 4.1 rotation + per-row affine).
+    Returns (codes u8[128], scale fp16 bits, offset fp16 bits)."""
+    x = np.ascontiguousarray(x_f16bits, dtype=np.uint16)
+    sg = np.ascontiguousarray(signs, dtype=np.int8)
+    codes = np.zeros(D, dtype=np.uint8)
+    s = np.zeros(1, dtype=np.uint16)
+    z = np.zeros(1, dtype=np.uint16)
+    lib().orc_affine_had_row(_ptr(x), _ptr(sg), L, _ptr(codes), _ptr(s), _ptr(z))
+    return codes, int(s[0]), int(z[0])
+
+
+def f32_to_f16_rd(x: float) -> int:
+    """binary32 -> binary16 bits rounded toward -infinity (hand-written)."""
+    return int(lib().orc_f32_to_f16_rd(float(np.float32(x))))
+
+
+def inv_sqrt_d() -> float:
+    """The binary32 constant 1/sqrt(128) of the rotated affine base."""
+    return float(lib().orc_inv_sqrt_d())
 
 
 def fwht_f32(w) -> np.ndarray:
@@ -282,7 +310,7 @@ class Cache:
     stage_v: np.ndarray = None
     stage_score: np.ndarray = None
     stage_n: int = 0
-    signs: np.ndarray = None          # [layers][kv_heads][128] int8 (TQ)
+    signs: np.ndarray = None          # [layers][kv_heads][128] int8 (TQ, rotated affine)
     cb_hi: tuple = None               # (centroids f32, thresholds f32) (TQ)
     cb_lo: tuple = None
 
@@ -436,7 +464,7 @@ def paper_code_bits(L: int) -> float:
 
 def metadata_bits(base: int) -> float:
     """fp16 metadata per value: two per 128-row for affine (0.25), one for TQ."""
-    return (2 if base == BASE_AFFINE else 1) * 16 / D
+    return (1 if base == BASE_TQ else 2) * 16 / D
 
 
 def effective_bits(base: int, L_hi: int, L_lo: int, r: float) -> float:
@@ -464,3 +492,30 @@ def score_kv_norm(x_f16bits, layer_begin: int = 0, layer_end: int | None = None)
     out = np.zeros((B, T), np.float32)
     lib().orc_score_kv_norm(_ptr(x), B, NL, H, T, layer_begin, le, _ptr(out))
     return out
+
+
+# ------------------------------------------ fake quantization (Sec. 4.1) ------
+
+def fake_quant(base: int, L_hi: int, L_lo: int, k, v, is_high=None, signs=None,
+               cb_hi=None, cb_lo=None):
+    """Quantize every row of K and V at its token's precision (Eq. 7; is_high None puts
+    every token at L_hi) and reconstruct to fp16 in binary32 in the order of
+    orc_fake_quant.  k, v: fp16 bits [B][NL][H][T][128]; cb_*: (centroids, thresholds)
+    fp32 for TQ.  Returns (k_out, v_out) fp16 bits."""
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    B, NL, H, T, d = k.shape
+    assert d == D and v.shape == k.shape
+    ko = np.zeros_like(k)
+    vo = np.zeros_like(v)
+    ih = None if is_high is None else np.ascontiguousarray(is_high, dtype=np.uint8)
+    sg = None if signs is None else np.ascontiguousarray(signs, dtype=np.int8)
+    z1 = np.zeros(8, np.float32)
+    ch, th = (z1, z1) if cb_hi is None else (np.ascontiguousarray(cb_hi[0], np.float32),
+                                             np.ascontiguousarray(cb_hi[1], np.float32))
+    cl, tl = (z1, z1) if cb_lo is None else (np.ascontiguousarray(cb_lo[0], np.float32),
+                                             np.ascontiguousarray(cb_lo[1], np.float32))
+    lib().orc_fake_quant(base, L_hi, L_lo, _ptr(k), _ptr(v), B, NL, H, T,
+                         None if ih is None else _ptr(ih), None if sg is None else _ptr(sg),
+                         _ptr(ch), _ptr(th), _ptr(cl), _ptr(tl), _ptr(ko), _ptr(vo))
+    return ko, vo

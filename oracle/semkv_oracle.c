@@ -10,6 +10,8 @@
  * What it computes
  *  - Per-row asymmetric affine quantization with fp16 scale/offset (Sec. 4.1
  *    "Memory accounting": two FP16 parameters per head-token row of dim 128).
+ *  - The same affine quantizer on Hadamard-rotated rows (Sec. 4.1: rotation before
+ *    the per-row quantizer): orthonormal (1/sqrt 128) H S, offset rounded down.
  *  - TurboQuant-MSE rows (Sec. 4.9): random sign flip + Walsh-Hadamard rotation,
  *    row norm stored in fp16, Gaussian Lloyd-Max codebook with L levels.
  *  - Mixed-radix packing at the paper's rates (Sec. 4.1: 3 five-level codes in
@@ -19,6 +21,7 @@
  *  - Dequantization of records to exact fp64 rows (used by the fp64 attention).
  *  - The KV-norm importance indicator (Sec. 3.3: key-norm ||K_i||_2 / value-norm
  *    ||V_i||_2 of the tensor being compressed), in a fixed summation order.
+ *  - Fake quantization: quantize and reconstruct to fp16 (Sec. 4.1's quality protocol).
  *
  * Floating point: build with -O2 -ffp-contract=off; every float operation below is
  * one IEEE binary32 operation rounded to nearest-even, in the order written.
@@ -31,7 +34,8 @@
  *  of that size stored the same way.  Symbols follow each other LSB first; quarter
  *  j starts at stream bit j * (bits of a quarter); stream bit i is bit i%8 of byte
  *  i/8; the row is zero-padded to whole bytes.
- *  affine record: [K row][V row][Ks][Kz][Vs][Vz]  (fp16 parameters)
+ *  affine record (also the rotated affine base): [K row][V row][Ks][Kz][Vs][Vz]
+ *  (fp16 parameters)
  *  TQ record:     [K row][V row][Kn][Vn]
  */
 #include <math.h>
@@ -70,6 +74,46 @@ uint16_t orc_f32_to_f16(float f) {
   uint32_t h = base + rounded;
   if (h >= 0x7C00u) h = 0x7C00u;
   return (uint16_t)(sign | h);
+}
+
+/* binary32 -> binary16 rounded toward -infinity (the largest binary16 value not
+ * above f), with subnormals; below -65504 -> -inf, above 65504 -> 65504. */
+uint16_t orc_f32_to_f16_rd(float f) {
+  uint32_t x;
+  memcpy(&x, &f, 4);
+  uint32_t sign = (x >> 16) & 0x8000u;
+  int exp = (int)((x >> 23) & 0xFFu);
+  uint32_t mant = x & 0x7FFFFFu;
+  if (exp == 0xFF) return (uint16_t)(sign | 0x7C00u | (mant ? 0x200u : 0u));
+  uint32_t mag; /* |f| truncated toward zero, as binary16 bits without the sign */
+  int inexact;
+  if (exp == 0) { /* binary32 zero or subnormal: below every nonzero binary16 */
+    mag = 0;
+    inexact = mant != 0;
+  } else {
+    uint32_t sig = mant | 0x800000u;
+    int e = exp - 127 + 15;
+    int shift;
+    uint32_t base;
+    if (e >= 1) {
+      shift = 13;
+      base = (uint32_t)(e - 1) << 10;
+    } else {
+      shift = 13 + (1 - e);
+      base = 0;
+    }
+    if (shift > 24) {
+      mag = 0;
+      inexact = 1;
+    } else {
+      mag = base + (sig >> shift);
+      inexact = (sig & ((1u << shift) - 1u)) != 0;
+    }
+  }
+  if (!sign) return (uint16_t)(mag >= 0x7C00u ? 0x7BFFu : mag);
+  if (inexact) mag += 1u; /* a negative value rounds away from zero */
+  if (mag >= 0x7C00u) mag = 0x7C00u;
+  return (uint16_t)(sign | mag);
 }
 
 float orc_f16_to_f32(uint16_t h) {
@@ -143,7 +187,7 @@ int orc_row_bytes(int L) {
 int orc_record_bytes(int base, int L) {
   int rb = orc_row_bytes(L);
   if (rb == 0) return 0;
-  return 2 * rb + (base == 0 ? 8 : 4);
+  return 2 * rb + (base == 1 ? 4 : 8);
 }
 
 static void put_bits(uint8_t* row, int pos, uint64_t val, int nbits) {
@@ -259,6 +303,56 @@ void orc_affine_row(const uint16_t* x, int L, uint8_t* codes, uint16_t* s_out,
   *z_out = z16;
 }
 
+/* 1/sqrt(128) = (1/sqrt 2)/8 rounded once to binary32: the normalisation of the
+ * orthonormal rotation (1/sqrt D) H S of the rotated affine base. */
+static const float kInvSqrtD = 0.0883883476483184405501f;
+float orc_inv_sqrt_d(void) { return kInvSqrtD; }
+
+void orc_fwht_f32(float* w);
+
+/* Hadamard-rotated affine row quantizer (Sec. 4.1: the per-row affine quantizer is
+ * applied after a Hadamard rotation; Sec. 4.9 names the rotation family).  In binary32:
+ *   u = fp32(1/sqrt 128) * FWHT(x * sign)             (orthonormal rotation of the row)
+ *   z16 = fp16 rounded toward -inf of min u, limited to >= -65504, so z <= min u
+ *   s16 = fp16_param((max u - z) / (L - 1))
+ *   c_j = clamp(rint((u_j - z) * fl(1/s)), 0, L-1), all 0 unless s > 0.
+ * Rows holding NaN or infinity are outside the supported inputs. */
+void orc_affine_had_row(const uint16_t* x, const int8_t* sgn, int L, uint8_t* codes,
+                        uint16_t* s_out, uint16_t* z_out) {
+  float u[D];
+  for (int j = 0; j < D; j++) u[j] = orc_f16_to_f32(x[j]) * (float)sgn[j];
+  orc_fwht_f32(u);
+  float mn = INFINITY, mx = -INFINITY;
+  for (int j = 0; j < D; j++) {
+    u[j] = u[j] * kInvSqrtD;
+    if (u[j] < mn) mn = u[j];
+    if (u[j] > mx) mx = u[j];
+  }
+  if (mn == 0.0f) mn = 0.0f;
+  if (mx == 0.0f) mx = 0.0f;
+  uint16_t z16 = orc_f32_to_f16_rd(mn);
+  if (z16 == 0xFC00u) z16 = 0xFBFFu;
+  float z = orc_f16_to_f32(z16);
+  float s32 = (mx - z) / (float)(L - 1);
+  uint16_t s16 = f16_param(s32);
+  float s = orc_f16_to_f32(s16);
+  if (!(s > 0.0f)) {
+    memset(codes, 0, D);
+  } else {
+    float inv = 1.0f / s;
+    for (int j = 0; j < D; j++) {
+      float d = u[j] - z;
+      float qv = d * inv;
+      int c = (int)nearbyintf(qv);
+      if (c < 0) c = 0;
+      if (c > L - 1) c = L - 1;
+      codes[j] = (uint8_t)c;
+    }
+  }
+  *s_out = s16;
+  *z_out = z16;
+}
+
 /* Unnormalised Walsh-Hadamard transform in binary32, butterfly stages h = 1, 2,
  * ..., 64; each butterfly maps (a, b) -> (a + b, a - b). */
 void orc_fwht_f32(float* w) {
@@ -360,6 +454,12 @@ int orc_quantize_tokens(int base, int Lhi, int Llo, const uint16_t* k, const uin
             orc_affine_row(k + row, L, ck, &p[0], &p[1]);
             orc_affine_row(v + row, L, cv, &p[2], &p[3]);
             memcpy(r + 2 * rb, p, 8);
+          } else if (base == 2) {
+            uint16_t p[4];
+            const int8_t* sg = signs + ((int64_t)l * H + h) * D;
+            orc_affine_had_row(k + row, sg, L, ck, &p[0], &p[1]);
+            orc_affine_had_row(v + row, sg, L, cv, &p[2], &p[3]);
+            memcpy(r + 2 * rb, p, 8);
           } else {
             uint16_t p[2];
             const int8_t* sg = signs + ((int64_t)l * H + h) * D;
@@ -389,8 +489,9 @@ static void fwht_f64(double* w) {
 }
 
 /* Dequantize `count` records of one (b, layer, head) into exact fp64 rows.
- *  affine: x^ = z + s * c               (exact in fp64)
- *  TQ:     x^ = (n / 128) * S H cb[c]   (x = S H (H S x) / 128, H H = 128 I) */
+ *  affine:         x^ = z + s * c                        (exact in fp64)
+ *  rotated affine: x^ = S H (z + s * c) / sqrt(128)      (the rotation's inverse)
+ *  TQ:             x^ = (n / 128) * S H cb[c]   (x = S H (H S x) / 128, H H = 128 I) */
 void orc_dequant_records(int base, int L, const uint8_t* recs, int64_t count,
                          const int8_t* sgn, const double* centroids, double* kout,
                          double* vout) {
@@ -401,15 +502,24 @@ void orc_dequant_records(int base, int L, const uint8_t* recs, int64_t count,
     orc_unpack_row(r, L, ck);
     orc_unpack_row(r + rb, L, cv);
     uint16_t p[4];
-    memcpy(p, r + 2 * rb, base == 0 ? 8 : 4);
+    memcpy(p, r + 2 * rb, base == 1 ? 4 : 8);
     double* ko = kout + i * D;
     double* vo = vout + i * D;
-    if (base == 0) {
+    if (base == 0 || base == 2) {
       double ks = orc_f16_to_f32(p[0]), kz = orc_f16_to_f32(p[1]);
       double vs = orc_f16_to_f32(p[2]), vz = orc_f16_to_f32(p[3]);
       for (int j = 0; j < D; j++) {
         ko[j] = kz + ks * ck[j];
         vo[j] = vz + vs * cv[j];
+      }
+      if (base == 2) {
+        fwht_f64(ko);
+        fwht_f64(vo);
+        const double r = 1.0 / sqrt((double)D);
+        for (int j = 0; j < D; j++) {
+          ko[j] = ko[j] * sgn[j] * r;
+          vo[j] = vo[j] * sgn[j] * r;
+        }
       }
     } else {
       double kn = orc_f16_to_f32(p[0]), vn = orc_f16_to_f32(p[1]);
@@ -428,6 +538,65 @@ void orc_dequant_records(int base, int L, const uint8_t* recs, int64_t count,
 }
 
 /* Element-wise conversions over arrays (for tests that sweep many values). */
+/* Fake quantization (Sec. 4.1: the quality experiments quantize and dequantize and
+ * compute in fp16): every row of K and V quantized at its token's precision (Eq. 7;
+ * is_high NULL puts every token at Lhi, a uniform grid point) and reconstructed to
+ * fp16 in binary32, in this order:
+ *   affine: x^_d = fp16( z + s * c_d )                       (multiply, then add)
+ *   rotated affine: y = FWHT(z + s * c);  x^_d = fp16( (sign_d y_d) * fp32(1/sqrt 128) )
+ *   TQ:     y = FWHT(cb[c]) (the quantizer's butterflies);  x^_d = fp16( (sign_d y_d) * (n / 128) )
+ * cent_*: fp32 centroids (TQ); x, out: [B][NL][H][T][128] fp16 bits. */
+static void fake_row(int base, const uint16_t* x, int L, const int8_t* sgn, const float* cent,
+                     const float* thr, uint16_t* out) {
+  uint8_t c[D];
+  if (base == 2) {
+    uint16_t s16, z16;
+    orc_affine_had_row(x, sgn, L, c, &s16, &z16);
+    const float s = orc_f16_to_f32(s16), z = orc_f16_to_f32(z16);
+    float y[D];
+    for (int j = 0; j < D; j++) {
+      const float t = s * (float)c[j];
+      y[j] = z + t;
+    }
+    orc_fwht_f32(y);
+    for (int j = 0; j < D; j++) out[j] = orc_f32_to_f16((y[j] * (float)sgn[j]) * kInvSqrtD);
+  } else if (base == 0) {
+    uint16_t s16, z16;
+    orc_affine_row(x, L, c, &s16, &z16);
+    const float s = orc_f16_to_f32(s16), z = orc_f16_to_f32(z16);
+    for (int j = 0; j < D; j++) {
+      const float t = s * (float)c[j];
+      out[j] = orc_f32_to_f16(z + t);
+    }
+  } else {
+    uint16_t n16;
+    orc_tq_row(x, sgn, L, thr, c, &n16);
+    const float nq = orc_f16_to_f32(n16) * 0.0078125f;
+    float y[D];
+    for (int j = 0; j < D; j++) y[j] = cent[c[j]];
+    orc_fwht_f32(y);
+    for (int j = 0; j < D; j++) out[j] = orc_f32_to_f16((y[j] * (float)sgn[j]) * nq);
+  }
+}
+
+void orc_fake_quant(int base, int Lhi, int Llo, const uint16_t* k, const uint16_t* v, int B,
+                    int NL, int H, int T, const uint8_t* is_high, const int8_t* signs,
+                    const float* cent_hi, const float* thr_hi, const float* cent_lo,
+                    const float* thr_lo, uint16_t* kout, uint16_t* vout) {
+  for (int b = 0; b < B; b++)
+    for (int l = 0; l < NL; l++)
+      for (int h = 0; h < H; h++)
+        for (int t = 0; t < T; t++) {
+          const int hi = is_high ? is_high[(int64_t)b * T + t] != 0 : 1;
+          const int64_t row = ((((int64_t)b * NL + l) * H + h) * T + t) * D;
+          const int8_t* sg = signs ? signs + ((int64_t)l * H + h) * D : NULL;
+          fake_row(base, k + row, hi ? Lhi : Llo, sg, hi ? cent_hi : cent_lo,
+                   hi ? thr_hi : thr_lo, kout + row);
+          fake_row(base, v + row, hi ? Lhi : Llo, sg, hi ? cent_hi : cent_lo,
+                   hi ? thr_hi : thr_lo, vout + row);
+        }
+}
+
 /* KV-norm indicator (Sec. 3.3, "KV-norm" family): token t of sequence b scores
  * ||x_{b,t}||_2 over the rows of layers [lb, le) and every KV head, x being the K or V
  * cache [B][NL][H][T][128] (fp16 bits).  Summation order, fixed so that equal inputs

@@ -159,6 +159,37 @@ semkv_status semkv_rank_assign(const float* scores, int32_t batch, int32_t T, ui
   return from_cuda(launch_rank_assign(a, (cudaStream_t)stream));
 }
 
+semkv_status semkv_fake_quant(const semkv_quant_desc* desc, const uint16_t* k, const uint16_t* v,
+                              int32_t batch, int32_t layers, int32_t kv_heads, int32_t T,
+                              const uint8_t* is_high, uint16_t* k_out, uint16_t* v_out,
+                              void* stream) {
+  semkv_status s = check_desc(desc);
+  if (s != SEMKV_OK) return s;
+  if (!k || !v || !k_out || !v_out || batch < 1 || layers < 1 || kv_heads < 1 || T < 1)
+    return SEMKV_EINVAL;
+  if (!aligned(k, 8) || !aligned(v, 8) || !aligned(k_out, 8) || !aligned(v_out, 8))
+    return SEMKV_EALIGN;
+  FakeArgs a;
+  a.base = desc->base;
+  a.L_hi = desc->levels_hi;
+  a.L_lo = desc->levels_lo;
+  a.k = k;
+  a.v = v;
+  a.B = batch;
+  a.NL = layers;
+  a.H = kv_heads;
+  a.T = T;
+  a.is_high = is_high;
+  a.signs = desc->signs;
+  a.thr_hi = desc->thresholds_hi;
+  a.thr_lo = desc->thresholds_lo;
+  a.cent_hi = desc->centroids_hi;
+  a.cent_lo = desc->centroids_lo;
+  a.k_out = k_out;
+  a.v_out = v_out;
+  return from_cuda(launch_fake_quant(a, device_sm_count(), (cudaStream_t)stream));
+}
+
 semkv_status semkv_score_kv_norm(const uint16_t* x, int32_t batch, int32_t layers,
                                  int32_t kv_heads, int32_t T, int32_t layer_begin,
                                  int32_t layer_end, float* scores, void* stream) {

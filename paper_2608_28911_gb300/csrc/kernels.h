@@ -43,6 +43,23 @@ struct RankArgs {
 size_t rank_workspace_words(int B, int T);
 cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream);
 
+// Fake quantization: quantize + reconstruct every row to fp16 (Sec. 4.1 protocol).
+struct FakeArgs {
+  int base, L_hi, L_lo;
+  const uint16_t* k;
+  const uint16_t* v;
+  int B, NL, H, T;
+  const uint8_t* is_high;   // [B][T] or null (every token at L_hi)
+  const int8_t* signs;      // [NL][H][128] (TQ)
+  const float* thr_hi;
+  const float* thr_lo;
+  const float* cent_hi;
+  const float* cent_lo;
+  uint16_t* k_out;
+  uint16_t* v_out;
+};
+cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t stream);
+
 // KV-norm importance scores (Sec. 3.3): ||x_{b,t}|| over layers [lb, le), all heads.
 struct ScoreArgs {
   const uint16_t* x;        // [B][NL][H][T][128] fp16

@@ -422,7 +422,118 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32)
   }
 }
 
+// ------------------------------------------------- fake quantization ---------
+// Every row quantized at its token's precision and reconstructed to fp16 (the quality
+// protocol of Sec. 4.1), in binary32 in this order:
+//   affine: x^_d = fp16( z + s * c_d )
+//   TQ:     y = FWHT(cb[c]) (the quantizer's butterflies);  x^_d = fp16( (sign_d y_d) * (n/128) )
+// One warp per (sequence, layer, KV head, token); lane l owns dims 4l..4l+3.
+
+__device__ __forceinline__ void store4_f16(uint16_t* row, int lane, const float y[4]) {
+  uint2 u;
+  u.x = (uint32_t)__half_as_ushort(__float2half_rn(y[0])) |
+        ((uint32_t)__half_as_ushort(__float2half_rn(y[1])) << 16);
+  u.y = (uint32_t)__half_as_ushort(__float2half_rn(y[2])) |
+        ((uint32_t)__half_as_ushort(__float2half_rn(y[3])) << 16);
+  *reinterpret_cast<uint2*>(row + 4 * lane) = u;
+}
+
+template <int BASE, int L>
+__device__ __forceinline__ void fake_row(const float x[4], const int8_t* sg, const float* thr_g,
+                                         const float* cent_g, uint16_t* out, int lane) {
+  float y[4];
+  if constexpr (BASE == SEMKV_BASE_AFFINE) {
+    const RowOut o = affine_row<L>(x);
+    const float s = f16_to_f32(o.p0), z = f16_to_f32(o.p1);
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      y[j] = __fadd_rn(z, __fmul_rn(s, (float)((o.codes >> (8 * j)) & 0xFFu)));
+  } else {
+    float thr[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) thr[t] = t < L - 1 ? thr_g[t] : 0.0f;
+    const RowOut o = tq_row<L>(x, sg, lane, thr);
+    float w[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) w[j] = cent_g[(o.codes >> (8 * j)) & 0xFFu];
+    {  // h = 1
+      const float a0 = w[0], b0 = w[1], a1 = w[2], b1 = w[3];
+      w[0] = __fadd_rn(a0, b0); w[1] = __fsub_rn(a0, b0);
+      w[2] = __fadd_rn(a1, b1); w[3] = __fsub_rn(a1, b1);
+    }
+    {  // h = 2
+      const float a0 = w[0], b0 = w[2], a1 = w[1], b1 = w[3];
+      w[0] = __fadd_rn(a0, b0); w[2] = __fsub_rn(a0, b0);
+      w[1] = __fadd_rn(a1, b1); w[3] = __fsub_rn(a1, b1);
+    }
+#pragma unroll
+    for (int k = 0; k < 5; ++k) {  // h = 4 << k: partner lane differs in bit k
+      const bool upper = (lane >> k) & 1;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float other = __shfl_xor_sync(0xffffffffu, w[j], 1 << k);
+        w[j] = upper ? __fsub_rn(other, w[j]) : __fadd_rn(w[j], other);
+      }
+    }
+    const float nq = f16_to_f32(o.p0) * 0.0078125f;
+    const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
+    const float sgn[4] = {(float)s4.x, (float)s4.y, (float)s4.z, (float)s4.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) y[j] = __fmul_rn(w[j] * sgn[j], nq);
+  }
+  store4_f16(out, lane, y);
+}
+
+template <int BASE>
+__global__ void __launch_bounds__(kWarpsPerBlock * 32) fake_quant_kernel(FakeArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int64_t total = (int64_t)a.B * a.NL * a.H * a.T;
+  const int64_t nwarps = (int64_t)gridDim.x * kWarpsPerBlock;
+  for (int64_t task = (int64_t)blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5); task < total;
+       task += nwarps) {
+    const int t = (int)(task % a.T);
+    int64_t r = task / a.T;
+    const int h = (int)(r % a.H);
+    r /= a.H;
+    const int l = (int)(r % a.NL);
+    const int b = (int)(r / a.NL);
+    const bool hi = a.is_high ? a.is_high[(int64_t)b * a.T + t] != 0 : true;
+    const int L = hi ? a.L_hi : a.L_lo;
+    const int64_t row = task * kHeadDim;
+    float kx[4], vx[4];
+    load4(a.k + row, lane, kx);
+    load4(a.v + row, lane, vx);
+    const int8_t* sg = a.signs ? a.signs + ((int64_t)l * a.H + h) * kHeadDim : nullptr;
+    const float* thr = hi ? a.thr_hi : a.thr_lo;
+    const float* cent = hi ? a.cent_hi : a.cent_lo;
+    switch (L) {
+#define SEMKV_FAKE_CASE(LV)                                             \
+      case LV:                                                          \
+        fake_row<BASE, LV>(kx, sg, thr, cent, a.k_out + row, lane);     \
+        fake_row<BASE, LV>(vx, sg, thr, cent, a.v_out + row, lane);     \
+        break;
+      SEMKV_FAKE_CASE(2) SEMKV_FAKE_CASE(3) SEMKV_FAKE_CASE(4) SEMKV_FAKE_CASE(5)
+      SEMKV_FAKE_CASE(6) SEMKV_FAKE_CASE(7) SEMKV_FAKE_CASE(8)
+#undef SEMKV_FAKE_CASE
+      default: break;
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t stream) {
+  const int64_t total = (int64_t)a.B * a.NL * a.H * a.T;
+  if (total == 0) return cudaSuccess;
+  int64_t blocks = (total + kWarpsPerBlock - 1) / kWarpsPerBlock;
+  const int64_t cap = (int64_t)num_sms * 32;  // grid-stride beyond this
+  if (blocks > cap) blocks = cap;
+  if (a.base == SEMKV_BASE_AFFINE)
+    fake_quant_kernel<SEMKV_BASE_AFFINE><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+  else
+    fake_quant_kernel<SEMKV_BASE_TQ><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
                                  cudaStream_t stream) {

@@ -75,6 +75,8 @@ def _load():
     L.semkv_rank_assign.argtypes = [p, i32, i32, u32, p, p, p, p, sz, p]
     L.semkv_rank_assign.restype = ctypes.c_int
     L.semkv_score_kv_norm.argtypes = [p, i32, i32, i32, i32, i32, i32, p, p]
+    L.semkv_fake_quant.argtypes = [p, p, p, i32, i32, i32, i32, p, p, p, p]
+    L.semkv_fake_quant.restype = ctypes.c_int
     L.semkv_score_kv_norm.restype = ctypes.c_int
     L.semkv_quantize_pack.argtypes = [ctypes.POINTER(QuantDescStruct), p, p, i32, p, p, u32,
                                       ctypes.POINTER(CacheStruct), p]
@@ -100,7 +102,7 @@ def _load():
 LIB = _load()
 EXPORTED = ["semkv_row_bytes", "semkv_record_bytes", "semkv_high_count_floor",
             "semkv_block_high_count", "semkv_lloyd_max_gaussian", "semkv_rank_workspace_bytes",
-            "semkv_rank_assign", "semkv_score_kv_norm", "semkv_quantize_pack", "semkv_append_block",
+            "semkv_rank_assign", "semkv_score_kv_norm", "semkv_fake_quant", "semkv_quantize_pack", "semkv_append_block",
             "semkv_decode_workspace_bytes", "semkv_decode_attention",
             "semkv_decode_attention_noalloc", "semkv_status_string"]
 
@@ -160,6 +162,15 @@ def semkv_rank_assign(scores: torch.Tensor, n_high: int, is_high: torch.Tensor,
     _check("semkv_rank_assign",
            LIB.semkv_rank_assign(_ptr(scores), B, T, n_high, _ptr(is_high), _ptr(slot),
                                  _ptr(rank), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def semkv_fake_quant(desc: "QuantDesc", k: torch.Tensor, v: torch.Tensor, k_out: torch.Tensor,
+                     v_out: torch.Tensor, is_high=None, stream=None):
+    """Quantize + reconstruct every row of k, v [B][NL][H][T][128] fp16 into k_out, v_out."""
+    B, NL, H, T, _ = k.shape
+    _check("semkv_fake_quant",
+           LIB.semkv_fake_quant(ctypes.byref(desc.s), _ptr(k), _ptr(v), B, NL, H, T,
+                                _ptr(is_high), _ptr(k_out), _ptr(v_out), _stream(stream)))
 
 
 def semkv_score_kv_norm(x: torch.Tensor, scores: torch.Tensor, layer_begin: int = 0,

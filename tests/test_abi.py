@@ -87,3 +87,24 @@ def test_rank_workspace_sizing_and_checks(lib):
     assert lib.semkv_rank_assign(fake, 2, 100, 3, fake, fake, fake, fake, 3199, None) == 6
     # misaligned workspace -> SEMKV_EALIGN
     assert lib.semkv_rank_assign(fake, 2, 100, 3, fake, fake, fake, fake + 2, 3200, None) == 2
+
+
+def test_fake_quant_validation(lib):
+    from paper_2608_28911_gb300.semkv import QuantDescStruct
+    p, i32 = ctypes.c_void_p, ctypes.c_int32
+    lib.semkv_fake_quant.argtypes = [p, p, p, i32, i32, i32, i32, p, p, p, p]
+    fake = 4096  # never dereferenced: every call below fails validation before a launch
+    d = QuantDescStruct(base=0, levels_hi=6, levels_lo=5, head_dim=128)
+    assert lib.semkv_fake_quant(None, fake, fake, 1, 1, 1, 1, None, fake, fake, None) == 1
+    assert lib.semkv_fake_quant(ctypes.byref(d), None, fake, 1, 1, 1, 1, None, fake, fake,
+                                None) == 1
+    assert lib.semkv_fake_quant(ctypes.byref(d), fake, fake, 1, 1, 1, 0, None, fake, fake,
+                                None) == 1
+    assert lib.semkv_fake_quant(ctypes.byref(d), fake + 4, fake, 1, 1, 1, 1, None, fake, fake,
+                                None) == 2
+    bad = QuantDescStruct(base=0, levels_hi=9, levels_lo=5, head_dim=128)
+    assert lib.semkv_fake_quant(ctypes.byref(bad), fake, fake, 1, 1, 1, 1, None, fake, fake,
+                                None) == 4
+    tq = QuantDescStruct(base=1, levels_hi=4, levels_lo=3, head_dim=128)  # no tables
+    assert lib.semkv_fake_quant(ctypes.byref(tq), fake, fake, 1, 1, 1, 1, None, fake, fake,
+                                None) == 1

@@ -217,3 +217,49 @@ def test_score_kv_norm_bit_exact_and_ranks(B, NL, H, T, lb, le):
     o_ih, o_sl, _ = oracle.rank_assign(want, n_high)
     assert np.array_equal(ih.cpu().numpy(), o_ih)
     assert np.array_equal(sl.cpu().numpy().view(np.uint32), o_sl)
+
+
+# -------------------------------------------------------- fake quantization ---
+
+@pytest.mark.parametrize("base,L_hi,L_lo,B,NL,H,T,mixed", [
+    (0, 6, 5, 2, 2, 2, 333, True),
+    (0, 5, 5, 1, 3, 2, 70, False),
+    (0, 2, 8, 1, 1, 4, 129, True),
+    (0, 3, 7, 2, 1, 1, 17, True),
+    (1, 4, 3, 2, 2, 2, 200, True),
+    (1, 2, 2, 1, 1, 2, 64, False),
+    (1, 8, 5, 1, 2, 2, 45, True),
+])
+def test_fake_quant_bit_exact(base, L_hi, L_lo, B, NL, H, T, mixed):
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    d = "cuda"
+    seed = 100 + T + L_hi
+    k, v = synthetic.kv(seed, B, NL, H, T)
+    k = k.astype(np.float32)
+    k[0, 0, 0, 0] = 1.25                     # constant row
+    k[0, 0, 0, 1] = 0.0                      # zero row (TQ: norm 0)
+    k[-1, -1, -1, -1] = np.linspace(-60000, 60000, 128)
+    k = k.astype(np.float16)
+    kb, vb = synthetic.f16_bits(k), synthetic.f16_bits(v)
+    ih = (np.random.default_rng(seed).random((B, T)) < 0.3).astype(np.uint8) if mixed else None
+    sg = synthetic.signs(seed, NL, H) if base == semkv.BASE_TQ else None
+    desc = semkv.QuantDesc(base, L_hi, L_lo, signs=sg)
+    kt = torch.from_numpy(k).to(d)
+    vt = torch.from_numpy(v).to(d)
+    ko, vo = torch.empty_like(kt), torch.empty_like(vt)
+    iht = torch.from_numpy(ih).to(d) if mixed else None
+    semkv.semkv_fake_quant(desc, kt, vt, ko, vo, is_high=iht)
+    torch.cuda.synchronize()
+    kw = {}
+    if base == semkv.BASE_TQ:
+        cbs = []
+        for L in (L_hi, L_lo):
+            _, c32, t32, _ = oracle.lloyd_max_gaussian(L)
+            cbs.append((c32, t32))
+        kw = dict(signs=sg, cb_hi=cbs[0], cb_lo=cbs[1])
+    o_k, o_v = oracle.fake_quant(base, L_hi, L_lo, kb, vb, is_high=ih, **kw)
+    g_k = ko.cpu().numpy().view(np.uint16)
+    g_v = vo.cpu().numpy().view(np.uint16)
+    assert np.array_equal(g_k, o_k), np.argwhere(g_k != o_k)[:5]
+    assert np.array_equal(g_v, o_v), np.argwhere(g_v != o_v)[:5]
