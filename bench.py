@@ -78,6 +78,14 @@ CONFIGS = {
                   block=128, seed=4, mode="token",
                   desc=f"4K-token prompt + generated tokens one per step, block-wise "
                        f"deferred quantization every 128 tokens, 1 layer ({_LLAMA}), affine 6/5"),
+    "had32k": dict(base=2, B=1, T=32768, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100),
+                   block=128, seed=6, mode="block",
+                   desc=f"batch 1 x 32K context, 1 layer of the Llama-3.1-8B KV shape "
+                        f"({_LLAMA}), Hadamard-rotated affine 6/5 levels at r=26%"),
+    "hb16x64k": dict(base=2, B=16, T=65536, NL=1, H=8, Hq=32, L_hi=6, L_lo=5, r=(26, 100),
+                     block=128, seed=3, mode="block",
+                     desc=f"batch 16 x 64K context, 1 layer of the Llama-3.1-8B KV shape "
+                          f"({_LLAMA}), Hadamard-rotated affine 6/5 levels at r=26%"),
     "tq32k": dict(base=1, B=1, T=32768, NL=1, H=8, Hq=32, L_hi=4, L_lo=3, r=(3, 4), block=128,
                   seed=5, mode="block",
                   desc=f"batch 1 x 32K context, 1 layer of the Mistral-7B KV shape ({_LLAMA}), "
@@ -195,7 +203,7 @@ def build_workload(cfg, dev):
     blk = cfg["block"]
     n_high = semkv.semkv_high_count_floor(T, r_num, r_den)
     n_high_blk = semkv.semkv_block_high_count(blk, r_num, r_den)
-    signs = synthetic.signs(cfg["seed"], NL, H) if cfg["base"] == semkv.BASE_TQ else None
+    signs = synthetic.signs(cfg["seed"], NL, H) if cfg["base"] != semkv.BASE_AFFINE else None
     desc = semkv.QuantDesc(cfg["base"], cfg["L_hi"], cfg["L_lo"], signs=signs, device=dev)
     cache = semkv.KVCache(desc, B, NL, H, Hq, hi_cap=n_high + n_high_blk,
                           lo_cap=T - n_high + blk - n_high_blk, block=blk, device=dev)
@@ -276,7 +284,6 @@ def gpu_arm(args, cfg, rank, world):
     B, T, NL, H, Hq, blk = cfg["B"], cfg["T"], cfg["NL"], cfg["H"], cfg["Hq"], cfg["block"]
     r_num, r_den = cfg["r"]
     token_mode = cfg["mode"] == "token"
-    tq = cfg["base"] == semkv.BASE_TQ
 
     # ---- prompt: rank + quantize + pack (A1-A5), timed for quantize GB/s
     is_high = torch.empty((B, T), dtype=torch.uint8, device=dev)
@@ -340,8 +347,9 @@ def gpu_arm(args, cfg, rank, world):
     base_counts = (cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens)
     nh_b = semkv.semkv_block_high_count(blk, r_num, r_den)
     # launches per decode call: (rotation for TQ,) pools, (stage,) combine
-    dec_launch = (1 if tq else 0) + 1 + 1
-    app_launch = 2 if tq else 3      # rank, (slot -> token scatter,) quantize
+    plain = cfg["base"] == semkv.BASE_AFFINE
+    dec_launch = (0 if plain else 1) + 1 + 1
+    app_launch = 3 if plain else 2      # rank, (slot -> token scatter,) quantize
 
     def decode_all(qv, ev=None):
         if ev is not None:
@@ -540,8 +548,9 @@ def oracle_sample(cfg, budget_s: float, max_steps: int | None = None):
     oc = oracle.Cache(base=base, L_hi=cfg["L_hi"], L_lo=cfg["L_lo"], batch=1, layers=1, kv_heads=1,
                       q_heads=G, block=blk, hi_cap=((n_high + nh_b + 15) // 16) * 16,
                       lo_cap=((T - n_high + blk + 15) // 16) * 16)
-    if base == oracle.BASE_TQ:
+    if base != oracle.BASE_AFFINE:
         oc.signs = synthetic.signs(cfg["seed"], 1, H)[:, :1]
+    if base == oracle.BASE_TQ:
         _, c32, t32, _ = oracle.lloyd_max_gaussian(cfg["L_hi"])
         oc.cb_hi = (c32, t32)
         _, c32, t32, _ = oracle.lloyd_max_gaussian(cfg["L_lo"])
@@ -599,7 +608,8 @@ def main():
     config = {"workload": cfg["desc"], "batch": cfg["B"], "context": cfg["T"],
               "layers": cfg["NL"], "kv_heads": cfg["H"], "q_heads": cfg["Hq"],
               "levels": [cfg["L_hi"], cfg["L_lo"]], "r": f"{cfg['r'][0]}/{cfg['r'][1]}",
-              "block": cfg["block"], "base": "TQ-MSE" if cfg["base"] == 1 else "affine",
+              "block": cfg["block"],
+              "base": {0: "affine", 1: "TQ-MSE", 2: "Hadamard-rotated affine"}[cfg["base"]],
               "step": "one generated token staged per step, block append every 128 steps"
               if cfg["mode"] == "token" else "append one 128-token block + decode every layer"}
 

@@ -64,12 +64,21 @@ typedef enum {
   SEMKV_EWORKSPACE = 6      /* workspace NULL or smaller than the size query says  */
 } semkv_status;
 
-enum { SEMKV_BASE_AFFINE = 0, SEMKV_BASE_TQ = 1 };
+enum { SEMKV_BASE_AFFINE = 0, SEMKV_BASE_TQ = 1, SEMKV_BASE_AFFINE_HAD = 2 };
 enum { SEMKV_HEAD_DIM = 128, SEMKV_MAX_LEVELS = 8 };
 
 /* Quantizer description (host struct; the pointers inside are device pointers).
  * base AFFINE: per-row asymmetric min/max quantizer with fp16 scale and offset
  *   (Sec. 4.1 "two FP16 parameters (offset and scale) per head-token row").
+ * base AFFINE_HAD: the same affine quantizer applied to the Hadamard-rotated row
+ *   (Sec. 4.1: rows are rotated before quantization), in binary32:
+ *     u = fp32(1/sqrt 128) * FWHT(x * sign)   (orthonormal (1/sqrt 128) H S; butterfly
+ *                                              stages 1, 2, ..., 64, each (a+b, a-b))
+ *     z = fp16 of min u rounded toward -infinity (limited to >= -65504), so z <= min u
+ *     s = fp16((max u - z) / (L - 1)), rounded to nearest and limited to 65504
+ *     c_j = clamp(rint((u_j - z) * fl(1/s)), 0, L - 1); all 0 unless s > 0.
+ *   Records as AFFINE; decoding rotates each query once and the output back once.
+ *   Needs signs.  Rows holding NaN or infinity are outside the supported inputs.
  * base TQ: TurboQuant-MSE (Sec. 4.9): sign flip + unnormalised Walsh-Hadamard
  *   transform of the row, divided by the row's fp16 norm, then a Gaussian Lloyd-Max
  *   scalar codebook with L levels (thresholds strictly-greater: ties go low).
@@ -78,7 +87,8 @@ typedef struct {
   int32_t base;
   int32_t levels_hi, levels_lo;
   int32_t head_dim;                 /* must be 128 */
-  const int8_t* signs;              /* TQ: device [layers][kv_heads][128] of +-1   */
+  const int8_t* signs;              /* TQ, AFFINE_HAD: device [layers][kv_heads][128]
+                                       of +-1, 4-byte aligned                       */
   const float* centroids_hi;        /* TQ: device [levels_hi]   ascending           */
   const float* thresholds_hi;       /* TQ: device [levels_hi-1] ascending           */
   const float* centroids_lo;        /* TQ: device [levels_lo]                       */

@@ -18,8 +18,14 @@ bool level_ok(int L) { return L >= 2 && L <= SEMKV_MAX_LEVELS; }
 semkv_status check_desc(const semkv_quant_desc* d) {
   if (!d) return SEMKV_EINVAL;
   if (d->head_dim != SEMKV_HEAD_DIM) return SEMKV_EUNSUPPORTED;
-  if (d->base != SEMKV_BASE_AFFINE && d->base != SEMKV_BASE_TQ) return SEMKV_EUNSUPPORTED;
+  if (d->base != SEMKV_BASE_AFFINE && d->base != SEMKV_BASE_TQ &&
+      d->base != SEMKV_BASE_AFFINE_HAD)
+    return SEMKV_EUNSUPPORTED;
   if (!level_ok(d->levels_hi) || !level_ok(d->levels_lo)) return SEMKV_EUNSUPPORTED;
+  if (d->base == SEMKV_BASE_AFFINE_HAD) {
+    if (!d->signs) return SEMKV_EINVAL;
+    if (!aligned(d->signs, 4)) return SEMKV_EALIGN;
+  }
   if (d->base == SEMKV_BASE_TQ) {
     if (!d->signs || !d->thresholds_hi || !d->thresholds_lo || !d->centroids_hi ||
         !d->centroids_lo)
@@ -69,7 +75,9 @@ extern "C" {
 size_t semkv_row_bytes(int32_t levels) { return level_ok(levels) ? (size_t)row_bytes_rt(levels) : 0; }
 
 size_t semkv_record_bytes(int32_t base, int32_t levels) {
-  if (!level_ok(levels) || (base != SEMKV_BASE_AFFINE && base != SEMKV_BASE_TQ)) return 0;
+  if (!level_ok(levels) ||
+      (base != SEMKV_BASE_AFFINE && base != SEMKV_BASE_TQ && base != SEMKV_BASE_AFFINE_HAD))
+    return 0;
   return (size_t)record_bytes_rt(base, levels);
 }
 
@@ -369,7 +377,8 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
   a.signs = desc->signs;
   a.cb_hi = desc->centroids_hi;
   a.cb_lo = desc->centroids_lo;
-  // rotated queries (TQ base) after the split-K partials in the workspace
+  // rotated queries (TQ and rotated affine bases) after the split-K partials
+  // in the workspace
   a.qrot = a.partials + (decode_workspace_floats(a.B, a.H, a.Hq) - (size_t)a.B * a.Hq * 128);
   a.err = cache->dev_error;
   a.plan = make_decode_plan(a.base, a.L_hi, a.L_lo, a.B, a.H, a.hi_count, a.lo_count, a.stage_n,

@@ -55,7 +55,7 @@ __host__ __device__ inline int row_bytes_rt(int L) {
 }
 __host__ __device__ inline int record_bytes_rt(int base, int L) {
   int rb = row_bytes_rt(L);
-  return rb == 0 ? 0 : 2 * rb + (base == SEMKV_BASE_AFFINE ? 8 : 4);
+  return rb == 0 ? 0 : 2 * rb + (base == SEMKV_BASE_TQ ? 4 : 8);
 }
 
 // --------------------------------------------------------------- helpers ------
@@ -67,6 +67,9 @@ __device__ __forceinline__ uint16_t f16_param(float f) {
   if ((h & 0x7FFFu) == 0x7C00u) h = (uint16_t)((h & 0x8000u) | 0x7BFFu);
   return h;
 }
+// 1/sqrt(128) rounded to binary32: the normalisation of the rotation (1/sqrt 128) H S
+constexpr float kInvSqrtD = 0x1.6a09e6p-4f;
+
 __device__ __forceinline__ float f16_to_f32(uint16_t h) {
   return __half2float(__ushort_as_half(h));
 }

@@ -500,7 +500,7 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
       const int p = 2 * j + i;
       float c0 = 0.0f, c1 = 0.0f;
       if (live && !upper) {
-        if constexpr (CODEC == 0) {
+        if (CODEC == 0 && a.base != SEMKV_BASE_AFFINE_HAD) {
           c0 = k_coef<L>(sh.q[g], t, p, 0) * qscale;
           c1 = k_coef<L>(sh.q[g], t, p, 1) * qscale;
         } else {
@@ -875,7 +875,9 @@ __device__ void run_pool_tq(const DecodeArgs& a, const Shared& sh, int which,
   }
 }
 
-// q' = H S q for every (sequence, query head): one warp each, lane l = dims 4l..4l+3
+// q' = H S q for every (sequence, query head), times fp32(1/sqrt 128) for the rotated
+// affine base (whose rows are stored in the orthonormal frame): one warp each, lane l =
+// dims 4l..4l+3
 __global__ void qrot_kernel(DecodeArgs a) {
   const int lane = threadIdx.x & 31;
   const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -897,9 +899,10 @@ __global__ void qrot_kernel(DecodeArgs a) {
       w[j] = upper ? other - w[j] : w[j] + other;
     }
   }
+  const float rs = a.base == SEMKV_BASE_AFFINE_HAD ? kInvSqrtD : 1.0f;
   float* dst = a.qrot + ((int64_t)b * a.Hq + qh) * 128 + 4 * lane;
 #pragma unroll
-  for (int j = 0; j < 4; ++j) dst[j] = w[j];
+  for (int j = 0; j < 4; ++j) dst[j] = w[j] * rs;
 }
 
 // ------------------------------------------------------- fp16 stage tokens ----
@@ -985,11 +988,15 @@ struct MergeArea {
 
 // the group's queries of pair (b, h) into shared memory, with their sums and maxima
 // (every thread of the CTA calls this; the caller orders it after earlier readers)
+// (rotated affine base: also the rotated queries into sh.qr, which the sums then follow)
 __device__ void load_group_q(const DecodeArgs& a, Shared& sh, int b, int h, int G) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool rot = a.base == SEMKV_BASE_AFFINE_HAD;
   for (int i = threadIdx.x; i < 8 * 128; i += kThreads) {
     const int c = i >> 7, d = i & 127;
-    sh.q[c][d] = c < G ? a.q[((int64_t)b * a.Hq + h * G + c) * 128 + d] : (uint16_t)0;
+    const int64_t at = ((int64_t)b * a.Hq + h * G + c) * 128 + d;
+    sh.q[c][d] = c < G ? a.q[at] : (uint16_t)0;
+    if (rot) sh.qr[c][d] = c < G ? a.qrot[at] : 0.0f;
   }
   __syncthreads();
   // per head: sum of q (the zero-point weight) and max |q| (the coefficient scale)
@@ -997,7 +1004,7 @@ __device__ void load_group_q(const DecodeArgs& a, Shared& sh, int b, int h, int 
   float s = 0.0f, mx = 0.0f;
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
-    const float x = f16_to_f32(sh.q[warp][4 * lane + j]);
+    const float x = rot ? sh.qr[warp][4 * lane + j] : f16_to_f32(sh.q[warp][4 * lane + j]);
     s += x;
     mx = fmaxf(mx, fabsf(x));
   }
@@ -1118,10 +1125,12 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
     }
   }
   const int8_t* sg = rotated ? a.signs + ((int64_t)a.layer * a.H + h) * 128 : nullptr;
+  // the rotated affine base stores rows in the orthonormal frame: x = S H u / sqrt(128)
+  const float rs = a.base == SEMKV_BASE_AFFINE_HAD ? kInvSqrtD : 1.0f;
   for (int i = threadIdx.x; i < G * 128; i += kThreads) {
     const int qh = i >> 7, d = i & 127;
     const float o = merged[qh * 128 + d];
-    part[16 + qh * 128 + d] = rotated ? o * (float)sg[d] : o;
+    part[16 + qh * 128 + d] = rotated ? o * ((float)sg[d] * rs) : o;
   }
   __syncthreads();  // the merge area (the ring) is free again
 }
@@ -1197,7 +1206,8 @@ __global__ void __launch_bounds__(kThreads, kCtasAffine) decode_affine_kernel(De
         default: break;
       }
       affine_rows(st, L, G, mg, merge_o);
-      merge_warps(a, 0, h, G, mg, merge_o, a.partials + (bh * P.stride + slot) * kPartialFloats);
+      merge_warps(a, a.base == SEMKV_BASE_AFFINE_HAD ? 3 : 0, h, G, mg, merge_o,
+                  a.partials + (bh * P.stride + slot) * kPartialFloats);
     }
   }
 }
@@ -1401,7 +1411,7 @@ DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int64_t 
   p.splits_st = st;
   const int64_t pairs = (int64_t)B * H;
   if (max_stride > kMaxSplits + 1) max_stride = kMaxSplits + 1;
-  if (base == SEMKV_BASE_AFFINE) {
+  if (base == SEMKV_BASE_AFFINE || base == SEMKV_BASE_AFFINE_HAD) {
     // balanced: one wave of equal CTAs over the weighted tiles of every pair
     p.balanced = 1;
     p.w_hi = tile_cost(L_hi);
@@ -1528,8 +1538,15 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
     const int pool_splits = P.splits_hi + P.splits_lo;
     if (pool_splits > 0)
       decode_kernel<1><<<dim3(pool_splits, a.H, a.B), kThreads, kRingBytes + kAqBytes, stream>>>(a);
-  } else if (P.ctas > 0) {
-    decode_affine_kernel<<<P.ctas, kThreads, kRingBytes + kAqBytes, stream>>>(a);
+  } else {
+    if (a.base == SEMKV_BASE_AFFINE_HAD) {  // the stage kernel reads the rotated q too
+      const int heads = a.B * a.Hq;
+      qrot_kernel<<<(heads + 7) / 8, 256, 0, stream>>>(a);
+      e = cudaGetLastError();
+      if (e != cudaSuccess) return e;
+    }
+    if (P.ctas > 0)
+      decode_affine_kernel<<<P.ctas, kThreads, kRingBytes + kAqBytes, stream>>>(a);
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;

@@ -68,13 +68,9 @@ __device__ __forceinline__ RowOut affine_row(const float x[4]) {
   return o;
 }
 
-template <int L>
-__device__ __forceinline__ RowOut tq_row(const float x[4], const int8_t* sg, int lane,
-                                         const float thr[8]) {
-  // sign flip (exact) then the Walsh-Hadamard butterflies in stage order
-  const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
-  float w[4] = {x[0] * (float)s4.x, x[1] * (float)s4.y, x[2] * (float)s4.z,
-                x[3] * (float)s4.w};
+// Unnormalised Walsh-Hadamard transform of a row held 4 values per lane (lane l owns
+// dims 4l..4l+3), butterfly stages h = 1, 2, ..., 64 in order, each (a + b, a - b).
+__device__ __forceinline__ void fwht_lanes(float w[4], int lane) {
   {  // h = 1: (0,1), (2,3)
     float a = w[0], b = w[1];
     w[0] = __fadd_rn(a, b); w[1] = __fsub_rn(a, b);
@@ -96,6 +92,16 @@ __device__ __forceinline__ RowOut tq_row(const float x[4], const int8_t* sg, int
       w[j] = upper ? __fsub_rn(other, w[j]) : __fadd_rn(w[j], other);
     }
   }
+}
+
+template <int L>
+__device__ __forceinline__ RowOut tq_row(const float x[4], const int8_t* sg, int lane,
+                                         const float thr[8]) {
+  // sign flip (exact) then the Walsh-Hadamard butterflies in stage order
+  const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
+  float w[4] = {x[0] * (float)s4.x, x[1] * (float)s4.y, x[2] * (float)s4.z,
+                x[3] * (float)s4.w};
+  fwht_lanes(w, lane);
   // norm with the fixed tree
   float acc = __fmul_rn(x[0], x[0]);
   acc = __fadd_rn(acc, __fmul_rn(x[1], x[1]));
@@ -116,6 +122,45 @@ __device__ __forceinline__ RowOut tq_row(const float x[4], const int8_t* sg, int
       int c = 0;
 #pragma unroll
       for (int t = 0; t < L - 1; ++t) c += (u > thr[t]) ? 1 : 0;
+      o.codes |= (uint32_t)c << (8 * j);
+    }
+  }
+  return o;
+}
+
+// Hadamard-rotated affine row: u = fp32(1/sqrt 128) FWHT(x sign); z = fp16 of min u
+// rounded toward -inf (limited to -65504); s = fp16_param((max u - z)/(L-1)); codes as
+// affine_row, all 0 unless s > 0.
+template <int L>
+__device__ __forceinline__ RowOut affine_had_row(const float x[4], const int8_t* sg, int lane) {
+  const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
+  float u[4] = {x[0] * (float)s4.x, x[1] * (float)s4.y, x[2] * (float)s4.z,
+                x[3] * (float)s4.w};
+  fwht_lanes(u, lane);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) u[j] = __fmul_rn(u[j], kInvSqrtD);
+  float mn = fminf(fminf(u[0], u[1]), fminf(u[2], u[3]));
+  float mx = fmaxf(fmaxf(u[0], u[1]), fmaxf(u[2], u[3]));
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  }
+  if (mn == 0.0f) mn = 0.0f;
+  if (mx == 0.0f) mx = 0.0f;
+  RowOut o;
+  o.p1 = __half_as_ushort(__float2half_rd(mn));
+  if (o.p1 == 0xFC00u) o.p1 = 0xFBFFu;
+  const float z = f16_to_f32(o.p1);
+  o.p0 = f16_param(__fdiv_rn(__fsub_rn(mx, z), (float)(L - 1)));
+  const float s = f16_to_f32(o.p0);
+  o.codes = 0;
+  if (s > 0.0f) {
+    const float inv = __fdiv_rn(1.0f, s);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      int c = __float2int_rn(__fmul_rn(__fsub_rn(u[j], z), inv));
+      c = min(max(c, 0), L - 1);
       o.codes |= (uint32_t)c << (8 * j);
     }
   }
@@ -158,6 +203,9 @@ __device__ void quantize_pair(const QuantArgs& a, const float kx[4], const float
   if constexpr (BASE == SEMKV_BASE_AFFINE) {
     ko = affine_row<L>(kx);
     vo = affine_row<L>(vx);
+  } else if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
+    ko = affine_had_row<L>(kx, sg, lane);
+    vo = affine_had_row<L>(vx, sg, lane);
   } else {
     float thr[8];
 #pragma unroll
@@ -165,7 +213,7 @@ __device__ void quantize_pair(const QuantArgs& a, const float kx[4], const float
     ko = tq_row<L>(kx, sg, lane, thr);
     vo = tq_row<L>(vx, sg, lane, thr);
   }
-  constexpr int kRec = 2 * F::RB + (BASE == SEMKV_BASE_AFFINE ? 8 : 4);
+  constexpr int kRec = 2 * F::RB + (BASE == SEMKV_BASE_TQ ? 4 : 8);
   constexpr int kRecWords = kRec / 4;
   reinterpret_cast<uint32_t*>(codes)[lane] = ko.codes;
   reinterpret_cast<uint32_t*>(codes)[32 + lane] = vo.codes;
@@ -173,7 +221,7 @@ __device__ void quantize_pair(const QuantArgs& a, const float kx[4], const float
   __syncwarp();
   pack_rows<L>(codes, rec, lane);
   if (lane == 0) {
-    if constexpr (BASE == SEMKV_BASE_AFFINE) {
+    if constexpr (BASE != SEMKV_BASE_TQ) {
       rec[(2 * F::RB) / 4] = (uint32_t)ko.p0 | ((uint32_t)ko.p1 << 16);
       rec[(2 * F::RB) / 4 + 1] = (uint32_t)vo.p0 | ((uint32_t)vo.p1 << 16);
     } else {
@@ -426,6 +474,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32)
 // Every row quantized at its token's precision and reconstructed to fp16 (the quality
 // protocol of Sec. 4.1), in binary32 in this order:
 //   affine: x^_d = fp16( z + s * c_d )
+//   rotated affine: y = FWHT(z + s * c);  x^_d = fp16( (sign_d y_d) * fp32(1/sqrt 128) )
 //   TQ:     y = FWHT(cb[c]) (the quantizer's butterflies);  x^_d = fp16( (sign_d y_d) * (n/128) )
 // One warp per (sequence, layer, KV head, token); lane l owns dims 4l..4l+3.
 
@@ -448,6 +497,18 @@ __device__ __forceinline__ void fake_row(const float x[4], const int8_t* sg, con
 #pragma unroll
     for (int j = 0; j < 4; ++j)
       y[j] = __fadd_rn(z, __fmul_rn(s, (float)((o.codes >> (8 * j)) & 0xFFu)));
+  } else if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
+    const RowOut o = affine_had_row<L>(x, sg, lane);
+    const float s = f16_to_f32(o.p0), z = f16_to_f32(o.p1);
+    float w[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      w[j] = __fadd_rn(z, __fmul_rn(s, (float)((o.codes >> (8 * j)) & 0xFFu)));
+    fwht_lanes(w, lane);
+    const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
+    const float sgn[4] = {(float)s4.x, (float)s4.y, (float)s4.z, (float)s4.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) y[j] = __fmul_rn(w[j] * sgn[j], kInvSqrtD);
   } else {
     float thr[8];
 #pragma unroll
@@ -456,25 +517,7 @@ __device__ __forceinline__ void fake_row(const float x[4], const int8_t* sg, con
     float w[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) w[j] = cent_g[(o.codes >> (8 * j)) & 0xFFu];
-    {  // h = 1
-      const float a0 = w[0], b0 = w[1], a1 = w[2], b1 = w[3];
-      w[0] = __fadd_rn(a0, b0); w[1] = __fsub_rn(a0, b0);
-      w[2] = __fadd_rn(a1, b1); w[3] = __fsub_rn(a1, b1);
-    }
-    {  // h = 2
-      const float a0 = w[0], b0 = w[2], a1 = w[1], b1 = w[3];
-      w[0] = __fadd_rn(a0, b0); w[2] = __fsub_rn(a0, b0);
-      w[1] = __fadd_rn(a1, b1); w[3] = __fsub_rn(a1, b1);
-    }
-#pragma unroll
-    for (int k = 0; k < 5; ++k) {  // h = 4 << k: partner lane differs in bit k
-      const bool upper = (lane >> k) & 1;
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float other = __shfl_xor_sync(0xffffffffu, w[j], 1 << k);
-        w[j] = upper ? __fsub_rn(other, w[j]) : __fadd_rn(w[j], other);
-      }
-    }
+    fwht_lanes(w, lane);
     const float nq = f16_to_f32(o.p0) * 0.0078125f;
     const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
     const float sgn[4] = {(float)s4.x, (float)s4.y, (float)s4.z, (float)s4.w};
@@ -530,6 +573,8 @@ cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t strea
   if (blocks > cap) blocks = cap;
   if (a.base == SEMKV_BASE_AFFINE)
     fake_quant_kernel<SEMKV_BASE_AFFINE><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+  else if (a.base == SEMKV_BASE_AFFINE_HAD)
+    fake_quant_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
   else
     fake_quant_kernel<SEMKV_BASE_TQ><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
   return cudaGetLastError();
@@ -558,7 +603,10 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
   int64_t blocks = (total + kWarpsPerBlock - 1) / kWarpsPerBlock;
   const int64_t cap_blocks = (int64_t)num_sms * 16;  // grid-stride beyond this
   if (blocks > cap_blocks) blocks = cap_blocks;
-  quantize_pack_kernel<SEMKV_BASE_TQ><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+  if (a.base == SEMKV_BASE_AFFINE_HAD)
+    quantize_pack_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+  else
+    quantize_pack_kernel<SEMKV_BASE_TQ><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
   return cudaGetLastError();
 }
 

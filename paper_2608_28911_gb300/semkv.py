@@ -16,7 +16,7 @@ import torch
 
 from . import build as _build
 
-BASE_AFFINE, BASE_TQ = 0, 1
+BASE_AFFINE, BASE_TQ, BASE_AFFINE_HAD = 0, 1, 2
 HEAD_DIM = 128
 
 _STATUS = {0: "ok", 1: "invalid argument", 2: "misaligned pointer or capacity",
@@ -245,6 +245,12 @@ class QuantDesc:
                 [t.data_ptr() for t in tabs]
             self.signs = sg
             self.codebooks = {"hi": (ch, th), "lo": (cl, tl)}
+        elif base == BASE_AFFINE_HAD:
+            assert signs is not None, "the rotated affine base needs a sign vector per (layer, head)"
+            sg = torch.as_tensor(signs, dtype=torch.int8).to(device).contiguous()
+            self._keep.append(sg)
+            s.signs = sg.data_ptr()
+            self.signs = sg
         self.s = s
 
 

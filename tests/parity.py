@@ -30,7 +30,7 @@ class Pair:
         self.base, self.B, self.NL, self.H, self.Hq, self.T = base, B, NL, H, Hq, T
         self.r_num, self.r_den, self.seed = r_num, r_den, seed
         self.n_high = oracle.high_count_floor(T, r_num, r_den)
-        signs = synthetic.signs(seed, NL, H) if base == oracle.BASE_TQ else None
+        signs = synthetic.signs(seed, NL, H) if base != oracle.BASE_AFFINE else None
         self.desc = semkv.QuantDesc(base, L_hi, L_lo, signs=signs, device=self.dev)
         self.cache = semkv.KVCache(self.desc, B, NL, H, Hq, hi_cap=self.n_high + extra_cap,
                                    lo_cap=T - self.n_high + extra_cap, block=block,
@@ -38,8 +38,9 @@ class Pair:
         self.oc = oracle.Cache(base=base, L_hi=L_hi, L_lo=L_lo, batch=B, layers=NL, kv_heads=H,
                                q_heads=Hq, block=block, hi_cap=self.cache.s.hi_cap,
                                lo_cap=self.cache.s.lo_cap)
-        if base == oracle.BASE_TQ:
+        if signs is not None:
             self.oc.signs = signs
+        if base == oracle.BASE_TQ:
             _, c32, t32, _ = oracle.lloyd_max_gaussian(L_hi)
             self.oc.cb_hi = (c32, t32)
             _, c32, t32, _ = oracle.lloyd_max_gaussian(L_lo)

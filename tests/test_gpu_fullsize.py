@@ -25,6 +25,16 @@ def test_mixed_65_batch1_32k_every_record_and_head():
     assert err <= ATOL and rel <= RTOL_L2, (err, rel)
 
 
+def test_had_65_batch1_32k_every_record_and_head():
+    # the same workload on the Hadamard-rotated affine base
+    p = Pair(2, 6, 5, 1, 1, 8, 32, 32768, 26, 100, seed=6)
+    p.quantize()
+    p.assert_records_equal()
+    got, ref = p.decode(0, 0)
+    err, rel = attention_errors(got, ref)
+    assert err <= ATOL and rel <= RTOL_L2, (err, rel)
+
+
 def test_batch16_64k_sampled_sequences_and_heads():
     import torch
     from paper_2608_28911_gb300 import semkv

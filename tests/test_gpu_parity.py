@@ -57,6 +57,10 @@ def test_rank_assign_bit_exact(T):
     (1, 4, 3, 1, 2, 2, 200, (3, 4)),        # TQ 4/3
     (1, 6, 5, 1, 1, 2, 90, (1, 4)),
     (1, 8, 2, 1, 1, 2, 90, (1, 4)),
+    (2, 6, 5, 2, 2, 2, 333, (26, 100)),     # Hadamard-rotated affine 6/5
+    (2, 5, 5, 1, 1, 2, 100, (0, 100)),
+    (2, 2, 8, 1, 1, 2, 70, (1, 2)),
+    (2, 3, 7, 1, 2, 1, 50, (1, 3)),
 ])
 def test_quantize_pack_bit_exact(base, L_hi, L_lo, B, NL, H, T, r):
     p = Pair(base, L_hi, L_lo, B, NL, H, 4 * H, T, r[0], r[1], seed=T + L_hi)
@@ -66,9 +70,11 @@ def test_quantize_pack_bit_exact(base, L_hi, L_lo, B, NL, H, T, r):
     assert int(p.cache.dev_error.item()) == 0
 
 
-def test_quantize_edge_rows_bit_exact():
-    # constant rows, signed zeros, tiny (subnormal-step) ranges and huge ranges
-    p = Pair(0, 6, 5, 1, 1, 2, 8, 64, 1, 2, seed=3)
+@pytest.mark.parametrize("base", [0, 2])
+def test_quantize_edge_rows_bit_exact(base):
+    # constant rows, signed zeros, tiny (subnormal-step) ranges and huge ranges (for the
+    # rotated base the rotated range passes 65504: the offset and scale saturate)
+    p = Pair(base, 6, 5, 1, 1, 2, 8, 64, 1, 2, seed=3)
     k = p.k.astype(np.float32)
     v = p.v.astype(np.float32)
     k[0, 0, 0, 0] = 1.5
@@ -114,8 +120,9 @@ def test_decode_attention_matches_oracle(L_hi, L_lo, B, NL, H, Hq, T, r):
         check_attention(p, layer)
 
 
-def test_decode_attention_with_staged_tail():
-    p = Pair(0, 6, 5, 2, 1, 2, 8, 300, 26, 100, seed=11, block=32)
+@pytest.mark.parametrize("base", [0, 2])
+def test_decode_attention_with_staged_tail(base):
+    p = Pair(base, 6, 5, 2, 1, 2, 8, 300, 26, 100, seed=11, block=32)
     p.quantize()
     k, v = synthetic.kv(12, 2, 1, 2, 20)
     s = synthetic.scores_zipf(12, 2, 20)
@@ -129,11 +136,12 @@ def test_decode_attention_with_staged_tail():
     check_attention(p)
 
 
-def test_append_blocks_and_flush_match_oracle():
+@pytest.mark.parametrize("base", [0, 2])
+def test_append_blocks_and_flush_match_oracle(base):
     import torch
     from paper_2608_28911_gb300 import semkv
     blk, T0, ngen = 32, 200, 2 * 32 + 9
-    p = Pair(0, 6, 5, 2, 2, 2, 8, T0, 26, 100, seed=21, block=blk, extra_cap=ngen)
+    p = Pair(base, 6, 5, 2, 2, 2, 8, T0, 26, 100, seed=21, block=blk, extra_cap=ngen)
     p.quantize()
     k, v = synthetic.kv(22, 2, 2, 2, ngen)
     s = synthetic.scores_zipf(22, 2, ngen)
@@ -156,6 +164,24 @@ def test_append_blocks_and_flush_match_oracle():
     p.assert_records_equal()
     assert p.cache.stage_n == 0 and p.cache.n_tokens == T0 + ngen
     check_attention(p, layer=1, qseed=99)
+
+
+# ------------------------------------------- Hadamard-rotated affine decode -----
+
+@pytest.mark.parametrize("L_hi,L_lo,B,NL,H,Hq,T,r", [
+    (6, 5, 2, 2, 2, 8, 333, (26, 100)),     # mixed, ragged tiles, layer 1 checked too
+    (6, 5, 1, 1, 8, 32, 2048, (26, 100)),   # Llama-3.1-8B layer shape, short context
+    (5, 5, 1, 1, 1, 4, 1024, (0, 100)),
+    (2, 3, 1, 1, 2, 8, 100, (1, 2)),
+    (8, 7, 1, 1, 2, 16, 150, (1, 4)),       # GQA group of 8
+    (6, 5, 1, 1, 1, 3, 150, (1, 4)),        # GQA group of 3
+])
+def test_had_decode_attention_matches_oracle(L_hi, L_lo, B, NL, H, Hq, T, r):
+    p = Pair(2, L_hi, L_lo, B, NL, H, Hq, T, r[0], r[1], seed=60 + T)
+    p.quantize()
+    p.assert_records_equal()
+    for layer in range(NL):
+        check_attention(p, layer)
 
 
 # ------------------------------------------------------------ TQ decode -----
@@ -229,6 +255,9 @@ def test_score_kv_norm_bit_exact_and_ranks(B, NL, H, T, lb, le):
     (1, 4, 3, 2, 2, 2, 200, True),
     (1, 2, 2, 1, 1, 2, 64, False),
     (1, 8, 5, 1, 2, 2, 45, True),
+    (2, 6, 5, 2, 2, 2, 150, True),
+    (2, 5, 5, 1, 1, 3, 40, False),
+    (2, 2, 8, 1, 2, 1, 33, True),
 ])
 def test_fake_quant_bit_exact(base, L_hi, L_lo, B, NL, H, T, mixed):
     import torch
@@ -243,7 +272,7 @@ def test_fake_quant_bit_exact(base, L_hi, L_lo, B, NL, H, T, mixed):
     k = k.astype(np.float16)
     kb, vb = synthetic.f16_bits(k), synthetic.f16_bits(v)
     ih = (np.random.default_rng(seed).random((B, T)) < 0.3).astype(np.uint8) if mixed else None
-    sg = synthetic.signs(seed, NL, H) if base == semkv.BASE_TQ else None
+    sg = synthetic.signs(seed, NL, H) if base != semkv.BASE_AFFINE else None
     desc = semkv.QuantDesc(base, L_hi, L_lo, signs=sg)
     kt = torch.from_numpy(k).to(d)
     vt = torch.from_numpy(v).to(d)
@@ -258,6 +287,8 @@ def test_fake_quant_bit_exact(base, L_hi, L_lo, B, NL, H, T, mixed):
             _, c32, t32, _ = oracle.lloyd_max_gaussian(L)
             cbs.append((c32, t32))
         kw = dict(signs=sg, cb_hi=cbs[0], cb_lo=cbs[1])
+    elif base == semkv.BASE_AFFINE_HAD:
+        kw = dict(signs=sg)
     o_k, o_v = oracle.fake_quant(base, L_hi, L_lo, kb, vb, is_high=ih, **kw)
     g_k = ko.cpu().numpy().view(np.uint16)
     g_v = vo.cpu().numpy().view(np.uint16)
