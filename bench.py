@@ -86,6 +86,11 @@ CONFIGS = {
                      block=128, seed=3, mode="block",
                      desc=f"batch 16 x 64K context, 1 layer of the Llama-3.1-8B KV shape "
                           f"({_LLAMA}), Hadamard-rotated affine 6/5 levels at r=26%"),
+    "tqd32k": dict(base=3, B=1, T=32768, NL=1, H=8, Hq=32, L_hi=4, L_lo=3, r=(3, 4), block=128,
+                   seed=5, mode="block",
+                   desc=f"batch 1 x 32K context, 1 layer of the Mistral-7B KV shape ({_LLAMA}), "
+                        f"TurboQuant-MSE-style base with a dense random rotation at 4/3 levels, "
+                        f"r=75%"),
     "tq32k": dict(base=1, B=1, T=32768, NL=1, H=8, Hq=32, L_hi=4, L_lo=3, r=(3, 4), block=128,
                   seed=5, mode="block",
                   desc=f"batch 1 x 32K context, 1 layer of the Mistral-7B KV shape ({_LLAMA}), "
@@ -203,8 +208,11 @@ def build_workload(cfg, dev):
     blk = cfg["block"]
     n_high = semkv.semkv_high_count_floor(T, r_num, r_den)
     n_high_blk = semkv.semkv_block_high_count(blk, r_num, r_den)
-    signs = synthetic.signs(cfg["seed"], NL, H) if cfg["base"] != semkv.BASE_AFFINE else None
-    desc = semkv.QuantDesc(cfg["base"], cfg["L_hi"], cfg["L_lo"], signs=signs, device=dev)
+    signs = (synthetic.signs(cfg["seed"], NL, H)
+             if cfg["base"] in (semkv.BASE_TQ, semkv.BASE_AFFINE_HAD) else None)
+    rot = synthetic.rotations(cfg["seed"], NL, H) if cfg["base"] == semkv.BASE_TQ_DENSE else None
+    desc = semkv.QuantDesc(cfg["base"], cfg["L_hi"], cfg["L_lo"], signs=signs, device=dev,
+                           rotation=rot)
     cache = semkv.KVCache(desc, B, NL, H, Hq, hi_cap=n_high + n_high_blk,
                           lo_cap=T - n_high + blk - n_high_blk, block=blk, device=dev)
     k = torch.empty((B, NL, H, T, 128), dtype=torch.float16, device=dev)
@@ -316,20 +324,24 @@ def gpu_arm(args, cfg, rank, world):
         if it > 0:
             st_.append(e0.elapsed_time(e1) * 1e-3)
     score_gbs = (B * NL * H * T * 128 * 2 + B * T * 4) / statistics.median(st_) / 1e9
-    # fake quantization of the prompt's K and V at the selected precisions (Sec. 4.1)
-    ko, vo = torch.empty_like(w["k"]), torch.empty_like(w["v"])
-    ft = []
-    for it in range(4):
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        torch.cuda.synchronize()
-        e0.record(stream)
-        semkv.semkv_fake_quant(desc, w["k"], w["v"], ko, vo, is_high=is_high)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        if it > 0:
-            ft.append(e0.elapsed_time(e1) * 1e-3)
-    fake_gbs = (B * NL * H * T * 128 * 2 * 4 + B * T) / statistics.median(ft) / 1e9
-    del ko, vo, w["k"], w["v"]
+    # fake quantization of the prompt's K and V at the selected precisions (Sec. 4.1;
+    # not provided for the dense-rotation base)
+    fake_gbs = None
+    if cfg["base"] != semkv.BASE_TQ_DENSE:
+        ko, vo = torch.empty_like(w["k"]), torch.empty_like(w["v"])
+        ft = []
+        for it in range(4):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record(stream)
+            semkv.semkv_fake_quant(desc, w["k"], w["v"], ko, vo, is_high=is_high)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if it > 0:
+                ft.append(e0.elapsed_time(e1) * 1e-3)
+        fake_gbs = (B * NL * H * T * 128 * 2 * 4 + B * T) / statistics.median(ft) / 1e9
+        del ko, vo
+    del w["k"], w["v"]
     torch.cuda.empty_cache()
 
     # ---- generation-time step
@@ -548,9 +560,11 @@ def oracle_sample(cfg, budget_s: float, max_steps: int | None = None):
     oc = oracle.Cache(base=base, L_hi=cfg["L_hi"], L_lo=cfg["L_lo"], batch=1, layers=1, kv_heads=1,
                       q_heads=G, block=blk, hi_cap=((n_high + nh_b + 15) // 16) * 16,
                       lo_cap=((T - n_high + blk + 15) // 16) * 16)
-    if base != oracle.BASE_AFFINE:
+    if base in (oracle.BASE_TQ, oracle.BASE_AFFINE_HAD):
         oc.signs = synthetic.signs(cfg["seed"], 1, H)[:, :1]
-    if base == oracle.BASE_TQ:
+    if base == oracle.BASE_TQ_DENSE:
+        oc.rotation = np.ascontiguousarray(synthetic.rotations(cfg["seed"], 1, H)[:, :1])
+    if base in (oracle.BASE_TQ, oracle.BASE_TQ_DENSE):
         _, c32, t32, _ = oracle.lloyd_max_gaussian(cfg["L_hi"])
         oc.cb_hi = (c32, t32)
         _, c32, t32, _ = oracle.lloyd_max_gaussian(cfg["L_lo"])
@@ -609,7 +623,8 @@ def main():
               "layers": cfg["NL"], "kv_heads": cfg["H"], "q_heads": cfg["Hq"],
               "levels": [cfg["L_hi"], cfg["L_lo"]], "r": f"{cfg['r'][0]}/{cfg['r'][1]}",
               "block": cfg["block"],
-              "base": {0: "affine", 1: "TQ-MSE", 2: "Hadamard-rotated affine"}[cfg["base"]],
+              "base": {0: "affine", 1: "TQ-MSE", 2: "Hadamard-rotated affine",
+                       3: "TQ-MSE, dense rotation"}[cfg["base"]],
               "step": "one generated token staged per step, block append every 128 steps"
               if cfg["mode"] == "token" else "append one 128-token block + decode every layer"}
 

@@ -64,7 +64,8 @@ typedef enum {
   SEMKV_EWORKSPACE = 6      /* workspace NULL or smaller than the size query says  */
 } semkv_status;
 
-enum { SEMKV_BASE_AFFINE = 0, SEMKV_BASE_TQ = 1, SEMKV_BASE_AFFINE_HAD = 2 };
+enum { SEMKV_BASE_AFFINE = 0, SEMKV_BASE_TQ = 1, SEMKV_BASE_AFFINE_HAD = 2,
+       SEMKV_BASE_TQ_DENSE = 3 };
 enum { SEMKV_HEAD_DIM = 128, SEMKV_MAX_LEVELS = 8 };
 
 /* Quantizer description (host struct; the pointers inside are device pointers).
@@ -82,6 +83,12 @@ enum { SEMKV_HEAD_DIM = 128, SEMKV_MAX_LEVELS = 8 };
  * base TQ: TurboQuant-MSE (Sec. 4.9): sign flip + unnormalised Walsh-Hadamard
  *   transform of the row, divided by the row's fp16 norm, then a Gaussian Lloyd-Max
  *   scalar codebook with L levels (thresholds strictly-greater: ties go low).
+ * base TQ_DENSE: TurboQuant-MSE with a dense random rotation (Sec. 4.9 "random
+ *   rotation"): w = M x with M the stored fp16 matrix ~ sqrt(128) Q (Q orthogonal) in
+ *   place of H S x; the rest as TQ (fp16 norm, u = w * fl(1/n), codebook).  w is formed
+ *   on the tensor cores (exact fp16 products, fp32 accumulation), so a code can differ
+ *   from the exactly rounded product's where u lies within rounding of a threshold.
+ *   Records as TQ; rows dequantize to (n/128) M^T cb[c].  Needs rotation + codebooks.
  * levels_hi / levels_lo: L for b_high / b_low, each in 2..8; equal = uniform. */
 typedef struct {
   int32_t base;
@@ -89,10 +96,13 @@ typedef struct {
   int32_t head_dim;                 /* must be 128 */
   const int8_t* signs;              /* TQ, AFFINE_HAD: device [layers][kv_heads][128]
                                        of +-1, 4-byte aligned                       */
-  const float* centroids_hi;        /* TQ: device [levels_hi]   ascending           */
+  const float* centroids_hi;        /* TQ, TQ_DENSE: device [levels_hi] ascending   */
   const float* thresholds_hi;       /* TQ: device [levels_hi-1] ascending           */
   const float* centroids_lo;        /* TQ: device [levels_lo]                       */
   const float* thresholds_lo;       /* TQ: device [levels_lo-1]                     */
+  const uint16_t* rotation;         /* TQ_DENSE: device fp16 [layers][kv_heads][128][128]
+                                       row-major (w_i = sum_j M_ij x_j), 16-byte
+                                       aligned; NULL for the other bases             */
 } semkv_quant_desc;
 
 /* One mixed-precision cache Ĉ_KV (Algorithm 1 output, extended by Algorithm 2).
@@ -189,8 +199,9 @@ semkv_status semkv_score_kv_norm(const uint16_t* x, int32_t batch, int32_t layer
 /* Token-wise quantization, Eq. 7 / Algorithm 1: quantize every row of the prompt
  * K/V with Q_{b_i} and write token i's record (for every layer and KV head) to
  * slot[b][i] of the high pool if is_high[b][i] else of the low pool; writes
- * hi_tok/lo_tok[b][slot] = i.  k, v: device fp16 [batch][layers][kv_heads][T][128].
- * is_high, slot: as produced by semkv_rank_assign for this T.  n_high: the number
+ * hi_tok/lo_tok[b][slot] = i.  k, v: device fp16 [batch][layers][kv_heads][T][128],
+ * 8-byte aligned (16-byte for TQ_DENSE, whose rows the tensor cores read; the same
+ * holds for the stage buffers in semkv_append_block).  is_high, slot: as produced by semkv_rank_assign for this T.  n_high: the number
  * of high tokens per sequence (used for the capacity check and the counts).
  * Sets cache->hi_count = n_high, lo_count = T - n_high, n_tokens = T and resets
  * stage_n to 0 (a prompt replaces whatever the cache held). */

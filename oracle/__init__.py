@@ -28,7 +28,7 @@ import numpy as np
 from .build import build_oracle
 
 D = 128
-BASE_AFFINE, BASE_TQ, BASE_AFFINE_HAD = 0, 1, 2
+BASE_AFFINE, BASE_TQ, BASE_AFFINE_HAD, BASE_TQ_DENSE = 0, 1, 2, 3
 
 _lib = None
 
@@ -64,9 +64,11 @@ def lib():
         L.orc_row_norm.restype = ctypes.c_float
         L.orc_quantize_tokens.argtypes = [i32, i32, i32, p, p, i32, i32, i32, i32, i32,
                                           p, p, i64, i64, i64, p, p, p, p, p, i64, i64,
-                                          p, p]
+                                          p, p, p]
         L.orc_quantize_tokens.restype = i32
-        L.orc_dequant_records.argtypes = [i32, i32, p, i64, p, p, p, p]
+        L.orc_dequant_records.argtypes = [i32, i32, p, i64, p, p, p, p, p]
+        L.orc_tq_dense_row.argtypes = [p, p, i32, p, p, p]
+        L.orc_tq_dense_w.argtypes = [p, p, p]
         L.orc_score_kv_norm.argtypes = [p, i32, i32, i32, i32, i32, i32, p]
         L.orc_fake_quant.argtypes = [i32, i32, i32, p, p, i32, i32, i32, i32, p, p, p, p, p, p,
                                      p, p]
@@ -192,6 +194,28 @@ def inv_sqrt_d() -> float:
     return float(lib().orc_inv_sqrt_d())
 
 
+def tq_dense_row(x_f16bits, rot_f16bits, L: int, thresholds):
+    """TurboQuant-MSE row under a dense rotation (fp16 matrix [128][128]).  Returns
+    (codes, norm fp16 bits)."""
+    x = np.ascontiguousarray(x_f16bits, dtype=np.uint16)
+    m = np.ascontiguousarray(rot_f16bits, dtype=np.uint16)
+    assert m.shape == (D, D)
+    thr = np.ascontiguousarray(thresholds, dtype=np.float32)
+    codes = np.zeros(D, dtype=np.uint8)
+    n = np.zeros(1, dtype=np.uint16)
+    lib().orc_tq_dense_row(_ptr(x), _ptr(m), L, _ptr(thr), _ptr(codes), _ptr(n))
+    return codes, int(n[0])
+
+
+def tq_dense_w(x_f16bits, rot_f16bits) -> np.ndarray:
+    """The rotated row w = M x of the dense TQ base (fp64 sum rounded to binary32)."""
+    x = np.ascontiguousarray(x_f16bits, dtype=np.uint16)
+    m = np.ascontiguousarray(rot_f16bits, dtype=np.uint16)
+    w = np.zeros(D, dtype=np.float32)
+    lib().orc_tq_dense_w(_ptr(x), _ptr(m), _ptr(w))
+    return w
+
+
 def fwht_f32(w) -> np.ndarray:
     a = np.array(w, dtype=np.float32)
     lib().orc_fwht_f32(_ptr(a))
@@ -313,6 +337,7 @@ class Cache:
     signs: np.ndarray = None          # [layers][kv_heads][128] int8 (TQ, rotated affine)
     cb_hi: tuple = None               # (centroids f32, thresholds f32) (TQ)
     cb_lo: tuple = None
+    rotation: np.ndarray = None       # [layers][kv_heads][128][128] fp16 bits (dense TQ)
 
     def __post_init__(self):
         B, NL, H = self.batch, self.layers, self.kv_heads
@@ -328,8 +353,18 @@ class Cache:
         if self.signs is None:
             self.signs = np.ones((NL, H, D), np.int8)
 
+    def _rot(self, layer=None, head=None):
+        """The dense rotation (fp16 bits) of every (layer, head), or of one, or None."""
+        if self.rotation is None:
+            return None
+        r = np.ascontiguousarray(self.rotation, dtype=np.uint16)
+        if layer is not None:
+            r = np.ascontiguousarray(r[layer, head])
+        self._rot_keep = r
+        return _ptr(r)
+
     def _thr(self, which):
-        if self.base != BASE_TQ:
+        if self.base not in (BASE_TQ, BASE_TQ_DENSE):
             return np.zeros(1, np.float32)
         return np.ascontiguousarray((self.cb_hi if which == "hi" else self.cb_lo)[1],
                                     dtype=np.float32)
@@ -351,7 +386,7 @@ def quantize_tokens(cache: Cache, k, v, n: int, is_high, slot, hi_base, lo_base,
                                    lo_base, tok_base, _ptr(signs), _ptr(thr_hi),
                                    _ptr(thr_lo), _ptr(cache.hi_pool), _ptr(cache.lo_pool),
                                    cache.hi_cap, cache.lo_cap, _ptr(cache.hi_tok),
-                                   _ptr(cache.lo_tok))
+                                   _ptr(cache.lo_tok), cache._rot())
     if rc != 0:
         raise ValueError("pool capacity exceeded")
 
@@ -393,7 +428,7 @@ def append_block(cache: Cache, r_num: int, r_den: int):
     cache.stage_n = 0
 
 
-def dequant_records(base: int, L: int, recs, signs_lh, centroids):
+def dequant_records(base: int, L: int, recs, signs_lh, centroids, rot_lh=None):
     """Exact fp64 rows of `count` records: affine z + s c; TQ (n/128) S H cb[c]."""
     recs = np.ascontiguousarray(recs, dtype=np.uint8)
     count = recs.shape[0]
@@ -402,8 +437,9 @@ def dequant_records(base: int, L: int, recs, signs_lh, centroids):
     sg = np.ascontiguousarray(signs_lh if signs_lh is not None else np.ones(D), np.int8)
     cb = np.ascontiguousarray(centroids if centroids is not None else np.zeros(1),
                               dtype=np.float64)
+    rot = None if rot_lh is None else np.ascontiguousarray(rot_lh, dtype=np.uint16)
     lib().orc_dequant_records(base, L, _ptr(recs), count, _ptr(sg), _ptr(cb),
-                              _ptr(kout), _ptr(vout))
+                              _ptr(kout), _ptr(vout), None if rot is None else _ptr(rot))
     return kout, vout
 
 
@@ -413,10 +449,11 @@ def dequant_cache_head(cache: Cache, b: int, layer: int, h: int):
     cb_hi = cache.cb_hi[0] if cache.cb_hi is not None else None
     cb_lo = cache.cb_lo[0] if cache.cb_lo is not None else None
     sg = cache.signs[layer, h]
+    rot = None if cache.rotation is None else cache.rotation[layer, h]
     kh, vh = dequant_records(cache.base, cache.L_hi,
-                             cache.hi_pool[b, layer, h, :cache.hi_count], sg, cb_hi)
+                             cache.hi_pool[b, layer, h, :cache.hi_count], sg, cb_hi, rot)
     kl, vl = dequant_records(cache.base, cache.L_lo,
-                             cache.lo_pool[b, layer, h, :cache.lo_count], sg, cb_lo)
+                             cache.lo_pool[b, layer, h, :cache.lo_count], sg, cb_lo, rot)
     n = cache.stage_n
     ks = f16_bits_to_f32(cache.stage_k[b, layer, h, :n]).astype(np.float64)
     vs = f16_bits_to_f32(cache.stage_v[b, layer, h, :n]).astype(np.float64)
@@ -464,7 +501,7 @@ def paper_code_bits(L: int) -> float:
 
 def metadata_bits(base: int) -> float:
     """fp16 metadata per value: two per 128-row for affine (0.25), one for TQ."""
-    return (1 if base == BASE_TQ else 2) * 16 / D
+    return (1 if base in (BASE_TQ, BASE_TQ_DENSE) else 2) * 16 / D
 
 
 def effective_bits(base: int, L_hi: int, L_lo: int, r: float) -> float:
@@ -502,6 +539,8 @@ def fake_quant(base: int, L_hi: int, L_lo: int, k, v, is_high=None, signs=None,
     every token at L_hi) and reconstruct to fp16 in binary32 in the order of
     orc_fake_quant.  k, v: fp16 bits [B][NL][H][T][128]; cb_*: (centroids, thresholds)
     fp32 for TQ.  Returns (k_out, v_out) fp16 bits."""
+    if base == BASE_TQ_DENSE:
+        raise NotImplementedError("fake quantization covers the affine, rotated affine and TQ bases")
     k = np.ascontiguousarray(k, dtype=np.uint16)
     v = np.ascontiguousarray(v, dtype=np.uint16)
     B, NL, H, T, d = k.shape

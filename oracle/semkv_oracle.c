@@ -12,6 +12,8 @@
  *    "Memory accounting": two FP16 parameters per head-token row of dim 128).
  *  - The same affine quantizer on Hadamard-rotated rows (Sec. 4.1: rotation before
  *    the per-row quantizer): orthonormal (1/sqrt 128) H S, offset rounded down.
+ *  - TurboQuant-MSE rows with a stored dense random orthogonal rotation (Sec. 4.9
+ *    "random rotation"), the rotated row taken as an fp64 sum rounded to binary32.
  *  - TurboQuant-MSE rows (Sec. 4.9): random sign flip + Walsh-Hadamard rotation,
  *    row norm stored in fp16, Gaussian Lloyd-Max codebook with L levels.
  *  - Mixed-radix packing at the paper's rates (Sec. 4.1: 3 five-level codes in
@@ -187,7 +189,7 @@ int orc_row_bytes(int L) {
 int orc_record_bytes(int base, int L) {
   int rb = orc_row_bytes(L);
   if (rb == 0) return 0;
-  return 2 * rb + (base == 1 ? 4 : 8);
+  return 2 * rb + ((base == 1 || base == 3) ? 4 : 8);
 }
 
 static void put_bits(uint8_t* row, int pos, uint64_t val, int nbits) {
@@ -415,6 +417,45 @@ void orc_tq_row(const uint16_t* x, const int8_t* sgn, int L, const float* thr,
   *n_out = n16;
 }
 
+/* TurboQuant-MSE row with a dense random rotation (Sec. 4.9: "random rotation" before
+ * the Lloyd-Max codebook; here a stored orthogonal matrix instead of the randomized
+ * Hadamard transform).  rot: the fp16 matrix M ~ sqrt(128) Q (Q orthogonal), row-major
+ * [128][128] fp16 bits, so that w = M x plays the part of H S x:
+ *   w_i = sum_j M_ij x_j                 (exact products, summed in fp64 in index order,
+ *                                        rounded once to binary32)
+ *   n16 = fp16(||x||) (the fixed tree of orc_row_norm); u_i = w_i * fl(1/n);
+ *   c_i = #{k : u_i > thr_k}; all codes 0 when n == 0. */
+void orc_tq_dense_w(const uint16_t* x, const uint16_t* rot, float* w) {
+  for (int i = 0; i < D; i++) {
+    double acc = 0.0;
+    for (int j = 0; j < D; j++)
+      acc += (double)orc_f16_to_f32(rot[i * D + j]) * (double)orc_f16_to_f32(x[j]);
+    w[i] = (float)acc;
+  }
+}
+
+void orc_tq_dense_row(const uint16_t* x, const uint16_t* rot, int L, const float* thr,
+                      uint8_t* codes, uint16_t* n_out) {
+  float xf[D], w[D];
+  for (int j = 0; j < D; j++) xf[j] = orc_f16_to_f32(x[j]);
+  orc_tq_dense_w(x, rot, w);
+  uint16_t n16 = f16_param(orc_row_norm(xf));
+  float n = orc_f16_to_f32(n16);
+  if (n == 0.0f) {
+    memset(codes, 0, D);
+  } else {
+    float inv = 1.0f / n;
+    for (int j = 0; j < D; j++) {
+      float u = w[j] * inv;
+      int c = 0;
+      for (int k = 0; k < L - 1; k++)
+        if (u > thr[k]) c++;
+      codes[j] = (uint8_t)c;
+    }
+  }
+  *n_out = n16;
+}
+
 /* --------------------------------------------------------- whole cache -------- */
 
 /* Quantize tokens 0..n-1 of a source K/V tensor [B][NL][H][Tsrc][128] (fp16 bits)
@@ -428,7 +469,8 @@ int orc_quantize_tokens(int base, int Lhi, int Llo, const uint16_t* k, const uin
                         const uint32_t* slot, int64_t hi_base, int64_t lo_base,
                         int64_t tok_base, const int8_t* signs, const float* thr_hi,
                         const float* thr_lo, uint8_t* hi_pool, uint8_t* lo_pool,
-                        int64_t hi_cap, int64_t lo_cap, int32_t* hi_tok, int32_t* lo_tok) {
+                        int64_t hi_cap, int64_t lo_cap, int32_t* hi_tok, int32_t* lo_tok,
+                        const uint16_t* rot) {
   int rec_hi = orc_record_bytes(base, Lhi), rec_lo = orc_record_bytes(base, Llo);
   for (int b = 0; b < B; b++) {
     for (int i = 0; i < n; i++) {
@@ -460,6 +502,13 @@ int orc_quantize_tokens(int base, int Lhi, int Llo, const uint16_t* k, const uin
             orc_affine_had_row(k + row, sg, L, ck, &p[0], &p[1]);
             orc_affine_had_row(v + row, sg, L, cv, &p[2], &p[3]);
             memcpy(r + 2 * rb, p, 8);
+          } else if (base == 3) {
+            uint16_t p[2];
+            const uint16_t* m = rot + ((int64_t)l * H + h) * D * D;
+            const float* thr = hi ? thr_hi : thr_lo;
+            orc_tq_dense_row(k + row, m, L, thr, ck, &p[0]);
+            orc_tq_dense_row(v + row, m, L, thr, cv, &p[1]);
+            memcpy(r + 2 * rb, p, 4);
           } else {
             uint16_t p[2];
             const int8_t* sg = signs + ((int64_t)l * H + h) * D;
@@ -491,10 +540,11 @@ static void fwht_f64(double* w) {
 /* Dequantize `count` records of one (b, layer, head) into exact fp64 rows.
  *  affine:         x^ = z + s * c                        (exact in fp64)
  *  rotated affine: x^ = S H (z + s * c) / sqrt(128)      (the rotation's inverse)
- *  TQ:             x^ = (n / 128) * S H cb[c]   (x = S H (H S x) / 128, H H = 128 I) */
+ *  TQ:             x^ = (n / 128) * S H cb[c]   (x = S H (H S x) / 128, H H = 128 I)
+ *  dense TQ:       x^ = (n / 128) * M^T cb[c]   (M = rot, M M^T ~ 128 I) */
 void orc_dequant_records(int base, int L, const uint8_t* recs, int64_t count,
                          const int8_t* sgn, const double* centroids, double* kout,
-                         double* vout) {
+                         double* vout, const uint16_t* rot) {
   int rb = orc_row_bytes(L), rec = orc_record_bytes(base, L);
   for (int64_t i = 0; i < count; i++) {
     const uint8_t* r = recs + i * rec;
@@ -502,7 +552,7 @@ void orc_dequant_records(int base, int L, const uint8_t* recs, int64_t count,
     orc_unpack_row(r, L, ck);
     orc_unpack_row(r + rb, L, cv);
     uint16_t p[4];
-    memcpy(p, r + 2 * rb, base == 1 ? 4 : 8);
+    memcpy(p, r + 2 * rb, (base == 1 || base == 3) ? 4 : 8);
     double* ko = kout + i * D;
     double* vo = vout + i * D;
     if (base == 0 || base == 2) {
@@ -520,6 +570,18 @@ void orc_dequant_records(int base, int L, const uint8_t* recs, int64_t count,
           ko[j] = ko[j] * sgn[j] * r;
           vo[j] = vo[j] * sgn[j] * r;
         }
+      }
+    } else if (base == 3) {
+      double kn = orc_f16_to_f32(p[0]), vn = orc_f16_to_f32(p[1]);
+      for (int d = 0; d < D; d++) {
+        double sk = 0.0, sv = 0.0;
+        for (int i2 = 0; i2 < D; i2++) {
+          const double m = orc_f16_to_f32(rot[i2 * D + d]);
+          sk += m * centroids[ck[i2]];
+          sv += m * centroids[cv[i2]];
+        }
+        ko[d] = sk * kn / D;
+        vo[d] = sv * vn / D;
       }
     } else {
       double kn = orc_f16_to_f32(p[0]), vn = orc_f16_to_f32(p[1]);

@@ -19,12 +19,18 @@ semkv_status check_desc(const semkv_quant_desc* d) {
   if (!d) return SEMKV_EINVAL;
   if (d->head_dim != SEMKV_HEAD_DIM) return SEMKV_EUNSUPPORTED;
   if (d->base != SEMKV_BASE_AFFINE && d->base != SEMKV_BASE_TQ &&
-      d->base != SEMKV_BASE_AFFINE_HAD)
+      d->base != SEMKV_BASE_AFFINE_HAD && d->base != SEMKV_BASE_TQ_DENSE)
     return SEMKV_EUNSUPPORTED;
   if (!level_ok(d->levels_hi) || !level_ok(d->levels_lo)) return SEMKV_EUNSUPPORTED;
   if (d->base == SEMKV_BASE_AFFINE_HAD) {
     if (!d->signs) return SEMKV_EINVAL;
     if (!aligned(d->signs, 4)) return SEMKV_EALIGN;
+  }
+  if (d->base == SEMKV_BASE_TQ_DENSE) {
+    if (!d->rotation || !d->thresholds_hi || !d->thresholds_lo || !d->centroids_hi ||
+        !d->centroids_lo)
+      return SEMKV_EINVAL;
+    if (!aligned(d->rotation, 16)) return SEMKV_EALIGN;
   }
   if (d->base == SEMKV_BASE_TQ) {
     if (!d->signs || !d->thresholds_hi || !d->thresholds_lo || !d->centroids_hi ||
@@ -75,9 +81,7 @@ extern "C" {
 size_t semkv_row_bytes(int32_t levels) { return level_ok(levels) ? (size_t)row_bytes_rt(levels) : 0; }
 
 size_t semkv_record_bytes(int32_t base, int32_t levels) {
-  if (!level_ok(levels) ||
-      (base != SEMKV_BASE_AFFINE && base != SEMKV_BASE_TQ && base != SEMKV_BASE_AFFINE_HAD))
-    return 0;
+  if (!level_ok(levels) || base < SEMKV_BASE_AFFINE || base > SEMKV_BASE_TQ_DENSE) return 0;
   return (size_t)record_bytes_rt(base, levels);
 }
 
@@ -173,6 +177,7 @@ semkv_status semkv_fake_quant(const semkv_quant_desc* desc, const uint16_t* k, c
                               void* stream) {
   semkv_status s = check_desc(desc);
   if (s != SEMKV_OK) return s;
+  if (desc->base == SEMKV_BASE_TQ_DENSE) return SEMKV_EUNSUPPORTED;
   if (!k || !v || !k_out || !v_out || batch < 1 || layers < 1 || kv_heads < 1 || T < 1)
     return SEMKV_EINVAL;
   if (!aligned(k, 8) || !aligned(v, 8) || !aligned(k_out, 8) || !aligned(v_out, 8))
@@ -226,6 +231,8 @@ semkv_status semkv_quantize_pack(const semkv_quant_desc* desc, const uint16_t* k
   if (s != SEMKV_OK) return s;
   if (!k || !v || !is_high || !slot || T < 1) return SEMKV_EINVAL;
   if (!aligned(k, 8) || !aligned(v, 8)) return SEMKV_EALIGN;
+  if (desc->base == SEMKV_BASE_TQ_DENSE && (!aligned(k, 16) || !aligned(v, 16)))
+    return SEMKV_EALIGN;  // the rows are staged in 16-byte chunks
   if (n_high > (uint32_t)T) return SEMKV_EINVAL;
   if ((int64_t)n_high > cache->hi_cap || (int64_t)(T - n_high) > cache->lo_cap)
     return SEMKV_ECAPACITY;
@@ -246,6 +253,7 @@ semkv_status semkv_quantize_pack(const semkv_quant_desc* desc, const uint16_t* k
   a.lo_base = 0;
   a.tok_base = 0;
   a.signs = desc->signs;
+  a.rot = desc->rotation;
   a.thr_hi = desc->thresholds_hi;
   a.thr_lo = desc->thresholds_lo;
   a.hi_pool = cache->hi_pool;
@@ -277,6 +285,9 @@ semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache
       !cache->blk_slot)
     return SEMKV_EINVAL;
   if (!aligned(cache->stage_k, 8) || !aligned(cache->stage_v, 8)) return SEMKV_EALIGN;
+  if (desc->base == SEMKV_BASE_TQ_DENSE &&
+      (!aligned(cache->stage_k, 16) || !aligned(cache->stage_v, 16)))
+    return SEMKV_EALIGN;
   const uint32_t n_high = semkv_block_high_count((uint32_t)n, r_num, r_den);
   if (cache->hi_count + n_high > cache->hi_cap || cache->lo_count + (n - n_high) > cache->lo_cap)
     return SEMKV_ECAPACITY;
@@ -309,6 +320,7 @@ semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache
   a.lo_base = cache->lo_count;
   a.tok_base = cache->n_tokens;
   a.signs = desc->signs;
+  a.rot = desc->rotation;
   a.thr_hi = desc->thresholds_hi;
   a.thr_lo = desc->thresholds_lo;
   a.hi_pool = cache->hi_pool;
@@ -375,6 +387,7 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
   a.partials = reinterpret_cast<float*>(ws);
   a.signs = desc->signs;
+  a.rot = desc->rotation;
   a.cb_hi = desc->centroids_hi;
   a.cb_lo = desc->centroids_lo;
   // rotated queries (TQ and rotated affine bases) after the split-K partials

@@ -55,7 +55,7 @@ __host__ __device__ inline int row_bytes_rt(int L) {
 }
 __host__ __device__ inline int record_bytes_rt(int base, int L) {
   int rb = row_bytes_rt(L);
-  return rb == 0 ? 0 : 2 * rb + (base == SEMKV_BASE_TQ ? 4 : 8);
+  return rb == 0 ? 0 : 2 * rb + ((base == SEMKV_BASE_TQ || base == SEMKV_BASE_TQ_DENSE) ? 4 : 8);
 }
 
 // --------------------------------------------------------------- helpers ------

@@ -883,8 +883,9 @@ __global__ void qrot_kernel(DecodeArgs a) {
   const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (gw >= a.B * a.Hq) return;
   const int b = gw / a.Hq, qh = gw % a.Hq, h = qh / (a.Hq / a.H);
-  const int8_t* sg = a.signs + ((int64_t)a.layer * a.H + h) * 128;
   const uint16_t* qrow = a.q + ((int64_t)b * a.Hq + qh) * 128;
+
+  const int8_t* sg = a.signs + ((int64_t)a.layer * a.H + h) * 128;
   float w[4];
 #pragma unroll
   for (int j = 0; j < 4; ++j) w[j] = f16_to_f32(qrow[4 * lane + j]) * (float)sg[4 * lane + j];
@@ -903,6 +904,35 @@ __global__ void qrot_kernel(DecodeArgs a) {
   float* dst = a.qrot + ((int64_t)b * a.Hq + qh) * 128 + 4 * lane;
 #pragma unroll
   for (int j = 0; j < 4; ++j) dst[j] = w[j] * rs;
+}
+
+// Dense rotation: q' = M q for the G query heads of each (sequence, KV head); one block
+// of 128 threads per pair, thread i taking row i of M (16 independent 16-byte loads)
+// against the group's queries staged in shared memory.
+__global__ void qrot_dense_kernel(DecodeArgs a) {
+  __shared__ float qs[8][128];
+  const int b = blockIdx.x / a.H, h = blockIdx.x % a.H;
+  const int G = a.Hq / a.H, i = threadIdx.x;
+  for (int x = threadIdx.x; x < G * 128; x += blockDim.x)
+    qs[x >> 7][x & 127] = f16_to_f32(a.q[((int64_t)b * a.Hq + h * G) * 128 + x]);
+  __syncthreads();
+  const uint4* row = reinterpret_cast<const uint4*>(a.rot + (((int64_t)a.layer * a.H + h) * 128 + i) * 128);
+  uint4 m[16];
+#pragma unroll
+  for (int c = 0; c < 16; ++c) m[c] = row[c];
+  for (int g = 0; g < G; ++g) {
+    float acc = 0.0f;
+#pragma unroll
+    for (int c = 0; c < 16; ++c) {
+      const uint32_t w[4] = {m[c].x, m[c].y, m[c].z, m[c].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        acc = fmaf(f16_to_f32((uint16_t)(w[e] & 0xFFFF)), qs[g][8 * c + 2 * e], acc);
+        acc = fmaf(f16_to_f32((uint16_t)(w[e] >> 16)), qs[g][8 * c + 2 * e + 1], acc);
+      }
+    }
+    a.qrot[((int64_t)b * a.Hq + h * G + g) * 128 + i] = acc;
+  }
 }
 
 // ------------------------------------------------------- fp16 stage tokens ----
@@ -1109,7 +1139,9 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
     merged[qh * 128 + d] = (kind == 0 || kind == 3) ? o + mg.cta_z[qh] : o;
   }
   __syncthreads();
-  const bool rotated = kind == 1 || kind == 3;
+  // (dense-rotation partials stay in the rotated domain: the combine turns their sum
+  // back once per head)
+  const bool rotated = (kind == 1 || kind == 3) && a.base != SEMKV_BASE_TQ_DENSE;
   if (rotated) {
     // back from the rotated domain: o = S H o' (unnormalised transform, stages 1..64)
     for (int hs = 1; hs < 128; hs <<= 1) {
@@ -1347,14 +1379,49 @@ __global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs
 // merge the partials of each (b, qh): one warp per head, 4 dims per lane.  The lanes
 // first take the partials' maxima and weights in parallel (weights kept in shared
 // memory), then sum the rows with independent loads.
+// o = M^T o' for one head (dense rotation): lane l holds dims 4l..4l+3 of o' on entry
+// and of o on return; buf is the warp's 128-float scratch, ms the pair's M in shared memory
+__device__ __forceinline__ void dense_back(const uint16_t* ms, float* buf, float (&o)[4],
+                                           int lane) {
+#pragma unroll
+  for (int e = 0; e < 4; ++e) buf[4 * lane + e] = o[e];
+  __syncwarp();
+  const uint16_t* m = ms + 4 * lane;
+  float u[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
+  for (int j = 0; j < 128; ++j) {
+    const uint2 mm = *reinterpret_cast<const uint2*>(m + j * 128);
+    const float x = buf[j];
+    u[0] = fmaf(f16_to_f32((uint16_t)(mm.x & 0xFFFF)), x, u[0]);
+    u[1] = fmaf(f16_to_f32((uint16_t)(mm.x >> 16)), x, u[1]);
+    u[2] = fmaf(f16_to_f32((uint16_t)(mm.y & 0xFFFF)), x, u[2]);
+    u[3] = fmaf(f16_to_f32((uint16_t)(mm.y >> 16)), x, u[3]);
+  }
+#pragma unroll
+  for (int e = 0; e < 4; ++e) o[e] = u[e];
+  __syncwarp();
+}
+
+// DENSE: one block of G warps per (sequence, KV head), the pair's rotation staged in
+// shared memory for the final M^T.
+template <bool DENSE>
 __global__ void combine_kernel(DecodeArgs a) {
   constexpr int kHeadsPerCta = 8;
   __shared__ float wsm[kHeadsPerCta][kMaxPartialsPerPair];
+  __shared__ float orot[DENSE ? kHeadsPerCta : 1][128];
+  __shared__ __align__(16) uint16_t ms[DENSE ? 128 * 128 : 8];
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
-  const int gw = blockIdx.x * kHeadsPerCta + wib;
+  const int G = a.Hq / a.H;
+  const int gw = DENSE ? (int)blockIdx.x * G + wib : (int)blockIdx.x * kHeadsPerCta + wib;
+  if constexpr (DENSE) {
+    const int hh = (int)blockIdx.x % a.H;
+    const uint4* src = reinterpret_cast<const uint4*>(a.rot + ((int64_t)a.layer * a.H + hh) * 128 * 128);
+    for (int x = threadIdx.x; x < 128 * 16; x += blockDim.x) reinterpret_cast<uint4*>(ms)[x] = src[x];
+    __syncthreads();
+  }
   if (gw >= a.B * a.Hq) return;
   const int b = gw / a.Hq, qh = gw % a.Hq;
-  const int G = a.Hq / a.H, h = qh / G, c = qh % G;
+  const int h = qh / G, c = qh % G;
   const int64_t bh = (int64_t)b * a.H + h;
   const int S = pair_partials(a.plan, bh);
   const float* base = a.partials + bh * a.plan.stride * kPartialFloats;
@@ -1372,9 +1439,14 @@ __global__ void combine_kernel(DecodeArgs a) {
 #pragma unroll
   for (int off = 16; off >= 1; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
   __syncwarp();
+  // dense rotation: the pool partials (all but the staged tail's, which comes last) are
+  // in the rotated domain; their weighted sum is turned back with M^T before the tail's
+  // partial is added
+  const int S_rot = DENSE ? S - a.plan.splits_st : -1;
   float o[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll 4
   for (int s = 0; s < S; ++s) {
+    if (DENSE && s == S_rot) dense_back(ms, orot[wib], o, lane);
     const float sc = wsm[wib][s];
     if (sc == 0.0f) continue;
     const float4 v = *reinterpret_cast<const float4*>(base + s * kPartialFloats + 16 + c * 128 + 4 * lane);
@@ -1383,6 +1455,7 @@ __global__ void combine_kernel(DecodeArgs a) {
     o[2] += sc * v.z;
     o[3] += sc * v.w;
   }
+  if (DENSE && S_rot == S) dense_back(ms, orot[wib], o, lane);  // no staged tail
   const float inv = 1.0f / lsum;
   float4 r = make_float4(o[0] * inv, o[1] * inv, o[2] * inv, o[3] * inv);
   *reinterpret_cast<float4*>(a.out + ((int64_t)b * a.Hq + qh) * 128 + 4 * lane) = r;
@@ -1530,7 +1603,14 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
   const DecodePlan& P = a.plan;
   if (P.stride < 1 || P.stride > kMaxSplits + 1) return cudaErrorInvalidValue;
   cudaError_t e = cudaSuccess;
-  if (a.base == SEMKV_BASE_TQ) {
+  if (a.base == SEMKV_BASE_TQ_DENSE) {
+    qrot_dense_kernel<<<a.B * a.H, 128, 0, stream>>>(a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int pool_splits = P.splits_hi + P.splits_lo;
+    if (pool_splits > 0)
+      decode_kernel<1><<<dim3(pool_splits, a.H, a.B), kThreads, kRingBytes + kAqBytes, stream>>>(a);
+  } else if (a.base == SEMKV_BASE_TQ) {
     const int heads = a.B * a.Hq;
     qrot_kernel<<<(heads + 7) / 8, 256, 0, stream>>>(a);
     e = cudaGetLastError();
@@ -1556,7 +1636,10 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
   }
   const int heads = a.B * a.Hq;
-  combine_kernel<<<(heads + 7) / 8, 256, 0, stream>>>(a);
+  if (a.base == SEMKV_BASE_TQ_DENSE)
+    combine_kernel<true><<<a.B * a.H, 32 * (a.Hq / a.H), 0, stream>>>(a);
+  else
+    combine_kernel<false><<<(heads + 7) / 8, 256, 0, stream>>>(a);
   return cudaGetLastError();
 }
 

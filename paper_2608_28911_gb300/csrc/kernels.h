@@ -16,6 +16,7 @@ struct QuantArgs {
   const uint32_t* slot;     // [B][n]
   int64_t hi_base, lo_base, tok_base;
   const int8_t* signs;      // [NL][H][128] (TQ)
+  const uint16_t* rot;      // [NL][H][128][128] fp16 (dense TQ)
   const float* thr_hi;
   const float* thr_lo;
   uint8_t* hi_pool;
@@ -96,6 +97,7 @@ struct DecodeArgs {
   float scale_log2;          // softmax scale * log2(e)
   float* partials;           // [B][H][splits][kPartialFloats]
   const int8_t* signs;       // TQ
+  const uint16_t* rot;       // dense TQ: [NL][H][128][128] fp16
   const float* cb_hi;        // TQ centroids
   const float* cb_lo;
   float* qrot;               // TQ: [B][Hq][128] rotated queries (workspace)

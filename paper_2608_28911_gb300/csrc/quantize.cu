@@ -22,6 +22,7 @@ namespace semkv {
 namespace {
 
 constexpr int kWarpsPerBlock = 8;
+constexpr uint32_t kSpinLimitQ = 1u << 22;  // bounded mbarrier polls
 constexpr int kMaxRecWords = 27;  // largest record: affine L=7/8, 2*48+8 = 104 B
 
 struct RowOut {
@@ -563,6 +564,253 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) fake_quant_kernel(FakeArg
   }
 }
 
+// ------------------------------------- dense-rotation TQ rows (tcgen05) --------
+// One CTA of 4 warps per 64 tokens of one (sequence, layer, KV head).  The 128 rows
+// of the tile (K and V of each token, rows 2i and 2i+1) are rotated on the tensor
+// cores: W[r][i] = sum_j X[r][j] M[i][j], tcgen05.mma kind::f16 with M = N = 128 and
+// K = 8 x 16, both operands K-major in shared memory without swizzle, the fp32
+// accumulator in tensor memory (128 lanes x 128 columns).  Thread r then owns row r:
+// the fixed-tree norm (from the staged row, while the MMAs run), the TMEM row, the
+// codes.  The warps pack the records as in quantize_pair.
+constexpr int kDenseTok = 64;
+constexpr uint32_t kDenseTile = 128 * 128 * 2;  // bytes of one operand tile
+// instruction descriptor: fp32 accumulate (bits 4-5 = 1), A and B fp16 (formats 0),
+// both K-major, N >> 3 at bits 17-22, M >> 4 at bits 24-28
+constexpr uint32_t kDenseIdesc = (1u << 4) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
+
+// core-matrix layout of a [128][128] fp16 K-major tile: 8 rows x 16 bytes per core
+// matrix, core matrices 128 bytes apart along K and 2048 bytes apart along rows; the
+// 16-byte chunk c = (rg, kg, rr) (rr fastest) sits at byte 16 c
+__device__ __forceinline__ uint32_t dense_off(int r, int k) {
+  return (uint32_t)((r >> 3) * 2048 + (k >> 3) * 128 + (r & 7) * 16 + (k & 7) * 2);
+}
+// shared-memory matrix descriptor: start >> 4 (bits 0-13), leading (K) core-matrix
+// offset 128 >> 4 (bits 16-29), stride (row-group) offset 2048 >> 4 (bits 32-45),
+// descriptor version 1 (bits 46-47), no swizzle
+__device__ __forceinline__ uint64_t dense_desc(uint32_t saddr) {
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)(128u >> 4) << 16) |
+         ((uint64_t)(2048u >> 4) << 32) | ((uint64_t)1 << 46);
+}
+__device__ __forceinline__ uint32_t dsmem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+// 32 columns of this warp's 32 TMEM lanes (lane i of the warp <- TMEM lane 32w + i)
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+        "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+        "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+        "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+template <int L>
+__device__ __forceinline__ void dense_pack(const uint8_t* codes, uint16_t nk, uint16_t nv,
+                                           uint8_t* dst, uint32_t* rec, int lane) {
+  using F = Fmt<L>;
+  constexpr int kRecWords = (2 * F::RB + 4) / 4;
+  if (lane < kRecWords) rec[lane] = 0u;
+  __syncwarp();
+  pack_rows<L>(codes, rec, lane);
+  if (lane == 0) rec[(2 * F::RB) / 4] = (uint32_t)nk | ((uint32_t)nv << 16);
+  __syncwarp();
+  if (lane < kRecWords) reinterpret_cast<uint32_t*>(dst)[lane] = rec[lane];
+  __syncwarp();
+}
+
+__global__ void __launch_bounds__(128) quantize_tq_dense_kernel(QuantArgs a) {
+  extern __shared__ __align__(1024) uint8_t dsm[];
+  uint8_t* xa = dsm;               // A: the tile's rows; after the MMAs, their codes
+  uint8_t* mb = dsm + kDenseTile;  // B: the rotation of (layer, head)
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ uint32_t tmem_base;
+  __shared__ uint16_t nrm[128];
+  __shared__ __align__(16) uint32_t rec_sm[4][kMaxRecWords + 1];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t bhs = (int64_t)a.B * a.NL * a.H;
+  const int t0 = blockIdx.x * kDenseTok;
+
+  if (tid == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(dsmem_u32(&bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 128;" ::"r"(
+                     dsmem_u32(&tmem_base))
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tb = tmem_base;
+
+  uint32_t phase = 0;
+  bool ok = true;
+  for (int64_t bhl = blockIdx.y; bhl < bhs && ok; bhl += gridDim.y) {
+    const int h = (int)(bhl % a.H);
+    const int l = (int)((bhl / a.H) % a.NL);
+    const int b = (int)(bhl / ((int64_t)a.H * a.NL));
+    // ---- stage both operands (16-byte chunk c goes to byte 16 c)
+    const uint4* msrc = reinterpret_cast<const uint4*>(a.rot + ((int64_t)l * a.H + h) * 128 * 128);
+    const int64_t row0 = (((int64_t)b * a.NL + l) * a.H + h) * a.Tsrc;
+    for (int c = tid; c < 128 * 16; c += 128) {
+      const int rr = c & 7, kg = (c >> 3) & 15, r = (c >> 7) * 8 + rr;
+      reinterpret_cast<uint4*>(mb)[c] = msrc[r * 16 + kg];
+      const int t = t0 + (r >> 1);
+      uint4 x = make_uint4(0u, 0u, 0u, 0u);
+      if (t < a.n) {
+        const uint16_t* src = ((r & 1) ? a.v : a.k) + (row0 + t) * 128;
+        x = reinterpret_cast<const uint4*>(src)[kg];
+      }
+      reinterpret_cast<uint4*>(xa)[c] = x;
+    }
+    // generic-proxy writes -> visible to the tensor cores (async proxy)
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    if (tid == 0) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const uint64_t da = dense_desc(dsmem_u32(xa) + k * 256);
+        const uint64_t db = dense_desc(dsmem_u32(mb) + k * 256);
+        asm volatile(
+            "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n"
+            " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tb),
+            "l"(da), "l"(db), "r"(kDenseIdesc), "r"((uint32_t)(k > 0))
+            : "memory");
+      }
+      asm volatile(
+          "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+              dsmem_u32(&bar))
+          : "memory");
+    }
+    // ---- row norm with the fixed tree (32 in-order partials of 4 squares, then the
+    // pairwise stages 16, 8, 4, 2, 1), from the staged row while the MMAs run
+    {
+      float p[32];
+#pragma unroll
+      for (int g = 0; g < 32; ++g) {
+        const uint2 u = *reinterpret_cast<const uint2*>(xa + dense_off(tid, 4 * g));
+        const float x0 = f16_to_f32((uint16_t)(u.x & 0xFFFF)), x1 = f16_to_f32((uint16_t)(u.x >> 16));
+        const float x2 = f16_to_f32((uint16_t)(u.y & 0xFFFF)), x3 = f16_to_f32((uint16_t)(u.y >> 16));
+        float acc = __fmul_rn(x0, x0);
+        acc = __fadd_rn(acc, __fmul_rn(x1, x1));
+        acc = __fadd_rn(acc, __fmul_rn(x2, x2));
+        p[g] = __fadd_rn(acc, __fmul_rn(x3, x3));
+      }
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1)
+#pragma unroll
+        for (int g = 0; g < off; ++g) p[g] = __fadd_rn(p[g], p[g + off]);
+      nrm[tid] = f16_param(__fsqrt_rn(p[0]));
+    }
+    ok = false;
+    for (uint32_t i = 0; i < kSpinLimitQ && !ok; ++i) {
+      uint32_t r;
+      asm volatile(
+          "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+          " selp.u32 %0, 1, 0, p;\n}"
+          : "=r"(r)
+          : "r"(dsmem_u32(&bar)), "r"(phase)
+          : "memory");
+      ok = r != 0;
+    }
+    phase ^= 1u;
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    ok = __syncthreads_and(ok) != 0;  // every norm is taken: the A tile may now hold the codes
+    if (!ok) {
+      if (tid == 0) raise_error(a.err, kDevWaitTimeout);
+      break;
+    }
+    // ---- codes of row tid: u = w * fl(1/n), c = #{k : u > thr_k}
+    {
+      const int t = t0 + (tid >> 1);
+      const bool hi = t < a.n && a.is_high[(int64_t)b * a.n + t] != 0;
+      const int L = hi ? a.L_hi : a.L_lo;
+      const float* thr_g = hi ? a.thr_hi : a.thr_lo;
+      float thr[7];
+#pragma unroll
+      for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? thr_g[k] : INFINITY;
+      const float n = f16_to_f32(nrm[tid]);
+      const float inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
+      uint32_t* crow = reinterpret_cast<uint32_t*>(xa + tid * 128);
+#pragma unroll
+      for (int ch = 0; ch < 4; ++ch) {
+        uint32_t v[32];
+        tmem_ld32(tb + ((uint32_t)(warp * 32) << 16) + (uint32_t)(ch * 32), v);
+        uint32_t wd[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          uint32_t word = 0u;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float u = __fmul_rn(__uint_as_float(v[4 * q + e]), inv);
+            int c = 0;
+#pragma unroll
+            for (int k = 0; k < 7; ++k) c += (u > thr[k]) ? 1 : 0;
+            word |= (uint32_t)(n != 0.0f ? c : 0) << (8 * e);
+          }
+          wd[q] = word;
+        }
+#pragma unroll
+        for (int s = 0; s < 8; ++s) {  // staggered by lane: fewer bank conflicts
+          const int q = (s + lane) & 7;
+          uint32_t val = wd[0];
+#pragma unroll
+          for (int j = 1; j < 8; ++j) val = q == j ? wd[j] : val;
+          crow[ch * 8 + q] = val;
+        }
+      }
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();  // codes complete; TMEM free for the next tile
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    // ---- records: warp w packs tokens w, w + 4, ...
+    for (int i = warp; i < kDenseTok; i += 4) {
+      const int t = t0 + i;
+      if (t >= a.n) break;
+      const bool hi = a.is_high[(int64_t)b * a.n + t] != 0;
+      const int64_t s = (hi ? a.hi_base : a.lo_base) + a.slot[(int64_t)b * a.n + t];
+      const int64_t cap = hi ? a.hi_cap : a.lo_cap;
+      if (s >= cap) {  // cannot happen after the host's capacity check
+        if (lane == 0) raise_error(a.err, kDevCapacity);
+        continue;
+      }
+      if (l == 0 && h == 0 && lane == 0) {
+        if (hi) a.hi_tok[(int64_t)b * a.hi_cap + s] = (int32_t)(a.tok_base + t);
+        else a.lo_tok[(int64_t)b * a.lo_cap + s] = (int32_t)(a.tok_base + t);
+      }
+      const int L = hi ? a.L_hi : a.L_lo;
+      const int rec = record_bytes_rt(SEMKV_BASE_TQ_DENSE, L);
+      uint8_t* dst = (hi ? a.hi_pool : a.lo_pool) + ((((int64_t)b * a.NL + l) * a.H + h) * cap + s) * rec;
+      const uint8_t* cp = xa + (2 * i) * 128;
+      const uint16_t nk = nrm[2 * i], nv = nrm[2 * i + 1];
+      switch (L) {
+        case 2: dense_pack<2>(cp, nk, nv, dst, rec_sm[warp], lane); break;
+        case 3: dense_pack<3>(cp, nk, nv, dst, rec_sm[warp], lane); break;
+        case 4: dense_pack<4>(cp, nk, nv, dst, rec_sm[warp], lane); break;
+        case 5: dense_pack<5>(cp, nk, nv, dst, rec_sm[warp], lane); break;
+        case 6: dense_pack<6>(cp, nk, nv, dst, rec_sm[warp], lane); break;
+        case 7: dense_pack<7>(cp, nk, nv, dst, rec_sm[warp], lane); break;
+        case 8: dense_pack<8>(cp, nk, nv, dst, rec_sm[warp], lane); break;
+        default: break;
+      }
+    }
+    __syncthreads();  // the tiles are free for the next (sequence, layer, head)
+  }
+  // release the tensor memory (after every TMEM read of this CTA)
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 0)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 128;" ::"r"(tb) : "memory");
+}
+
 }  // namespace
 
 cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t stream) {
@@ -603,6 +851,20 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
   int64_t blocks = (total + kWarpsPerBlock - 1) / kWarpsPerBlock;
   const int64_t cap_blocks = (int64_t)num_sms * 16;  // grid-stride beyond this
   if (blocks > cap_blocks) blocks = cap_blocks;
+  if (a.base == SEMKV_BASE_TQ_DENSE) {
+    static bool attr_set = false;
+    if (!attr_set) {
+      const cudaError_t e = cudaFuncSetAttribute(
+          quantize_tq_dense_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kDenseTile);
+      if (e != cudaSuccess) return e;
+      attr_set = true;
+    }
+    const int64_t bhs = (int64_t)a.B * a.NL * a.H;
+    const dim3 grid((unsigned)((a.n + kDenseTok - 1) / kDenseTok),
+                    (unsigned)(bhs < 65535 ? bhs : 65535));
+    quantize_tq_dense_kernel<<<grid, 128, 2 * kDenseTile, stream>>>(a);
+    return cudaGetLastError();
+  }
   if (a.base == SEMKV_BASE_AFFINE_HAD)
     quantize_pack_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
   else

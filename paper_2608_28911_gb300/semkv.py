@@ -12,11 +12,13 @@ from __future__ import annotations
 import ctypes
 import os
 
+import numpy as np
+
 import torch
 
 from . import build as _build
 
-BASE_AFFINE, BASE_TQ, BASE_AFFINE_HAD = 0, 1, 2
+BASE_AFFINE, BASE_TQ, BASE_AFFINE_HAD, BASE_TQ_DENSE = 0, 1, 2, 3
 HEAD_DIM = 128
 
 _STATUS = {0: "ok", 1: "invalid argument", 2: "misaligned pointer or capacity",
@@ -34,7 +36,7 @@ class QuantDescStruct(ctypes.Structure):
                 ("levels_lo", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("signs", ctypes.c_void_p), ("centroids_hi", ctypes.c_void_p),
                 ("thresholds_hi", ctypes.c_void_p), ("centroids_lo", ctypes.c_void_p),
-                ("thresholds_lo", ctypes.c_void_p)]
+                ("thresholds_lo", ctypes.c_void_p), ("rotation", ctypes.c_void_p)]
 
 
 class CacheStruct(ctypes.Structure):
@@ -228,22 +230,30 @@ class QuantDesc:
     """A semkv_quant_desc whose device tables are torch tensors kept alive here."""
 
     def __init__(self, base: int, levels_hi: int, levels_lo: int, signs=None,
-                 device="cuda"):
+                 device="cuda", rotation=None):
         self.base, self.levels_hi, self.levels_lo = base, levels_hi, levels_lo
         self._keep = []
         s = QuantDescStruct(base=base, levels_hi=levels_hi, levels_lo=levels_lo,
                             head_dim=HEAD_DIM)
-        if base == BASE_TQ:
-            assert signs is not None, "the TQ base needs a sign vector per (layer, head)"
-            sg = torch.as_tensor(signs, dtype=torch.int8).to(device).contiguous()
+        if base in (BASE_TQ, BASE_TQ_DENSE):
+            if base == BASE_TQ:
+                assert signs is not None, "the TQ base needs a sign vector per (layer, head)"
+                sg = torch.as_tensor(signs, dtype=torch.int8).to(device).contiguous()
+                self._keep.append(sg)
+                s.signs = sg.data_ptr()
+                self.signs = sg
+            else:
+                assert rotation is not None, "the dense TQ base needs a rotation per (layer, head)"
+                rt = torch.as_tensor(np.ascontiguousarray(rotation).view(np.int16)).to(device)
+                self._keep.append(rt.contiguous())
+                s.rotation = self._keep[-1].data_ptr()
+                self.rotation = self._keep[-1]
             ch, th = semkv_lloyd_max_gaussian(levels_hi)
             cl, tl = semkv_lloyd_max_gaussian(levels_lo)
             tabs = [t.to(device).contiguous() for t in (ch, th, cl, tl)]
-            self._keep += [sg, *tabs]
-            s.signs = sg.data_ptr()
+            self._keep += tabs
             s.centroids_hi, s.thresholds_hi, s.centroids_lo, s.thresholds_lo = \
                 [t.data_ptr() for t in tabs]
-            self.signs = sg
             self.codebooks = {"hi": (ch, th), "lo": (cl, tl)}
         elif base == BASE_AFFINE_HAD:
             assert signs is not None, "the rotated affine base needs a sign vector per (layer, head)"

@@ -10,17 +10,19 @@ KV shape (8 KV heads, head_dim 128, 32 query heads, Sec. 4.5) and:
   - q: fp16 N(0,1);
   - scores: float32(Zipf(1.1)) per (sequence, token): integer-valued with heavy
     ties, which exercises the tie rule of the top-r selection;
-  - signs: +-1 per (layer, KV head, dim) for the TurboQuant-style rotation.
+  - signs: +-1 per (layer, KV head, dim) for the TurboQuant-style rotation;
+  - rotations: a Haar-random orthogonal Q per (layer, KV head) (QR of a Gaussian
+    matrix with the signs of R's diagonal taken into Q), stored as fp16 of sqrt(128) Q.
 Streams: numpy PCG64 seeded with seed*1000 + {0 K, 1 V, 2 q, 3 scores, 4 signs,
-5 outlier channels} + 10000*layer, so a many-layer cache is reproducible layer by
-layer.
+5 outlier channels, 6 rotations} + 10000*layer, so a many-layer cache is reproducible
+layer by layer.
 """
 from __future__ import annotations
 
 import numpy as np
 
 HEAD_DIM = 128
-STREAM_K, STREAM_V, STREAM_Q, STREAM_SCORES, STREAM_SIGNS, STREAM_OUTLIERS = range(6)
+STREAM_K, STREAM_V, STREAM_Q, STREAM_SCORES, STREAM_SIGNS, STREAM_OUTLIERS, STREAM_ROT = range(7)
 
 
 def _rng(seed: int, stream: int, layer: int = 0) -> np.random.Generator:
@@ -73,6 +75,18 @@ def signs(seed: int, layers: int, kv_heads: int) -> np.ndarray:
     """+-1 int8 [layers][kv_heads][128] for the randomized Hadamard rotation."""
     r = _rng(seed, STREAM_SIGNS)
     return np.where(r.random((layers, kv_heads, HEAD_DIM)) < 0.5, -1, 1).astype(np.int8)
+
+
+def rotations(seed: int, layers: int, kv_heads: int) -> np.ndarray:
+    """fp16 bits [layers][kv_heads][128][128] of sqrt(128) Q, Q Haar-random orthogonal."""
+    out = np.empty((layers, kv_heads, HEAD_DIM, HEAD_DIM), np.float16)
+    for l in range(layers):
+        r = _rng(seed, STREAM_ROT, l)
+        for h in range(kv_heads):
+            q, rr = np.linalg.qr(r.standard_normal((HEAD_DIM, HEAD_DIM)))
+            q = q * np.where(np.diag(rr) < 0, -1.0, 1.0)[None, :]
+            out[l, h] = (np.sqrt(HEAD_DIM) * q).astype(np.float16)
+    return out.view(np.uint16)
 
 
 def f16_bits(a: np.ndarray) -> np.ndarray:

@@ -30,8 +30,11 @@ class Pair:
         self.base, self.B, self.NL, self.H, self.Hq, self.T = base, B, NL, H, Hq, T
         self.r_num, self.r_den, self.seed = r_num, r_den, seed
         self.n_high = oracle.high_count_floor(T, r_num, r_den)
-        signs = synthetic.signs(seed, NL, H) if base != oracle.BASE_AFFINE else None
-        self.desc = semkv.QuantDesc(base, L_hi, L_lo, signs=signs, device=self.dev)
+        signs = (synthetic.signs(seed, NL, H)
+                 if base in (oracle.BASE_TQ, oracle.BASE_AFFINE_HAD) else None)
+        rot = synthetic.rotations(seed, NL, H) if base == oracle.BASE_TQ_DENSE else None
+        self.desc = semkv.QuantDesc(base, L_hi, L_lo, signs=signs, device=self.dev,
+                                    rotation=rot)
         self.cache = semkv.KVCache(self.desc, B, NL, H, Hq, hi_cap=self.n_high + extra_cap,
                                    lo_cap=T - self.n_high + extra_cap, block=block,
                                    device=self.dev)
@@ -40,7 +43,8 @@ class Pair:
                                lo_cap=self.cache.s.lo_cap)
         if signs is not None:
             self.oc.signs = signs
-        if base == oracle.BASE_TQ:
+        self.oc.rotation = rot
+        if base in (oracle.BASE_TQ, oracle.BASE_TQ_DENSE):
             _, c32, t32, _ = oracle.lloyd_max_gaussian(L_hi)
             self.oc.cb_hi = (c32, t32)
             _, c32, t32, _ = oracle.lloyd_max_gaussian(L_lo)
@@ -77,6 +81,57 @@ class Pair:
                 raise AssertionError(f"{name} pool differs at {len(bad)} records, first {bad[:3]}")
         assert np.array_equal(c.hi_tok.cpu().numpy()[:, :oc.hi_count], oc.hi_tok[:, :oc.hi_count])
         assert np.array_equal(c.lo_tok.cpu().numpy()[:, :oc.lo_count], oc.lo_tok[:, :oc.lo_count])
+
+    def assert_records_equal_up_to_ties(self, k=None, v=None, eps=1e-4):
+        """Dense-rotation TQ: the GPU forms w = M x on the tensor cores, the oracle rounds
+        the exact product once, so a code may differ by one where u sits within rounding
+        of the threshold between them.  Norms, token maps and every other code match."""
+        c, oc = self.cache, self.oc
+        k = self.k if k is None else k
+        v = self.v if v is None else v
+        assert c.hi_count == oc.hi_count and c.lo_count == oc.lo_count
+        assert np.array_equal(c.hi_tok.cpu().numpy()[:, :oc.hi_count], oc.hi_tok[:, :oc.hi_count])
+        assert np.array_equal(c.lo_tok.cpu().numpy()[:, :oc.lo_count], oc.lo_tok[:, :oc.lo_count])
+        flips = total = 0
+        for name, L, cnt, gp, op, tok in (
+                ("hi", oc.L_hi, oc.hi_count, c.hi_pool, oc.hi_pool, oc.hi_tok),
+                ("lo", oc.L_lo, oc.lo_count, c.lo_pool, oc.lo_pool, oc.lo_tok)):
+            if cnt == 0:
+                continue
+            got = gp.cpu().numpy()[..., :cnt, :]
+            want = op[..., :cnt, :]
+            rb = oracle.row_bytes(L)
+            assert np.array_equal(got[..., 2 * rb:2 * rb + 4], want[..., 2 * rb:2 * rb + 4]), name
+            bad = np.argwhere(np.any(got != want, axis=-1))
+            thr = (oc.cb_hi if name == "hi" else oc.cb_lo)[1].astype(np.float32)
+            for b, l, h, s in bad:
+                t = tok[b, s]
+                for row, src in ((0, k), (1, v)):
+                    cg = oracle.unpack_row(got[b, l, h, s, row * rb:(row + 1) * rb], L)
+                    co = oracle.unpack_row(want[b, l, h, s, row * rb:(row + 1) * rb], L)
+                    diff = np.nonzero(cg != co)[0]
+                    if diff.size == 0:
+                        continue
+                    x = synthetic.f16_bits(src[b, l, h, t])
+                    w = oracle.tq_dense_w(x, oc.rotation[l, h])
+                    n16 = want[b, l, h, s, 2 * rb + 2 * row:2 * rb + 2 * row + 2].view(np.uint16)[0]
+                    n = np.float32(np.uint16(n16).view(np.float16))
+                    u = (w * (np.float32(1) / n)).astype(np.float64)
+                    lo = np.minimum(cg[diff], co[diff]).astype(int)
+                    assert np.all(np.abs(cg[diff].astype(int) - co[diff].astype(int)) == 1)
+                    gap = np.abs(u[diff] - thr[lo].astype(np.float64))
+                    assert np.all(gap <= eps * (1 + np.abs(u[diff]))), (name, b, l, h, s, gap.max())
+                    flips += diff.size
+            total += got.shape[0] * got.shape[1] * got.shape[2] * cnt * 256
+        assert flips <= max(4, total * 1e-4), (flips, total)
+        return flips
+
+    def adopt_gpu_records(self):
+        """Attention parity independent of quantization ties: the oracle takes the GPU's
+        pools as they are."""
+        oc = self.oc
+        oc.hi_pool[..., :oc.hi_count, :] = self.cache.hi_pool.cpu().numpy()[..., :oc.hi_count, :]
+        oc.lo_pool[..., :oc.lo_count, :] = self.cache.lo_pool.cpu().numpy()[..., :oc.lo_count, :]
 
     def decode(self, layer=0, qseed=0, heads=None):
         torch, semkv = self.torch, self.semkv

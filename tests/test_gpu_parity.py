@@ -184,6 +184,53 @@ def test_had_decode_attention_matches_oracle(L_hi, L_lo, B, NL, H, Hq, T, r):
         check_attention(p, layer)
 
 
+# --------------------------------------------- dense-rotation TQ (tcgen05) -----
+
+@pytest.mark.parametrize("L_hi,L_lo,B,NL,H,Hq,T,r", [
+    (4, 3, 1, 2, 2, 8, 333, (3, 4)),        # the 2.0/1.585-bit mix at r = 75%, ragged
+    (4, 3, 2, 1, 8, 32, 1100, (3, 4)),      # Mistral-7B layer shape, short context
+    (2, 2, 1, 1, 2, 4, 64, (0, 1)),         # one full 64-token tile
+    (8, 5, 1, 1, 2, 16, 150, (1, 4)),       # CUDA-core decode path, GQA group of 8
+    (3, 2, 1, 1, 1, 4, 1, (1, 1)),          # a single token
+])
+def test_dense_tq_quantize_and_decode(L_hi, L_lo, B, NL, H, Hq, T, r):
+    p = Pair(3, L_hi, L_lo, B, NL, H, Hq, T, r[0], r[1], seed=70 + T)
+    p.quantize()
+    assert np.array_equal(p.is_high.cpu().numpy(), p.o_is_high)
+    p.assert_records_equal_up_to_ties()
+    assert int(p.cache.dev_error.item()) == 0
+    p.adopt_gpu_records()
+    for layer in range(NL):
+        check_attention(p, layer)
+
+
+def test_dense_tq_append_blocks_and_staged_tail():
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    blk, T0, ngen = 32, 150, 2 * 32 + 5
+    p = Pair(3, 4, 3, 1, 2, 2, 8, T0, 3, 4, seed=81, block=blk, extra_cap=ngen)
+    p.quantize()
+    p.assert_records_equal_up_to_ties()
+    k, v = synthetic.kv(82, 1, 2, 2, ngen)
+    s = synthetic.scores_zipf(82, 1, ngen)
+    for g in range(ngen):
+        kt = torch.from_numpy(np.ascontiguousarray(k[:, :, :, g])).to(p.dev)
+        vt = torch.from_numpy(np.ascontiguousarray(v[:, :, :, g])).to(p.dev)
+        p.cache.stage_token(kt, vt, torch.from_numpy(np.ascontiguousarray(s[:, g])).to(p.dev))
+        oracle.stage_token(p.oc, synthetic.f16_bits(k[:, :, :, g]), synthetic.f16_bits(v[:, :, :, g]),
+                           s[:, g])
+        if p.cache.stage_n == blk:
+            semkv.semkv_append_block(p.desc, p.cache, 3, 4)
+            oracle.append_block(p.oc, 3, 4)
+            torch.cuda.synchronize()
+            allk = np.concatenate([p.k, k], axis=3)
+            allv = np.concatenate([p.v, v], axis=3)
+            p.assert_records_equal_up_to_ties(allk, allv)
+    p.adopt_gpu_records()
+    check_attention(p, layer=1, qseed=5)     # pools + the 5 staged fp16 tokens
+    assert int(p.cache.dev_error.item()) == 0
+
+
 # ------------------------------------------------------------ TQ decode -----
 
 @pytest.mark.parametrize("L_hi,L_lo,B,NL,H,Hq,T,r", [
