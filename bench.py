@@ -360,8 +360,9 @@ def gpu_arm(args, cfg, rank, world):
     nh_b = semkv.semkv_block_high_count(blk, r_num, r_den)
     # launches per decode call: (rotation for TQ,) pools, (stage,) combine
     plain = cfg["base"] == semkv.BASE_AFFINE
-    dec_launch = (0 if plain else 1) + 1 + 1
-    app_launch = 3 if plain else 2      # rank, (slot -> token scatter,) quantize
+    dec_launch = (0 if plain else 1) + 1 + 1     # (query rotation,) pools, combine
+    # rank, slot -> token scatter (not for the dense rotation), quantize
+    app_launch = 2 if cfg["base"] == semkv.BASE_TQ_DENSE else 3
 
     def decode_all(qv, ev=None):
         if ev is not None:

@@ -195,95 +195,6 @@ __device__ __forceinline__ void pack_rows(const uint8_t* codes, uint32_t* rec, i
   }
 }
 
-template <int BASE, int L>
-__device__ void quantize_pair(const QuantArgs& a, const float kx[4], const float vx[4],
-                              const int8_t* sg, const float* thr_g, uint8_t* dst,
-                              uint8_t* codes, uint32_t* rec, int lane) {
-  using F = Fmt<L>;
-  RowOut ko, vo;
-  if constexpr (BASE == SEMKV_BASE_AFFINE) {
-    ko = affine_row<L>(kx);
-    vo = affine_row<L>(vx);
-  } else if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
-    ko = affine_had_row<L>(kx, sg, lane);
-    vo = affine_had_row<L>(vx, sg, lane);
-  } else {
-    float thr[8];
-#pragma unroll
-    for (int t = 0; t < 8; ++t) thr[t] = t < L - 1 ? thr_g[t] : 0.0f;
-    ko = tq_row<L>(kx, sg, lane, thr);
-    vo = tq_row<L>(vx, sg, lane, thr);
-  }
-  constexpr int kRec = 2 * F::RB + (BASE == SEMKV_BASE_TQ ? 4 : 8);
-  constexpr int kRecWords = kRec / 4;
-  reinterpret_cast<uint32_t*>(codes)[lane] = ko.codes;
-  reinterpret_cast<uint32_t*>(codes)[32 + lane] = vo.codes;
-  if (lane < kRecWords) rec[lane] = 0u;
-  __syncwarp();
-  pack_rows<L>(codes, rec, lane);
-  if (lane == 0) {
-    if constexpr (BASE != SEMKV_BASE_TQ) {
-      rec[(2 * F::RB) / 4] = (uint32_t)ko.p0 | ((uint32_t)ko.p1 << 16);
-      rec[(2 * F::RB) / 4 + 1] = (uint32_t)vo.p0 | ((uint32_t)vo.p1 << 16);
-    } else {
-      rec[(2 * F::RB) / 4] = (uint32_t)ko.p0 | ((uint32_t)vo.p0 << 16);
-    }
-  }
-  __syncwarp();
-  if (lane < kRecWords) reinterpret_cast<uint32_t*>(dst)[lane] = rec[lane];
-  __syncwarp();
-}
-
-template <int BASE>
-__global__ void __launch_bounds__(kWarpsPerBlock * 32)
-    quantize_pack_kernel(QuantArgs a) {
-  __shared__ __align__(16) uint8_t codes_sm[kWarpsPerBlock][256];
-  __shared__ __align__(16) uint32_t rec_sm[kWarpsPerBlock][kMaxRecWords + 1];
-  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
-  const int64_t total = (int64_t)a.B * a.NL * a.H * a.n;
-  const int64_t nwarps = (int64_t)gridDim.x * kWarpsPerBlock;
-  for (int64_t task = (int64_t)blockIdx.x * kWarpsPerBlock + wib; task < total; task += nwarps) {
-    const int i = (int)(task % a.n);
-    int64_t r = task / a.n;
-    const int h = (int)(r % a.H);
-    r /= a.H;
-    const int l = (int)(r % a.NL);
-    const int b = (int)(r / a.NL);
-    const bool hi = a.is_high[(int64_t)b * a.n + i] != 0;
-    const int64_t s = (hi ? a.hi_base : a.lo_base) + a.slot[(int64_t)b * a.n + i];
-    const int64_t cap = hi ? a.hi_cap : a.lo_cap;
-    if (s >= cap) {  // cannot happen after the host's capacity check; never write out of range
-      if (lane == 0) raise_error(a.err, kDevCapacity);
-      continue;
-    }
-    if (l == 0 && h == 0 && lane == 0) {
-      if (hi) a.hi_tok[(int64_t)b * a.hi_cap + s] = (int32_t)(a.tok_base + i);
-      else a.lo_tok[(int64_t)b * a.lo_cap + s] = (int32_t)(a.tok_base + i);
-    }
-    const int64_t row = ((((int64_t)b * a.NL + l) * a.H + h) * a.Tsrc + i) * kHeadDim;
-    float kx[4], vx[4];
-    load4(a.k + row, lane, kx);
-    load4(a.v + row, lane, vx);
-    const int L = hi ? a.L_hi : a.L_lo;
-    const int rec = record_bytes_rt(BASE, L);
-    uint8_t* dst = (hi ? a.hi_pool : a.lo_pool) + ((((int64_t)b * a.NL + l) * a.H + h) * cap + s) * rec;
-    const int8_t* sg = a.signs ? a.signs + ((int64_t)l * a.H + h) * kHeadDim : nullptr;
-    const float* thr = hi ? a.thr_hi : a.thr_lo;
-    uint8_t* cs = codes_sm[wib];
-    uint32_t* rs = rec_sm[wib];
-    switch (L) {
-      case 2: quantize_pair<BASE, 2>(a, kx, vx, sg, thr, dst, cs, rs, lane); break;
-      case 3: quantize_pair<BASE, 3>(a, kx, vx, sg, thr, dst, cs, rs, lane); break;
-      case 4: quantize_pair<BASE, 4>(a, kx, vx, sg, thr, dst, cs, rs, lane); break;
-      case 5: quantize_pair<BASE, 5>(a, kx, vx, sg, thr, dst, cs, rs, lane); break;
-      case 6: quantize_pair<BASE, 6>(a, kx, vx, sg, thr, dst, cs, rs, lane); break;
-      case 7: quantize_pair<BASE, 7>(a, kx, vx, sg, thr, dst, cs, rs, lane); break;
-      case 8: quantize_pair<BASE, 8>(a, kx, vx, sg, thr, dst, cs, rs, lane); break;
-      default: break;
-    }
-  }
-}
-
 // ------------------------------------------------- affine pools, by slot -----
 // Affine records are built by destination slot: a warp takes units of 8 consecutive
 // slots of one pool of one (sequence, layer, KV head), so the level count is uniform
@@ -326,26 +237,32 @@ __device__ __forceinline__ void quarter_field(const uint32_t (&m)[32], uint32_t 
   using F = Fmt<L>;
   constexpr uint32_t kMagic = 0x4B400000u;
   w[0] = w[1] = w[2] = 0u;
+  if constexpr (F::G == 1 && F::LG == (1u << F::W)) {
+    // L = 2, 4, 8: ceil(c 2^W / L) = c, each code its own W-bit symbol
 #pragma unroll
-  for (int sy = 0; sy < F::NG; ++sy) {
-    uint32_t t = 0, wsum = 0;
+    for (int sy = 0; sy < 32; ++sy) put_bits(w, sy * F::W, F::W, m[sy] - kMagic);
+  } else {
 #pragma unroll
-    for (int k = 0; k < F::G; ++k) {
-      t = t * (uint32_t)L + m[sy * F::G + k];
-      wsum = wsum * (uint32_t)L + 1u;
+    for (int sy = 0; sy < F::NG; ++sy) {
+      uint32_t t = 0, wsum = 0;
+#pragma unroll
+      for (int k = 0; k < F::G; ++k) {
+        t = t * (uint32_t)L + m[sy * F::G + k];
+        wsum = wsum * (uint32_t)L + 1u;
+      }
+      t -= wsum * kMagic;
+      put_bits(w, sy * F::W, F::W, ((t << F::W) + F::LG - 1u) / F::LG);
     }
-    t -= wsum * kMagic;
-    put_bits(w, sy * F::W, F::W, ((t << F::W) + F::LG - 1u) / F::LG);
-  }
-  if constexpr (F::R > 0) {
-    uint32_t t = 0, wsum = 0;
+    if constexpr (F::R > 0) {
+      uint32_t t = 0, wsum = 0;
 #pragma unroll
-    for (int k = 0; k < F::R; ++k) {
-      t = t * (uint32_t)L + m[32 - F::R + k];
-      wsum = wsum * (uint32_t)L + 1u;
+      for (int k = 0; k < F::R; ++k) {
+        t = t * (uint32_t)L + m[32 - F::R + k];
+        wsum = wsum * (uint32_t)L + 1u;
+      }
+      t -= wsum * kMagic;
+      put_bits(w, F::NG * F::W, F::WT, ((t << F::WT) + F::LR - 1u) / F::LR);
     }
-    t -= wsum * kMagic;
-    put_bits(w, F::NG * F::W, F::WT, ((t << F::WT) + F::LR - 1u) / F::LR);
   }
 }
 
@@ -471,6 +388,256 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32)
   }
 }
 
+// ------------------------------- rotated bases by slot, one thread per row -----
+// TQ and rotated affine records built by destination slot, as for the affine base: a
+// CTA of 128 threads takes 64 consecutive slots of one pool of one (sequence, layer,
+// KV head), so the level count is uniform.  Thread r owns row r of the tile (K of slot
+// r/2 when r is even, V when odd).  Its 128 values live in registers and the
+// Walsh-Hadamard butterflies run inside the thread in the quantizer's stage order
+// (the same roundings as the lane-distributed form), followed by the norm or the
+// min/max, the codes and the quarter bit fields.  The warps then assemble each
+// record's words from the two rows' bits and write them with 4-byte stores.
+constexpr int kRowSlots = 64;
+constexpr int kRowStride = 272;  // bytes per staged row: 256 + 16 spreads the banks
+constexpr int kRowBitWords = 13;  // words per row's bit image (12 used at most)
+
+// packed binary32 pairs (two independent IEEE operations, rounded to nearest)
+__device__ __forceinline__ unsigned long long f2_add(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ unsigned long long f2_sub(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ unsigned long long f2_pack(float lo, float hi) {
+  return (unsigned long long)__float_as_uint(lo) | ((unsigned long long)__float_as_uint(hi) << 32);
+}
+__device__ __forceinline__ float f2_lo(unsigned long long v) { return __uint_as_float((uint32_t)v); }
+__device__ __forceinline__ float f2_hi(unsigned long long v) {
+  return __uint_as_float((uint32_t)(v >> 32));
+}
+
+// OR the 96-bit field v at bit pos (compile-time after unrolling) of a row's words
+template <int N>
+__device__ __forceinline__ void or_field(uint32_t (&w)[N], int pos, const uint32_t (&v)[3]) {
+  const int wd = pos >> 5, sh = pos & 31;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const uint32_t lo = k < 3 ? v[k] : 0u, prev = k > 0 ? v[k - 1] : 0u;
+    const uint32_t part = sh == 0 ? lo : (lo << sh) | (prev >> (32 - sh));
+    if (wd + k < N) w[wd + k] |= part;
+  }
+}
+
+template <int BASE, int L>
+__device__ void rows_block(const QuantArgs& a, int b, int l, int h, bool hi, int64_t s0,
+                           int nslots, uint8_t* stage, uint32_t* bits, uint32_t* par) {
+  using F = Fmt<L>;
+  constexpr int kWords = (4 * F::QB + 31) / 32;
+  constexpr int kRecW = (2 * F::RB + (BASE == SEMKV_BASE_TQ ? 4 : 8)) / 4;
+  static_assert(kWords <= 12 && F::QB <= 96, "row image size");
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t cap = hi ? a.hi_cap : a.lo_cap;
+  const int64_t pbase = hi ? a.hi_base : a.lo_base;
+  const int64_t bh = ((int64_t)b * a.NL + l) * a.H + h;
+  const int32_t* tokmap = (hi ? a.hi_tok : a.lo_tok) + (int64_t)b * cap + pbase;
+  // ---- stage the rows of the block's slots (coalesced 16-byte chunks)
+  for (int c = tid; c < 128 * 16; c += 128) {
+    const int r = c >> 4, ch = c & 15, i = r >> 1;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (i < nslots) {
+      const int64_t t = (int64_t)tokmap[s0 + i] - a.tok_base;
+      const uint16_t* src = ((r & 1) ? a.v : a.k) + (bh * a.Tsrc + t) * kHeadDim;
+      v = __ldg(reinterpret_cast<const uint4*>(src) + ch);
+    }
+    *reinterpret_cast<uint4*>(stage + r * kRowStride + ch * 16) = v;
+  }
+  __syncthreads();
+  // ---- row tid: values, signs
+  float x[128];
+#pragma unroll
+  for (int ch = 0; ch < 16; ++ch) {
+    const uint4 u = *reinterpret_cast<const uint4*>(stage + tid * kRowStride + ch * 16);
+    const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
+      x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
+    }
+  }
+  uint32_t param;
+  float zq = 0.0f, invq = 0.0f;  // affine: offset and 1/s;  TQ: 1/n in invq
+  bool live;
+  if constexpr (BASE == SEMKV_BASE_TQ) {
+    // norm of the row with the fixed tree: 32 in-order partials of 4 squares, then the
+    // pairwise stages 16, 8, 4, 2, 1 (partials g and g + 16 formed together, so the
+    // first stage needs 16 registers)
+    float pn[16];
+#pragma unroll
+    for (int g = 0; g < 16; ++g) {
+      float acc[2];
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const int gg = g + 16 * hh;
+        float v = __fmul_rn(x[4 * gg], x[4 * gg]);
+#pragma unroll
+        for (int k = 1; k < 4; ++k) v = __fadd_rn(v, __fmul_rn(x[4 * gg + k], x[4 * gg + k]));
+        acc[hh] = v;
+      }
+      pn[g] = __fadd_rn(acc[0], acc[1]);
+    }
+#pragma unroll
+    for (int off = 8; off >= 1; off >>= 1)
+#pragma unroll
+      for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
+    const uint16_t n16 = f16_param(__fsqrt_rn(pn[0]));
+    param = n16;
+    const float n = f16_to_f32(n16);
+    live = n != 0.0f;
+    invq = live ? __fdiv_rn(1.0f, n) : 0.0f;
+  }
+  const int8_t* sg = a.signs + ((int64_t)l * a.H + h) * kHeadDim;
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    const char4 s4 = __ldg(reinterpret_cast<const char4*>(sg) + j);
+    x[4 * j] *= (float)s4.x;
+    x[4 * j + 1] *= (float)s4.y;
+    x[4 * j + 2] *= (float)s4.z;
+    x[4 * j + 3] *= (float)s4.w;
+  }
+  // ---- Walsh-Hadamard butterflies, stages 1, 2, ..., 64: stage 1 inside each pair
+  // (2k, 2k+1), the later stages on packed pairs (pair k with pair k + hs/2)
+  unsigned long long xp[64];
+#pragma unroll
+  for (int k = 0; k < 64; ++k) {
+    const float p0 = x[2 * k], p1 = x[2 * k + 1];
+    xp[k] = f2_pack(__fadd_rn(p0, p1), __fsub_rn(p0, p1));
+  }
+#pragma unroll
+  for (int hs = 2; hs < 128; hs <<= 1) {
+#pragma unroll
+    for (int k = 0; k < 64; ++k) {
+      if ((2 * k) & hs) continue;
+      const unsigned long long p0 = xp[k], p1 = xp[k + hs / 2];
+      xp[k] = f2_add(p0, p1);
+      xp[k + hs / 2] = f2_sub(p0, p1);
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 64; ++k) {
+    x[2 * k] = f2_lo(xp[k]);
+    x[2 * k + 1] = f2_hi(xp[k]);
+  }
+  if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
+    float mn = INFINITY, mx = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 128; ++j) {
+      x[j] = __fmul_rn(x[j], kInvSqrtD);
+      mn = fminf(mn, x[j]);
+      mx = fmaxf(mx, x[j]);
+    }
+    if (mn == 0.0f) mn = 0.0f;
+    if (mx == 0.0f) mx = 0.0f;
+    uint16_t z16 = __half_as_ushort(__float2half_rd(mn));
+    if (z16 == 0xFC00u) z16 = 0xFBFFu;
+    zq = f16_to_f32(z16);
+    const uint16_t s16 = f16_param(__fdiv_rn(__fsub_rn(mx, zq), (float)(L - 1)));
+    const float sv = f16_to_f32(s16);
+    live = sv > 0.0f;
+    invq = live ? __fdiv_rn(1.0f, sv) : 0.0f;
+    param = (uint32_t)s16 | ((uint32_t)z16 << 16);
+  }
+  // ---- codes, quarter by quarter, as magic-number patterns 1.5 * 2^23 + c
+  uint32_t w[12];
+#pragma unroll
+  for (int k = 0; k < 12; ++k) w[k] = 0u;
+  const bool hi_row = hi;  // (the level count is the pool's)
+  (void)hi_row;
+  float thr[7];
+  if constexpr (BASE == SEMKV_BASE_TQ) {
+    const float* tg = hi ? a.thr_hi : a.thr_lo;
+#pragma unroll
+    for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? tg[k] : INFINITY;
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint32_t m[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const float xv = x[32 * q + j];
+      if constexpr (BASE == SEMKV_BASE_TQ) {
+        const float u = __fmul_rn(xv, invq);
+        int c = 0;
+#pragma unroll
+        for (int k = 0; k < L - 1; ++k) c += (u > thr[k]) ? 1 : 0;
+        m[j] = 0x4B400000u + (uint32_t)(live ? c : 0);
+      } else {
+        // rint(clamp(v)) = clamp(rint(v)) for integer bounds; + 1.5 * 2^23 rounds to even
+        const float y = fminf(fmaxf(__fmul_rn(__fsub_rn(xv, zq), invq), 0.0f), (float)(L - 1));
+        m[j] = live ? __float_as_uint(__fadd_rn(y, 12582912.0f)) : 0x4B400000u;
+      }
+    }
+    uint32_t fw[3];
+    quarter_field<L>(m, fw);
+    or_field<12>(w, q * F::QB, fw);
+  }
+#pragma unroll
+  for (int k = 0; k < kWords; ++k) bits[tid * kRowBitWords + k] = w[k];
+  par[tid] = param;
+  __syncthreads();
+  // ---- records: warp takes slots warp, warp + 4, ...; lane j writes word j
+  uint32_t* recs = reinterpret_cast<uint32_t*>(hi ? a.hi_pool : a.lo_pool) + (bh * cap + pbase + s0) * kRecW;
+  for (int i = warp; i < nslots; i += 4) {
+    for (int j = lane; j < kRecW; j += 32) {
+      uint32_t word = 0u;
+      if (4 * j >= 2 * F::RB) {
+        const int pj = j - (2 * F::RB) / 4;
+        if constexpr (BASE == SEMKV_BASE_TQ) word = par[2 * i] | (par[2 * i + 1] << 16);
+        else word = par[2 * i + pj];
+      } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int byte = 4 * j + e;
+          const int row = byte < F::RB ? 2 * i : 2 * i + 1;
+          const int rb = byte < F::RB ? byte : byte - F::RB;
+          const uint32_t v = rb < F::RB ? (bits[row * kRowBitWords + (rb >> 2)] >> (8 * (rb & 3))) & 0xFFu : 0u;
+          word |= v << (8 * e);
+        }
+      }
+      recs[(int64_t)i * kRecW + j] = word;
+    }
+  }
+  __syncthreads();  // the staging area is free for the next block
+}
+
+template <int BASE>
+__global__ void __launch_bounds__(128, 3) quantize_rows_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
+  __shared__ __align__(16) uint8_t stage[128 * kRowStride];
+  __shared__ uint32_t bits[128 * kRowBitWords];
+  __shared__ uint32_t par[128];
+  const bool hi = blockIdx.z == 0;
+  const int64_t n_pool = hi ? n_hi : n_lo;
+  const int bhs = a.B * a.NL * a.H;
+  const int L = hi ? a.L_hi : a.L_lo;
+  for (int64_t s0 = (int64_t)blockIdx.x * kRowSlots; s0 < n_pool; s0 += (int64_t)gridDim.x * kRowSlots) {
+    const int nslots = (int)min((int64_t)kRowSlots, n_pool - s0);
+    for (int bhi = blockIdx.y; bhi < bhs; bhi += gridDim.y) {
+      const int h = bhi % a.H, l = (bhi / a.H) % a.NL, b = bhi / (a.H * a.NL);
+      switch (L) {
+#define SEMKV_ROWS_CASE(LV) \
+        case LV: rows_block<BASE, LV>(a, b, l, h, hi, s0, nslots, stage, bits, par); break;
+        SEMKV_ROWS_CASE(2) SEMKV_ROWS_CASE(3) SEMKV_ROWS_CASE(4) SEMKV_ROWS_CASE(5)
+        SEMKV_ROWS_CASE(6) SEMKV_ROWS_CASE(7) SEMKV_ROWS_CASE(8)
+#undef SEMKV_ROWS_CASE
+        default: break;
+      }
+    }
+  }
+}
+
 // ------------------------------------------------- fake quantization ---------
 // Every row quantized at its token's precision and reconstructed to fp16 (the quality
 // protocol of Sec. 4.1), in binary32 in this order:
@@ -571,7 +738,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) fake_quant_kernel(FakeArg
 // K = 8 x 16, both operands K-major in shared memory without swizzle, the fp32
 // accumulator in tensor memory (128 lanes x 128 columns).  Thread r then owns row r:
 // the fixed-tree norm (from the staged row, while the MMAs run), the TMEM row, the
-// codes.  The warps pack the records as in quantize_pair.
+// codes.  The warps pack the records with pack_rows.
 constexpr int kDenseTok = 64;
 constexpr uint32_t kDenseTile = 128 * 128 * 2;  // bytes of one operand tile
 // instruction descriptor: fp32 accumulate (bits 4-5 = 1), A and B fp16 (formats 0),
@@ -830,6 +997,7 @@ cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t strea
 
 cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
                                  cudaStream_t stream) {
+  (void)num_sms;
   const int64_t total = (int64_t)a.B * a.NL * a.H * a.n;
   if (total == 0) return cudaSuccess;
   if (a.base == SEMKV_BASE_AFFINE) {
@@ -848,9 +1016,6 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
     quantize_affine_kernel<<<grid, kWarpsPerBlock * 32, 0, stream>>>(a, n_hi, a.n - n_hi);
     return cudaGetLastError();
   }
-  int64_t blocks = (total + kWarpsPerBlock - 1) / kWarpsPerBlock;
-  const int64_t cap_blocks = (int64_t)num_sms * 16;  // grid-stride beyond this
-  if (blocks > cap_blocks) blocks = cap_blocks;
   if (a.base == SEMKV_BASE_TQ_DENSE) {
     static bool attr_set = false;
     if (!attr_set) {
@@ -865,10 +1030,21 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
     quantize_tq_dense_kernel<<<grid, 128, 2 * kDenseTile, stream>>>(a);
     return cudaGetLastError();
   }
+  // TQ and rotated affine: slot -> token maps, then one thread per row by slot
+  const int64_t pairs = (int64_t)a.B * a.n;
+  scatter_tok_kernel<<<(unsigned)((pairs + 255) / 256), 256, 0, stream>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int64_t bhs = (int64_t)a.B * a.NL * a.H;
+  const int64_t n_max = n_hi > a.n - n_hi ? n_hi : a.n - n_hi;
+  int64_t bx = (n_max + kRowSlots - 1) / kRowSlots;
+  if (bx < 1) bx = 1;
+  if (bx > 65535) bx = 65535;
+  const dim3 grid((unsigned)bx, (unsigned)(bhs < 65535 ? bhs : 65535), 2);
   if (a.base == SEMKV_BASE_AFFINE_HAD)
-    quantize_pack_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+    quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD><<<grid, 128, 0, stream>>>(a, n_hi, a.n - n_hi);
   else
-    quantize_pack_kernel<SEMKV_BASE_TQ><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+    quantize_rows_kernel<SEMKV_BASE_TQ><<<grid, 128, 0, stream>>>(a, n_hi, a.n - n_hi);
   return cudaGetLastError();
 }
 

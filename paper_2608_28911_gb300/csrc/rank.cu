@@ -5,9 +5,10 @@
 // One 1024-thread CTA per sequence.  Sequences of at most 1024 tokens (the blocks of
 // Algorithm 2) take a single pass: each thread counts the keys ahead of its own.
 // Longer ones: scores become order-preserving 32-bit keys
-// (NaN -> 0, below every number; -0 -> +0).  A 4-pass MSB-first radix select over
-// 8-bit digits finds theta, the key of the n_high-th largest score, and `need`, how
-// many keys equal to theta are taken (the earliest ones).  One sweep with a block
+// (NaN -> 0, below every number; -0 -> +0), kept in shared memory for sequences of up
+// to 40960 tokens.  A 4-pass MSB-first radix select over 8-bit digits finds theta,
+// the key of the n_high-th largest score, and `need`, how many keys equal to theta
+// are taken (the earliest ones).  One sweep with a block
 // scan of packed (greater, equal) counts then gives, for token i,
 //   high(i)        = key_i > theta  or  (key_i == theta and eq_before(i) < need)
 //   high_before(i) = gt_before(i) + min(eq_before(i), need)
@@ -91,9 +92,49 @@ __global__ void __launch_bounds__(kThreads) rank_small_kernel(RankArgs a) {
   }
 }
 
+// keys of sequences up to this length are kept in shared memory across the passes
+constexpr uint32_t kSmemKeys = 40960;
+constexpr int kSelItems = 8;  // keys per thread per loop trip (independent loads)
+
+// warp 0: the bin holding the k-th largest key among the 256 counts, and how many
+// larger keys the bins above it hold (a suffix scan, 8 bins per lane)
+__device__ __forceinline__ void select_bin(const uint32_t* hist, uint32_t k, uint32_t* bin_out,
+                                           uint32_t* above_out) {
+  const int lane = threadIdx.x & 31;
+  // lane l owns bins 255 - 8l down to 248 - 8l (descending key order)
+  uint32_t c[8], sum = 0;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    c[e] = hist[255 - 8 * lane - e];
+    sum += c[e];
+  }
+  uint32_t incl = sum;  // inclusive scan over lanes of the per-lane sums
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += y;
+  }
+  const uint32_t excl = incl - sum;  // keys in bins above this lane's
+  const bool mine = excl < k && incl >= k;
+  if (mine) {
+    uint32_t cum = excl;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      if (cum + c[e] >= k) {
+        *bin_out = 255u - 8u * lane - (uint32_t)e;
+        *above_out = cum;
+        break;
+      }
+      cum += c[e];
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kThreads) rank_assign_kernel(RankArgs a) {
+  extern __shared__ uint32_t skeys[];  // the sequence's keys when T <= kSmemKeys
   __shared__ uint32_t hist[256];
-  __shared__ uint32_t sel_prefix, sel_k;
+  __shared__ uint32_t whist[kThreads / 32][256];  // one histogram per warp: no contention
+  __shared__ uint32_t sel_bin, sel_above;
   __shared__ uint64_t warp_sums[32];
   const int b = blockIdx.x;
   const float* s = a.scores + (int64_t)b * a.ld;
@@ -110,47 +151,47 @@ __global__ void __launch_bounds__(kThreads) rank_assign_kernel(RankArgs a) {
     }
     return;
   }
+  const bool in_smem = T <= kSmemKeys;
+  if (in_smem) {
+    for (uint32_t i = tid; i < T; i += kThreads) skeys[i] = order_key(s[i]);
+    __syncthreads();
+  }
 
   // ---- radix select: theta = key of the n_high-th largest, need = ties taken
   uint32_t prefix = 0, mask = 0, k = a.n_high;
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
-    for (int i = tid; i < 256; i += kThreads) hist[i] = 0;
+    uint32_t* wh = whist[tid >> 5];
+    for (int i = tid; i < (kThreads / 32) * 256; i += kThreads) (&whist[0][0])[i] = 0;
     __syncthreads();
-    for (uint32_t i0 = 0; i0 < T; i0 += kThreads) {
-      const uint32_t i = i0 + tid;
-      bool cand = false;
-      uint32_t bin = 0;
-      if (i < T) {
-        const uint32_t key = order_key(s[i]);
-        cand = (key & mask) == prefix;
-        bin = (key >> shift) & 0xFFu;
+    for (uint32_t i0 = 0; i0 < T; i0 += kThreads * kSelItems) {
+      uint32_t key[kSelItems];
+#pragma unroll
+      for (int j = 0; j < kSelItems; ++j) {
+        const uint32_t i = i0 + j * kThreads + tid;
+        key[j] = i < T ? (in_smem ? skeys[i] : order_key(s[i])) : 0u;
       }
-      // warp-aggregated histogram update: equal bins of a warp add once
-      const uint32_t active = __ballot_sync(0xffffffffu, cand);
-      if (cand) {
-        const uint32_t peers = __match_any_sync(active, bin);
-        const int leader = __ffs(peers) - 1;
-        if ((tid & 31) == leader) atomicAdd(&hist[bin], (uint32_t)__popc(peers));
+#pragma unroll
+      for (int j = 0; j < kSelItems; ++j) {
+        const uint32_t i = i0 + j * kThreads + tid;
+        const bool cand = i < T && (key[j] & mask) == prefix;
+        const uint32_t bin = (key[j] >> shift) & 0xFFu;
+        // the warp's own histogram: shared-memory atomics without cross-warp contention
+        if (cand) atomicAdd(&wh[bin], 1u);
       }
     }
     __syncthreads();
-    if (tid == 0) {
-      uint32_t cum = 0, chosen = 0;
-      for (int bin = 255; bin >= 0; --bin) {
-        const uint32_t c = hist[bin];
-        if (cum + c >= k) {
-          chosen = (uint32_t)bin;
-          break;
-        }
-        cum += c;
-      }
-      sel_prefix = prefix | (chosen << shift);
-      sel_k = k - cum;
+    for (int i = tid; i < 256; i += kThreads) {
+      uint32_t c = 0;
+#pragma unroll 8
+      for (int w = 0; w < kThreads / 32; ++w) c += whist[w][i];
+      hist[i] = c;
     }
     __syncthreads();
-    prefix = sel_prefix;
-    k = sel_k;
+    if (tid < 32) select_bin(hist, k, &sel_bin, &sel_above);
+    __syncthreads();
+    prefix |= sel_bin << shift;
+    k -= sel_above;
     mask |= 0xFFu << shift;
     __syncthreads();
   }
@@ -164,7 +205,7 @@ __global__ void __launch_bounds__(kThreads) rank_assign_kernel(RankArgs a) {
 #pragma unroll
     for (int j = 0; j < kItems; ++j) {
       const uint32_t i = c0 + tid * kItems + j;
-      keys[j] = i < T ? order_key(s[i]) : 0u;
+      keys[j] = i < T ? (in_smem ? skeys[i] : order_key(s[i])) : 0u;
       if (i < T) local += (keys[j] > theta ? 1ull : 0ull) | ((keys[j] == theta ? 1ull : 0ull) << 32);
     }
     uint64_t total;
@@ -289,10 +330,20 @@ size_t rank_workspace_words(int B, int T) { return (size_t)B * 4 * (size_t)T; }
 
 cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream) {
   if (a.B == 0 || a.T == 0) return cudaSuccess;
-  if (a.T <= kThreads)
+  if (a.T <= kThreads) {
     rank_small_kernel<<<a.B, kThreads, 0, stream>>>(a);
-  else
-    rank_assign_kernel<<<a.B, kThreads, 0, stream>>>(a);
+  } else {
+    static bool attr_set = false;
+    if (!attr_set) {
+      const cudaError_t e = cudaFuncSetAttribute(rank_assign_kernel,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)(kSmemKeys * sizeof(uint32_t)));
+      if (e != cudaSuccess) return e;
+      attr_set = true;
+    }
+    const size_t smem = (uint32_t)a.T <= kSmemKeys ? (size_t)a.T * sizeof(uint32_t) : 0;
+    rank_assign_kernel<<<a.B, kThreads, smem, stream>>>(a);
+  }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || !a.rank) return e;
   rank_sort_kernel<<<a.B, kThreads, 0, stream>>>(a, a.ws);
