@@ -1,19 +1,21 @@
 // quantize.cu — token-wise mixed-precision quantization and mixed-radix packing
-// (Eq. 7; Sec. 4.1 affine base; Sec. 4.9 TurboQuant-MSE base).
+// (Eq. 7; Sec. 4.1 affine base and its Hadamard-rotated form; Sec. 4.9 TurboQuant-MSE
+// base with the randomized Hadamard or a dense random rotation), and fake quantization.
 //
-// One warp per (sequence, layer, KV head, token): lane l holds dims 4l..4l+3 of the
-// token's K row and V row (one 8-byte load each, 256 contiguous bytes per warp per
-// row).  The warp reduces the row statistics with shuffles, computes the 4+4 codes
-// per lane, stages the 256 codes in shared memory, builds every group symbol of both
-// rows in parallel (one lane per symbol), ORs the symbols into a shared record image
-// and writes the record to its pool slot with coalesced 4-byte stores.
+// Records are built by destination slot: after a slot -> token map (scatter_tok_kernel),
+// the affine kernel gives a warp 8 consecutive slots of one pool (lanes own half rows);
+// the rotated bases give a 128-thread CTA 64 slots (one thread per row, the whole row
+// in registers).  Either way a CTA's level count is uniform and its record writes are
+// contiguous.  The dense rotation runs its 128 x 128 product on tcgen05 instead.
 //
 // Arithmetic (binary32, round to nearest even, no contraction), per row x:
 //  affine: s = fp16((max-min)/(L-1)) limited to 65504, z = fp16(min);
 //          c = clamp(rint((x - z) * fl(1/s)), 0, L-1)   (all 0 when s == 0)
+//  rotated affine: u = fl(1/sqrt 128) * FWHT(x * sign); z = fp16 of min u rounded
+//          toward -inf (limited to -65504); s and c as affine on u (all 0 unless s > 0)
 //  TQ:     w = FWHT(x * sign) with butterflies h = 1..64; n = fp16(sqrt(sum x^2))
-//          with the sum taken as 32 in-order partials of 4 squares then an xor
-//          butterfly over lanes 16, 8, 4, 2, 1; u = w * fl(1/n); c = #{k: u > t_k}
+//          with the sum taken as 32 in-order partials of 4 squares then pairwise
+//          stages 16, 8, 4, 2, 1; u = w * fl(1/n); c = #{k: u > t_k}
 #include "common.cuh"
 #include "kernels.h"
 
@@ -24,149 +26,6 @@ namespace {
 constexpr int kWarpsPerBlock = 8;
 constexpr uint32_t kSpinLimitQ = 1u << 22;  // bounded mbarrier polls
 constexpr int kMaxRecWords = 27;  // largest record: affine L=7/8, 2*48+8 = 104 B
-
-struct RowOut {
-  uint32_t codes;  // four 8-bit codes, dims 4l..4l+3
-  uint16_t p0;     // affine: scale; TQ: norm
-  uint16_t p1;     // affine: offset
-};
-
-__device__ __forceinline__ void load4(const uint16_t* row, int lane, float x[4]) {
-  uint2 u = *reinterpret_cast<const uint2*>(row + 4 * lane);
-  x[0] = f16_to_f32((uint16_t)(u.x & 0xFFFF));
-  x[1] = f16_to_f32((uint16_t)(u.x >> 16));
-  x[2] = f16_to_f32((uint16_t)(u.y & 0xFFFF));
-  x[3] = f16_to_f32((uint16_t)(u.y >> 16));
-}
-
-template <int L>
-__device__ __forceinline__ RowOut affine_row(const float x[4]) {
-  float mn = fminf(fminf(x[0], x[1]), fminf(x[2], x[3]));
-  float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) {
-    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-  }
-  // a zero extreme is taken as +0 (fmin/fmax may return either signed zero)
-  if (mn == 0.0f) mn = 0.0f;
-  if (mx == 0.0f) mx = 0.0f;
-  const float s32 = __fdiv_rn(__fsub_rn(mx, mn), (float)(L - 1));
-  RowOut o;
-  o.p0 = f16_param(s32);
-  o.p1 = __half_as_ushort(__float2half_rn(mn));
-  const float s = f16_to_f32(o.p0), z = f16_to_f32(o.p1);
-  o.codes = 0;
-  if (s != 0.0f) {
-    const float inv = __fdiv_rn(1.0f, s);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      int c = __float2int_rn(__fmul_rn(__fsub_rn(x[j], z), inv));
-      c = min(max(c, 0), L - 1);
-      o.codes |= (uint32_t)c << (8 * j);
-    }
-  }
-  return o;
-}
-
-// Unnormalised Walsh-Hadamard transform of a row held 4 values per lane (lane l owns
-// dims 4l..4l+3), butterfly stages h = 1, 2, ..., 64 in order, each (a + b, a - b).
-__device__ __forceinline__ void fwht_lanes(float w[4], int lane) {
-  {  // h = 1: (0,1), (2,3)
-    float a = w[0], b = w[1];
-    w[0] = __fadd_rn(a, b); w[1] = __fsub_rn(a, b);
-    a = w[2]; b = w[3];
-    w[2] = __fadd_rn(a, b); w[3] = __fsub_rn(a, b);
-  }
-  {  // h = 2: (0,2), (1,3)
-    float a = w[0], b = w[2];
-    w[0] = __fadd_rn(a, b); w[2] = __fsub_rn(a, b);
-    a = w[1]; b = w[3];
-    w[1] = __fadd_rn(a, b); w[3] = __fsub_rn(a, b);
-  }
-#pragma unroll
-  for (int k = 0; k < 5; ++k) {  // h = 4 << k: partner lane differs in bit k
-    const bool upper = (lane >> k) & 1;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float other = __shfl_xor_sync(0xffffffffu, w[j], 1 << k);
-      w[j] = upper ? __fsub_rn(other, w[j]) : __fadd_rn(w[j], other);
-    }
-  }
-}
-
-template <int L>
-__device__ __forceinline__ RowOut tq_row(const float x[4], const int8_t* sg, int lane,
-                                         const float thr[8]) {
-  // sign flip (exact) then the Walsh-Hadamard butterflies in stage order
-  const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
-  float w[4] = {x[0] * (float)s4.x, x[1] * (float)s4.y, x[2] * (float)s4.z,
-                x[3] * (float)s4.w};
-  fwht_lanes(w, lane);
-  // norm with the fixed tree
-  float acc = __fmul_rn(x[0], x[0]);
-  acc = __fadd_rn(acc, __fmul_rn(x[1], x[1]));
-  acc = __fadd_rn(acc, __fmul_rn(x[2], x[2]));
-  acc = __fadd_rn(acc, __fmul_rn(x[3], x[3]));
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) acc = __fadd_rn(acc, __shfl_xor_sync(0xffffffffu, acc, off));
-  RowOut o;
-  o.p0 = f16_param(__fsqrt_rn(acc));
-  o.p1 = 0;
-  o.codes = 0;
-  const float n = f16_to_f32(o.p0);
-  if (n != 0.0f) {
-    const float inv = __fdiv_rn(1.0f, n);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float u = __fmul_rn(w[j], inv);
-      int c = 0;
-#pragma unroll
-      for (int t = 0; t < L - 1; ++t) c += (u > thr[t]) ? 1 : 0;
-      o.codes |= (uint32_t)c << (8 * j);
-    }
-  }
-  return o;
-}
-
-// Hadamard-rotated affine row: u = fp32(1/sqrt 128) FWHT(x sign); z = fp16 of min u
-// rounded toward -inf (limited to -65504); s = fp16_param((max u - z)/(L-1)); codes as
-// affine_row, all 0 unless s > 0.
-template <int L>
-__device__ __forceinline__ RowOut affine_had_row(const float x[4], const int8_t* sg, int lane) {
-  const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
-  float u[4] = {x[0] * (float)s4.x, x[1] * (float)s4.y, x[2] * (float)s4.z,
-                x[3] * (float)s4.w};
-  fwht_lanes(u, lane);
-#pragma unroll
-  for (int j = 0; j < 4; ++j) u[j] = __fmul_rn(u[j], kInvSqrtD);
-  float mn = fminf(fminf(u[0], u[1]), fminf(u[2], u[3]));
-  float mx = fmaxf(fmaxf(u[0], u[1]), fmaxf(u[2], u[3]));
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) {
-    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-  }
-  if (mn == 0.0f) mn = 0.0f;
-  if (mx == 0.0f) mx = 0.0f;
-  RowOut o;
-  o.p1 = __half_as_ushort(__float2half_rd(mn));
-  if (o.p1 == 0xFC00u) o.p1 = 0xFBFFu;
-  const float z = f16_to_f32(o.p1);
-  o.p0 = f16_param(__fdiv_rn(__fsub_rn(mx, z), (float)(L - 1)));
-  const float s = f16_to_f32(o.p0);
-  o.codes = 0;
-  if (s > 0.0f) {
-    const float inv = __fdiv_rn(1.0f, s);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      int c = __float2int_rn(__fmul_rn(__fsub_rn(u[j], z), inv));
-      c = min(max(c, 0), L - 1);
-      o.codes |= (uint32_t)c << (8 * j);
-    }
-  }
-  return o;
-}
 
 // Build every symbol of the K and V rows from the staged codes and OR it into the
 // record image (both rows: 2 * 4 * (NG + tail) symbols, one lane per symbol).
@@ -420,6 +279,34 @@ __device__ __forceinline__ float f2_hi(unsigned long long v) {
   return __uint_as_float((uint32_t)(v >> 32));
 }
 
+// In-thread unnormalised Walsh-Hadamard transform of one row, butterfly stages 1, 2,
+// ..., 64 in order, each (a + b, a - b) rounded to nearest: stage 1 inside each pair
+// (2k, 2k+1), the later stages on packed pairs (pair k with pair k + hs/2).  The same
+// roundings as any other evaluation of these butterflies in this stage order.
+__device__ __forceinline__ void fwht128(float (&x)[128]) {
+  unsigned long long xp[64];
+#pragma unroll
+  for (int k = 0; k < 64; ++k) {
+    const float p0 = x[2 * k], p1 = x[2 * k + 1];
+    xp[k] = f2_pack(__fadd_rn(p0, p1), __fsub_rn(p0, p1));
+  }
+#pragma unroll
+  for (int hs = 2; hs < 128; hs <<= 1) {
+#pragma unroll
+    for (int k = 0; k < 64; ++k) {
+      if ((2 * k) & hs) continue;
+      const unsigned long long p0 = xp[k], p1 = xp[k + hs / 2];
+      xp[k] = f2_add(p0, p1);
+      xp[k + hs / 2] = f2_sub(p0, p1);
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 64; ++k) {
+    x[2 * k] = f2_lo(xp[k]);
+    x[2 * k + 1] = f2_hi(xp[k]);
+  }
+}
+
 // OR the 96-bit field v at bit pos (compile-time after unrolling) of a row's words
 template <int N>
 __device__ __forceinline__ void or_field(uint32_t (&w)[N], int pos, const uint32_t (&v)[3]) {
@@ -508,29 +395,8 @@ __device__ void rows_block(const QuantArgs& a, int b, int l, int h, bool hi, int
     x[4 * j + 2] *= (float)s4.z;
     x[4 * j + 3] *= (float)s4.w;
   }
-  // ---- Walsh-Hadamard butterflies, stages 1, 2, ..., 64: stage 1 inside each pair
-  // (2k, 2k+1), the later stages on packed pairs (pair k with pair k + hs/2)
-  unsigned long long xp[64];
-#pragma unroll
-  for (int k = 0; k < 64; ++k) {
-    const float p0 = x[2 * k], p1 = x[2 * k + 1];
-    xp[k] = f2_pack(__fadd_rn(p0, p1), __fsub_rn(p0, p1));
-  }
-#pragma unroll
-  for (int hs = 2; hs < 128; hs <<= 1) {
-#pragma unroll
-    for (int k = 0; k < 64; ++k) {
-      if ((2 * k) & hs) continue;
-      const unsigned long long p0 = xp[k], p1 = xp[k + hs / 2];
-      xp[k] = f2_add(p0, p1);
-      xp[k + hs / 2] = f2_sub(p0, p1);
-    }
-  }
-#pragma unroll
-  for (int k = 0; k < 64; ++k) {
-    x[2 * k] = f2_lo(xp[k]);
-    x[2 * k + 1] = f2_hi(xp[k]);
-  }
+  // ---- Walsh-Hadamard butterflies, stages 1, 2, ..., 64
+  fwht128(x);
   if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
     float mn = INFINITY, mx = -INFINITY;
 #pragma unroll
@@ -644,89 +510,171 @@ __global__ void __launch_bounds__(128, 3) quantize_rows_kernel(QuantArgs a, int6
 //   affine: x^_d = fp16( z + s * c_d )
 //   rotated affine: y = FWHT(z + s * c);  x^_d = fp16( (sign_d y_d) * fp32(1/sqrt 128) )
 //   TQ:     y = FWHT(cb[c]) (the quantizer's butterflies);  x^_d = fp16( (sign_d y_d) * (n/128) )
-// One warp per (sequence, layer, KV head, token); lane l owns dims 4l..4l+3.
+// A CTA of 128 threads takes 64 tokens of one (sequence, layer, KV head): thread r
+// owns row r (K of token r/2 when r is even, V when odd), in registers; rows are
+// staged through shared memory on the way in and out for coalesced transfers.
 
-__device__ __forceinline__ void store4_f16(uint16_t* row, int lane, const float y[4]) {
-  uint2 u;
-  u.x = (uint32_t)__half_as_ushort(__float2half_rn(y[0])) |
-        ((uint32_t)__half_as_ushort(__float2half_rn(y[1])) << 16);
-  u.y = (uint32_t)__half_as_ushort(__float2half_rn(y[2])) |
-        ((uint32_t)__half_as_ushort(__float2half_rn(y[3])) << 16);
-  *reinterpret_cast<uint2*>(row + 4 * lane) = u;
-}
-
-template <int BASE, int L>
-__device__ __forceinline__ void fake_row(const float x[4], const int8_t* sg, const float* thr_g,
-                                         const float* cent_g, uint16_t* out, int lane) {
-  float y[4];
-  if constexpr (BASE == SEMKV_BASE_AFFINE) {
-    const RowOut o = affine_row<L>(x);
-    const float s = f16_to_f32(o.p0), z = f16_to_f32(o.p1);
+__device__ __forceinline__ void load_signs(const int8_t* sg, float (&x)[128]) {
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
-      y[j] = __fadd_rn(z, __fmul_rn(s, (float)((o.codes >> (8 * j)) & 0xFFu)));
-  } else if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
-    const RowOut o = affine_had_row<L>(x, sg, lane);
-    const float s = f16_to_f32(o.p0), z = f16_to_f32(o.p1);
-    float w[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-      w[j] = __fadd_rn(z, __fmul_rn(s, (float)((o.codes >> (8 * j)) & 0xFFu)));
-    fwht_lanes(w, lane);
-    const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
-    const float sgn[4] = {(float)s4.x, (float)s4.y, (float)s4.z, (float)s4.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) y[j] = __fmul_rn(w[j] * sgn[j], kInvSqrtD);
-  } else {
-    float thr[8];
-#pragma unroll
-    for (int t = 0; t < 8; ++t) thr[t] = t < L - 1 ? thr_g[t] : 0.0f;
-    const RowOut o = tq_row<L>(x, sg, lane, thr);
-    float w[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) w[j] = cent_g[(o.codes >> (8 * j)) & 0xFFu];
-    fwht_lanes(w, lane);
-    const float nq = f16_to_f32(o.p0) * 0.0078125f;
-    const char4 s4 = *reinterpret_cast<const char4*>(sg + 4 * lane);
-    const float sgn[4] = {(float)s4.x, (float)s4.y, (float)s4.z, (float)s4.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) y[j] = __fmul_rn(w[j] * sgn[j], nq);
+  for (int j = 0; j < 32; ++j) {
+    const char4 s4 = __ldg(reinterpret_cast<const char4*>(sg) + j);
+    x[4 * j] *= (float)s4.x;
+    x[4 * j + 1] *= (float)s4.y;
+    x[4 * j + 2] *= (float)s4.z;
+    x[4 * j + 3] *= (float)s4.w;
   }
-  store4_f16(out, lane, y);
 }
 
 template <int BASE>
-__global__ void __launch_bounds__(kWarpsPerBlock * 32) fake_quant_kernel(FakeArgs a) {
-  const int lane = threadIdx.x & 31;
-  const int64_t total = (int64_t)a.B * a.NL * a.H * a.T;
-  const int64_t nwarps = (int64_t)gridDim.x * kWarpsPerBlock;
-  for (int64_t task = (int64_t)blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5); task < total;
-       task += nwarps) {
-    const int t = (int)(task % a.T);
-    int64_t r = task / a.T;
-    const int h = (int)(r % a.H);
-    r /= a.H;
-    const int l = (int)(r % a.NL);
-    const int b = (int)(r / a.NL);
-    const bool hi = a.is_high ? a.is_high[(int64_t)b * a.T + t] != 0 : true;
-    const int L = hi ? a.L_hi : a.L_lo;
-    const int64_t row = task * kHeadDim;
-    float kx[4], vx[4];
-    load4(a.k + row, lane, kx);
-    load4(a.v + row, lane, vx);
-    const int8_t* sg = a.signs ? a.signs + ((int64_t)l * a.H + h) * kHeadDim : nullptr;
-    const float* thr = hi ? a.thr_hi : a.thr_lo;
-    const float* cent = hi ? a.cent_hi : a.cent_lo;
-    switch (L) {
-#define SEMKV_FAKE_CASE(LV)                                             \
-      case LV:                                                          \
-        fake_row<BASE, LV>(kx, sg, thr, cent, a.k_out + row, lane);     \
-        fake_row<BASE, LV>(vx, sg, thr, cent, a.v_out + row, lane);     \
-        break;
-      SEMKV_FAKE_CASE(2) SEMKV_FAKE_CASE(3) SEMKV_FAKE_CASE(4) SEMKV_FAKE_CASE(5)
-      SEMKV_FAKE_CASE(6) SEMKV_FAKE_CASE(7) SEMKV_FAKE_CASE(8)
-#undef SEMKV_FAKE_CASE
-      default: break;
+__global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : 3) fake_rows_kernel(FakeArgs a) {
+  __shared__ __align__(16) uint8_t stage[128 * kRowStride];
+  __shared__ float cbs[2][8];
+  const int tid = threadIdx.x;
+  if (BASE == SEMKV_BASE_TQ && tid < 16) {
+    const int which = tid >> 3, k = tid & 7;
+    const int L = which ? a.L_lo : a.L_hi;
+    cbs[which][k] = k < L ? (which ? a.cent_lo : a.cent_hi)[k] : 0.0f;
+  }
+  const int64_t bhs = (int64_t)a.B * a.NL * a.H;
+  for (int64_t bhi = blockIdx.y; bhi < bhs; bhi += gridDim.y) {
+    const int h = (int)(bhi % a.H), l = (int)((bhi / a.H) % a.NL);
+    const int b = (int)(bhi / ((int64_t)a.H * a.NL));
+    for (int t0 = blockIdx.x * kRowSlots; t0 < a.T; t0 += gridDim.x * kRowSlots) {
+      const int nt = min(kRowSlots, a.T - t0);
+      const int64_t row0 = bhi * a.T + t0;
+      for (int c = tid; c < 128 * 16; c += 128) {
+        const int r = c >> 4, ch = c & 15, i = r >> 1;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (i < nt) v = __ldg(reinterpret_cast<const uint4*>(((r & 1) ? a.v : a.k) + (row0 + i) * kHeadDim) + ch);
+        *reinterpret_cast<uint4*>(stage + r * kRowStride + ch * 16) = v;
+      }
+      __syncthreads();
+      const int i = tid >> 1;
+      const bool hi = i < nt && (a.is_high == nullptr || a.is_high[(int64_t)b * a.T + t0 + i] != 0);
+      const int L = (a.is_high == nullptr || hi) ? a.L_hi : a.L_lo;
+      float x[128];
+#pragma unroll
+      for (int ch = 0; ch < 16; ++ch) {
+        const uint4 u = *reinterpret_cast<const uint4*>(stage + tid * kRowStride + ch * 16);
+        const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
+          x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
+        }
+      }
+      const int8_t* sg = a.signs ? a.signs + ((int64_t)l * a.H + h) * kHeadDim : nullptr;
+      if constexpr (BASE == SEMKV_BASE_AFFINE) {
+        // x^_d = fp16(z + s c_d)
+        float mn = x[0], mx = x[0];
+#pragma unroll
+        for (int j = 1; j < 128; ++j) {
+          mn = fminf(mn, x[j]);
+          mx = fmaxf(mx, x[j]);
+        }
+        if (mn == 0.0f) mn = 0.0f;
+        if (mx == 0.0f) mx = 0.0f;
+        const uint16_t s16 = f16_param(__fdiv_rn(__fsub_rn(mx, mn), (float)(L - 1)));
+        const float sv = f16_to_f32(s16), z = f16_to_f32(__half_as_ushort(__float2half_rn(mn)));
+        const float inv = sv != 0.0f ? __fdiv_rn(1.0f, sv) : 0.0f;
+#pragma unroll
+        for (int j = 0; j < 128; ++j) {
+          int c = 0;
+          if (sv != 0.0f) c = min(max(__float2int_rn(__fmul_rn(__fsub_rn(x[j], z), inv)), 0), L - 1);
+          x[j] = __fadd_rn(z, __fmul_rn(sv, (float)c));
+        }
+      } else if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
+        // y = FWHT(z + s c);  x^_d = fp16((sign_d y_d) * fp32(1/sqrt 128))
+        load_signs(sg, x);
+        fwht128(x);
+        float mn = INFINITY, mx = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < 128; ++j) {
+          x[j] = __fmul_rn(x[j], kInvSqrtD);
+          mn = fminf(mn, x[j]);
+          mx = fmaxf(mx, x[j]);
+        }
+        if (mn == 0.0f) mn = 0.0f;
+        if (mx == 0.0f) mx = 0.0f;
+        uint16_t z16 = __half_as_ushort(__float2half_rd(mn));
+        if (z16 == 0xFC00u) z16 = 0xFBFFu;
+        const float z = f16_to_f32(z16);
+        const float sv = f16_to_f32(f16_param(__fdiv_rn(__fsub_rn(mx, z), (float)(L - 1))));
+        const bool live = sv > 0.0f;
+        const float inv = live ? __fdiv_rn(1.0f, sv) : 0.0f;
+#pragma unroll
+        for (int j = 0; j < 128; ++j) {
+          int c = 0;
+          if (live) c = min(max(__float2int_rn(__fmul_rn(__fsub_rn(x[j], z), inv)), 0), L - 1);
+          x[j] = __fadd_rn(z, __fmul_rn(sv, (float)c));
+        }
+        fwht128(x);
+        load_signs(sg, x);
+#pragma unroll
+        for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], kInvSqrtD);
+      } else {
+        // y = FWHT(cb[c]);  x^_d = fp16((sign_d y_d) * (n / 128))
+        float pn[16];
+#pragma unroll
+        for (int g = 0; g < 16; ++g) {
+          float acc[2];
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            const int gg = g + 16 * hh;
+            float v = __fmul_rn(x[4 * gg], x[4 * gg]);
+#pragma unroll
+            for (int k = 1; k < 4; ++k) v = __fadd_rn(v, __fmul_rn(x[4 * gg + k], x[4 * gg + k]));
+            acc[hh] = v;
+          }
+          pn[g] = __fadd_rn(acc[0], acc[1]);
+        }
+#pragma unroll
+        for (int off = 8; off >= 1; off >>= 1)
+#pragma unroll
+          for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
+        const uint16_t n16 = f16_param(__fsqrt_rn(pn[0]));
+        const float n = f16_to_f32(n16);
+        const float inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
+        const float* thr_g = hi || a.is_high == nullptr ? a.thr_hi : a.thr_lo;
+        const float* cb = cbs[(hi || a.is_high == nullptr) ? 0 : 1];
+        float thr[7];
+#pragma unroll
+        for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? thr_g[k] : INFINITY;
+        load_signs(sg, x);
+        fwht128(x);
+#pragma unroll
+        for (int j = 0; j < 128; ++j) {
+          const float u = __fmul_rn(x[j], inv);
+          int c = 0;
+#pragma unroll
+          for (int k = 0; k < 7; ++k) c += (u > thr[k]) ? 1 : 0;
+          x[j] = cb[n != 0.0f ? c : 0];
+        }
+        fwht128(x);
+        load_signs(sg, x);
+        const float nq = n * 0.0078125f;
+#pragma unroll
+        for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], nq);
+      }
+      __syncthreads();  // every row is read: the stage takes the outputs
+#pragma unroll
+      for (int ch = 0; ch < 16; ++ch) {
+        uint4 u;
+        uint32_t* wv = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          wv[e] = (uint32_t)__half_as_ushort(__float2half_rn(x[8 * ch + 2 * e])) |
+                  ((uint32_t)__half_as_ushort(__float2half_rn(x[8 * ch + 2 * e + 1])) << 16);
+        *reinterpret_cast<uint4*>(stage + tid * kRowStride + ch * 16) = u;
+      }
+      __syncthreads();
+      for (int c = tid; c < 128 * 16; c += 128) {
+        const int r = c >> 4, ch = c & 15, ii = r >> 1;
+        if (ii < nt)
+          reinterpret_cast<uint4*>(((r & 1) ? a.v_out : a.k_out) + (row0 + ii) * kHeadDim)[ch] =
+              *reinterpret_cast<const uint4*>(stage + r * kRowStride + ch * 16);
+      }
+      __syncthreads();
     }
   }
 }
@@ -981,17 +929,19 @@ __global__ void __launch_bounds__(128) quantize_tq_dense_kernel(QuantArgs a) {
 }  // namespace
 
 cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t stream) {
+  (void)num_sms;
   const int64_t total = (int64_t)a.B * a.NL * a.H * a.T;
   if (total == 0) return cudaSuccess;
-  int64_t blocks = (total + kWarpsPerBlock - 1) / kWarpsPerBlock;
-  const int64_t cap = (int64_t)num_sms * 32;  // grid-stride beyond this
-  if (blocks > cap) blocks = cap;
+  const int64_t bhs = (int64_t)a.B * a.NL * a.H;
+  int64_t bx = ((int64_t)a.T + kRowSlots - 1) / kRowSlots;
+  if (bx > 65535) bx = 65535;
+  const dim3 grid((unsigned)bx, (unsigned)(bhs < 65535 ? bhs : 65535));
   if (a.base == SEMKV_BASE_AFFINE)
-    fake_quant_kernel<SEMKV_BASE_AFFINE><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+    fake_rows_kernel<SEMKV_BASE_AFFINE><<<grid, 128, 0, stream>>>(a);
   else if (a.base == SEMKV_BASE_AFFINE_HAD)
-    fake_quant_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+    fake_rows_kernel<SEMKV_BASE_AFFINE_HAD><<<grid, 128, 0, stream>>>(a);
   else
-    fake_quant_kernel<SEMKV_BASE_TQ><<<(unsigned)blocks, kWarpsPerBlock * 32, 0, stream>>>(a);
+    fake_rows_kernel<SEMKV_BASE_TQ><<<grid, 128, 0, stream>>>(a);
   return cudaGetLastError();
 }
 
