@@ -13,6 +13,8 @@
 //   high(i)        = key_i > theta  or  (key_i == theta and eq_before(i) < need)
 //   high_before(i) = gt_before(i) + min(eq_before(i), need)
 //   slot(i)        = high(i) ? high_before(i) : i - high_before(i).
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -227,6 +229,158 @@ __global__ void __launch_bounds__(kThreads) rank_assign_kernel(RankArgs a) {
   }
 }
 
+// ---- long sequences on a thread-block cluster -----------------------------------
+// The same selection and sweep with one sequence spread over a cluster of kCluster
+// CTAs: CTA r keeps the keys of tokens [r chunk, (r+1) chunk) in its shared memory and
+// counts them into its own histograms; each pass every CTA sums the cluster's 256-bin
+// histograms through distributed shared memory and takes the same bin (the choice is
+// deterministic); for the sweep each CTA adds the (greater, equal) totals of the CTAs
+// before it, so every token sees the counts of all earlier tokens of the sequence.
+constexpr int kCluster = 8;
+
+__global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
+    rank_cluster_kernel(RankArgs a) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cluster = cg::this_cluster();
+  extern __shared__ uint32_t ckeys[];
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t whist[kThreads / 32][256];
+  __shared__ uint32_t sel_bin, sel_above;
+  __shared__ uint64_t warp_sums[32];
+  __shared__ uint64_t chunk_total;
+  const int rank_in = (int)cluster.block_rank();
+  const int b = blockIdx.x / kCluster;
+  const float* s = a.scores + (int64_t)b * a.ld;
+  uint8_t* is_high = a.is_high + (int64_t)b * a.T;
+  uint32_t* slot = a.slot + (int64_t)b * a.T;
+  const uint32_t T = (uint32_t)a.T;
+  const uint32_t chunk = (T + kCluster - 1) / kCluster;
+  const uint32_t c_begin = min(T, (uint32_t)rank_in * chunk);
+  const uint32_t c_end = min(T, c_begin + chunk);
+  const uint32_t nloc = c_end - c_begin;
+  const int tid = threadIdx.x;
+
+  if (a.n_high == 0 || a.n_high == T) {  // the same branch in every CTA of the cluster
+    const uint8_t all = a.n_high == T ? 1 : 0;
+    for (uint32_t i = c_begin + tid; i < c_end; i += kThreads) {
+      is_high[i] = all;
+      slot[i] = i;
+    }
+    return;
+  }
+  for (uint32_t i = tid; i < nloc; i += kThreads) ckeys[i] = order_key(s[c_begin + i]);
+
+  uint32_t prefix = 0, mask = 0, k = a.n_high;
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    uint32_t* wh = whist[tid >> 5];
+    for (int i = tid; i < (kThreads / 32) * 256; i += kThreads) (&whist[0][0])[i] = 0;
+    __syncthreads();
+    for (uint32_t i0 = 0; i0 < nloc; i0 += kThreads * kSelItems) {
+      uint32_t key[kSelItems];
+#pragma unroll
+      for (int j = 0; j < kSelItems; ++j) {
+        const uint32_t i = i0 + j * kThreads + tid;
+        key[j] = i < nloc ? ckeys[i] : 0u;
+      }
+#pragma unroll
+      for (int j = 0; j < kSelItems; ++j) {
+        const uint32_t i = i0 + j * kThreads + tid;
+        if (i < nloc && (key[j] & mask) == prefix) atomicAdd(&wh[(key[j] >> shift) & 0xFFu], 1u);
+      }
+    }
+    __syncthreads();
+    for (int i = tid; i < 256; i += kThreads) {
+      uint32_t c = 0;
+#pragma unroll 8
+      for (int w = 0; w < kThreads / 32; ++w) c += whist[w][i];
+      hist[i] = c;
+    }
+    cluster.sync();  // every CTA's histogram is complete
+    if (tid < 32) {
+      // the cluster's counts, summed in CTA order (each CTA reaches the same totals)
+      uint32_t tot[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) tot[e] = 0;
+      for (int r = 0; r < kCluster; ++r) {
+        const uint32_t* rh = cluster.map_shared_rank(hist, r);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) tot[e] += rh[255 - 8 * tid - e];
+      }
+      // select_bin over the summed counts (lane l holds bins 255 - 8l .. 248 - 8l)
+      uint32_t sum = 0;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) sum += tot[e];
+      uint32_t incl = sum;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (tid >= off) incl += y;
+      }
+      const uint32_t excl = incl - sum;
+      if (excl < k && incl >= k) {
+        uint32_t cum = excl;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          if (cum + tot[e] >= k) {
+            sel_bin = 255u - 8u * tid - (uint32_t)e;
+            sel_above = cum;
+            break;
+          }
+          cum += tot[e];
+        }
+      }
+    }
+    cluster.sync();  // every CTA has read the others' histograms: they may be reset
+    prefix |= sel_bin << shift;
+    k -= sel_above;
+    mask |= 0xFFu << shift;
+  }
+  const uint32_t theta = prefix, need = k;
+
+  // ---- this CTA's (greater, equal) totals, then the totals of the CTAs before it
+  {
+    uint64_t local = 0;
+    for (uint32_t i = tid; i < nloc; i += kThreads)
+      local += (ckeys[i] > theta ? 1ull : 0ull) | ((ckeys[i] == theta ? 1ull : 0ull) << 32);
+    uint64_t total;
+    (void)block_exclusive_scan(local, warp_sums, &total);
+    if (tid == 0) chunk_total = total;
+  }
+  cluster.sync();
+  uint64_t run = 0;
+  for (int r = 0; r < rank_in; ++r) run += *cluster.map_shared_rank(&chunk_total, r);
+  cluster.sync();  // no CTA leaves while another still reads its shared memory
+
+  for (uint32_t c0 = 0; c0 < nloc; c0 += kThreads * kItems) {
+    uint32_t keys[kItems];
+    uint64_t local = 0;
+#pragma unroll
+    for (int j = 0; j < kItems; ++j) {
+      const uint32_t i = c0 + tid * kItems + j;
+      keys[j] = i < nloc ? ckeys[i] : 0u;
+      if (i < nloc) local += (keys[j] > theta ? 1ull : 0ull) | ((keys[j] == theta ? 1ull : 0ull) << 32);
+    }
+    uint64_t total;
+    uint64_t before = run + block_exclusive_scan(local, warp_sums, &total);
+#pragma unroll
+    for (int j = 0; j < kItems; ++j) {
+      const uint32_t il = c0 + tid * kItems + j;
+      if (il >= nloc) break;
+      const uint32_t i = c_begin + il;
+      const uint32_t gt_b = (uint32_t)(before & 0xFFFFFFFFu);
+      const uint32_t eq_b = (uint32_t)(before >> 32);
+      const bool gt = keys[j] > theta, eq = keys[j] == theta;
+      const bool hi = gt || (eq && eq_b < need);
+      const uint32_t hib = gt_b + min(eq_b, need);
+      is_high[i] = hi ? 1 : 0;
+      slot[i] = hi ? hib : i - hib;
+      before += (gt ? 1ull : 0ull) | ((eq ? 1ull : 0ull) << 32);
+    }
+    run += total;
+  }
+}
+
 // ---- full ranks (optional output): a stable LSD radix sort of the inverted keys
 // (ascending inverted key = descending score; a stable pass keeps equal keys in index
 // order, which is the tie rule), 4-bit digits in 8 passes, one CTA per sequence,
@@ -330,8 +484,19 @@ size_t rank_workspace_words(int B, int T) { return (size_t)B * 4 * (size_t)T; }
 
 cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream) {
   if (a.B == 0 || a.T == 0) return cudaSuccess;
+  const uint32_t chunk = ((uint32_t)a.T + kCluster - 1) / kCluster;
   if (a.T <= kThreads) {
     rank_small_kernel<<<a.B, kThreads, 0, stream>>>(a);
+  } else if (a.T >= 8192 && chunk <= kSmemKeys) {
+    static bool cattr_set = false;
+    if (!cattr_set) {
+      const cudaError_t e = cudaFuncSetAttribute(rank_cluster_kernel,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)(kSmemKeys * sizeof(uint32_t)));
+      if (e != cudaSuccess) return e;
+      cattr_set = true;
+    }
+    rank_cluster_kernel<<<a.B * kCluster, kThreads, (size_t)chunk * sizeof(uint32_t), stream>>>(a);
   } else {
     static bool attr_set = false;
     if (!attr_set) {
