@@ -16,6 +16,9 @@
 //  TQ:     w = FWHT(x * sign) with butterflies h = 1..64; n = fp16(sqrt(sum x^2))
 //          with the sum taken as 32 in-order partials of 4 squares then pairwise
 //          stages 16, 8, 4, 2, 1; u = w * fl(1/n); c = #{k: u > t_k}
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -27,40 +30,13 @@ constexpr int kWarpsPerBlock = 8;
 constexpr uint32_t kSpinLimitQ = 1u << 22;  // bounded mbarrier polls
 constexpr int kMaxRecWords = 27;  // largest record: affine L=7/8, 2*48+8 = 104 B
 
-// Build every symbol of the K and V rows from the staged codes and OR it into the
-// record image (both rows: 2 * 4 * (NG + tail) symbols, one lane per symbol).
-template <int L>
-__device__ __forceinline__ void pack_rows(const uint8_t* codes, uint32_t* rec, int lane) {
-  using F = Fmt<L>;
-  constexpr int kSymQ = F::NG + (F::R > 0 ? 1 : 0);
-  constexpr int kSymRow = 4 * kSymQ;
-  for (int idx = lane; idx < 2 * kSymRow; idx += 32) {
-    const int row = idx / kSymRow;
-    const int j = idx - row * kSymRow;
-    const int q = j / kSymQ;
-    const int s = j - q * kSymQ;
-    const bool tail = s == F::NG;
-    const int n = tail ? F::R : F::G;
-    const int w = tail ? F::WT : F::W;
-    const uint32_t m = tail ? F::LR : F::LG;
-    const int d0 = 32 * q + (tail ? 32 - F::R : s * F::G);
-    uint32_t t = 0;
-    for (int k = 0; k < n; ++k) t = t * (uint32_t)L + codes[row * 128 + d0 + k];
-    const uint32_t beta = ((t << w) + m - 1u) / m;
-    const int pos = row * 8 * F::RB + q * F::QB + s * F::W;
-    const int word = pos >> 5, sh = pos & 31;
-    atomicOr(&rec[word], beta << sh);
-    if (sh + w > 32) atomicOr(&rec[word + 1], beta >> (32 - sh));
-  }
-}
-
 // ------------------------------------------------- affine pools, by slot -----
 // Affine records are built by destination slot: a warp takes units of 8 consecutive
 // slots of one pool of one (sequence, layer, KV head), so the level count is uniform
 // across the warp and the records it writes are contiguous.  Lane 4i + 2r + f handles
 // half f (dims 64f..64f+63, quarters 2f and 2f+1) of row r (0 = K, 1 = V) of the i-th
 // slot's token: 128 contiguous bytes in, two quarter bit fields out.  The same
-// arithmetic as affine_row, and symbols beta = ceil(t 2^W / L^G) as in pack_rows.
+// arithmetic as the header states, and symbols beta = ceil(t 2^W / L^G) (the record format).
 
 constexpr int kAffineSlots = 8;
 
@@ -680,36 +656,55 @@ __global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : 3) fake_rows_
 }
 
 // ------------------------------------- dense-rotation TQ rows (tcgen05) --------
-// One CTA of 4 warps per 64 tokens of one (sequence, layer, KV head).  The 128 rows
-// of the tile (K and V of each token, rows 2i and 2i+1) are rotated on the tensor
-// cores: W[r][i] = sum_j X[r][j] M[i][j], tcgen05.mma kind::f16 with M = N = 128 and
-// K = 8 x 16, both operands K-major in shared memory without swizzle, the fp32
-// accumulator in tensor memory (128 lanes x 128 columns).  Thread r then owns row r:
-// the fixed-tree norm (from the staged row, while the MMAs run), the TMEM row, the
-// codes.  The warps pack the records with pack_rows.
+// Persistent CTAs of 8 warps (two per SM), each over a contiguous range of 64-token
+// tiles of one (sequence, layer, KV head).  The head's rotation M (128 x 128 fp16, the
+// A operand) is staged once per CTA.  The K and V rows of a tile arrive by TMA, one 3-D
+// tensor copy each (dims: 8 values, rows, 16 groups of 8 values), so they land as
+// 8-row x 16-byte core matrices, K-major without swizzle, completing on an mbarrier;
+// the next tile's copy starts as soon as the MMAs have read the current one, under the
+// codes and the packing.  One thread issues D^T = M X^T on tcgen05 (kind::f16,
+// M = 128 output dims, N = 64 tokens, K = 8 x 16) for the K rows and for the V rows into
+// 128 fp32 columns of tensor memory and commits to an mbarrier.  Meanwhile the threads
+// take the rows' fixed-tree norms from the tile (two threads per row); then warp w
+// reads TMEM lanes 32 (w % 4).. (output dims) of the K (w < 4) or V (w >= 4) columns,
+// writes the codes into a row-major code tile; a thread per row builds the row's
+// bit image (the quarter fields) and the warps write the records word by word.
 constexpr int kDenseTok = 64;
-constexpr uint32_t kDenseTile = 128 * 128 * 2;  // bytes of one operand tile
+constexpr int kDenseThreads = 256;
+constexpr uint32_t kDenseM = 128 * 128 * 2;   // the rotation, bytes
+constexpr uint32_t kDenseBox = 64 * 128 * 2;  // one TMA box: 64 rows of K or of V
+constexpr uint32_t kDenseSmem = kDenseM + 2 * kDenseBox + 128 * 128 + 1024;  // + codes, align
 // instruction descriptor: fp32 accumulate (bits 4-5 = 1), A and B fp16 (formats 0),
 // both K-major, N >> 3 at bits 17-22, M >> 4 at bits 24-28
-constexpr uint32_t kDenseIdesc = (1u << 4) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
+constexpr uint32_t kDenseIdesc = (1u << 4) | ((64u >> 3) << 17) | ((128u >> 4) << 24);
 
-// core-matrix layout of a [128][128] fp16 K-major tile: 8 rows x 16 bytes per core
-// matrix, core matrices 128 bytes apart along K and 2048 bytes apart along rows; the
-// 16-byte chunk c = (rg, kg, rr) (rr fastest) sits at byte 16 c
-__device__ __forceinline__ uint32_t dense_off(int r, int k) {
-  return (uint32_t)((r >> 3) * 2048 + (k >> 3) * 128 + (r & 7) * 16 + (k & 7) * 2);
-}
-// shared-memory matrix descriptor: start >> 4 (bits 0-13), leading (K) core-matrix
-// offset 128 >> 4 (bits 16-29), stride (row-group) offset 2048 >> 4 (bits 32-45),
-// descriptor version 1 (bits 46-47), no swizzle
-__device__ __forceinline__ uint64_t dense_desc(uint32_t saddr) {
-  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)(128u >> 4) << 16) |
-         ((uint64_t)(2048u >> 4) << 32) | ((uint64_t)1 << 46);
+// shared-memory matrix descriptor without swizzle: start >> 4 (bits 0-13), leading
+// (K-direction) core-matrix offset >> 4 (bits 16-29), stride (8-row group) offset >> 4
+// (bits 32-45), descriptor version 1 (bits 46-47)
+__device__ __forceinline__ uint64_t umma_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+         ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46);
 }
 __device__ __forceinline__ uint32_t dsmem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
 }
-// 32 columns of this warp's 32 TMEM lanes (lane i of the warp <- TMEM lane 32w + i)
+__device__ __forceinline__ void dbar_init(uint64_t* bar) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(dsmem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool dbar_wait(uint64_t* bar, uint32_t parity) {
+  for (uint32_t i = 0; i < kSpinLimitQ; ++i) {
+    uint32_t r;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(r)
+        : "r"(dsmem_u32(bar)), "r"(parity)
+        : "memory");
+    if (r) return true;
+  }
+  return false;
+}
+// 32 columns of this warp's 32 TMEM lanes (lane i of the warp <- TMEM lane 32 (w % 4) + i)
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
@@ -723,34 +718,63 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// the bit image of one row of 128 codes (bytes) as the record stores it
 template <int L>
-__device__ __forceinline__ void dense_pack(const uint8_t* codes, uint16_t nk, uint16_t nv,
-                                           uint8_t* dst, uint32_t* rec, int lane) {
+__device__ __forceinline__ void row_bits(const uint8_t* crow, uint32_t* out) {
   using F = Fmt<L>;
-  constexpr int kRecWords = (2 * F::RB + 4) / 4;
-  if (lane < kRecWords) rec[lane] = 0u;
-  __syncwarp();
-  pack_rows<L>(codes, rec, lane);
-  if (lane == 0) rec[(2 * F::RB) / 4] = (uint32_t)nk | ((uint32_t)nv << 16);
-  __syncwarp();
-  if (lane < kRecWords) reinterpret_cast<uint32_t*>(dst)[lane] = rec[lane];
-  __syncwarp();
+  constexpr int kWords = (4 * F::QB + 31) / 32;
+  uint32_t w[12];
+#pragma unroll
+  for (int k = 0; k < 12; ++k) w[k] = 0u;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint32_t m[32];
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {
+      const uint4 u0 = *reinterpret_cast<const uint4*>(crow + 32 * q + 16 * c);
+      const uint32_t wv[4] = {u0.x, u0.y, u0.z, u0.w};
+#pragma unroll
+      for (int e = 0; e < 16; ++e) m[16 * c + e] = 0x4B400000u + ((wv[e >> 2] >> (8 * (e & 3))) & 0xFFu);
+    }
+    uint32_t fw[3];
+    quarter_field<L>(m, fw);
+    or_field<12>(w, q * F::QB, fw);
+  }
+#pragma unroll
+  for (int k = 0; k < kWords; ++k) out[k] = w[k];
 }
 
-__global__ void __launch_bounds__(128) quantize_tq_dense_kernel(QuantArgs a) {
-  extern __shared__ __align__(1024) uint8_t dsm[];
-  uint8_t* xa = dsm;               // A: the tile's rows; after the MMAs, their codes
-  uint8_t* mb = dsm + kDenseTile;  // B: the rotation of (layer, head)
-  __shared__ __align__(8) uint64_t bar;
+__global__ void __launch_bounds__(kDenseThreads, 2)
+    quantize_tq_dense_kernel(const __grid_constant__ CUtensorMap tmk,
+                             const __grid_constant__ CUtensorMap tmv, QuantArgs a) {
+  extern __shared__ uint8_t dsm_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~(uintptr_t)1023);
+  uint8_t* ma = base;                       // A: the rotation, core-matrix layout
+  uint8_t* xk = base + kDenseM;             // the tile: K box, then V box
+  uint8_t* codes = xk + 2 * kDenseBox;      // [128 rows: K of token t = 2t, V = 2t+1][128]
+  __shared__ __align__(8) uint64_t tma_bar, mma_bar;
   __shared__ uint32_t tmem_base;
   __shared__ uint16_t nrm[128];
-  __shared__ __align__(16) uint32_t rec_sm[4][kMaxRecWords + 1];
+  __shared__ float invs[128];
+  __shared__ uint8_t tokhi[kDenseTok];
+  __shared__ uint32_t rbits[128 * kRowBitWords];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t bhs = (int64_t)a.B * a.NL * a.H;
-  const int t0 = blockIdx.x * kDenseTok;
+  const int64_t bhl = blockIdx.y;
+  const int h = (int)(bhl % a.H), l = (int)((bhl / a.H) % a.NL);
+  const int b = (int)(bhl / ((int64_t)a.H * a.NL));
+  const int tiles = (a.n + kDenseTok - 1) / kDenseTok;
+  const int per = (tiles + (int)gridDim.x - 1) / (int)gridDim.x;
+  const int j0 = min(tiles, (int)blockIdx.x * per), j1 = min(tiles, j0 + per);
+  float th_hi[7], th_lo[7];
+#pragma unroll
+  for (int k = 0; k < 7; ++k) {
+    th_hi[k] = k < a.L_hi - 1 ? a.thr_hi[k] : INFINITY;
+    th_lo[k] = k < a.L_lo - 1 ? a.thr_lo[k] : INFINITY;
+  }
 
   if (tid == 0) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(dsmem_u32(&bar)) : "memory");
+    dbar_init(&tma_bar);
+    dbar_init(&mma_bar);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -759,138 +783,158 @@ __global__ void __launch_bounds__(128) quantize_tq_dense_kernel(QuantArgs a) {
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
+  // the rotation: 16-byte chunk c = (row group, k group, row in group) at byte 16 c
+  const uint4* msrc = reinterpret_cast<const uint4*>(a.rot + ((int64_t)l * a.H + h) * 128 * 128);
+  for (int c = tid; c < 128 * 16; c += kDenseThreads) {
+    const int rr = c & 7, kg = (c >> 3) & 15, r = (c >> 7) * 8 + rr;
+    reinterpret_cast<uint4*>(ma)[c] = msrc[r * 16 + kg];
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tb = tmem_base;
+  const int row_base = (int)(bhl * a.Tsrc);  // first row of this (b, l, h) in the row view
 
-  uint32_t phase = 0;
+  auto issue_tma = [&](int j) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(dsmem_u32(&tma_bar)),
+                 "r"(2 * kDenseBox)
+                 : "memory");
+    const int row = row_base + j * kDenseTok;
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dsmem_u32(xk)),
+        "l"(reinterpret_cast<uint64_t>(&tmk)), "r"(0), "r"(row), "r"(0), "r"(dsmem_u32(&tma_bar))
+        : "memory");
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dsmem_u32(xk + kDenseBox)),
+        "l"(reinterpret_cast<uint64_t>(&tmv)), "r"(0), "r"(row), "r"(0), "r"(dsmem_u32(&tma_bar))
+        : "memory");
+  };
+  if (tid == 0 && j0 < j1) issue_tma(j0);
   bool ok = true;
-  for (int64_t bhl = blockIdx.y; bhl < bhs && ok; bhl += gridDim.y) {
-    const int h = (int)(bhl % a.H);
-    const int l = (int)((bhl / a.H) % a.NL);
-    const int b = (int)(bhl / ((int64_t)a.H * a.NL));
-    // ---- stage both operands (16-byte chunk c goes to byte 16 c)
-    const uint4* msrc = reinterpret_cast<const uint4*>(a.rot + ((int64_t)l * a.H + h) * 128 * 128);
-    const int64_t row0 = (((int64_t)b * a.NL + l) * a.H + h) * a.Tsrc;
-    for (int c = tid; c < 128 * 16; c += 128) {
-      const int rr = c & 7, kg = (c >> 3) & 15, r = (c >> 7) * 8 + rr;
-      reinterpret_cast<uint4*>(mb)[c] = msrc[r * 16 + kg];
-      const int t = t0 + (r >> 1);
-      uint4 x = make_uint4(0u, 0u, 0u, 0u);
-      if (t < a.n) {
-        const uint16_t* src = ((r & 1) ? a.v : a.k) + (row0 + t) * 128;
-        x = reinterpret_cast<const uint4*>(src)[kg];
-      }
-      reinterpret_cast<uint4*>(xa)[c] = x;
-    }
-    // generic-proxy writes -> visible to the tensor cores (async proxy)
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
+  for (int j = j0; j < j1 && ok; ++j) {
+    const uint32_t par = (uint32_t)((j - j0) & 1);
+    ok = __syncthreads_and(dbar_wait(&tma_bar, par)) != 0;
+    if (!ok) break;
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     if (tid == 0) {
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const uint64_t da = dense_desc(dsmem_u32(xa) + k * 256);
-        const uint64_t db = dense_desc(dsmem_u32(mb) + k * 256);
-        asm volatile(
-            "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n"
-            " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tb),
-            "l"(da), "l"(db), "r"(kDenseIdesc), "r"((uint32_t)(k > 0))
-            : "memory");
+      for (int half = 0; half < 2; ++half) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const uint64_t da = umma_desc(dsmem_u32(ma) + k * 256, 128, 2048);
+          const uint64_t db = umma_desc(dsmem_u32(xk + half * kDenseBox) + k * 2048, 1024, 128);
+          asm volatile(
+              "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n"
+              " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(
+                  tb + (uint32_t)(half * 64)),
+              "l"(da), "l"(db), "r"(kDenseIdesc), "r"((uint32_t)(k > 0))
+              : "memory");
+        }
       }
       asm volatile(
           "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-              dsmem_u32(&bar))
+              dsmem_u32(&mma_bar))
           : "memory");
     }
-    // ---- row norm with the fixed tree (32 in-order partials of 4 squares, then the
-    // pairwise stages 16, 8, 4, 2, 1), from the staged row while the MMAs run
+    // ---- while the MMAs run: norms (fixed tree: 32 in-order partials of 4 squares,
+    // stages 16 .. 1), two threads per row (lanes 2r' and 2r'+1: dims 0..63 and 64..127,
+    // which hold partials 0..15 and 16..31), and the tokens' precisions
     {
-      float p[32];
+      const int rowi = tid >> 1, part = tid & 1;
+      const int half = rowi >> 6, tok = rowi & 63;
+      const uint8_t* box = xk + half * kDenseBox;
+      float p[16];
 #pragma unroll
-      for (int g = 0; g < 32; ++g) {
-        const uint2 u = *reinterpret_cast<const uint2*>(xa + dense_off(tid, 4 * g));
-        const float x0 = f16_to_f32((uint16_t)(u.x & 0xFFFF)), x1 = f16_to_f32((uint16_t)(u.x >> 16));
-        const float x2 = f16_to_f32((uint16_t)(u.y & 0xFFFF)), x3 = f16_to_f32((uint16_t)(u.y >> 16));
-        float acc = __fmul_rn(x0, x0);
-        acc = __fadd_rn(acc, __fmul_rn(x1, x1));
-        acc = __fadd_rn(acc, __fmul_rn(x2, x2));
-        p[g] = __fadd_rn(acc, __fmul_rn(x3, x3));
+      for (int q = 0; q < 8; ++q) {
+        const uint4 u = *reinterpret_cast<const uint4*>(box + (8 * part + q) * 1024 + tok * 16);
+        const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int g2 = 0; g2 < 2; ++g2) {
+          const float x0 = f16_to_f32((uint16_t)(wv[2 * g2] & 0xFFFF)), x1 = f16_to_f32((uint16_t)(wv[2 * g2] >> 16));
+          const float x2 = f16_to_f32((uint16_t)(wv[2 * g2 + 1] & 0xFFFF)), x3 = f16_to_f32((uint16_t)(wv[2 * g2 + 1] >> 16));
+          float acc = __fmul_rn(x0, x0);
+          acc = __fadd_rn(acc, __fmul_rn(x1, x1));
+          acc = __fadd_rn(acc, __fmul_rn(x2, x2));
+          p[2 * q + g2] = __fadd_rn(acc, __fmul_rn(x3, x3));
+        }
+      }
+      // stage 16 pairs partial g (dims 0..63) with g + 16 (dims 64..127)
+#pragma unroll
+      for (int g = 0; g < 16; ++g) {
+        const float other = __shfl_xor_sync(0xffffffffu, p[g], 1);
+        p[g] = part == 0 ? __fadd_rn(p[g], other) : __fadd_rn(other, p[g]);
       }
 #pragma unroll
-      for (int off = 16; off >= 1; off >>= 1)
+      for (int off = 8; off >= 1; off >>= 1)
 #pragma unroll
         for (int g = 0; g < off; ++g) p[g] = __fadd_rn(p[g], p[g + off]);
-      nrm[tid] = f16_param(__fsqrt_rn(p[0]));
+      if (part == 0) {
+        const uint16_t n16 = f16_param(__fsqrt_rn(p[0]));
+        const float n = f16_to_f32(n16);
+        nrm[2 * tok + half] = n16;
+        invs[2 * tok + half] = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
+      }
+      if (tid < kDenseTok) {
+        const int t = j * kDenseTok + tid;
+        tokhi[tid] = (t < a.n && a.is_high[(int64_t)b * a.n + t] != 0) ? 1 : 0;
+      }
     }
-    ok = false;
-    for (uint32_t i = 0; i < kSpinLimitQ && !ok; ++i) {
-      uint32_t r;
-      asm volatile(
-          "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-          " selp.u32 %0, 1, 0, p;\n}"
-          : "=r"(r)
-          : "r"(dsmem_u32(&bar)), "r"(phase)
-          : "memory");
-      ok = r != 0;
-    }
-    phase ^= 1u;
+    ok = __syncthreads_and(dbar_wait(&mma_bar, par)) != 0;  // also: norms visible
+    if (!ok) break;
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    ok = __syncthreads_and(ok) != 0;  // every norm is taken: the A tile may now hold the codes
-    if (!ok) {
-      if (tid == 0) raise_error(a.err, kDevWaitTimeout);
-      break;
-    }
-    // ---- codes of row tid: u = w * fl(1/n), c = #{k : u > thr_k}
+    if (tid == 0 && j + 1 < j1) issue_tma(j + 1);  // the MMAs have read the tile
+    // ---- codes: warp w, output dims 32 (w % 4) + lane, K (w < 4) or V columns; the
+    // token (and its precision and 1/n) is the same across the warp
     {
-      const int t = t0 + (tid >> 1);
-      const bool hi = t < a.n && a.is_high[(int64_t)b * a.n + t] != 0;
-      const int L = hi ? a.L_hi : a.L_lo;
-      const float* thr_g = hi ? a.thr_hi : a.thr_lo;
-      float thr[7];
+      const int half = warp >> 2, d = 32 * (warp & 3) + lane;
 #pragma unroll
-      for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? thr_g[k] : INFINITY;
-      const float n = f16_to_f32(nrm[tid]);
-      const float inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
-      uint32_t* crow = reinterpret_cast<uint32_t*>(xa + tid * 128);
-#pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {
+      for (int ch = 0; ch < 2; ++ch) {
         uint32_t v[32];
-        tmem_ld32(tb + ((uint32_t)(warp * 32) << 16) + (uint32_t)(ch * 32), v);
-        uint32_t wd[8];
+        tmem_ld32(tb + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(half * 64 + ch * 32), v);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          uint32_t word = 0u;
+        for (int e = 0; e < 32; ++e) {
+          const int tok = ch * 32 + e, row = 2 * tok + half;
+          const float inv = invs[row];
+          const float u = __fmul_rn(__uint_as_float(v[e]), inv);
+          int c = 0;
+          if (tokhi[tok]) {
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float u = __fmul_rn(__uint_as_float(v[4 * q + e]), inv);
-            int c = 0;
+            for (int k = 0; k < 7; ++k) c += u > th_hi[k] ? 1 : 0;
+          } else {
 #pragma unroll
-            for (int k = 0; k < 7; ++k) c += (u > thr[k]) ? 1 : 0;
-            word |= (uint32_t)(n != 0.0f ? c : 0) << (8 * e);
+            for (int k = 0; k < 7; ++k) c += u > th_lo[k] ? 1 : 0;
           }
-          wd[q] = word;
-        }
-#pragma unroll
-        for (int s = 0; s < 8; ++s) {  // staggered by lane: fewer bank conflicts
-          const int q = (s + lane) & 7;
-          uint32_t val = wd[0];
-#pragma unroll
-          for (int j = 1; j < 8; ++j) val = q == j ? wd[j] : val;
-          crow[ch * 8 + q] = val;
+          codes[row * 128 + d] = (uint8_t)(inv != 0.0f ? c : 0);
         }
       }
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();  // codes complete; TMEM free for the next tile
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    // ---- records: warp w packs tokens w, w + 4, ...
-    for (int i = warp; i < kDenseTok; i += 4) {
-      const int t = t0 + i;
+    __syncthreads();  // the code tile is complete; the accumulator may be reused
+    // ---- bit images: thread r < 128 packs row r (the record's quarter fields)
+    if (tid < 128) {
+      const int L = tokhi[tid >> 1] ? a.L_hi : a.L_lo;
+      uint32_t* out = rbits + tid * kRowBitWords;
+      const uint8_t* crow = codes + tid * 128;
+      switch (L) {
+        case 2: row_bits<2>(crow, out); break;
+        case 3: row_bits<3>(crow, out); break;
+        case 4: row_bits<4>(crow, out); break;
+        case 5: row_bits<5>(crow, out); break;
+        case 6: row_bits<6>(crow, out); break;
+        case 7: row_bits<7>(crow, out); break;
+        case 8: row_bits<8>(crow, out); break;
+        default: break;
+      }
+    }
+    __syncthreads();
+    // ---- records: warp w writes tokens w, w + 8, ...; lane j word j
+    for (int i = warp; i < kDenseTok; i += kDenseThreads / 32) {
+      const int t = j * kDenseTok + i;
       if (t >= a.n) break;
-      const bool hi = a.is_high[(int64_t)b * a.n + t] != 0;
+      const bool hi = tokhi[i] != 0;
       const int64_t s = (hi ? a.hi_base : a.lo_base) + a.slot[(int64_t)b * a.n + t];
       const int64_t cap = hi ? a.hi_cap : a.lo_cap;
       if (s >= cap) {  // cannot happen after the host's capacity check
@@ -902,24 +946,27 @@ __global__ void __launch_bounds__(128) quantize_tq_dense_kernel(QuantArgs a) {
         else a.lo_tok[(int64_t)b * a.lo_cap + s] = (int32_t)(a.tok_base + t);
       }
       const int L = hi ? a.L_hi : a.L_lo;
-      const int rec = record_bytes_rt(SEMKV_BASE_TQ_DENSE, L);
-      uint8_t* dst = (hi ? a.hi_pool : a.lo_pool) + ((((int64_t)b * a.NL + l) * a.H + h) * cap + s) * rec;
-      const uint8_t* cp = xa + (2 * i) * 128;
-      const uint16_t nk = nrm[2 * i], nv = nrm[2 * i + 1];
-      switch (L) {
-        case 2: dense_pack<2>(cp, nk, nv, dst, rec_sm[warp], lane); break;
-        case 3: dense_pack<3>(cp, nk, nv, dst, rec_sm[warp], lane); break;
-        case 4: dense_pack<4>(cp, nk, nv, dst, rec_sm[warp], lane); break;
-        case 5: dense_pack<5>(cp, nk, nv, dst, rec_sm[warp], lane); break;
-        case 6: dense_pack<6>(cp, nk, nv, dst, rec_sm[warp], lane); break;
-        case 7: dense_pack<7>(cp, nk, nv, dst, rec_sm[warp], lane); break;
-        case 8: dense_pack<8>(cp, nk, nv, dst, rec_sm[warp], lane); break;
-        default: break;
+      const int RB = row_bytes_rt(L), recw = (2 * RB + 4) / 4;
+      uint32_t* dst = reinterpret_cast<uint32_t*>((hi ? a.hi_pool : a.lo_pool) + ((bhl * cap) + s) * (2 * RB + 4));
+      if (lane < recw) {
+        uint32_t word = 0u;
+        if (4 * lane >= 2 * RB) {
+          word = (uint32_t)nrm[2 * i] | ((uint32_t)nrm[2 * i + 1] << 16);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int byte = 4 * lane + e;
+            const int row = byte < RB ? 2 * i : 2 * i + 1;
+            const int rb = byte < RB ? byte : byte - RB;
+            word |= ((rbits[row * kRowBitWords + (rb >> 2)] >> (8 * (rb & 3))) & 0xFFu) << (8 * e);
+          }
+        }
+        dst[lane] = word;
       }
     }
-    __syncthreads();  // the tiles are free for the next (sequence, layer, head)
+    __syncthreads();  // the code tile, norms and precisions are free for the next tile
   }
-  // release the tensor memory (after every TMEM read of this CTA)
+  if (!ok && tid == 0) raise_error(a.err, kDevWaitTimeout);
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (warp == 0)
@@ -947,7 +994,6 @@ cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t strea
 
 cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
                                  cudaStream_t stream) {
-  (void)num_sms;
   const int64_t total = (int64_t)a.B * a.NL * a.H * a.n;
   if (total == 0) return cudaSuccess;
   if (a.base == SEMKV_BASE_AFFINE) {
@@ -968,16 +1014,42 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
   }
   if (a.base == SEMKV_BASE_TQ_DENSE) {
     static bool attr_set = false;
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     if (!attr_set) {
-      const cudaError_t e = cudaFuncSetAttribute(
-          quantize_tq_dense_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kDenseTile);
+      cudaError_t e = cudaFuncSetAttribute(quantize_tq_dense_kernel,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)kDenseSmem);
       if (e != cudaSuccess) return e;
+      cudaDriverEntryPointQueryResult q;
+      e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&encode),
+                                           12000, cudaEnableDefault, &q);
+      if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !encode)
+        return e != cudaSuccess ? e : cudaErrorNotSupported;
       attr_set = true;
     }
+    // rows of K (V) as a 3-D view: 8 values, every (sequence, layer, head, token) row,
+    // 16 groups of 8 values; a box of 64 rows lands as 8-row x 16-byte core matrices
     const int64_t bhs = (int64_t)a.B * a.NL * a.H;
-    const dim3 grid((unsigned)((a.n + kDenseTok - 1) / kDenseTok),
-                    (unsigned)(bhs < 65535 ? bhs : 65535));
-    quantize_tq_dense_kernel<<<grid, 128, 2 * kDenseTile, stream>>>(a);
+    const cuuint64_t dims[3] = {8, (cuuint64_t)(bhs * a.Tsrc), 16};
+    const cuuint64_t strides[2] = {256, 16};
+    const cuuint32_t box[3] = {8, (cuuint32_t)kDenseTok, 16};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    CUtensorMap tmk, tmv;
+    for (int t = 0; t < 2; ++t) {
+      const CUresult r = encode(t ? &tmv : &tmk, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3,
+                                const_cast<uint16_t*>(t ? a.v : a.k), dims, strides, box, estr,
+                                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    }
+    const int tiles = (a.n + kDenseTok - 1) / kDenseTok;
+    int64_t splits = (2 * (int64_t)num_sms + bhs - 1) / bhs;  // about two CTAs per SM
+    if (splits > tiles) splits = tiles;
+    if (splits < 1) splits = 1;
+    if (bhs > 65535) return cudaErrorInvalidValue;
+    const dim3 grid((unsigned)splits, (unsigned)bhs);
+    quantize_tq_dense_kernel<<<grid, kDenseThreads, kDenseSmem, stream>>>(tmk, tmv, a);
     return cudaGetLastError();
   }
   // TQ and rotated affine: slot -> token maps, then one thread per row by slot

@@ -178,3 +178,47 @@ def test_value_norm_scores_batch16_64k_sampled_sequences():
     for b, vb in host.items():
         want = oracle.score_kv_norm(synthetic.f16_bits(vb))[0]
         assert np.array_equal(got[b].view(np.uint32), want.view(np.uint32)), b
+
+
+def test_fake_quant_batch16_64k_sampled_sequences():
+    # the batch-16 x 64K prompt's K and V, reconstructed at the 6/5 split of the
+    # rank; sequences 3 and 14 compared with the oracle bit for bit
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    B, T, H = 16, 65536, 8
+    dev = torch.device("cuda:0")
+    n_high = oracle.high_count_floor(T, 26, 100)
+    desc = semkv.QuantDesc(semkv.BASE_AFFINE, 6, 5, device=dev)
+    k = torch.empty((B, 1, H, T, 128), dtype=torch.float16, device=dev)
+    v = torch.empty_like(k)
+    s = np.stack([synthetic.scores_zipf(600 + b, 1, T)[0] for b in range(B)])
+    host = {}
+    for b in range(B):
+        kb, vb = synthetic.kv(600 + b, 1, 1, H, T)
+        k[b].copy_(torch.from_numpy(kb[0]))
+        v[b].copy_(torch.from_numpy(vb[0]))
+        if b in (3, 14):
+            host[b] = (kb, vb)
+    is_high = torch.empty((B, T), dtype=torch.uint8, device=dev)
+    slot = torch.empty((B, T), dtype=torch.int32, device=dev)
+    semkv.semkv_rank_assign(torch.from_numpy(s).to(dev), n_high, is_high, slot)
+    ko, vo = torch.empty_like(k), torch.empty_like(v)
+    semkv.semkv_fake_quant(desc, k, v, ko, vo, is_high=is_high)
+    torch.cuda.synchronize()
+    ih = is_high.cpu().numpy()
+    for b, (kb, vb) in host.items():
+        o_k, o_v = oracle.fake_quant(0, 6, 5, synthetic.f16_bits(kb), synthetic.f16_bits(vb),
+                                     is_high=ih[b:b + 1])
+        assert np.array_equal(ko[b:b + 1].cpu().numpy().view(np.uint16), o_k), b
+        assert np.array_equal(vo[b:b + 1].cpu().numpy().view(np.uint16), o_v), b
+
+
+def test_dense_tq_43_32k_every_record_up_to_ties_and_heads():
+    # the TQ 4/3 workload on the dense random rotation (tcgen05 quantize)
+    p = Pair(3, 4, 3, 1, 1, 8, 32, 32768, 3, 4, seed=5)
+    p.quantize()
+    p.assert_records_equal_up_to_ties()
+    p.adopt_gpu_records()
+    got, ref = p.decode(0, 0)
+    err, rel = attention_errors(got, ref)
+    assert err <= ATOL and rel <= RTOL_L2, (err, rel)
