@@ -261,11 +261,13 @@ def pre_decode_work(k, cache, blk, token_mode, base_counts, r_num, r_den, desc,
     """The host and device work of step k that precedes its decode calls: staging and,
     when due, the block append (with the appended slots rewound first)."""
     if not token_mode:
+        # the block's K/V and scores already sit in device buffers laid out as the
+        # stage (the caller's): point the cache's stage at them
         j = k % nblocks
         cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
-        cache.stage_k.copy_(blocks_k[:, :, :, j * blk:(j + 1) * blk])
-        cache.stage_v.copy_(blocks_v[:, :, :, j * blk:(j + 1) * blk])
-        cache.stage_score.copy_(blocks_s[:, j * blk:(j + 1) * blk])
+        cache.s.stage_k = blocks_k[j].data_ptr()
+        cache.s.stage_v = blocks_v[j].data_ptr()
+        cache.s.stage_score = blocks_s[j].data_ptr()
         cache.s.stage_n = blk
         semkv.semkv_append_block(desc, cache, r_num, r_den)
     else:
@@ -348,9 +350,17 @@ def gpu_arm(args, cfg, rank, world):
     nblocks = 4
     gk, gv = synthetic.kv(cfg["seed"] * 100 + 99, B, NL, H, blk * nblocks)
     gs = synthetic.scores_zipf(cfg["seed"] * 100 + 99, B, blk * nblocks)
-    blocks_k = torch.from_numpy(gk).to(dev)
-    blocks_v = torch.from_numpy(gv).to(dev)
-    blocks_s = torch.from_numpy(gs).to(dev)
+    if token_mode:
+        blocks_k = torch.from_numpy(gk).to(dev)
+        blocks_v = torch.from_numpy(gv).to(dev)
+        blocks_s = torch.from_numpy(gs).to(dev)
+    else:  # per block, contiguous in the stage layout [B][NL][H][blk][128]
+        blocks_k = [torch.from_numpy(np.ascontiguousarray(gk[:, :, :, j * blk:(j + 1) * blk])).to(dev)
+                    for j in range(nblocks)]
+        blocks_v = [torch.from_numpy(np.ascontiguousarray(gv[:, :, :, j * blk:(j + 1) * blk])).to(dev)
+                    for j in range(nblocks)]
+        blocks_s = [torch.from_numpy(np.ascontiguousarray(gs[:, j * blk:(j + 1) * blk])).to(dev)
+                    for j in range(nblocks)]
     q_all = torch.from_numpy(np.stack([synthetic.queries(cfg["seed"], B, Hq, step=i)
                                        for i in range(nblocks)])).to(dev)
     out = torch.empty((B, Hq, 128), dtype=torch.float32, device=dev)
@@ -468,6 +478,9 @@ def gpu_arm(args, cfg, rank, world):
             elapsed = sum(a.elapsed_time(b) for a, b in sev) * 1e-3
     dec_times = [a.elapsed_time(b) * 1e-3 for a, b in evs]
     err = int(cache.dev_error.item())
+    # the cache's own stage buffers again (the steps above pointed it at the blocks)
+    cache.s.stage_k, cache.s.stage_v = cache.stage_k.data_ptr(), cache.stage_v.data_ptr()
+    cache.s.stage_score = cache.stage_score.data_ptr()
 
     # ---- end to end through the public API with host buffers
     # contiguous pinned host buffers per block (per token in the block-wise workload),
@@ -520,20 +533,83 @@ def gpu_arm(args, cfg, rank, world):
             semkv.semkv_decode_attention(desc, cache, layer, qdev, out, scale, ws)
         pin_out.copy_(out, non_blocking=True)
 
+    # Block mode overlaps the copies with the compute, as a serving loop would: a copy
+    # stream uploads step i+1's block and queries into the other of two staging
+    # buffers (the cache's stage pointers are the caller's) while step i runs, and
+    # reads step i's output back after it; every copy stays inside the timed region.
+    copy_s = torch.cuda.Stream()
+    nbuf = 2
+    bufs = [dict(k=torch.empty_like(cache.stage_k), v=torch.empty_like(cache.stage_v),
+                 s=torch.empty_like(cache.stage_score), q=torch.empty_like(qdev),
+                 o=torch.empty_like(out)) for _ in range(nbuf)]
+    pin_outs = [torch.empty_like(pin_out).pin_memory() for _ in range(nbuf)]
+    up_ev = [torch.cuda.Event() for _ in range(nbuf)]
+    done_ev = [torch.cuda.Event() for _ in range(nbuf)]
+
+    def upload(i):
+        j, bb = i % nblocks, bufs[i % nbuf]
+        with torch.cuda.stream(copy_s):
+            if i >= nbuf:
+                copy_s.wait_event(done_ev[i % nbuf])  # step i - 2 is done with this buffer
+            bb["k"].copy_(pin_k[j], non_blocking=True)
+            bb["v"].copy_(pin_v[j], non_blocking=True)
+            bb["s"].copy_(pin_s[j], non_blocking=True)
+            bb["q"].copy_(pin_q[j], non_blocking=True)
+            up_ev[i % nbuf].record(copy_s)
+
+    def compute(i):
+        bb = bufs[i % nbuf]
+        stream.wait_event(up_ev[i % nbuf])
+        cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens = base_counts
+        cache.s.stage_k, cache.s.stage_v = bb["k"].data_ptr(), bb["v"].data_ptr()
+        cache.s.stage_score = bb["s"].data_ptr()
+        cache.s.stage_n = blk
+        semkv.semkv_append_block(desc, cache, r_num, r_den)
+        for layer in range(NL):
+            semkv.semkv_decode_attention(desc, cache, layer, bb["q"], bb["o"], scale, ws)
+        done_ev[i % nbuf].record(stream)
+        with torch.cuda.stream(copy_s):
+            copy_s.wait_event(done_ev[i % nbuf])
+            pin_outs[i % nbuf].copy_(bb["o"], non_blocking=True)
+
+    def run_pipelined(n):
+        upload(0)
+        for i in range(n):
+            if i + 1 < n:
+                upload(i + 1)
+            compute(i)
+
     e2e_steps = max(3, min(args.steps, 200))
     if token_mode:
         e2e_steps = max(blk, (e2e_steps // blk) * blk)
         cache.s.stage_n = 0
-    for i in range(3 if not token_mode else blk):
-        step_e2e(i)
+        for i in range(blk):
+            step_e2e(i)
+    else:
+        run_pipelined(3)
+        torch.cuda.synchronize()
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for i in range(e2e_steps):
-        step_e2e(i)
+    if token_mode:
+        for i in range(e2e_steps):
+            step_e2e(i)
+    else:
+        run_pipelined(e2e_steps)
+        stream.wait_stream(copy_s)  # the last read-back is inside the timed region
     e1.record(stream)
     barrier()
     e2e_time = e0.elapsed_time(e1) * 1e-3 / e2e_steps
+    if not token_mode:
+        # the pipelined loop computes what the serial one does: recheck its last step
+        torch.cuda.synchronize()
+        cache.s.stage_k, cache.s.stage_v = cache.stage_k.data_ptr(), cache.stage_v.data_ptr()
+        cache.s.stage_score = cache.stage_score.data_ptr()
+        got = pin_outs[(e2e_steps - 1) % nbuf].clone()
+        step_e2e(e2e_steps - 1)
+        torch.cuda.synchronize()
+        if not torch.equal(got, pin_out):
+            raise RuntimeError("pipelined end-to-end step differs from the serial step")
 
     elapsed, e2e_time = max_over_ranks([elapsed, e2e_time], device=dev)
     return dict(elapsed=elapsed, dec_times=dec_times, dec_bytes=dec_bytes, app_bytes=app_bytes,
