@@ -1461,6 +1461,72 @@ __global__ void combine_kernel(DecodeArgs a) {
   *reinterpret_cast<float4*>(a.out + ((int64_t)b * a.Hq + qh) * 128 + 4 * lane) = r;
 }
 
+// Merge the partials of one (b, qh) with a CTA of 8 warps: every thread takes partials
+// for the maximum and the weights, then warp w sums the rows of partials w, w + 8, ...
+// (lane = 4 dims) and the 8 row sums are added in warp order.  For the small batches,
+// whose (b, h) pairs are spread over dozens of CTAs, this keeps the combine short.
+__global__ void __launch_bounds__(256) combine_wide_kernel(DecodeArgs a) {
+  __shared__ float wsm[kMaxPartialsPerPair];
+  __shared__ float red[8][128];
+  __shared__ float red_m[8], red_l[8];
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  const int gw = blockIdx.x;
+  const int b = gw / a.Hq, qh = gw % a.Hq;
+  const int G = a.Hq / a.H, h = qh / G, c = qh % G;
+  const int64_t bh = (int64_t)b * a.H + h;
+  const int S = pair_partials(a.plan, bh);
+  const float* base = a.partials + bh * a.plan.stride * kPartialFloats;
+  float M = -INFINITY;
+  for (int s = tid; s < S; s += 256) M = fmaxf(M, base[s * kPartialFloats + c]);
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+  if (lane == 0) red_m[w] = M;
+  __syncthreads();
+  M = red_m[0];
+#pragma unroll
+  for (int i = 1; i < 8; ++i) M = fmaxf(M, red_m[i]);
+  float lsum = 0.0f;
+  for (int s = tid; s < S; s += 256) {
+    const float ms = base[s * kPartialFloats + c];
+    const float sc = (M == -INFINITY || ms == -INFINITY) ? 0.0f : exp2f(ms - M);
+    wsm[s] = sc;
+    lsum += sc * base[s * kPartialFloats + 8 + c];
+  }
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
+  if (lane == 0) red_l[w] = lsum;
+  __syncthreads();
+  float o[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int s = w; s < S; s += 8) {
+    const float sc = wsm[s];
+    if (sc == 0.0f) continue;
+    const float4 v = *reinterpret_cast<const float4*>(base + s * kPartialFloats + 16 + c * 128 + 4 * lane);
+    o[0] += sc * v.x;
+    o[1] += sc * v.y;
+    o[2] += sc * v.z;
+    o[3] += sc * v.w;
+  }
+#pragma unroll
+  for (int e = 0; e < 4; ++e) red[w][4 * lane + e] = o[e];
+  __syncthreads();
+  if (w == 0) {
+    float l = red_l[0];
+#pragma unroll
+    for (int i = 1; i < 8; ++i) l += red_l[i];
+    const float inv = 1.0f / l;
+    float r[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      float x = red[0][4 * lane + e];
+#pragma unroll
+      for (int i = 1; i < 8; ++i) x += red[i][4 * lane + e];
+      r[e] = x * inv;
+    }
+    *reinterpret_cast<float4*>(a.out + ((int64_t)b * a.Hq + qh) * 128 + 4 * lane) =
+        make_float4(r[0], r[1], r[2], r[3]);
+  }
+}
+
 }  // namespace
 
 // relative cost of a 16-token tile per level count (decode instructions per tile)
@@ -1639,7 +1705,7 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
   if (a.base == SEMKV_BASE_TQ_DENSE)
     combine_kernel<true><<<a.B * a.H, 32 * (a.Hq / a.H), 0, stream>>>(a);
   else
-    combine_kernel<false><<<(heads + 7) / 8, 256, 0, stream>>>(a);
+    combine_wide_kernel<<<heads, 256, 0, stream>>>(a);
   return cudaGetLastError();
 }
 
