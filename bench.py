@@ -753,7 +753,10 @@ def main():
         "fake_quant_gbs": r["fake_gbs"],
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": profiled_traffic(args.config),
-                     "kernel": "decode_kernel+combine_kernel (semkv_decode_attention)",
+                     "kernel": {0: "decode_affine_kernel + combine_wide_kernel", 2: "decode_affine_kernel + combine_wide_kernel",
+                                1: "decode_kernel<1> + combine_wide_kernel",
+                                3: "decode_kernel<1> + combine_kernel<dense>"}[cfg["base"]]
+                               + " (semkv_decode_attention)",
                      "peak_kind": f"{peak_kind} hbm_gbs"},
         "e2e": {"value": job_gbs(step_bytes, world, r["e2e_time"]), "unit": "GB/s",
                 "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
