@@ -250,7 +250,9 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
  *    any stream capture.
  *  - Limit: batch * kv_heads * (one partial per non-empty pool, plus one when tokens
  *    are staged) must fit in 2016 partials; larger requests return SEMKV_EWORKSPACE.
- *    Within the limit the split count is reduced to fit.
+ *    Within the limit the split count is reduced to fit.  The rotated bases (TQ,
+ *    AFFINE_HAD, TQ_DENSE) also keep their rotated queries in a second static array
+ *    of 4096 query heads (batch * q_heads beyond it: SEMKV_EWORKSPACE).
  *  - All calls share the array, which keeps the last call's contents (each call
  *    overwrites every partial it reads, so nothing needs clearing).  Calls whose
  *    kernels overlap on the GPU (e.g. on two streams, or two host threads) race on

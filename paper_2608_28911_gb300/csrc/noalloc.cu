@@ -16,24 +16,32 @@
 // Every GPU that loads the library holds this array until the process exits.
 static constexpr size_t kScratchFloats = (size_t)2016 * semkv::kPartialFloats;
 static __device__ __align__(256) float g_decode_scratch[kScratchFloats];
+// 2 MiB of rotated queries (the rotated bases): 4096 query heads of 128 floats
+static constexpr size_t kQrotFloats = (size_t)4096 * 128;
+static __device__ __align__(256) float g_qrot_scratch[kQrotFloats];
 
 namespace {
 
 constexpr int kMaxDevices = 64;
 float* g_scratch_addr[kMaxDevices] = {nullptr};
+float* g_qrot_addr[kMaxDevices] = {nullptr};
 
-// The device address of the array on the current device.  In host code the name
-// g_decode_scratch is only a host-side stand-in, so the address is looked up once per
-// device (with that device current) and cached.
-semkv_status scratch_address(float** out) {
+// The device addresses of the arrays on the current device.  In host code their names
+// are only host-side stand-ins, so the addresses are looked up once per device (with
+// that device current) and cached.
+semkv_status scratch_address(float** out, float** qrot) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return SEMKV_ECUDA;
   if (!g_scratch_addr[dev]) {
     void* p = nullptr;
+    void* r = nullptr;
     if (cudaGetSymbolAddress(&p, g_decode_scratch) != cudaSuccess || !p) return SEMKV_ECUDA;
+    if (cudaGetSymbolAddress(&r, g_qrot_scratch) != cudaSuccess || !r) return SEMKV_ECUDA;
     g_scratch_addr[dev] = static_cast<float*>(p);
+    g_qrot_addr[dev] = static_cast<float*>(r);
   }
   *out = g_scratch_addr[dev];
+  *qrot = g_qrot_addr[dev];
   return SEMKV_OK;
 }
 
@@ -49,10 +57,21 @@ extern "C" semkv_status semkv_decode_attention_noalloc(const semkv_quant_desc* d
   if (!desc || !cache) return SEMKV_EINVAL;
   if (desc->head_dim != SEMKV_HEAD_DIM || cache->head_dim != SEMKV_HEAD_DIM)
     return SEMKV_EUNSUPPORTED;
-  if (desc->base != SEMKV_BASE_AFFINE) return SEMKV_EUNSUPPORTED;
+  if (desc->base < SEMKV_BASE_AFFINE || desc->base > SEMKV_BASE_TQ_DENSE) return SEMKV_EUNSUPPORTED;
   if (desc->levels_hi < 2 || desc->levels_hi > SEMKV_MAX_LEVELS || desc->levels_lo < 2 ||
       desc->levels_lo > SEMKV_MAX_LEVELS)
     return SEMKV_EUNSUPPORTED;
+  if (desc->base == SEMKV_BASE_TQ || desc->base == SEMKV_BASE_AFFINE_HAD) {
+    if (!desc->signs) return SEMKV_EINVAL;
+    if (!aligned(desc->signs, 4)) return SEMKV_EALIGN;
+  }
+  if (desc->base == SEMKV_BASE_TQ_DENSE) {
+    if (!desc->rotation) return SEMKV_EINVAL;
+    if (!aligned(desc->rotation, 16)) return SEMKV_EALIGN;
+  }
+  if ((desc->base == SEMKV_BASE_TQ || desc->base == SEMKV_BASE_TQ_DENSE) &&
+      (!desc->centroids_hi || !desc->centroids_lo || !desc->thresholds_hi || !desc->thresholds_lo))
+    return SEMKV_EINVAL;
   const semkv_cache* c = cache;
   if (c->batch < 1 || c->layers < 1 || c->kv_heads < 1 || c->q_heads < 1) return SEMKV_EINVAL;
   if (c->q_heads % c->kv_heads != 0) return SEMKV_EINVAL;
@@ -82,8 +101,12 @@ extern "C" semkv_status semkv_decode_attention_noalloc(const semkv_quant_desc* d
                                            sms, cap);
   if (cap < 1 || plan.stride > cap) return SEMKV_EWORKSPACE;  // exceeds the static scratch
 
+  const bool rotated = desc->base != SEMKV_BASE_AFFINE;
+  if (rotated && (size_t)c->batch * c->q_heads * 128 > kQrotFloats) return SEMKV_EWORKSPACE;
+
   float* scratch = nullptr;
-  semkv_status s = scratch_address(&scratch);
+  float* qrot = nullptr;
+  semkv_status s = scratch_address(&scratch, &qrot);
   if (s != SEMKV_OK) return s;
 
   DecodeArgs a;
@@ -111,9 +134,10 @@ extern "C" semkv_status semkv_decode_attention_noalloc(const semkv_quant_desc* d
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
   a.partials = scratch;  // fully overwritten by each call: nothing needs clearing
   a.signs = desc->signs;
+  a.rot = desc->rotation;
   a.cb_hi = desc->centroids_hi;
   a.cb_lo = desc->centroids_lo;
-  a.qrot = nullptr;
+  a.qrot = rotated ? qrot : nullptr;
   a.err = c->dev_error;
   a.plan = plan;
   return launch_decode_attention(a, (cudaStream_t)stream) == cudaSuccess ? SEMKV_OK : SEMKV_ECUDA;

@@ -49,6 +49,20 @@ def test_noalloc_matches_workspace_entry_point(B, H, Hq, T):
     assert int(p.cache.dev_error.item()) == 0
 
 
+@pytest.mark.parametrize("base,L_hi,L_lo", [(1, 4, 3), (2, 6, 5), (3, 4, 3)])
+def test_noalloc_rotated_bases(base, L_hi, L_lo):
+    # TQ, Hadamard-rotated affine and dense-rotation TQ: the rotated queries live in
+    # the library's second static array
+    p = Pair(base, L_hi, L_lo, 2, 1, 8, 32, 2000, 3, 4, seed=320 + base)
+    p.quantize()
+    for qseed in (0, 1):
+        ref, outs = _run_both(p, qseed)
+        for got in outs:
+            err, rel = attention_errors(got, ref)
+            assert err <= ATOL and rel <= RTOL_L2, (err, rel)
+    assert int(p.cache.dev_error.item()) == 0
+
+
 def test_noalloc_rejects_requests_beyond_the_array():
     import torch
     from paper_2608_28911_gb300 import semkv
