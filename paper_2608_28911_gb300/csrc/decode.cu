@@ -14,9 +14,10 @@
 // beta = ceil(t 2^W / L^G), so F_k = floor(beta L^(k+1) / 2^W) is the number formed by
 // the first k+1 digits and c_k = F_k - L F_{k-1}.  Read as an fp32 bit pattern, beta
 // is the denormal beta * 2^-149; one multiply rounded toward zero by the exact
-// constant L^(k+1)/2^W yields a float whose bit pattern is F_k.  For five-level
-// groups two symbols share one multiply (beta_a + 65536 beta_b is still a denormal)
-// and a mask separates the halves.  Integers (all < 256) become fp16 values with a
+// constant L^(k+1)/2^W yields a float whose bit pattern is F_k; the packed binary32
+// forms (mul/fma.rz.f32x2) take two symbols, or two constants, per instruction.  For
+// five-level groups two symbols also share one lane of a multiply (beta_a + 65536 beta_b
+// is still a denormal) and a mask separates the halves.  Integers (all < 256) become fp16 values with a
 // byte placed over them (1024 + v) and one f16x2 subtract.
 //  - QK^T as S = Q' F^T on mma.sync m16n8k16 (M = heads, N = 8 tokens, K = 128 F
 //    slots): the q coefficient of F_k is q'_k = q_{d_k} - L q_{d_{k+1}} when F_k
@@ -133,6 +134,30 @@ __device__ __forceinline__ uint32_t fdig(uint32_t beta, float c) {
 __device__ __forceinline__ uint32_t fdig1024(uint32_t beta, float c) {
   return __float_as_uint(__fmaf_rz(__uint_as_float(beta), c, __uint_as_float(0x6400u)));
 }
+// fdig and fdig1024 of two symbols (or one symbol and two constants) in one packed
+// binary32 instruction: lane 0 takes (a, ca), lane 1 (b, cb)
+__device__ __forceinline__ unsigned long long u2_pack(uint32_t lo, uint32_t hi) {
+  return (unsigned long long)lo | ((unsigned long long)hi << 32);
+}
+__device__ __forceinline__ void fdig_x2(uint32_t a, uint32_t b, float ca, float cb,
+                                        uint32_t& ra, uint32_t& rb) {
+  unsigned long long y;
+  asm("mul.rz.f32x2 %0, %1, %2;"
+      : "=l"(y)
+      : "l"(u2_pack(a, b)), "l"(u2_pack(__float_as_uint(ca), __float_as_uint(cb))));
+  ra = (uint32_t)y;
+  rb = (uint32_t)(y >> 32);
+}
+__device__ __forceinline__ void fdig1024_x2(uint32_t a, uint32_t b, float ca, float cb,
+                                            uint32_t& ra, uint32_t& rb) {
+  unsigned long long y;
+  asm("fma.rz.f32x2 %0, %1, %2, %3;"
+      : "=l"(y)
+      : "l"(u2_pack(a, b)), "l"(u2_pack(__float_as_uint(ca), __float_as_uint(cb))),
+        "l"(0x0000640000006400ull));
+  ra = (uint32_t)y;
+  rb = (uint32_t)(y >> 32);
+}
 // the low halves of a and b side by side
 __device__ __forceinline__ uint32_t fpair(uint32_t a, uint32_t b) {
   return __byte_perm(a, b, 0x5410);
@@ -247,11 +272,44 @@ struct Dec {
       }
     }
   }
+  // sym of two symbols at once, in packed instructions
+  __device__ __forceinline__ static void sym2(uint32_t ba, uint32_t bb, uint32_t* fa,
+                                              uint32_t* fb) {
+    if constexpr (G == 1) {
+      if constexpr (L == 7) {
+        fdig1024_x2(ba, bb, 7.0f / 8.0f, 7.0f / 8.0f, fa[0], fb[0]);
+      } else {
+        fa[0] = ba | 0x6400u;
+        fb[0] = bb | 0x6400u;
+      }
+    } else if constexpr (L == 6) {
+      constexpr float c1 = 6.0f / 8192.0f, c2 = 36.0f / 8192.0f, c3 = 216.0f / 8192.0f;
+      fdig1024_x2(ba, bb, c1, c1, fa[0], fb[0]);
+      fdig1024_x2(ba, bb, c2, c2, fa[1], fb[1]);
+      const uint32_t xa = (ba * 36u) & 8191u, xb = (bb * 36u) & 8191u;
+      fdig1024_x2(xa, xb, c1, c1, fa[2], fb[2]);
+      fdig1024_x2(xa, xb, c2, c2, fa[3], fb[3]);
+      fdig1024_x2(xa, xb, c3, c3, fa[4], fb[4]);
+    } else {
+      float c = (float)L / (float)(1u << F::W);
+#pragma unroll
+      for (int k = 0; k < G; ++k) {
+        fdig1024_x2(ba, bb, c, c, fa[k], fb[k]);
+        c *= (float)L;
+      }
+    }
+  }
   // 1024 + F values of the two-code tail symbol
   __device__ __forceinline__ static void tail(uint32_t beta, uint32_t* f) {
     constexpr float c = (float)L / (float)(1u << F::WT);
-    f[0] = fdig1024(beta, c);
-    f[1] = fdig1024(beta, c * (float)L);
+    fdig1024_x2(beta, beta, c, c * (float)L, f[0], f[1]);
+  }
+  // the tails of two symbols: fa, fb as in tail
+  __device__ __forceinline__ static void tail2(uint32_t ba, uint32_t bb, uint32_t* fa,
+                                               uint32_t* fb) {
+    constexpr float c = (float)L / (float)(1u << F::WT);
+    fdig1024_x2(ba, bb, c, c, fa[0], fb[0]);
+    fdig1024_x2(ba, bb, c * (float)L, c * (float)L, fa[1], fb[1]);
   }
   // does F slot k of a group carry a share of digit k+1?
   __host__ __device__ static constexpr bool chained(int k) { return k + 1 < G && k + 1 != kRestart; }
@@ -263,9 +321,24 @@ struct Dec {
 // one multiply gives both halves' F_k (bytes 0 and 2; the fraction lands in byte 1).
 constexpr uint32_t kM7 = 0x007F007Fu;
 __device__ __forceinline__ void l5_fpairs(uint32_t u, uint32_t* X) {
-  X[0] = bytes_to_h2(fdig(u, 5.0f / 128.0f));
-  X[1] = bytes_to_h2(fdig(u, 25.0f / 128.0f));
+  uint32_t P0, P1;
+  fdig_x2(u, u, 5.0f / 128.0f, 25.0f / 128.0f, P0, P1);
+  X[0] = bytes_to_h2(P0);
+  X[1] = bytes_to_h2(P1);
   X[2] = bytes_to_h2(fdig(u, 125.0f / 128.0f));
+}
+// l5_fpairs of two registers at once
+__device__ __forceinline__ void l5_fpairs2(uint32_t u, uint32_t v, uint32_t* X, uint32_t* Y) {
+  uint32_t P, Q;
+  fdig_x2(u, v, 5.0f / 128.0f, 5.0f / 128.0f, P, Q);
+  X[0] = bytes_to_h2(P);
+  Y[0] = bytes_to_h2(Q);
+  fdig_x2(u, v, 25.0f / 128.0f, 25.0f / 128.0f, P, Q);
+  X[1] = bytes_to_h2(P);
+  Y[1] = bytes_to_h2(Q);
+  fdig_x2(u, v, 125.0f / 128.0f, 125.0f / 128.0f, P, Q);
+  X[2] = bytes_to_h2(P);
+  Y[2] = bytes_to_h2(Q);
 }
 // symbol pairs from two windows: symbol j of window a in the low half and of window b
 // in the high half, j = 0..4 (bits 7j)
@@ -283,8 +356,10 @@ __device__ __forceinline__ void l5_pairs(uint32_t a0, uint32_t a1, uint32_t b0, 
 // the two-code five-level tail of two windows at once (5-bit symbols, u < 2^21):
 // F_0 and F_1 pairs (bytes 0 and 2); the fraction of the high symbol lands in bits 11..15
 __device__ __forceinline__ void l5_tail_pairs(uint32_t ut, uint32_t& X0, uint32_t& X1) {
-  X0 = bytes_to_h2(fdig(ut, 5.0f / 32.0f));
-  X1 = bytes_to_h2(fdig(ut, 25.0f / 32.0f));
+  uint32_t P0, P1;
+  fdig_x2(ut, ut, 5.0f / 32.0f, 25.0f / 32.0f, P0, P1);
+  X0 = bytes_to_h2(P0);
+  X1 = bytes_to_h2(P1);
 }
 
 // F side of S = Q' F^T: the fp16 F-value pairs of one quarter row of one token (both
@@ -300,8 +375,9 @@ __device__ __forceinline__ void k_quarter(const Window& w, uint32_t (&f)[8][2]) 
     uint32_t u[5];
     // symbol s + 5 sits 35 bits after symbol s
     l5_pairs(w.q0, w.q1, __funnelshift_r(w.q1, w.q2, 3), w.q2 >> 3, u);
-#pragma unroll
-    for (int s = 0; s < 5; ++s) l5_fpairs(u[s], h + 3 * s);
+    l5_fpairs2(u[0], u[1], h, h + 3);
+    l5_fpairs2(u[2], u[3], h + 6, h + 9);
+    l5_fpairs(u[4], h + 12);
     uint32_t ft[2];
     D::tail(wbits(w, 70, 5), ft);
     h[15] = hsub1024(fpair(ft[0], ft[1]));
@@ -309,8 +385,7 @@ __device__ __forceinline__ void k_quarter(const Window& w, uint32_t (&f)[8][2]) 
 #pragma unroll
     for (int s = 0; s < D::kHalf; ++s) {
       uint32_t fa[D::G], fb[D::G];
-      D::sym(wbits(w, s * F::W, F::W), fa);
-      D::sym(wbits(w, (s + D::kHalf) * F::W, F::W), fb);
+      D::sym2(wbits(w, s * F::W, F::W), wbits(w, (s + D::kHalf) * F::W, F::W), fa, fb);
 #pragma unroll
       for (int k = 0; k < D::G; ++k) h[s * D::G + k] = hsub1024(fpair(fa[k], fb[k]));
     }
@@ -366,13 +441,15 @@ __device__ __forceinline__ void v_half_pair(const Window& wa, const Window& wb, 
   if constexpr (L == 5) {
     uint32_t u[5];
     l5_pairs(wa.q0, wa.q1, wb.q0, wb.q1, u);
+    uint32_t X[5][3];
+    l5_fpairs2(u[0], u[1], X[0], X[1]);
+    l5_fpairs2(u[2], u[3], X[2], X[3]);
+    l5_fpairs(u[4], X[4]);
 #pragma unroll
     for (int j = 0; j < 5; ++j) {
-      uint32_t X[3];
-      l5_fpairs(u[j], X);
-      h[3 * j] = X[0];
-      h[3 * j + 1] = hdigit<5>(X[0], X[1]);
-      h[3 * j + 2] = hdigit<5>(X[1], X[2]);
+      h[3 * j] = X[j][0];
+      h[3 * j + 1] = hdigit<5>(X[j][0], X[j][1]);
+      h[3 * j + 2] = hdigit<5>(X[j][1], X[j][2]);
     }
     uint32_t X0, X1;
     l5_tail_pairs(fpair(wbits_rt(wa, tpos, 5), wbits_rt(wb, tpos, 5)), X0, X1);
@@ -381,8 +458,7 @@ __device__ __forceinline__ void v_half_pair(const Window& wa, const Window& wb, 
 #pragma unroll
     for (int j = 0; j < D::kHalf; ++j) {
       uint32_t fa[D::G], fb[D::G], X[D::G];
-      D::sym(wbits(wa, j * F::W, F::W), fa);
-      D::sym(wbits(wb, j * F::W, F::W), fb);
+      D::sym2(wbits(wa, j * F::W, F::W), wbits(wb, j * F::W, F::W), fa, fb);
 #pragma unroll
       for (int k = 0; k < D::G; ++k) X[k] = hsub1024(fpair(fa[k], fb[k]));
 #pragma unroll
@@ -391,8 +467,7 @@ __device__ __forceinline__ void v_half_pair(const Window& wa, const Window& wb, 
     }
     if constexpr (F::R > 0) {
       uint32_t fa[2], fb[2];
-      D::tail(wbits_rt(wa, tpos, F::WT), fa);
-      D::tail(wbits_rt(wb, tpos, F::WT), fb);
+      D::tail2(wbits_rt(wa, tpos, F::WT), wbits_rt(wb, tpos, F::WT), fa, fb);
       const uint32_t X0 = hsub1024(fpair(fa[0], fb[0]));
       const uint32_t X1 = hsub1024(fpair(fa[1], fb[1]));
       h[15] = hh ? hdigit<L>(X0, X1) : X0;
