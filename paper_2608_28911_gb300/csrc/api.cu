@@ -301,6 +301,19 @@ semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache
   r.slot = cache->blk_slot;
   r.rank = nullptr;
   r.ws = nullptr;
+  // a block of at most 1024 tokens is ranked by one single-pass kernel, which then
+  // writes the slot -> token maps too (no separate scatter launch)
+  const bool maps_in_rank = n <= 1024 && desc->base != SEMKV_BASE_TQ_DENSE;
+  if (maps_in_rank) {
+    r.hi_tok = cache->hi_tok;
+    r.lo_tok = cache->lo_tok;
+    r.hi_base = cache->hi_count;
+    r.lo_base = cache->lo_count;
+    r.hi_cap = cache->hi_cap;
+    r.lo_cap = cache->lo_cap;
+    r.tok_base = cache->n_tokens;
+    r.err = cache->dev_error;
+  }
   s = from_cuda(launch_rank_assign(r, (cudaStream_t)stream));
   if (s != SEMKV_OK) return s;
   QuantArgs a;
@@ -330,7 +343,8 @@ semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache
   a.hi_tok = cache->hi_tok;
   a.lo_tok = cache->lo_tok;
   a.err = cache->dev_error;
-  s = from_cuda(launch_quantize_pack(a, n_high, device_sm_count(), (cudaStream_t)stream));
+  s = from_cuda(launch_quantize_pack(a, n_high, device_sm_count(), (cudaStream_t)stream,
+                                     maps_in_rank));
   if (s != SEMKV_OK) return s;
   cache->hi_count += n_high;
   cache->lo_count += n - (int64_t)n_high;

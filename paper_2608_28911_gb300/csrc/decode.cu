@@ -542,7 +542,8 @@ struct Shared {
 template <int L, bool PACKED, int CODEC = 0>
 __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint4* aq_all,
                          uint64_t* bars, const uint8_t* pool_bh, int64_t count, int t_begin,
-                         int t_end, int G, WarpState& st, int& ring_it, int which = 0) {
+                         int t_end, int G, WarpState& st, int& ring_it, int which = 0,
+                         bool prefilled = false) {
   using D = Dec<L>;
   using F = typename D::F;
   static_assert(CODEC != 2 || L == 4, "the cubic decomposition is for four levels");
@@ -603,7 +604,7 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
 
   const int nmine = t_end - t_begin <= warp ? 0 : (t_end - t_begin - warp + kWarps - 1) / kWarps;
   const int count32 = (int)count;  // a pool holds fewer than 2^31 slots
-  if (lane == 0) {
+  if (lane == 0 && !prefilled) {
     // the ring may have been the merge area: order those writes before the copies
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     for (int i = 0; i < kStages && i < nmine; ++i) {
@@ -1242,14 +1243,36 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
   __syncthreads();  // the merge area (the ring) is free again
 }
 
+// The first copies of a segment, as run_pool would start them: issued before the
+// queries are loaded and the coefficient fragments built, so those overlap the copies.
+// The ring must be free (no merge in progress).
+__device__ void ring_fill(uint8_t* ring, uint64_t* bars, const uint8_t* pool_bh,
+                          uint32_t tile_bytes, int t_begin, int t_end, int ring_it) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nmine = t_end - t_begin <= warp ? 0 : (t_end - t_begin - warp + kWarps - 1) / kWarps;
+  uint8_t* my_ring = ring + warp * kStages * kStageBytes;
+  uint64_t* my_bar = bars + warp * kStages;
+  if (lane == 0) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    for (int i = 0; i < kStages && i < nmine; ++i) {
+      const int tile = t_begin + warp + i * kWarps;
+      const int sl = (ring_it + i) % kStages;
+      mbar_expect_tx(&my_bar[sl], tile_bytes);
+      bulk_g2s(my_ring + sl * kStageBytes, pool_bh + (int64_t)tile * tile_bytes, tile_bytes,
+               &my_bar[sl]);
+    }
+  }
+  __syncwarp();
+}
+
 template <int L>
 __device__ void run_pool_any_g(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint4* aq_all,
                                uint64_t* bars, const uint8_t* pool_bh, int64_t count, int t0,
                                int t1, int G, WarpState& st, int& ring_it) {
   if (G <= 4)
-    run_pool<L, true>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it);
+    run_pool<L, true>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it, 0, true);
   else
-    run_pool<L, false>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it);
+    run_pool<L, false>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it, 0, true);
 }
 
 // Affine pools, balanced plan: CTA c takes the weighted range [c per, (c+1) per) of the
@@ -1289,19 +1312,20 @@ __global__ void __launch_bounds__(kThreads, kCtasAffine) decode_affine_kernel(De
       int n_hi, n_lo;
       pair_slots(P, bh, n_hi, n_lo);
       const int slot = (int)((int64_t)blockIdx.x - S / P.per) + (src ? n_hi : 0);
+      const int L = src ? a.L_lo : a.L_hi;
+      const int64_t cap = src ? a.lo_cap : a.hi_cap;
+      const int64_t count = src ? a.lo_count : a.hi_count;
+      const uint8_t* pool = src ? a.lo_pool : a.hi_pool;
+      const int rec = record_bytes_rt(SEMKV_BASE_AFFINE, L);
+      const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
+      uint64_t* bars = &sh.bar[0][0];
+      ring_fill(ring, bars, pool_bh, (uint32_t)(kTile * rec), t0, t1, ring_it);
       if (bh != loaded) {
         load_group_q(a, sh, b, h, G);
         loaded = bh;
       }
       WarpState st;
       state_init(st);
-      const int L = src ? a.L_lo : a.L_hi;
-      const int64_t cap = src ? a.lo_cap : a.hi_cap;
-      const int64_t count = src ? a.lo_count : a.hi_count;
-      const uint8_t* pool = src ? a.lo_pool : a.hi_pool;
-      const uint8_t* pool_bh =
-          pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * record_bytes_rt(SEMKV_BASE_AFFINE, L);
-      uint64_t* bars = &sh.bar[0][0];
       switch (L) {
         case 2: run_pool_any_g<2>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it); break;
         case 3: run_pool_any_g<3>(a, sh, ring, aq_all, bars, pool_bh, count, t0, t1, G, st, ring_it); break;

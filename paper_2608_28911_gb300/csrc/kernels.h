@@ -26,9 +26,11 @@ struct QuantArgs {
   int32_t* lo_tok;
   int32_t* err;
 };
-// n_hi: how many of the n tokens go to the high pool (the rest go to the low pool)
+// n_hi: how many of the n tokens go to the high pool (the rest go to the low pool).
+// maps_ready: the slot -> token maps of these tokens are already written (by the rank
+// kernel of a block append); otherwise a scatter kernel writes them first.
 cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
-                                 cudaStream_t stream);
+                                 cudaStream_t stream, bool maps_ready = false);
 
 // Top-r selection of each sequence (Eqs. 4-5).
 struct RankArgs {
@@ -40,6 +42,13 @@ struct RankArgs {
   uint32_t* slot;           // [B][T]
   uint32_t* rank;           // [B][T] or null
   uint32_t* ws;             // rank_workspace_words(B, T) words when rank is set
+  // Optional, T <= 1024 only (a block append): when hi_tok is set the kernel also
+  // writes the pools' slot -> token maps, hi_tok[b][hi_base + slot] = tok_base + i
+  // (lo likewise), and raises kDevCapacity in err for a slot past the capacity.
+  int32_t* hi_tok = nullptr;
+  int32_t* lo_tok = nullptr;
+  int64_t hi_base = 0, lo_base = 0, hi_cap = 0, lo_cap = 0, tok_base = 0;
+  int32_t* err = nullptr;
 };
 size_t rank_workspace_words(int B, int T);
 cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream);

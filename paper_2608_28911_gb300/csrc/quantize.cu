@@ -993,20 +993,26 @@ cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t strea
 }
 
 cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
-                                 cudaStream_t stream) {
+                                 cudaStream_t stream, bool maps_ready) {
   const int64_t total = (int64_t)a.B * a.NL * a.H * a.n;
   if (total == 0) return cudaSuccess;
   if (a.base == SEMKV_BASE_AFFINE) {
-    const int64_t pairs = (int64_t)a.B * a.n;
-    scatter_tok_kernel<<<(unsigned)((pairs + 255) / 256), 256, 0, stream>>>(a);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    // about 8 units per warp for the larger pool; the (sequence, layer, head) index
-    // runs over grid y (and loops past its limit of 65535)
+    if (!maps_ready) {
+      const int64_t pairs = (int64_t)a.B * a.n;
+      scatter_tok_kernel<<<(unsigned)((pairs + 255) / 256), 256, 0, stream>>>(a);
+      const cudaError_t e = cudaGetLastError();
+      if (e != cudaSuccess) return e;
+    }
+    // units per warp for the larger pool: enough warps for about one wave of 3 CTAs
+    // per SM, at most 8 units each; the (sequence, layer, head) index runs over grid y
+    // (and loops past its limit of 65535)
     const int64_t bhs = (int64_t)a.B * a.NL * a.H;
     const int64_t n_max = n_hi > a.n - n_hi ? n_hi : a.n - n_hi;
     const int64_t units = (n_max + kAffineSlots - 1) / kAffineSlots;
-    int64_t bx = (units + 8 * kWarpsPerBlock - 1) / (8 * kWarpsPerBlock);
+    const int64_t resident = (int64_t)(num_sms > 0 ? num_sms : 1) * 3 * kWarpsPerBlock;
+    int64_t per_warp = (2 * (bhs < 65535 ? bhs : 65535) * units + resident - 1) / resident;
+    per_warp = per_warp < 1 ? 1 : (per_warp > 8 ? 8 : per_warp);
+    int64_t bx = (units + per_warp * kWarpsPerBlock - 1) / (per_warp * kWarpsPerBlock);
     if (bx < 1) bx = 1;
     dim3 grid((unsigned)bx, (unsigned)(bhs < 65535 ? bhs : 65535), 2);
     quantize_affine_kernel<<<grid, kWarpsPerBlock * 32, 0, stream>>>(a, n_hi, a.n - n_hi);
@@ -1053,10 +1059,12 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
     return cudaGetLastError();
   }
   // TQ and rotated affine: slot -> token maps, then one thread per row by slot
-  const int64_t pairs = (int64_t)a.B * a.n;
-  scatter_tok_kernel<<<(unsigned)((pairs + 255) / 256), 256, 0, stream>>>(a);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
+  if (!maps_ready) {
+    const int64_t pairs = (int64_t)a.B * a.n;
+    scatter_tok_kernel<<<(unsigned)((pairs + 255) / 256), 256, 0, stream>>>(a);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
   const int64_t bhs = (int64_t)a.B * a.NL * a.H;
   const int64_t n_max = n_hi > a.n - n_hi ? n_hi : a.n - n_hi;
   int64_t bx = (n_max + kRowSlots - 1) / kRowSlots;

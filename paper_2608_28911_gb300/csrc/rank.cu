@@ -76,6 +76,7 @@ __global__ void __launch_bounds__(kThreads) rank_small_kernel(RankArgs a) {
   __syncthreads();
   uint32_t rank = 0;
   if (tid < T) {
+#pragma unroll 8
     for (int j = 0; j < T; ++j) {
       const uint32_t kj = keys[j];
       rank += (kj > mine || (kj == mine && j < tid)) ? 1u : 0u;
@@ -89,8 +90,18 @@ __global__ void __launch_bounds__(kThreads) rank_small_kernel(RankArgs a) {
   uint32_t before = __popc(bal & ((1u << lane) - 1u));
   for (int w = 0; w < warp; ++w) before += warp_hi[w];
   if (tid < T) {
+    const uint32_t slot = hi ? before : (uint32_t)tid - before;
     a.is_high[(int64_t)b * T + tid] = hi ? 1 : 0;
-    a.slot[(int64_t)b * T + tid] = hi ? before : (uint32_t)tid - before;
+    a.slot[(int64_t)b * T + tid] = slot;
+    if (a.hi_tok != nullptr) {
+      // a block append: the pools' slot -> token maps as well
+      const int64_t s = (hi ? a.hi_base : a.lo_base) + slot;
+      const int64_t cap = hi ? a.hi_cap : a.lo_cap;
+      if (s >= cap)  // cannot happen after the host's capacity check
+        raise_error(a.err, kDevCapacity);
+      else
+        (hi ? a.hi_tok : a.lo_tok)[(int64_t)b * cap + s] = (int32_t)(a.tok_base + tid);
+    }
   }
 }
 
