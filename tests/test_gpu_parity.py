@@ -166,6 +166,33 @@ def test_append_blocks_and_flush_match_oracle(base):
     check_attention(p, layer=1, qseed=99)
 
 
+@pytest.mark.parametrize("base,blk", [(0, 1024), (0, 1000), (1, 1024), (1, 1000)])
+def test_append_large_block_matches_oracle(base, blk):
+    """The largest block the cache allows (1024 tokens) and a ragged one: one pass ranks
+    the block and writes the pools' slot maps, then the block is packed."""
+    import torch
+    from paper_2608_28911_gb300 import semkv
+    T0, ngen = 64, blk + 3
+    p = Pair(base, 4 if base == 1 else 6, 3 if base == 1 else 5, 1, 1, 2, 8, T0, 26, 100,
+             seed=23, block=blk, extra_cap=ngen)
+    p.quantize()
+    k, v = synthetic.kv(24, 1, 1, 2, ngen)
+    s = synthetic.scores_zipf(24, 1, ngen)
+    for g in range(ngen):
+        kt = torch.from_numpy(np.ascontiguousarray(k[:, :, :, g])).to(p.dev)
+        vt = torch.from_numpy(np.ascontiguousarray(v[:, :, :, g])).to(p.dev)
+        p.cache.stage_token(kt, vt, torch.from_numpy(np.ascontiguousarray(s[:, g])).to(p.dev))
+        oracle.stage_token(p.oc, synthetic.f16_bits(k[:, :, :, g]), synthetic.f16_bits(v[:, :, :, g]),
+                           s[:, g])
+        if p.cache.stage_n == blk:
+            semkv.semkv_append_block(p.desc, p.cache, 26, 100)
+            oracle.append_block(p.oc, 26, 100)
+            torch.cuda.synchronize()
+            p.assert_records_equal()
+    assert p.cache.stage_n == 3 and int(p.cache.dev_error.item()) == 0
+    check_attention(p, layer=0, qseed=7)     # pools + the 3 staged fp16 tokens
+
+
 # ------------------------------------------- Hadamard-rotated affine decode -----
 
 @pytest.mark.parametrize("L_hi,L_lo,B,NL,H,Hq,T,r", [
