@@ -502,7 +502,8 @@ __device__ __forceinline__ void load_signs(const int8_t* sg, float (&x)[128]) {
 }
 
 template <int BASE>
-__global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : 3) fake_rows_kernel(FakeArgs a) {
+__global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : (BASE == SEMKV_BASE_AFFINE ? 5 : 3))
+    fake_rows_kernel(FakeArgs a) {
   __shared__ __align__(16) uint8_t stage[128 * kRowStride];
   __shared__ float cbs[2][8];
   const int tid = threadIdx.x;
@@ -528,121 +529,146 @@ __global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : 3) fake_rows_
       const int i = tid >> 1;
       const bool hi = i < nt && (a.is_high == nullptr || a.is_high[(int64_t)b * a.T + t0 + i] != 0);
       const int L = (a.is_high == nullptr || hi) ? a.L_hi : a.L_lo;
-      float x[128];
-#pragma unroll
-      for (int ch = 0; ch < 16; ++ch) {
-        const uint4 u = *reinterpret_cast<const uint4*>(stage + tid * kRowStride + ch * 16);
-        const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
-          x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
-        }
-      }
       const int8_t* sg = a.signs ? a.signs + ((int64_t)l * a.H + h) * kHeadDim : nullptr;
+      uint32_t ov[64];  // the row's fp16 outputs, in pairs
       if constexpr (BASE == SEMKV_BASE_AFFINE) {
-        // x^_d = fp16(z + s c_d)
-        float mn = x[0], mx = x[0];
+        // x^_d = fp16(z + s c_d), the row kept as fp16 pairs (fewer registers, more CTAs)
+        uint32_t hv[64];
 #pragma unroll
-        for (int j = 1; j < 128; ++j) {
-          mn = fminf(mn, x[j]);
-          mx = fmaxf(mx, x[j]);
+        for (int ch = 0; ch < 16; ++ch) {
+          const uint4 u = *reinterpret_cast<const uint4*>(stage + tid * kRowStride + ch * 16);
+          hv[4 * ch] = u.x;
+          hv[4 * ch + 1] = u.y;
+          hv[4 * ch + 2] = u.z;
+          hv[4 * ch + 3] = u.w;
         }
+        // row minimum and maximum on fp16 pairs (exact)
+        __half2 mn2 = *reinterpret_cast<const __half2*>(&hv[0]), mx2 = mn2;
+#pragma unroll
+        for (int j = 1; j < 64; ++j) {
+          const __half2 x2 = *reinterpret_cast<const __half2*>(&hv[j]);
+          mn2 = __hmin2(mn2, x2);
+          mx2 = __hmax2(mx2, x2);
+        }
+        float mn = fminf(__low2float(mn2), __high2float(mn2));
+        float mx = fmaxf(__low2float(mx2), __high2float(mx2));
         if (mn == 0.0f) mn = 0.0f;
         if (mx == 0.0f) mx = 0.0f;
         const uint16_t s16 = f16_param(__fdiv_rn(__fsub_rn(mx, mn), (float)(L - 1)));
         const float sv = f16_to_f32(s16), z = f16_to_f32(__half_as_ushort(__float2half_rn(mn)));
         const float inv = sv != 0.0f ? __fdiv_rn(1.0f, sv) : 0.0f;
+        // c = rint(min((x - z) / s, L - 1)) as an integer-valued float (x >= z: z is the
+        // row minimum; inv = 0 when s = 0, so every code is 0): adding and taking off
+        // 1.5 * 2^23 rounds to nearest even, as the float-to-int conversion would
 #pragma unroll
-        for (int j = 0; j < 128; ++j) {
-          int c = 0;
-          if (sv != 0.0f) c = min(max(__float2int_rn(__fmul_rn(__fsub_rn(x[j], z), inv)), 0), L - 1);
-          x[j] = __fadd_rn(z, __fmul_rn(sv, (float)c));
-        }
-      } else if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
-        // y = FWHT(z + s c);  x^_d = fp16((sign_d y_d) * fp32(1/sqrt 128))
-        load_signs(sg, x);
-        fwht128(x);
-        float mn = INFINITY, mx = -INFINITY;
+        for (int j = 0; j < 64; ++j) {
+          float r[2];
 #pragma unroll
-        for (int j = 0; j < 128; ++j) {
-          x[j] = __fmul_rn(x[j], kInvSqrtD);
-          mn = fminf(mn, x[j]);
-          mx = fmaxf(mx, x[j]);
-        }
-        if (mn == 0.0f) mn = 0.0f;
-        if (mx == 0.0f) mx = 0.0f;
-        uint16_t z16 = __half_as_ushort(__float2half_rd(mn));
-        if (z16 == 0xFC00u) z16 = 0xFBFFu;
-        const float z = f16_to_f32(z16);
-        const float sv = f16_to_f32(f16_param(__fdiv_rn(__fsub_rn(mx, z), (float)(L - 1))));
-        const bool live = sv > 0.0f;
-        const float inv = live ? __fdiv_rn(1.0f, sv) : 0.0f;
-#pragma unroll
-        for (int j = 0; j < 128; ++j) {
-          int c = 0;
-          if (live) c = min(max(__float2int_rn(__fmul_rn(__fsub_rn(x[j], z), inv)), 0), L - 1);
-          x[j] = __fadd_rn(z, __fmul_rn(sv, (float)c));
-        }
-        fwht128(x);
-        load_signs(sg, x);
-#pragma unroll
-        for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], kInvSqrtD);
-      } else {
-        // y = FWHT(cb[c]);  x^_d = fp16((sign_d y_d) * (n / 128))
-        float pn[16];
-#pragma unroll
-        for (int g = 0; g < 16; ++g) {
-          float acc[2];
-#pragma unroll
-          for (int hh = 0; hh < 2; ++hh) {
-            const int gg = g + 16 * hh;
-            float v = __fmul_rn(x[4 * gg], x[4 * gg]);
-#pragma unroll
-            for (int k = 1; k < 4; ++k) v = __fadd_rn(v, __fmul_rn(x[4 * gg + k], x[4 * gg + k]));
-            acc[hh] = v;
+          for (int e = 0; e < 2; ++e) {
+            const float x = f16_to_f32((uint16_t)(hv[j] >> (16 * e)));
+            const float y = fminf(__fmul_rn(__fsub_rn(x, z), inv), (float)(L - 1));
+            const float c = __fsub_rn(__fadd_rn(y, 12582912.0f), 12582912.0f);
+            r[e] = __fadd_rn(z, __fmul_rn(sv, c));
           }
-          pn[g] = __fadd_rn(acc[0], acc[1]);
+          const __half2 h2 = __floats2half2_rn(r[0], r[1]);
+          ov[j] = *reinterpret_cast<const uint32_t*>(&h2);
+        }
+      } else {
+        float x[128];
+#pragma unroll
+        for (int ch = 0; ch < 16; ++ch) {
+          const uint4 u = *reinterpret_cast<const uint4*>(stage + tid * kRowStride + ch * 16);
+          const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
+            x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
+          }
+        }
+        if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
+          // y = FWHT(z + s c);  x^_d = fp16((sign_d y_d) * fp32(1/sqrt 128))
+          load_signs(sg, x);
+          fwht128(x);
+          float mn = INFINITY, mx = -INFINITY;
+#pragma unroll
+          for (int j = 0; j < 128; ++j) {
+            x[j] = __fmul_rn(x[j], kInvSqrtD);
+            mn = fminf(mn, x[j]);
+            mx = fmaxf(mx, x[j]);
+          }
+          if (mn == 0.0f) mn = 0.0f;
+          if (mx == 0.0f) mx = 0.0f;
+          uint16_t z16 = __half_as_ushort(__float2half_rd(mn));
+          if (z16 == 0xFC00u) z16 = 0xFBFFu;
+          const float z = f16_to_f32(z16);
+          const float sv = f16_to_f32(f16_param(__fdiv_rn(__fsub_rn(mx, z), (float)(L - 1))));
+          const bool live = sv > 0.0f;
+          const float inv = live ? __fdiv_rn(1.0f, sv) : 0.0f;
+#pragma unroll
+          for (int j = 0; j < 128; ++j) {
+            int c = 0;
+            if (live) c = min(max(__float2int_rn(__fmul_rn(__fsub_rn(x[j], z), inv)), 0), L - 1);
+            x[j] = __fadd_rn(z, __fmul_rn(sv, (float)c));
+          }
+          fwht128(x);
+          load_signs(sg, x);
+#pragma unroll
+          for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], kInvSqrtD);
+        } else {
+          // y = FWHT(cb[c]);  x^_d = fp16((sign_d y_d) * (n / 128))
+          float pn[16];
+#pragma unroll
+          for (int g = 0; g < 16; ++g) {
+            float acc[2];
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+              const int gg = g + 16 * hh;
+              float v = __fmul_rn(x[4 * gg], x[4 * gg]);
+#pragma unroll
+              for (int k = 1; k < 4; ++k) v = __fadd_rn(v, __fmul_rn(x[4 * gg + k], x[4 * gg + k]));
+              acc[hh] = v;
+            }
+            pn[g] = __fadd_rn(acc[0], acc[1]);
+          }
+#pragma unroll
+          for (int off = 8; off >= 1; off >>= 1)
+#pragma unroll
+            for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
+          const uint16_t n16 = f16_param(__fsqrt_rn(pn[0]));
+          const float n = f16_to_f32(n16);
+          const float inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
+          const float* thr_g = hi || a.is_high == nullptr ? a.thr_hi : a.thr_lo;
+          const float* cb = cbs[(hi || a.is_high == nullptr) ? 0 : 1];
+          float thr[7];
+#pragma unroll
+          for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? thr_g[k] : INFINITY;
+          load_signs(sg, x);
+          fwht128(x);
+#pragma unroll
+          for (int j = 0; j < 128; ++j) {
+            const float u = __fmul_rn(x[j], inv);
+            int c = 0;
+#pragma unroll
+            for (int k = 0; k < 7; ++k) c += (u > thr[k]) ? 1 : 0;
+            x[j] = cb[n != 0.0f ? c : 0];
+          }
+          fwht128(x);
+          load_signs(sg, x);
+          const float nq = n * 0.0078125f;
+#pragma unroll
+          for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], nq);
         }
 #pragma unroll
-        for (int off = 8; off >= 1; off >>= 1)
-#pragma unroll
-          for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
-        const uint16_t n16 = f16_param(__fsqrt_rn(pn[0]));
-        const float n = f16_to_f32(n16);
-        const float inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
-        const float* thr_g = hi || a.is_high == nullptr ? a.thr_hi : a.thr_lo;
-        const float* cb = cbs[(hi || a.is_high == nullptr) ? 0 : 1];
-        float thr[7];
-#pragma unroll
-        for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? thr_g[k] : INFINITY;
-        load_signs(sg, x);
-        fwht128(x);
-#pragma unroll
-        for (int j = 0; j < 128; ++j) {
-          const float u = __fmul_rn(x[j], inv);
-          int c = 0;
-#pragma unroll
-          for (int k = 0; k < 7; ++k) c += (u > thr[k]) ? 1 : 0;
-          x[j] = cb[n != 0.0f ? c : 0];
+        for (int j = 0; j < 64; ++j) {
+          const __half2 h2 = __floats2half2_rn(x[2 * j], x[2 * j + 1]);
+          ov[j] = *reinterpret_cast<const uint32_t*>(&h2);
         }
-        fwht128(x);
-        load_signs(sg, x);
-        const float nq = n * 0.0078125f;
-#pragma unroll
-        for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], nq);
       }
       __syncthreads();  // every row is read: the stage takes the outputs
 #pragma unroll
-      for (int ch = 0; ch < 16; ++ch) {
-        uint4 u;
-        uint32_t* wv = reinterpret_cast<uint32_t*>(&u);
-#pragma unroll
-        for (int e = 0; e < 4; ++e)
-          wv[e] = (uint32_t)__half_as_ushort(__float2half_rn(x[8 * ch + 2 * e])) |
-                  ((uint32_t)__half_as_ushort(__float2half_rn(x[8 * ch + 2 * e + 1])) << 16);
-        *reinterpret_cast<uint4*>(stage + tid * kRowStride + ch * 16) = u;
-      }
+      for (int ch = 0; ch < 16; ++ch)
+        *reinterpret_cast<uint4*>(stage + tid * kRowStride + ch * 16) =
+            make_uint4(ov[4 * ch], ov[4 * ch + 1], ov[4 * ch + 2], ov[4 * ch + 3]);
       __syncthreads();
       for (int c = tid; c < 128 * 16; c += 128) {
         const int r = c >> 4, ch = c & 15, ii = r >> 1;
