@@ -197,7 +197,7 @@ __global__ void scatter_tok_kernel(QuantArgs a) {
 }
 
 // grid (x, sequence*layer*head, pool): each warp strides over that pool's units
-__global__ void __launch_bounds__(kWarpsPerBlock * 32)
+__global__ void __launch_bounds__(kWarpsPerBlock * 32, 4)
     quantize_affine_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
   __shared__ __align__(16) uint32_t img_sm[kWarpsPerBlock][kAffineSlots * kMaxRecWords];
   const int wib = threadIdx.x >> 5;
@@ -1029,16 +1029,25 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
       const cudaError_t e = cudaGetLastError();
       if (e != cudaSuccess) return e;
     }
-    // units per warp for the larger pool: enough warps for about one wave of 3 CTAs
-    // per SM, at most 8 units each; the (sequence, layer, head) index runs over grid y
-    // (and loops past its limit of 65535)
+    // grid x from a simple wave model: with R resident CTAs (4 per SM), the pass takes
+    // about ceil(CTAs / R) waves of ceil(units / (8 bx)) units per warp; take the
+    // cheapest bx (at most 16 units per warp).  The (sequence, layer, head) index runs
+    // over grid y (and loops past its limit of 65535)
     const int64_t bhs = (int64_t)a.B * a.NL * a.H;
     const int64_t n_max = n_hi > a.n - n_hi ? n_hi : a.n - n_hi;
     const int64_t units = (n_max + kAffineSlots - 1) / kAffineSlots;
-    const int64_t resident = (int64_t)(num_sms > 0 ? num_sms : 1) * 3 * kWarpsPerBlock;
-    int64_t per_warp = (2 * (bhs < 65535 ? bhs : 65535) * units + resident - 1) / resident;
-    per_warp = per_warp < 1 ? 1 : (per_warp > 8 ? 8 : per_warp);
-    int64_t bx = (units + per_warp * kWarpsPerBlock - 1) / (per_warp * kWarpsPerBlock);
+    const int64_t resident = (int64_t)(num_sms > 0 ? num_sms : 1) * 4;
+    const int64_t rows = 2 * (bhs < 65535 ? bhs : 65535);
+    int64_t bx = 1, best = -1;
+    for (int64_t pw = 16; pw >= 1; --pw) {
+      const int64_t cand = (units + pw * kWarpsPerBlock - 1) / (pw * kWarpsPerBlock);
+      const int64_t per = (units + cand * kWarpsPerBlock - 1) / (cand * kWarpsPerBlock);
+      const int64_t cost = ((cand * rows + resident - 1) / resident) * per;
+      if (best < 0 || cost * 50 < best * 49) {  // a near tie keeps the larger units
+        best = cost;
+        bx = cand;
+      }
+    }
     if (bx < 1) bx = 1;
     dim3 grid((unsigned)bx, (unsigned)(bhs < 65535 ? bhs : 65535), 2);
     quantize_affine_kernel<<<grid, kWarpsPerBlock * 32, 0, stream>>>(a, n_hi, a.n - n_hi);
