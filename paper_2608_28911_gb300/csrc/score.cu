@@ -27,7 +27,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32)
     float acc = 0.0f;
     for (int l = a.lb; l < a.le; ++l) {
       const uint16_t* lrow = a.x + (((int64_t)b * a.NL + l) * a.H * a.T + t) * kHeadDim + 4 * lane;
-#pragma unroll 4
+#pragma unroll 8
       for (int h = 0; h < a.H; ++h) {
         const uint2 u = *reinterpret_cast<const uint2*>(lrow + (int64_t)h * a.T * kHeadDim);
         const float x0 = f16_to_f32((uint16_t)(u.x & 0xFFFF)), x1 = f16_to_f32((uint16_t)(u.x >> 16));
