@@ -173,8 +173,9 @@ semkv_status semkv_rank_assign(const float* scores, int32_t batch, int32_t T,
  * reconstructed to fp16, in binary32 in this order:
  *   affine: out_d = fp16( z + s * c_d )
  *   TQ:     y = unnormalised FWHT(cb[c]) (stages 1..64);  out_d = fp16( (sign_d * y_d) * (n/128) )
- * k, v, k_out, v_out: device fp16 [batch][layers][kv_heads][T][128], 8-byte aligned,
- * caller-owned (outputs may not alias inputs); is_high: device u8 [batch][T] or NULL.
+ * k, v, k_out, v_out: device fp16 [batch][layers][kv_heads][T][128], 16-byte aligned
+ * (rows move in 16-byte chunks), caller-owned (outputs may not alias inputs); is_high:
+ * device u8 [batch][T] or NULL.
  * Errors: SEMKV_EINVAL, SEMKV_EALIGN, SEMKV_EUNSUPPORTED (level counts, base). */
 semkv_status semkv_fake_quant(const semkv_quant_desc* desc, const uint16_t* k, const uint16_t* v,
                               int32_t batch, int32_t layers, int32_t kv_heads, int32_t T,
@@ -200,8 +201,9 @@ semkv_status semkv_score_kv_norm(const uint16_t* x, int32_t batch, int32_t layer
  * K/V with Q_{b_i} and write token i's record (for every layer and KV head) to
  * slot[b][i] of the high pool if is_high[b][i] else of the low pool; writes
  * hi_tok/lo_tok[b][slot] = i.  k, v: device fp16 [batch][layers][kv_heads][T][128],
- * 8-byte aligned (16-byte for TQ_DENSE, whose rows the tensor cores read; the same
- * holds for the stage buffers in semkv_append_block).  is_high, slot: as produced by semkv_rank_assign for this T.  n_high: the number
+ * 8-byte aligned for AFFINE, 16-byte aligned for the other bases (their rows arrive by
+ * bulk or tensor copies in 16-byte units); the same holds for the stage buffers in
+ * semkv_append_block.  is_high, slot: as produced by semkv_rank_assign for this T.  n_high: the number
  * of high tokens per sequence (used for the capacity check and the counts).
  * Sets cache->hi_count = n_high, lo_count = T - n_high, n_tokens = T and resets
  * stage_n to 0 (a prompt replaces whatever the cache held). */

@@ -180,7 +180,7 @@ semkv_status semkv_fake_quant(const semkv_quant_desc* desc, const uint16_t* k, c
   if (desc->base == SEMKV_BASE_TQ_DENSE) return SEMKV_EUNSUPPORTED;
   if (!k || !v || !k_out || !v_out || batch < 1 || layers < 1 || kv_heads < 1 || T < 1)
     return SEMKV_EINVAL;
-  if (!aligned(k, 8) || !aligned(v, 8) || !aligned(k_out, 8) || !aligned(v_out, 8))
+  if (!aligned(k, 16) || !aligned(v, 16) || !aligned(k_out, 16) || !aligned(v_out, 16))
     return SEMKV_EALIGN;
   FakeArgs a;
   a.base = desc->base;
@@ -231,8 +231,8 @@ semkv_status semkv_quantize_pack(const semkv_quant_desc* desc, const uint16_t* k
   if (s != SEMKV_OK) return s;
   if (!k || !v || !is_high || !slot || T < 1) return SEMKV_EINVAL;
   if (!aligned(k, 8) || !aligned(v, 8)) return SEMKV_EALIGN;
-  if (desc->base == SEMKV_BASE_TQ_DENSE && (!aligned(k, 16) || !aligned(v, 16)))
-    return SEMKV_EALIGN;  // the rows are staged in 16-byte chunks
+  if (desc->base != SEMKV_BASE_AFFINE && (!aligned(k, 16) || !aligned(v, 16)))
+    return SEMKV_EALIGN;  // the rows arrive by bulk or tensor copies in 16-byte units
   if (n_high > (uint32_t)T) return SEMKV_EINVAL;
   if ((int64_t)n_high > cache->hi_cap || (int64_t)(T - n_high) > cache->lo_cap)
     return SEMKV_ECAPACITY;
@@ -285,7 +285,7 @@ semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache
       !cache->blk_slot)
     return SEMKV_EINVAL;
   if (!aligned(cache->stage_k, 8) || !aligned(cache->stage_v, 8)) return SEMKV_EALIGN;
-  if (desc->base == SEMKV_BASE_TQ_DENSE &&
+  if (desc->base != SEMKV_BASE_AFFINE &&
       (!aligned(cache->stage_k, 16) || !aligned(cache->stage_v, 16)))
     return SEMKV_EALIGN;
   const uint32_t n_high = semkv_block_high_count((uint32_t)n, r_num, r_den);

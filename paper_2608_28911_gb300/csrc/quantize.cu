@@ -297,7 +297,7 @@ __device__ __forceinline__ void or_field(uint32_t (&w)[N], int pos, const uint32
 
 template <int BASE, int L>
 __device__ void rows_block(const QuantArgs& a, int b, int l, int h, bool hi, int64_t s0,
-                           int nslots, uint8_t* stage, uint32_t* bits, uint32_t* par) {
+                           int nslots, uint8_t* stage) {
   using F = Fmt<L>;
   constexpr int kWords = (4 * F::QB + 31) / 32;
   constexpr int kRecW = (2 * F::RB + (BASE == SEMKV_BASE_TQ ? 4 : 8)) / 4;
@@ -306,30 +306,23 @@ __device__ void rows_block(const QuantArgs& a, int b, int l, int h, bool hi, int
   const int64_t cap = hi ? a.hi_cap : a.lo_cap;
   const int64_t pbase = hi ? a.hi_base : a.lo_base;
   const int64_t bh = ((int64_t)b * a.NL + l) * a.H + h;
-  const int32_t* tokmap = (hi ? a.hi_tok : a.lo_tok) + (int64_t)b * cap + pbase;
-  // ---- stage the rows of the block's slots (coalesced 16-byte chunks)
-  for (int c = tid; c < 128 * 16; c += 128) {
-    const int r = c >> 4, ch = c & 15, i = r >> 1;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (i < nslots) {
-      const int64_t t = (int64_t)tokmap[s0 + i] - a.tok_base;
-      const uint16_t* src = ((r & 1) ? a.v : a.k) + (bh * a.Tsrc + t) * kHeadDim;
-      v = __ldg(reinterpret_cast<const uint4*>(src) + ch);
-    }
-    *reinterpret_cast<uint4*>(stage + r * kRowStride + ch * 16) = v;
-  }
-  __syncthreads();
-  // ---- row tid: values, signs
+  // ---- row tid (its 256 bytes arrived in its own slot of the stage; rows past the
+  // block's slots are zeros)
   float x[128];
+  if ((tid >> 1) < nslots) {
 #pragma unroll
-  for (int ch = 0; ch < 16; ++ch) {
-    const uint4 u = *reinterpret_cast<const uint4*>(stage + tid * kRowStride + ch * 16);
-    const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+    for (int ch = 0; ch < 16; ++ch) {
+      const uint4 u = *reinterpret_cast<const uint4*>(stage + tid * kRowStride + ch * 16);
+      const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
-      x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
+      for (int e = 0; e < 4; ++e) {
+        x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
+        x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
+      }
     }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 128; ++j) x[j] = 0.0f;
   }
   uint32_t param;
   float zq = 0.0f, invq = 0.0f;  // affine: offset and 1/s;  TQ: 1/n in invq
@@ -426,9 +419,11 @@ __device__ void rows_block(const QuantArgs& a, int b, int l, int h, bool hi, int
     quarter_field<L>(m, fw);
     or_field<12>(w, q * F::QB, fw);
   }
+  // the row's bit image and parameters go to its own slot (its values are in registers)
+  uint32_t* mine = reinterpret_cast<uint32_t*>(stage + tid * kRowStride);
 #pragma unroll
-  for (int k = 0; k < kWords; ++k) bits[tid * kRowBitWords + k] = w[k];
-  par[tid] = param;
+  for (int k = 0; k < kWords; ++k) mine[k] = w[k];
+  mine[kRowBitWords] = param;
   __syncthreads();
   // ---- records: warp takes slots warp, warp + 4, ...; lane j writes word j
   uint32_t* recs = reinterpret_cast<uint32_t*>(hi ? a.hi_pool : a.lo_pool) + (bh * cap + pbase + s0) * kRecW;
@@ -437,49 +432,151 @@ __device__ void rows_block(const QuantArgs& a, int b, int l, int h, bool hi, int
       uint32_t word = 0u;
       if (4 * j >= 2 * F::RB) {
         const int pj = j - (2 * F::RB) / 4;
-        if constexpr (BASE == SEMKV_BASE_TQ) word = par[2 * i] | (par[2 * i + 1] << 16);
-        else word = par[2 * i + pj];
+        const uint32_t p0 = reinterpret_cast<const uint32_t*>(stage + (2 * i) * kRowStride)[kRowBitWords];
+        const uint32_t p1 = reinterpret_cast<const uint32_t*>(stage + (2 * i + 1) * kRowStride)[kRowBitWords];
+        if constexpr (BASE == SEMKV_BASE_TQ) word = p0 | (p1 << 16);
+        else word = pj ? p1 : p0;
       } else {
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const int byte = 4 * j + e;
           const int row = byte < F::RB ? 2 * i : 2 * i + 1;
           const int rb = byte < F::RB ? byte : byte - F::RB;
-          const uint32_t v = rb < F::RB ? (bits[row * kRowBitWords + (rb >> 2)] >> (8 * (rb & 3))) & 0xFFu : 0u;
+          const uint32_t v = rb < F::RB ? (reinterpret_cast<const uint32_t*>(stage + row * kRowStride)[rb >> 2] >>
+                                           (8 * (rb & 3))) & 0xFFu
+                                        : 0u;
           word |= v << (8 * e);
         }
       }
       recs[(int64_t)i * kRecW + j] = word;
     }
   }
-  __syncthreads();  // the staging area is free for the next block
+  __syncthreads();  // the stage is free for the copies of a later block
+}
+
+// ---- mbarriers
+__device__ __forceinline__ uint32_t dsmem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void dbar_init(uint64_t* bar) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(dsmem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool dbar_wait(uint64_t* bar, uint32_t parity) {
+  for (uint32_t i = 0; i < kSpinLimitQ; ++i) {
+    uint32_t r;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(r)
+        : "r"(dsmem_u32(bar)), "r"(parity)
+        : "memory");
+    if (r) return true;
+  }
+  return false;
+}
+
+// Persistent CTAs over the blocks (64 slots of one pool of one (sequence, layer, KV
+// head)), in a two-stage pipeline: while a block is quantized, the rows of the CTA's
+// next block are already on their way.  Thread r brings its own row r with one 256-byte
+// cp.async.bulk into its own 272-byte slot of the stage (so a slot is only ever touched
+// by its thread until the records are assembled); every thread arrives once per phase
+// on the stage's mbarrier (count 128), announcing its bytes.  Waits are bounded.
+constexpr int kRowStageBytes = 128 * kRowStride;
+static_assert(kRowBitWords + 1 <= kRowStride / 4, "bit image and parameters fit a row slot");
+
+__device__ __forceinline__ void rbar_init128(uint64_t* bar) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], 128;" ::"r"(dsmem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void rbar_arrive(uint64_t* bar, uint32_t tx_bytes) {
+  if (tx_bytes)
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(dsmem_u32(bar)),
+                 "r"(tx_bytes)
+                 : "memory");
+  else
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(dsmem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void bulk_g2s_row(void* dst, const void* src, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], 256, [%2];" ::"r"(
+          dsmem_u32(dst)),
+      "l"(src), "r"(dsmem_u32(bar))
+      : "memory");
+}
+
+// block t of the pass: (sequence, layer, head) index, pool, first slot, slot count
+struct RowsTile {
+  int bhi;
+  bool hi;
+  int64_t s0;
+  int nslots;
+};
+__device__ __forceinline__ RowsTile rows_tile(int64_t t, int64_t n_hi, int64_t n_lo) {
+  const int64_t nb_hi = (n_hi + kRowSlots - 1) / kRowSlots;
+  const int64_t nb_lo = (n_lo + kRowSlots - 1) / kRowSlots;
+  const int64_t r = t % (nb_hi + nb_lo);
+  RowsTile x;
+  x.bhi = (int)(t / (nb_hi + nb_lo));
+  x.hi = r < nb_hi;
+  x.s0 = (x.hi ? r : r - nb_hi) * kRowSlots;
+  x.nslots = (int)min((int64_t)kRowSlots, (x.hi ? n_hi : n_lo) - x.s0);
+  return x;
 }
 
 template <int BASE>
 __global__ void __launch_bounds__(128, 3) quantize_rows_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
-  __shared__ __align__(16) uint8_t stage[128 * kRowStride];
-  __shared__ uint32_t bits[128 * kRowBitWords];
-  __shared__ uint32_t par[128];
-  const bool hi = blockIdx.z == 0;
-  const int64_t n_pool = hi ? n_hi : n_lo;
-  const int bhs = a.B * a.NL * a.H;
-  const int L = hi ? a.L_hi : a.L_lo;
-  for (int64_t s0 = (int64_t)blockIdx.x * kRowSlots; s0 < n_pool; s0 += (int64_t)gridDim.x * kRowSlots) {
-    const int nslots = (int)min((int64_t)kRowSlots, n_pool - s0);
-    for (int bhi = blockIdx.y; bhi < bhs; bhi += gridDim.y) {
-      const int h = bhi % a.H, l = (bhi / a.H) % a.NL, b = bhi / (a.H * a.NL);
-      switch (L) {
+  extern __shared__ __align__(128) uint8_t rstage[];  // 2 stages of 128 row slots
+  __shared__ __align__(8) uint64_t rbar[2];
+  const int tid = threadIdx.x;
+  if (tid < 2) rbar_init128(&rbar[tid]);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  __syncthreads();
+  const int64_t bhs = (int64_t)a.B * a.NL * a.H;
+  const int64_t per_bh = (n_hi + kRowSlots - 1) / kRowSlots + (n_lo + kRowSlots - 1) / kRowSlots;
+  const int64_t total = bhs * per_bh;
+  // this thread's row of block t into stage st
+  auto issue = [&](int64_t t, int st) {
+    const RowsTile x = rows_tile(t, n_hi, n_lo);
+    const int i = tid >> 1;
+    if (i < x.nslots) {
+      const int h = x.bhi % a.H, l = (x.bhi / a.H) % a.NL, b = x.bhi / (a.H * a.NL);
+      const int64_t cap = x.hi ? a.hi_cap : a.lo_cap;
+      const int32_t* tokmap = (x.hi ? a.hi_tok : a.lo_tok) + (int64_t)b * cap + (x.hi ? a.hi_base : a.lo_base);
+      const int64_t tk = (int64_t)tokmap[x.s0 + i] - a.tok_base;
+      const int64_t bh = ((int64_t)b * a.NL + l) * a.H + h;
+      const uint16_t* src = ((tid & 1) ? a.v : a.k) + (bh * a.Tsrc + tk) * kHeadDim;
+      // this slot was last read (and written) through the generic proxy
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      rbar_arrive(&rbar[st], 256u);
+      bulk_g2s_row(rstage + st * kRowStageBytes + tid * kRowStride, src, &rbar[st]);
+    } else {
+      rbar_arrive(&rbar[st], 0u);
+    }
+  };
+  int64_t t = blockIdx.x;
+  if (t < total) issue(t, 0);
+  for (int k = 0; t < total; t += gridDim.x, ++k) {
+    const int st = k & 1;
+    const bool next = t + gridDim.x < total;
+    if (next) issue(t + gridDim.x, st ^ 1);
+    if (!__syncthreads_and(dbar_wait(&rbar[st], (uint32_t)((k >> 1) & 1)))) {
+      // a copy never landed: record it, let the other stage's copies finish, stop
+      if (tid == 0) raise_error(a.err, kDevWaitTimeout);
+      if (next) dbar_wait(&rbar[st ^ 1], (uint32_t)(((k + 1) >> 1) & 1));
+      return;
+    }
+    const RowsTile x = rows_tile(t, n_hi, n_lo);
+    const int h = x.bhi % a.H, l = (x.bhi / a.H) % a.NL, b = x.bhi / (a.H * a.NL);
+    uint8_t* stage = rstage + st * kRowStageBytes;
+    switch (x.hi ? a.L_hi : a.L_lo) {
 #define SEMKV_ROWS_CASE(LV) \
-        case LV: rows_block<BASE, LV>(a, b, l, h, hi, s0, nslots, stage, bits, par); break;
-        SEMKV_ROWS_CASE(2) SEMKV_ROWS_CASE(3) SEMKV_ROWS_CASE(4) SEMKV_ROWS_CASE(5)
-        SEMKV_ROWS_CASE(6) SEMKV_ROWS_CASE(7) SEMKV_ROWS_CASE(8)
+      case LV: rows_block<BASE, LV>(a, b, l, h, x.hi, x.s0, x.nslots, stage); break;
+      SEMKV_ROWS_CASE(2) SEMKV_ROWS_CASE(3) SEMKV_ROWS_CASE(4) SEMKV_ROWS_CASE(5)
+      SEMKV_ROWS_CASE(6) SEMKV_ROWS_CASE(7) SEMKV_ROWS_CASE(8)
 #undef SEMKV_ROWS_CASE
-        default: break;
-      }
+      default: break;
     }
   }
 }
-
 // ------------------------------------------------- fake quantization ---------
 // Every row quantized at its token's precision and reconstructed to fp16 (the quality
 // protocol of Sec. 4.1), in binary32 in this order:
@@ -710,25 +807,6 @@ constexpr uint32_t kDenseIdesc = (1u << 4) | ((64u >> 3) << 17) | ((128u >> 4) <
 __device__ __forceinline__ uint64_t umma_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
   return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
          ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46);
-}
-__device__ __forceinline__ uint32_t dsmem_u32(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
-}
-__device__ __forceinline__ void dbar_init(uint64_t* bar) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(dsmem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ bool dbar_wait(uint64_t* bar, uint32_t parity) {
-  for (uint32_t i = 0; i < kSpinLimitQ; ++i) {
-    uint32_t r;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-        " selp.u32 %0, 1, 0, p;\n}"
-        : "=r"(r)
-        : "r"(dsmem_u32(bar)), "r"(parity)
-        : "memory");
-    if (r) return true;
-  }
-  return false;
 }
 // 32 columns of this warp's 32 TMEM lanes (lane i of the warp <- TMEM lane 32 (w % 4) + i)
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
@@ -1100,16 +1178,30 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
+  // persistent CTAs (3 per SM) over every block of both pools
   const int64_t bhs = (int64_t)a.B * a.NL * a.H;
-  const int64_t n_max = n_hi > a.n - n_hi ? n_hi : a.n - n_hi;
-  int64_t bx = (n_max + kRowSlots - 1) / kRowSlots;
-  if (bx < 1) bx = 1;
-  if (bx > 65535) bx = 65535;
-  const dim3 grid((unsigned)bx, (unsigned)(bhs < 65535 ? bhs : 65535), 2);
+  const int64_t blocks = bhs * ((n_hi + kRowSlots - 1) / kRowSlots +
+                                (a.n - n_hi + kRowSlots - 1) / kRowSlots);
+  int64_t ctas = (int64_t)(num_sms > 0 ? num_sms : 1) * 3;
+  if (ctas > blocks) ctas = blocks;
+  if (ctas < 1) return cudaSuccess;
+  static bool rows_attr = false;
+  if (!rows_attr) {
+    cudaError_t e = cudaFuncSetAttribute(quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         2 * kRowStageBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(quantize_rows_kernel<SEMKV_BASE_TQ>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kRowStageBytes);
+    if (e != cudaSuccess) return e;
+    rows_attr = true;
+  }
   if (a.base == SEMKV_BASE_AFFINE_HAD)
-    quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD><<<grid, 128, 0, stream>>>(a, n_hi, a.n - n_hi);
+    quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)ctas, 128, 2 * kRowStageBytes, stream>>>(
+        a, n_hi, a.n - n_hi);
   else
-    quantize_rows_kernel<SEMKV_BASE_TQ><<<grid, 128, 0, stream>>>(a, n_hi, a.n - n_hi);
+    quantize_rows_kernel<SEMKV_BASE_TQ><<<(unsigned)ctas, 128, 2 * kRowStageBytes, stream>>>(
+        a, n_hi, a.n - n_hi);
   return cudaGetLastError();
 }
 

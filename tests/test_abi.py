@@ -102,6 +102,9 @@ def test_fake_quant_validation(lib):
                                 None) == 1
     assert lib.semkv_fake_quant(ctypes.byref(d), fake + 4, fake, 1, 1, 1, 1, None, fake, fake,
                                 None) == 2
+    # rows move in 16-byte chunks: 8-byte aligned buffers are refused too
+    assert lib.semkv_fake_quant(ctypes.byref(d), fake, fake, 1, 1, 1, 1, None, fake + 8, fake,
+                                None) == 2
     bad = QuantDescStruct(base=0, levels_hi=9, levels_lo=5, head_dim=128)
     assert lib.semkv_fake_quant(ctypes.byref(bad), fake, fake, 1, 1, 1, 1, None, fake, fake,
                                 None) == 4
