@@ -67,6 +67,7 @@ struct FakeArgs {
   const float* cent_lo;
   uint16_t* k_out;
   uint16_t* v_out;
+  int32_t* err = nullptr;   // device error word, or null (the call has none)
 };
 cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t stream);
 

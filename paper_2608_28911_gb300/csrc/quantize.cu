@@ -598,20 +598,97 @@ __device__ __forceinline__ void load_signs(const int8_t* sg, float (&x)[128]) {
   }
 }
 
+// The rotated-affine and TQ fake quantization of one row in registers (in: the row's
+// fp16 values as binary32; out: the reconstruction before its fp16 rounding).  sel_hi:
+// the row takes the high pool's tables (its token is high, or every token is).
 template <int BASE>
-__global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : (BASE == SEMKV_BASE_AFFINE ? 5 : 3))
-    fake_rows_kernel(FakeArgs a) {
-  __shared__ __align__(16) uint8_t stage[128 * kRowStride];
-  __shared__ float cbs[2][8];
-  const int tid = threadIdx.x;
-  if (BASE == SEMKV_BASE_TQ && tid < 16) {
-    const int which = tid >> 3, k = tid & 7;
-    const int L = which ? a.L_lo : a.L_hi;
-    cbs[which][k] = k < L ? (which ? a.cent_lo : a.cent_hi)[k] : 0.0f;
+__device__ __forceinline__ void fake_float_row(float (&x)[128], int L, bool sel_hi,
+                                               const int8_t* sg, const float (*cbs)[8],
+                                               const FakeArgs& a) {
+  if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
+    // y = FWHT(z + s c);  x^_d = fp16((sign_d y_d) * fp32(1/sqrt 128))
+    load_signs(sg, x);
+    fwht128(x);
+    float mn = INFINITY, mx = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 128; ++j) {
+      x[j] = __fmul_rn(x[j], kInvSqrtD);
+      mn = fminf(mn, x[j]);
+      mx = fmaxf(mx, x[j]);
+    }
+    if (mn == 0.0f) mn = 0.0f;
+    if (mx == 0.0f) mx = 0.0f;
+    uint16_t z16 = __half_as_ushort(__float2half_rd(mn));
+    if (z16 == 0xFC00u) z16 = 0xFBFFu;
+    const float z = f16_to_f32(z16);
+    const float sv = f16_to_f32(f16_param(__fdiv_rn(__fsub_rn(mx, z), (float)(L - 1))));
+    const bool live = sv > 0.0f;
+    const float inv = live ? __fdiv_rn(1.0f, sv) : 0.0f;
+#pragma unroll
+    for (int j = 0; j < 128; ++j) {
+      // c = rint(clamp((x - z) / s)) as an integer-valued float (magic-number rounding,
+      // to nearest even); every code is 0 when s = 0 (inv = 0)
+      const float y = fminf(fmaxf(__fmul_rn(__fsub_rn(x[j], z), inv), 0.0f), (float)(L - 1));
+      const float c = __fsub_rn(__fadd_rn(y, 12582912.0f), 12582912.0f);
+      x[j] = __fadd_rn(z, __fmul_rn(sv, c));
+    }
+    fwht128(x);
+    load_signs(sg, x);
+#pragma unroll
+    for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], kInvSqrtD);
+  } else {
+    // y = FWHT(cb[c]);  x^_d = fp16((sign_d y_d) * (n / 128))
+    float pn[16];
+#pragma unroll
+    for (int g = 0; g < 16; ++g) {
+      float acc[2];
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const int gg = g + 16 * hh;
+        float v = __fmul_rn(x[4 * gg], x[4 * gg]);
+#pragma unroll
+        for (int k = 1; k < 4; ++k) v = __fadd_rn(v, __fmul_rn(x[4 * gg + k], x[4 * gg + k]));
+        acc[hh] = v;
+      }
+      pn[g] = __fadd_rn(acc[0], acc[1]);
+    }
+#pragma unroll
+    for (int off = 8; off >= 1; off >>= 1)
+#pragma unroll
+      for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
+    const uint16_t n16 = f16_param(__fsqrt_rn(pn[0]));
+    const float n = f16_to_f32(n16);
+    const float inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
+    const float* thr_g = sel_hi ? a.thr_hi : a.thr_lo;
+    const float* cb = cbs[sel_hi ? 0 : 1];
+    float thr[7];
+#pragma unroll
+    for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? thr_g[k] : INFINITY;
+    load_signs(sg, x);
+    fwht128(x);
+#pragma unroll
+    for (int j = 0; j < 128; ++j) {
+      const float u = __fmul_rn(x[j], inv);
+      int c = 0;
+#pragma unroll
+      for (int k = 0; k < 7; ++k) c += (u > thr[k]) ? 1 : 0;
+      x[j] = cb[n != 0.0f ? c : 0];
+    }
+    fwht128(x);
+    load_signs(sg, x);
+    const float nq = n * 0.0078125f;
+#pragma unroll
+    for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], nq);
   }
+}
+
+// Affine base: a CTA per 64-token block, rows staged through shared memory in and out
+// (coalesced), each row kept as fp16 pairs (96 registers: 5 CTAs per SM).
+__global__ void __launch_bounds__(128, 5) fake_affine_kernel(FakeArgs a) {
+  __shared__ __align__(16) uint8_t stage[128 * kRowStride];
+  const int tid = threadIdx.x;
   const int64_t bhs = (int64_t)a.B * a.NL * a.H;
   for (int64_t bhi = blockIdx.y; bhi < bhs; bhi += gridDim.y) {
-    const int h = (int)(bhi % a.H), l = (int)((bhi / a.H) % a.NL);
     const int b = (int)(bhi / ((int64_t)a.H * a.NL));
     for (int t0 = blockIdx.x * kRowSlots; t0 < a.T; t0 += gridDim.x * kRowSlots) {
       const int nt = min(kRowSlots, a.T - t0);
@@ -626,9 +703,8 @@ __global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : (BASE == SEMK
       const int i = tid >> 1;
       const bool hi = i < nt && (a.is_high == nullptr || a.is_high[(int64_t)b * a.T + t0 + i] != 0);
       const int L = (a.is_high == nullptr || hi) ? a.L_hi : a.L_lo;
-      const int8_t* sg = a.signs ? a.signs + ((int64_t)l * a.H + h) * kHeadDim : nullptr;
       uint32_t ov[64];  // the row's fp16 outputs, in pairs
-      if constexpr (BASE == SEMKV_BASE_AFFINE) {
+      {
         // x^_d = fp16(z + s c_d), the row kept as fp16 pairs (fewer registers, more CTAs)
         uint32_t hv[64];
 #pragma unroll
@@ -670,96 +746,6 @@ __global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : (BASE == SEMK
           const __half2 h2 = __floats2half2_rn(r[0], r[1]);
           ov[j] = *reinterpret_cast<const uint32_t*>(&h2);
         }
-      } else {
-        float x[128];
-#pragma unroll
-        for (int ch = 0; ch < 16; ++ch) {
-          const uint4 u = *reinterpret_cast<const uint4*>(stage + tid * kRowStride + ch * 16);
-          const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
-            x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
-          }
-        }
-        if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
-          // y = FWHT(z + s c);  x^_d = fp16((sign_d y_d) * fp32(1/sqrt 128))
-          load_signs(sg, x);
-          fwht128(x);
-          float mn = INFINITY, mx = -INFINITY;
-#pragma unroll
-          for (int j = 0; j < 128; ++j) {
-            x[j] = __fmul_rn(x[j], kInvSqrtD);
-            mn = fminf(mn, x[j]);
-            mx = fmaxf(mx, x[j]);
-          }
-          if (mn == 0.0f) mn = 0.0f;
-          if (mx == 0.0f) mx = 0.0f;
-          uint16_t z16 = __half_as_ushort(__float2half_rd(mn));
-          if (z16 == 0xFC00u) z16 = 0xFBFFu;
-          const float z = f16_to_f32(z16);
-          const float sv = f16_to_f32(f16_param(__fdiv_rn(__fsub_rn(mx, z), (float)(L - 1))));
-          const bool live = sv > 0.0f;
-          const float inv = live ? __fdiv_rn(1.0f, sv) : 0.0f;
-#pragma unroll
-          for (int j = 0; j < 128; ++j) {
-            int c = 0;
-            if (live) c = min(max(__float2int_rn(__fmul_rn(__fsub_rn(x[j], z), inv)), 0), L - 1);
-            x[j] = __fadd_rn(z, __fmul_rn(sv, (float)c));
-          }
-          fwht128(x);
-          load_signs(sg, x);
-#pragma unroll
-          for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], kInvSqrtD);
-        } else {
-          // y = FWHT(cb[c]);  x^_d = fp16((sign_d y_d) * (n / 128))
-          float pn[16];
-#pragma unroll
-          for (int g = 0; g < 16; ++g) {
-            float acc[2];
-#pragma unroll
-            for (int hh = 0; hh < 2; ++hh) {
-              const int gg = g + 16 * hh;
-              float v = __fmul_rn(x[4 * gg], x[4 * gg]);
-#pragma unroll
-              for (int k = 1; k < 4; ++k) v = __fadd_rn(v, __fmul_rn(x[4 * gg + k], x[4 * gg + k]));
-              acc[hh] = v;
-            }
-            pn[g] = __fadd_rn(acc[0], acc[1]);
-          }
-#pragma unroll
-          for (int off = 8; off >= 1; off >>= 1)
-#pragma unroll
-            for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
-          const uint16_t n16 = f16_param(__fsqrt_rn(pn[0]));
-          const float n = f16_to_f32(n16);
-          const float inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
-          const float* thr_g = hi || a.is_high == nullptr ? a.thr_hi : a.thr_lo;
-          const float* cb = cbs[(hi || a.is_high == nullptr) ? 0 : 1];
-          float thr[7];
-#pragma unroll
-          for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? thr_g[k] : INFINITY;
-          load_signs(sg, x);
-          fwht128(x);
-#pragma unroll
-          for (int j = 0; j < 128; ++j) {
-            const float u = __fmul_rn(x[j], inv);
-            int c = 0;
-#pragma unroll
-            for (int k = 0; k < 7; ++k) c += (u > thr[k]) ? 1 : 0;
-            x[j] = cb[n != 0.0f ? c : 0];
-          }
-          fwht128(x);
-          load_signs(sg, x);
-          const float nq = n * 0.0078125f;
-#pragma unroll
-          for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], nq);
-        }
-#pragma unroll
-        for (int j = 0; j < 64; ++j) {
-          const __half2 h2 = __floats2half2_rn(x[2 * j], x[2 * j + 1]);
-          ov[j] = *reinterpret_cast<const uint32_t*>(&h2);
-        }
       }
       __syncthreads();  // every row is read: the stage takes the outputs
 #pragma unroll
@@ -776,6 +762,98 @@ __global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : (BASE == SEMK
       __syncthreads();
     }
   }
+}
+
+// Rotated affine and TQ: persistent CTAs over the 64-token blocks, each row moved by its
+// own thread with bulk copies in both directions: the rows of the CTA's next block are
+// loaded into the other stage while this block is computed, and each thread writes its
+// reconstructed row back from its own slot with one 256-byte bulk store.  A slot is only
+// ever touched by its thread, so the blocks need no CTA barrier; before a slot takes new
+// rows, its thread waits until its previous store has read it.  Waits are bounded.
+__device__ __forceinline__ void bulk_s2g_row(void* dst, const void* src) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], 256;" ::"l"(dst),
+               "r"(dsmem_u32(src))
+               : "memory");
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+
+template <int BASE>
+__global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : 3) fake_rows_kernel(FakeArgs a) {
+  extern __shared__ __align__(128) uint8_t fstage[];  // 2 stages of 128 row slots
+  __shared__ __align__(8) uint64_t fbar[2];
+  __shared__ float cbs[2][8];
+  const int tid = threadIdx.x;
+  if (tid < 2) rbar_init128(&fbar[tid]);
+  if (BASE == SEMKV_BASE_TQ && tid < 16) {
+    const int which = tid >> 3, k = tid & 7;
+    const int L = which ? a.L_lo : a.L_hi;
+    cbs[which][k] = k < L ? (which ? a.cent_lo : a.cent_hi)[k] : 0.0f;
+  }
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  __syncthreads();
+  const int64_t bhs = (int64_t)a.B * a.NL * a.H;
+  const int64_t nblk = ((int64_t)a.T + kRowSlots - 1) / kRowSlots;
+  const int64_t total = bhs * nblk;
+  const int i = tid >> 1;
+  auto issue = [&](int64_t t, int st) {
+    const int64_t bhi = t / nblk;
+    const int t0 = (int)(t % nblk) * kRowSlots;
+    if (i < a.T - t0) {
+      const uint16_t* src = ((tid & 1) ? a.v : a.k) + (bhi * a.T + t0 + i) * kHeadDim;
+      asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");  // the slot's last store
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      rbar_arrive(&fbar[st], 256u);
+      bulk_g2s_row(fstage + st * kRowStageBytes + tid * kRowStride, src, &fbar[st]);
+    } else {
+      rbar_arrive(&fbar[st], 0u);
+    }
+  };
+  int64_t t = blockIdx.x;
+  if (t < total) issue(t, 0);
+  for (int k = 0; t < total; t += gridDim.x, ++k) {
+    const int st = k & 1;
+    const bool next = t + gridDim.x < total;
+    if (next) issue(t + gridDim.x, st ^ 1);
+    if (!__syncthreads_and(dbar_wait(&fbar[st], (uint32_t)((k >> 1) & 1)))) {
+      // a copy never landed: record it, let the other stage's copies finish, stop
+      if (tid == 0) raise_error(a.err, kDevWaitTimeout);
+      if (next) dbar_wait(&fbar[st ^ 1], (uint32_t)(((k + 1) >> 1) & 1));
+      break;
+    }
+    const int64_t bhi = t / nblk;
+    const int t0 = (int)(t % nblk) * kRowSlots;
+    if (i >= a.T - t0) continue;  // past the sequence's end
+    const int h = (int)(bhi % a.H), l = (int)((bhi / a.H) % a.NL);
+    const int b = (int)(bhi / ((int64_t)a.H * a.NL));
+    const bool sel_hi = a.is_high == nullptr || a.is_high[(int64_t)b * a.T + t0 + i] != 0;
+    const int L = sel_hi ? a.L_hi : a.L_lo;
+    uint8_t* slot = fstage + st * kRowStageBytes + tid * kRowStride;
+    float x[128];
+#pragma unroll
+    for (int ch = 0; ch < 16; ++ch) {
+      const uint4 u = *reinterpret_cast<const uint4*>(slot + ch * 16);
+      const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
+        x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
+      }
+    }
+    fake_float_row<BASE>(x, L, sel_hi, a.signs + ((int64_t)l * a.H + h) * kHeadDim, cbs, a);
+#pragma unroll
+    for (int ch = 0; ch < 16; ++ch) {
+      uint32_t w[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const __half2 h2 = __floats2half2_rn(x[8 * ch + 2 * e], x[8 * ch + 2 * e + 1]);
+        w[e] = *reinterpret_cast<const uint32_t*>(&h2);
+      }
+      *reinterpret_cast<uint4*>(slot + ch * 16) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the row, to the async proxy
+    bulk_s2g_row(((tid & 1) ? a.v_out : a.k_out) + (bhi * a.T + t0 + i) * kHeadDim, slot);
+  }
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");  // every store done before exit
 }
 
 // ------------------------------------- dense-rotation TQ rows (tcgen05) --------
@@ -1080,19 +1158,33 @@ __global__ void __launch_bounds__(kDenseThreads, 2)
 }  // namespace
 
 cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t stream) {
-  (void)num_sms;
   const int64_t total = (int64_t)a.B * a.NL * a.H * a.T;
   if (total == 0) return cudaSuccess;
   const int64_t bhs = (int64_t)a.B * a.NL * a.H;
-  int64_t bx = ((int64_t)a.T + kRowSlots - 1) / kRowSlots;
-  if (bx > 65535) bx = 65535;
-  const dim3 grid((unsigned)bx, (unsigned)(bhs < 65535 ? bhs : 65535));
-  if (a.base == SEMKV_BASE_AFFINE)
-    fake_rows_kernel<SEMKV_BASE_AFFINE><<<grid, 128, 0, stream>>>(a);
-  else if (a.base == SEMKV_BASE_AFFINE_HAD)
-    fake_rows_kernel<SEMKV_BASE_AFFINE_HAD><<<grid, 128, 0, stream>>>(a);
+  const int64_t nblk = ((int64_t)a.T + kRowSlots - 1) / kRowSlots;
+  if (a.base == SEMKV_BASE_AFFINE) {
+    const dim3 grid((unsigned)(nblk < 65535 ? nblk : 65535), (unsigned)(bhs < 65535 ? bhs : 65535));
+    fake_affine_kernel<<<grid, 128, 0, stream>>>(a);
+    return cudaGetLastError();
+  }
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(fake_rows_kernel<SEMKV_BASE_AFFINE_HAD>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         2 * kRowStageBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(fake_rows_kernel<SEMKV_BASE_TQ>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kRowStageBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  // persistent: 3 CTAs per SM (2 for TQ, whose registers allow no more)
+  int64_t ctas = (int64_t)(num_sms > 0 ? num_sms : 1) * (a.base == SEMKV_BASE_TQ ? 2 : 3);
+  if (ctas > bhs * nblk) ctas = bhs * nblk;
+  if (a.base == SEMKV_BASE_AFFINE_HAD)
+    fake_rows_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)ctas, 128, 2 * kRowStageBytes, stream>>>(a);
   else
-    fake_rows_kernel<SEMKV_BASE_TQ><<<grid, 128, 0, stream>>>(a);
+    fake_rows_kernel<SEMKV_BASE_TQ><<<(unsigned)ctas, 128, 2 * kRowStageBytes, stream>>>(a);
   return cudaGetLastError();
 }
 
