@@ -371,8 +371,8 @@ def gpu_arm(args, cfg, rank, world):
     # launches per decode call: (rotation for TQ,) pools, (stage,) combine
     plain = cfg["base"] == semkv.BASE_AFFINE
     dec_launch = (0 if plain else 1) + 1 + 1     # (query rotation,) pools, combine
-    # rank, slot -> token scatter (not for the dense rotation), quantize
-    app_launch = 2 if cfg["base"] == semkv.BASE_TQ_DENSE else 3
+    # a block append: the block rank (which also writes the slot -> token maps), quantize
+    app_launch = 2
 
     def decode_all(qv, ev=None):
         if ev is not None:
