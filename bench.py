@@ -368,9 +368,10 @@ def gpu_arm(args, cfg, rank, world):
     scale = 1.0 / math.sqrt(128)
     base_counts = (cache.s.hi_count, cache.s.lo_count, cache.s.n_tokens)
     nh_b = semkv.semkv_block_high_count(blk, r_num, r_den)
-    # launches per decode call: (rotation for TQ,) pools, (stage,) combine
+    # launches per decode call: (query rotation,) pools, combine (plus the stage kernel
+    # while tokens are staged)
     plain = cfg["base"] == semkv.BASE_AFFINE
-    dec_launch = (0 if plain else 1) + 1 + 1     # (query rotation,) pools, combine
+    dec_launch = (0 if plain else 1) + 1 + 1
     # a block append: the block rank (which also writes the slot -> token maps), quantize
     app_launch = 2
 
@@ -753,9 +754,9 @@ def main():
         "fake_quant_gbs": r["fake_gbs"],
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": profiled_traffic(args.config),
-                     "kernel": {0: "decode_affine_kernel + combine_wide_kernel", 2: "decode_affine_kernel + combine_wide_kernel",
-                                1: "decode_kernel<1> + combine_wide_kernel",
-                                3: "decode_kernel<1> + combine_kernel<dense>"}[cfg["base"]]
+                     "kernel": {0: "decode_affine_kernel + combine_wide_kernel", 2: "qrot_kernel + decode_affine_kernel + combine_wide_kernel",
+                                1: "qrot_kernel + decode_kernel<1> + combine_wide_kernel",
+                                3: "qrot_dense_kernel + decode_kernel<1> + combine_kernel<dense>"}[cfg["base"]]
                                + " (semkv_decode_attention)",
                      "peak_kind": f"{peak_kind} hbm_gbs"},
         "e2e": {"value": job_gbs(step_bytes, world, r["e2e_time"]), "unit": "GB/s",
