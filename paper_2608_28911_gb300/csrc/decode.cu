@@ -1518,6 +1518,9 @@ __global__ void combine_kernel(DecodeArgs a) {
     for (int x = threadIdx.x; x < 128 * 16; x += blockDim.x) reinterpret_cast<uint4*>(ms)[x] = src[x];
     __syncthreads();
   }
+  // launched as a programmatic dependent of the pool kernels: the rotation above is
+  // staged while they finish; their partials are read only after this wait
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   if (gw >= a.B * a.Hq) return;
   const int b = gw / a.Hq, qh = gw % a.Hq;
   const int h = qh / G, c = qh % G;
@@ -1568,6 +1571,8 @@ __global__ void __launch_bounds__(256) combine_wide_kernel(DecodeArgs a) {
   __shared__ float wsm[kMaxPartialsPerPair];
   __shared__ float red[8][128];
   __shared__ float red_m[8], red_l[8];
+  // launched as a programmatic dependent of the pool kernels: wait for their partials
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const int gw = blockIdx.x;
   const int b = gw / a.Hq, qh = gw % a.Hq;
@@ -1800,12 +1805,25 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
+  // the combine starts as a programmatic dependent launch: its launch (and, for the
+  // dense rotation, the staging of M) overlaps the tail of the kernels before it
   const int heads = a.B * a.Hq;
-  if (a.base == SEMKV_BASE_TQ_DENSE)
-    combine_kernel<true><<<a.B * a.H, 32 * (a.Hq / a.H), 0, stream>>>(a);
-  else
-    combine_wide_kernel<<<heads, 256, 0, stream>>>(a);
-  return cudaGetLastError();
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.dynamicSmemBytes = 0;
+  if (a.base == SEMKV_BASE_TQ_DENSE) {
+    cfg.gridDim = dim3((unsigned)(a.B * a.H));
+    cfg.blockDim = dim3((unsigned)(32 * (a.Hq / a.H)));
+    return cudaLaunchKernelEx(&cfg, combine_kernel<true>, a);
+  }
+  cfg.gridDim = dim3((unsigned)heads);
+  cfg.blockDim = dim3(256);
+  return cudaLaunchKernelEx(&cfg, combine_wide_kernel, a);
 }
 
 }  // namespace semkv
