@@ -176,7 +176,10 @@ semkv_status semkv_rank_assign(const float* scores, int32_t batch, int32_t T,
  * k, v, k_out, v_out: device fp16 [batch][layers][kv_heads][T][128], 16-byte aligned
  * (rows move in 16-byte chunks), caller-owned (outputs may not alias inputs); is_high:
  * device u8 [batch][T] or NULL.
- * Errors: SEMKV_EINVAL, SEMKV_EALIGN, SEMKV_EUNSUPPORTED (level counts, base). */
+ * Errors: SEMKV_EINVAL, SEMKV_EALIGN, SEMKV_EUNSUPPORTED (level counts, base).  There is
+ * no device error word: the rotated bases move rows with bulk copies whose waits are
+ * bounded, and a copy that never completed would stop its CTA, leaving the rows it had
+ * not yet written unchanged. */
 semkv_status semkv_fake_quant(const semkv_quant_desc* desc, const uint16_t* k, const uint16_t* v,
                               int32_t batch, int32_t layers, int32_t kv_heads, int32_t T,
                               const uint8_t* is_high, uint16_t* k_out, uint16_t* v_out,
