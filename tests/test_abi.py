@@ -111,3 +111,35 @@ def test_fake_quant_validation(lib):
     tq = QuantDescStruct(base=1, levels_hi=4, levels_lo=3, head_dim=128)  # no tables
     assert lib.semkv_fake_quant(ctypes.byref(tq), fake, fake, 1, 1, 1, 1, None, fake, fake,
                                 None) == 1
+
+
+def test_row_alignment_rules_per_base(lib):
+    """K/V rows move in 16-byte units (bulk or tensor copies) for every base but the
+    affine one, which also takes 8-byte aligned rows; misaligned rows are refused with
+    SEMKV_EALIGN before anything is launched."""
+    from paper_2608_28911_gb300.semkv import CacheStruct, QuantDescStruct
+    p, i32, u32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_uint32
+    lib.semkv_quantize_pack.argtypes = [p, p, p, i32, p, p, u32, p, p]
+    lib.semkv_append_block.argtypes = [p, p, u32, u32, p]
+    fake = 1 << 20  # never dereferenced: every call below fails validation before a launch
+    c = CacheStruct(batch=1, layers=1, kv_heads=1, q_heads=4, head_dim=128, block=16,
+                    hi_pool=fake, lo_pool=fake, hi_cap=16, lo_cap=16, hi_tok=fake,
+                    lo_tok=fake, stage_k=fake + 8, stage_v=fake, stage_score=fake,
+                    stage_n=4, blk_is_high=fake, blk_slot=fake, dev_error=fake)
+    aff = QuantDescStruct(base=0, levels_hi=6, levels_lo=5, head_dim=128)
+    tq = QuantDescStruct(base=1, levels_hi=4, levels_lo=3, head_dim=128, signs=fake,
+                         centroids_hi=fake, thresholds_hi=fake, centroids_lo=fake,
+                         thresholds_lo=fake)
+    had = QuantDescStruct(base=2, levels_hi=6, levels_lo=5, head_dim=128, signs=fake)
+    for d in (tq, had):
+        # rows 8-byte but not 16-byte aligned
+        assert lib.semkv_quantize_pack(ctypes.byref(d), fake + 8, fake, 16, fake, fake, 4,
+                                       ctypes.byref(c), None) == 2
+        assert lib.semkv_quantize_pack(ctypes.byref(d), fake, fake + 8, 16, fake, fake, 4,
+                                       ctypes.byref(c), None) == 2
+        assert lib.semkv_append_block(ctypes.byref(d), ctypes.byref(c), 1, 4, None) == 2
+    # the affine base refuses rows that are not even 8-byte aligned
+    assert lib.semkv_quantize_pack(ctypes.byref(aff), fake + 4, fake, 16, fake, fake, 4,
+                                   ctypes.byref(c), None) == 2
+    c.stage_k = fake + 4
+    assert lib.semkv_append_block(ctypes.byref(aff), ctypes.byref(c), 1, 4, None) == 2
