@@ -1296,6 +1296,7 @@ __global__ void __launch_bounds__(kThreads, kCtasAffine) decode_affine_kernel(De
   if (threadIdx.x < kWarps * kStages) mbar_init(&sh.bar[0][0] + threadIdx.x);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncthreads();
+  pdl_wait();  // the records, queries and stage partial come from earlier work
   int ring_it = 0;  // tiles this warp has taken through its ring (barrier phases)
   int64_t loaded = -1;
   for (int64_t bh = start / P.W; bh < pairs && bh * P.W < end; ++bh) {
@@ -1795,8 +1796,11 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
       e = cudaGetLastError();
       if (e != cudaSuccess) return e;
     }
-    if (P.ctas > 0)
-      decode_affine_kernel<<<P.ctas, kThreads, kRingBytes + kAqBytes, stream>>>(a);
+    if (P.ctas > 0) {
+      e = launch_pdl(decode_affine_kernel, dim3(P.ctas), dim3(kThreads), kRingBytes + kAqBytes,
+                     stream, a);
+      if (e != cudaSuccess) return e;
+    }
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;

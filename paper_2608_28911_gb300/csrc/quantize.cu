@@ -201,6 +201,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 4)
     quantize_affine_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
   __shared__ __align__(16) uint32_t img_sm[kWarpsPerBlock][kAffineSlots * kMaxRecWords];
   const int wib = threadIdx.x >> 5;
+  pdl_wait();  // the slot maps and the rows come from earlier work on the stream
   const bool hi = blockIdx.z == 0;
   const int64_t n_pool = hi ? n_hi : n_lo;
   const int64_t u_begin = (int64_t)blockIdx.x * kWarpsPerBlock + wib;
@@ -1220,8 +1221,8 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
     }
     if (bx < 1) bx = 1;
     dim3 grid((unsigned)bx, (unsigned)(bhs < 65535 ? bhs : 65535), 2);
-    quantize_affine_kernel<<<grid, kWarpsPerBlock * 32, 0, stream>>>(a, n_hi, a.n - n_hi);
-    return cudaGetLastError();
+    return launch_pdl(quantize_affine_kernel, grid, dim3(kWarpsPerBlock * 32), 0, stream, a, n_hi,
+                      a.n - n_hi);
   }
   if (a.base == SEMKV_BASE_TQ_DENSE) {
     static bool attr_set = false;

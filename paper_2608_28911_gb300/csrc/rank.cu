@@ -70,6 +70,7 @@ __global__ void __launch_bounds__(kThreads) rank_small_kernel(RankArgs a) {
   __shared__ uint32_t warp_hi[32];
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int T = a.T;
+  pdl_wait();  // the scores (and the maps) belong to earlier work on the stream
   const float* s = a.scores + (int64_t)b * a.ld;
   const uint32_t mine = tid < T ? order_key(s[tid]) : 0u;
   keys[tid] = mine;
@@ -497,7 +498,8 @@ cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream) {
   if (a.B == 0 || a.T == 0) return cudaSuccess;
   const uint32_t chunk = ((uint32_t)a.T + kCluster - 1) / kCluster;
   if (a.T <= kThreads) {
-    rank_small_kernel<<<a.B, kThreads, 0, stream>>>(a);
+    const cudaError_t e = launch_pdl(rank_small_kernel, dim3(a.B), dim3(kThreads), 0, stream, a);
+    if (e != cudaSuccess) return e;
   } else if (a.T >= 8192 && chunk <= kSmemKeys) {
     static bool cattr_set = false;
     if (!cattr_set) {
