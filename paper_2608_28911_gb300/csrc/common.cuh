@@ -81,6 +81,21 @@ __device__ __forceinline__ void raise_error(int32_t* err, int32_t code) {
   if (err) atomicCAS(err, 0, code);
 }
 
+// Kernel attributes (the opt-in dynamic shared memory size) are per device: set() runs
+// the first time a launcher is called on each device.
+constexpr int kAttrDevices = 64;
+template <typename F>
+inline cudaError_t once_per_device(bool (&done)[kAttrDevices], F set) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kAttrDevices) return cudaErrorInvalidDevice;
+  if (done[dev]) return cudaSuccess;
+  e = set();
+  if (e == cudaSuccess) done[dev] = true;
+  return e;
+}
+
 // Programmatic dependent launch: the kernel may be scheduled while the previous kernel
 // on the stream drains; it must call pdl_wait() before touching what that kernel (or
 // anything earlier on the stream) wrote.  pdl_wait is a no-op for an ordinary launch.

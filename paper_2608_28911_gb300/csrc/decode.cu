@@ -129,13 +129,9 @@ __device__ __forceinline__ void mma16816(float c[4], uint32_t a0, uint32_t a1, u
 __device__ __forceinline__ uint32_t fdig(uint32_t beta, float c) {
   return __float_as_uint(__fmul_rz(__uint_as_float(beta), c));
 }
-// the same with 0x6400 added in the denormal grid: the low 16 bits are then the fp16
-// value 1024 + F (F < 1024)
-__device__ __forceinline__ uint32_t fdig1024(uint32_t beta, float c) {
-  return __float_as_uint(__fmaf_rz(__uint_as_float(beta), c, __uint_as_float(0x6400u)));
-}
-// fdig and fdig1024 of two symbols (or one symbol and two constants) in one packed
-// binary32 instruction: lane 0 takes (a, ca), lane 1 (b, cb)
+// fdig of two symbols (or one symbol and two constants) in one packed binary32
+// instruction, lane 0 taking (a, ca) and lane 1 (b, cb); fdig1024_x2 adds 0x6400 in the
+// denormal grid, so the low 16 bits are the fp16 value 1024 + F (F < 1024)
 __device__ __forceinline__ unsigned long long u2_pack(uint32_t lo, uint32_t hi) {
   return (unsigned long long)lo | ((unsigned long long)hi << 32);
 }
@@ -250,29 +246,8 @@ struct Dec {
   static constexpr int G = F::G;
   static constexpr int kHalf = F::NG / 2;                     // symbols per half quarter
   static constexpr int kRestart = (L == 6) ? 2 : G;           // F chain restarts here
-  // 1024 + F values of one full symbol, in the low 16 bits of each word (F < 256)
-  __device__ __forceinline__ static void sym(uint32_t beta, uint32_t* f) {
-    if constexpr (G == 1) {
-      // L = 2, 4, 8 store the code itself; seven levels take one multiply
-      f[0] = L == 7 ? fdig1024(beta, 7.0f / 8.0f) : (beta | 0x6400u);
-    } else if constexpr (L == 6) {
-      constexpr float c1 = 6.0f / 8192.0f, c2 = 36.0f / 8192.0f, c3 = 216.0f / 8192.0f;
-      f[0] = fdig1024(beta, c1);
-      f[1] = fdig1024(beta, c2);
-      const uint32_t x = (beta * 36u) & 8191u;  // remainder after two digits
-      f[2] = fdig1024(x, c1);
-      f[3] = fdig1024(x, c2);
-      f[4] = fdig1024(x, c3);
-    } else {
-      float c = (float)L / (float)(1u << F::W);
-#pragma unroll
-      for (int k = 0; k < G; ++k) {
-        f[k] = fdig1024(beta, c);
-        c *= (float)L;
-      }
-    }
-  }
-  // sym of two symbols at once, in packed instructions
+  // 1024 + F values of two full symbols (fa, fb: the low 16 bits of each word, F < 256),
+  // two per packed instruction
   __device__ __forceinline__ static void sym2(uint32_t ba, uint32_t bb, uint32_t* fa,
                                               uint32_t* fb) {
     if constexpr (G == 1) {
@@ -1757,19 +1732,21 @@ size_t decode_workspace_floats(int B, int H, int Hq) {
 }
 
 cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(decode_affine_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kRingBytes + kAqBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               kRingBytes + kAqBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(decode_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               kRingBytes);
+  static bool attr_set[kAttrDevices] = {};
+  {
+    const cudaError_t e = once_per_device(attr_set, [] {
+      cudaError_t r = cudaFuncSetAttribute(decode_affine_kernel,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           kRingBytes + kAqBytes);
+      if (r == cudaSuccess)
+        r = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kRingBytes + kAqBytes);
+      if (r == cudaSuccess)
+        r = cudaFuncSetAttribute(decode_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kRingBytes);
+      return r;
+    });
     if (e != cudaSuccess) return e;
-    attr_set = true;
   }
   const DecodePlan& P = a.plan;
   if (P.stride < 1 || P.stride > kMaxSplits + 1) return cudaErrorInvalidValue;

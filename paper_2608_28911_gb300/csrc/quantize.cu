@@ -1168,17 +1168,17 @@ cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t strea
     fake_affine_kernel<<<grid, 128, 0, stream>>>(a);
     return cudaGetLastError();
   }
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(fake_rows_kernel<SEMKV_BASE_AFFINE_HAD>,
+  static bool attr_set[kAttrDevices] = {};
+  const cudaError_t e = once_per_device(attr_set, [] {
+    cudaError_t r = cudaFuncSetAttribute(fake_rows_kernel<SEMKV_BASE_AFFINE_HAD>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          2 * kRowStageBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(fake_rows_kernel<SEMKV_BASE_TQ>,
+    if (r == cudaSuccess)
+      r = cudaFuncSetAttribute(fake_rows_kernel<SEMKV_BASE_TQ>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kRowStageBytes);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+    return r;
+  });
+  if (e != cudaSuccess) return e;
   // persistent: 3 CTAs per SM (2 for TQ, whose registers allow no more)
   int64_t ctas = (int64_t)(num_sms > 0 ? num_sms : 1) * (a.base == SEMKV_BASE_TQ ? 2 : 3);
   if (ctas > bhs * nblk) ctas = bhs * nblk;
@@ -1225,19 +1225,21 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
                       a.n - n_hi);
   }
   if (a.base == SEMKV_BASE_TQ_DENSE) {
-    static bool attr_set = false;
+    static bool attr_set[kAttrDevices] = {};
     static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
-    if (!attr_set) {
-      cudaError_t e = cudaFuncSetAttribute(quantize_tq_dense_kernel,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)kDenseSmem);
-      if (e != cudaSuccess) return e;
+    cudaError_t e = once_per_device(attr_set, [] {
+      return cudaFuncSetAttribute(quantize_tq_dense_kernel,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDenseSmem);
+    });
+    if (e != cudaSuccess) return e;
+    if (!encode) {  // the driver's entry point (the same for every device)
       cudaDriverEntryPointQueryResult q;
-      e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&encode),
+      PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+      e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&fn),
                                            12000, cudaEnableDefault, &q);
-      if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !encode)
+      if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
         return e != cudaSuccess ? e : cudaErrorNotSupported;
-      attr_set = true;
+      encode = fn;
     }
     // rows of K (V) as a 3-D view: 8 values, every (sequence, layer, head, token) row,
     // 16 groups of 8 values; a box of 64 rows lands as 8-row x 16-byte core matrices
@@ -1278,16 +1280,18 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
   int64_t ctas = (int64_t)(num_sms > 0 ? num_sms : 1) * 3;
   if (ctas > blocks) ctas = blocks;
   if (ctas < 1) return cudaSuccess;
-  static bool rows_attr = false;
-  if (!rows_attr) {
-    cudaError_t e = cudaFuncSetAttribute(quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         2 * kRowStageBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(quantize_rows_kernel<SEMKV_BASE_TQ>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kRowStageBytes);
+  static bool rows_attr[kAttrDevices] = {};
+  {
+    const cudaError_t e = once_per_device(rows_attr, [] {
+      cudaError_t r = cudaFuncSetAttribute(quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           2 * kRowStageBytes);
+      if (r == cudaSuccess)
+        r = cudaFuncSetAttribute(quantize_rows_kernel<SEMKV_BASE_TQ>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kRowStageBytes);
+      return r;
+    });
     if (e != cudaSuccess) return e;
-    rows_attr = true;
   }
   if (a.base == SEMKV_BASE_AFFINE_HAD)
     quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)ctas, 128, 2 * kRowStageBytes, stream>>>(

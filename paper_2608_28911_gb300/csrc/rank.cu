@@ -501,24 +501,20 @@ cudaError_t launch_rank_assign(const RankArgs& a, cudaStream_t stream) {
     const cudaError_t e = launch_pdl(rank_small_kernel, dim3(a.B), dim3(kThreads), 0, stream, a);
     if (e != cudaSuccess) return e;
   } else if (a.T >= 8192 && chunk <= kSmemKeys) {
-    static bool cattr_set = false;
-    if (!cattr_set) {
-      const cudaError_t e = cudaFuncSetAttribute(rank_cluster_kernel,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)(kSmemKeys * sizeof(uint32_t)));
-      if (e != cudaSuccess) return e;
-      cattr_set = true;
-    }
+    static bool cattr_set[kAttrDevices] = {};
+    const cudaError_t e = once_per_device(cattr_set, [] {
+      return cudaFuncSetAttribute(rank_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)(kSmemKeys * sizeof(uint32_t)));
+    });
+    if (e != cudaSuccess) return e;
     rank_cluster_kernel<<<a.B * kCluster, kThreads, (size_t)chunk * sizeof(uint32_t), stream>>>(a);
   } else {
-    static bool attr_set = false;
-    if (!attr_set) {
-      const cudaError_t e = cudaFuncSetAttribute(rank_assign_kernel,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)(kSmemKeys * sizeof(uint32_t)));
-      if (e != cudaSuccess) return e;
-      attr_set = true;
-    }
+    static bool attr_set[kAttrDevices] = {};
+    const cudaError_t e = once_per_device(attr_set, [] {
+      return cudaFuncSetAttribute(rank_assign_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)(kSmemKeys * sizeof(uint32_t)));
+    });
+    if (e != cudaSuccess) return e;
     const size_t smem = (uint32_t)a.T <= kSmemKeys ? (size_t)a.T * sizeof(uint32_t) : 0;
     rank_assign_kernel<<<a.B, kThreads, smem, stream>>>(a);
   }
