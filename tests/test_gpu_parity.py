@@ -120,6 +120,18 @@ def test_decode_attention_matches_oracle(L_hi, L_lo, B, NL, H, Hq, T, r):
         check_attention(p, layer)
 
 
+@pytest.mark.parametrize("L", [2, 7, 8])
+def test_uniform_grid_points_quantize_and_decode(L):
+    """The uniform grid points of the cliff sweep (1.0, 2.807, 3.0 bits per code): every
+    token at L levels (r = 0, the high pool empty), records bit-exact, attention within
+    tolerance."""
+    p = Pair(0, L, L, 1, 1, 2, 8, 300, 0, 100, seed=40 + L)
+    p.quantize()
+    assert np.array_equal(p.is_high.cpu().numpy(), p.o_is_high)
+    p.assert_records_equal()
+    check_attention(p)
+
+
 @pytest.mark.parametrize("base", [0, 2])
 def test_decode_attention_with_staged_tail(base):
     p = Pair(base, 6, 5, 2, 1, 2, 8, 300, 26, 100, seed=11, block=32)
