@@ -136,11 +136,26 @@ class Pair:
     def decode(self, layer=0, qseed=0, heads=None):
         torch, semkv = self.torch, self.semkv
         q = synthetic.queries(self.seed + 100 * qseed, self.B, self.Hq)
-        out = torch.empty((self.B, self.Hq, 128), dtype=torch.float32, device=self.dev)
+        # the output sits between two canary regions that must come back untouched
+        n, pad, canary = self.B * self.Hq * 128, 64, -1234.5
+        big = torch.full((n + 2 * pad,), canary, dtype=torch.float32, device=self.dev)
+        out = big[pad:pad + n].view(self.B, self.Hq, 128)
         ws = self.cache.workspace()
         scale = 1.0 / math.sqrt(128)
         semkv.semkv_decode_attention(self.desc, self.cache, layer, torch.from_numpy(q).to(self.dev),
                                      out, scale, ws)
         torch.cuda.synchronize()
+        g = big.cpu().numpy()
+        assert np.all(g[:pad] == canary) and np.all(g[pad + n:] == canary), "decode wrote past out"
         ref = oracle.decode_attention(self.oc, layer, synthetic.f16_bits(q), scale, heads=heads)
-        return out.cpu().numpy(), ref
+        return g[pad:pad + n].reshape(self.B, self.Hq, 128), ref
+
+    def assert_untouched_past_counts(self):
+        """Canaries: the pools were zero-filled and the slot maps filled with -1 when the
+        cache was allocated; nothing may be written past the counts."""
+        c = self.cache
+        hc, lc = c.s.hi_count, c.s.lo_count
+        assert not c.hi_pool.cpu().numpy()[..., hc:, :].any()
+        assert not c.lo_pool.cpu().numpy()[..., lc:, :].any()
+        assert np.all(c.hi_tok.cpu().numpy()[:, hc:] == -1)
+        assert np.all(c.lo_tok.cpu().numpy()[:, lc:] == -1)

@@ -67,6 +67,7 @@ def test_quantize_pack_bit_exact(base, L_hi, L_lo, B, NL, H, T, r):
     p.quantize()
     assert np.array_equal(p.is_high.cpu().numpy(), p.o_is_high)
     p.assert_records_equal()
+    p.assert_untouched_past_counts()
     assert int(p.cache.dev_error.item()) == 0
 
 
@@ -362,10 +363,18 @@ def test_fake_quant_bit_exact(base, L_hi, L_lo, B, NL, H, T, mixed):
     desc = semkv.QuantDesc(base, L_hi, L_lo, signs=sg)
     kt = torch.from_numpy(k).to(d)
     vt = torch.from_numpy(v).to(d)
-    ko, vo = torch.empty_like(kt), torch.empty_like(vt)
+    # outputs between canary regions (fp16 bit pattern 0x7BCD) that must stay untouched
+    n, pad, canary = kt.numel(), 64, 0x7BCD
+    kbig = torch.full((n + 2 * pad,), canary, dtype=torch.int16, device=d)
+    vbig = torch.full((n + 2 * pad,), canary, dtype=torch.int16, device=d)
+    ko = kbig[pad:pad + n].view(torch.float16).view(kt.shape)
+    vo = vbig[pad:pad + n].view(torch.float16).view(vt.shape)
     iht = torch.from_numpy(ih).to(d) if mixed else None
     semkv.semkv_fake_quant(desc, kt, vt, ko, vo, is_high=iht)
     torch.cuda.synchronize()
+    for big in (kbig, vbig):
+        g = big.cpu().numpy()
+        assert np.all(g[:pad] == canary) and np.all(g[pad + n:] == canary), "wrote past the output"
     kw = {}
     if base == semkv.BASE_TQ:
         cbs = []
