@@ -35,49 +35,70 @@ def test_had_65_batch1_32k_every_record_and_head():
     assert err <= ATOL and rel <= RTOL_L2, (err, rel)
 
 
-def test_batch16_64k_sampled_sequences_and_heads():
+def test_batch16_64k_timed_step_sampled_sequences_every_head():
+    """The benchmark's step at its full size: batch 16 x 64K prompt (rank + quantize),
+    one appended 128-token block (Algorithm 2), then decode over 65536 + 128 tokens in
+    the same launch configuration.  Four sequences are redone by the oracle: their
+    records bit for bit and every query head's attention."""
     import torch
     from paper_2608_28911_gb300 import semkv
-    B, T, H, Hq = 16, 65536, 8, 32
+    B, T, H, Hq, blk = 16, 65536, 8, 32, 128
     dev = torch.device("cuda:0")
     n_high = oracle.high_count_floor(T, 26, 100)
+    n_blk = oracle.block_high_count(blk, 26, 100)
     desc = semkv.QuantDesc(semkv.BASE_AFFINE, 6, 5, device=dev)
-    cache = semkv.KVCache(desc, B, 1, H, Hq, hi_cap=n_high, lo_cap=T - n_high, device=dev)
+    cache = semkv.KVCache(desc, B, 1, H, Hq, hi_cap=n_high + n_blk,
+                          lo_cap=T - n_high + blk - n_blk, block=blk, device=dev)
     k = torch.empty((B, 1, H, T, 128), dtype=torch.float16, device=dev)
     v = torch.empty_like(k)
     s = np.stack([synthetic.scores_zipf(300 + b, 1, T)[0] for b in range(B)])
+    kblk, vblk = synthetic.kv(399, B, 1, H, blk)
+    sblk = synthetic.scores_zipf(399, B, blk)
+    check = (0, 5, 11, 15)
     host = {}
     for b in range(B):
         kb, vb = synthetic.kv(300 + b, 1, 1, H, T)
         k[b].copy_(torch.from_numpy(kb[0]))
         v[b].copy_(torch.from_numpy(vb[0]))
-        if b in (0, 11):
+        if b in check:
             host[b] = (kb, vb)
     is_high = torch.empty((B, T), dtype=torch.uint8, device=dev)
     slot = torch.empty((B, T), dtype=torch.int32, device=dev)
     semkv.semkv_rank_assign(torch.from_numpy(s).to(dev), n_high, is_high, slot)
     semkv.semkv_quantize_pack(desc, k, v, is_high, slot, n_high, cache)
+    del k, v
+    # the block, staged as a serving loop fills the stage, then appended
+    cache.stage_k[:, :, :, :blk].copy_(torch.from_numpy(kblk))
+    cache.stage_v[:, :, :, :blk].copy_(torch.from_numpy(vblk))
+    cache.stage_score[:, :blk].copy_(torch.from_numpy(sblk))
+    cache.s.stage_n = blk
+    semkv.semkv_append_block(desc, cache, 26, 100)
+    assert cache.hi_count == n_high + n_blk and cache.stage_n == 0
     q = synthetic.queries(300, B, Hq)
     out = torch.empty((B, Hq, 128), dtype=torch.float32, device=dev)
     semkv.semkv_decode_attention(desc, cache, 0, torch.from_numpy(q).to(dev), out,
                                  1 / math.sqrt(128), cache.workspace())
     torch.cuda.synchronize()
+    assert int(cache.dev_error.item()) == 0
     o_is_high, _, _ = oracle.rank_assign(s, n_high)
     assert np.array_equal(is_high.cpu().numpy(), o_is_high)
     got = out.cpu().numpy()
+    hc, lc = cache.hi_count, cache.lo_count
     for b, (kb, vb) in host.items():
         oc = oracle.Cache(base=0, L_hi=6, L_lo=5, batch=1, layers=1, kv_heads=H, q_heads=Hq,
-                          block=128, hi_cap=cache.s.hi_cap, lo_cap=cache.s.lo_cap)
+                          block=blk, hi_cap=cache.s.hi_cap, lo_cap=cache.s.lo_cap)
         oracle.quantize_prompt(oc, synthetic.f16_bits(kb), synthetic.f16_bits(vb), s[b:b + 1], 26, 100)
-        assert np.array_equal(cache.hi_pool[b:b + 1].cpu().numpy()[..., :n_high, :],
-                              oc.hi_pool[..., :n_high, :])
-        assert np.array_equal(cache.lo_pool[b:b + 1].cpu().numpy()[..., :T - n_high, :],
-                              oc.lo_pool[..., :T - n_high, :])
-        heads = [(0, qh) for qh in (0, 13, 31)]
-        ref = oracle.decode_attention(oc, 0, synthetic.f16_bits(q[b:b + 1]), 1 / math.sqrt(128),
-                                      heads=heads)
-        sel = np.array([qh for _, qh in heads])
-        err, rel = attention_errors(got[b:b + 1, sel], ref[:, sel])
+        kb16, vb16 = synthetic.f16_bits(kblk[b:b + 1]), synthetic.f16_bits(vblk[b:b + 1])
+        for g in range(blk):
+            oracle.stage_token(oc, kb16[:, :, :, g], vb16[:, :, :, g], sblk[b:b + 1, g])
+        oracle.append_block(oc, 26, 100)
+        assert (oc.hi_count, oc.lo_count) == (hc, lc)
+        assert np.array_equal(cache.hi_pool[b:b + 1].cpu().numpy()[..., :hc, :], oc.hi_pool[..., :hc, :])
+        assert np.array_equal(cache.lo_pool[b:b + 1].cpu().numpy()[..., :lc, :], oc.lo_pool[..., :lc, :])
+        assert np.array_equal(cache.hi_tok[b:b + 1].cpu().numpy()[:, :hc], oc.hi_tok[:, :hc])
+        assert np.array_equal(cache.lo_tok[b:b + 1].cpu().numpy()[:, :lc], oc.lo_tok[:, :lc])
+        ref = oracle.decode_attention(oc, 0, synthetic.f16_bits(q[b:b + 1]), 1 / math.sqrt(128))
+        err, rel = attention_errors(got[b:b + 1], ref)
         assert err <= ATOL and rel <= RTOL_L2, (b, err, rel)
 
 
@@ -182,7 +203,8 @@ def test_value_norm_scores_batch16_64k_sampled_sequences():
 
 def test_fake_quant_batch16_64k_sampled_sequences():
     # the batch-16 x 64K prompt's K and V, reconstructed at the 6/5 split of the
-    # rank; sequences 3 and 14 compared with the oracle bit for bit
+    # rank; sequences 3 and 14 compared with the oracle bit for bit, the oracle taking
+    # its own top-r selection
     import torch
     from paper_2608_28911_gb300 import semkv
     B, T, H = 16, 65536, 8
@@ -207,8 +229,11 @@ def test_fake_quant_batch16_64k_sampled_sequences():
     torch.cuda.synchronize()
     ih = is_high.cpu().numpy()
     for b, (kb, vb) in host.items():
+        # the oracle makes its own selection (Eq. 4-5), which must be the GPU's
+        o_ih, _, _ = oracle.rank_assign(s[b:b + 1], n_high)
+        assert np.array_equal(ih[b:b + 1], o_ih), b
         o_k, o_v = oracle.fake_quant(0, 6, 5, synthetic.f16_bits(kb), synthetic.f16_bits(vb),
-                                     is_high=ih[b:b + 1])
+                                     is_high=o_ih)
         assert np.array_equal(ko[b:b + 1].cpu().numpy().view(np.uint16), o_k), b
         assert np.array_equal(vo[b:b + 1].cpu().numpy().view(np.uint16), o_v), b
 
