@@ -233,7 +233,11 @@ semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache
  * dequantized rows (affine: z + s*c; TQ: n/128 * S H cb[c]).  Computed split-K over
  * the tokens with an online softmax and a final combine.
  * q: device fp16 [batch][q_heads][128]; out: device f32 [batch][q_heads][128].
- * ws: device workspace of semkv_decode_workspace_bytes(cache) bytes, 16-B aligned. */
+ * ws: device workspace of semkv_decode_workspace_bytes(cache) bytes, 16-B aligned.
+ * Accuracy: against fp64 attention over the same dequantized cache, max-abs error
+ * <= 2e-3 and relative L2 <= 1e-3 for values of magnitude below 64; binary32 carries
+ * relative error, so for larger values the absolute error grows as about 1e-6 *
+ * max|v^| (all of fp16's range, including subnormal steps, is supported). */
 size_t semkv_decode_workspace_bytes(const semkv_cache* cache);
 semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_cache* cache,
                                     int32_t layer, const uint16_t* q, float* out,
@@ -245,19 +249,23 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
  * Who needs it: a caller whose host framework owns all device memory and gives this
  * library only the cache and the tensors of the call, or a serving loop that must
  * not call cudaMalloc between decode steps (an allocation can synchronise the device).
- * It computes exactly what semkv_decode_attention computes (same kernels, affine base
- * only), but keeps the split-K partial results in a static device array of 8 MiB
+ * It computes what semkv_decode_attention computes, for every base, with the same
+ * kernels, but keeps the split-K partial results in a static device array of 8 MiB
  * (2016 partials) that the library owns, instead of a caller workspace; it calls no
  * cudaMalloc, cudaFree or allocating routine.  Every GPU that loads the library
  * holds that array until the process exits.
  *  - Set-up: the first call on each device looks up the array's device address
- *    (cudaGetSymbolAddress) with that device current; make that first call before
- *    any stream capture.
- *  - Limit: batch * kv_heads * (one partial per non-empty pool, plus one when tokens
- *    are staged) must fit in 2016 partials; larger requests return SEMKV_EWORKSPACE.
- *    Within the limit the split count is reduced to fit.  The rotated bases (TQ,
- *    AFFINE_HAD, TQ_DENSE) also keep their rotated queries in a second static array
- *    of 4096 query heads (batch * q_heads beyond it: SEMKV_EWORKSPACE).
+ *    (cudaGetSymbolAddress) with that device current and caches it; make that first
+ *    call before any stream capture.  The cached address is not refreshed after
+ *    cudaDeviceReset.  Host threads may make their first calls concurrently.
+ *  - Limit: each (sequence, KV head) pair gets cap = min(65, 2016 / (batch *
+ *    kv_heads)) partial slots, and the split count is reduced to fit them.  The
+ *    affine bases (balanced plan) need cap >= 3 + stage, i.e. batch * kv_heads <= 672,
+ *    or <= 504 with staged tokens; the TQ bases (split plan) need cap >= one per
+ *    non-empty pool + stage, i.e. batch * kv_heads * (pools + stage) <= 2016.
+ *    Larger requests return SEMKV_EWORKSPACE before anything is launched.  The rotated
+ *    bases (TQ, AFFINE_HAD, TQ_DENSE) also keep their rotated queries in a second
+ *    static array of 4096 query heads (batch * q_heads beyond it: SEMKV_EWORKSPACE).
  *  - All calls share the array, which keeps the last call's contents (each call
  *    overwrites every partial it reads, so nothing needs clearing).  Calls whose
  *    kernels overlap on the GPU (e.g. on two streams, or two host threads) race on
@@ -267,6 +275,18 @@ semkv_status semkv_decode_attention_noalloc(const semkv_quant_desc* desc,
                                             const semkv_cache* cache, int32_t layer,
                                             const uint16_t* q, float* out, float softmax_scale,
                                             void* stream);
+
+/* Failure-detection check (not a step of the paper's method).  Every kernel that
+ * waits on a bulk copy uses one bounded mbarrier wait: after a fixed number of polls
+ * (2^22) it gives up, writes 1 (a wait that timed out) into the device error word and
+ * the kernel returns, so a lost copy never hangs the GPU and the context stays usable.
+ * This entry point runs that same wait in one CTA of 4 warps on a barrier that nothing
+ * arrives on, with the caller's poll limit `polls` (1 .. 2^22): each warp's wait runs
+ * out and writes 1 into *dev_error (device int32, 4-byte aligned; the first error
+ * written wins, so clear it first to see this one).  It lets a test make a wait run
+ * out on purpose without faulting or hanging anything.  Stream-ordered; errors:
+ * SEMKV_EINVAL (NULL dev_error, polls out of range), SEMKV_EALIGN, SEMKV_ECUDA. */
+semkv_status semkv_debug_wait_timeout(int32_t* dev_error, uint32_t polls, void* stream);
 
 /* Human-readable name of a status code (static string). */
 const char* semkv_status_string(semkv_status s);

@@ -14,7 +14,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 OUT = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT, "libsemkv.so")
-SOURCES = ["api.cu", "quantize.cu", "rank.cu", "decode.cu", "noalloc.cu", "score.cu"]
+SOURCES = ["api.cu", "quantize.cu", "rank.cu", "decode.cu", "noalloc.cu", "score.cu",
+           "failure.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-ftz=false", "-prec-div=true", "-prec-sqrt=true", "--expt-relaxed-constexpr", "-Xcompiler", "-fPIC",
          "-I", INCLUDE]

@@ -4,60 +4,13 @@
 #include <cstdint>
 #include <cstring>
 
+#include "checks.h"
 #include "common.cuh"
 #include "kernels.h"
 
 using namespace semkv;
 
 namespace {
-
-bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
-
-bool level_ok(int L) { return L >= 2 && L <= SEMKV_MAX_LEVELS; }
-
-semkv_status check_desc(const semkv_quant_desc* d) {
-  if (!d) return SEMKV_EINVAL;
-  if (d->head_dim != SEMKV_HEAD_DIM) return SEMKV_EUNSUPPORTED;
-  if (d->base != SEMKV_BASE_AFFINE && d->base != SEMKV_BASE_TQ &&
-      d->base != SEMKV_BASE_AFFINE_HAD && d->base != SEMKV_BASE_TQ_DENSE)
-    return SEMKV_EUNSUPPORTED;
-  if (!level_ok(d->levels_hi) || !level_ok(d->levels_lo)) return SEMKV_EUNSUPPORTED;
-  if (d->base == SEMKV_BASE_AFFINE_HAD) {
-    if (!d->signs) return SEMKV_EINVAL;
-    if (!aligned(d->signs, 4)) return SEMKV_EALIGN;
-  }
-  if (d->base == SEMKV_BASE_TQ_DENSE) {
-    if (!d->rotation || !d->thresholds_hi || !d->thresholds_lo || !d->centroids_hi ||
-        !d->centroids_lo)
-      return SEMKV_EINVAL;
-    if (!aligned(d->rotation, 16)) return SEMKV_EALIGN;
-  }
-  if (d->base == SEMKV_BASE_TQ) {
-    if (!d->signs || !d->thresholds_hi || !d->thresholds_lo || !d->centroids_hi ||
-        !d->centroids_lo)
-      return SEMKV_EINVAL;
-    if (!aligned(d->signs, 4)) return SEMKV_EALIGN;
-  }
-  return SEMKV_OK;
-}
-
-semkv_status check_cache(const semkv_cache* c) {
-  if (!c) return SEMKV_EINVAL;
-  if (c->batch < 1 || c->layers < 1 || c->kv_heads < 1 || c->q_heads < 1) return SEMKV_EINVAL;
-  if (c->head_dim != SEMKV_HEAD_DIM) return SEMKV_EUNSUPPORTED;
-  if (c->q_heads % c->kv_heads != 0) return SEMKV_EINVAL;
-  if (c->q_heads / c->kv_heads > 8) return SEMKV_EUNSUPPORTED;
-  if (c->block < 1 || c->block > 1024) return SEMKV_EINVAL;
-  if (!c->hi_pool || !c->lo_pool || !c->hi_tok || !c->lo_tok) return SEMKV_EINVAL;
-  if (!aligned(c->hi_pool, 16) || !aligned(c->lo_pool, 16)) return SEMKV_EALIGN;
-  if (c->hi_cap < 0 || c->lo_cap < 0 || c->hi_cap % 16 || c->lo_cap % 16) return SEMKV_EALIGN;
-  // slot indices are 32-bit inside the kernels
-  if (c->hi_cap > (int64_t)1 << 30 || c->lo_cap > (int64_t)1 << 30) return SEMKV_EUNSUPPORTED;
-  if (c->hi_count < 0 || c->lo_count < 0 || c->hi_count > c->hi_cap || c->lo_count > c->lo_cap)
-    return SEMKV_EINVAL;
-  if (c->stage_n < 0 || c->stage_n > c->block) return SEMKV_EINVAL;
-  return SEMKV_OK;
-}
 
 semkv_status from_cuda(cudaError_t e) { return e == cudaSuccess ? SEMKV_OK : SEMKV_ECUDA; }
 
@@ -362,52 +315,17 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
                                     int32_t layer, const uint16_t* q, float* out,
                                     float softmax_scale, void* ws, size_t ws_bytes,
                                     void* stream) {
-  semkv_status s = check_desc(desc);
+  semkv_status s = check_decode(desc, cache, layer, q, out);
   if (s != SEMKV_OK) return s;
-  s = check_cache(cache);
-  if (s != SEMKV_OK) return s;
-  if (!q || !out || layer < 0 || layer >= cache->layers) return SEMKV_EINVAL;
-  if (!aligned(out, 16)) return SEMKV_EALIGN;
-  if (cache->hi_count + cache->lo_count + cache->stage_n == 0) return SEMKV_EINVAL;
-  if (cache->stage_n > 0 && (!cache->stage_k || !cache->stage_v)) return SEMKV_EINVAL;
-  if (cache->stage_n > 0 && (!aligned(cache->stage_k, 8) || !aligned(cache->stage_v, 8)))
-    return SEMKV_EALIGN;
   if (!ws || !aligned(ws, 16)) return SEMKV_EWORKSPACE;
   if (ws_bytes < semkv_decode_workspace_bytes(cache)) return SEMKV_EWORKSPACE;
   const int sms = device_sm_count();
   if (sms <= 0) return SEMKV_ECUDA;
-  DecodeArgs a;
-  std::memset(&a, 0, sizeof(a));
-  a.base = desc->base;
-  a.L_hi = desc->levels_hi;
-  a.L_lo = desc->levels_lo;
-  a.B = cache->batch;
-  a.NL = cache->layers;
-  a.H = cache->kv_heads;
-  a.Hq = cache->q_heads;
-  a.layer = layer;
-  a.hi_pool = cache->hi_pool;
-  a.lo_pool = cache->lo_pool;
-  a.hi_cap = cache->hi_cap;
-  a.lo_cap = cache->lo_cap;
-  a.hi_count = cache->hi_count;
-  a.lo_count = cache->lo_count;
-  a.stage_k = cache->stage_k;
-  a.stage_v = cache->stage_v;
-  a.block = cache->block;
-  a.stage_n = cache->stage_n;
-  a.q = q;
-  a.out = out;
-  a.scale_log2 = softmax_scale * 1.4426950408889634f;
+  DecodeArgs a = decode_args(desc, cache, layer, q, out, softmax_scale);
   a.partials = reinterpret_cast<float*>(ws);
-  a.signs = desc->signs;
-  a.rot = desc->rotation;
-  a.cb_hi = desc->centroids_hi;
-  a.cb_lo = desc->centroids_lo;
   // rotated queries (TQ and rotated affine bases) after the split-K partials
   // in the workspace
   a.qrot = a.partials + (decode_workspace_floats(a.B, a.H, a.Hq) - (size_t)a.B * a.Hq * 128);
-  a.err = cache->dev_error;
   a.plan = make_decode_plan(a.base, a.L_hi, a.L_lo, a.B, a.H, a.hi_count, a.lo_count, a.stage_n,
                             sms, kMaxPartialsPerPair);
   return from_cuda(launch_decode_attention(a, (cudaStream_t)stream));

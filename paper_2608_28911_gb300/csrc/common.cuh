@@ -81,6 +81,26 @@ __device__ __forceinline__ void raise_error(int32_t* err, int32_t code) {
   if (err) atomicCAS(err, 0, code);
 }
 
+// Bounded mbarrier wait, the one every kernel uses: polls the barrier's phase at most
+// `polls` times and returns false if it never completed, so a copy that never lands
+// cannot hang a kernel (the caller records kDevWaitTimeout and returns).
+constexpr uint32_t kWaitPolls = 1u << 22;
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity,
+                                                  uint32_t polls = kWaitPolls) {
+  const uint32_t addr = (uint32_t)__cvta_generic_to_shared(bar);
+  for (uint32_t i = 0; i < polls; ++i) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(addr), "r"(parity)
+        : "memory");
+    if (ok) return true;
+  }
+  return false;
+}
+
 // Kernel attributes (the opt-in dynamic shared memory size) are per device: set() runs
 // the first time a launcher is called on each device.
 constexpr int kAttrDevices = 64;

@@ -24,8 +24,9 @@
 //    carries a share of digit k+1, scaled by a power of two and split into fp16 hi
 //    and lo rows; logit = scale log2e (s acc + z sum q).  The output fragment is
 //    the B operand of the PV product as it stands (at most one exchange of halves).
-//  - softmax in base 2 against a per-head reference exponent e that keeps p and
-//    p * s_v below 2^14; e moves, and the running sums are rescaled, only when a tile
+//  - softmax in base 2 against a per-head reference exponent e that keeps
+//    P' = p * s_v below 2^14 (the largest near 2^12) and p below 2^52; e moves, and
+//    the running sums are rescaled, only when a tile
 //    would exceed that bound.
 //  - P V as O^T = C^T P'^T (M = 128 dims, N = 8 columns, K = 16 tokens) on the digits
 //    c_k (formed lane-wise as F_k - L F_{k-1} in f16x2), with P' = p * s_v as fp16
@@ -60,7 +61,7 @@ constexpr int kAqBytes = 8 * 32 * 16;   // q-coefficient A fragments: 8 k-steps 
 constexpr int kCtasAffine = 2;          // resident CTAs per SM: affine pools / other sources
 constexpr int kCtasOther = 2;
 constexpr int kMaxSplits = 64;                     // pool splits per (b, h)
-constexpr uint32_t kSpinLimit = 1u << 22;
+constexpr float kPMax = 0x1p52f;                   // bound on p = 2^(logit - e)
 
 static_assert(kStageBytes % 16 == 0, "bulk copies need 16-byte aligned stages");
 static_assert(kRingBytes >= (kWarps * 8 * 128 + 8 * 128) * 4, "merge area reuses the ring");
@@ -97,20 +98,9 @@ __device__ __forceinline__ void bulk_refill(bool pred, void* dst, const void* sr
       "r"(smem_u32(bar)), "r"(bytes), "r"(smem_u32(dst)), "l"(src)
       : "memory");
 }
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// bounded wait: false after kSpinLimit polls
+// bounded wait: false after kWaitPolls polls
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i)
-    if (mbar_try_wait(bar, parity)) return true;
-  return false;
+  return mbar_wait_bounded(bar, parity);
 }
 
 __device__ __forceinline__ void mma16816(float c[4], uint32_t a0, uint32_t a1, uint32_t a2,
@@ -500,7 +490,7 @@ struct Shared {
 //   largest is near 2^13 and split into fp16 hi (row g) and lo (row g+8) parts.  The
 //   output fragment (rows = heads, columns = tokens 2t, 2t+1) is, after adding hi and
 //   lo, already laid out as the B fragment the PV product needs: no transposition.
-//  p = 2^(logit - e) with a per-head reference e chosen so p and p*s_v stay <= 2^14:
+//  p = 2^(logit - e) with a per-head reference e chosen so p*s_v stays <= 2^14 and p <= 2^52:
 //   e moves (and the sums are rescaled) only when a tile would exceed that.
 //  O^T += C^T P'^T (M = 128 V rows, K = 16 tokens) with P' = p*s_v as fp16 hi + lo
 //   (PACKED: columns 0..3 hi and 4..7 lo of heads 0..3; else two passes).
@@ -689,14 +679,17 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
       }
       p[i] = valid[i] ? ex2(lg[i] - st.e) : 0.0f;
       P[i] = p[i] * sv[i];
-      bad |= !(p[i] <= 16384.0f) || !(fabsf(P[i]) <= 16384.0f);
+      bad |= !(p[i] <= kPMax) || !(fabsf(P[i]) <= 16384.0f);
     }
     if (__any_sync(0xffffffffu, bad)) {
-      // move e up to (max over the head's tokens of logit + log2 max(s_v, 1)) - 12
+      // move e up to (max over the head's tokens of logit + log2 max(s_v, 2^-40)) - 12:
+      // the largest P' lands near 2^12, well inside fp16's normal range even when the
+      // value rows' steps are tiny, and p stays below 2^52 so the fp32 sums of p and
+      // p z_v cannot overflow
       float mx = -INFINITY;
 #pragma unroll
       for (int i = 0; i < NT; ++i)
-        if (valid[i]) mx = fmaxf(mx, lg[i] + fmaxf(0.0f, __log2f(fabsf(sv[i]))));
+        if (valid[i]) mx = fmaxf(mx, lg[i] + fmaxf(-40.0f, __log2f(fabsf(sv[i]))));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
       if (PACKED) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
@@ -1647,9 +1640,11 @@ DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int64_t 
     int64_t per = (total + target - 1) / target;
     const int64_t min_work = (int64_t)(p.w_hi > p.w_lo ? p.w_hi : p.w_lo) * kWarps * 2;
     if (per < min_work) per = min_work;
-    // a segment of length x meets at most x / per + 2 CTAs: keep a pair's partials
-    // (hi + lo + stage) within max_stride
-    const int64_t avail = (int64_t)max_stride - st - 4;
+    // A pair's weighted range of length W meets at most ceil(W / per) + 1 CTA ranges,
+    // and the hi | lo boundary splits at most one of those pieces in two: the pair
+    // writes at most ceil(W / per) + 2 pool partials.  Keep them, plus the stage's,
+    // within max_stride: ceil(W / per) <= max_stride - st - 2.
+    const int64_t avail = (int64_t)max_stride - st - 2;
     if (avail < 1) {
       p.per = per;
       p.ctas = 0;

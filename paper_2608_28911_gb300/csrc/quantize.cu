@@ -27,7 +27,6 @@ namespace semkv {
 namespace {
 
 constexpr int kWarpsPerBlock = 8;
-constexpr uint32_t kSpinLimitQ = 1u << 22;  // bounded mbarrier polls
 constexpr int kMaxRecWords = 27;  // largest record: affine L=7/8, 2*48+8 = 104 B
 
 // ------------------------------------------------- affine pools, by slot -----
@@ -463,17 +462,7 @@ __device__ __forceinline__ void dbar_init(uint64_t* bar) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(dsmem_u32(bar)) : "memory");
 }
 __device__ __forceinline__ bool dbar_wait(uint64_t* bar, uint32_t parity) {
-  for (uint32_t i = 0; i < kSpinLimitQ; ++i) {
-    uint32_t r;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-        " selp.u32 %0, 1, 0, p;\n}"
-        : "=r"(r)
-        : "r"(dsmem_u32(bar)), "r"(parity)
-        : "memory");
-    if (r) return true;
-  }
-  return false;
+  return mbar_wait_bounded(bar, parity);
 }
 
 // Persistent CTAs over the blocks (64 slots of one pool of one (sequence, layer, KV

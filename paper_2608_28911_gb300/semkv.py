@@ -96,6 +96,8 @@ def _load():
                                                  ctypes.POINTER(CacheStruct), i32, p, p,
                                                  ctypes.c_float, p]
     L.semkv_decode_attention_noalloc.restype = ctypes.c_int
+    L.semkv_debug_wait_timeout.argtypes = [p, u32, p]
+    L.semkv_debug_wait_timeout.restype = ctypes.c_int
     L.semkv_status_string.argtypes = [ctypes.c_int]
     L.semkv_status_string.restype = ctypes.c_char_p
     return L
@@ -106,7 +108,7 @@ EXPORTED = ["semkv_row_bytes", "semkv_record_bytes", "semkv_high_count_floor",
             "semkv_block_high_count", "semkv_lloyd_max_gaussian", "semkv_rank_workspace_bytes",
             "semkv_rank_assign", "semkv_score_kv_norm", "semkv_fake_quant", "semkv_quantize_pack", "semkv_append_block",
             "semkv_decode_workspace_bytes", "semkv_decode_attention",
-            "semkv_decode_attention_noalloc", "semkv_status_string"]
+            "semkv_decode_attention_noalloc", "semkv_debug_wait_timeout", "semkv_status_string"]
 
 
 def _ptr(t):
@@ -222,6 +224,13 @@ def semkv_decode_attention_noalloc(desc: "QuantDesc", cache: "KVCache", layer: i
            LIB.semkv_decode_attention_noalloc(ctypes.byref(desc.s), ctypes.byref(cache.s), layer,
                                               _ptr(q), _ptr(out), softmax_scale,
                                               _stream(stream)))
+
+
+def semkv_debug_wait_timeout(dev_error: torch.Tensor, polls: int, stream=None):
+    """Run the kernels' bounded mbarrier wait on a barrier nothing arrives on, giving up
+    after `polls` polls: the wait reports a timeout (1) in dev_error (device int32)."""
+    _check("semkv_debug_wait_timeout",
+           LIB.semkv_debug_wait_timeout(_ptr(dev_error), polls, _stream(stream)))
 
 
 # ------------------------------------------------------- owning wrappers ------

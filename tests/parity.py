@@ -133,9 +133,13 @@ class Pair:
         oc.hi_pool[..., :oc.hi_count, :] = self.cache.hi_pool.cpu().numpy()[..., :oc.hi_count, :]
         oc.lo_pool[..., :oc.lo_count, :] = self.cache.lo_pool.cpu().numpy()[..., :oc.lo_count, :]
 
-    def decode(self, layer=0, qseed=0, heads=None):
+    def decode(self, layer=0, qseed=0, heads=None, q=None):
+        """Decode through the C ABI and through the oracle on the same queries (drawn
+        from the seeded stream unless `q`, fp16 [B][Hq][128], is given)."""
         torch, semkv = self.torch, self.semkv
-        q = synthetic.queries(self.seed + 100 * qseed, self.B, self.Hq)
+        if q is None:
+            q = synthetic.queries(self.seed + 100 * qseed, self.B, self.Hq)
+        q = np.ascontiguousarray(q, dtype=np.float16)
         # the output sits between two canary regions that must come back untouched
         n, pad, canary = self.B * self.Hq * 128, 64, -1234.5
         big = torch.full((n + 2 * pad,), canary, dtype=torch.float32, device=self.dev)
@@ -149,6 +153,19 @@ class Pair:
         assert np.all(g[:pad] == canary) and np.all(g[pad + n:] == canary), "decode wrote past out"
         ref = oracle.decode_attention(self.oc, layer, synthetic.f16_bits(q), scale, heads=heads)
         return g[pad:pad + n].reshape(self.B, self.Hq, 128), ref
+
+    def stage(self, k, v, s):
+        """Stage tokens (fp16 k, v [B][NL][H][n][128], scores [B][n]) into the GPU cache
+        and the oracle's, one at a time (Algorithm 2's per-token step)."""
+        torch = self.torch
+        for g in range(k.shape[3]):
+            kg = np.ascontiguousarray(k[:, :, :, g], dtype=np.float16)
+            vg = np.ascontiguousarray(v[:, :, :, g], dtype=np.float16)
+            sg = np.ascontiguousarray(s[:, g], dtype=np.float32)
+            self.cache.stage_token(torch.from_numpy(kg).to(self.dev),
+                                   torch.from_numpy(vg).to(self.dev),
+                                   torch.from_numpy(sg).to(self.dev))
+            oracle.stage_token(self.oc, synthetic.f16_bits(kg), synthetic.f16_bits(vg), sg)
 
     def assert_untouched_past_counts(self):
         """Canaries: the pools were zero-filled and the slot maps filled with -1 when the
