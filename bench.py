@@ -754,7 +754,8 @@ def main():
         "fake_quant_gbs": r["fake_gbs"],
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": profiled_traffic(args.config),
-                     "kernel": {0: "decode_affine_kernel + combine_wide_kernel", 2: "qrot_kernel + decode_affine_kernel + combine_wide_kernel",
+                     "kernel": {0: "decode_affine_fast_kernel + combine_wide_kernel",
+                                2: "qrot_kernel + decode_affine_fast_kernel + combine_wide_kernel",
                                 1: "qrot_kernel + decode_kernel<1> + combine_wide_kernel",
                                 3: "qrot_dense_kernel + decode_kernel<1> + combine_kernel<dense>"}[cfg["base"]]
                                + " (semkv_decode_attention)",

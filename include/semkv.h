@@ -236,7 +236,7 @@ semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache
  * ws: device workspace of semkv_decode_workspace_bytes(cache) bytes, 16-B aligned.
  * Accuracy: against fp64 attention over the same dequantized cache, max-abs error
  * <= 2e-3 and relative L2 <= 1e-3 for values of magnitude below 64; binary32 carries
- * relative error, so for larger values the absolute error grows as about 1e-6 *
+ * relative error, so for larger values the absolute error grows as up to 8e-6 *
  * max|v^| (all of fp16's range, including subnormal steps, is supported). */
 size_t semkv_decode_workspace_bytes(const semkv_cache* cache);
 semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_cache* cache,

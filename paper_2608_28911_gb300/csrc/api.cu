@@ -326,7 +326,7 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
   // rotated queries (TQ and rotated affine bases) after the split-K partials
   // in the workspace
   a.qrot = a.partials + (decode_workspace_floats(a.B, a.H, a.Hq) - (size_t)a.B * a.Hq * 128);
-  a.plan = make_decode_plan(a.base, a.L_hi, a.L_lo, a.B, a.H, a.hi_count, a.lo_count, a.stage_n,
+  a.plan = make_decode_plan(a.base, a.L_hi, a.L_lo, a.B, a.H, a.Hq, a.hi_count, a.lo_count, a.stage_n,
                             sms, kMaxPartialsPerPair);
   return from_cuda(launch_decode_attention(a, (cudaStream_t)stream));
 }

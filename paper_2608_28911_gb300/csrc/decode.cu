@@ -39,6 +39,13 @@
 //
 // Per warp: a 4-deep ring of cp.async.bulk tile copies completing on per-stage
 // mbarriers (bounded waits that report a timeout in the error word).
+//
+// The description above is that of decode_affine_kernel, which serves every level
+// count and GQA group size.  Five- and six-level affine pools with groups of up to
+// four heads (the workloads' shape) run decode_affine_fast_kernel instead: the same
+// plan, ring and merge, with S^T = F Q'^T (eight MMAs per tile, the coefficients in
+// B fragments), five-level digits on the f16x2 FMA pipe, and the softmax in packed
+// binary32 (see "affine pools: fast path" below).
 #include <float.h>
 
 #include <cstring>
@@ -58,8 +65,10 @@ constexpr int kMaxRec = 104;
 constexpr int kStageBytes = kTile * kMaxRec + 16;  // +16: window loads may run 12 B past a tile
 constexpr int kRingBytes = kWarps * kStages * kStageBytes;
 constexpr int kAqBytes = 8 * 32 * 16;   // q-coefficient A fragments: 8 k-steps x 32 lanes x uint4
+constexpr int kQbBytes = 8 * 32 * 8;    // fast path: coefficient B fragments, 8 steps x 32 lanes x uint2
 constexpr int kCtasAffine = 2;          // resident CTAs per SM: affine pools / other sources
 constexpr int kCtasOther = 2;
+constexpr int kCtasFast = 2;           // resident CTAs per SM: the fast affine path (127 registers)
 constexpr int kMaxSplits = 64;                     // pool splits per (b, h)
 constexpr float kPMax = 0x1p52f;                   // bound on p = 2^(logit - e)
 
@@ -789,6 +798,402 @@ __device__ void run_pool(const DecodeArgs& a, const Shared& sh, uint8_t* ring, u
   ring_it += nmine;
 }
 
+// ==================================================== affine pools: fast path =====
+// Five- and six-level affine pools with GQA groups of up to four heads (the shape of
+// the paper's models and of every workload here), in a kernel of its own so that it
+// gets its own register budget (decode_affine_fast_kernel).
+//
+// S^T = F Q'^T on m16n8k16: M = the tile's 16 tokens, N = 8 columns (column 2h holds
+// the hi part of head h's coefficients, 2h + 1 the lo part), K = 16 F slots per step,
+// 8 steps: eight MMAs per tile.  Lane (g, t) supplies the F values of quarter t of
+// tokens g and g + 8 (A fragment) and the coefficients of head g>>1, part g&1, for the
+// same slots (B fragment: 16 registers built once per segment, no per-tile loads); its
+// output holds the logits of tokens g and g + 8 for head t.  The softmax runs on those
+// two logits per lane; four shuffles and two byte permutes hand P' = p s_v to the
+// lanes that hold it in the PV product's B fragment.
+//
+// Five-level symbols are decoded on the f16x2 FMA pipe.  The mask that extracts a
+// pair of symbols also lays the fp16 exponent of 1024 over them, giving the halves
+// B = 1024 + beta.  fma(B, 5^(k+1)/128, 1025.5 - 1024 * 5^(k+1)/128) is then
+// 1026 + F_k + (f - 1/2) before rounding, f the fraction of beta 5^(k+1)/128: a
+// multiple of 1/128, nonzero unless beta = 0 (5 is prime to 128).  So it rounds to
+// 1026 + F_k: for f > 0 the offset f - 1/2 lies strictly inside (-1/2, 1/2), and for
+// beta = 0 the tie 1025.5 goes to the even 1026.  Subtracting 1026 leaves F_k.  (Every
+// constant is exact in fp16; the values stay in [1024, 2048), where fp16's step is 1.)
+// Six-level symbols keep the binary32 multiplies of Dec<6> (their 13-bit symbols do
+// not fit fp16's 11 bits).
+
+__device__ __forceinline__ uint32_t hfma2u(uint32_t a, uint32_t b, uint32_t c) {
+  uint32_t r;
+  asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(c));
+  return r;
+}
+// x - 1026 on both halves
+__device__ __forceinline__ uint32_t hsub1026(uint32_t x) {
+  uint32_t r;
+  asm("add.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(x), "r"(0xE402E402u));
+  return r;
+}
+// (x & m) | ov in one LOP3: ov (the fp16 exponent of 1024 in both halves) comes from a
+// register the caller made once, so the two constants never both need an immediate
+__device__ __forceinline__ uint32_t and_or(uint32_t x, uint32_t m, uint32_t ov) {
+  uint32_t r;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(r) : "r"(x), "r"(m), "r"(ov));
+  return r;
+}
+__device__ __forceinline__ uint32_t overlay1024() {
+  uint32_t ov;
+  asm volatile("mov.b32 %0, 0x64006400;" : "=r"(ov));
+  return ov;
+}
+
+// fp16 constants of the five-level digit fmas: 5^(k+1)/128 and 1025.5 - 1024 5^(k+1)/128
+__host__ __device__ constexpr uint32_t l5_mul(int k) {
+  return k == 0 ? 0x29002900u : k == 1 ? 0x32403240u : 0x3BD03BD0u;
+}
+__host__ __device__ constexpr uint32_t l5_add(int k) {
+  return k == 0 ? 0x63B363B3u : k == 1 ? 0x62736273u : 0x4E604E60u;
+}
+// the two-code tail (5 bits): F_0 = floor(beta 5/32), F_1 = floor(beta 25/32)
+constexpr uint32_t kL5TMul0 = 0x31003100u, kL5TAdd0 = 0x62C362C3u;
+constexpr uint32_t kL5TMul1 = 0x3A403A40u, kL5TAdd1 = 0x5B0C5B0Cu;
+constexpr uint32_t kL5TMulK = 0x3A403100u, kL5TAddK = 0x5B0C62C3u;  // F_0 low, F_1 high
+
+// B = 1024 + beta pairs of five symbols: symbol j (bits 7j) of the window (a0, a1)
+// in the low half and of the window (b0, b1) in the high half
+__device__ __forceinline__ void l5_pairsB(uint32_t a0, uint32_t a1, uint32_t b0, uint32_t b1,
+                                          uint32_t ov, uint32_t (&B)[5]) {
+  const uint32_t C = fpair(a0, b0);                                 // bits 0..15 of each
+  B[0] = and_or(C, kM7, ov);
+  B[1] = and_or(C >> 7, kM7, ov);
+  B[2] = and_or(__byte_perm(a0, b0, 0x6521) >> 6, kM7, ov);         // bits 8..23, >> 6
+  B[3] = and_or(__byte_perm(a0, b0, 0x7632) >> 5, kM7, ov);         // bits 16..31, >> 5
+  B[4] = and_or(fpair(__funnelshift_r(a0, a1, 28), __funnelshift_r(b0, b1, 28)), kM7, ov);
+}
+
+// K side: the B pairs of one quarter (symbols s and s + 5, 35 bits apart) and its tail
+// (in both halves).  Register p of the quarter's A-fragment halves: p < 15: F_(p%3)
+// of symbols p/3 (low half) and p/3 + 5 (high half); p = 15: the tail's F_0, F_1.
+__device__ __forceinline__ void k5_B(const Window& w, uint32_t ov, uint32_t (&B)[5], uint32_t& Bt) {
+  l5_pairsB(w.q0, w.q1, __funnelshift_r(w.q1, w.q2, 3), w.q2 >> 3, ov, B);
+  Bt = ((w.q2 >> 6) & 0x1Fu) * 0x00010001u + 0x64006400u;          // quarter bits 70..74
+}
+__device__ __forceinline__ uint32_t k5_reg(const uint32_t (&B)[5], uint32_t Bt, int p) {
+  return p < 15 ? hsub1026(hfma2u(B[p / 3], l5_mul(p % 3), l5_add(p % 3)))
+                : hsub1026(hfma2u(Bt, kL5TMulK, kL5TAddK));
+}
+// V side: the B pairs (tokens of wa low, wb high) of lane group g's half quarter and
+// the pair of its tail symbols (70 bits on for half 0, 35 for half 1); the digits of
+// one symbol; the tail's digit hh (F_hh - 5 hh F_0)
+__device__ __forceinline__ void v5_B(const Window& wa, const Window& wb, int hh, uint32_t ov,
+                                     uint32_t (&B)[5], uint32_t& Bt) {
+  l5_pairsB(wa.q0, wa.q1, wb.q0, wb.q1, ov, B);
+  const uint32_t ta = hh ? (wa.q1 >> 3) : (wa.q2 >> 6);
+  const uint32_t tb = hh ? (wb.q1 >> 3) : (wb.q2 >> 6);
+  Bt = and_or(fpair(ta, tb), 0x001F001Fu, ov);
+}
+__device__ __forceinline__ void v5_digits(uint32_t B, uint32_t& d0, uint32_t& d1, uint32_t& d2) {
+  const uint32_t F0 = hsub1026(hfma2u(B, l5_mul(0), l5_add(0)));
+  const uint32_t F1 = hsub1026(hfma2u(B, l5_mul(1), l5_add(1)));
+  const uint32_t F2 = hsub1026(hfma2u(B, l5_mul(2), l5_add(2)));
+  d0 = F0;
+  d1 = hdigit<5>(F0, F1);
+  d2 = hdigit<5>(F1, F2);
+}
+__device__ __forceinline__ uint32_t v5_tail(uint32_t Bt, uint32_t tmul, uint32_t tadd, uint32_t tneg) {
+  const uint32_t T0 = hsub1026(hfma2u(Bt, kL5TMul0, kL5TAdd0));
+  const uint32_t Th = hsub1026(hfma2u(Bt, tmul, tadd));
+  return hfma2u(T0, tneg, Th);
+}
+
+// packed binary32 pairs (Blackwell's f32x2 arithmetic: one instruction for two lanes)
+__device__ __forceinline__ unsigned long long f2_bits(float2 v) {
+  return (unsigned long long)__float_as_uint(v.x) | ((unsigned long long)__float_as_uint(v.y) << 32);
+}
+__device__ __forceinline__ float2 f2_of(unsigned long long r) {
+  return make_float2(__uint_as_float((uint32_t)r), __uint_as_float((uint32_t)(r >> 32)));
+}
+__device__ __forceinline__ float2 f2_fma(float2 a, float2 b, float2 c) {
+  unsigned long long r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(f2_bits(a)), "l"(f2_bits(b)), "l"(f2_bits(c)));
+  return f2_of(r);
+}
+__device__ __forceinline__ float2 f2_mul(float2 a, float2 b) {
+  unsigned long long r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(f2_bits(a)), "l"(f2_bits(b)));
+  return f2_of(r);
+}
+__device__ __forceinline__ float2 f2_add(float2 a, float2 b) {
+  unsigned long long r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(f2_bits(a)), "l"(f2_bits(b)));
+  return f2_of(r);
+}
+__device__ __forceinline__ float2 neg_f2(float2 a) { return make_float2(-a.x, -a.y); }
+// fp16 pair (low half = x) <-> two binary32
+__device__ __forceinline__ float2 h2_to_f2(uint32_t h) {
+  return make_float2(f16_to_f32((uint16_t)(h & 0xFFFFu)), f16_to_f32((uint16_t)(h >> 16)));
+}
+__device__ __forceinline__ uint32_t f2_to_h2(float2 v) { return pack_h2(v.x, v.y); }
+
+struct FastState {
+  float O[8][4];  // O^T accumulators: V rows x columns 2t, 2t+1
+  float e;        // reference exponent of head t (base 2)
+  float l, l2;    // partial sums of p over this lane's tokens g and g + 8 of head t
+  float zs, zs2;  // partial sums of p z_v
+};
+
+__device__ __forceinline__ void fast_init(FastState& st) {
+#pragma unroll
+  for (int m = 0; m < 8; ++m)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) st.O[m][i] = 0.0f;
+  st.e = -INFINITY;
+  st.l = st.l2 = 0.0f;
+  st.zs = st.zs2 = 0.0f;
+}
+
+// the power-of-two scale that brings head coefficients near 2^13
+__device__ __forceinline__ float coef_scale(float qmax, int L) {
+  return qmax > 0.0f ? pow2_floor(fminf(8192.0f / ((float)(L + 1) * qmax), 1e30f)) : 1.0f;
+}
+
+// One warp streams its tiles of one (pair, pool) segment (see the section comment).
+// ring_it: tiles this warp has taken through its ring so far (barrier phases).
+template <int L>
+__device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint2* qbs,
+                              uint64_t* bars, const uint8_t* pool_bh, int64_t count,
+                              int t_begin, int t_end, int G, FastState& st, int& ring_it) {
+  using D = Dec<L>;
+  using F = typename D::F;
+  constexpr int kRec = 2 * F::RB + 8;
+  constexpr uint32_t kTileBytes = kTile * kRec;
+  static_assert(kTileBytes % 16 == 0, "tile size must be a multiple of 16 bytes");
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int g = lane >> 2, t = lane & 3;
+  uint8_t* my_ring = ring + warp * kStages * kStageBytes;
+  uint64_t* my_bar = bars + warp * kStages;
+  const bool rot = a.base == SEMKV_BASE_AFFINE_HAD;
+
+  // B fragments: coefficients of head g>>1 (hi part for even g, lo part for odd g) for
+  // the slots of lane (g, t), the same for every warp: warp 0 writes them to shared
+  // memory, every warp loads its lane's pair per step (one conflict-free 8-byte load)
+  __syncthreads();  // the previous segment's fragments and the merge area are no longer read
+  if (warp == 0) {
+    const int hb = g >> 1;
+    const float sc = coef_scale(sh.qmax[hb], L);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      uint32_t r[2];
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int p = 2 * j + i;
+        float c0 = 0.0f, c1 = 0.0f;
+        if (hb < G) {
+          if (rot) {
+            c0 = k_coef<L>(sh.qr[hb], t, p, 0) * sc;
+            c1 = k_coef<L>(sh.qr[hb], t, p, 1) * sc;
+          } else {
+            c0 = k_coef<L>(sh.q[hb], t, p, 0) * sc;
+            c1 = k_coef<L>(sh.q[hb], t, p, 1) * sc;
+          }
+        }
+        uint32_t hi, lo;
+        split_h2(c0, c1, hi, lo);
+        r[i] = (g & 1) ? lo : hi;
+      }
+      qbs[32 * j + lane] = make_uint2(r[0], r[1]);
+    }
+  }
+  __syncthreads();
+  const uint2* qb = qbs + lane;
+  // logits of head t
+  const bool live = t < G;
+  const float cS = a.scale_log2 / coef_scale(sh.qmax[t], L);
+  const float cZ = a.scale_log2 * sh.sumq[t];
+  // O columns 2t, 2t+1 belong to heads (2t)&3, (2t+1)&3, whose e lives in lanes 0..3
+  const int oh0 = (2 * t) & 3, oh1 = oh0 + 1;
+  // P' hand-over: this lane's PV column g is head g&3, part g>>2; its rows are tokens
+  // 2t, 2t+1 (lanes 8t + (g&3), + 4) and 2t+8, 2t+9
+  const int srcX = 8 * t + (g & 3), srcY = srcX + 4;
+  const uint32_t psel = (g >> 2) ? 0x7632u : 0x5410u;
+  // V half quarter of lane group g, and its tail digit's constants
+  const int qv = g >> 1, hh = g & 1;
+  const int vpos = 8 * F::RB + qv * F::QB + hh * D::kHalf * F::W;
+  const int tpos = F::NG * F::W - hh * D::kHalf * F::W;
+  const uint32_t tmul = hh ? kL5TMul1 : kL5TMul0, tadd = hh ? kL5TAdd1 : kL5TAdd0;
+  const uint32_t tneg = hh ? 0xC500C500u : 0u;
+  const uint32_t ov = overlay1024();
+  const int kpos = t * F::QB;
+
+  const int nmine = t_end - t_begin <= warp ? 0 : (t_end - t_begin - warp + kWarps - 1) / kWarps;
+  // tokens left in the pool from this warp's current tile on (a pool holds fewer than
+  // 2^31 slots), the source of the refill kStages tiles ahead, the ring position
+  int left = (int)count - (t_begin + warp) * kTile;
+  const uint8_t* refill_src = pool_bh + (int64_t)(t_begin + warp + kStages * kWarps) * kTileBytes;
+  int stage = ring_it % kStages;
+  uint32_t phase = (uint32_t)((ring_it / kStages) & 1);
+  bool ok = true;
+  int it = 0;
+  for (; it < nmine; ++it) {
+    if (!mbar_wait(&my_bar[stage], phase)) {
+      ok = false;
+      break;
+    }
+    const uint8_t* tb = my_ring + stage * kStageBytes;
+    const int nvalid = min(kTile, left);
+
+    // ---- S^T = F Q'^T: tokens g (rows g) and g + 8, heads in column pairs
+    float s[4] = {0.f, 0.f, 0.f, 0.f};
+    {
+      if constexpr (L == 5) {
+        uint32_t Ba[5], Bb[5], Ta, Tb;
+        k5_B(load_window(tb + g * kRec, kpos), ov, Ba, Ta);
+        k5_B(load_window(tb + (g + 8) * kRec, kpos), ov, Bb, Tb);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+        {
+          const uint2 c = qb[32 * j];
+          mma16816(s, k5_reg(Ba, Ta, 2 * j), k5_reg(Bb, Tb, 2 * j), k5_reg(Ba, Ta, 2 * j + 1),
+                   k5_reg(Bb, Tb, 2 * j + 1), c.x, c.y);
+        }
+      } else {
+        uint32_t fa[8][2], fb[8][2];
+        k_quarter<L>(load_window(tb + g * kRec, kpos), fa);
+        k_quarter<L>(load_window(tb + (g + 8) * kRec, kpos), fb);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+        {
+          const uint2 c = qb[32 * j];
+          mma16816(s, fa[j][0], fb[j][0], fa[j][1], fb[j][1], c.x, c.y);
+        }
+      }
+    }
+    // ---- softmax of head t over tokens g and g + 8
+    const uint32_t* pr0 = reinterpret_cast<const uint32_t*>(tb + g * kRec + 2 * F::RB);
+    const uint32_t* pr1 = reinterpret_cast<const uint32_t*>(tb + (g + 8) * kRec + 2 * F::RB);
+    const bool v0 = live && g < nvalid, v1 = live && g + 8 < nvalid;
+    const uint32_t kp0 = pr0[0], kp1 = pr1[0];
+    // rows past the pool's count are not data: keep whatever they hold out of the sums
+    const uint32_t vp0 = v0 ? pr0[1] : 0u, vp1 = v1 ? pr1[1] : 0u;
+    // both tokens at once in packed binary32 (x: token g, y: token g + 8)
+    const float2 k0 = h2_to_f2(kp0), k1 = h2_to_f2(kp1), vv0 = h2_to_f2(vp0), vv1 = h2_to_f2(vp1);
+    const float2 lg = f2_fma(f2_mul(make_float2(k0.x, k1.x), make_float2(cS, cS)),
+                             make_float2(s[0] + s[1], s[2] + s[3]),
+                             f2_mul(make_float2(k0.y, k1.y), make_float2(cZ, cZ)));
+    const float2 sv = make_float2(vv0.x, vv1.x), zv = make_float2(vv0.y, vv1.y);
+    float2 dl = f2_add(lg, make_float2(-st.e, -st.e));
+    float2 p = make_float2(v0 ? ex2(dl.x) : 0.0f, v1 ? ex2(dl.y) : 0.0f);
+    float2 P = f2_mul(p, sv);
+    const bool bad = !(fmaxf(p.x, p.y) <= kPMax) || !(fmaxf(fabsf(P.x), fabsf(P.y)) <= 16384.0f);
+    if (__any_sync(0xffffffffu, bad)) {
+      // e of each head moves up to (max over its tokens of logit + log2 max(s_v, 2^-40))
+      // - 12: the largest P' lands near 2^12, p stays below 2^52
+      float mx = -INFINITY;
+      if (v0) mx = lg.x + fmaxf(-40.0f, __log2f(fabsf(sv.x)));
+      if (v1) mx = fmaxf(mx, lg.y + fmaxf(-40.0f, __log2f(fabsf(sv.y))));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+      const float e_new = fmaxf(st.e, mx - 12.0f);
+      const float al = st.e == -INFINITY ? 0.0f : ex2(st.e - e_new);
+      st.e = e_new;
+      st.l *= al;
+      st.l2 *= al;
+      st.zs *= al;
+      st.zs2 *= al;
+      const float a0 = __shfl_sync(0xffffffffu, al, oh0);
+      const float a1 = __shfl_sync(0xffffffffu, al, oh1);
+#pragma unroll
+      for (int m = 0; m < 8; ++m) {
+        st.O[m][0] *= a0;
+        st.O[m][1] *= a1;
+        st.O[m][2] *= a0;
+        st.O[m][3] *= a1;
+      }
+      dl = f2_add(lg, make_float2(-st.e, -st.e));
+      p = make_float2(v0 ? ex2(dl.x) : 0.0f, v1 ? ex2(dl.y) : 0.0f);
+      P = f2_mul(p, sv);
+    }
+    {
+      // the two tokens' sums stay apart (l, l2 and zs, zs2) so one packed op adds both
+      const float2 l2 = f2_add(make_float2(st.l, st.l2), p);
+      const float2 z2 = f2_fma(p, zv, make_float2(st.zs, st.zs2));
+      st.l = l2.x;
+      st.l2 = l2.y;
+      st.zs = z2.x;
+      st.zs2 = z2.y;
+    }
+    // ---- P'^T as the PV product's B fragment (rows = tokens, column g)
+    uint32_t b0, b1;
+    {
+      // fp16 hi and lo parts of both tokens' P', then (hi, lo) per token
+      const uint32_t hp = f2_to_h2(P);
+      const float2 lo = f2_add(P, neg_f2(h2_to_f2(hp)));
+      const uint32_t lp = f2_to_h2(lo);
+      const uint32_t W0 = __byte_perm(hp, lp, 0x5410), W1 = __byte_perm(hp, lp, 0x7632);
+      const uint32_t x0 = __shfl_sync(0xffffffffu, W0, srcX);
+      const uint32_t x1 = __shfl_sync(0xffffffffu, W1, srcX);
+      const uint32_t y0 = __shfl_sync(0xffffffffu, W0, srcY);
+      const uint32_t y1 = __shfl_sync(0xffffffffu, W1, srcY);
+      b0 = __byte_perm(x0, y0, psel);
+      b1 = __byte_perm(x1, y1, psel);
+    }
+    // ---- O^T += C^T P'^T
+    {
+      const Window w0 = load_window(tb + (2 * t) * kRec, vpos);
+      const Window w1 = load_window(tb + (2 * t + 1) * kRec, vpos);
+      const Window w2 = load_window(tb + (2 * t + 8) * kRec, vpos);
+      const Window w3 = load_window(tb + (2 * t + 9) * kRec, vpos);
+      if constexpr (L == 5) {
+        // symbol by symbol: after symbol j, rows 0 .. 3j + 2 are ready and the m-blocks
+        // up to (3j + 1) / 2 go to the tensor cores
+        uint32_t B0[5], B1[5], T0, T1;
+        v5_B(w0, w1, hh, ov, B0, T0);
+        v5_B(w2, w3, hh, ov, B1, T1);
+        uint32_t r0[16], r1[16];
+#pragma unroll
+        for (int j = 0; j < 5; ++j) {
+          v5_digits(B0[j], r0[3 * j], r0[3 * j + 1], r0[3 * j + 2]);
+          v5_digits(B1[j], r1[3 * j], r1[3 * j + 1], r1[3 * j + 2]);
+#pragma unroll
+          for (int m = (3 * j - 2 < 0 ? 0 : (3 * j - 2) / 2 + 1); m <= (3 * j + 1) / 2; ++m)
+            mma16816(st.O[m], r0[2 * m], r0[2 * m + 1], r1[2 * m], r1[2 * m + 1], b0, b1);
+        }
+        r0[15] = v5_tail(T0, tmul, tadd, tneg);
+        r1[15] = v5_tail(T1, tmul, tadd, tneg);
+        mma16816(st.O[7], r0[14], r0[15], r1[14], r1[15], b0, b1);
+      } else {
+        uint32_t VA[8][4];
+        v_half_pair<L, 0>(w0, w1, tpos, hh, VA);
+        v_half_pair<L, 2>(w2, w3, tpos, hh, VA);
+#pragma unroll
+        for (int m = 0; m < 8; ++m)
+          mma16816(st.O[m], VA[m][0], VA[m][1], VA[m][2], VA[m][3], b0, b1);
+      }
+    }
+    __syncwarp();
+    // the stage is free again: lane 0 starts the copy of the tile kStages ahead
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    bulk_refill(lane == 0 && it + kStages < nmine, my_ring + stage * kStageBytes, refill_src,
+                kTileBytes, &my_bar[stage]);
+    refill_src += (int64_t)kWarps * kTileBytes;
+    left -= kWarps * kTile;
+    if (++stage == kStages) {
+      stage = 0;
+      phase ^= 1u;
+    }
+  }
+  if (!ok) {
+    // a copy never completed: record it, give the copies still in flight a bounded
+    // chance to land, and drop this warp's contribution
+    if (lane == 0) raise_error(a.err, kDevWaitTimeout);
+    for (int j = it; j < nmine && j < it + kStages; ++j)
+      mbar_wait(&my_bar[(ring_it + j) % kStages], (uint32_t)(((ring_it + j) / kStages) & 1));
+    fast_init(st);
+  }
+  ring_it += nmine;
+}
+
 // ------------------------------------------------- TurboQuant-MSE records -----
 // Dequantized rows are x^ = (n/128) S H cb[c] (Sec. 4.9), so q . x^ = (n/128) q' . cb[c]
 // with q' = H S q, and sum p x^ = S H (sum p (n/128) cb[c]): scores and the weighted
@@ -1312,6 +1717,112 @@ __global__ void __launch_bounds__(kThreads, kCtasAffine) decode_affine_kernel(De
   }
 }
 
+// A fast-path warp's state into the merge area, in the layout merge_warps reads: per
+// head (e, l, zs), and O rows for columns 0..7 (columns 4..7 are the lo parts of
+// heads 0..3, folded in by merge_warps); rows 16m + g (+8) are V rows u = 2m (+1) of
+// lane group g, i.e. output dims v_dim(g, u).
+template <int L>
+__device__ void fast_rows(FastState& st, int G, MergeArea& mg, float* merge_o) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int g = lane >> 2, t = lane & 3;
+  // l and zs of head t: both tokens' sums of the lanes 4g + t for every g
+  st.l += st.l2;
+  st.zs += st.zs2;
+#pragma unroll
+  for (int off = 4; off <= 16; off <<= 1) {
+    st.l += __shfl_xor_sync(0xffffffffu, st.l, off);
+    st.zs += __shfl_xor_sync(0xffffffffu, st.zs, off);
+  }
+  __syncthreads();  // every warp is done with the ring: reuse it as the merge area
+  if (g == 0 && t < G) {
+    mg.m[warp * 8 + t] = st.e;
+    mg.l[warp * 8 + t] = st.l;
+    mg.z[warp * 8 + t] = st.zs;
+  }
+#pragma unroll
+  for (int c = 0; c < 2; ++c) {
+    const int col = 2 * t + c;
+    if ((col & 3) < G) {
+#pragma unroll
+      for (int m = 0; m < 8; ++m)
+#pragma unroll
+        for (int r = 0; r < 2; ++r)
+          merge_o[(warp * 8 + col) * 128 + v_dim<L>(g, 2 * m + r)] = st.O[m][2 * r + c];
+    }
+  }
+}
+
+
+template <int L>
+__device__ __forceinline__ void run_fast_l(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
+                                           uint2* qbs, uint64_t* bars, const uint8_t* pool_bh,
+                                           int64_t count, int t0, int t1, int G, FastState& st,
+                                           int& ring_it, MergeArea& mg, float* merge_o) {
+  run_pool_fast<L>(a, sh, ring, qbs, bars, pool_bh, count, t0, t1, G, st, ring_it);
+  fast_rows<L>(st, G, mg, merge_o);
+}
+
+// The balanced plan of decode_affine_kernel, run by the fast path: CTA c takes the
+// weighted range [c per, (c+1) per) of the concatenated [hi | lo] tile sequence of every
+// (b, h), one partial per (pair, pool) segment it touches.
+__global__ void __launch_bounds__(kThreads, kCtasFast) decode_affine_fast_kernel(DecodeArgs a) {
+  extern __shared__ __align__(128) uint8_t dyn[];
+  __shared__ Shared sh;
+  __shared__ MergeArea mg;
+  uint8_t* ring = dyn;
+  uint2* qbs = reinterpret_cast<uint2*>(dyn + kRingBytes);  // [8 steps][32 lanes]
+  float* merge_o = reinterpret_cast<float*>(dyn);  // [kWarps][8][128] rows, then [8][128]
+  const DecodePlan& P = a.plan;
+  const int G = a.Hq / a.H;
+  const int64_t pairs = (int64_t)a.B * a.H;
+  const int64_t total = pairs * P.W;
+  const int64_t start = (int64_t)blockIdx.x * P.per;
+  const int64_t end = min(start + P.per, total);
+
+  if (threadIdx.x < kWarps * kStages) mbar_init(&sh.bar[0][0] + threadIdx.x);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  __syncthreads();
+  pdl_wait();  // the records, queries and stage partial come from earlier work
+  int ring_it = 0;  // tiles this warp has taken through its ring (barrier phases)
+  int64_t loaded = -1;
+  for (int64_t bh = start / P.W; bh < pairs && bh * P.W < end; ++bh) {
+    const int b = (int)(bh / a.H), h = (int)(bh % a.H);
+    for (int src = 0; src < 2; ++src) {
+      const int tiles = src ? P.tiles_lo : P.tiles_hi;
+      const int w = src ? P.w_lo : P.w_hi;
+      const int64_t S = bh * P.W + (src ? (int64_t)P.w_hi * P.tiles_hi : 0);
+      const int64_t E = S + (int64_t)w * tiles;
+      if (E <= S || E <= start || S >= end) continue;
+      const int64_t x0 = max(start, S) - S, x1 = min(end, E) - S;
+      const int t0 = (int)((x0 + w - 1) / w);
+      const int t1 = (int)min((int64_t)tiles, (x1 + w - 1) / w);
+      int n_hi, n_lo;
+      pair_slots(P, bh, n_hi, n_lo);
+      const int slot = (int)((int64_t)blockIdx.x - S / P.per) + (src ? n_hi : 0);
+      const int L = src ? a.L_lo : a.L_hi;
+      const int64_t cap = src ? a.lo_cap : a.hi_cap;
+      const int64_t count = src ? a.lo_count : a.hi_count;
+      const uint8_t* pool = src ? a.lo_pool : a.hi_pool;
+      const int rec = record_bytes_rt(SEMKV_BASE_AFFINE, L);
+      const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
+      uint64_t* bars = &sh.bar[0][0];
+      ring_fill(ring, bars, pool_bh, (uint32_t)(kTile * rec), t0, t1, ring_it);
+      if (bh != loaded) {
+        load_group_q(a, sh, b, h, G);
+        loaded = bh;
+      }
+      FastState st;
+      fast_init(st);
+      if (L == 5)
+        run_fast_l<5>(a, sh, ring, qbs, bars, pool_bh, count, t0, t1, G, st, ring_it, mg, merge_o);
+      else
+        run_fast_l<6>(a, sh, ring, qbs, bars, pool_bh, count, t0, t1, G, st, ring_it, mg, merge_o);
+      merge_warps(a, a.base == SEMKV_BASE_AFFINE_HAD ? 3 : 0, h, G, mg, merge_o,
+                  a.partials + (bh * P.stride + slot) * kPartialFloats);
+    }
+  }
+}
+
 // TQ pools (KIND 1, one CTA per split) and the fp16 stage (KIND 2, one CTA per pair).
 template <int KIND>
 __global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs a) {
@@ -1612,7 +2123,7 @@ static int tile_cost(int L) {
   }
 }
 
-DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int64_t hi_count,
+DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int Hq, int64_t hi_count,
                             int64_t lo_count, int stage_n, int num_sms, int max_stride) {
   DecodePlan p;
   std::memset(&p, 0, sizeof(p));
@@ -1626,6 +2137,7 @@ DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int64_t 
   if (base == SEMKV_BASE_AFFINE || base == SEMKV_BASE_AFFINE_HAD) {
     // balanced: one wave of equal CTAs over the weighted tiles of every pair
     p.balanced = 1;
+    p.fast = (Hq / H <= 4 && (L_hi == 5 || L_hi == 6) && (L_lo == 5 || L_lo == 6)) ? 1 : 0;
     p.w_hi = tile_cost(L_hi);
     p.w_lo = tile_cost(L_lo);
     p.W = (int64_t)p.w_hi * p.tiles_hi + (int64_t)p.w_lo * p.tiles_lo;
@@ -1636,7 +2148,7 @@ DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int64_t 
       p.stride = st;
       return p;
     }
-    const int64_t target = (int64_t)num_sms * kCtasAffine;
+    const int64_t target = (int64_t)num_sms * (p.fast ? kCtasFast : kCtasAffine);
     int64_t per = (total + target - 1) / target;
     const int64_t min_work = (int64_t)(p.w_hi > p.w_lo ? p.w_hi : p.w_lo) * kWarps * 2;
     if (per < min_work) per = min_work;
@@ -1734,6 +2246,9 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            kRingBytes + kAqBytes);
       if (r == cudaSuccess)
+        r = cudaFuncSetAttribute(decode_affine_fast_kernel,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes + kQbBytes);
+      if (r == cudaSuccess)
         r = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kRingBytes + kAqBytes);
       if (r == cudaSuccess)
@@ -1768,7 +2283,11 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
       e = cudaGetLastError();
       if (e != cudaSuccess) return e;
     }
-    if (P.ctas > 0) {
+    if (P.ctas > 0 && P.fast) {
+      e = launch_pdl(decode_affine_fast_kernel, dim3(P.ctas), dim3(kThreads), kRingBytes + kQbBytes,
+                     stream, a);
+      if (e != cudaSuccess) return e;
+    } else if (P.ctas > 0) {
       e = launch_pdl(decode_affine_kernel, dim3(P.ctas), dim3(kThreads), kRingBytes + kAqBytes,
                      stream, a);
       if (e != cudaSuccess) return e;

@@ -92,6 +92,9 @@ struct DecodePlan {
   int64_t W;                             // weighted length of one (b, h)
   int64_t per;                           // weighted length per CTA
   int ctas;
+  // affine pools with five- and six-level codes and GQA groups of up to 4 heads: the
+  // fast kernel (3 resident CTAs per SM) runs the balanced plan
+  int fast;
 };
 struct DecodeArgs {
   int base, L_hi, L_lo;
@@ -117,7 +120,7 @@ struct DecodeArgs {
 constexpr int kPartialFloats = 16 + 8 * 128;  // m[8], l[8], o[8][128]
 // max_stride: partial slots available per (b, h); a plan whose stride exceeds it
 // cannot be run with that workspace
-DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int64_t hi_count,
+DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int Hq, int64_t hi_count,
                             int64_t lo_count, int stage_n, int num_sms, int max_stride);
 constexpr int kMaxPartialsPerPair = 65;
 size_t decode_workspace_floats(int B, int H, int Hq);

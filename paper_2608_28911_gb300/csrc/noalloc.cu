@@ -72,7 +72,7 @@ extern "C" semkv_status semkv_decode_attention_noalloc(const semkv_quant_desc* d
   const int64_t cap64 = (int64_t)kScratchPartials / pairs;
   const int cap = (int)(cap64 < kMaxPartialsPerPair ? cap64 : kMaxPartialsPerPair);
   const DecodePlan plan = make_decode_plan(desc->base, desc->levels_hi, desc->levels_lo, c->batch,
-                                           c->kv_heads, c->hi_count, c->lo_count, c->stage_n,
+                                           c->kv_heads, c->q_heads, c->hi_count, c->lo_count, c->stage_n,
                                            sms, cap);
   if (cap < 1 || plan.stride > cap) return SEMKV_EWORKSPACE;  // exceeds the static scratch
 

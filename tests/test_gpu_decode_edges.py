@@ -20,11 +20,12 @@ plan, then the combine), on the plain affine 6/5, the Hadamard-rotated affine 6/
 the TurboQuant-MSE 4/3 bases, most with a staged fp16 tail.
 
 Tolerance: max-abs 2e-3 and relative L2 1e-3 at the synthetic scale (|v| below 64).
-Binary32 carries a relative error, so the absolute bound follows the values' scale:
-where every value is scaled by a power of two sigma it is 2e-3 * sigma; where a few
-rows are far larger it is max(2e-3, 1e-6 * max|v^|) (P' reaches the tensor cores as
-fp16 hi + lo, about 2^-22 relative, and sums run in fp32, so an output's error is a
-few 1e-7 of the largest value it averages).
+Binary32 carries a relative, not an absolute, error, so the absolute bound follows the
+values' scale: where every value is scaled by a power of two sigma it is 2e-3 * sigma;
+where a few rows are far larger it is max(2e-3, 8e-6 * max|v^|).  The tensor cores
+round each fp32 accumulation toward zero (at most one binary32 ulp, 2^-23 relative,
+per MMA) and a warp chains its PV products over up to ~64 tiles of a segment, so an
+output may drift by 64 * 2^-23 = 8e-6 of the largest value it averages.
 """
 import numpy as np
 import pytest
@@ -65,7 +66,7 @@ def _value_max(p):
 def _check(p, q, atol=None):
     got, ref = p.decode(q=q)
     if atol is None:
-        atol = max(ATOL, 1e-6 * _value_max(p))
+        atol = max(ATOL, 8e-6 * _value_max(p))
     err, rel = attention_errors(got, ref)
     assert err <= atol and rel <= RTOL_L2, (err, rel, atol)
     assert int(p.cache.dev_error.item()) == 0
@@ -165,14 +166,13 @@ def test_few_value_rows_near_fp16_limit(base, L_hi, L_lo, r):
 
 @pytest.mark.parametrize("base,L_hi,L_lo,r", BASES)
 def test_all_value_rows_scaled_up(base, L_hi, L_lo, r):
-    # values x 1024: the rows' ranges reach +-30000..60000 everywhere (the absolute
-    # bound is then 1e-6 * max|v^|, about 0.04)
+    # values x 1024: the rows' ranges reach +-30000..60000 everywhere
     sigma = 1024.0
     p = _pair(base, L_hi, L_lo, r, seed=550 + base)
     p.v = (p.v.astype(np.float32) * sigma).astype(np.float16)
     p.quantize()
     _stage_tail(p, 551 + base, vscale=sigma)
-    _check(p, synthetic.queries(552 + base, p.B, p.Hq))
+    _check(p, synthetic.queries(552 + base, p.B, p.Hq), atol=ATOL * sigma)
 
 
 @pytest.mark.parametrize("base,L_hi,L_lo,r", BASES)
