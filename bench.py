@@ -622,38 +622,39 @@ def gpu_arm(args, cfg, rank, world):
 
 # ------------------------------------------------------------ CPU oracle ------
 
-def oracle_sample(cfg, budget_s: float, max_steps: int | None = None):
+def oracle_sample(cfg, budget_s: float, max_steps: int | None = None, pair: int = 0):
     """The CPU oracle as it stands on a bounded sample of the same workload: one
-    (sequence, KV head) of the batch and one layer, at full context -- append one
-    block and run fp64 decode attention for that head's query heads -- repeated until
-    the time budget is spent.  Returns (GB/s of algorithmic bytes, sample description,
-    steps, seconds)."""
+    (sequence, KV head) of the batch (`pair`) and one layer, at full context -- append
+    one block and run fp64 decode attention for that head's query heads -- repeated
+    until the time budget (or max_steps) is spent.  Returns (GB/s of algorithmic bytes,
+    sample description, steps, seconds)."""
     import oracle
     T, Hq, H, blk = cfg["T"], cfg["Hq"], cfg["H"], cfg["block"]
     base = cfg["base"]
     r_num, r_den = cfg["r"]
     G = Hq // H
+    b, h = divmod(pair % (cfg["B"] * H), H)
     n_high = oracle.high_count_floor(T, r_num, r_den)
     nh_b = oracle.block_high_count(blk, r_num, r_den)
     oc = oracle.Cache(base=base, L_hi=cfg["L_hi"], L_lo=cfg["L_lo"], batch=1, layers=1, kv_heads=1,
                       q_heads=G, block=blk, hi_cap=((n_high + nh_b + 15) // 16) * 16,
                       lo_cap=((T - n_high + blk + 15) // 16) * 16)
     if base in (oracle.BASE_TQ, oracle.BASE_AFFINE_HAD):
-        oc.signs = synthetic.signs(cfg["seed"], 1, H)[:, :1]
+        oc.signs = np.ascontiguousarray(synthetic.signs(cfg["seed"], 1, H)[:, h:h + 1])
     if base == oracle.BASE_TQ_DENSE:
-        oc.rotation = np.ascontiguousarray(synthetic.rotations(cfg["seed"], 1, H)[:, :1])
+        oc.rotation = np.ascontiguousarray(synthetic.rotations(cfg["seed"], 1, H)[:, h:h + 1])
     if base in (oracle.BASE_TQ, oracle.BASE_TQ_DENSE):
         _, c32, t32, _ = oracle.lloyd_max_gaussian(cfg["L_hi"])
         oc.cb_hi = (c32, t32)
         _, c32, t32, _ = oracle.lloyd_max_gaussian(cfg["L_lo"])
         oc.cb_lo = (c32, t32)
-    kb, vb = synthetic.kv_layer(cfg["seed"] * 100, 0, 1, H, T)
-    s = synthetic.scores_zipf(cfg["seed"] * 100, 1, T)
-    oracle.quantize_prompt(oc, synthetic.f16_bits(kb[:, None, :1]), synthetic.f16_bits(vb[:, None, :1]),
-                           s, r_num, r_den)
+    kb, vb = synthetic.kv_layer(cfg["seed"] * 100 + b, 0, 1, H, T)
+    s = synthetic.scores_zipf(cfg["seed"] * 100 + b, 1, T)
+    oracle.quantize_prompt(oc, synthetic.f16_bits(kb[:, None, h:h + 1]),
+                           synthetic.f16_bits(vb[:, None, h:h + 1]), s, r_num, r_den)
     gk, gv = synthetic.kv(cfg["seed"] * 100 + 99, 1, 1, H, blk)
     gs = synthetic.scores_zipf(cfg["seed"] * 100 + 99, 1, blk)
-    q = synthetic.f16_bits(synthetic.queries(cfg["seed"], 1, Hq)[:, :G])
+    q = synthetic.f16_bits(synthetic.queries(cfg["seed"], 1, Hq)[:, h * G:(h + 1) * G])
     counts = (oc.hi_count, oc.lo_count, oc.n_tokens)
     rh, rl = oracle.record_bytes(base, cfg["L_hi"]), oracle.record_bytes(base, cfg["L_lo"])
     per_step = ((n_high + nh_b) * rh + (T - n_high + blk - nh_b) * rl + G * 128 * 6
@@ -661,8 +662,8 @@ def oracle_sample(cfg, budget_s: float, max_steps: int | None = None):
     steps, t_start = 0, time.perf_counter()
     while True:
         oc.hi_count, oc.lo_count, oc.n_tokens = counts
-        oc.stage_k[0, 0, 0, :blk] = synthetic.f16_bits(gk[0, 0, 0])
-        oc.stage_v[0, 0, 0, :blk] = synthetic.f16_bits(gv[0, 0, 0])
+        oc.stage_k[0, 0, 0, :blk] = synthetic.f16_bits(gk[0, 0, h])
+        oc.stage_v[0, 0, 0, :blk] = synthetic.f16_bits(gv[0, 0, h])
         oc.stage_score[0, :blk] = gs[0]
         oc.stage_n = blk
         oracle.append_block(oc, r_num, r_den)
@@ -675,6 +676,56 @@ def oracle_sample(cfg, budget_s: float, max_steps: int | None = None):
               f"full {T}-token context: append one {blk}-token block + fp64 decode attention "
               f"for its {G} query heads, x{steps} repetitions")
     return per_step * steps / el / 1e9, sample, steps, el
+
+
+def _oracle_worker(args):
+    """One process of the multi-core baseline (module level, so a spawned process can
+    import it): the oracle on its own (sequence, KV head) pair."""
+    cfg_name, budget_s, max_steps, pair = args
+    gbs, _, steps, el = oracle_sample(CONFIGS[cfg_name], budget_s, max_steps, pair)
+    return gbs * el * 1e9, steps, el
+
+
+def host_cpus():
+    """(usable cores, CPU model) of this host."""
+    n = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    model = ""
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu part")):
+                model = line.split(":", 1)[1].strip()
+                break
+        if not model:
+            r = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10)
+            m = re.search(r"Model name:\s*(.+)", r.stdout)
+            model = m.group(1).strip() if m else ""
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return n, model
+
+
+def oracle_sample_cores(cfg_name, budget_s: float, max_steps: int | None = None, cores=None):
+    """The oracle as it stands on every host core at once: one spawned process per core,
+    each on its own (sequence, KV head) pair of the workload (the pairs are independent,
+    as on the GPU).  Returns (GB/s of all processes' bytes over the wall time, sample,
+    cores, CPU model, wall seconds)."""
+    import multiprocessing as mp
+    n, model = host_cpus()
+    n = cores or n
+    cfg = CONFIGS[cfg_name]
+    pairs = cfg["B"] * cfg["H"]
+    ctx = mp.get_context("spawn")    # a fresh interpreter per process: no CUDA state inherited
+    t0 = time.perf_counter()
+    with ctx.Pool(n) as pool:
+        res = pool.map(_oracle_worker, [(cfg_name, budget_s, max_steps, i % pairs) for i in range(n)])
+    wall = time.perf_counter() - t0
+    total_bytes = sum(r[0] for r in res)
+    busy = max(r[2] for r in res)
+    sample = (f"{n} processes, one per core, each on its own (sequence, KV head) pair of "
+              f"{pairs}, 1 of {cfg['NL']} layers, at full {cfg['T']}-token context: append one "
+              f"{cfg['block']}-token block + fp64 decode attention, "
+              f"x{min(r[1] for r in res)}-{max(r[1] for r in res)} repetitions each")
+    return total_bytes / busy / 1e9, sample, n, model, wall
 
 
 # ------------------------------------------------------------------ main ------
@@ -709,13 +760,16 @@ def main():
     if args.impl == "reference":
         if rank != 0:
             return
-        gbs, sample, steps, el = oracle_sample(cfg, 0, max_steps=args.warmup + args.steps)
+        # every host core runs the oracle on its own pair; a step = one block append +
+        # decode on each of them
+        steps = args.warmup + args.steps
+        gbs, sample, cores, model, wall = oracle_sample_cores(args.config, 0, max_steps=steps)
         line = {"impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s",
                 "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-                "ms_per_step": el / steps * 1e3, "higher_is_better": True, "scaling": "weak",
+                "ms_per_step": wall / steps * 1e3, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config,
-                "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": 1, "kind": "oracle",
-                                 "sample": sample},
+                "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
+                                 "cpu": model, "sample": sample},
                 "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}}
         print(json.dumps(line))
@@ -767,9 +821,12 @@ def main():
         "device_error": r["err"],
     }
     if world == 1 and args.cpu_seconds > 0:
-        gbs, sample, steps, el = oracle_sample(cfg, args.cpu_seconds)
-        line["cpu_baseline"] = {"value": gbs, "unit": "GB/s", "cores": 1, "kind": "oracle",
-                                "sample": sample}
+        # the oracle on every host core (the baseline), and on one core alongside
+        gbs, sample, cores, model, _ = oracle_sample_cores(args.config, args.cpu_seconds / 2)
+        gbs1, sample1, _, _ = oracle_sample(cfg, args.cpu_seconds / 2)
+        line["cpu_baseline"] = {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
+                                "cpu": model, "sample": sample,
+                                "single_core": {"value": gbs1, "unit": "GB/s", "sample": sample1}}
     print(json.dumps(line))
 
 

@@ -82,10 +82,14 @@ class Pair:
         assert np.array_equal(c.hi_tok.cpu().numpy()[:, :oc.hi_count], oc.hi_tok[:, :oc.hi_count])
         assert np.array_equal(c.lo_tok.cpu().numpy()[:, :oc.lo_count], oc.lo_tok[:, :oc.lo_count])
 
-    def assert_records_equal_up_to_ties(self, k=None, v=None, eps=1e-4):
+    def assert_records_equal_up_to_ties(self, k=None, v=None, eps=2e-4):
         """Dense-rotation TQ: the GPU forms w = M x on the tensor cores, the oracle rounds
         the exact product once, so a code may differ by one where u sits within rounding
-        of the threshold between them.  Norms, token maps and every other code match."""
+        of the threshold between them.  Norms, token maps and every other code match.
+        eps: the worst case of 8 chained MMAs of 16 products, each MMA truncating its 17
+        addends below one binary32 unit of the largest (8 * 17 * 2^-23 * ||M_i|| ||x|| / n,
+        about 1.8e-4 with ||M_i|| ~ sqrt(128), n ~ ||x||).  The share of flipped codes is
+        bounded by 1e-4, five times its expectation for spread-out truncation errors."""
         c, oc = self.cache, self.oc
         k = self.k if k is None else k
         v = self.v if v is None else v
