@@ -120,6 +120,13 @@ inline cudaError_t once_per_device(bool (&done)[kAttrDevices], F set) {
 // on the stream drains; it must call pdl_wait() before touching what that kernel (or
 // anything earlier on the stream) wrote.  pdl_wait is a no-op for an ordinary launch.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Let the next kernel on the stream be scheduled now (its CTAs take SM slots as this
+// kernel's CTAs leave).  It fires once every CTA of this grid has issued it or exited,
+// so a dependent never holds resources that a CTA of this grid still waits for, and
+// the dependent still waits (pdl_wait) before it reads what this kernel writes.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 template <typename... Params, typename... Args>
 inline cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
                               cudaStream_t stream, Args&&... args) {

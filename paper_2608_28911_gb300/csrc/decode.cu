@@ -1670,6 +1670,7 @@ __global__ void __launch_bounds__(kThreads, kCtasAffine) decode_affine_kernel(De
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncthreads();
   pdl_wait();  // the records, queries and stage partial come from earlier work
+  pdl_trigger();
   int ring_it = 0;  // tiles this warp has taken through its ring (barrier phases)
   int64_t loaded = -1;
   for (int64_t bh = start / P.W; bh < pairs && bh * P.W < end; ++bh) {
@@ -1783,6 +1784,7 @@ __global__ void __launch_bounds__(kThreads, kCtasFast) decode_affine_fast_kernel
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncthreads();
   pdl_wait();  // the records, queries and stage partial come from earlier work
+  pdl_trigger();
   int ring_it = 0;  // tiles this warp has taken through its ring (barrier phases)
   int64_t loaded = -1;
   for (int64_t bh = start / P.W; bh < pairs && bh * P.W < end; ++bh) {
@@ -2001,6 +2003,7 @@ __global__ void combine_kernel(DecodeArgs a) {
   // launched as a programmatic dependent of the pool kernels: the rotation above is
   // staged while they finish; their partials are read only after this wait
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  pdl_trigger();
   if (gw >= a.B * a.Hq) return;
   const int b = gw / a.Hq, qh = gw % a.Hq;
   const int h = qh / G, c = qh % G;
@@ -2053,6 +2056,7 @@ __global__ void __launch_bounds__(256) combine_wide_kernel(DecodeArgs a) {
   __shared__ float red_m[8], red_l[8];
   // launched as a programmatic dependent of the pool kernels: wait for their partials
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  pdl_trigger();
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const int gw = blockIdx.x;
   const int b = gw / a.Hq, qh = gw % a.Hq;

@@ -201,6 +201,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 4)
   __shared__ __align__(16) uint32_t img_sm[kWarpsPerBlock][kAffineSlots * kMaxRecWords];
   const int wib = threadIdx.x >> 5;
   pdl_wait();  // the slot maps and the rows come from earlier work on the stream
+  pdl_trigger();
   const bool hi = blockIdx.z == 0;
   const int64_t n_pool = hi ? n_hi : n_lo;
   const int64_t u_begin = (int64_t)blockIdx.x * kWarpsPerBlock + wib;

@@ -71,6 +71,7 @@ __global__ void __launch_bounds__(kThreads) rank_small_kernel(RankArgs a) {
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int T = a.T;
   pdl_wait();  // the scores (and the maps) belong to earlier work on the stream
+  pdl_trigger();
   const float* s = a.scores + (int64_t)b * a.ld;
   const uint32_t mine = tid < T ? order_key(s[tid]) : 0u;
   keys[tid] = mine;
