@@ -975,34 +975,33 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
   const bool rot = a.base == SEMKV_BASE_AFFINE_HAD;
 
   // B fragments: coefficients of head g>>1 (hi part for even g, lo part for odd g) for
-  // the slots of lane (g, t), the same for every warp: warp 0 writes them to shared
-  // memory, every warp loads its lane's pair per step (one conflict-free 8-byte load)
+  // the slots of lane (g, t), the same for every warp: warp w builds step w for every
+  // lane into shared memory, then every warp loads its lane's pair per step (one
+  // conflict-free 8-byte load)
+  static_assert(kWarps >= 8, "one warp per coefficient step");
   __syncthreads();  // the previous segment's fragments and the merge area are no longer read
-  if (warp == 0) {
-    const int hb = g >> 1;
+  if (warp < 8) {
+    const int hb = g >> 1, j = warp;
     const float sc = coef_scale(sh.qmax[hb], L);
+    uint32_t r[2];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      uint32_t r[2];
-#pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        const int p = 2 * j + i;
-        float c0 = 0.0f, c1 = 0.0f;
-        if (hb < G) {
-          if (rot) {
-            c0 = k_coef<L>(sh.qr[hb], t, p, 0) * sc;
-            c1 = k_coef<L>(sh.qr[hb], t, p, 1) * sc;
-          } else {
-            c0 = k_coef<L>(sh.q[hb], t, p, 0) * sc;
-            c1 = k_coef<L>(sh.q[hb], t, p, 1) * sc;
-          }
+    for (int i = 0; i < 2; ++i) {
+      const int p = 2 * j + i;
+      float c0 = 0.0f, c1 = 0.0f;
+      if (hb < G) {
+        if (rot) {
+          c0 = k_coef<L>(sh.qr[hb], t, p, 0) * sc;
+          c1 = k_coef<L>(sh.qr[hb], t, p, 1) * sc;
+        } else {
+          c0 = k_coef<L>(sh.q[hb], t, p, 0) * sc;
+          c1 = k_coef<L>(sh.q[hb], t, p, 1) * sc;
         }
-        uint32_t hi, lo;
-        split_h2(c0, c1, hi, lo);
-        r[i] = (g & 1) ? lo : hi;
       }
-      qbs[32 * j + lane] = make_uint2(r[0], r[1]);
+      uint32_t hi, lo;
+      split_h2(c0, c1, hi, lo);
+      r[i] = (g & 1) ? lo : hi;
     }
+    qbs[32 * j + lane] = make_uint2(r[0], r[1]);
   }
   __syncthreads();
   const uint2* qb = qbs + lane;
@@ -1573,6 +1572,9 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
     mg.cta_z[qh] = zsum;
   }
   __syncthreads();
+  // (dense-rotation partials stay in the rotated domain: the combine turns their sum
+  // back once per head)
+  const bool rotated = (kind == 1 || kind == 3) && a.base != SEMKV_BASE_TQ_DENSE;
   float* merged = merge_o + kWarps * 8 * 128;  // [8][128], after the warp rows
   for (int i = threadIdx.x; i < G * 128; i += kThreads) {
     const int qh = i >> 7, d = i & 127;
@@ -1585,12 +1587,15 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
         o += sc * v;
       }
     }
-    merged[qh * 128 + d] = (kind == 0 || kind == 3) ? o + mg.cta_z[qh] : o;
+    o = (kind == 0 || kind == 3) ? o + mg.cta_z[qh] : o;
+    if (rotated) merged[qh * 128 + d] = o;
+    else part[16 + qh * 128 + d] = o;   // nothing to turn back: straight to the partial
+  }
+  if (!rotated) {
+    __syncthreads();  // the merge area (the ring) is free again
+    return;
   }
   __syncthreads();
-  // (dense-rotation partials stay in the rotated domain: the combine turns their sum
-  // back once per head)
-  const bool rotated = (kind == 1 || kind == 3) && a.base != SEMKV_BASE_TQ_DENSE;
   if (rotated) {
     // back from the rotated domain: o = S H o' (unnormalised transform, stages 1..64)
     for (int hs = 1; hs < 128; hs <<= 1) {
