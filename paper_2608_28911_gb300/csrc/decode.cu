@@ -935,6 +935,30 @@ __device__ __forceinline__ float2 h2_to_f2(uint32_t h) {
 }
 __device__ __forceinline__ uint32_t f2_to_h2(float2 v) { return pack_h2(v.x, v.y); }
 
+// A 96-bit window read with 32-bit shared-memory addressing: addr is the shared address
+// of the word holding the window's first bit, sh the bit offset in it.  (volatile keeps
+// the loads after the tile's mbarrier wait.)
+__device__ __forceinline__ Window load_window_s(uint32_t addr, uint32_t sh) {
+  uint32_t w0, w1, w2, w3;
+  asm volatile(
+      "ld.shared.u32 %0, [%4];\n\t"
+      "ld.shared.u32 %1, [%4+4];\n\t"
+      "ld.shared.u32 %2, [%4+8];\n\t"
+      "ld.shared.u32 %3, [%4+12];"
+      : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
+      : "r"(addr));
+  Window r;
+  r.q0 = __funnelshift_r(w0, w1, sh);
+  r.q1 = __funnelshift_r(w1, w2, sh);
+  r.q2 = __funnelshift_r(w2, w3, sh);
+  return r;
+}
+__device__ __forceinline__ uint2 ld_shared_u2(uint32_t addr) {
+  uint32_t x, y;
+  asm volatile("ld.shared.u32 %0, [%2];\n\tld.shared.u32 %1, [%2+4];" : "=r"(x), "=r"(y) : "r"(addr));
+  return make_uint2(x, y);
+}
+
 struct FastState {
   float O[8][4];  // O^T accumulators: V rows x columns 2t, 2t+1
   float e;        // reference exponent of head t (base 2)
@@ -1023,6 +1047,12 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
   const uint32_t tneg = hh ? 0xC500C500u : 0u;
   const uint32_t ov = overlay1024();
   const int kpos = t * F::QB;
+  // 32-bit shared addresses: the ring, and per lane the word offsets of its windows in a
+  // tile and their bit shifts
+  const uint32_t ring_s = smem_u32(my_ring);
+  const uint32_t kw0 = g * kRec + 4 * (kpos >> 5), kw1 = kw0 + 8 * kRec, ksh = kpos & 31;
+  const uint32_t vw0 = 2 * t * kRec + 4 * (vpos >> 5), vsh = vpos & 31;
+  const uint32_t pw0 = g * kRec + 2 * F::RB, pw1 = pw0 + 8 * kRec;
 
   const int nmine = t_end - t_begin <= warp ? 0 : (t_end - t_begin - warp + kWarps - 1) / kWarps;
   // tokens left in the pool from this warp's current tile on (a pool holds fewer than
@@ -1038,7 +1068,7 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
       ok = false;
       break;
     }
-    const uint8_t* tb = my_ring + stage * kStageBytes;
+    const uint32_t ts = ring_s + stage * kStageBytes;
     const int nvalid = min(kTile, left);
 
     // ---- S^T = F Q'^T: tokens g (rows g) and g + 8, heads in column pairs
@@ -1046,8 +1076,8 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
     {
       if constexpr (L == 5) {
         uint32_t Ba[5], Bb[5], Ta, Tb;
-        k5_B(load_window(tb + g * kRec, kpos), ov, Ba, Ta);
-        k5_B(load_window(tb + (g + 8) * kRec, kpos), ov, Bb, Tb);
+        k5_B(load_window_s(ts + kw0, ksh), ov, Ba, Ta);
+        k5_B(load_window_s(ts + kw1, ksh), ov, Bb, Tb);
 #pragma unroll
         for (int j = 0; j < 8; ++j)
         {
@@ -1057,8 +1087,8 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
         }
       } else {
         uint32_t fa[8][2], fb[8][2];
-        k_quarter<L>(load_window(tb + g * kRec, kpos), fa);
-        k_quarter<L>(load_window(tb + (g + 8) * kRec, kpos), fb);
+        k_quarter<L>(load_window_s(ts + kw0, ksh), fa);
+        k_quarter<L>(load_window_s(ts + kw1, ksh), fb);
 #pragma unroll
         for (int j = 0; j < 8; ++j)
         {
@@ -1068,12 +1098,11 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
       }
     }
     // ---- softmax of head t over tokens g and g + 8
-    const uint32_t* pr0 = reinterpret_cast<const uint32_t*>(tb + g * kRec + 2 * F::RB);
-    const uint32_t* pr1 = reinterpret_cast<const uint32_t*>(tb + (g + 8) * kRec + 2 * F::RB);
     const bool v0 = live && g < nvalid, v1 = live && g + 8 < nvalid;
-    const uint32_t kp0 = pr0[0], kp1 = pr1[0];
+    const uint2 pr0 = ld_shared_u2(ts + pw0), pr1 = ld_shared_u2(ts + pw1);
+    const uint32_t kp0 = pr0.x, kp1 = pr1.x;
     // rows past the pool's count are not data: keep whatever they hold out of the sums
-    const uint32_t vp0 = v0 ? pr0[1] : 0u, vp1 = v1 ? pr1[1] : 0u;
+    const uint32_t vp0 = v0 ? pr0.y : 0u, vp1 = v1 ? pr1.y : 0u;
     // both tokens at once in packed binary32 (x: token g, y: token g + 8)
     const float2 k0 = h2_to_f2(kp0), k1 = h2_to_f2(kp1), vv0 = h2_to_f2(vp0), vv1 = h2_to_f2(vp1);
     const float2 lg = f2_fma(f2_mul(make_float2(k0.x, k1.x), make_float2(cS, cS)),
@@ -1139,10 +1168,10 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
     }
     // ---- O^T += C^T P'^T
     {
-      const Window w0 = load_window(tb + (2 * t) * kRec, vpos);
-      const Window w1 = load_window(tb + (2 * t + 1) * kRec, vpos);
-      const Window w2 = load_window(tb + (2 * t + 8) * kRec, vpos);
-      const Window w3 = load_window(tb + (2 * t + 9) * kRec, vpos);
+      const Window w0 = load_window_s(ts + vw0, vsh);
+      const Window w1 = load_window_s(ts + vw0 + kRec, vsh);
+      const Window w2 = load_window_s(ts + vw0 + 8 * kRec, vsh);
+      const Window w3 = load_window_s(ts + vw0 + 9 * kRec, vsh);
       if constexpr (L == 5) {
         // symbol by symbol: after symbol j, rows 0 .. 3j + 2 are ready and the m-blocks
         // up to (3j + 1) / 2 go to the tensor cores
