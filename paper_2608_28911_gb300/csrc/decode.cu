@@ -1871,6 +1871,7 @@ __global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs
   const int64_t bh = (int64_t)b * a.H + h;
   const int G = a.Hq / a.H;
   int split = blockIdx.x;
+  if (KIND == 2 && !a.stage_overlaps_pools) pdl_wait();
   if (KIND == 2) {
     if (P.balanced) {
       int n_hi, n_lo;
@@ -1989,6 +1990,9 @@ __global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs
     }
   }
   merge_warps(a, kind, h, G, mg, merge_o, a.partials + (bh * P.stride + split) * kPartialFloats);
+  // a stage kernel that ran alongside the pool kernel completes only after it: the
+  // combine, which waits for this kernel, then sees every pool partial too
+  if (KIND == 2) pdl_wait();
 }
 
 // merge the partials of each (b, qh): one warp per head, 4 dims per lane.  The lanes
@@ -2334,7 +2338,15 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (P.splits_st > 0) {
-    decode_kernel<2><<<dim3(1, a.H, a.B), kThreads, kRingBytes, stream>>>(a);
+    // after an affine pool kernel (which triggers its dependents once it has waited for
+    // its own inputs) the stage kernel starts alongside it; otherwise it runs in order
+    DecodeArgs as = a;
+    as.stage_overlaps_pools = (a.base == SEMKV_BASE_AFFINE || a.base == SEMKV_BASE_AFFINE_HAD) && P.ctas > 0;
+    if (as.stage_overlaps_pools)
+      e = launch_pdl(decode_kernel<2>, dim3(1, a.H, a.B), dim3(kThreads), kRingBytes, stream, as);
+    else
+      decode_kernel<2><<<dim3(1, a.H, a.B), kThreads, kRingBytes, stream>>>(as);
+    if (e != cudaSuccess) return e;
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }

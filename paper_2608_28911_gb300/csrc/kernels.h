@@ -115,6 +115,9 @@ struct DecodeArgs {
   const float* cb_lo;
   float* qrot;               // TQ: [B][Hq][128] rotated queries (workspace)
   int32_t* err;
+  // the fp16 stage kernel runs as a programmatic dependent of the affine pool kernel:
+  // it reads its inputs at once and waits for that kernel only before it exits
+  int stage_overlaps_pools;
   DecodePlan plan;
 };
 constexpr int kPartialFloats = 16 + 8 * 128;  // m[8], l[8], o[8][128]
