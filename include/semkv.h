@@ -263,9 +263,9 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
  *    affine bases (balanced plan) need cap >= 3 + stage, i.e. batch * kv_heads <= 672,
  *    or <= 504 with staged tokens; the TQ bases (split plan) need cap >= one per
  *    non-empty pool + stage, i.e. batch * kv_heads * (pools + stage) <= 2016.
- *    Larger requests return SEMKV_EWORKSPACE before anything is launched.  The rotated
- *    bases (TQ, AFFINE_HAD, TQ_DENSE) also keep their rotated queries in a second
- *    static array of 4096 query heads (batch * q_heads beyond it: SEMKV_EWORKSPACE).
+ *    Larger requests return SEMKV_EWORKSPACE before anything is launched.  The dense-
+ *    rotation base (TQ_DENSE) also keeps its rotated queries in a second static array
+ *    of 4096 query heads (batch * q_heads beyond it: SEMKV_EWORKSPACE).
  *  - All calls share the array, which keeps the last call's contents (each call
  *    overwrites every partial it reads, so nothing needs clearing).  Calls whose
  *    kernels overlap on the GPU (e.g. on two streams, or two host threads) race on

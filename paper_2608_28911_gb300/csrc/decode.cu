@@ -1352,37 +1352,6 @@ __device__ void run_pool_tq(const DecodeArgs& a, const Shared& sh, int which,
   }
 }
 
-// q' = H S q for every (sequence, query head), times fp32(1/sqrt 128) for the rotated
-// affine base (whose rows are stored in the orthonormal frame): one warp each, lane l =
-// dims 4l..4l+3
-__global__ void qrot_kernel(DecodeArgs a) {
-  const int lane = threadIdx.x & 31;
-  const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (gw >= a.B * a.Hq) return;
-  const int b = gw / a.Hq, qh = gw % a.Hq, h = qh / (a.Hq / a.H);
-  const uint16_t* qrow = a.q + ((int64_t)b * a.Hq + qh) * 128;
-
-  const int8_t* sg = a.signs + ((int64_t)a.layer * a.H + h) * 128;
-  float w[4];
-#pragma unroll
-  for (int j = 0; j < 4; ++j) w[j] = f16_to_f32(qrow[4 * lane + j]) * (float)sg[4 * lane + j];
-  float t0 = w[0] + w[1], t1 = w[0] - w[1], t2 = w[2] + w[3], t3 = w[2] - w[3];
-  w[0] = t0 + t2; w[2] = t0 - t2; w[1] = t1 + t3; w[3] = t1 - t3;
-#pragma unroll
-  for (int k = 0; k < 5; ++k) {
-    const bool upper = (lane >> k) & 1;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float other = __shfl_xor_sync(0xffffffffu, w[j], 1 << k);
-      w[j] = upper ? other - w[j] : w[j] + other;
-    }
-  }
-  const float rs = a.base == SEMKV_BASE_AFFINE_HAD ? kInvSqrtD : 1.0f;
-  float* dst = a.qrot + ((int64_t)b * a.Hq + qh) * 128 + 4 * lane;
-#pragma unroll
-  for (int j = 0; j < 4; ++j) dst[j] = w[j] * rs;
-}
-
 // Dense rotation: q' = M q for the G query heads of each (sequence, KV head); one block
 // of 128 threads per pair, thread i taking row i of M (16 independent 16-byte loads)
 // against the group's queries staged in shared memory.
@@ -1498,16 +1467,48 @@ struct MergeArea {
 // (rotated affine base: also the rotated queries into sh.qr, which the sums then follow)
 __device__ void load_group_q(const DecodeArgs& a, Shared& sh, int b, int h, int G) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const bool rot = a.base == SEMKV_BASE_AFFINE_HAD;
+  // the Walsh-Hadamard bases take their rotated queries q' = H S q (times fl32(1/sqrt
+  // 128) for the rotated affine base, whose rows are stored in the orthonormal frame);
+  // the dense rotation's q' = M q comes from qrot_dense_kernel
+  const bool wht = a.base == SEMKV_BASE_AFFINE_HAD || a.base == SEMKV_BASE_TQ;
+  const bool rot = wht || a.base == SEMKV_BASE_TQ_DENSE;
   for (int i = threadIdx.x; i < 8 * 128; i += kThreads) {
     const int c = i >> 7, d = i & 127;
     const int64_t at = ((int64_t)b * a.Hq + h * G + c) * 128 + d;
     sh.q[c][d] = c < G ? a.q[at] : (uint16_t)0;
-    if (rot) sh.qr[c][d] = c < G ? a.qrot[at] : 0.0f;
+    if (a.base == SEMKV_BASE_TQ_DENSE) sh.qr[c][d] = c < G ? a.qrot[at] : 0.0f;
   }
   __syncthreads();
-  // per head: sum of q (the zero-point weight) and max |q| (the coefficient scale)
   static_assert(kWarps == 8, "one warp per head slot");
+  if (wht) {
+    // warp w rotates head w: lane l holds dims 4l..4l+3; butterfly stages 1, 2 inside
+    // the lane, then 4..64 across lanes, each (a + b, a - b) rounded to nearest
+    const int8_t* sg = a.signs + ((int64_t)a.layer * a.H + h) * 128;
+    float w[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      w[j] = warp < G ? f16_to_f32(sh.q[warp][4 * lane + j]) * (float)sg[4 * lane + j] : 0.0f;
+    const float t0 = w[0] + w[1], t1 = w[0] - w[1], t2 = w[2] + w[3], t3 = w[2] - w[3];
+    w[0] = t0 + t2;
+    w[2] = t0 - t2;
+    w[1] = t1 + t3;
+    w[3] = t1 - t3;
+#pragma unroll
+    for (int k = 0; k < 5; ++k) {
+      const bool upper = (lane >> k) & 1;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float other = __shfl_xor_sync(0xffffffffu, w[j], 1 << k);
+        w[j] = upper ? other - w[j] : w[j] + other;
+      }
+    }
+    const float rs = a.base == SEMKV_BASE_AFFINE_HAD ? kInvSqrtD : 1.0f;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) sh.qr[warp][4 * lane + j] = w[j] * rs;
+    __syncwarp();
+  }
+  // per head: sum of q (the zero-point weight) and max |q| (the coefficient scale), of
+  // the rotated queries for the rotated bases
   float s = 0.0f, mx = 0.0f;
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
@@ -1871,6 +1872,10 @@ __global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs
   const int64_t bh = (int64_t)b * a.H + h;
   const int G = a.Hq / a.H;
   int split = blockIdx.x;
+  if (KIND == 1) {
+    pdl_wait();  // the records and queries (and the dense rotation's q') come from earlier work
+    pdl_trigger();
+  }
   if (KIND == 2 && !a.stage_overlaps_pools) pdl_wait();
   if (KIND == 2) {
     if (P.balanced) {
@@ -1884,10 +1889,6 @@ __global__ void __launch_bounds__(kThreads, kCtasOther) decode_kernel(DecodeArgs
   load_group_q(a, sh, b, h, G);
   __shared__ int tq_path;  // TQ: 1 when this pool's codebook takes the tensor-core path
   if (KIND == 1) {
-    for (int i = threadIdx.x; i < 8 * 128; i += kThreads) {
-      const int c = i >> 7, d = i & 127;
-      sh.qr[c][d] = c < G ? a.qrot[((int64_t)b * a.Hq + h * G + c) * 128 + d] : 0.0f;
-    }
     if (threadIdx.x < 16) {
       const int which = threadIdx.x >> 3, k = threadIdx.x & 7;
       const int L = which == 0 ? a.L_hi : a.L_lo;
@@ -2303,45 +2304,38 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
   const DecodePlan& P = a.plan;
   if (P.stride < 1 || P.stride > kMaxSplits + 1) return cudaErrorInvalidValue;
   cudaError_t e = cudaSuccess;
-  if (a.base == SEMKV_BASE_TQ_DENSE) {
-    qrot_dense_kernel<<<a.B * a.H, 128, 0, stream>>>(a);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    const int pool_splits = P.splits_hi + P.splits_lo;
-    if (pool_splits > 0)
-      decode_kernel<1><<<dim3(pool_splits, a.H, a.B), kThreads, kRingBytes + kAqBytes, stream>>>(a);
-  } else if (a.base == SEMKV_BASE_TQ) {
-    const int heads = a.B * a.Hq;
-    qrot_kernel<<<(heads + 7) / 8, 256, 0, stream>>>(a);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    const int pool_splits = P.splits_hi + P.splits_lo;
-    if (pool_splits > 0)
-      decode_kernel<1><<<dim3(pool_splits, a.H, a.B), kThreads, kRingBytes + kAqBytes, stream>>>(a);
-  } else {
-    if (a.base == SEMKV_BASE_AFFINE_HAD) {  // the stage kernel reads the rotated q too
-      const int heads = a.B * a.Hq;
-      qrot_kernel<<<(heads + 7) / 8, 256, 0, stream>>>(a);
+  bool pools_launched = false;
+  if (a.base == SEMKV_BASE_TQ_DENSE || a.base == SEMKV_BASE_TQ) {
+    if (a.base == SEMKV_BASE_TQ_DENSE) {
+      qrot_dense_kernel<<<a.B * a.H, 128, 0, stream>>>(a);
       e = cudaGetLastError();
       if (e != cudaSuccess) return e;
     }
-    if (P.ctas > 0 && P.fast) {
+    const int pool_splits = P.splits_hi + P.splits_lo;
+    if (pool_splits > 0) {
+      e = launch_pdl(decode_kernel<1>, dim3(pool_splits, a.H, a.B), dim3(kThreads),
+                     kRingBytes + kAqBytes, stream, a);
+      if (e != cudaSuccess) return e;
+      pools_launched = true;
+    }
+  } else if (P.ctas > 0) {
+    // (the rotated affine base rotates its queries inside the pool and stage kernels)
+    if (P.fast)
       e = launch_pdl(decode_affine_fast_kernel, dim3(P.ctas), dim3(kThreads), kRingBytes + kQbBytes,
                      stream, a);
-      if (e != cudaSuccess) return e;
-    } else if (P.ctas > 0) {
+    else
       e = launch_pdl(decode_affine_kernel, dim3(P.ctas), dim3(kThreads), kRingBytes + kAqBytes,
                      stream, a);
-      if (e != cudaSuccess) return e;
-    }
+    if (e != cudaSuccess) return e;
+    pools_launched = true;
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (P.splits_st > 0) {
-    // after an affine pool kernel (which triggers its dependents once it has waited for
-    // its own inputs) the stage kernel starts alongside it; otherwise it runs in order
+    // after a pool kernel (which triggers its dependents once it has waited for its own
+    // inputs) the stage kernel starts alongside it; otherwise it runs in order
     DecodeArgs as = a;
-    as.stage_overlaps_pools = (a.base == SEMKV_BASE_AFFINE || a.base == SEMKV_BASE_AFFINE_HAD) && P.ctas > 0;
+    as.stage_overlaps_pools = pools_launched ? 1 : 0;
     if (as.stage_overlaps_pools)
       e = launch_pdl(decode_kernel<2>, dim3(1, a.H, a.B), dim3(kThreads), kRingBytes, stream, as);
     else

@@ -18,7 +18,7 @@
 static constexpr size_t kScratchPartials = 2016;
 static constexpr size_t kScratchFloats = kScratchPartials * semkv::kPartialFloats;
 static __device__ __align__(256) float g_decode_scratch[kScratchFloats];
-// 2 MiB of rotated queries (the rotated bases): 4096 query heads of 128 floats
+// 2 MiB of rotated queries (the dense-rotation base): 4096 query heads of 128 floats
 static constexpr size_t kQrotFloats = (size_t)4096 * 128;
 static __device__ __align__(256) float g_qrot_scratch[kQrotFloats];
 
@@ -76,7 +76,9 @@ extern "C" semkv_status semkv_decode_attention_noalloc(const semkv_quant_desc* d
                                            sms, cap);
   if (cap < 1 || plan.stride > cap) return SEMKV_EWORKSPACE;  // exceeds the static scratch
 
-  const bool rotated = desc->base != SEMKV_BASE_AFFINE;
+  // only the dense rotation keeps its rotated queries in memory (the Walsh-Hadamard bases
+  // rotate them inside the kernels)
+  const bool rotated = desc->base == SEMKV_BASE_TQ_DENSE;
   if (rotated && (size_t)c->batch * c->q_heads * 128 > kQrotFloats) return SEMKV_EWORKSPACE;
 
   float* scratch = nullptr;
