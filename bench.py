@@ -691,16 +691,19 @@ def host_cpus():
     n = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
     model = ""
     try:
-        for line in open("/proc/cpuinfo"):
-            if line.lower().startswith(("model name", "cpu part")):
-                model = line.split(":", 1)[1].strip()
-                break
-        if not model:
-            r = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10)
-            m = re.search(r"Model name:\s*(.+)", r.stdout)
-            model = m.group(1).strip() if m else ""
+        r = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10)
+        m = re.search(r"Model name:\s*(.+)", r.stdout)
+        model = m.group(1).strip() if m else ""
     except (OSError, subprocess.SubprocessError):
         pass
+    if not model:
+        try:
+            for line in open("/proc/cpuinfo"):
+                if line.lower().startswith(("model name", "cpu part")):
+                    model = line.split(":", 1)[1].strip()
+                    break
+        except OSError:
+            pass
     return n, model
 
 
