@@ -185,7 +185,7 @@ semkv_status semkv_quantize_pack(const semkv_quant_desc* desc, const uint16_t* k
   if (!k || !v || !is_high || !slot || T < 1) return SEMKV_EINVAL;
   if (!aligned(k, 8) || !aligned(v, 8)) return SEMKV_EALIGN;
   if (desc->base != SEMKV_BASE_AFFINE && (!aligned(k, 16) || !aligned(v, 16)))
-    return SEMKV_EALIGN;  // the rows arrive by bulk or tensor copies in 16-byte units
+    return SEMKV_EALIGN;  // the rows arrive by async or tensor copies in 16-byte units
   if (n_high > (uint32_t)T) return SEMKV_EINVAL;
   if ((int64_t)n_high > cache->hi_cap || (int64_t)(T - n_high) > cache->lo_cap)
     return SEMKV_ECAPACITY;

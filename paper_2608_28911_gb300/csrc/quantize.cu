@@ -224,18 +224,30 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 4)
   }
 }
 
-// ------------------------------- rotated bases by slot, one thread per row -----
+// ------------------------------ rotated bases by slot, two threads per row -----
 // TQ and rotated affine records built by destination slot, as for the affine base: a
-// CTA of 128 threads takes 64 consecutive slots of one pool of one (sequence, layer,
-// KV head), so the level count is uniform.  Thread r owns row r of the tile (K of slot
-// r/2 when r is even, V when odd).  Its 128 values live in registers and the
-// Walsh-Hadamard butterflies run inside the thread in the quantizer's stage order
-// (the same roundings as the lane-distributed form), followed by the norm or the
-// min/max, the codes and the quarter bit fields.  The warps then assemble each
-// record's words from the two rows' bits and write them with 4-byte stores.
+// CTA of 256 threads takes 64 consecutive slots of one pool of one (sequence, layer,
+// KV head), so the level count is uniform.  Thread tid holds half f = tid & 1 (dims
+// 64f .. 64f + 63, quarters 2f and 2f + 1) of row tid >> 1 of the block (K of slot
+// tid >> 2 when bit 1 of tid is 0, V when it is 1), in registers as 32 packed pairs
+// (x_j, x_{j+32}).  The Walsh-Hadamard butterflies run in the quantizer's stage order
+// (the same roundings as any other evaluation of them): stages 1..16 as packed
+// operations across pairs, stage 32 inside each pair, stage 64 with the partner lane.
+// Then the norm or the min/max (combined across the two halves), the codes, the two
+// quarters' bit fields; the threads then assemble the block's record words from the
+// rows' bit images and write them in order with 4-byte stores.
 constexpr int kRowSlots = 64;
 constexpr int kRowStride = 272;  // bytes per staged row: 256 + 16 spreads the banks
 constexpr int kRowBitWords = 13;  // words per row's bit image (12 used at most)
+constexpr int kRows2Threads = 256;
+constexpr int kHalfStride = 144;  // bytes per half-row slot: 128 + 16 (9 x 16 B: the 8 lanes
+                                  // of a quarter warp reach distinct banks)
+constexpr int kRows2StageBytes = kRows2Threads * kHalfStride;
+// resident CTAs per SM (80 registers a thread).  The TQ path at 4 and more levels keeps
+// its packed thresholds in registers too and spills a few words at this budget; it still
+// ran 6% faster than at 2 CTAs per SM (128 registers, no spills).
+constexpr int rows2_ctas(int) { return 3; }
+static_assert(kRowBitWords + 1 <= kHalfStride / 4, "bit image and parameters fit a half slot");
 
 // packed binary32 pairs (two independent IEEE operations, rounded to nearest)
 __device__ __forceinline__ unsigned long long f2_add(unsigned long long a, unsigned long long b) {
@@ -296,58 +308,241 @@ __device__ __forceinline__ void or_field(uint32_t (&w)[N], int pos, const uint32
   }
 }
 
-template <int BASE, int L>
-__device__ void rows_block(const QuantArgs& a, int b, int l, int h, bool hi, int64_t s0,
-                           int nslots, uint8_t* stage) {
+// packed binary32 multiply and fused multiply-add (one rounding each).  The code
+// generator may fuse a packed multiply into a packed add or subtract that consumes it,
+// .rn notwithstanding (measured), so bit-exact paths use f2_mul only where the product
+// is exact (squares of fp16 values) and the scalar __fmul_rn (never fused) elsewhere.
+__device__ __forceinline__ unsigned long long f2_mul(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ unsigned long long f2_fma(unsigned long long a, unsigned long long b,
+                                                     unsigned long long c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+// all ones when a > b (false for a NaN operand), else 0
+__device__ __forceinline__ uint32_t gt_mask(float a, float b) {
+  uint32_t d;
+  asm("set.gt.u32.f32 %0, %1, %2;" : "=r"(d) : "f"(a), "f"(b));
+  return d;
+}
+
+// Butterfly stages 1, 2, 4, 8, 16 and 32 of the row transform over one half of the row,
+// held as packed pairs xp[j] = (x_j, x_{j+32}) (half-local indices): stages 1..16 pair
+// registers j and j + hs and so run packed, stage 32 works inside each register.  Each
+// butterfly is (a + b, a - b), rounded to nearest.
+__device__ __forceinline__ void fwht_half(unsigned long long (&xp)[32]) {
+#pragma unroll
+  for (int hs = 1; hs < 32; hs <<= 1) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      if (j & hs) continue;
+      const unsigned long long p0 = xp[j], p1 = xp[j + hs];
+      xp[j] = f2_add(p0, p1);
+      xp[j + hs] = f2_sub(p0, p1);
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    const float lo = f2_lo(xp[j]), hi = f2_hi(xp[j]);
+    xp[j] = f2_pack(__fadd_rn(lo, hi), __fsub_rn(lo, hi));
+  }
+}
+
+// The bit field of one quarter from its 32 codes c_j = m[j] - kOff (kOff: 1.5 * 2^23 for
+// magic-number patterns, 0 for plain codes), as quarter_field.
+template <int L, uint32_t kOff>
+__device__ __forceinline__ void quarter_field_off(const uint32_t (&m)[32], uint32_t (&w)[3]) {
   using F = Fmt<L>;
-  constexpr int kWords = (4 * F::QB + 31) / 32;
-  constexpr int kRecW = (2 * F::RB + (BASE == SEMKV_BASE_TQ ? 4 : 8)) / 4;
-  static_assert(kWords <= 12 && F::QB <= 96, "row image size");
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t cap = hi ? a.hi_cap : a.lo_cap;
-  const int64_t pbase = hi ? a.hi_base : a.lo_base;
-  const int64_t bh = ((int64_t)b * a.NL + l) * a.H + h;
-  // ---- row tid (its 256 bytes arrived in its own slot of the stage; rows past the
-  // block's slots are zeros)
-  float x[128];
-  if ((tid >> 1) < nslots) {
+  w[0] = w[1] = w[2] = 0u;
+  if constexpr (F::G == 1 && F::LG == (1u << F::W)) {
 #pragma unroll
-    for (int ch = 0; ch < 16; ++ch) {
-      const uint4 u = *reinterpret_cast<const uint4*>(stage + tid * kRowStride + ch * 16);
-      const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+    for (int sy = 0; sy < 32; ++sy) put_bits(w, sy * F::W, F::W, m[sy] - kOff);
+  } else {
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
-        x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
+    for (int sy = 0; sy < F::NG; ++sy) {
+      uint32_t t = 0, wsum = 0;
+#pragma unroll
+      for (int k = 0; k < F::G; ++k) {
+        t = t * (uint32_t)L + m[sy * F::G + k];
+        wsum = wsum * (uint32_t)L + 1u;
+      }
+      t -= wsum * kOff;
+      put_bits(w, sy * F::W, F::W, ((t << F::W) + F::LG - 1u) / F::LG);
+    }
+    if constexpr (F::R > 0) {
+      uint32_t t = 0, wsum = 0;
+#pragma unroll
+      for (int k = 0; k < F::R; ++k) {
+        t = t * (uint32_t)L + m[32 - F::R + k];
+        wsum = wsum * (uint32_t)L + 1u;
+      }
+      t -= wsum * kOff;
+      put_bits(w, F::NG * F::W, F::WT, ((t << F::WT) + F::LR - 1u) / F::LR);
+    }
+  }
+}
+
+// TQ codes of both quarters of a half, straight into their bit fields.  u2[j] holds the
+// pair (u of quarter 0, u of quarter 1) at dim j of the quarters; t2[k] the pair
+// (thr_k, thr_k), ascending, with a zero threshold taken as +0.  d = thr_k - u rounds to
+// a value below zero exactly when u > thr_k (binary32 subtraction of unequal values is
+// never zero, and with +0 thresholds an equal pair gives +0), so bit 31 of d is the
+// comparison, and c = sum_k [u > thr_k] is a thermometer code: c = 1 + ... + 1.
+//   L = 2, 4, 8: the code's binary digits from those bits (parities and middles of the
+//   thermometer), shifted into the field most significant bit first, one funnel shift
+//   per bit (code j occupies bits jW .. jW + W - 1 of the field);
+//   other L: c as a sum of the bits, radix groups as quarter_field.
+template <int L>
+__device__ __forceinline__ void tq_fields(const unsigned long long (&u2)[32],
+                                          const unsigned long long (&t2)[7],
+                                          uint32_t (&w0)[3], uint32_t (&w1)[3]) {
+  using F = Fmt<L>;
+  w0[0] = w0[1] = w0[2] = 0u;
+  w1[0] = w1[1] = w1[2] = 0u;
+  if constexpr (F::G == 1 && F::LG == (1u << F::W)) {
+    constexpr int W = F::W;
+    uint32_t a0 = 0u, a1 = 0u;
+#pragma unroll
+    for (int j = 31; j >= 0; --j) {
+      uint32_t dl[7], dh[7];
+#pragma unroll
+      for (int k = 0; k < L - 1; ++k) {
+        const unsigned long long d = f2_sub(t2[k], u2[j]);
+        dl[k] = (uint32_t)d;
+        dh[k] = (uint32_t)(d >> 32);
+      }
+#pragma unroll
+      for (int b = W - 1; b >= 0; --b) {
+        uint32_t bl, bh;
+        if constexpr (L == 2) {
+          bl = dl[0]; bh = dh[0];
+        } else if constexpr (L == 4) {
+          if (b == 1) { bl = dl[1]; bh = dh[1]; }
+          else { bl = dl[0] ^ dl[1] ^ dl[2]; bh = dh[0] ^ dh[1] ^ dh[2]; }
+        } else {
+          if (b == 2) { bl = dl[3]; bh = dh[3]; }
+          else if (b == 1) { bl = dl[1] ^ dl[3] ^ dl[5]; bh = dh[1] ^ dh[3] ^ dh[5]; }
+          else {
+            bl = dl[0] ^ dl[1] ^ dl[2] ^ dl[3] ^ dl[4] ^ dl[5] ^ dl[6];
+            bh = dh[0] ^ dh[1] ^ dh[2] ^ dh[3] ^ dh[4] ^ dh[5] ^ dh[6];
+          }
+        }
+        a0 = __funnelshift_l(bl, a0, 1);
+        a1 = __funnelshift_l(bh, a1, 1);
+        const int pbit = j * W + b;
+        if ((pbit & 31) == 0) {
+          w0[pbit >> 5] = a0;
+          w1[pbit >> 5] = a1;
+        }
       }
     }
   } else {
+    // c = sum of the comparison bits; symbols beta = ceil(t 2^W / L^G) as quarter_field
+    auto code = [&](int j, uint32_t& cl, uint32_t& ch) {
+      cl = 0u; ch = 0u;
 #pragma unroll
-    for (int j = 0; j < 128; ++j) x[j] = 0.0f;
-  }
-  uint32_t param;
-  float zq = 0.0f, invq = 0.0f;  // affine: offset and 1/s;  TQ: 1/n in invq
-  bool live;
-  if constexpr (BASE == SEMKV_BASE_TQ) {
-    // norm of the row with the fixed tree: 32 in-order partials of 4 squares, then the
-    // pairwise stages 16, 8, 4, 2, 1 (partials g and g + 16 formed together, so the
-    // first stage needs 16 registers)
-    float pn[16];
-#pragma unroll
-    for (int g = 0; g < 16; ++g) {
-      float acc[2];
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        const int gg = g + 16 * hh;
-        float v = __fmul_rn(x[4 * gg], x[4 * gg]);
-#pragma unroll
-        for (int k = 1; k < 4; ++k) v = __fadd_rn(v, __fmul_rn(x[4 * gg + k], x[4 * gg + k]));
-        acc[hh] = v;
+      for (int k = 0; k < L - 1; ++k) {
+        const unsigned long long d = f2_sub(t2[k], u2[j]);
+        cl += (uint32_t)d >> 31;
+        ch += (uint32_t)(d >> 32) >> 31;
       }
-      pn[g] = __fadd_rn(acc[0], acc[1]);
+    };
+#pragma unroll
+    for (int sy = 0; sy < F::NG; ++sy) {
+      uint32_t tl = 0u, th = 0u;
+#pragma unroll
+      for (int k = 0; k < F::G; ++k) {
+        uint32_t cl, ch;
+        code(sy * F::G + k, cl, ch);
+        tl = tl * (uint32_t)L + cl;
+        th = th * (uint32_t)L + ch;
+      }
+      put_bits(w0, sy * F::W, F::W, ((tl << F::W) + F::LG - 1u) / F::LG);
+      put_bits(w1, sy * F::W, F::W, ((th << F::W) + F::LG - 1u) / F::LG);
+    }
+    if constexpr (F::R > 0) {
+      uint32_t tl = 0u, th = 0u;
+#pragma unroll
+      for (int k = 0; k < F::R; ++k) {
+        uint32_t cl, ch;
+        code(32 - F::R + k, cl, ch);
+        tl = tl * (uint32_t)L + cl;
+        th = th * (uint32_t)L + ch;
+      }
+      put_bits(w0, F::NG * F::W, F::WT, ((tl << F::WT) + F::LR - 1u) / F::LR);
+      put_bits(w1, F::NG * F::W, F::WT, ((th << F::WT) + F::LR - 1u) / F::LR);
+    }
+  }
+}
+
+// One half of every row of a 64-slot block (see above).  stage: the block's half-row
+// slots (thread tid's 128 bytes at tid * kHalfStride); smask: the (layer, head)'s sign
+// masks, one word per fp16 pair of dims (0x8000 in a half whose sign is -1).
+template <int BASE, int L>
+__device__ void rows_half(const QuantArgs& a, int b, int l, int h, bool hi, int64_t s0,
+                          int nslots, uint8_t* stage, const uint32_t* smask) {
+  using F = Fmt<L>;
+  constexpr int kWords = (4 * F::QB + 31) / 32;
+  constexpr int kRecW = (2 * F::RB + (BASE == SEMKV_BASE_TQ ? 4 : 8)) / 4;
+  constexpr int kSh = (2 * F::QB) & 31;        // bit offset of half 1 in its first word
+  constexpr int kWb = (2 * F::QB) >> 5;        // that word
+  constexpr int kW0 = (2 * F::QB + 31) / 32;   // words half 0 touches
+  constexpr int kW1 = (kSh + 2 * F::QB + 31) / 32;  // words half 1 touches, from kWb
+  static_assert(kWords <= 12 && F::QB <= 96 && kW1 <= 7, "row image size");
+  const int tid = threadIdx.x, f = tid & 1;
+  const int64_t cap = hi ? a.hi_cap : a.lo_cap;
+  const int64_t pbase = hi ? a.hi_base : a.lo_base;
+  const int64_t bh = ((int64_t)b * a.NL + l) * a.H + h;
+  // ---- the half, sign-flipped on its fp16 bits (the signs are +-1), as pairs
+  unsigned long long xp[32];
+  if ((tid >> 2) < nslots) {
+    const uint4* src = reinterpret_cast<const uint4*>(stage + tid * kHalfStride);
+    const uint4* msk = reinterpret_cast<const uint4*>(smask + 32 * f);
+    uint32_t wv[32];
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const uint4 u = src[c], m = msk[c];
+      wv[4 * c] = u.x ^ m.x; wv[4 * c + 1] = u.y ^ m.y;
+      wv[4 * c + 2] = u.z ^ m.z; wv[4 * c + 3] = u.w ^ m.w;
     }
 #pragma unroll
-    for (int off = 8; off >= 1; off >>= 1)
+    for (int j = 0; j < 32; ++j) {
+      const uint32_t lo = wv[j >> 1], hi2 = wv[16 + (j >> 1)];
+      const int sh = 16 * (j & 1);
+      xp[j] = f2_pack(f16_to_f32((uint16_t)(lo >> sh)), f16_to_f32((uint16_t)(hi2 >> sh)));
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) xp[j] = 0ull;
+  }
+  uint32_t param;
+  float invq;  // TQ: 1/n;  affine: 1/s
+  float zq = 0.0f;
+  bool live;
+  if constexpr (BASE == SEMKV_BASE_TQ) {
+    // the norm's fixed tree: 32 in-order partials of 4 squares (this half holds partials
+    // 16f + g in the low lanes, 16f + g + 8 in the high ones), then the pairwise stages
+    // 16 (across the halves), 8, 4, 2, 1
+    // (a square of an fp16 value is exact in binary32, so a fused x * x + v rounds as
+    // the separate multiply and add do)
+    float pn[8];
+#pragma unroll
+    for (int g = 0; g < 8; ++g) {
+      unsigned long long v = f2_mul(xp[4 * g], xp[4 * g]);
+#pragma unroll
+      for (int k = 1; k < 4; ++k) v = f2_add(v, f2_mul(xp[4 * g + k], xp[4 * g + k]));
+      const float plo = __shfl_xor_sync(0xffffffffu, f2_lo(v), 1);
+      const float phi = __shfl_xor_sync(0xffffffffu, f2_hi(v), 1);
+      // partials g + (g + 16) and (g + 8) + (g + 24): the same sums in both halves
+      const unsigned long long sp = f2_add(v, f2_pack(plo, phi));
+      pn[g] = __fadd_rn(f2_lo(sp), f2_hi(sp));
+    }
+#pragma unroll
+    for (int off = 4; off >= 1; off >>= 1)
 #pragma unroll
       for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
     const uint16_t n16 = f16_param(__fsqrt_rn(pn[0]));
@@ -356,25 +551,31 @@ __device__ void rows_block(const QuantArgs& a, int b, int l, int h, bool hi, int
     live = n != 0.0f;
     invq = live ? __fdiv_rn(1.0f, n) : 0.0f;
   }
-  const int8_t* sg = a.signs + ((int64_t)l * a.H + h) * kHeadDim;
+  // ---- butterflies: stages 1..32 in the thread, stage 64 with the partner half.  Half 0
+  // keeps a + b and half 1 a - b (a from half 0): fma(own, +-1, partner), whose product
+  // is exact, rounds partner +- own once, which is that sum or difference.
+  fwht_half(xp);
+  {
+    const float sg = f ? -1.0f : 1.0f;
+    const unsigned long long sg2 = f2_pack(sg, sg);
 #pragma unroll
-  for (int j = 0; j < 32; ++j) {
-    const char4 s4 = __ldg(reinterpret_cast<const char4*>(sg) + j);
-    x[4 * j] *= (float)s4.x;
-    x[4 * j + 1] *= (float)s4.y;
-    x[4 * j + 2] *= (float)s4.z;
-    x[4 * j + 3] *= (float)s4.w;
+    for (int j = 0; j < 32; ++j) {
+      const float plo = __shfl_xor_sync(0xffffffffu, f2_lo(xp[j]), 1);
+      const float phi = __shfl_xor_sync(0xffffffffu, f2_hi(xp[j]), 1);
+      xp[j] = f2_fma(xp[j], sg2, f2_pack(plo, phi));
+    }
   }
-  // ---- Walsh-Hadamard butterflies, stages 1, 2, ..., 64
-  fwht128(x);
   if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
     float mn = INFINITY, mx = -INFINITY;
 #pragma unroll
-    for (int j = 0; j < 128; ++j) {
-      x[j] = __fmul_rn(x[j], kInvSqrtD);
-      mn = fminf(mn, x[j]);
-      mx = fmaxf(mx, x[j]);
+    for (int j = 0; j < 32; ++j) {
+      xp[j] = f2_pack(__fmul_rn(f2_lo(xp[j]), kInvSqrtD), __fmul_rn(f2_hi(xp[j]), kInvSqrtD));
+      mn = fminf(mn, fminf(f2_lo(xp[j]), f2_hi(xp[j])));
+      mx = fmaxf(mx, fmaxf(f2_lo(xp[j]), f2_hi(xp[j])));
     }
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, 1));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+    // a zero extreme is taken as +0 (min/max may return either signed zero)
     if (mn == 0.0f) mn = 0.0f;
     if (mx == 0.0f) mx = 0.0f;
     uint16_t z16 = __half_as_ushort(__float2half_rd(mn));
@@ -383,74 +584,96 @@ __device__ void rows_block(const QuantArgs& a, int b, int l, int h, bool hi, int
     const uint16_t s16 = f16_param(__fdiv_rn(__fsub_rn(mx, zq), (float)(L - 1)));
     const float sv = f16_to_f32(s16);
     live = sv > 0.0f;
+    // 1/s, or 0 when s == 0: then every (u - z) * 0 clamps and rounds to code 0
     invq = live ? __fdiv_rn(1.0f, sv) : 0.0f;
     param = (uint32_t)s16 | ((uint32_t)z16 << 16);
   }
-  // ---- codes, quarter by quarter, as magic-number patterns 1.5 * 2^23 + c
-  uint32_t w[12];
+  // ---- codes, quarter 2f from the low lanes, then quarter 2f + 1 from the high ones
+  uint32_t lw[7];
 #pragma unroll
-  for (int k = 0; k < 12; ++k) w[k] = 0u;
-  const bool hi_row = hi;  // (the level count is the pool's)
-  (void)hi_row;
-  float thr[7];
+  for (int k = 0; k < 7; ++k) lw[k] = 0u;
+  const unsigned long long inv2 = f2_pack(invq, invq);
   if constexpr (BASE == SEMKV_BASE_TQ) {
+    // c = #{k : u > thr_k} (ties go low); a zero-norm row compares against +inf
     const float* tg = hi ? a.thr_hi : a.thr_lo;
+    unsigned long long t2[7];
 #pragma unroll
-    for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? tg[k] : INFINITY;
-  }
+    for (int k = 0; k < L - 1; ++k) {
+      const float tk = live ? __fadd_rn(__ldg(tg + k), 0.0f) : INFINITY;
+      t2[k] = f2_pack(tk, tk);
+    }
+    // u = y * fl(1/n), rounded before the comparisons subtract it
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    uint32_t m[32];
+    for (int j = 0; j < 32; ++j) xp[j] = f2_pack(__fmul_rn(f2_lo(xp[j]), invq), __fmul_rn(f2_hi(xp[j]), invq));
+    uint32_t fw0[3], fw1[3];
+    tq_fields<L>(xp, t2, fw0, fw1);
+    or_field<7>(lw, 0, fw0);
+    or_field<7>(lw, F::QB, fw1);
+  } else {
+    // rint(clamp((u - z) / s)) = clamp(rint(...)) for integer bounds; + 1.5 * 2^23 rounds
+    // to nearest even and leaves the code in the low bits of the pattern
+    const unsigned long long z2 = f2_pack(zq, zq);
+    const unsigned long long mg2 = f2_pack(12582912.0f, 12582912.0f);
 #pragma unroll
     for (int j = 0; j < 32; ++j) {
-      const float xv = x[32 * q + j];
-      if constexpr (BASE == SEMKV_BASE_TQ) {
-        const float u = __fmul_rn(xv, invq);
-        int c = 0;
-#pragma unroll
-        for (int k = 0; k < L - 1; ++k) c += (u > thr[k]) ? 1 : 0;
-        m[j] = 0x4B400000u + (uint32_t)(live ? c : 0);
-      } else {
-        // rint(clamp(v)) = clamp(rint(v)) for integer bounds; + 1.5 * 2^23 rounds to even
-        const float y = fminf(fmaxf(__fmul_rn(__fsub_rn(xv, zq), invq), 0.0f), (float)(L - 1));
-        m[j] = live ? __float_as_uint(__fadd_rn(y, 12582912.0f)) : 0x4B400000u;
-      }
+      const unsigned long long d = f2_mul(f2_sub(xp[j], z2), inv2);
+      const float ylo = fminf(fmaxf(f2_lo(d), 0.0f), (float)(L - 1));
+      const float yhi = fminf(fmaxf(f2_hi(d), 0.0f), (float)(L - 1));
+      xp[j] = f2_add(f2_pack(ylo, yhi), mg2);
     }
-    uint32_t fw[3];
-    quarter_field<L>(m, fw);
-    or_field<12>(w, q * F::QB, fw);
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      uint32_t m[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) m[j] = __float_as_uint(q ? f2_hi(xp[j]) : f2_lo(xp[j]));
+      uint32_t fw[3];
+      quarter_field_off<L, 0x4B400000u>(m, fw);
+      or_field<7>(lw, q * F::QB, fw);
+    }
   }
-  // the row's bit image and parameters go to its own slot (its values are in registers)
-  uint32_t* mine = reinterpret_cast<uint32_t*>(stage + tid * kRowStride);
+  // ---- the row's bit image and parameters, in half 0's slot: half 0 writes words
+  // 0..kWb (word kWb with half 1's low bits when half 1 starts inside it), half 1 the rest
+  uint32_t* img = reinterpret_cast<uint32_t*>(stage + (tid & ~1) * kHalfStride);
+  if constexpr (kSh != 0) {
 #pragma unroll
-  for (int k = 0; k < kWords; ++k) mine[k] = w[k];
-  mine[kRowBitWords] = param;
-  __syncthreads();
-  // ---- records: warp takes slots warp, warp + 4, ...; lane j writes word j
-  uint32_t* recs = reinterpret_cast<uint32_t*>(hi ? a.hi_pool : a.lo_pool) + (bh * cap + pbase + s0) * kRecW;
-  for (int i = warp; i < nslots; i += 4) {
-    for (int j = lane; j < kRecW; j += 32) {
-      uint32_t word = 0u;
-      if (4 * j >= 2 * F::RB) {
-        const int pj = j - (2 * F::RB) / 4;
-        const uint32_t p0 = reinterpret_cast<const uint32_t*>(stage + (2 * i) * kRowStride)[kRowBitWords];
-        const uint32_t p1 = reinterpret_cast<const uint32_t*>(stage + (2 * i + 1) * kRowStride)[kRowBitWords];
-        if constexpr (BASE == SEMKV_BASE_TQ) word = p0 | (p1 << 16);
-        else word = pj ? p1 : p0;
-      } else {
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int byte = 4 * j + e;
-          const int row = byte < F::RB ? 2 * i : 2 * i + 1;
-          const int rb = byte < F::RB ? byte : byte - F::RB;
-          const uint32_t v = rb < F::RB ? (reinterpret_cast<const uint32_t*>(stage + row * kRowStride)[rb >> 2] >>
-                                           (8 * (rb & 3))) & 0xFFu
-                                        : 0u;
-          word |= v << (8 * e);
-        }
-      }
-      recs[(int64_t)i * kRecW + j] = word;
+    for (int k = kW1 - 1; k >= 0; --k) {
+      const uint32_t v = (lw[k] << kSh) | (k > 0 ? lw[k - 1] >> (32 - kSh) : 0u);
+      if (f) lw[k] = v;
     }
+  }
+  const uint32_t first1 = __shfl_xor_sync(0xffffffffu, lw[0], 1);
+  __syncwarp();  // both halves' values were read from the slots
+  if ((tid >> 2) < nslots) {
+    if (f == 0) {
+#pragma unroll
+      for (int k = 0; k < kW0; ++k) img[k] = (kSh != 0 && k == kWb) ? (lw[k] | first1) : lw[k];
+      img[kRowBitWords] = param;
+    } else {
+#pragma unroll
+      for (int k = (kSh != 0 ? 1 : 0); k < kW1; ++k) img[kWb + k] = lw[k];
+    }
+  }
+  __syncthreads();
+  // ---- records: the block's words in order, one 4-byte word per thread and step
+  uint32_t* recs = reinterpret_cast<uint32_t*>(hi ? a.hi_pool : a.lo_pool) + (bh * cap + pbase + s0) * kRecW;
+  const int nw = nslots * kRecW;
+  for (int wi = tid; wi < nw; wi += kRows2Threads) {
+    const int i = wi / kRecW, j = wi - i * kRecW;
+    const uint32_t* K = reinterpret_cast<const uint32_t*>(stage + (4 * i) * kHalfStride);
+    const uint32_t* V = reinterpret_cast<const uint32_t*>(stage + (4 * i + 2) * kHalfStride);
+    uint32_t word;
+    if (4 * j >= 2 * F::RB) {
+      const int pj = j - (2 * F::RB) / 4;
+      if constexpr (BASE == SEMKV_BASE_TQ) word = K[kRowBitWords] | (V[kRowBitWords] << 16);
+      else word = pj ? V[kRowBitWords] : K[kRowBitWords];
+    } else if (4 * j + 4 <= F::RB) {
+      word = K[j];
+    } else {
+      const int vb = 4 * j - F::RB;  // byte of the V row at this word's first byte
+      if (vb >= 0) word = __funnelshift_r(V[vb >> 2], V[(vb >> 2) + 1], 8 * (vb & 3));
+      else word = K[j] | (V[0] << (8 * -vb));
+    }
+    recs[wi] = word;
   }
   __syncthreads();  // the stage is free for the copies of a later block
 }
@@ -494,78 +717,102 @@ __device__ __forceinline__ void bulk_g2s_row(void* dst, const void* src, uint64_
       : "memory");
 }
 
-// block t of the pass: (sequence, layer, head) index, pool, first slot, slot count
+// block t of the pass, decoded once: (sequence, layer, KV head), pool, first slot and
+// slot count (32-bit arithmetic: the launcher keeps the block count below 2^31)
 struct RowsTile {
-  int bhi;
+  int b, l, h;
   bool hi;
-  int64_t s0;
-  int nslots;
+  int s0, nslots;
 };
-__device__ __forceinline__ RowsTile rows_tile(int64_t t, int64_t n_hi, int64_t n_lo) {
-  const int64_t nb_hi = (n_hi + kRowSlots - 1) / kRowSlots;
-  const int64_t nb_lo = (n_lo + kRowSlots - 1) / kRowSlots;
-  const int64_t r = t % (nb_hi + nb_lo);
+__device__ __forceinline__ RowsTile rows_tile(uint32_t t, uint32_t nb_hi, uint32_t per_bh,
+                                              uint32_t n_hi, uint32_t n_lo, uint32_t H,
+                                              uint32_t NL) {
   RowsTile x;
-  x.bhi = (int)(t / (nb_hi + nb_lo));
+  const uint32_t bhi = t / per_bh, r = t - bhi * per_bh;
   x.hi = r < nb_hi;
-  x.s0 = (x.hi ? r : r - nb_hi) * kRowSlots;
-  x.nslots = (int)min((int64_t)kRowSlots, (x.hi ? n_hi : n_lo) - x.s0);
+  x.s0 = (int)((x.hi ? r : r - nb_hi) * kRowSlots);
+  x.nslots = min(kRowSlots, (int)(x.hi ? n_hi : n_lo) - x.s0);
+  const uint32_t q = bhi / H;
+  x.h = (int)(bhi - q * H);
+  x.b = (int)(q / NL);
+  x.l = (int)(q - (uint32_t)x.b * NL);
   return x;
 }
 
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dsmem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Persistent CTAs of 256 threads over the blocks (64 slots of one pool of one (sequence,
+// layer, KV head)), in a two-stage pipeline: while a block is quantized, the halves of
+// the CTA's next block are already on their way.  Thread tid brings half tid & 1 of its
+// row into its own slot of the stage with eight 16-byte cp.async copies (one commit
+// group per block), and the first 64 threads write the next block's sign masks; a
+// thread waits for its own group, then the CTA barrier publishes the stage.
 template <int BASE>
-__global__ void __launch_bounds__(128, 3) quantize_rows_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
-  extern __shared__ __align__(128) uint8_t rstage[];  // 2 stages of 128 row slots
-  __shared__ __align__(8) uint64_t rbar[2];
+__global__ void __launch_bounds__(kRows2Threads, rows2_ctas(BASE)) quantize_rows_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
+  extern __shared__ __align__(128) uint8_t rstage[];  // 2 stages of 256 half-row slots
+  __shared__ __align__(16) uint32_t smask[2][64];
   const int tid = threadIdx.x;
-  if (tid < 2) rbar_init128(&rbar[tid]);
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  __syncthreads();
-  const int64_t bhs = (int64_t)a.B * a.NL * a.H;
-  const int64_t per_bh = (n_hi + kRowSlots - 1) / kRowSlots + (n_lo + kRowSlots - 1) / kRowSlots;
-  const int64_t total = bhs * per_bh;
-  // this thread's row of block t into stage st
-  auto issue = [&](int64_t t, int st) {
-    const RowsTile x = rows_tile(t, n_hi, n_lo);
-    const int i = tid >> 1;
-    if (i < x.nslots) {
-      const int h = x.bhi % a.H, l = (x.bhi / a.H) % a.NL, b = x.bhi / (a.H * a.NL);
-      const int64_t cap = x.hi ? a.hi_cap : a.lo_cap;
-      const int32_t* tokmap = (x.hi ? a.hi_tok : a.lo_tok) + (int64_t)b * cap + (x.hi ? a.hi_base : a.lo_base);
-      const int64_t tk = (int64_t)tokmap[x.s0 + i] - a.tok_base;
-      const int64_t bh = ((int64_t)b * a.NL + l) * a.H + h;
-      const uint16_t* src = ((tid & 1) ? a.v : a.k) + (bh * a.Tsrc + tk) * kHeadDim;
-      // this slot was last read (and written) through the generic proxy
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      rbar_arrive(&rbar[st], 256u);
-      bulk_g2s_row(rstage + st * kRowStageBytes + tid * kRowStride, src, &rbar[st]);
-    } else {
-      rbar_arrive(&rbar[st], 0u);
-    }
+  const uint32_t nb_hi = (uint32_t)((n_hi + kRowSlots - 1) / kRowSlots);
+  const uint32_t per_bh = nb_hi + (uint32_t)((n_lo + kRowSlots - 1) / kRowSlots);
+  const uint32_t total = (uint32_t)a.B * a.NL * a.H * per_bh;
+  auto tile = [&](uint32_t t) {
+    return rows_tile(t, nb_hi, per_bh, (uint32_t)n_hi, (uint32_t)n_lo, a.H, a.NL);
   };
-  int64_t t = blockIdx.x;
-  if (t < total) issue(t, 0);
+  // this thread's half row of block x into stage st (and, for tid < 64, a sign mask word)
+  auto issue = [&](const RowsTile& x, int st) {
+    if (tid < 64) {
+      const char2 s2 = *reinterpret_cast<const char2*>(a.signs + ((int64_t)x.l * a.H + x.h) * kHeadDim + 2 * tid);
+      smask[st][tid] = (s2.x < 0 ? 0x8000u : 0u) | (s2.y < 0 ? 0x80000000u : 0u);
+    }
+    const int i = tid >> 2;
+    if (i < x.nslots) {
+      const int64_t cap = x.hi ? a.hi_cap : a.lo_cap;
+      const int32_t* tokmap = (x.hi ? a.hi_tok : a.lo_tok) + (int64_t)x.b * cap + (x.hi ? a.hi_base : a.lo_base);
+      const int64_t tk = (int64_t)tokmap[x.s0 + i] - a.tok_base;
+      const int64_t bh = ((int64_t)x.b * a.NL + x.l) * a.H + x.h;
+      const uint16_t* src = (((tid >> 1) & 1) ? a.v : a.k) + (bh * a.Tsrc + tk) * kHeadDim + 64 * (tid & 1);
+      uint8_t* dst = rstage + st * kRows2StageBytes + tid * kHalfStride;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) cp_async16(dst + 16 * c, src + 8 * c);
+    }
+    cp_async_commit();
+  };
+  uint32_t t = blockIdx.x;
+  RowsTile cur{};
+  if (t < total) {
+    cur = tile(t);
+    issue(cur, 0);
+  }
   for (int k = 0; t < total; t += gridDim.x, ++k) {
     const int st = k & 1;
-    const bool next = t + gridDim.x < total;
-    if (next) issue(t + gridDim.x, st ^ 1);
-    if (!__syncthreads_and(dbar_wait(&rbar[st], (uint32_t)((k >> 1) & 1)))) {
-      // a copy never landed: record it, let the other stage's copies finish, stop
-      if (tid == 0) raise_error(a.err, kDevWaitTimeout);
-      if (next) dbar_wait(&rbar[st ^ 1], (uint32_t)(((k + 1) >> 1) & 1));
-      return;
+    RowsTile nxt{};
+    if (t + gridDim.x < total) {
+      nxt = tile(t + gridDim.x);
+      issue(nxt, st ^ 1);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
     }
-    const RowsTile x = rows_tile(t, n_hi, n_lo);
-    const int h = x.bhi % a.H, l = (x.bhi / a.H) % a.NL, b = x.bhi / (a.H * a.NL);
-    uint8_t* stage = rstage + st * kRowStageBytes;
-    switch (x.hi ? a.L_hi : a.L_lo) {
+    __syncthreads();
+    uint8_t* stage = rstage + st * kRows2StageBytes;
+    switch (cur.hi ? a.L_hi : a.L_lo) {
 #define SEMKV_ROWS_CASE(LV) \
-      case LV: rows_block<BASE, LV>(a, b, l, h, x.hi, x.s0, x.nslots, stage); break;
+      case LV: rows_half<BASE, LV>(a, cur.b, cur.l, cur.h, cur.hi, cur.s0, cur.nslots, stage, smask[st]); break;
       SEMKV_ROWS_CASE(2) SEMKV_ROWS_CASE(3) SEMKV_ROWS_CASE(4) SEMKV_ROWS_CASE(5)
       SEMKV_ROWS_CASE(6) SEMKV_ROWS_CASE(7) SEMKV_ROWS_CASE(8)
 #undef SEMKV_ROWS_CASE
-      default: break;
+      default: __syncthreads(); break;
     }
+    cur = nxt;
   }
 }
 // ------------------------------------------------- fake quantization ---------
@@ -1263,32 +1510,33 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  // persistent CTAs (3 per SM) over every block of both pools
+  // persistent CTAs (rows2_ctas per SM) over every block of both pools
   const int64_t bhs = (int64_t)a.B * a.NL * a.H;
   const int64_t blocks = bhs * ((n_hi + kRowSlots - 1) / kRowSlots +
                                 (a.n - n_hi + kRowSlots - 1) / kRowSlots);
-  int64_t ctas = (int64_t)(num_sms > 0 ? num_sms : 1) * 3;
+  int64_t ctas = (int64_t)(num_sms > 0 ? num_sms : 1) * rows2_ctas(a.base);
   if (ctas > blocks) ctas = blocks;
   if (ctas < 1) return cudaSuccess;
+  if (blocks + ctas > INT32_MAX) return cudaErrorInvalidValue;  // block indices are 32-bit
   static bool rows_attr[kAttrDevices] = {};
   {
     const cudaError_t e = once_per_device(rows_attr, [] {
       cudaError_t r = cudaFuncSetAttribute(quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           2 * kRowStageBytes);
+                                           2 * kRows2StageBytes);
       if (r == cudaSuccess)
         r = cudaFuncSetAttribute(quantize_rows_kernel<SEMKV_BASE_TQ>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kRowStageBytes);
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kRows2StageBytes);
       return r;
     });
     if (e != cudaSuccess) return e;
   }
   if (a.base == SEMKV_BASE_AFFINE_HAD)
-    quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)ctas, 128, 2 * kRowStageBytes, stream>>>(
-        a, n_hi, a.n - n_hi);
+    quantize_rows_kernel<SEMKV_BASE_AFFINE_HAD>
+        <<<(unsigned)ctas, kRows2Threads, 2 * kRows2StageBytes, stream>>>(a, n_hi, a.n - n_hi);
   else
-    quantize_rows_kernel<SEMKV_BASE_TQ><<<(unsigned)ctas, 128, 2 * kRowStageBytes, stream>>>(
-        a, n_hi, a.n - n_hi);
+    quantize_rows_kernel<SEMKV_BASE_TQ>
+        <<<(unsigned)ctas, kRows2Threads, 2 * kRows2StageBytes, stream>>>(a, n_hi, a.n - n_hi);
   return cudaGetLastError();
 }
 

@@ -71,10 +71,11 @@ def test_quantize_pack_bit_exact(base, L_hi, L_lo, B, NL, H, T, r):
     assert int(p.cache.dev_error.item()) == 0
 
 
-@pytest.mark.parametrize("base", [0, 2])
+@pytest.mark.parametrize("base", [0, 1, 2])
 def test_quantize_edge_rows_bit_exact(base):
     # constant rows, signed zeros, tiny (subnormal-step) ranges and huge ranges (for the
-    # rotated base the rotated range passes 65504: the offset and scale saturate)
+    # rotated base the rotated range passes 65504: the offset and scale saturate; for TQ
+    # the norm saturates and a zero row has norm 0, all codes 0)
     p = Pair(base, 6, 5, 1, 1, 2, 8, 64, 1, 2, seed=3)
     k = p.k.astype(np.float32)
     v = p.v.astype(np.float32)
@@ -87,6 +88,47 @@ def test_quantize_edge_rows_bit_exact(base):
     v[0, 0, 1, 5, 0] = 65504.0
     v[0, 0, 1, 5, 1] = -65504.0
     p.k, p.v = k.astype(np.float16), v.astype(np.float16)
+    p.quantize()
+    p.assert_records_equal()
+
+
+# TQ rows in which some u = y * fl(1/n) equals a codebook threshold exactly (found by a
+# search over seeded inputs: token, dim).  Ties go low (Sec. 4.9's quantizer compares
+# strictly), and in the rows marked + the exact product y * fl(1/n) lies above the
+# threshold, so a quantizer that fused the multiply into its comparison would round the
+# code up there.
+@pytest.mark.parametrize("seed,L,row,tok,dim", [
+    (21, 4, "v", 1214, 122),     # +
+    (27, 4, "v", 866, 73),       # +
+    (104, 4, "k", 2720, 122),    # +
+    (110, 4, "v", 1758, 125),    # +
+    (15, 4, "v", 563, 8),
+    (153, 3, "k", 3621, 35),     # +
+    (197, 3, "k", 2525, 115),    # +
+    (62, 3, "k", 1718, 61),
+])
+def test_tq_threshold_ties_bit_exact(seed, L, row, tok, dim):
+    p = Pair(1, L, L, 1, 1, 1, 4, 4096, 1, 1, seed=seed)
+    # the input still holds the tie: u at (tok, dim) equals a threshold
+    x = (p.k if row == "k" else p.v)[0, 0, 0, tok].astype(np.float32)
+    w = x * synthetic.signs(seed, 1, 1)[0, 0].astype(np.float32)
+    hs = 1
+    while hs < 128:
+        i = np.arange(128)[(np.arange(128) & hs) == 0]
+        a, b = w[i].copy(), w[i + hs].copy()
+        w[i], w[i + hs] = a + b, a - b
+        hs <<= 1
+    sq = x * x
+    part = sq[0::4].copy()
+    for k in range(1, 4):
+        part = part + sq[k::4]
+    pn = part[:16] + part[16:]
+    while len(pn) > 1:
+        pn = pn[:len(pn) // 2] + pn[len(pn) // 2:]
+    n = np.float32(np.float16(np.sqrt(pn[0])))
+    u = np.float32(w[dim] * (np.float32(1) / n))
+    _, _, thr, _ = oracle.lloyd_max_gaussian(L)
+    assert u in thr.astype(np.float32)
     p.quantize()
     p.assert_records_equal()
 
