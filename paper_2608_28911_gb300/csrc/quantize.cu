@@ -653,12 +653,15 @@ __device__ void rows_half(const QuantArgs& a, int b, int l, int h, bool hi, int6
       for (int k = (kSh != 0 ? 1 : 0); k < kW1; ++k) img[kWb + k] = lw[k];
     }
   }
-  __syncthreads();
-  // ---- records: the block's words in order, one 4-byte word per thread and step
-  uint32_t* recs = reinterpret_cast<uint32_t*>(hi ? a.hi_pool : a.lo_pool) + (bh * cap + pbase + s0) * kRecW;
-  const int nw = nslots * kRecW;
-  for (int wi = tid; wi < nw; wi += kRows2Threads) {
-    const int i = wi / kRecW, j = wi - i * kRecW;
+  // ---- records: slot i's two rows are threads 4i .. 4i + 3, so each warp assembles its
+  // own 8 slots' records (contiguous words, one 4-byte word per lane and step)
+  __syncwarp();
+  const int warp = tid >> 5, lane = tid & 31;
+  const int ns = min(8, nslots - 8 * warp);
+  uint32_t* recs = reinterpret_cast<uint32_t*>(hi ? a.hi_pool : a.lo_pool) +
+                   (bh * cap + pbase + s0 + 8 * warp) * kRecW;
+  for (int wi = lane; wi < ns * kRecW; wi += 32) {
+    const int i = 8 * warp + wi / kRecW, j = wi - (wi / kRecW) * kRecW;
     const uint32_t* K = reinterpret_cast<const uint32_t*>(stage + (4 * i) * kHalfStride);
     const uint32_t* V = reinterpret_cast<const uint32_t*>(stage + (4 * i + 2) * kHalfStride);
     uint32_t word;
@@ -675,7 +678,6 @@ __device__ void rows_half(const QuantArgs& a, int b, int l, int h, bool hi, int6
     }
     recs[wi] = word;
   }
-  __syncthreads();  // the stage is free for the copies of a later block
 }
 
 // ---- mbarriers
@@ -755,7 +757,8 @@ __device__ __forceinline__ void cp_async_wait() {
 // the CTA's next block are already on their way.  Thread tid brings half tid & 1 of its
 // row into its own slot of the stage with eight 16-byte cp.async copies (one commit
 // group per block), and the first 64 threads write the next block's sign masks; a
-// thread waits for its own group, then the CTA barrier publishes the stage.
+// thread waits for its own group, then the CTA barrier (the only one per block)
+// publishes the stage.
 template <int BASE>
 __global__ void __launch_bounds__(kRows2Threads, rows2_ctas(BASE)) quantize_rows_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
   extern __shared__ __align__(128) uint8_t rstage[];  // 2 stages of 256 half-row slots
@@ -794,15 +797,16 @@ __global__ void __launch_bounds__(kRows2Threads, rows2_ctas(BASE)) quantize_rows
   }
   for (int k = 0; t < total; t += gridDim.x, ++k) {
     const int st = k & 1;
+    // this thread's copies of block k have landed; after the barrier every thread's have,
+    // and every warp is done with the other stage (block k - 1), which the copies of
+    // block k + 1 then take over
+    cp_async_wait<0>();
+    __syncthreads();
     RowsTile nxt{};
     if (t + gridDim.x < total) {
       nxt = tile(t + gridDim.x);
       issue(nxt, st ^ 1);
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
     }
-    __syncthreads();
     uint8_t* stage = rstage + st * kRows2StageBytes;
     switch (cur.hi ? a.L_hi : a.L_lo) {
 #define SEMKV_ROWS_CASE(LV) \
@@ -810,7 +814,7 @@ __global__ void __launch_bounds__(kRows2Threads, rows2_ctas(BASE)) quantize_rows
       SEMKV_ROWS_CASE(2) SEMKV_ROWS_CASE(3) SEMKV_ROWS_CASE(4) SEMKV_ROWS_CASE(5)
       SEMKV_ROWS_CASE(6) SEMKV_ROWS_CASE(7) SEMKV_ROWS_CASE(8)
 #undef SEMKV_ROWS_CASE
-      default: __syncthreads(); break;
+      default: break;
     }
     cur = nxt;
   }
