@@ -323,12 +323,6 @@ __device__ __forceinline__ unsigned long long f2_fma(unsigned long long a, unsig
   asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
   return d;
 }
-// all ones when a > b (false for a NaN operand), else 0
-__device__ __forceinline__ uint32_t gt_mask(float a, float b) {
-  uint32_t d;
-  asm("set.gt.u32.f32 %0, %1, %2;" : "=r"(d) : "f"(a), "f"(b));
-  return d;
-}
 
 // Butterfly stages 1, 2, 4, 8, 16 and 32 of the row transform over one half of the row,
 // held as packed pairs xp[j] = (x_j, x_{j+32}) (half-local indices): stages 1..16 pair
@@ -1099,27 +1093,29 @@ __global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : 3) fake_rows_
 }
 
 // ------------------------------------- dense-rotation TQ rows (tcgen05) --------
-// Persistent CTAs of 8 warps (two per SM), each over a contiguous range of 64-token
-// tiles of one (sequence, layer, KV head).  The head's rotation M (128 x 128 fp16, the
-// A operand) is staged once per CTA.  The K and V rows of a tile arrive by TMA, one 3-D
-// tensor copy each (dims: 8 values, rows, 16 groups of 8 values), so they land as
-// 8-row x 16-byte core matrices, K-major without swizzle, completing on an mbarrier;
-// the next tile's copy starts as soon as the MMAs have read the current one, under the
-// codes and the packing.  One thread issues D^T = M X^T on tcgen05 (kind::f16,
-// M = 128 output dims, N = 64 tokens, K = 8 x 16) for the K rows and for the V rows into
-// 128 fp32 columns of tensor memory and commits to an mbarrier.  Meanwhile the threads
-// take the rows' fixed-tree norms from the tile (two threads per row); then warp w
-// reads TMEM lanes 32 (w % 4).. (output dims) of the K (w < 4) or V (w >= 4) columns,
-// writes the codes into a row-major code tile; a thread per row builds the row's
-// bit image (the quarter fields) and the warps write the records word by word.
-constexpr int kDenseTok = 64;
+// Blocks of 64 slots of one pool of one (sequence, layer, KV head), as for the other
+// bases: 128 rows (row r: K of slot r/2 when r is even, V when odd), one level count.
+// Persistent CTAs of two groups of 4 warps (two CTAs per SM), each CTA over a range of
+// blocks of one (sequence, layer, KV head) whose rotation M (128 x 128 fp16, the B
+// operand, K-major: output dims x input dims) it stages once.  A group takes every other
+// block of the range: thread r of the group brings row r with sixteen 16-byte cp.async
+// copies into the group's A tile (K-major 8-row x 16-byte core matrices: byte
+// kg * 2048 + r * 16 holds dims 8 kg .. 8 kg + 7), then one thread issues
+// D = X M^T on tcgen05 (kind::f16, M = 128 rows, N = 128 output dims, K = 8 x 16) into
+// the group's 128 columns of tensor memory, so TMEM lane r is row r and column c its
+// output dim c.  While the MMAs run, thread r takes its row's fixed-tree norm from the
+// tile; once they have completed it starts the copies of the group's next block and
+// reads its row's w = M x a quarter (32 columns) at a time: u = w * fl(1/n), the codes
+// from the thresholds, the quarter bit fields, and the row's bytes straight into its
+// record.  The two groups' accumulators are distinct, so one group's MMAs overlap the
+// other's epilogue.
 constexpr int kDenseThreads = 256;
 constexpr uint32_t kDenseM = 128 * 128 * 2;   // the rotation, bytes
-constexpr uint32_t kDenseBox = 64 * 128 * 2;  // one TMA box: 64 rows of K or of V
-constexpr uint32_t kDenseSmem = kDenseM + 2 * kDenseBox + 128 * 128 + 1024;  // + codes, align
+constexpr uint32_t kDenseA = 128 * 128 * 2;   // one group's tile of 128 rows
+constexpr uint32_t kDenseSmem = kDenseM + 2 * kDenseA + 1024;  // + alignment
 // instruction descriptor: fp32 accumulate (bits 4-5 = 1), A and B fp16 (formats 0),
 // both K-major, N >> 3 at bits 17-22, M >> 4 at bits 24-28
-constexpr uint32_t kDenseIdesc = (1u << 4) | ((64u >> 3) << 17) | ((128u >> 4) << 24);
+constexpr uint32_t kDenseIdesc = (1u << 4) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
 
 // shared-memory matrix descriptor without swizzle: start >> 4 (bits 0-13), leading
 // (K-direction) core-matrix offset >> 4 (bits 16-29), stride (8-row group) offset >> 4
@@ -1141,68 +1137,153 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
       : "r"(taddr));
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+// barrier of the 128 threads of group g (named barrier 1 + g), with an AND of p
+__device__ __forceinline__ bool group_sync_and(int g, bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n"
+      " barrier.cta.red.and.pred q, %2, 128, p;\n selp.u32 %0, 1, 0, q;\n}"
+      : "=r"(r)
+      : "r"((uint32_t)p), "r"(1 + g)
+      : "memory");
+  return r != 0;
+}
 
-// the bit image of one row of 128 codes (bytes) as the record stores it
+// The field of one quarter from its 32 values u (thresholds as in tq_fields: t2[k] the
+// pair (thr_k, thr_k)); pairs of neighbouring dims share each packed subtraction.
 template <int L>
-__device__ __forceinline__ void row_bits(const uint8_t* crow, uint32_t* out) {
+__device__ __forceinline__ void tq_quarter(const float (&u)[32], const unsigned long long (&t2)[7],
+                                           uint32_t (&w)[3]) {
   using F = Fmt<L>;
-  constexpr int kWords = (4 * F::QB + 31) / 32;
-  uint32_t w[12];
+  w[0] = w[1] = w[2] = 0u;
+  if constexpr (F::G == 1 && F::LG == (1u << F::W)) {
+    constexpr int W = F::W;
+    uint32_t acc = 0u;
 #pragma unroll
-  for (int k = 0; k < 12; ++k) w[k] = 0u;
+    for (int jp = 15; jp >= 0; --jp) {
+      uint32_t dl[7], dh[7];
+#pragma unroll
+      for (int k = 0; k < L - 1; ++k) {
+        const unsigned long long d = f2_sub(t2[k], f2_pack(u[2 * jp], u[2 * jp + 1]));
+        dl[k] = (uint32_t)d;
+        dh[k] = (uint32_t)(d >> 32);
+      }
+#pragma unroll
+      for (int e = 1; e >= 0; --e) {  // dim 2jp + 1 first: most significant bit first
+        const uint32_t* dd = e ? dh : dl;
+        const int j = 2 * jp + e;
+#pragma unroll
+        for (int b = W - 1; b >= 0; --b) {
+          uint32_t bit;
+          if constexpr (L == 2) bit = dd[0];
+          else if constexpr (L == 4) bit = b == 1 ? dd[1] : (dd[0] ^ dd[1] ^ dd[2]);
+          else bit = b == 2 ? dd[3] : b == 1 ? (dd[1] ^ dd[3] ^ dd[5])
+                                             : (dd[0] ^ dd[1] ^ dd[2] ^ dd[3] ^ dd[4] ^ dd[5] ^ dd[6]);
+          acc = __funnelshift_l(bit, acc, 1);
+          const int pbit = j * W + b;
+          if ((pbit & 31) == 0) w[pbit >> 5] = acc;
+        }
+      }
+    }
+  } else {
+    uint32_t t = 0u;
+#pragma unroll
+    for (int jp = 0; jp < 16; ++jp) {
+      uint32_t c[2] = {0u, 0u};
+#pragma unroll
+      for (int k = 0; k < L - 1; ++k) {
+        const unsigned long long d = f2_sub(t2[k], f2_pack(u[2 * jp], u[2 * jp + 1]));
+        c[0] += (uint32_t)d >> 31;
+        c[1] += (uint32_t)(d >> 32) >> 31;
+      }
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int j = 2 * jp + e;
+        if (j < F::NG * F::G) {
+          const int k = j % F::G, sy = j / F::G;
+          t = (k == 0 ? 0u : t * (uint32_t)L) + c[e];
+          if (k == F::G - 1) put_bits(w, sy * F::W, F::W, ((t << F::W) + F::LG - 1u) / F::LG);
+        } else {
+          const int k = j - F::NG * F::G;
+          t = (k == 0 ? 0u : t * (uint32_t)L) + c[e];
+          if (k == F::R - 1) put_bits(w, F::NG * F::W, F::WT, ((t << F::WT) + F::LR - 1u) / F::LR);
+        }
+      }
+    }
+  }
+}
+
+// Row r of a block: codes from TMEM (taddr: this warp's lanes, the group's columns), the
+// quarter fields, and the row's bytes into its record (rec: the record; kind 0 = K at
+// byte 0, 1 = V at byte RB; its fp16 norm at byte 2 RB + 2 kind)
+template <int L>
+__device__ __forceinline__ void dense_row(uint32_t taddr, const float* thr, float inv, bool live,
+                                          uint16_t n16, uint8_t* rec, int kind, bool store) {
+  using F = Fmt<L>;
+  constexpr int RB = F::RB;
+  unsigned long long t2[7];
+#pragma unroll
+  for (int k = 0; k < L - 1; ++k) {
+    const float tk = live ? __fadd_rn(__ldg(thr + k), 0.0f) : INFINITY;
+    t2[k] = f2_pack(tk, tk);
+  }
+  uint32_t w[13];
+#pragma unroll
+  for (int k = 0; k < 13; ++k) w[k] = 0u;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    uint32_t m[32];
+    uint32_t v[32];
+    tmem_ld32(taddr + 32 * q, v);
+    float u[32];
+    // u = w * fl(1/n), rounded before the comparisons subtract it
 #pragma unroll
-    for (int c = 0; c < 2; ++c) {
-      const uint4 u0 = *reinterpret_cast<const uint4*>(crow + 32 * q + 16 * c);
-      const uint32_t wv[4] = {u0.x, u0.y, u0.z, u0.w};
-#pragma unroll
-      for (int e = 0; e < 16; ++e) m[16 * c + e] = 0x4B400000u + ((wv[e >> 2] >> (8 * (e & 3))) & 0xFFu);
-    }
+    for (int j = 0; j < 32; ++j) u[j] = __fmul_rn(__uint_as_float(v[j]), inv);
     uint32_t fw[3];
-    quarter_field<L>(m, fw);
-    or_field<12>(w, q * F::QB, fw);
+    tq_quarter<L>(u, t2, fw);
+    or_field<13>(w, q * F::QB, fw);
   }
+  if (!store) return;
+  // the row's RB bytes: word-aligned for K; V starts 2 bytes into a word when RB = 2 mod 4
+  if (kind == 0 || (RB & 3) == 0) {
+    uint32_t* dst = reinterpret_cast<uint32_t*>(rec + kind * RB);
 #pragma unroll
-  for (int k = 0; k < kWords; ++k) out[k] = w[k];
+    for (int k = 0; k < RB / 4; ++k) dst[k] = w[k];
+    if constexpr ((RB & 3) != 0)
+      *reinterpret_cast<uint16_t*>(rec + kind * RB + 4 * (RB / 4)) = (uint16_t)w[RB / 4];
+  } else {
+    *reinterpret_cast<uint16_t*>(rec + RB) = (uint16_t)w[0];
+    uint32_t* dst = reinterpret_cast<uint32_t*>(rec + RB + 2);
+#pragma unroll
+    for (int k = 0; k < (RB - 2) / 4; ++k) dst[k] = __funnelshift_r(w[k], w[k + 1], 16);
+  }
+  *reinterpret_cast<uint16_t*>(rec + 2 * RB + 2 * kind) = n16;
 }
 
 __global__ void __launch_bounds__(kDenseThreads, 2)
-    quantize_tq_dense_kernel(const __grid_constant__ CUtensorMap tmk,
-                             const __grid_constant__ CUtensorMap tmv, QuantArgs a) {
+    quantize_tq_dense_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
   extern __shared__ uint8_t dsm_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~(uintptr_t)1023);
-  uint8_t* ma = base;                       // A: the rotation, core-matrix layout
-  uint8_t* xk = base + kDenseM;             // the tile: K box, then V box
-  uint8_t* codes = xk + 2 * kDenseBox;      // [128 rows: K of token t = 2t, V = 2t+1][128]
-  __shared__ __align__(8) uint64_t tma_bar, mma_bar;
+  uint8_t* mb = base;                       // B: the rotation, core-matrix layout
+  __shared__ __align__(8) uint64_t mma_bar[2];
   __shared__ uint32_t tmem_base;
-  __shared__ uint16_t nrm[128];
-  __shared__ float invs[128];
-  __shared__ uint8_t tokhi[kDenseTok];
-  __shared__ uint32_t rbits[128 * kRowBitWords];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int grp = warp >> 2, row = 32 * (warp & 3) + lane;
+  uint8_t* xa = base + kDenseM + grp * kDenseA;  // A: this group's rows
   const int64_t bhl = blockIdx.y;
   const int h = (int)(bhl % a.H), l = (int)((bhl / a.H) % a.NL);
   const int b = (int)(bhl / ((int64_t)a.H * a.NL));
-  const int tiles = (a.n + kDenseTok - 1) / kDenseTok;
+  const int nb_hi = (int)((n_hi + kRowSlots - 1) / kRowSlots);
+  const int tiles = nb_hi + (int)((n_lo + kRowSlots - 1) / kRowSlots);
   const int per = (tiles + (int)gridDim.x - 1) / (int)gridDim.x;
   const int j0 = min(tiles, (int)blockIdx.x * per), j1 = min(tiles, j0 + per);
-  float th_hi[7], th_lo[7];
-#pragma unroll
-  for (int k = 0; k < 7; ++k) {
-    th_hi[k] = k < a.L_hi - 1 ? a.thr_hi[k] : INFINITY;
-    th_lo[k] = k < a.L_lo - 1 ? a.thr_lo[k] : INFINITY;
-  }
 
   if (tid == 0) {
-    dbar_init(&tma_bar);
-    dbar_init(&mma_bar);
+    dbar_init(&mma_bar[0]);
+    dbar_init(&mma_bar[1]);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 128;" ::"r"(
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(
                      dsmem_u32(&tmem_base))
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
@@ -1211,190 +1292,131 @@ __global__ void __launch_bounds__(kDenseThreads, 2)
   const uint4* msrc = reinterpret_cast<const uint4*>(a.rot + ((int64_t)l * a.H + h) * 128 * 128);
   for (int c = tid; c < 128 * 16; c += kDenseThreads) {
     const int rr = c & 7, kg = (c >> 3) & 15, r = (c >> 7) * 8 + rr;
-    reinterpret_cast<uint4*>(ma)[c] = msrc[r * 16 + kg];
+    reinterpret_cast<uint4*>(mb)[c] = msrc[r * 16 + kg];
   }
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tb = tmem_base;
-  const int row_base = (int)(bhl * a.Tsrc);  // first row of this (b, l, h) in the row view
+  const uint32_t tcol = tb + (uint32_t)(grp * 128);           // this group's accumulator
+  const uint32_t tlane = tcol + ((uint32_t)(32 * (warp & 3)) << 16);
+  const int64_t bh = bhl;  // (sequence, layer, head) index of the pools and the rows
 
-  auto issue_tma = [&](int j) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(dsmem_u32(&tma_bar)),
-                 "r"(2 * kDenseBox)
-                 : "memory");
-    const int row = row_base + j * kDenseTok;
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dsmem_u32(xk)),
-        "l"(reinterpret_cast<uint64_t>(&tmk)), "r"(0), "r"(row), "r"(0), "r"(dsmem_u32(&tma_bar))
-        : "memory");
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dsmem_u32(xk + kDenseBox)),
-        "l"(reinterpret_cast<uint64_t>(&tmv)), "r"(0), "r"(row), "r"(0), "r"(dsmem_u32(&tma_bar))
-        : "memory");
+  // block j of the range: pool, first slot, slots
+  auto block = [&](int j, bool& hi, int& s0, int& ns) {
+    hi = j < nb_hi;
+    s0 = (hi ? j : j - nb_hi) * kRowSlots;
+    ns = (int)min((int64_t)kRowSlots, (hi ? n_hi : n_lo) - s0);
   };
-  if (tid == 0 && j0 < j1) issue_tma(j0);
+  // this thread's row of block j into the group's tile
+  auto load_row = [&](int j) {
+    bool hi;
+    int s0, ns;
+    block(j, hi, s0, ns);
+    if ((row >> 1) < ns) {
+      const int64_t cap = hi ? a.hi_cap : a.lo_cap;
+      const int32_t* tokmap = (hi ? a.hi_tok : a.lo_tok) + (int64_t)b * cap + (hi ? a.hi_base : a.lo_base);
+      const int64_t tk = (int64_t)tokmap[s0 + (row >> 1)] - a.tok_base;
+      const uint16_t* src = ((row & 1) ? a.v : a.k) + (bh * a.Tsrc + tk) * kHeadDim;
+#pragma unroll
+      for (int kg = 0; kg < 16; ++kg) cp_async16(xa + kg * 2048 + row * 16, src + 8 * kg);
+    }
+    cp_async_commit();
+  };
+
   bool ok = true;
-  for (int j = j0; j < j1 && ok; ++j) {
-    const uint32_t par = (uint32_t)((j - j0) & 1);
-    ok = __syncthreads_and(dbar_wait(&tma_bar, par)) != 0;
-    if (!ok) break;
+  int j = j0 + grp;
+  if (j < j1) load_row(j);
+  for (int it = 0; j < j1; j += 2, ++it) {
+    bool hi;
+    int s0, ns;
+    block(j, hi, s0, ns);
+    const bool mine = (row >> 1) < ns;
+    cp_async_wait<0>();
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the rows, for the MMAs
+    group_sync_and(grp, true);
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    if (tid == 0) {
+    if (row == 0) {
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          const uint64_t da = umma_desc(dsmem_u32(ma) + k * 256, 128, 2048);
-          const uint64_t db = umma_desc(dsmem_u32(xk + half * kDenseBox) + k * 2048, 1024, 128);
-          asm volatile(
-              "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n"
-              " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(
-                  tb + (uint32_t)(half * 64)),
-              "l"(da), "l"(db), "r"(kDenseIdesc), "r"((uint32_t)(k > 0))
-              : "memory");
-        }
+      for (int k = 0; k < 8; ++k) {
+        const uint64_t da = umma_desc(dsmem_u32(xa) + k * 4096, 2048, 128);
+        const uint64_t db = umma_desc(dsmem_u32(mb) + k * 256, 128, 2048);
+        asm volatile(
+            "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n"
+            " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tcol),
+            "l"(da), "l"(db), "r"(kDenseIdesc), "r"((uint32_t)(k > 0))
+            : "memory");
       }
       asm volatile(
           "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-              dsmem_u32(&mma_bar))
+              dsmem_u32(&mma_bar[grp]))
           : "memory");
     }
-    // ---- while the MMAs run: norms (fixed tree: 32 in-order partials of 4 squares,
-    // stages 16 .. 1), two threads per row (lanes 2r' and 2r'+1: dims 0..63 and 64..127,
-    // which hold partials 0..15 and 16..31), and the tokens' precisions
+    // ---- while the MMAs run: the row's norm (fixed tree: 32 in-order partials of 4
+    // squares, then the pairwise stages 16, 8, 4, 2, 1).  Partials g and g + 16 are
+    // formed as a pair from chunks kg and kg + 8 (a square of an fp16 value is exact, so
+    // a fused multiply-add rounds as the separate operations)
+    uint16_t n16 = 0;
+    float inv = 0.0f;
     {
-      const int rowi = tid >> 1, part = tid & 1;
-      const int half = rowi >> 6, tok = rowi & 63;
-      const uint8_t* box = xk + half * kDenseBox;
-      float p[16];
+      float pn[16];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const uint4 u = *reinterpret_cast<const uint4*>(box + (8 * part + q) * 1024 + tok * 16);
-        const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+      for (int kg = 0; kg < 8; ++kg) {
+        const uint4 ua = *reinterpret_cast<const uint4*>(xa + kg * 2048 + row * 16);
+        const uint4 ub = *reinterpret_cast<const uint4*>(xa + (kg + 8) * 2048 + row * 16);
+        const uint32_t wa[4] = {ua.x, ua.y, ua.z, ua.w}, wb[4] = {ub.x, ub.y, ub.z, ub.w};
 #pragma unroll
         for (int g2 = 0; g2 < 2; ++g2) {
-          const float x0 = f16_to_f32((uint16_t)(wv[2 * g2] & 0xFFFF)), x1 = f16_to_f32((uint16_t)(wv[2 * g2] >> 16));
-          const float x2 = f16_to_f32((uint16_t)(wv[2 * g2 + 1] & 0xFFFF)), x3 = f16_to_f32((uint16_t)(wv[2 * g2 + 1] >> 16));
-          float acc = __fmul_rn(x0, x0);
-          acc = __fadd_rn(acc, __fmul_rn(x1, x1));
-          acc = __fadd_rn(acc, __fmul_rn(x2, x2));
-          p[2 * q + g2] = __fadd_rn(acc, __fmul_rn(x3, x3));
-        }
-      }
-      // stage 16 pairs partial g (dims 0..63) with g + 16 (dims 64..127)
+          unsigned long long acc = 0ull;
 #pragma unroll
-      for (int g = 0; g < 16; ++g) {
-        const float other = __shfl_xor_sync(0xffffffffu, p[g], 1);
-        p[g] = part == 0 ? __fadd_rn(p[g], other) : __fadd_rn(other, p[g]);
+          for (int e = 0; e < 4; ++e) {
+            const uint32_t xw = wa[2 * g2 + (e >> 1)], yw = wb[2 * g2 + (e >> 1)];
+            const int sh = 16 * (e & 1);
+            const unsigned long long x2 = f2_pack(f16_to_f32((uint16_t)(xw >> sh)), f16_to_f32((uint16_t)(yw >> sh)));
+            acc = e == 0 ? f2_mul(x2, x2) : f2_add(acc, f2_mul(x2, x2));
+          }
+          // partials 2kg + g2 and 2kg + g2 + 16, then their sum (stage 16)
+          pn[2 * kg + g2] = __fadd_rn(f2_lo(acc), f2_hi(acc));
+        }
       }
 #pragma unroll
       for (int off = 8; off >= 1; off >>= 1)
 #pragma unroll
-        for (int g = 0; g < off; ++g) p[g] = __fadd_rn(p[g], p[g + off]);
-      if (part == 0) {
-        const uint16_t n16 = f16_param(__fsqrt_rn(p[0]));
-        const float n = f16_to_f32(n16);
-        nrm[2 * tok + half] = n16;
-        invs[2 * tok + half] = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
-      }
-      if (tid < kDenseTok) {
-        const int t = j * kDenseTok + tid;
-        tokhi[tid] = (t < a.n && a.is_high[(int64_t)b * a.n + t] != 0) ? 1 : 0;
-      }
+        for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
+      n16 = f16_param(__fsqrt_rn(pn[0]));
+      const float n = f16_to_f32(n16);
+      inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
     }
-    ok = __syncthreads_and(dbar_wait(&mma_bar, par)) != 0;  // also: norms visible
-    if (!ok) break;
+    ok = group_sync_and(grp, mbar_wait_bounded(&mma_bar[grp], (uint32_t)(it & 1)));
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    if (tid == 0 && j + 1 < j1) issue_tma(j + 1);  // the MMAs have read the tile
-    // ---- codes: warp w, output dims 32 (w % 4) + lane, K (w < 4) or V columns; the
-    // token (and its precision and 1/n) is the same across the warp
-    {
-      const int half = warp >> 2, d = 32 * (warp & 3) + lane;
-#pragma unroll
-      for (int ch = 0; ch < 2; ++ch) {
-        uint32_t v[32];
-        tmem_ld32(tb + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(half * 64 + ch * 32), v);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int tok = ch * 32 + e, row = 2 * tok + half;
-          const float inv = invs[row];
-          const float u = __fmul_rn(__uint_as_float(v[e]), inv);
-          int c = 0;
-          if (tokhi[tok]) {
-#pragma unroll
-            for (int k = 0; k < 7; ++k) c += u > th_hi[k] ? 1 : 0;
-          } else {
-#pragma unroll
-            for (int k = 0; k < 7; ++k) c += u > th_lo[k] ? 1 : 0;
-          }
-          codes[row * 128 + d] = (uint8_t)(inv != 0.0f ? c : 0);
-        }
-      }
+    if (!ok) break;
+    // the MMAs have read the tile and this thread its row: the next block's row
+    if (j + 2 < j1) load_row(j + 2);
+    // ---- codes and the record
+    const int64_t cap = hi ? a.hi_cap : a.lo_cap;
+    const int L = hi ? a.L_hi : a.L_lo;
+    const int rec_bytes = 2 * row_bytes_rt(L) + 4;
+    uint8_t* rec = (hi ? a.hi_pool : a.lo_pool) +
+                   (bh * cap + (hi ? a.hi_base : a.lo_base) + s0 + (row >> 1)) * rec_bytes;
+    const float* thr = hi ? a.thr_hi : a.thr_lo;
+    const bool live = n16 != 0;
+    switch (L) {
+#define SEMKV_DENSE_CASE(LV) \
+      case LV: dense_row<LV>(tlane, thr, inv, live, n16, rec, row & 1, mine); break;
+      SEMKV_DENSE_CASE(2) SEMKV_DENSE_CASE(3) SEMKV_DENSE_CASE(4) SEMKV_DENSE_CASE(5)
+      SEMKV_DENSE_CASE(6) SEMKV_DENSE_CASE(7) SEMKV_DENSE_CASE(8)
+#undef SEMKV_DENSE_CASE
+      default: break;
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();  // the code tile is complete; the accumulator may be reused
-    // ---- bit images: thread r < 128 packs row r (the record's quarter fields)
-    if (tid < 128) {
-      const int L = tokhi[tid >> 1] ? a.L_hi : a.L_lo;
-      uint32_t* out = rbits + tid * kRowBitWords;
-      const uint8_t* crow = codes + tid * 128;
-      switch (L) {
-        case 2: row_bits<2>(crow, out); break;
-        case 3: row_bits<3>(crow, out); break;
-        case 4: row_bits<4>(crow, out); break;
-        case 5: row_bits<5>(crow, out); break;
-        case 6: row_bits<6>(crow, out); break;
-        case 7: row_bits<7>(crow, out); break;
-        case 8: row_bits<8>(crow, out); break;
-        default: break;
-      }
-    }
-    __syncthreads();
-    // ---- records: warp w writes tokens w, w + 8, ...; lane j word j
-    for (int i = warp; i < kDenseTok; i += kDenseThreads / 32) {
-      const int t = j * kDenseTok + i;
-      if (t >= a.n) break;
-      const bool hi = tokhi[i] != 0;
-      const int64_t s = (hi ? a.hi_base : a.lo_base) + a.slot[(int64_t)b * a.n + t];
-      const int64_t cap = hi ? a.hi_cap : a.lo_cap;
-      if (s >= cap) {  // cannot happen after the host's capacity check
-        if (lane == 0) raise_error(a.err, kDevCapacity);
-        continue;
-      }
-      if (l == 0 && h == 0 && lane == 0) {
-        if (hi) a.hi_tok[(int64_t)b * a.hi_cap + s] = (int32_t)(a.tok_base + t);
-        else a.lo_tok[(int64_t)b * a.lo_cap + s] = (int32_t)(a.tok_base + t);
-      }
-      const int L = hi ? a.L_hi : a.L_lo;
-      const int RB = row_bytes_rt(L), recw = (2 * RB + 4) / 4;
-      uint32_t* dst = reinterpret_cast<uint32_t*>((hi ? a.hi_pool : a.lo_pool) + ((bhl * cap) + s) * (2 * RB + 4));
-      if (lane < recw) {
-        uint32_t word = 0u;
-        if (4 * lane >= 2 * RB) {
-          word = (uint32_t)nrm[2 * i] | ((uint32_t)nrm[2 * i + 1] << 16);
-        } else {
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int byte = 4 * lane + e;
-            const int row = byte < RB ? 2 * i : 2 * i + 1;
-            const int rb = byte < RB ? byte : byte - RB;
-            word |= ((rbits[row * kRowBitWords + (rb >> 2)] >> (8 * (rb & 3))) & 0xFFu) << (8 * e);
-          }
-        }
-        dst[lane] = word;
-      }
-    }
-    __syncthreads();  // the code tile, norms and precisions are free for the next tile
   }
-  if (!ok && tid == 0) raise_error(a.err, kDevWaitTimeout);
+  if (!ok && row == 0) raise_error(a.err, kDevWaitTimeout);
+  cp_async_wait<0>();
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (warp == 0)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 128;" ::"r"(tb) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tb) : "memory");
 }
 
 }  // namespace
@@ -1465,54 +1487,30 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
     return launch_pdl(quantize_affine_kernel, grid, dim3(kWarpsPerBlock * 32), 0, stream, a, n_hi,
                       a.n - n_hi);
   }
-  if (a.base == SEMKV_BASE_TQ_DENSE) {
-    static bool attr_set[kAttrDevices] = {};
-    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
-    cudaError_t e = once_per_device(attr_set, [] {
-      return cudaFuncSetAttribute(quantize_tq_dense_kernel,
-                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDenseSmem);
-    });
-    if (e != cudaSuccess) return e;
-    if (!encode) {  // the driver's entry point (the same for every device)
-      cudaDriverEntryPointQueryResult q;
-      PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-      e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&fn),
-                                           12000, cudaEnableDefault, &q);
-      if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
-        return e != cudaSuccess ? e : cudaErrorNotSupported;
-      encode = fn;
-    }
-    // rows of K (V) as a 3-D view: 8 values, every (sequence, layer, head, token) row,
-    // 16 groups of 8 values; a box of 64 rows lands as 8-row x 16-byte core matrices
-    const int64_t bhs = (int64_t)a.B * a.NL * a.H;
-    const cuuint64_t dims[3] = {8, (cuuint64_t)(bhs * a.Tsrc), 16};
-    const cuuint64_t strides[2] = {256, 16};
-    const cuuint32_t box[3] = {8, (cuuint32_t)kDenseTok, 16};
-    const cuuint32_t estr[3] = {1, 1, 1};
-    CUtensorMap tmk, tmv;
-    for (int t = 0; t < 2; ++t) {
-      const CUresult r = encode(t ? &tmv : &tmk, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3,
-                                const_cast<uint16_t*>(t ? a.v : a.k), dims, strides, box, estr,
-                                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                                CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-                                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-      if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-    }
-    const int tiles = (a.n + kDenseTok - 1) / kDenseTok;
-    int64_t splits = (2 * (int64_t)num_sms + bhs - 1) / bhs;  // about two CTAs per SM
-    if (splits > tiles) splits = tiles;
-    if (splits < 1) splits = 1;
-    if (bhs > 65535) return cudaErrorInvalidValue;
-    const dim3 grid((unsigned)splits, (unsigned)bhs);
-    quantize_tq_dense_kernel<<<grid, kDenseThreads, kDenseSmem, stream>>>(tmk, tmv, a);
-    return cudaGetLastError();
-  }
-  // TQ and rotated affine: slot -> token maps, then one thread per row by slot
+  // TQ, rotated affine and dense-rotation TQ: slot -> token maps, then the rows by slot
   if (!maps_ready) {
     const int64_t pairs = (int64_t)a.B * a.n;
     scatter_tok_kernel<<<(unsigned)((pairs + 255) / 256), 256, 0, stream>>>(a);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+  }
+  if (a.base == SEMKV_BASE_TQ_DENSE) {
+    static bool attr_set[kAttrDevices] = {};
+    const cudaError_t e = once_per_device(attr_set, [] {
+      return cudaFuncSetAttribute(quantize_tq_dense_kernel,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDenseSmem);
+    });
+    if (e != cudaSuccess) return e;
+    const int64_t bhs = (int64_t)a.B * a.NL * a.H;
+    if (bhs > 65535) return cudaErrorInvalidValue;
+    const int64_t tiles = (n_hi + kRowSlots - 1) / kRowSlots + (a.n - n_hi + kRowSlots - 1) / kRowSlots;
+    int64_t splits = (2 * (int64_t)num_sms + bhs - 1) / bhs;  // about two CTAs per SM
+    // (each CTA's two groups take alternate blocks of its range)
+    if (splits > (tiles + 1) / 2) splits = (tiles + 1) / 2;
+    if (splits < 1) splits = 1;
+    const dim3 grid((unsigned)splits, (unsigned)bhs);
+    quantize_tq_dense_kernel<<<grid, kDenseThreads, kDenseSmem, stream>>>(a, n_hi, a.n - n_hi);
+    return cudaGetLastError();
   }
   // persistent CTAs (rows2_ctas per SM) over every block of both pools
   const int64_t bhs = (int64_t)a.B * a.NL * a.H;
