@@ -268,34 +268,6 @@ __device__ __forceinline__ float f2_hi(unsigned long long v) {
   return __uint_as_float((uint32_t)(v >> 32));
 }
 
-// In-thread unnormalised Walsh-Hadamard transform of one row, butterfly stages 1, 2,
-// ..., 64 in order, each (a + b, a - b) rounded to nearest: stage 1 inside each pair
-// (2k, 2k+1), the later stages on packed pairs (pair k with pair k + hs/2).  The same
-// roundings as any other evaluation of these butterflies in this stage order.
-__device__ __forceinline__ void fwht128(float (&x)[128]) {
-  unsigned long long xp[64];
-#pragma unroll
-  for (int k = 0; k < 64; ++k) {
-    const float p0 = x[2 * k], p1 = x[2 * k + 1];
-    xp[k] = f2_pack(__fadd_rn(p0, p1), __fsub_rn(p0, p1));
-  }
-#pragma unroll
-  for (int hs = 2; hs < 128; hs <<= 1) {
-#pragma unroll
-    for (int k = 0; k < 64; ++k) {
-      if ((2 * k) & hs) continue;
-      const unsigned long long p0 = xp[k], p1 = xp[k + hs / 2];
-      xp[k] = f2_add(p0, p1);
-      xp[k + hs / 2] = f2_sub(p0, p1);
-    }
-  }
-#pragma unroll
-  for (int k = 0; k < 64; ++k) {
-    x[2 * k] = f2_lo(xp[k]);
-    x[2 * k + 1] = f2_hi(xp[k]);
-  }
-}
-
 // OR the 96-bit field v at bit pos (compile-time after unrolling) of a row's words
 template <int N>
 __device__ __forceinline__ void or_field(uint32_t (&w)[N], int pos, const uint32_t (&v)[3]) {
@@ -674,45 +646,13 @@ __device__ void rows_half(const QuantArgs& a, int b, int l, int h, bool hi, int6
   }
 }
 
-// ---- mbarriers
+// ---- shared addresses and mbarriers
 __device__ __forceinline__ uint32_t dsmem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
 }
 __device__ __forceinline__ void dbar_init(uint64_t* bar) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(dsmem_u32(bar)) : "memory");
 }
-__device__ __forceinline__ bool dbar_wait(uint64_t* bar, uint32_t parity) {
-  return mbar_wait_bounded(bar, parity);
-}
-
-// Persistent CTAs over the blocks (64 slots of one pool of one (sequence, layer, KV
-// head)), in a two-stage pipeline: while a block is quantized, the rows of the CTA's
-// next block are already on their way.  Thread r brings its own row r with one 256-byte
-// cp.async.bulk into its own 272-byte slot of the stage (so a slot is only ever touched
-// by its thread until the records are assembled); every thread arrives once per phase
-// on the stage's mbarrier (count 128), announcing its bytes.  Waits are bounded.
-constexpr int kRowStageBytes = 128 * kRowStride;
-static_assert(kRowBitWords + 1 <= kRowStride / 4, "bit image and parameters fit a row slot");
-
-__device__ __forceinline__ void rbar_init128(uint64_t* bar) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], 128;" ::"r"(dsmem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ void rbar_arrive(uint64_t* bar, uint32_t tx_bytes) {
-  if (tx_bytes)
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(dsmem_u32(bar)),
-                 "r"(tx_bytes)
-                 : "memory");
-  else
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(dsmem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ void bulk_g2s_row(void* dst, const void* src, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], 256, [%2];" ::"r"(
-          dsmem_u32(dst)),
-      "l"(src), "r"(dsmem_u32(bar))
-      : "memory");
-}
-
 // block t of the pass, decoded once: (sequence, layer, KV head), pool, first slot and
 // slot count (32-bit arithmetic: the launcher keeps the block count below 2^31)
 struct RowsTile {
@@ -823,101 +763,6 @@ __global__ void __launch_bounds__(kRows2Threads, rows2_ctas(BASE)) quantize_rows
 // owns row r (K of token r/2 when r is even, V when odd), in registers; rows are
 // staged through shared memory on the way in and out for coalesced transfers.
 
-__device__ __forceinline__ void load_signs(const int8_t* sg, float (&x)[128]) {
-#pragma unroll
-  for (int j = 0; j < 32; ++j) {
-    const char4 s4 = __ldg(reinterpret_cast<const char4*>(sg) + j);
-    x[4 * j] *= (float)s4.x;
-    x[4 * j + 1] *= (float)s4.y;
-    x[4 * j + 2] *= (float)s4.z;
-    x[4 * j + 3] *= (float)s4.w;
-  }
-}
-
-// The rotated-affine and TQ fake quantization of one row in registers (in: the row's
-// fp16 values as binary32; out: the reconstruction before its fp16 rounding).  sel_hi:
-// the row takes the high pool's tables (its token is high, or every token is).
-template <int BASE>
-__device__ __forceinline__ void fake_float_row(float (&x)[128], int L, bool sel_hi,
-                                               const int8_t* sg, const float (*cbs)[8],
-                                               const FakeArgs& a) {
-  if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
-    // y = FWHT(z + s c);  x^_d = fp16((sign_d y_d) * fp32(1/sqrt 128))
-    load_signs(sg, x);
-    fwht128(x);
-    float mn = INFINITY, mx = -INFINITY;
-#pragma unroll
-    for (int j = 0; j < 128; ++j) {
-      x[j] = __fmul_rn(x[j], kInvSqrtD);
-      mn = fminf(mn, x[j]);
-      mx = fmaxf(mx, x[j]);
-    }
-    if (mn == 0.0f) mn = 0.0f;
-    if (mx == 0.0f) mx = 0.0f;
-    uint16_t z16 = __half_as_ushort(__float2half_rd(mn));
-    if (z16 == 0xFC00u) z16 = 0xFBFFu;
-    const float z = f16_to_f32(z16);
-    const float sv = f16_to_f32(f16_param(__fdiv_rn(__fsub_rn(mx, z), (float)(L - 1))));
-    const bool live = sv > 0.0f;
-    const float inv = live ? __fdiv_rn(1.0f, sv) : 0.0f;
-#pragma unroll
-    for (int j = 0; j < 128; ++j) {
-      // c = rint(clamp((x - z) / s)) as an integer-valued float (magic-number rounding,
-      // to nearest even); every code is 0 when s = 0 (inv = 0)
-      const float y = fminf(fmaxf(__fmul_rn(__fsub_rn(x[j], z), inv), 0.0f), (float)(L - 1));
-      const float c = __fsub_rn(__fadd_rn(y, 12582912.0f), 12582912.0f);
-      x[j] = __fadd_rn(z, __fmul_rn(sv, c));
-    }
-    fwht128(x);
-    load_signs(sg, x);
-#pragma unroll
-    for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], kInvSqrtD);
-  } else {
-    // y = FWHT(cb[c]);  x^_d = fp16((sign_d y_d) * (n / 128))
-    float pn[16];
-#pragma unroll
-    for (int g = 0; g < 16; ++g) {
-      float acc[2];
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        const int gg = g + 16 * hh;
-        float v = __fmul_rn(x[4 * gg], x[4 * gg]);
-#pragma unroll
-        for (int k = 1; k < 4; ++k) v = __fadd_rn(v, __fmul_rn(x[4 * gg + k], x[4 * gg + k]));
-        acc[hh] = v;
-      }
-      pn[g] = __fadd_rn(acc[0], acc[1]);
-    }
-#pragma unroll
-    for (int off = 8; off >= 1; off >>= 1)
-#pragma unroll
-      for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
-    const uint16_t n16 = f16_param(__fsqrt_rn(pn[0]));
-    const float n = f16_to_f32(n16);
-    const float inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
-    const float* thr_g = sel_hi ? a.thr_hi : a.thr_lo;
-    const float* cb = cbs[sel_hi ? 0 : 1];
-    float thr[7];
-#pragma unroll
-    for (int k = 0; k < 7; ++k) thr[k] = k < L - 1 ? thr_g[k] : INFINITY;
-    load_signs(sg, x);
-    fwht128(x);
-#pragma unroll
-    for (int j = 0; j < 128; ++j) {
-      const float u = __fmul_rn(x[j], inv);
-      int c = 0;
-#pragma unroll
-      for (int k = 0; k < 7; ++k) c += (u > thr[k]) ? 1 : 0;
-      x[j] = cb[n != 0.0f ? c : 0];
-    }
-    fwht128(x);
-    load_signs(sg, x);
-    const float nq = n * 0.0078125f;
-#pragma unroll
-    for (int j = 0; j < 128; ++j) x[j] = __fmul_rn(x[j], nq);
-  }
-}
-
 // Affine base: a CTA per 64-token block, rows staged through shared memory in and out
 // (coalesced), each row kept as fp16 pairs (96 registers: 5 CTAs per SM).
 __global__ void __launch_bounds__(128, 5) fake_affine_kernel(FakeArgs a) {
@@ -1000,96 +845,223 @@ __global__ void __launch_bounds__(128, 5) fake_affine_kernel(FakeArgs a) {
   }
 }
 
-// Rotated affine and TQ: persistent CTAs over the 64-token blocks, each row moved by its
-// own thread with bulk copies in both directions: the rows of the CTA's next block are
-// loaded into the other stage while this block is computed, and each thread writes its
-// reconstructed row back from its own slot with one 256-byte bulk store.  A slot is only
-// ever touched by its thread, so the blocks need no CTA barrier; before a slot takes new
-// rows, its thread waits until its previous store has read it.  Waits are bounded.
-__device__ __forceinline__ void bulk_s2g_row(void* dst, const void* src) {
-  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], 256;" ::"l"(dst),
-               "r"(dsmem_u32(src))
-               : "memory");
-  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+// Rotated affine and TQ: two threads per row, as the rows quantizer.  Persistent CTAs of
+// 256 threads over the 64-token blocks of every (sequence, layer, KV head): thread tid
+// holds half f = tid & 1 of row tid >> 1 (K of token tid >> 2 when bit 1 is 0, V when 1)
+// as 32 packed pairs (x_j, x_{j+32}), the next block's halves arriving by 16-byte
+// cp.async copies under the current block (one CTA barrier per block).  Both
+// transforms run the quantizer's butterflies (stages 1..32 in the thread, stage 64 with
+// the partner lane); the reconstruction is written back as fp16 with 16-byte stores.
+
+// stage 64 of the butterflies across the two halves of a row (half 0 keeps a + b, half 1
+// a - b, a from half 0): fma(own, +-1, partner) rounds partner +- own once
+__device__ __forceinline__ void fwht_stage64(unsigned long long (&xp)[32], unsigned long long sg2) {
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    const float plo = __shfl_xor_sync(0xffffffffu, f2_lo(xp[j]), 1);
+    const float phi = __shfl_xor_sync(0xffffffffu, f2_hi(xp[j]), 1);
+    xp[j] = f2_fma(xp[j], sg2, f2_pack(plo, phi));
+  }
+}
+
+// The codebook entry of each of a pair's two values: c = #{k : u > thr_k} over the
+// kLmax - 1 thresholds (the row's own L - 1 of them, then +inf), from the sign bits of
+// thr_k - u as in tq_fields
+template <int kLmax>
+__device__ __forceinline__ unsigned long long tq_dequant2(unsigned long long u2,
+                                                          const unsigned long long (&t2)[7],
+                                                          const float* cb) {
+  uint32_t cl = 0u, ch = 0u;
+#pragma unroll
+  for (int k = 0; k < kLmax - 1; ++k) {
+    const unsigned long long d = f2_sub(t2[k], u2);
+    cl += (uint32_t)d >> 31;
+    ch += (uint32_t)(d >> 32) >> 31;
+  }
+  return f2_pack(cb[cl], cb[ch]);
+}
+
+// One half of a row (see above): slot holds its fp16 values, mask the sign masks of its
+// dims; out: the reconstruction's fp16 pairs for dims 64f + 2p, 64f + 2p + 1.
+template <int BASE, int kLmax>
+__device__ __forceinline__ void fake_half(const uint8_t* slot, const uint32_t* mask, int f, int L,
+                                          bool sel_hi, const float (*cbs)[8], const FakeArgs& a,
+                                          uint32_t (&out)[32]) {
+  unsigned long long xp[32];
+  {
+    const uint4* src = reinterpret_cast<const uint4*>(slot);
+    const uint4* msk = reinterpret_cast<const uint4*>(mask);
+    uint32_t wv[32];
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const uint4 u = src[c], m = msk[c];
+      wv[4 * c] = u.x ^ m.x; wv[4 * c + 1] = u.y ^ m.y;
+      wv[4 * c + 2] = u.z ^ m.z; wv[4 * c + 3] = u.w ^ m.w;
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const uint32_t lo = wv[j >> 1], hi2 = wv[16 + (j >> 1)];
+      const int sh = 16 * (j & 1);
+      xp[j] = f2_pack(f16_to_f32((uint16_t)(lo >> sh)), f16_to_f32((uint16_t)(hi2 >> sh)));
+    }
+  }
+  const float sg = f ? -1.0f : 1.0f;
+  const unsigned long long sg2 = f2_pack(sg, sg);
+  float post;  // the reconstruction's final factor: fp32(1/sqrt 128), or n / 128
+  if constexpr (BASE == SEMKV_BASE_AFFINE_HAD) {
+    // y = FWHT(z + s c);  x^_d = fp16((sign_d y_d) * fp32(1/sqrt 128))
+    fwht_half(xp);
+    fwht_stage64(xp, sg2);
+    float mn = INFINITY, mx = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      xp[j] = f2_pack(__fmul_rn(f2_lo(xp[j]), kInvSqrtD), __fmul_rn(f2_hi(xp[j]), kInvSqrtD));
+      mn = fminf(mn, fminf(f2_lo(xp[j]), f2_hi(xp[j])));
+      mx = fmaxf(mx, fmaxf(f2_lo(xp[j]), f2_hi(xp[j])));
+    }
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, 1));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+    if (mn == 0.0f) mn = 0.0f;
+    if (mx == 0.0f) mx = 0.0f;
+    uint16_t z16 = __half_as_ushort(__float2half_rd(mn));
+    if (z16 == 0xFC00u) z16 = 0xFBFFu;
+    const float z = f16_to_f32(z16);
+    const float sv = f16_to_f32(f16_param(__fdiv_rn(__fsub_rn(mx, z), (float)(L - 1))));
+    const float inv = sv > 0.0f ? __fdiv_rn(1.0f, sv) : 0.0f;
+    const unsigned long long z2 = f2_pack(z, z), inv2 = f2_pack(inv, inv), s2 = f2_pack(sv, sv);
+    const unsigned long long mg2 = f2_pack(12582912.0f, 12582912.0f);
+    const float top = (float)(L - 1);
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      // c = rint(clamp((x - z) / s)) as an integer-valued float (every code 0 when s = 0);
+      // z + s c: s c is exact (an fp16 value times an integer below 8), so the fused
+      // multiply-add rounds as the separate multiply and add
+      const unsigned long long d = f2_mul(f2_sub(xp[j], z2), inv2);
+      const float ylo = fminf(fmaxf(f2_lo(d), 0.0f), top), yhi = fminf(fmaxf(f2_hi(d), 0.0f), top);
+      const unsigned long long c2 = f2_sub(f2_add(f2_pack(ylo, yhi), mg2), mg2);
+      xp[j] = f2_fma(s2, c2, z2);
+    }
+    post = kInvSqrtD;
+  } else {
+    // y = FWHT(cb[c]);  x^_d = fp16((sign_d y_d) * (n / 128))
+    float pn[8];
+#pragma unroll
+    for (int g = 0; g < 8; ++g) {
+      // (a square of an fp16 value is exact: a fused x * x + v rounds as the separate ops)
+      unsigned long long v = f2_mul(xp[4 * g], xp[4 * g]);
+#pragma unroll
+      for (int k = 1; k < 4; ++k) v = f2_add(v, f2_mul(xp[4 * g + k], xp[4 * g + k]));
+      const float plo = __shfl_xor_sync(0xffffffffu, f2_lo(v), 1);
+      const float phi = __shfl_xor_sync(0xffffffffu, f2_hi(v), 1);
+      const unsigned long long sp = f2_add(v, f2_pack(plo, phi));
+      pn[g] = __fadd_rn(f2_lo(sp), f2_hi(sp));
+    }
+#pragma unroll
+    for (int off = 4; off >= 1; off >>= 1)
+#pragma unroll
+      for (int g = 0; g < off; ++g) pn[g] = __fadd_rn(pn[g], pn[g + off]);
+    const float n = f16_to_f32(f16_param(__fsqrt_rn(pn[0])));
+    const float inv = n != 0.0f ? __fdiv_rn(1.0f, n) : 0.0f;
+    const float* tg = sel_hi ? a.thr_hi : a.thr_lo;
+    unsigned long long t2[7];
+#pragma unroll
+    for (int k = 0; k < kLmax - 1; ++k) {
+      // a zero-norm row compares against +inf (all codes 0)
+      const float tk = (n != 0.0f && k < L - 1) ? __fadd_rn(__ldg(tg + k), 0.0f) : INFINITY;
+      t2[k] = f2_pack(tk, tk);
+    }
+    fwht_half(xp);
+    fwht_stage64(xp, sg2);
+    const float* cb = cbs[sel_hi ? 0 : 1];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      // u = y * fl(1/n), rounded before the comparisons subtract it
+      const unsigned long long u2 = f2_pack(__fmul_rn(f2_lo(xp[j]), inv), __fmul_rn(f2_hi(xp[j]), inv));
+      xp[j] = tq_dequant2<kLmax>(u2, t2, cb);
+    }
+    post = n * 0.0078125f;
+  }
+  fwht_half(xp);
+  fwht_stage64(xp, sg2);
+  // (sign_d y_d) * post = sign_d (y_d * post): the product rounds to fp16 next, no add
+  const unsigned long long p2 = f2_pack(post, post);
+#pragma unroll
+  for (int j = 0; j < 32; ++j) xp[j] = f2_mul(xp[j], p2);
+#pragma unroll
+  for (int p = 0; p < 16; ++p) {
+    const __half2 h0 = __floats2half2_rn(f2_lo(xp[2 * p]), f2_lo(xp[2 * p + 1]));
+    const __half2 h1 = __floats2half2_rn(f2_hi(xp[2 * p]), f2_hi(xp[2 * p + 1]));
+    out[p] = *reinterpret_cast<const uint32_t*>(&h0) ^ mask[p];
+    out[16 + p] = *reinterpret_cast<const uint32_t*>(&h1) ^ mask[16 + p];
+  }
 }
 
 template <int BASE>
-__global__ void __launch_bounds__(128, BASE == SEMKV_BASE_TQ ? 2 : 3) fake_rows_kernel(FakeArgs a) {
-  extern __shared__ __align__(128) uint8_t fstage[];  // 2 stages of 128 row slots
-  __shared__ __align__(8) uint64_t fbar[2];
+__global__ void __launch_bounds__(kRows2Threads, 2) fake_rows_kernel(FakeArgs a, int Lmax) {
+  extern __shared__ __align__(128) uint8_t fstage[];  // 2 stages of 256 half-row slots
+  __shared__ __align__(16) uint32_t smask[2][64];
   __shared__ float cbs[2][8];
-  const int tid = threadIdx.x;
-  if (tid < 2) rbar_init128(&fbar[tid]);
+  const int tid = threadIdx.x, f = tid & 1, r = tid >> 1, i = r >> 1;
   if (BASE == SEMKV_BASE_TQ && tid < 16) {
     const int which = tid >> 3, k = tid & 7;
     const int L = which ? a.L_lo : a.L_hi;
     cbs[which][k] = k < L ? (which ? a.cent_lo : a.cent_hi)[k] : 0.0f;
   }
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  __syncthreads();
-  const int64_t bhs = (int64_t)a.B * a.NL * a.H;
-  const int64_t nblk = ((int64_t)a.T + kRowSlots - 1) / kRowSlots;
-  const int64_t total = bhs * nblk;
-  const int i = tid >> 1;
-  auto issue = [&](int64_t t, int st) {
-    const int64_t bhi = t / nblk;
-    const int t0 = (int)(t % nblk) * kRowSlots;
-    if (i < a.T - t0) {
-      const uint16_t* src = ((tid & 1) ? a.v : a.k) + (bhi * a.T + t0 + i) * kHeadDim;
-      asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");  // the slot's last store
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      rbar_arrive(&fbar[st], 256u);
-      bulk_g2s_row(fstage + st * kRowStageBytes + tid * kRowStride, src, &fbar[st]);
-    } else {
-      rbar_arrive(&fbar[st], 0u);
-    }
+  const uint32_t nblk = (uint32_t)((a.T + kRowSlots - 1) / kRowSlots);
+  const uint32_t total = (uint32_t)a.B * a.NL * a.H * nblk;
+  // block t: (sequence, layer, head) index and first token
+  auto decode = [&](uint32_t t, uint32_t& bhi, int& t0) {
+    bhi = t / nblk;
+    t0 = (int)(t - bhi * nblk) * kRowSlots;
   };
-  int64_t t = blockIdx.x;
+  auto issue = [&](uint32_t t, int st) {
+    uint32_t bhi;
+    int t0;
+    decode(t, bhi, t0);
+    if (tid < 64) {
+      const uint32_t q = bhi / (uint32_t)a.H;
+      const int h = (int)(bhi - q * a.H), l = (int)(q % (uint32_t)a.NL);
+      const char2 s2 = *reinterpret_cast<const char2*>(a.signs + ((int64_t)l * a.H + h) * kHeadDim + 2 * tid);
+      smask[st][tid] = (s2.x < 0 ? 0x8000u : 0u) | (s2.y < 0 ? 0x80000000u : 0u);
+    }
+    if (i < a.T - t0) {
+      const uint16_t* src = ((r & 1) ? a.v : a.k) + ((int64_t)bhi * a.T + t0 + i) * kHeadDim + 64 * f;
+      uint8_t* dst = fstage + st * kRows2StageBytes + tid * kHalfStride;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) cp_async16(dst + 16 * c, src + 8 * c);
+    }
+    cp_async_commit();
+  };
+  uint32_t t = blockIdx.x;
   if (t < total) issue(t, 0);
   for (int k = 0; t < total; t += gridDim.x, ++k) {
     const int st = k & 1;
-    const bool next = t + gridDim.x < total;
-    if (next) issue(t + gridDim.x, st ^ 1);
-    if (!__syncthreads_and(dbar_wait(&fbar[st], (uint32_t)((k >> 1) & 1)))) {
-      // a copy never landed: record it, let the other stage's copies finish, stop
-      if (tid == 0) raise_error(a.err, kDevWaitTimeout);
-      if (next) dbar_wait(&fbar[st ^ 1], (uint32_t)(((k + 1) >> 1) & 1));
-      break;
-    }
-    const int64_t bhi = t / nblk;
-    const int t0 = (int)(t % nblk) * kRowSlots;
-    if (i >= a.T - t0) continue;  // past the sequence's end
-    const int h = (int)(bhi % a.H), l = (int)((bhi / a.H) % a.NL);
-    const int b = (int)(bhi / ((int64_t)a.H * a.NL));
-    const bool sel_hi = a.is_high == nullptr || a.is_high[(int64_t)b * a.T + t0 + i] != 0;
+    cp_async_wait<0>();
+    __syncthreads();  // the stage and its masks are published; the other stage is free
+    if (t + gridDim.x < total) issue(t + gridDim.x, st ^ 1);
+    uint32_t bhi;
+    int t0;
+    decode(t, bhi, t0);
+    const int b = (int)(bhi / ((uint32_t)a.H * a.NL));
+    const bool live = i < a.T - t0;
+    const bool sel_hi = a.is_high == nullptr || (live && a.is_high[(int64_t)b * a.T + t0 + i] != 0);
     const int L = sel_hi ? a.L_hi : a.L_lo;
-    uint8_t* slot = fstage + st * kRowStageBytes + tid * kRowStride;
-    float x[128];
-#pragma unroll
-    for (int ch = 0; ch < 16; ++ch) {
-      const uint4 u = *reinterpret_cast<const uint4*>(slot + ch * 16);
-      const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        x[8 * ch + 2 * e] = f16_to_f32((uint16_t)(wv[e] & 0xFFFFu));
-        x[8 * ch + 2 * e + 1] = f16_to_f32((uint16_t)(wv[e] >> 16));
-      }
+    const uint8_t* slot = fstage + st * kRows2StageBytes + tid * kHalfStride;
+    uint32_t out[32];
+    switch (BASE == SEMKV_BASE_TQ ? Lmax : 2) {
+#define SEMKV_FAKE_CASE(LV) \
+      case LV: fake_half<BASE, LV>(slot, smask[st] + 32 * f, f, L, sel_hi, cbs, a, out); break;
+      SEMKV_FAKE_CASE(2) SEMKV_FAKE_CASE(3) SEMKV_FAKE_CASE(4) SEMKV_FAKE_CASE(5)
+      SEMKV_FAKE_CASE(6) SEMKV_FAKE_CASE(7) SEMKV_FAKE_CASE(8)
+#undef SEMKV_FAKE_CASE
+      default: break;
     }
-    fake_float_row<BASE>(x, L, sel_hi, a.signs + ((int64_t)l * a.H + h) * kHeadDim, cbs, a);
+    if (live) {
+      uint4* dst = reinterpret_cast<uint4*>(((r & 1) ? a.v_out : a.k_out) + ((int64_t)bhi * a.T + t0 + i) * kHeadDim + 64 * f);
 #pragma unroll
-    for (int ch = 0; ch < 16; ++ch) {
-      uint32_t w[4];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const __half2 h2 = __floats2half2_rn(x[8 * ch + 2 * e], x[8 * ch + 2 * e + 1]);
-        w[e] = *reinterpret_cast<const uint32_t*>(&h2);
-      }
-      *reinterpret_cast<uint4*>(slot + ch * 16) = make_uint4(w[0], w[1], w[2], w[3]);
+      for (int c = 0; c < 8; ++c) dst[c] = make_uint4(out[4 * c], out[4 * c + 1], out[4 * c + 2], out[4 * c + 3]);
     }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the row, to the async proxy
-    bulk_s2g_row(((tid & 1) ? a.v_out : a.k_out) + (bhi * a.T + t0 + i) * kHeadDim, slot);
   }
-  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");  // every store done before exit
 }
 
 // ------------------------------------- dense-rotation TQ rows (tcgen05) --------
@@ -1435,20 +1407,25 @@ cudaError_t launch_fake_quant(const FakeArgs& a, int num_sms, cudaStream_t strea
   const cudaError_t e = once_per_device(attr_set, [] {
     cudaError_t r = cudaFuncSetAttribute(fake_rows_kernel<SEMKV_BASE_AFFINE_HAD>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         2 * kRowStageBytes);
+                                         2 * kRows2StageBytes);
     if (r == cudaSuccess)
       r = cudaFuncSetAttribute(fake_rows_kernel<SEMKV_BASE_TQ>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kRowStageBytes);
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kRows2StageBytes);
     return r;
   });
   if (e != cudaSuccess) return e;
-  // persistent: 3 CTAs per SM (2 for TQ, whose registers allow no more)
-  int64_t ctas = (int64_t)(num_sms > 0 ? num_sms : 1) * (a.base == SEMKV_BASE_TQ ? 2 : 3);
+  // persistent: 2 CTAs of 256 threads per SM (128 registers: both transforms' pairs and
+  // the dequantization constants spill at 80); block indices are 32-bit
+  if (bhs * nblk > INT32_MAX / 2) return cudaErrorInvalidValue;
+  int64_t ctas = (int64_t)(num_sms > 0 ? num_sms : 1) * 2;
   if (ctas > bhs * nblk) ctas = bhs * nblk;
+  const int Lmax = a.L_hi > a.L_lo ? a.L_hi : a.L_lo;
   if (a.base == SEMKV_BASE_AFFINE_HAD)
-    fake_rows_kernel<SEMKV_BASE_AFFINE_HAD><<<(unsigned)ctas, 128, 2 * kRowStageBytes, stream>>>(a);
+    fake_rows_kernel<SEMKV_BASE_AFFINE_HAD>
+        <<<(unsigned)ctas, kRows2Threads, 2 * kRows2StageBytes, stream>>>(a, Lmax);
   else
-    fake_rows_kernel<SEMKV_BASE_TQ><<<(unsigned)ctas, 128, 2 * kRowStageBytes, stream>>>(a);
+    fake_rows_kernel<SEMKV_BASE_TQ>
+        <<<(unsigned)ctas, kRows2Threads, 2 * kRows2StageBytes, stream>>>(a, Lmax);
   return cudaGetLastError();
 }
 
