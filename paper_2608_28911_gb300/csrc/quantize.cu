@@ -30,26 +30,28 @@ constexpr int kWarpsPerBlock = 8;
 constexpr int kMaxRecWords = 27;  // largest record: affine L=7/8, 2*48+8 = 104 B
 
 // ------------------------------------------------- affine pools, by slot -----
-// Affine records are built by destination slot: a warp takes units of 8 consecutive
+// Affine records are built by destination slot: a warp takes units of 4 consecutive
 // slots of one pool of one (sequence, layer, KV head), so the level count is uniform
-// across the warp and the records it writes are contiguous.  Lane 4i + 2r + f handles
-// half f (dims 64f..64f+63, quarters 2f and 2f+1) of row r (0 = K, 1 = V) of the i-th
-// slot's token: 128 contiguous bytes in, two quarter bit fields out.  The same
-// arithmetic as the header states, and symbols beta = ceil(t 2^W / L^G) (the record format).
+// across the warp and the records it writes are contiguous.  Lane 8i + 4r + q handles
+// quarter q (dims 32q..32q+31) of row r (0 = K, 1 = V) of the i-th slot's token: 64
+// contiguous bytes in, one quarter bit field out (a quarter per lane keeps the lane's
+// state small: 48 registers, 40 warps per SM).  The same arithmetic as the header states, and
+// symbols beta = ceil(t 2^W / L^G) (the record format).
 
-constexpr int kAffineSlots = 8;
+constexpr int kAffineSlots = 4;
+constexpr int kAffineCtas = 5;  // resident CTAs of 8 warps per SM (48 registers)
 
-// 64 fp16 values of one half row (16-byte loads when the source allows)
-__device__ __forceinline__ void load_half(const uint16_t* src, bool vec16, uint32_t (&h)[32]) {
+// 32 fp16 values of one quarter row (16-byte loads when the source allows)
+__device__ __forceinline__ void load_quarter(const uint16_t* src, bool vec16, uint32_t (&h)[16]) {
   if (vec16) {
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < 4; ++j) {
       const uint4 u = __ldg(reinterpret_cast<const uint4*>(src) + j);
       h[4 * j] = u.x; h[4 * j + 1] = u.y; h[4 * j + 2] = u.z; h[4 * j + 3] = u.w;
     }
   } else {
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
+    for (int j = 0; j < 8; ++j) {
       const uint2 u = __ldg(reinterpret_cast<const uint2*>(src) + j);
       h[2 * j] = u.x; h[2 * j + 1] = u.y;
     }
@@ -100,6 +102,38 @@ __device__ __forceinline__ void quarter_field(const uint32_t (&m)[32], uint32_t 
   }
 }
 
+// One code of a quarter's field, streamed in order (j = 0..31, compile-time after
+// unrolling): m is the magic-number pattern 1.5 * 2^23 + c_j, t the running radix value
+// of the open symbol; each completed symbol's beta goes into the field, as quarter_field.
+template <int L>
+__device__ __forceinline__ void field_push(uint32_t (&w)[3], uint32_t& t, int j, uint32_t m) {
+  using F = Fmt<L>;
+  constexpr uint32_t kMagic = 0x4B400000u;
+  if constexpr (F::G == 1 && F::LG == (1u << F::W)) {
+    put_bits(w, j * F::W, F::W, m - kMagic);
+  } else {
+    if (j < F::NG * F::G) {
+      const int k = j % F::G, sy = j / F::G;
+      t = (k == 0 ? 0u : t * (uint32_t)L) + m;
+      if (k == F::G - 1) {
+        uint32_t wsum = 0;
+        for (int q = 0; q < F::G; ++q) wsum = wsum * (uint32_t)L + 1u;
+        const uint32_t tt = t - wsum * kMagic;
+        put_bits(w, sy * F::W, F::W, ((tt << F::W) + F::LG - 1u) / F::LG);
+      }
+    } else {
+      const int k = j - F::NG * F::G;
+      t = (k == 0 ? 0u : t * (uint32_t)L) + m;
+      if (k == F::R - 1) {
+        uint32_t wsum = 0;
+        for (int q = 0; q < F::R; ++q) wsum = wsum * (uint32_t)L + 1u;
+        const uint32_t tt = t - wsum * kMagic;
+        put_bits(w, F::NG * F::W, F::WT, ((tt << F::WT) + F::LR - 1u) / F::LR);
+      }
+    }
+  }
+}
+
 template <int L>
 __device__ void affine_units(const QuantArgs& a, int b, int l, int h, bool hi, int64_t n_pool,
                              int64_t u_begin, int64_t u_step, bool vec16, uint32_t* img) {
@@ -107,12 +141,12 @@ __device__ void affine_units(const QuantArgs& a, int b, int l, int h, bool hi, i
   constexpr int kRecW = (2 * F::RB + 8) / 4;
   static_assert(F::QB <= 96, "a quarter fits three words");
   const int lane = threadIdx.x & 31;
-  const int ti = lane >> 2, row = (lane >> 1) & 1, hf = lane & 1;
+  const int ti = lane >> 3, row = (lane >> 2) & 1, qd = lane & 3;
   const int64_t cap = hi ? a.hi_cap : a.lo_cap;
   const int64_t base = hi ? a.hi_base : a.lo_base;
   const int64_t bh = ((int64_t)b * a.NL + l) * a.H + h;
   const int32_t* tokmap = (hi ? a.hi_tok : a.lo_tok) + (int64_t)b * cap + base;
-  const uint16_t* src = (row ? a.v : a.k) + bh * a.Tsrc * kHeadDim + 64 * hf;
+  const uint16_t* src = (row ? a.v : a.k) + bh * a.Tsrc * kHeadDim + 32 * qd;
   const int64_t tok_base = a.tok_base;
   uint32_t* recs = reinterpret_cast<uint32_t*>(hi ? a.hi_pool : a.lo_pool) + (bh * cap + base) * kRecW;
   const int64_t units = (n_pool + kAffineSlots - 1) / kAffineSlots;
@@ -121,17 +155,17 @@ __device__ void affine_units(const QuantArgs& a, int b, int l, int h, bool hi, i
     const int nslots = (int)min((int64_t)kAffineSlots, n_pool - s0);
     const bool active = ti < nslots;
     for (int i = lane; i < kAffineSlots * kRecW; i += 32) img[i] = 0u;
-    uint32_t hv[32];
+    uint32_t hv[16];
     if (active) {
-      load_half(src + ((int64_t)tokmap[s0 + ti] - tok_base) * kHeadDim, vec16, hv);
+      load_quarter(src + ((int64_t)tokmap[s0 + ti] - tok_base) * kHeadDim, vec16, hv);
     } else {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) hv[j] = 0u;
+      for (int j = 0; j < 16; ++j) hv[j] = 0u;
     }
-    // row minimum and maximum: fp16 pairs (exact), then the row's other half
+    // row minimum and maximum: fp16 pairs (exact), then the row's other quarters
     __half2 mn2 = *reinterpret_cast<const __half2*>(&hv[0]), mx2 = mn2;
 #pragma unroll
-    for (int j = 1; j < 32; ++j) {
+    for (int j = 1; j < 16; ++j) {
       const __half2 x2 = *reinterpret_cast<const __half2*>(&hv[j]);
       mn2 = __hmin2(mn2, x2);
       mx2 = __hmax2(mx2, x2);
@@ -140,6 +174,8 @@ __device__ void affine_units(const QuantArgs& a, int b, int l, int h, bool hi, i
     float mx = fmaxf(__low2float(mx2), __high2float(mx2));
     mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, 1));
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, 2));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
     // a zero extreme is taken as +0 (min/max may return either signed zero)
     if (mn == 0.0f) mn = 0.0f;
     if (mx == 0.0f) mx = 0.0f;
@@ -149,30 +185,26 @@ __device__ void affine_units(const QuantArgs& a, int b, int l, int h, bool hi, i
     // 1/s, or 0 when s == 0 (then every value rounds to code 0)
     const float inv = sc != 0.0f ? __fdiv_rn(1.0f, sc) : 0.0f;
     __syncwarp();
+    // the codes stream into the quarter's field (no array of them: fewer registers)
+    uint32_t w[3] = {0u, 0u, 0u}, t = 0u;
 #pragma unroll
-    for (int qq = 0; qq < 2; ++qq) {
-      uint32_t m[32];
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const float x = f16_to_f32((uint16_t)(hv[16 * qq + (j >> 1)] >> (16 * (j & 1))));
-        // rint((x - z) / s) clamped to L-1 (the difference is >= 0: z is the row
-        // minimum); adding 1.5 * 2^23 rounds to nearest even
-        const float y = fminf(__fmul_rn(__fsub_rn(x, z), inv), (float)(L - 1));
-        m[j] = __float_as_uint(__fadd_rn(y, 12582912.0f));
-      }
-      uint32_t w[3];
-      quarter_field<L>(m, w);
-      if (active) {
-        uint32_t* r = img + ti * kRecW;
-        const int pos = row * 8 * F::RB + (2 * hf + qq) * F::QB;  // the quarter's first bit
-        const int wd = pos >> 5, sh = pos & 31;
-        atomicOr(&r[wd], w[0] << sh);
-        if (sh + F::QB > 32) atomicOr(&r[wd + 1], __funnelshift_l(w[0], w[1], sh));
-        if (sh + F::QB > 64) atomicOr(&r[wd + 2], __funnelshift_l(w[1], w[2], sh));
-        if (sh + F::QB > 96) atomicOr(&r[wd + 3], __funnelshift_l(w[2], 0u, sh));
-      }
+    for (int j = 0; j < 32; ++j) {
+      const float x = f16_to_f32((uint16_t)(hv[j >> 1] >> (16 * (j & 1))));
+      // rint((x - z) / s) clamped to L-1 (the difference is >= 0: z is the row
+      // minimum); adding 1.5 * 2^23 rounds to nearest even
+      const float y = fminf(__fmul_rn(__fsub_rn(x, z), inv), (float)(L - 1));
+      field_push<L>(w, t, j, __float_as_uint(__fadd_rn(y, 12582912.0f)));
     }
-    if (active && hf == 0) img[ti * kRecW + (2 * F::RB) / 4 + row] = (uint32_t)s16 | ((uint32_t)z16 << 16);
+    if (active) {
+      uint32_t* r = img + ti * kRecW;
+      const int pos = row * 8 * F::RB + qd * F::QB;  // the quarter's first bit
+      const int wd = pos >> 5, sh = pos & 31;
+      atomicOr(&r[wd], w[0] << sh);
+      if (sh + F::QB > 32) atomicOr(&r[wd + 1], __funnelshift_l(w[0], w[1], sh));
+      if (sh + F::QB > 64) atomicOr(&r[wd + 2], __funnelshift_l(w[1], w[2], sh));
+      if (sh + F::QB > 96) atomicOr(&r[wd + 3], __funnelshift_l(w[2], 0u, sh));
+      if (qd == 0) r[(2 * F::RB) / 4 + row] = (uint32_t)s16 | ((uint32_t)z16 << 16);
+    }
     __syncwarp();
     uint32_t* dst = recs + s0 * kRecW;
     for (int i = lane; i < nslots * kRecW; i += 32) dst[i] = img[i];
@@ -196,7 +228,7 @@ __global__ void scatter_tok_kernel(QuantArgs a) {
 }
 
 // grid (x, sequence*layer*head, pool): each warp strides over that pool's units
-__global__ void __launch_bounds__(kWarpsPerBlock * 32, 4)
+__global__ void __launch_bounds__(kWarpsPerBlock * 32, kAffineCtas)
     quantize_affine_kernel(QuantArgs a, int64_t n_hi, int64_t n_lo) {
   __shared__ __align__(16) uint32_t img_sm[kWarpsPerBlock][kAffineSlots * kMaxRecWords];
   const int wib = threadIdx.x >> 5;
@@ -1440,14 +1472,14 @@ cudaError_t launch_quantize_pack(const QuantArgs& a, int64_t n_hi, int num_sms,
       const cudaError_t e = cudaGetLastError();
       if (e != cudaSuccess) return e;
     }
-    // grid x from a simple wave model: with R resident CTAs (4 per SM), the pass takes
+    // grid x from a simple wave model: with R resident CTAs (kAffineCtas per SM), the pass takes
     // about ceil(CTAs / R) waves of ceil(units / (8 bx)) units per warp; take the
     // cheapest bx (at most 16 units per warp).  The (sequence, layer, head) index runs
     // over grid y (and loops past its limit of 65535)
     const int64_t bhs = (int64_t)a.B * a.NL * a.H;
     const int64_t n_max = n_hi > a.n - n_hi ? n_hi : a.n - n_hi;
     const int64_t units = (n_max + kAffineSlots - 1) / kAffineSlots;
-    const int64_t resident = (int64_t)(num_sms > 0 ? num_sms : 1) * 4;
+    const int64_t resident = (int64_t)(num_sms > 0 ? num_sms : 1) * kAffineCtas;
     const int64_t rows = 2 * (bhs < 65535 ? bhs : 65535);
     int64_t bx = 1, best = -1;
     for (int64_t pw = 16; pw >= 1; --pw) {
