@@ -1109,7 +1109,8 @@ __global__ void __launch_bounds__(kRows2Threads, 2) fake_rows_kernel(FakeArgs a,
 // the group's 128 columns of tensor memory, so TMEM lane r is row r and column c its
 // output dim c.  While the MMAs run, thread r takes its row's fixed-tree norm from the
 // tile; once they have completed it starts the copies of the group's next block and
-// reads its row's w = M x a quarter (32 columns) at a time: u = w * fl(1/n), the codes
+// reads its row's w = M x a quarter (32 columns) at a time, the next quarter's load in
+// flight while one is coded: u = w * fl(1/n), the codes
 // from the thresholds, the quarter bit fields, and the row's bytes straight into its
 // record.  The two groups' accumulators are distinct, so one group's MMAs overlap the
 // other's epilogue.
@@ -1128,8 +1129,10 @@ __device__ __forceinline__ uint64_t umma_desc(uint32_t saddr, uint32_t lbo, uint
   return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
          ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46);
 }
-// 32 columns of this warp's 32 TMEM lanes (lane i of the warp <- TMEM lane 32 (w % 4) + i)
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+// 32 columns of this warp's 32 TMEM lanes (lane i of the warp <- TMEM lane 32 (w % 4) + i):
+// the load, and the wait that makes them readable.  The wait takes the registers as
+// in-out operands, so no use of them can be scheduled before it.
+__device__ __forceinline__ void tmem_ld32_start(uint32_t taddr, uint32_t (&v)[32]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
       "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
@@ -1139,7 +1142,22 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
         "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
         "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
       : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_ld_wait(uint32_t (&v)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]),
+                 "+r"(v[6]), "+r"(v[7]), "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]),
+                 "+r"(v[12]), "+r"(v[13]), "+r"(v[14]), "+r"(v[15]), "+r"(v[16]), "+r"(v[17]),
+                 "+r"(v[18]), "+r"(v[19]), "+r"(v[20]), "+r"(v[21]), "+r"(v[22]), "+r"(v[23]),
+                 "+r"(v[24]), "+r"(v[25]), "+r"(v[26]), "+r"(v[27]), "+r"(v[28]), "+r"(v[29]),
+                 "+r"(v[30]), "+r"(v[31])
+               :
+               : "memory");
+}
+__device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+  return v;
 }
 // barrier of the 128 threads of group g (named barrier 1 + g), with an AND of p
 __device__ __forceinline__ bool group_sync_and(int g, bool p) {
@@ -1234,14 +1252,18 @@ __device__ __forceinline__ void dense_row(uint32_t taddr, const float* thr, floa
   uint32_t w[13];
 #pragma unroll
   for (int k = 0; k < 13; ++k) w[k] = 0u;
+  // quarter q + 1's columns load while quarter q is coded
+  uint32_t vb[2][32];
+  tmem_ld32_start(taddr, vb[0]);
+  tmem_ld_wait(vb[0]);
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    uint32_t v[32];
-    tmem_ld32(taddr + 32 * q, v);
+    if (q < 3) tmem_ld32_start(taddr + 32 * (q + 1), vb[(q + 1) & 1]);
     float u[32];
     // u = w * fl(1/n), rounded before the comparisons subtract it
 #pragma unroll
-    for (int j = 0; j < 32; ++j) u[j] = __fmul_rn(__uint_as_float(v[j]), inv);
+    for (int j = 0; j < 32; ++j) u[j] = __fmul_rn(__uint_as_float(vb[q & 1][j]), inv);
+    if (q < 3) tmem_ld_wait(vb[(q + 1) & 1]);
     uint32_t fw[3];
     tq_quarter<L>(u, t2, fw);
     or_field<13>(w, q * F::QB, fw);
@@ -1364,11 +1386,12 @@ __global__ void __launch_bounds__(kDenseThreads, 2)
     uint16_t n16 = 0;
     float inv = 0.0f;
     {
+      const uint32_t xs = dsmem_u32(xa);  // (shared-space loads: the tile is in shared memory)
       float pn[16];
 #pragma unroll
       for (int kg = 0; kg < 8; ++kg) {
-        const uint4 ua = *reinterpret_cast<const uint4*>(xa + kg * 2048 + row * 16);
-        const uint4 ub = *reinterpret_cast<const uint4*>(xa + (kg + 8) * 2048 + row * 16);
+        const uint4 ua = ld_shared_v4(xs + kg * 2048 + row * 16);
+        const uint4 ub = ld_shared_v4(xs + (kg + 8) * 2048 + row * 16);
         const uint32_t wa[4] = {ua.x, ua.y, ua.z, ua.w}, wb[4] = {ub.x, ub.y, ub.z, ub.w};
 #pragma unroll
         for (int g2 = 0; g2 < 2; ++g2) {
