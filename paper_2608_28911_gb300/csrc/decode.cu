@@ -2090,7 +2090,6 @@ __global__ void combine_kernel(DecodeArgs a) {
 // (lane = 4 dims) and the 8 row sums are added in warp order.  For the small batches,
 // whose (b, h) pairs are spread over dozens of CTAs, this keeps the combine short.
 __global__ void __launch_bounds__(256) combine_wide_kernel(DecodeArgs a) {
-  __shared__ float wsm[kMaxPartialsPerPair];
   __shared__ float red[8][128];
   __shared__ float red_m[8], red_l[8];
   // launched as a programmatic dependent of the pool kernels: wait for their partials
@@ -2103,54 +2102,53 @@ __global__ void __launch_bounds__(256) combine_wide_kernel(DecodeArgs a) {
   const int64_t bh = (int64_t)b * a.H + h;
   const int S = pair_partials(a.plan, bh);
   const float* base = a.partials + bh * a.plan.stride * kPartialFloats;
-  float M = -INFINITY;
-  for (int s = tid; s < S; s += 256) M = fmaxf(M, base[s * kPartialFloats + c]);
+  // one pass: warp w merges partials w, w + 8, ... (each lane dims 4 lane .. 4 lane + 3)
+  // against its own maximum, so every load is issued before any result is needed;
+  // then the 8 warps' sums are merged against the overall maximum
+  constexpr int kPer = (kMaxPartialsPerPair + 7) / 8;
+  float ms[kPer];
+  float Mw = -INFINITY;
 #pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-  if (lane == 0) red_m[w] = M;
-  __syncthreads();
-  M = red_m[0];
-#pragma unroll
-  for (int i = 1; i < 8; ++i) M = fmaxf(M, red_m[i]);
-  float lsum = 0.0f;
-  for (int s = tid; s < S; s += 256) {
-    const float ms = base[s * kPartialFloats + c];
-    const float sc = (M == -INFINITY || ms == -INFINITY) ? 0.0f : exp2f(ms - M);
-    wsm[s] = sc;
-    lsum += sc * base[s * kPartialFloats + 8 + c];
+  for (int i = 0; i < kPer; ++i) {
+    const int s = w + 8 * i;
+    ms[i] = s < S ? base[s * kPartialFloats + c] : -INFINITY;
+    Mw = fmaxf(Mw, ms[i]);
   }
+  float lw = 0.0f, o[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
-  if (lane == 0) red_l[w] = lsum;
-  __syncthreads();
-  float o[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int s = w; s < S; s += 8) {
-    const float sc = wsm[s];
-    if (sc == 0.0f) continue;
+  for (int i = 0; i < kPer; ++i) {
+    const int s = w + 8 * i;
+    if (s >= S || ms[i] == -INFINITY) continue;
+    const float sc = exp2f(ms[i] - Mw);
     const float4 v = *reinterpret_cast<const float4*>(base + s * kPartialFloats + 16 + c * 128 + 4 * lane);
+    lw += sc * base[s * kPartialFloats + 8 + c];
     o[0] += sc * v.x;
     o[1] += sc * v.y;
     o[2] += sc * v.z;
     o[3] += sc * v.w;
   }
+  if (lane == 0) {
+    red_m[w] = Mw;
+    red_l[w] = lw;
+  }
 #pragma unroll
   for (int e = 0; e < 4; ++e) red[w][4 * lane + e] = o[e];
   __syncthreads();
   if (w == 0) {
-    float l = red_l[0];
+    float M = red_m[0];
 #pragma unroll
-    for (int i = 1; i < 8; ++i) l += red_l[i];
-    const float inv = 1.0f / l;
-    float r[4];
+    for (int i = 1; i < 8; ++i) M = fmaxf(M, red_m[i]);
+    float l = 0.0f, r[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      float x = red[0][4 * lane + e];
+    for (int i = 0; i < 8; ++i) {
+      const float sc = red_m[i] == -INFINITY ? 0.0f : exp2f(red_m[i] - M);
+      l += sc * red_l[i];
 #pragma unroll
-      for (int i = 1; i < 8; ++i) x += red[i][4 * lane + e];
-      r[e] = x * inv;
+      for (int e = 0; e < 4; ++e) r[e] += sc * red[i][4 * lane + e];
     }
+    const float inv = 1.0f / l;
     *reinterpret_cast<float4*>(a.out + ((int64_t)b * a.Hq + qh) * 128 + 4 * lane) =
-        make_float4(r[0], r[1], r[2], r[3]);
+        make_float4(r[0] * inv, r[1] * inv, r[2] * inv, r[3] * inv);
   }
 }
 
