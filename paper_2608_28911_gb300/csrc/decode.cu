@@ -73,6 +73,17 @@ constexpr int kMaxSplits = 64;                     // pool splits per (b, h)
 constexpr float kPMax = 0x1p52f;                   // bound on p = 2^(logit - e)
 
 static_assert(kStageBytes % 16 == 0, "bulk copies need 16-byte aligned stages");
+// The fast path copies two tiles (32 consecutive slots) per bulk copy into a ring of
+// kFastStages stages per warp: one wait, one refill and one round of ring bookkeeping
+// serve 32 tokens.
+constexpr int kChunk = 2;                  // tiles per copy on the fast path
+constexpr int kFastStages = 3;
+constexpr int kFastRec = 92;               // largest fast-path record (six levels)
+constexpr int kFastStageBytes = kChunk * kTile * kFastRec + 16;  // +16: window over-read
+constexpr int kFastRingBytes = kWarps * kFastStages * kFastStageBytes;
+static_assert(kFastStageBytes % 16 == 0, "bulk copies need 16-byte aligned stages");
+static_assert(kFastStages <= kStages, "the fast path uses the first barriers of each warp");
+static_assert(kFastRingBytes >= (kWarps * 8 * 128 + 8 * 128) * 4, "merge area reuses the ring");
 static_assert(kRingBytes >= (kWarps * 8 * 128 + 8 * 128) * 4, "merge area reuses the ring");
 
 // ------------------------------------------------------------------ PTX -------
@@ -981,8 +992,10 @@ __device__ __forceinline__ float coef_scale(float qmax, int L) {
   return qmax > 0.0f ? pow2_floor(fminf(8192.0f / ((float)(L + 1) * qmax), 1e30f)) : 1.0f;
 }
 
-// One warp streams its tiles of one (pair, pool) segment (see the section comment).
-// ring_it: tiles this warp has taken through its ring so far (barrier phases).
+// One warp streams its tiles of one (pair, pool) segment (see the section comment),
+// two consecutive tiles per copy: the segment's tiles [t_begin, t_end) form chunks of
+// kChunk tiles (the last may hold one) and warp w takes chunks w, w + kWarps, ...
+// ring_it: chunks this warp has taken through its ring so far (barrier phases).
 template <int L>
 __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint2* qbs,
                               uint64_t* bars, const uint8_t* pool_bh, int64_t count,
@@ -994,7 +1007,7 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
   static_assert(kTileBytes % 16 == 0, "tile size must be a multiple of 16 bytes");
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int g = lane >> 2, t = lane & 3;
-  uint8_t* my_ring = ring + warp * kStages * kStageBytes;
+  uint8_t* my_ring = ring + warp * kFastStages * kFastStageBytes;
   uint64_t* my_bar = bars + warp * kStages;
   const bool rot = a.base == SEMKV_BASE_AFFINE_HAD;
 
@@ -1054,23 +1067,8 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
   const uint32_t vw0 = 2 * t * kRec + 4 * (vpos >> 5), vsh = vpos & 31;
   const uint32_t pw0 = g * kRec + 2 * F::RB, pw1 = pw0 + 8 * kRec;
 
-  const int nmine = t_end - t_begin <= warp ? 0 : (t_end - t_begin - warp + kWarps - 1) / kWarps;
-  // tokens left in the pool from this warp's current tile on (a pool holds fewer than
-  // 2^31 slots), the source of the refill kStages tiles ahead, the ring position
-  int left = (int)count - (t_begin + warp) * kTile;
-  const uint8_t* refill_src = pool_bh + (int64_t)(t_begin + warp + kStages * kWarps) * kTileBytes;
-  int stage = ring_it % kStages;
-  uint32_t phase = (uint32_t)((ring_it / kStages) & 1);
-  bool ok = true;
-  int it = 0;
-  for (; it < nmine; ++it) {
-    if (!mbar_wait(&my_bar[stage], phase)) {
-      ok = false;
-      break;
-    }
-    const uint32_t ts = ring_s + stage * kStageBytes;
-    const int nvalid = min(kTile, left);
-
+  // one 16-token tile at shared address ts whose first nvalid rows are tokens of the pool
+  auto run_tile = [&](const uint32_t ts, const int nvalid) {
     // ---- S^T = F Q'^T: tokens g (rows g) and g + 8, heads in column pairs
     float s[4] = {0.f, 0.f, 0.f, 0.f};
     {
@@ -1199,14 +1197,37 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
           mma16816(st.O[m], VA[m][0], VA[m][1], VA[m][2], VA[m][3], b0, b1);
       }
     }
+  };
+
+  const int nchunks = (t_end - t_begin + kChunk - 1) / kChunk;
+  const int nmine = nchunks <= warp ? 0 : (nchunks - warp + kWarps - 1) / kWarps;
+  // first tile of this warp's current chunk (a pool holds fewer than 2^31 slots), the
+  // ring position
+  int tile = t_begin + warp * kChunk;
+  int stage = ring_it % kFastStages;
+  uint32_t phase = (uint32_t)((ring_it / kFastStages) & 1);
+  bool ok = true;
+  int it = 0;
+  for (; it < nmine; ++it) {
+    if (!mbar_wait(&my_bar[stage], phase)) {
+      ok = false;
+      break;
+    }
+    const uint32_t cs = ring_s + stage * kFastStageBytes;
+    const int left = (int)count - tile * kTile;  // tokens of the pool from this chunk on
+    run_tile(cs, min(kTile, left));
+#pragma unroll
+    for (int j = 1; j < kChunk; ++j)
+      if (tile + j < t_end) run_tile(cs + j * kTileBytes, min(kTile, left - j * kTile));
     __syncwarp();
-    // the stage is free again: lane 0 starts the copy of the tile kStages ahead
+    // the stage is free again: lane 0 starts the copy of the chunk kFastStages ahead
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    bulk_refill(lane == 0 && it + kStages < nmine, my_ring + stage * kStageBytes, refill_src,
-                kTileBytes, &my_bar[stage]);
-    refill_src += (int64_t)kWarps * kTileBytes;
-    left -= kWarps * kTile;
-    if (++stage == kStages) {
+    const int nt = tile + kFastStages * kWarps * kChunk;
+    bulk_refill(lane == 0 && it + kFastStages < nmine, my_ring + stage * kFastStageBytes,
+                pool_bh + (int64_t)nt * kTileBytes, (uint32_t)min(kChunk, t_end - nt) * kTileBytes,
+                &my_bar[stage]);
+    tile += kWarps * kChunk;
+    if (++stage == kFastStages) {
       stage = 0;
       phase ^= 1u;
     }
@@ -1215,8 +1236,9 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
     // a copy never completed: record it, give the copies still in flight a bounded
     // chance to land, and drop this warp's contribution
     if (lane == 0) raise_error(a.err, kDevWaitTimeout);
-    for (int j = it; j < nmine && j < it + kStages; ++j)
-      mbar_wait(&my_bar[(ring_it + j) % kStages], (uint32_t)(((ring_it + j) / kStages) & 1));
+    for (int j = it; j < nmine && j < it + kFastStages; ++j)
+      mbar_wait(&my_bar[(ring_it + j) % kFastStages],
+                (uint32_t)(((ring_it + j) / kFastStages) & 1));
     fast_init(st);
   }
   ring_it += nmine;
@@ -1673,6 +1695,30 @@ __device__ void ring_fill(uint8_t* ring, uint64_t* bars, const uint8_t* pool_bh,
   __syncwarp();
 }
 
+// The first copies of a fast-path segment (chunks of kChunk tiles), as run_pool_fast
+// would start them, issued before the queries are loaded and the coefficient fragments
+// built.  The ring must be free (no merge in progress).
+__device__ void ring_fill_fast(uint8_t* ring, uint64_t* bars, const uint8_t* pool_bh,
+                               uint32_t tile_bytes, int t_begin, int t_end, int ring_it) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nchunks = (t_end - t_begin + kChunk - 1) / kChunk;
+  const int nmine = nchunks <= warp ? 0 : (nchunks - warp + kWarps - 1) / kWarps;
+  uint8_t* my_ring = ring + warp * kFastStages * kFastStageBytes;
+  uint64_t* my_bar = bars + warp * kStages;
+  if (lane == 0) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    for (int i = 0; i < kFastStages && i < nmine; ++i) {
+      const int first = t_begin + (warp + i * kWarps) * kChunk;
+      const uint32_t bytes = (uint32_t)min(kChunk, t_end - first) * tile_bytes;
+      const int sl = (ring_it + i) % kFastStages;
+      mbar_expect_tx(&my_bar[sl], bytes);
+      bulk_g2s(my_ring + sl * kFastStageBytes, pool_bh + (int64_t)first * tile_bytes, bytes,
+               &my_bar[sl]);
+    }
+  }
+  __syncwarp();
+}
+
 template <int L>
 __device__ void run_pool_any_g(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint4* aq_all,
                                uint64_t* bars, const uint8_t* pool_bh, int64_t count, int t0,
@@ -1806,7 +1852,7 @@ __global__ void __launch_bounds__(kThreads, kCtasFast) decode_affine_fast_kernel
   __shared__ Shared sh;
   __shared__ MergeArea mg;
   uint8_t* ring = dyn;
-  uint2* qbs = reinterpret_cast<uint2*>(dyn + kRingBytes);  // [8 steps][32 lanes]
+  uint2* qbs = reinterpret_cast<uint2*>(dyn + kFastRingBytes);  // [8 steps][32 lanes]
   float* merge_o = reinterpret_cast<float*>(dyn);  // [kWarps][8][128] rows, then [8][128]
   const DecodePlan& P = a.plan;
   const int G = a.Hq / a.H;
@@ -1843,7 +1889,7 @@ __global__ void __launch_bounds__(kThreads, kCtasFast) decode_affine_fast_kernel
       const int rec = record_bytes_rt(SEMKV_BASE_AFFINE, L);
       const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
       uint64_t* bars = &sh.bar[0][0];
-      ring_fill(ring, bars, pool_bh, (uint32_t)(kTile * rec), t0, t1, ring_it);
+      ring_fill_fast(ring, bars, pool_bh, (uint32_t)(kTile * rec), t0, t1, ring_it);
       if (bh != loaded) {
         load_group_q(a, sh, b, h, G);
         loaded = bh;
@@ -2288,7 +2334,8 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
                                            kRingBytes + kAqBytes);
       if (r == cudaSuccess)
         r = cudaFuncSetAttribute(decode_affine_fast_kernel,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes + kQbBytes);
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kFastRingBytes + kQbBytes);
       if (r == cudaSuccess)
         r = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kRingBytes + kAqBytes);
@@ -2319,8 +2366,8 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
   } else if (P.ctas > 0) {
     // (the rotated affine base rotates its queries inside the pool and stage kernels)
     if (P.fast)
-      e = launch_pdl(decode_affine_fast_kernel, dim3(P.ctas), dim3(kThreads), kRingBytes + kQbBytes,
-                     stream, a);
+      e = launch_pdl(decode_affine_fast_kernel, dim3(P.ctas), dim3(kThreads),
+                     kFastRingBytes + kQbBytes, stream, a);
     else
       e = launch_pdl(decode_affine_kernel, dim3(P.ctas), dim3(kThreads), kRingBytes + kAqBytes,
                      stream, a);
