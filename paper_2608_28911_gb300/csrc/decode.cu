@@ -2210,6 +2210,48 @@ static int tile_cost(int L) {
   }
 }
 
+// the fixed cost of a segment in a CTA (queries, coefficient fragments, the first
+// copies' latency, the merge), in tile weights: about 16 five-level tiles
+constexpr int64_t kSegmentCost = 16 * 7;
+
+// Replace the balanced plan p by its aligned form (see make_decode_plan) when that is
+// cheaper.  target: resident CTAs; st: 1 with a staged tail.
+static void aligned_plan(DecodePlan& p, int64_t pairs, int64_t target, int st, int max_stride) {
+  const int64_t th = p.tiles_hi, tl = p.tiles_lo;
+  const int64_t per_pair = target / pairs;
+  const int pools = (th > 0) + (tl > 0);
+  if (pools == 0 || per_pair < pools) return;
+  const int64_t Th = th > 0 ? th : 1, Tl = tl > 0 ? tl : 1;
+  if (Th * Tl > ((int64_t)1 << 40)) return;  // weights must stay small integers
+  // CTAs per segment: every warp gets a chunk or more, at most the partial slots allow
+  const int64_t max_n = (int64_t)max_stride - st;
+  const int64_t cap_hi = th > 0 ? (th / 16 > 1 ? th / 16 : 1) : 0;
+  const int64_t cap_lo = tl > 0 ? (tl / 16 > 1 ? tl / 16 : 1) : 0;
+  int64_t best_h = 0, best_l = 0, best = INT64_MAX;
+  for (int64_t nh = th > 0 ? 1 : 0; nh <= (th > 0 ? cap_hi : 0); ++nh) {
+    int64_t nl = tl > 0 ? per_pair - nh : 0;
+    if (nl > cap_lo) nl = cap_lo;
+    if (nh + nl > max_n) nl = max_n - nh;
+    if (tl > 0 && nl < 1) continue;
+    const int64_t ch = nh ? (th + nh - 1) / nh * p.w_hi : 0;
+    const int64_t cl = nl ? (tl + nl - 1) / nl * p.w_lo : 0;
+    const int64_t c = ch > cl ? ch : cl;
+    if (c < best) {
+      best = c;
+      best_h = nh;
+      best_l = nl;
+    }
+  }
+  if (best == INT64_MAX || best >= p.per + kSegmentCost) return;
+  const int64_t wh = best_h * Tl, wl = best_l * Th;
+  if (wh > INT32_MAX || wl > INT32_MAX) return;
+  p.w_hi = (int)wh;
+  p.w_lo = (int)wl;
+  p.per = Th * Tl;
+  p.W = (best_h + best_l) * p.per;
+  p.ctas = (int)(pairs * (best_h + best_l));
+}
+
 DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int Hq, int64_t hi_count,
                             int64_t lo_count, int stage_n, int num_sms, int max_stride) {
   DecodePlan p;
@@ -2254,6 +2296,15 @@ DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int Hq, 
     if (per < per_min) per = per_min;
     p.per = per;
     p.ctas = (int)((total + per - 1) / per);
+    // When the CTAs outnumber the pairs' segments (few sequences), ranges of equal
+    // weight cut across the hi | lo and pair boundaries, and a CTA whose range holds a
+    // boundary sets up, streams and merges two segments.  Aligned alternative: n_hi
+    // CTAs per hi segment and n_lo per lo segment, each taking an equal share of its
+    // segment's tiles.  It is the same range arithmetic with the weights w_hi' =
+    // n_hi T_lo and w_lo' = n_lo T_hi and per' = T_hi T_lo (T = the tile counts, 1 for
+    // an empty pool), so that a segment is exactly n_hi (n_lo) ranges long.  Taken when
+    // its longest range is shorter than per plus one segment's fixed cost.
+    aligned_plan(p, pairs, target, st, max_stride);
     int worst = 0;
     for (int64_t bh = 0; bh < pairs; ++bh) {
       int n_hi, n_lo;
