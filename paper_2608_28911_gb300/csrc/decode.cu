@@ -68,7 +68,7 @@ constexpr int kAqBytes = 8 * 32 * 16;   // q-coefficient A fragments: 8 k-steps 
 constexpr int kQbBytes = 8 * 32 * 8;    // fast path: coefficient B fragments, 8 steps x 32 lanes x uint2
 constexpr int kCtasAffine = 2;          // resident CTAs per SM: affine pools / other sources
 constexpr int kCtasOther = 2;
-constexpr int kCtasFast = 2;           // resident CTAs per SM: the fast affine path (127 registers)
+constexpr int kCtasFast = 2;           // resident CTAs per SM: the fast affine path with 8 warps
 constexpr int kMaxSplits = 64;                     // pool splits per (b, h)
 constexpr float kPMax = 0x1p52f;                   // bound on p = 2^(logit - e)
 
@@ -80,10 +80,21 @@ constexpr int kChunk = 2;                  // tiles per copy on the fast path
 constexpr int kFastStages = 3;
 constexpr int kFastRec = 92;               // largest fast-path record (six levels)
 constexpr int kFastStageBytes = kChunk * kTile * kFastRec + 16;  // +16: window over-read
-constexpr int kFastRingBytes = kWarps * kFastStages * kFastStageBytes;
+// The fast path has two CTA shapes.  Over long straddled ranges (many sequences) it runs
+// one CTA of 16 warps per SM: the warp schedulers favour the warps of the CTA that
+// reached an SM first, so of two 8-warp CTAs with equal ranges one finishes long before
+// the other, which then runs alone at half occupancy, while the warps of one CTA advance
+// evenly.  With segment-aligned ranges (few sequences), two CTAs of 8 warps per SM, whose
+// set-up and merge overlap each other's tiles.
+constexpr int kFastWarps = 16;
+constexpr int kMaxWarps = 16;                // warps of the largest CTA (barriers, merge area)
+template <int NW>
+constexpr int fast_ring_bytes() { return NW * kFastStages * kFastStageBytes; }
 static_assert(kFastStageBytes % 16 == 0, "bulk copies need 16-byte aligned stages");
 static_assert(kFastStages <= kStages, "the fast path uses the first barriers of each warp");
-static_assert(kFastRingBytes >= (kWarps * 8 * 128 + 8 * 128) * 4, "merge area reuses the ring");
+static_assert(fast_ring_bytes<kWarps>() >= (kWarps * 8 * 128 + 8 * 128) * 4 &&
+                  fast_ring_bytes<kFastWarps>() >= (kFastWarps * 8 * 128 + 8 * 128) * 4,
+              "merge area reuses the ring");
 static_assert(kRingBytes >= (kWarps * 8 * 128 + 8 * 128) * 4, "merge area reuses the ring");
 
 // ------------------------------------------------------------------ PTX -------
@@ -499,7 +510,7 @@ struct Shared {
   float sumq[8];            // sum over dims of each head's q (q' for TQ records)
   float qmax[8];            // max |q_d| of each head (q' for TQ records)
   float cdec[2][3];         // TQ tensor path, per pool: centroids as cz + cs c (+ c3 phi^3)
-  uint64_t bar[kWarps][kStages];
+  uint64_t bar[kMaxWarps][kStages];
 };
 
 // ------------------------------------------------------------ pool tiles ------
@@ -994,9 +1005,9 @@ __device__ __forceinline__ float coef_scale(float qmax, int L) {
 
 // One warp streams its tiles of one (pair, pool) segment (see the section comment),
 // two consecutive tiles per copy: the segment's tiles [t_begin, t_end) form chunks of
-// kChunk tiles (the last may hold one) and warp w takes chunks w, w + kWarps, ...
+// kChunk tiles (the last may hold one) and warp w of NW takes chunks w, w + NW, ...
 // ring_it: chunks this warp has taken through its ring so far (barrier phases).
-template <int L>
+template <int L, int NW>
 __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ring, uint2* qbs,
                               uint64_t* bars, const uint8_t* pool_bh, int64_t count,
                               int t_begin, int t_end, int G, FastState& st, int& ring_it) {
@@ -1200,7 +1211,7 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
   };
 
   const int nchunks = (t_end - t_begin + kChunk - 1) / kChunk;
-  const int nmine = nchunks <= warp ? 0 : (nchunks - warp + kWarps - 1) / kWarps;
+  const int nmine = nchunks <= warp ? 0 : (nchunks - warp + NW - 1) / NW;
   // first tile of this warp's current chunk (a pool holds fewer than 2^31 slots), the
   // ring position
   int tile = t_begin + warp * kChunk;
@@ -1222,11 +1233,11 @@ __device__ void run_pool_fast(const DecodeArgs& a, const Shared& sh, uint8_t* ri
     __syncwarp();
     // the stage is free again: lane 0 starts the copy of the chunk kFastStages ahead
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    const int nt = tile + kFastStages * kWarps * kChunk;
+    const int nt = tile + kFastStages * NW * kChunk;
     bulk_refill(lane == 0 && it + kFastStages < nmine, my_ring + stage * kFastStageBytes,
                 pool_bh + (int64_t)nt * kTileBytes, (uint32_t)min(kChunk, t_end - nt) * kTileBytes,
                 &my_bar[stage]);
-    tile += kWarps * kChunk;
+    tile += NW * kChunk;
     if (++stage == kFastStages) {
       stage = 0;
       phase ^= 1u;
@@ -1480,13 +1491,14 @@ __host__ __device__ inline int pair_partials(const DecodePlan& P, int64_t bh) {
 }
 
 struct MergeArea {
-  float m[kWarps * 8], l[kWarps * 8], z[kWarps * 8];
-  float scale[kWarps * 8], cta_z[8];
+  float m[kMaxWarps * 8], l[kMaxWarps * 8], z[kMaxWarps * 8];
+  float scale[kMaxWarps * 8], cta_z[8];
 };
 
 // the group's queries of pair (b, h) into shared memory, with their sums and maxima
 // (every thread of the CTA calls this; the caller orders it after earlier readers)
 // (rotated affine base: also the rotated queries into sh.qr, which the sums then follow)
+template <int NW = kWarps>
 __device__ void load_group_q(const DecodeArgs& a, Shared& sh, int b, int h, int G) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   // the Walsh-Hadamard bases take their rotated queries q' = H S q (times fl32(1/sqrt
@@ -1494,14 +1506,15 @@ __device__ void load_group_q(const DecodeArgs& a, Shared& sh, int b, int h, int 
   // the dense rotation's q' = M q comes from qrot_dense_kernel
   const bool wht = a.base == SEMKV_BASE_AFFINE_HAD || a.base == SEMKV_BASE_TQ;
   const bool rot = wht || a.base == SEMKV_BASE_TQ_DENSE;
-  for (int i = threadIdx.x; i < 8 * 128; i += kThreads) {
+  for (int i = threadIdx.x; i < 8 * 128; i += NW * 32) {
     const int c = i >> 7, d = i & 127;
     const int64_t at = ((int64_t)b * a.Hq + h * G + c) * 128 + d;
     sh.q[c][d] = c < G ? a.q[at] : (uint16_t)0;
     if (a.base == SEMKV_BASE_TQ_DENSE) sh.qr[c][d] = c < G ? a.qrot[at] : 0.0f;
   }
   __syncthreads();
-  static_assert(kWarps == 8, "one warp per head slot");
+  // warp w < 8 takes head slot w (a CTA of more warps leaves the rest idle here)
+  if (warp < 8) {
   if (wht) {
     // warp w rotates head w: lane l holds dims 4l..4l+3; butterfly stages 1, 2 inside
     // the lane, then 4..64 across lanes, each (a + b, a - b) rounded to nearest
@@ -1546,6 +1559,7 @@ __device__ void load_group_q(const DecodeArgs& a, Shared& sh, int b, int h, int 
   if (lane == 0) {
     sh.sumq[warp] = s;
     sh.qmax[warp] = mx;
+  }
   }
   __syncthreads();
 }
@@ -1599,16 +1613,18 @@ __device__ void affine_rows(WarpState& st, int L, int G, MergeArea& mg, float* m
 // affine pool rows (sum p' c; plus sum p z; lo rows folded for G <= 4); 1: TQ rows
 // from the CUDA-core path (rotated back); 2: staged rows (plain sums); 3: TQ rows from
 // the tensor-core path (as kind 0, then rotated back).
+template <int NW = kWarps>
 __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeArea& mg,
                             float* merge_o, float* part) {
+  constexpr int nw = NW;  // warps of this CTA
   __syncthreads();
   if (threadIdx.x < 8) {
     const int qh = threadIdx.x;
     float M = -INFINITY;
     if (qh < G)
-      for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mg.m[w * 8 + qh]);
+      for (int w = 0; w < nw; ++w) M = fmaxf(M, mg.m[w * 8 + qh]);
     float lsum = 0.0f, zsum = 0.0f;
-    for (int w = 0; w < kWarps; ++w) {
+    for (int w = 0; w < nw; ++w) {
       const float mw = qh < G ? mg.m[w * 8 + qh] : -INFINITY;
       const float sc = (M == -INFINITY || mw == -INFINITY) ? 0.0f : exp2f(mw - M);
       mg.scale[w * 8 + qh] = sc;
@@ -1627,11 +1643,11 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
   // (dense-rotation partials stay in the rotated domain: the combine turns their sum
   // back once per head)
   const bool rotated = (kind == 1 || kind == 3) && a.base != SEMKV_BASE_TQ_DENSE;
-  float* merged = merge_o + kWarps * 8 * 128;  // [8][128], after the warp rows
-  for (int i = threadIdx.x; i < G * 128; i += kThreads) {
+  float* merged = merge_o + nw * 8 * 128;  // [8][128], after the warp rows
+  for (int i = threadIdx.x; i < G * 128; i += NW * 32) {
     const int qh = i >> 7, d = i & 127;
     float o = 0.0f;
-    for (int w = 0; w < kWarps; ++w) {
+    for (int w = 0; w < nw; ++w) {
       const float sc = mg.scale[w * 8 + qh];
       if (sc != 0.0f) {
         float v = merge_o[(w * 8 + qh) * 128 + d];
@@ -1651,7 +1667,7 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
   if (rotated) {
     // back from the rotated domain: o = S H o' (unnormalised transform, stages 1..64)
     for (int hs = 1; hs < 128; hs <<= 1) {
-      for (int i = threadIdx.x; i < G * 64; i += kThreads) {
+      for (int i = threadIdx.x; i < G * 64; i += NW * 32) {
         const int qh = i >> 6, j = i & 63;
         const int lo = (j / hs) * 2 * hs + (j % hs);
         float* r = merged + qh * 128;
@@ -1665,7 +1681,7 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
   const int8_t* sg = rotated ? a.signs + ((int64_t)a.layer * a.H + h) * 128 : nullptr;
   // the rotated affine base stores rows in the orthonormal frame: x = S H u / sqrt(128)
   const float rs = a.base == SEMKV_BASE_AFFINE_HAD ? kInvSqrtD : 1.0f;
-  for (int i = threadIdx.x; i < G * 128; i += kThreads) {
+  for (int i = threadIdx.x; i < G * 128; i += NW * 32) {
     const int qh = i >> 7, d = i & 127;
     const float o = merged[qh * 128 + d];
     part[16 + qh * 128 + d] = rotated ? o * ((float)sg[d] * rs) : o;
@@ -1698,17 +1714,18 @@ __device__ void ring_fill(uint8_t* ring, uint64_t* bars, const uint8_t* pool_bh,
 // The first copies of a fast-path segment (chunks of kChunk tiles), as run_pool_fast
 // would start them, issued before the queries are loaded and the coefficient fragments
 // built.  The ring must be free (no merge in progress).
+template <int NW>
 __device__ void ring_fill_fast(uint8_t* ring, uint64_t* bars, const uint8_t* pool_bh,
                                uint32_t tile_bytes, int t_begin, int t_end, int ring_it) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int nchunks = (t_end - t_begin + kChunk - 1) / kChunk;
-  const int nmine = nchunks <= warp ? 0 : (nchunks - warp + kWarps - 1) / kWarps;
+  const int nmine = nchunks <= warp ? 0 : (nchunks - warp + NW - 1) / NW;
   uint8_t* my_ring = ring + warp * kFastStages * kFastStageBytes;
   uint64_t* my_bar = bars + warp * kStages;
   if (lane == 0) {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     for (int i = 0; i < kFastStages && i < nmine; ++i) {
-      const int first = t_begin + (warp + i * kWarps) * kChunk;
+      const int first = t_begin + (warp + i * NW) * kChunk;
       const uint32_t bytes = (uint32_t)min(kChunk, t_end - first) * tile_bytes;
       const int sl = (ring_it + i) % kFastStages;
       mbar_expect_tx(&my_bar[sl], bytes);
@@ -1835,25 +1852,27 @@ __device__ void fast_rows(FastState& st, int G, MergeArea& mg, float* merge_o) {
 }
 
 
-template <int L>
+template <int L, int NW>
 __device__ __forceinline__ void run_fast_l(const DecodeArgs& a, const Shared& sh, uint8_t* ring,
                                            uint2* qbs, uint64_t* bars, const uint8_t* pool_bh,
                                            int64_t count, int t0, int t1, int G, FastState& st,
                                            int& ring_it, MergeArea& mg, float* merge_o) {
-  run_pool_fast<L>(a, sh, ring, qbs, bars, pool_bh, count, t0, t1, G, st, ring_it);
+  run_pool_fast<L, NW>(a, sh, ring, qbs, bars, pool_bh, count, t0, t1, G, st, ring_it);
   fast_rows<L>(st, G, mg, merge_o);
 }
 
 // The balanced plan of decode_affine_kernel, run by the fast path: CTA c takes the
 // weighted range [c per, (c+1) per) of the concatenated [hi | lo] tile sequence of every
 // (b, h), one partial per (pair, pool) segment it touches.
-__global__ void __launch_bounds__(kThreads, kCtasFast) decode_affine_fast_kernel(DecodeArgs a) {
+template <int NW>
+__global__ void __launch_bounds__(NW * 32, NW == kWarps ? kCtasFast : 1)
+    decode_affine_fast_kernel(DecodeArgs a) {
   extern __shared__ __align__(128) uint8_t dyn[];
   __shared__ Shared sh;
   __shared__ MergeArea mg;
   uint8_t* ring = dyn;
-  uint2* qbs = reinterpret_cast<uint2*>(dyn + kFastRingBytes);  // [8 steps][32 lanes]
-  float* merge_o = reinterpret_cast<float*>(dyn);  // [kWarps][8][128] rows, then [8][128]
+  uint2* qbs = reinterpret_cast<uint2*>(dyn + fast_ring_bytes<NW>());  // [8 steps][32 lanes]
+  float* merge_o = reinterpret_cast<float*>(dyn);  // [NW][8][128] rows, then [8][128]
   const DecodePlan& P = a.plan;
   const int G = a.Hq / a.H;
   const int64_t pairs = (int64_t)a.B * a.H;
@@ -1861,7 +1880,7 @@ __global__ void __launch_bounds__(kThreads, kCtasFast) decode_affine_fast_kernel
   const int64_t start = (int64_t)blockIdx.x * P.per;
   const int64_t end = min(start + P.per, total);
 
-  if (threadIdx.x < kWarps * kStages) mbar_init(&sh.bar[0][0] + threadIdx.x);
+  if (threadIdx.x < NW * kStages) mbar_init(&sh.bar[0][0] + threadIdx.x);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncthreads();
   pdl_wait();  // the records, queries and stage partial come from earlier work
@@ -1889,18 +1908,20 @@ __global__ void __launch_bounds__(kThreads, kCtasFast) decode_affine_fast_kernel
       const int rec = record_bytes_rt(SEMKV_BASE_AFFINE, L);
       const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
       uint64_t* bars = &sh.bar[0][0];
-      ring_fill_fast(ring, bars, pool_bh, (uint32_t)(kTile * rec), t0, t1, ring_it);
+      ring_fill_fast<NW>(ring, bars, pool_bh, (uint32_t)(kTile * rec), t0, t1, ring_it);
       if (bh != loaded) {
-        load_group_q(a, sh, b, h, G);
+        load_group_q<NW>(a, sh, b, h, G);
         loaded = bh;
       }
       FastState st;
       fast_init(st);
       if (L == 5)
-        run_fast_l<5>(a, sh, ring, qbs, bars, pool_bh, count, t0, t1, G, st, ring_it, mg, merge_o);
+        run_fast_l<5, NW>(a, sh, ring, qbs, bars, pool_bh, count, t0, t1, G, st, ring_it, mg,
+                          merge_o);
       else
-        run_fast_l<6>(a, sh, ring, qbs, bars, pool_bh, count, t0, t1, G, st, ring_it, mg, merge_o);
-      merge_warps(a, a.base == SEMKV_BASE_AFFINE_HAD ? 3 : 0, h, G, mg, merge_o,
+        run_fast_l<6, NW>(a, sh, ring, qbs, bars, pool_bh, count, t0, t1, G, st, ring_it, mg,
+                          merge_o);
+      merge_warps<NW>(a, a.base == SEMKV_BASE_AFFINE_HAD ? 3 : 0, h, G, mg, merge_o,
                   a.partials + (bh * P.stride + slot) * kPartialFloats);
     }
   }
@@ -2216,17 +2237,19 @@ constexpr int64_t kSegmentCost = 16 * 7;
 
 // Replace the balanced plan p by its aligned form (see make_decode_plan) when that is
 // cheaper.  target: resident CTAs; st: 1 with a staged tail.
-static void aligned_plan(DecodePlan& p, int64_t pairs, int64_t target, int st, int max_stride) {
+static bool aligned_plan(DecodePlan& p, int64_t pairs, int64_t target, int st, int max_stride,
+                         int64_t min_tiles) {
   const int64_t th = p.tiles_hi, tl = p.tiles_lo;
   const int64_t per_pair = target / pairs;
   const int pools = (th > 0) + (tl > 0);
-  if (pools == 0 || per_pair < pools) return;
+  if (pools == 0 || per_pair < pools) return false;
   const int64_t Th = th > 0 ? th : 1, Tl = tl > 0 ? tl : 1;
-  if (Th * Tl > ((int64_t)1 << 40)) return;  // weights must stay small integers
-  // CTAs per segment: every warp gets a chunk or more, at most the partial slots allow
+  if (Th * Tl > ((int64_t)1 << 40)) return false;  // weights must stay small integers
+  // CTAs per segment: min_tiles or more per CTA (a chunk or more per warp), at most the
+  // partial slots allow
   const int64_t max_n = (int64_t)max_stride - st;
-  const int64_t cap_hi = th > 0 ? (th / 16 > 1 ? th / 16 : 1) : 0;
-  const int64_t cap_lo = tl > 0 ? (tl / 16 > 1 ? tl / 16 : 1) : 0;
+  const int64_t cap_hi = th > 0 ? (th / min_tiles > 1 ? th / min_tiles : 1) : 0;
+  const int64_t cap_lo = tl > 0 ? (tl / min_tiles > 1 ? tl / min_tiles : 1) : 0;
   int64_t best_h = 0, best_l = 0, best = INT64_MAX;
   for (int64_t nh = th > 0 ? 1 : 0; nh <= (th > 0 ? cap_hi : 0); ++nh) {
     int64_t nl = tl > 0 ? per_pair - nh : 0;
@@ -2242,14 +2265,15 @@ static void aligned_plan(DecodePlan& p, int64_t pairs, int64_t target, int st, i
       best_l = nl;
     }
   }
-  if (best == INT64_MAX || best >= p.per + kSegmentCost) return;
+  if (best == INT64_MAX || best >= p.per + kSegmentCost) return false;
   const int64_t wh = best_h * Tl, wl = best_l * Th;
-  if (wh > INT32_MAX || wl > INT32_MAX) return;
+  if (wh > INT32_MAX || wl > INT32_MAX) return false;
   p.w_hi = (int)wh;
   p.w_lo = (int)wl;
   p.per = Th * Tl;
   p.W = (best_h + best_l) * p.per;
   p.ctas = (int)(pairs * (best_h + best_l));
+  return true;
 }
 
 DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int Hq, int64_t hi_count,
@@ -2277,25 +2301,30 @@ DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int Hq, 
       p.stride = st;
       return p;
     }
-    const int64_t target = (int64_t)num_sms * (p.fast ? kCtasFast : kCtasAffine);
-    int64_t per = (total + target - 1) / target;
-    const int64_t min_work = (int64_t)(p.w_hi > p.w_lo ? p.w_hi : p.w_lo) * kWarps * 2;
-    if (per < min_work) per = min_work;
     // A pair's weighted range of length W meets at most ceil(W / per) + 1 CTA ranges,
     // and the hi | lo boundary splits at most one of those pieces in two: the pair
     // writes at most ceil(W / per) + 2 pool partials.  Keep them, plus the stage's,
     // within max_stride: ceil(W / per) <= max_stride - st - 2.
     const int64_t avail = (int64_t)max_stride - st - 2;
-    if (avail < 1) {
+    const int64_t w_max = p.w_hi > p.w_lo ? p.w_hi : p.w_lo;
+    // equal ranges for `target` CTAs of at least min_tiles tiles' weight each
+    auto straddled = [&](int64_t target, int64_t min_tiles) {
+      int64_t per = (total + target - 1) / target;
+      if (per < w_max * min_tiles) per = w_max * min_tiles;
+      const int64_t per_min = (p.W + avail - 1) / avail;
+      if (per < per_min) per = per_min;
       p.per = per;
+      p.ctas = (int)((total + per - 1) / per);
+    };
+    if (avail < 1) {
+      p.per = 1;
       p.ctas = 0;
       p.stride = max_stride + 1;  // infeasible: the caller reports the workspace as short
       return p;
     }
-    const int64_t per_min = (p.W + avail - 1) / avail;
-    if (per < per_min) per = per_min;
-    p.per = per;
-    p.ctas = (int)((total + per - 1) / per);
+    // CTAs of 8 warps, two per SM (a copy of one or two tiles per warp and step)
+    p.warps = kWarps;
+    straddled((int64_t)num_sms * (p.fast ? kCtasFast : kCtasAffine), kWarps * 2);
     // When the CTAs outnumber the pairs' segments (few sequences), ranges of equal
     // weight cut across the hi | lo and pair boundaries, and a CTA whose range holds a
     // boundary sets up, streams and merges two segments.  Aligned alternative: n_hi
@@ -2304,7 +2333,13 @@ DecodePlan make_decode_plan(int base, int L_hi, int L_lo, int B, int H, int Hq, 
     // n_hi T_lo and w_lo' = n_lo T_hi and per' = T_hi T_lo (T = the tile counts, 1 for
     // an empty pool), so that a segment is exactly n_hi (n_lo) ranges long.  Taken when
     // its longest range is shorter than per plus one segment's fixed cost.
-    aligned_plan(p, pairs, target, st, max_stride);
+    const bool aligned = aligned_plan(p, pairs, (int64_t)num_sms * (p.fast ? kCtasFast : kCtasAffine),
+                                      st, max_stride, kWarps * 2);
+    // Otherwise the fast kernel runs one CTA of 16 warps per SM (see fast_ring_bytes)
+    if (p.fast && !aligned) {
+      p.warps = kFastWarps;
+      straddled(num_sms, kFastWarps * kChunk);
+    }
     int worst = 0;
     for (int64_t bh = 0; bh < pairs; ++bh) {
       int n_hi, n_lo;
@@ -2384,9 +2419,13 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            kRingBytes + kAqBytes);
       if (r == cudaSuccess)
-        r = cudaFuncSetAttribute(decode_affine_fast_kernel,
+        r = cudaFuncSetAttribute(decode_affine_fast_kernel<kWarps>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kFastRingBytes + kQbBytes);
+                                 fast_ring_bytes<kWarps>() + kQbBytes);
+      if (r == cudaSuccess)
+        r = cudaFuncSetAttribute(decode_affine_fast_kernel<kFastWarps>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 fast_ring_bytes<kFastWarps>() + kQbBytes);
       if (r == cudaSuccess)
         r = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kRingBytes + kAqBytes);
@@ -2417,8 +2456,11 @@ cudaError_t launch_decode_attention(const DecodeArgs& a, cudaStream_t stream) {
   } else if (P.ctas > 0) {
     // (the rotated affine base rotates its queries inside the pool and stage kernels)
     if (P.fast)
-      e = launch_pdl(decode_affine_fast_kernel, dim3(P.ctas), dim3(kThreads),
-                     kFastRingBytes + kQbBytes, stream, a);
+      e = P.warps == kFastWarps
+              ? launch_pdl(decode_affine_fast_kernel<kFastWarps>, dim3(P.ctas),
+                           dim3(kFastWarps * 32), fast_ring_bytes<kFastWarps>() + kQbBytes, stream, a)
+              : launch_pdl(decode_affine_fast_kernel<kWarps>, dim3(P.ctas), dim3(kWarps * 32),
+                           fast_ring_bytes<kWarps>() + kQbBytes, stream, a);
     else
       e = launch_pdl(decode_affine_kernel, dim3(P.ctas), dim3(kThreads), kRingBytes + kAqBytes,
                      stream, a);

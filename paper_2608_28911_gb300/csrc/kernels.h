@@ -93,8 +93,9 @@ struct DecodePlan {
   int64_t per;                           // weighted length per CTA
   int ctas;
   // affine pools with five- and six-level codes and GQA groups of up to 4 heads: the
-  // fast kernel (3 resident CTAs per SM) runs the balanced plan
+  // fast kernel runs the balanced plan, with CTAs of `warps` warps (8: two per SM, 16: one)
   int fast;
+  int warps;
 };
 struct DecodeArgs {
   int base, L_hi, L_lo;

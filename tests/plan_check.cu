@@ -5,8 +5,8 @@
 // alone, the tile range each CTA of the balanced plan takes (the arithmetic of the
 // affine pool kernels) and its partial slot, and requires: every tile of the pool in
 // exactly one CTA's range, slots inside the pair's stride (the stage's slot after the
-// pools'), the CTA count within one wave of resident CTAs, and the stride within the
-// caller's limit.  Cases: the workloads' shapes, tiny and one-sided pools, staged tails,
+// pools'), the CTA count within one wave of resident CTAs (two 8-warp or one 16-warp CTA
+// per SM), and the stride within the caller's limit.  Cases: the workloads' shapes, tiny and one-sided pools, staged tails,
 // reduced strides (the no-allocation entry point), and seeded random shapes.
 #include <cstdio>
 #include <cstdlib>
@@ -25,6 +25,7 @@ static int check(int L_hi, int L_lo, int B, int H, int Hq, long hi, long lo, int
   const long total = pairs * P.W;
   int bad = 0;
   if (P.ctas > 2L * sms) bad++;
+  if (P.fast && P.warps == 16 && P.ctas > sms) bad++;   // one 16-warp CTA per SM
   for (long bh = 0; bh < pairs; ++bh) {
     int n_hi, n_lo;
     pair_slots(P, bh, n_hi, n_lo);
@@ -51,9 +52,9 @@ static int check(int L_hi, int L_lo, int B, int H, int Hq, long hi, long lo, int
   }
   if (verbose || bad)
     printf("L%d/%d B%d H%d hi %ld lo %ld stage %d sms %d max_stride %d: ctas %d stride %d "
-           "per %lld w %d/%d: %s\n",
+           "per %lld w %d/%d warps %d: %s\n",
            L_hi, L_lo, B, H, hi, lo, st, sms, max_stride, P.ctas, P.stride, (long long)P.per,
-           P.w_hi, P.w_lo, bad ? "BAD" : "ok");
+           P.w_hi, P.w_lo, P.warps, bad ? "BAD" : "ok");
   return bad ? 1 : 0;
 }
 
