@@ -73,6 +73,11 @@ constexpr int kMaxSplits = 64;                     // pool splits per (b, h)
 constexpr float kPMax = 0x1p52f;                   // bound on p = 2^(logit - e)
 
 static_assert(kStageBytes % 16 == 0, "bulk copies need 16-byte aligned stages");
+// merge area rows: kMoStride floats per (warp, column) row, dim d at d + d / 32 (each
+// quarter one bank further on), so that the lanes writing one dim of each quarter, or
+// four consecutive dims each, reach distinct banks
+constexpr int kMoStride = 132;
+__host__ __device__ constexpr int mo_at(int row, int d) { return row * kMoStride + d + (d >> 5); }
 // The fast path copies two tiles (32 consecutive slots) per bulk copy into a ring of
 // kFastStages stages per warp: one wait, one refill and one round of ring bookkeeping
 // serve 32 tokens.
@@ -92,10 +97,10 @@ template <int NW>
 constexpr int fast_ring_bytes() { return NW * kFastStages * kFastStageBytes; }
 static_assert(kFastStageBytes % 16 == 0, "bulk copies need 16-byte aligned stages");
 static_assert(kFastStages <= kStages, "the fast path uses the first barriers of each warp");
-static_assert(fast_ring_bytes<kWarps>() >= (kWarps * 8 * 128 + 8 * 128) * 4 &&
-                  fast_ring_bytes<kFastWarps>() >= (kFastWarps * 8 * 128 + 8 * 128) * 4,
+static_assert(fast_ring_bytes<kWarps>() >= (kWarps * 8 * kMoStride + 8 * 128) * 4 &&
+                  fast_ring_bytes<kFastWarps>() >= (kFastWarps * 8 * kMoStride + 8 * 128) * 4,
               "merge area reuses the ring");
-static_assert(kRingBytes >= (kWarps * 8 * 128 + 8 * 128) * 4, "merge area reuses the ring");
+static_assert(kRingBytes >= (kWarps * 8 * kMoStride + 8 * 128) * 4, "merge area reuses the ring");
 
 // ------------------------------------------------------------------ PTX -------
 
@@ -1381,7 +1386,7 @@ __device__ void run_pool_tq(const DecodeArgs& a, const Shared& sh, int which,
       z_out[warp * 8 + c] = 0.0f;
     }
 #pragma unroll
-    for (int j = 0; j < 4; ++j) o_out[(warp * 8 + c) * 128 + 4 * lane + j] = o[c][j];
+    for (int j = 0; j < 4; ++j) o_out[mo_at(warp * 8 + c, 4 * lane + j)] = o[c][j];
   }
 }
 
@@ -1467,7 +1472,7 @@ __device__ void run_stage(const DecodeArgs& a, const Shared& sh, int b, int h, i
       z_out[warp * 8 + c] = 0.0f;
     }
 #pragma unroll
-    for (int j = 0; j < 4; ++j) o_out[(warp * 8 + c) * 128 + 4 * lane + j] = o[c][j];
+    for (int j = 0; j < 4; ++j) o_out[mo_at(warp * 8 + c, 4 * lane + j)] = o[c][j];
   }
 }
 
@@ -1498,19 +1503,46 @@ struct MergeArea {
 // the group's queries of pair (b, h) into shared memory, with their sums and maxima
 // (every thread of the CTA calls this; the caller orders it after earlier readers)
 // (rotated affine base: also the rotated queries into sh.qr, which the sums then follow)
+// A CTA of NW warps' share of the group's query values (thread i: values i, i + 32 NW,
+// ...): loaded into registers before a segment's first copies are issued, so that the
+// loads do not queue behind the copies
+template <int NW>
+struct QPrefetch {
+  static constexpr int kN = (8 * 128 + NW * 32 - 1) / (NW * 32);
+  uint16_t v[kN];
+};
+template <int NW>
+__device__ __forceinline__ void q_prefetch(const DecodeArgs& a, int b, int h, int G,
+                                           QPrefetch<NW>& pre) {
+#pragma unroll
+  for (int k = 0; k < QPrefetch<NW>::kN; ++k) {
+    const int i = threadIdx.x + k * NW * 32, c = i >> 7, d = i & 127;
+    pre.v[k] = (i < 8 * 128 && c < G) ? a.q[((int64_t)b * a.Hq + h * G + c) * 128 + d] : (uint16_t)0;
+  }
+}
+
 template <int NW = kWarps>
-__device__ void load_group_q(const DecodeArgs& a, Shared& sh, int b, int h, int G) {
+__device__ void load_group_q(const DecodeArgs& a, Shared& sh, int b, int h, int G,
+                             const QPrefetch<NW>* pre = nullptr) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   // the Walsh-Hadamard bases take their rotated queries q' = H S q (times fl32(1/sqrt
   // 128) for the rotated affine base, whose rows are stored in the orthonormal frame);
   // the dense rotation's q' = M q comes from qrot_dense_kernel
   const bool wht = a.base == SEMKV_BASE_AFFINE_HAD || a.base == SEMKV_BASE_TQ;
   const bool rot = wht || a.base == SEMKV_BASE_TQ_DENSE;
-  for (int i = threadIdx.x; i < 8 * 128; i += NW * 32) {
-    const int c = i >> 7, d = i & 127;
-    const int64_t at = ((int64_t)b * a.Hq + h * G + c) * 128 + d;
-    sh.q[c][d] = c < G ? a.q[at] : (uint16_t)0;
-    if (a.base == SEMKV_BASE_TQ_DENSE) sh.qr[c][d] = c < G ? a.qrot[at] : 0.0f;
+  if (pre) {
+#pragma unroll
+    for (int k = 0; k < QPrefetch<NW>::kN; ++k) {
+      const int i = threadIdx.x + k * NW * 32;
+      if (i < 8 * 128) sh.q[i >> 7][i & 127] = pre->v[k];
+    }
+  } else {
+    for (int i = threadIdx.x; i < 8 * 128; i += NW * 32) {
+      const int c = i >> 7, d = i & 127;
+      const int64_t at = ((int64_t)b * a.Hq + h * G + c) * 128 + d;
+      sh.q[c][d] = c < G ? a.q[at] : (uint16_t)0;
+      if (a.base == SEMKV_BASE_TQ_DENSE) sh.qr[c][d] = c < G ? a.qrot[at] : 0.0f;
+    }
   }
   __syncthreads();
   // warp w < 8 takes head slot w (a CTA of more warps leaves the rest idle here)
@@ -1602,7 +1634,7 @@ __device__ void affine_rows(WarpState& st, int L, int G, MergeArea& mg, float* m
             case 7: dim = v_dim<7>(g, 2 * m + r); break;
             default: dim = v_dim<8>(g, 2 * m + r); break;
           }
-          merge_o[(warp * 8 + qh) * 128 + dim] = st.O[m][2 * r + c];
+          merge_o[mo_at(warp * 8 + qh, dim)] = st.O[m][2 * r + c];
         }
       }
     }
@@ -1643,15 +1675,15 @@ __device__ void merge_warps(const DecodeArgs& a, int kind, int h, int G, MergeAr
   // (dense-rotation partials stay in the rotated domain: the combine turns their sum
   // back once per head)
   const bool rotated = (kind == 1 || kind == 3) && a.base != SEMKV_BASE_TQ_DENSE;
-  float* merged = merge_o + nw * 8 * 128;  // [8][128], after the warp rows
+  float* merged = merge_o + nw * 8 * kMoStride;  // [8][128], after the warp rows
   for (int i = threadIdx.x; i < G * 128; i += NW * 32) {
     const int qh = i >> 7, d = i & 127;
     float o = 0.0f;
     for (int w = 0; w < nw; ++w) {
       const float sc = mg.scale[w * 8 + qh];
       if (sc != 0.0f) {
-        float v = merge_o[(w * 8 + qh) * 128 + d];
-        if ((kind == 0 || kind == 3) && G <= 4) v += merge_o[(w * 8 + qh + 4) * 128 + d];
+        float v = merge_o[mo_at(w * 8 + qh, d)];
+        if ((kind == 0 || kind == 3) && G <= 4) v += merge_o[mo_at(w * 8 + qh + 4, d)];
         o += sc * v;
       }
     }
@@ -1846,7 +1878,7 @@ __device__ void fast_rows(FastState& st, int G, MergeArea& mg, float* merge_o) {
       for (int m = 0; m < 8; ++m)
 #pragma unroll
         for (int r = 0; r < 2; ++r)
-          merge_o[(warp * 8 + col) * 128 + v_dim<L>(g, 2 * m + r)] = st.O[m][2 * r + c];
+          merge_o[mo_at(warp * 8 + col, v_dim<L>(g, 2 * m + r))] = st.O[m][2 * r + c];
     }
   }
 }
@@ -1908,9 +1940,14 @@ __global__ void __launch_bounds__(NW * 32, NW == kWarps ? kCtasFast : 1)
       const int rec = record_bytes_rt(SEMKV_BASE_AFFINE, L);
       const uint8_t* pool_bh = pool + (((int64_t)b * a.NL + a.layer) * a.H + h) * cap * rec;
       uint64_t* bars = &sh.bar[0][0];
+      // the queries' loads first, then the segment's first copies, then the queries
+      // into shared memory
+      const bool new_q = bh != loaded;
+      QPrefetch<NW> pre;
+      if (new_q) q_prefetch<NW>(a, b, h, G, pre);
       ring_fill_fast<NW>(ring, bars, pool_bh, (uint32_t)(kTile * rec), t0, t1, ring_it);
-      if (bh != loaded) {
-        load_group_q<NW>(a, sh, b, h, G);
+      if (new_q) {
+        load_group_q<NW>(a, sh, b, h, G, &pre);
         loaded = bh;
       }
       FastState st;
