@@ -6,9 +6,12 @@
 // h = qh / G (G = q_heads / kv_heads <= 8).  Affine rows dequantize as z + s*c.
 //
 // Work split.  The tokens of each (b, h) are cut into 16-token tiles, per source
-// (high pool, low pool, fp16 stage).  A CTA of 8 warps handles a contiguous range of
-// tiles of ONE source (so its level count L is uniform), the warps taking tiles
-// round-robin; a final kernel merges the per-CTA partials (m, l, o) per (b, qh).
+// (high pool, low pool, fp16 stage).  A CTA runs each (b, h, pool) segment of its range
+// of tiles in turn (so the level count L is uniform within a segment), its warps taking
+// the segment's tiles round-robin (two at a time on the fast path), and writes one
+// partial (m, l, o) per segment; a final kernel merges the partials per (b, qh).  The
+// affine pools take a balanced plan (equal weighted ranges over all pairs, or ranges
+// aligned to the segments when the sequences are few), the TQ pools a split plan.
 //
 // Decoding on the FMA pipe.  A group symbol is stored as the W-bit integer
 // beta = ceil(t 2^W / L^G), so F_k = floor(beta L^(k+1) / 2^W) is the number formed by
