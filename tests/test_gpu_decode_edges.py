@@ -17,7 +17,9 @@ takes part):
 
 Each case runs at T = 4096 (hi + lo pools over several CTAs of the balanced or split
 plan, then the combine), on the plain affine 6/5, the Hadamard-rotated affine 6/5 and
-the TurboQuant-MSE 4/3 bases, most with a staged fp16 tail.
+the TurboQuant-MSE 4/3 bases, most with a staged fp16 tail.  One more case runs sharp
+queries and dominant tokens over 320 (sequence, KV head) pairs, where the affine pools
+take equal ranges on 16-warp CTAs that each hold several segments.
 
 Tolerance: max-abs 2e-3 and relative L2 1e-3 at the synthetic scale (|v| below 64).
 Binary32 carries a relative, not an absolute, error, so the absolute bound follows the
@@ -210,3 +212,47 @@ def test_logit_shift_leaves_output_unchanged():
     assert np.max(np.abs(r0 - r1)) < 1e-9          # the oracle: shift invariant
     err, rel = attention_errors(g1, g0)
     assert err <= ATOL and rel <= RTOL_L2, (err, rel)
+
+
+# ----------------------------- the equal-range plan: several segments per CTA -----
+
+@pytest.mark.parametrize("base", [0, 2])
+def test_sharp_softmax_and_dominant_token_equal_range_plan(base):
+    """Many (sequence, KV head) pairs: 320 here, more than the CTAs of one wave, so the
+    affine pools run equal weighted ranges on one CTA of 16 warps per SM, each CTA taking
+    several segments (hi and lo pools of consecutive pairs) and loading new queries for
+    each pair.  Queries scaled x16, and in every fifth sequence the last low-pool token
+    dominates query head 0 of KV head 0 (logit 640, the rest below about 200); a staged
+    fp16 tail.  Sampled heads, those heads included, against the oracle."""
+    B, H, Hq, T_ = 40, 8, 32, 1200
+    r = (26, 100)
+    p = Pair(base, 6, 5, B, 1, H, Hq, T_, r[0], r[1], seed=560 + base, block=64)
+    q = synthetic.queries(561 + base, B, Hq).astype(np.float32) * 16
+    is_high, _, _ = oracle.rank_assign(p.s, oracle.high_count_floor(T_, r[0], r[1]))
+    k = p.k.astype(np.float32)
+    for b in range(0, B, 5):
+        t_star = int(np.nonzero(is_high[b] == 0)[0][-1])
+        qv = q[b, 0]
+        # logit 640: the x16 queries put the other tokens' logits below about 200
+        k[b, 0, 0, t_star] = 640.0 * np.sqrt(128.0) * qv / float(qv @ qv)
+    p.k = k.astype(np.float16)
+    p.quantize()
+    _stage_tail(p, 562 + base)
+    rng = np.random.default_rng(563 + base)
+    heads = [(b, 0) for b in range(0, B, 5)]
+    heads += [(int(b), int(qh)) for b, qh in zip(rng.integers(0, B, 24), rng.integers(0, Hq, 24))]
+    q16 = q.astype(np.float16)
+    got, ref = p.decode(q=q16, heads=heads)
+    sel = np.zeros((B, Hq), bool)
+    for b, qh in heads:
+        sel[b, qh] = True
+    err, rel = attention_errors(got[sel], ref[sel])
+    assert err <= ATOL and rel <= RTOL_L2, (err, rel)
+    assert np.isfinite(got).all()
+    assert int(p.cache.dev_error.item()) == 0
+    # the dominant tokens did dominate: those heads' outputs are their value rows
+    for b in range(0, B, 5):
+        K, V = oracle.dequant_cache_head(p.oc, b, 0, 0)
+        lg = K @ q16[b, 0].astype(np.float64) / np.sqrt(128.0)
+        j = int(np.argmax(lg))
+        assert lg[j] - np.partition(lg, -2)[-2] > 20.0
