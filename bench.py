@@ -433,6 +433,18 @@ def gpu_arm(args, cfg, rank, world):
             with torch.cuda.graph(gd):
                 decode_all(q_for(k))
             parts.append((ga, gd))
+        # block mode: each step also as ONE graph (the append and the decode together, so
+        # the programmatic dependent launches overlap their boundary too), which times
+        # the step; the pairs above time the decode alone.  (Every block-mode step rewinds
+        # the counts first, so capturing the steps again finds the same host state.)
+        whole = []
+        if not token_mode:
+            for k in range(n_distinct):
+                gw = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(gw):
+                    pre_decode(k)
+                    decode_all(q_for(k))
+                whole.append(gw)
         torch.cuda.synchronize()
 
         def step(i, ev=None, _parts=parts):   # noqa: F811 (the graph replay of the step)
@@ -446,6 +458,12 @@ def gpu_arm(args, cfg, rank, world):
         for i in range(args.warmup):
             step(i)
         torch.cuda.synchronize()
+        if whole:
+            def step_whole(i, _whole=whole):
+                _whole[i % len(_whole)].replay()
+            for i in range(args.warmup):
+                step_whole(i)
+            torch.cuda.synchronize()
 
     def barrier():
         if world > 1:
@@ -455,13 +473,20 @@ def gpu_arm(args, cfg, rank, world):
 
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in range(args.steps)]
+    # the step as a whole (one graph per step where there is one), and the decode alone
+    # (its calls bracketed by events); the same steps, timed twice
+    step_timed = step_whole if (args.graph and not token_mode) else step
+    dec_loop = args.graph and not token_mode
     with ClockSampler(dev.index) as clk:
         if not flush:
             t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             barrier()
             t0.record(stream)
             for i in range(args.steps):
-                step(i, evs[i])
+                if dec_loop:
+                    step_timed(i)
+                else:
+                    step(i, evs[i])
             t1.record(stream)
             barrier()
             elapsed = t0.elapsed_time(t1) * 1e-3
@@ -473,10 +498,21 @@ def gpu_arm(args, cfg, rank, world):
             for i in range(args.steps):
                 scrub.fill_(i & 0xFF)
                 sev[i][0].record(stream)
-                step(i, evs[i])
+                if dec_loop:
+                    step_timed(i)
+                else:
+                    step(i, evs[i])
                 sev[i][1].record(stream)
             barrier()
             elapsed = sum(a.elapsed_time(b) for a, b in sev) * 1e-3
+        if dec_loop:
+            # the decode alone: the same steps replayed as (append, decode) graph pairs
+            barrier()
+            for i in range(args.steps):
+                if flush:
+                    scrub.fill_(i & 0xFF)
+                step(i, evs[i])
+            barrier()
     dec_times = [a.elapsed_time(b) * 1e-3 for a, b in evs]
     err = int(cache.dev_error.item())
     # the cache's own stage buffers again (the steps above pointed it at the blocks)
