@@ -66,6 +66,7 @@ const char* semkv_status_string(semkv_status s) {
 // Lloyd-Max quantizer of N(0,1) (Sec. 4.9): Lloyd iteration in fp64 until the
 // centroids stop moving; thresholds are centroid midpoints.
 semkv_status semkv_lloyd_max_gaussian(int32_t levels, float* centroids, float* thresholds) {
+  const TraceRange trace("semkv_lloyd_max_gaussian");
   if (levels < 2 || levels > 64 || !centroids || !thresholds) return SEMKV_EINVAL;
   const int L = levels;
   double c[64], nc[64], t[65];
@@ -105,6 +106,7 @@ size_t semkv_rank_workspace_bytes(int32_t batch, int32_t T, int32_t want_rank) {
 semkv_status semkv_rank_assign(const float* scores, int32_t batch, int32_t T, uint32_t n_high,
                                uint8_t* is_high, uint32_t* slot, uint32_t* rank, void* ws,
                                size_t ws_bytes, void* stream) {
+  const TraceRange trace("semkv_rank_assign");
   if (!scores || !is_high || !slot || batch < 0 || T < 1 || T > (1 << 24)) return SEMKV_EINVAL;
   if (n_high > (uint32_t)T) return SEMKV_EINVAL;
   if (rank) {
@@ -128,6 +130,7 @@ semkv_status semkv_fake_quant(const semkv_quant_desc* desc, const uint16_t* k, c
                               int32_t batch, int32_t layers, int32_t kv_heads, int32_t T,
                               const uint8_t* is_high, uint16_t* k_out, uint16_t* v_out,
                               void* stream) {
+  const TraceRange trace("semkv_fake_quant");
   semkv_status s = check_desc(desc);
   if (s != SEMKV_OK) return s;
   if (desc->base == SEMKV_BASE_TQ_DENSE) return SEMKV_EUNSUPPORTED;
@@ -159,6 +162,7 @@ semkv_status semkv_fake_quant(const semkv_quant_desc* desc, const uint16_t* k, c
 semkv_status semkv_score_kv_norm(const uint16_t* x, int32_t batch, int32_t layers,
                                  int32_t kv_heads, int32_t T, int32_t layer_begin,
                                  int32_t layer_end, float* scores, void* stream) {
+  const TraceRange trace("semkv_score_kv_norm");
   if (!x || !scores || batch < 1 || layers < 1 || kv_heads < 1 || T < 1) return SEMKV_EINVAL;
   if (layer_begin < 0 || layer_end > layers || layer_begin >= layer_end) return SEMKV_EINVAL;
   if (!aligned(x, 8) || !aligned(scores, 4)) return SEMKV_EALIGN;
@@ -178,6 +182,7 @@ semkv_status semkv_quantize_pack(const semkv_quant_desc* desc, const uint16_t* k
                                  const uint16_t* v, int32_t T, const uint8_t* is_high,
                                  const uint32_t* slot, uint32_t n_high, semkv_cache* cache,
                                  void* stream) {
+  const TraceRange trace("semkv_quantize_pack");
   semkv_status s = check_desc(desc);
   if (s != SEMKV_OK) return s;
   s = check_cache(cache);
@@ -227,6 +232,7 @@ semkv_status semkv_quantize_pack(const semkv_quant_desc* desc, const uint16_t* k
 
 semkv_status semkv_append_block(const semkv_quant_desc* desc, semkv_cache* cache,
                                 uint32_t r_num, uint32_t r_den, void* stream) {
+  const TraceRange trace("semkv_append_block");
   semkv_status s = check_desc(desc);
   if (s != SEMKV_OK) return s;
   s = check_cache(cache);
@@ -315,6 +321,7 @@ semkv_status semkv_decode_attention(const semkv_quant_desc* desc, const semkv_ca
                                     int32_t layer, const uint16_t* q, float* out,
                                     float softmax_scale, void* ws, size_t ws_bytes,
                                     void* stream) {
+  const TraceRange trace("semkv_decode_attention");
   semkv_status s = check_decode(desc, cache, layer, q, out);
   if (s != SEMKV_OK) return s;
   if (!ws || !aligned(ws, 16)) return SEMKV_EWORKSPACE;

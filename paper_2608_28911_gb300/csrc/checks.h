@@ -5,10 +5,22 @@
 #include <cstdint>
 #include <cstring>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/semkv.h"
 #include "kernels.h"
 
 namespace semkv {
+
+// An NVTX range named after the C-ABI call, open for the call's host-side extent (its
+// checks and launches), so a profiler's timeline shows which call enqueued which kernels.
+// Without a profiler attached the push and pop do nothing.
+struct TraceRange {
+  explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+  ~TraceRange() { nvtxRangePop(); }
+  TraceRange(const TraceRange&) = delete;
+  TraceRange& operator=(const TraceRange&) = delete;
+};
 
 inline bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
 

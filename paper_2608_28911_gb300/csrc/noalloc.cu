@@ -60,6 +60,7 @@ extern "C" semkv_status semkv_decode_attention_noalloc(const semkv_quant_desc* d
                                                        const semkv_cache* cache, int32_t layer,
                                                        const uint16_t* q, float* out,
                                                        float softmax_scale, void* stream) {
+  const semkv::TraceRange trace("semkv_decode_attention_noalloc");
   using namespace semkv;
   semkv_status st = check_decode(desc, cache, layer, q, out);
   if (st != SEMKV_OK) return st;
